@@ -1,0 +1,165 @@
+"""ctypes front end of the plain-C oracle (``oracle.c``).
+
+TEST INFRASTRUCTURE ONLY: imported by the test suite, the smoke check and the
+benchmark's CPU-baseline leg.  The product package never imports it.
+
+Functions take and return numpy arrays.  Each returns ``(status, outputs...)``
+with the same status codes as the product library (0 ok, -1 invalid, -2 range,
+-3 unbounded).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+
+MODE_SNAPSHOT, MODE_SEQUENTIAL, MODE_ALG1_SNAPSHOT, MODE_ALG1_SEQUENTIAL = 0, 1, 2, 3
+
+
+def build(force: bool = False) -> str:
+    """Compile ``liboracle.so`` with the host C compiler (plain C11, -O2)."""
+    if force or not os.path.exists(_LIB) or (
+            os.path.getmtime(_LIB) < max(os.path.getmtime(_SRC),
+                                         os.path.getmtime(os.path.join(_HERE, "oracle.h")))):
+        tmp = _LIB + f".{os.getpid()}.tmp"
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-shared", "-fPIC",
+                               "-o", tmp, _SRC])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+_lib = None
+
+_i32p = np.ctypeslib.ndpointer(np.int32, flags="C_CONTIGUOUS")
+_i64p = np.ctypeslib.ndpointer(np.int64, flags="C_CONTIGUOUS")
+
+
+class StreamCfg(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int64), ("D", ctypes.c_int32),
+                ("H", ctypes.c_int32), ("cap", ctypes.c_int32),
+                ("batch", ctypes.c_int32), ("window", ctypes.c_int32),
+                ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32)]
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        L = ctypes.CDLL(build())
+        L.oracle_rank.restype = ctypes.c_int64
+        L.oracle_rank.argtypes = [ctypes.c_int64, ctypes.c_uint32]
+        L.oracle_calibrate.argtypes = [_i32p, _i32p, ctypes.c_int64,
+                                       ctypes.c_uint32,
+                                       ctypes.POINTER(ctypes.c_int64)]
+        L.oracle_bound.argtypes = [_i32p, ctypes.c_int64, ctypes.c_int64, _i32p]
+        L.oracle_occupancy.argtypes = [ctypes.c_int32, ctypes.c_int32, _i64p,
+                                       ctypes.c_int64, _i32p, _i32p, _i32p,
+                                       _i32p]
+        L.oracle_occupancy_cell.restype = ctypes.c_int64
+        L.oracle_occupancy_cell.argtypes = [ctypes.c_int32, _i64p,
+                                            ctypes.c_int32, ctypes.c_int32,
+                                            _i32p, _i32p, _i32p]
+        vp = ctypes.c_void_p
+        L.oracle_dispatch.argtypes = [ctypes.c_int32, ctypes.c_int32,
+                                      ctypes.c_int32, ctypes.c_int32, vp, vp,
+                                      vp, vp, ctypes.c_int64, vp, vp, vp,
+                                      ctypes.c_int64, vp, vp, vp, vp]
+        L.oracle_order_local.argtypes = [ctypes.c_int64, ctypes.c_int32, vp, vp,
+                                         vp, vp, ctypes.c_int32, vp, vp]
+        L.oracle_stream.argtypes = [ctypes.POINTER(StreamCfg), _i64p, _i32p,
+                                    _i32p, _i32p, _i32p, _i32p, _i64p]
+        _lib = L
+    return _lib
+
+
+def _c32(a):
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+def _c64(a):
+    return np.ascontiguousarray(a, dtype=np.int64)
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def rank(n: int, alpha_ppm: int) -> int:
+    return int(lib().oracle_rank(n, alpha_ppm))
+
+
+def calibrate(true_len, pred_len, alpha_ppm: int):
+    t, p = _c32(true_len), _c32(pred_len)
+    q = ctypes.c_int64(0)
+    st = lib().oracle_calibrate(t, p, t.shape[0], alpha_ppm, ctypes.byref(q))
+    return st, int(q.value)
+
+
+def bound(pred, q: int):
+    p = _c32(pred)
+    out = np.empty_like(p)
+    st = lib().oracle_bound(p, p.shape[0], q, out)
+    return st, out
+
+
+def occupancy(D: int, H: int, res_off, prompt, gen, bnd):
+    off = _c64(res_off)
+    p, g, u = _c32(prompt), _c32(gen), _c32(bnd)
+    K = np.empty((D, H), dtype=np.int32)
+    st = lib().oracle_occupancy(D, H, off, p.shape[0], p, g, u, K.reshape(-1))
+    return st, K
+
+
+def occupancy_cell(H: int, res_off, k: int, t: int, prompt, gen, bnd) -> int:
+    return int(lib().oracle_occupancy_cell(H, _c64(res_off), k, t, _c32(prompt),
+                                           _c32(gen), _c32(bnd)))
+
+
+def dispatch(mode: int, D: int, H: int, S: int, K, cap, Q, cand_prompt,
+             cand_bound, res_off=None, prompt=None, gen=None, bnd=None):
+    """Returns (status, choice, headroom, K_after, Q_after).  K and Q are
+    copied; SEQUENTIAL modes update the copies in place."""
+    Kc = None if K is None else _c32(K).copy()
+    Qc = _c32(Q).copy()
+    capc = _c32(cap)
+    cp, cb = _c32(cand_prompt), _c32(cand_bound)
+    J = cp.shape[0]
+    choice = np.empty(J, dtype=np.int32)
+    head = np.empty(J, dtype=np.int64)
+    off = None if res_off is None else _c64(res_off)
+    pr = None if prompt is None else _c32(prompt)
+    ge = None if gen is None else _c32(gen)
+    bo = None if bnd is None else _c32(bnd)
+    R = 0 if pr is None else pr.shape[0]
+    st = lib().oracle_dispatch(mode, D, H, S, _ptr(Kc), _ptr(capc), _ptr(Qc),
+                               _ptr(off), R, _ptr(pr), _ptr(ge), _ptr(bo), J,
+                               _ptr(cp), _ptr(cb), _ptr(choice), _ptr(head))
+    return st, choice, head, Kc, Qc
+
+
+def order_local(D: int, dec, bnd, wait, arrival, max_wait: int):
+    d, b, w, a = _c32(dec), _c32(bnd), _c32(wait), _c32(arrival)
+    N = d.shape[0]
+    perm = np.empty(N, dtype=np.int32)
+    seg = np.empty(D + 1, dtype=np.int64)
+    st = lib().oracle_order_local(N, D, _ptr(d), _ptr(b), _ptr(w), _ptr(a),
+                                  max_wait, _ptr(perm), _ptr(seg))
+    return st, perm, seg
+
+
+def stream(N, D, H, cap, batch, window, alpha_ppm, max_wait, arrival_ms,
+           prompt, true_len, pred):
+    cfg = StreamCfg(N, D, H, cap, batch, window, alpha_ppm, max_wait)
+    nb = (N + batch - 1) // batch
+    choice = np.empty(N, dtype=np.int32)
+    q = np.empty(nb, dtype=np.int32)
+    stats = np.empty(4 * nb, dtype=np.int64)
+    st = lib().oracle_stream(ctypes.byref(cfg), _c64(arrival_ms[:N]),
+                             _c32(prompt[:N]), _c32(true_len[:N]),
+                             _c32(pred[:N]), choice, q, stats)
+    return st, choice, q, stats.reshape(nb, 4)
