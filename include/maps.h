@@ -1,0 +1,202 @@
+/*
+ * maps.h -- C ABI of the MAPS memory-aware predictive scheduler hot path,
+ * implemented as integer-only CUDA kernels for GB300 (sm_103a).
+ *
+ * The four calls follow the scheduler's problem statement (Sec. 3.3): decoders
+ * d_k with KV-token capacity C_k and waiting-queue length Q_k; requests with a
+ * prompt length, a predicted output length, and a calibrated upper bound on
+ * it (Sec. 3.2).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * Memory.   Every array argument is DEVICE memory owned by the caller, except
+ *           where an argument name ends in `_host`.  The library allocates
+ *           nothing: calls that need scratch memory take a caller-provided
+ *           workspace `ws` of `ws_bytes` bytes, sized by the matching
+ *           `maps_*_workspace_size()` query.  A workspace must be zero-filled
+ *           before its first use and must be 256-byte aligned.  One
+ *           workspace may serve several calls in sequence on one stream;
+ *           calls that run concurrently need separate workspaces.
+ * Streams.  `stream` is a cudaStream_t passed as void*.  Calls enqueue work
+ *           on it and return without waiting, except where a `_host` output
+ *           is non-NULL: then the call synchronises the stream and returns
+ *           the full status, data-dependent errors included.
+ * Layout.   Arrays are dense and row-major; int32 unless stated.  K is
+ *           [D][H].  Residents of decoder k are the index range
+ *           [res_off[k], res_off[k+1]) of the resident arrays (CSR).
+ * Status.   Every call returns an int status.  Argument errors (NULL
+ *           pointers, negative sizes, a workspace too small or misaligned)
+ *           are returned at once and nothing is enqueued.  Errors that depend
+ *           on device data (a value outside its domain, an int32 overflow, a
+ *           bounded device wait that expired) are recorded in a sticky status
+ *           word inside the workspace; read and clear it with maps_check().
+ *           Outputs are unspecified when a call or a later maps_check()
+ *           reports an error.  No exception crosses the interface and no
+ *           kernel traps.
+ * Domain.   Lengths (prompt p, generated g, bounds U), capacities, queue
+ *           lengths and K values must be >= 0; a negative one is reported as
+ *           MAPS_E_RANGE.
+ */
+#ifndef MAPS_H
+#define MAPS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MAPS_OK 0
+#define MAPS_E_INVALID (-1)   /* bad argument: NULL, size, alignment, mode */
+#define MAPS_E_RANGE (-2)     /* device data outside its domain or int32 range */
+#define MAPS_E_UNBOUNDED (-3) /* conformal rank exceeds n: no finite bound */
+#define MAPS_E_TIMEOUT (-4)   /* a bounded device wait expired */
+#define MAPS_E_CUDA (-5)      /* CUDA runtime error; see maps_last_cuda_error */
+#define MAPS_E_WORKSPACE (-6) /* workspace smaller than the size query asked */
+
+#define MAPS_MODE_SNAPSHOT 0
+#define MAPS_MODE_SEQUENTIAL 1
+#define MAPS_MODE_ALG1_SNAPSHOT 2
+#define MAPS_MODE_ALG1_SEQUENTIAL 3
+
+/* Library version, major*10000 + minor*100 + patch. */
+int maps_version(void);
+
+/* The cudaError_t behind the last MAPS_E_CUDA returned by this thread. */
+int maps_last_cuda_error(void);
+
+/* Synchronises `stream`, returns the workspace's sticky device status
+ * (MAPS_OK or the first error any kernel recorded in it) and clears it. */
+int maps_check(void *ws, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Uncertainty-aware calibration, Sec. 3.2.
+ *
+ * Scores s_i = max(0, true_len[i] - pred_len[i]) (Eq. nonconformity) over the
+ * calibration set of n completed requests; q = the k-th smallest score with
+ * k = ceil((1 - alpha)(n + 1)), alpha = alpha_ppm / 1e6 (the rank is exact
+ * integer arithmetic); then, for m query predictions, the calibrated upper
+ * bounds bound_out[i] = query_pred[i] + q (Eq. conformal_upper).
+ *
+ *   true_len, pred_len  [n] int32, device.
+ *   alpha_ppm           miscoverage in parts per million, 0 < alpha_ppm < 1e6.
+ *   query_pred, m       [m] predictions to bound (m may be 0, then both NULL).
+ *   bound_out           [m] int32 output, device.
+ *   q_dev_out           int32 scalar output, device (may be NULL).
+ *   q_host_out          int32 scalar output, host (may be NULL; non-NULL
+ *                       synchronises the stream).
+ * Returns MAPS_E_UNBOUNDED at once, enqueuing nothing, when k > n (including
+ * n = 0): the bound is unavailable and Alg. 1 falls back to round robin.
+ * q > INT32_MAX or a bound above INT32_MAX is MAPS_E_RANGE.
+ * Requires n <= 2^40.
+ * ---------------------------------------------------------------------- */
+size_t maps_calibrate_workspace_size(int64_t n, int64_t m);
+int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
+                   uint32_t alpha_ppm, const int32_t *query_pred, int64_t m,
+                   int32_t *bound_out, int32_t *q_dev_out, int32_t *q_host_out,
+                   void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Projected KV-token occupancy over a step horizon.
+ *
+ * Built on the KV footprint M(r) = L_p + L_out (App. A, Eq. kv_demand) and the
+ * occupancy K_d(t) of Eq. (admission): at step t in [0, H) a resident r of
+ * decoder k with prompt p, g tokens generated and bound U holds p + g + t + 1
+ * KV tokens while t < e_r = min(max(U - g, 1), H) (a resident past its bound
+ * is kept for one step), so
+ *     K[k][t] = sum over residents r of k with t < e_r of (p + g + 1 + t).
+ *
+ *   D, H                decoders (>= 1) and horizon steps (>= 1).
+ *   res_off             [D+1] int64 CSR offsets into the resident arrays,
+ *                       non-decreasing within [0, R].
+ *   R                   length of prompt / gen / bound.
+ *   prompt, gen, bound  [R] int32 resident prompt lengths, generated tokens,
+ *                       calibrated bounds.
+ *   K_out               [D][H] int32 output.
+ * A K value above INT32_MAX, offsets out of order or a negative length is
+ * MAPS_E_RANGE (via maps_check).
+ * ---------------------------------------------------------------------- */
+size_t maps_project_occupancy_workspace_size(int32_t D, int32_t H, int64_t R);
+int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
+                           int64_t R, const int32_t *prompt, const int32_t *gen,
+                           const int32_t *bound, int32_t *K_out, void *ws,
+                           size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Global memory-aware dispatch, Sec. 3.3 and Alg. 1.
+ *
+ * Horizon modes (SNAPSHOT, SEQUENTIAL).  Candidate j (prompt p_j, bound U_j)
+ * is live for u_j = min(max(U_j, 1), H) steps holding p_j + t + 1 tokens, so
+ * on decoder k its peak is
+ *     peak_jk = max_{t < u_j} (K[k][t] + p_j + t + 1),  h_jk = cap[k] - peak_jk.
+ * Decoder k is feasible iff h_jk >= 0.  The choice is the feasible decoder
+ * with the smallest Q[k]; if none is feasible, the decoder with the largest
+ * headroom h_jk (the fallback to the most available capacity).  Ties go to
+ * the lowest decoder index.  SNAPSHOT scores every candidate against the same
+ * state.  SEQUENTIAL takes candidates in index order and, after each choice,
+ * reserves the footprint at the chosen decoder: K[k*][t] += p_j + t + 1 for
+ * t < u_j and Q[k*] += 1, in place.
+ *
+ * ALG1 modes (ALG1_SNAPSHOT, ALG1_SEQUENTIAL): Algorithm 1 literally, with
+ * block size S: B_need_j = ceil((p_j + U_j) / S) (Eq. feasibility);
+ * B_eff_k = floor(cap[k] / S) - sum over residents of
+ * ceil((p + max(U, g + 1)) / S) (free blocks minus what each ongoing request
+ * holds or has reserved at its bound); feasible iff B_need_j <= B_eff_k; argmin
+ * Q over the feasible set, else argmax B_eff; headroom = B_eff - B_need.
+ * ALG1_SEQUENTIAL subtracts B_need from B_eff[k*] and adds 1 to Q[k*] after
+ * each choice.  K is not read in the ALG1 modes.
+ *
+ *   mode                MAPS_MODE_*.
+ *   D, H, S             decoders (1 <= D <= 1024), horizon, block size (ALG1).
+ *   K                   [D][H] int32 occupancy (horizon modes; updated in
+ *                       place by SEQUENTIAL).
+ *   cap, Q              [D] int32 capacities and queue lengths (Q updated in
+ *                       place by the SEQUENTIAL modes).
+ *   res_off, R, prompt, gen, bound   residents as in maps_project_occupancy
+ *                       (ALG1 modes only; else NULL / 0).
+ *   J                   number of candidates.
+ *   cand_prompt, cand_bound   [J] int32.
+ *   choice_out          [J] int32 output decoder index.
+ *   headroom_out        [J] int64 output headroom at the chosen decoder
+ *                       (tokens, or blocks in ALG1 modes); may be NULL.
+ * ---------------------------------------------------------------------- */
+size_t maps_dispatch_workspace_size(int32_t mode, int32_t D, int32_t H,
+                                    int64_t J);
+int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K,
+                  const int32_t *cap, int32_t *Q, const int64_t *res_off,
+                  int64_t R, const int32_t *prompt, const int32_t *gen,
+                  const int32_t *bound, int64_t J, const int32_t *cand_prompt,
+                  const int32_t *cand_bound, int32_t *choice_out,
+                  int64_t *headroom_out, void *ws, size_t ws_bytes,
+                  void *stream);
+
+/* ------------------------------------------------------------------------
+ * Local SJF reordering, Sec. 3.3: Order(Q_k) = argsort of the calibrated
+ * bound, with the maximum-waiting-time promotion.
+ *
+ * Entries are grouped by decoder; within a decoder, entries with
+ * wait > max_wait come first in arrival order, then the rest by ascending
+ * bound, ties by arrival, then by entry index.
+ *
+ *   N, D                entries (N <= INT32_MAX) and decoders (>= 1).
+ *   dec                 [N] int32 decoder of each entry, in [0, D).
+ *   bound               [N] int32 calibrated bound (>= 0).
+ *   wait                [N] int32 steps waited so far.
+ *   arrival             [N] int32 arrival index (>= 0).
+ *   max_wait            promotion threshold in steps.
+ *   perm_out            [N] int32 output: entry indices in queue order.
+ *   seg_off_out         [D+1] int64 output: decoder k's entries are
+ *                       perm_out[seg_off_out[k] .. seg_off_out[k+1]).
+ * ---------------------------------------------------------------------- */
+size_t maps_order_local_workspace_size(int64_t N, int32_t D);
+int maps_order_local(int64_t N, int32_t D, const int32_t *dec,
+                     const int32_t *bound, const int32_t *wait,
+                     const int32_t *arrival, int32_t max_wait,
+                     int32_t *perm_out, int64_t *seg_off_out, void *ws,
+                     size_t ws_bytes, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MAPS_H */

@@ -1,0 +1,217 @@
+// calibrate.cu -- uncertainty-aware calibration (Sec. 3.2) on the GPU.
+//
+// q is the k-th smallest one-sided score s_i = max(0, L_i - Lhat_i) with
+// k = ceil((1 - alpha)(n + 1)).  The scores are unsigned 32-bit (the
+// difference of two int32 values clamped at 0 fits), so q is found by a
+// most-significant-digit radix select over three digits (11, 11, 10 bits):
+// each pass histograms the digit of the scores whose higher digits match the
+// prefix chosen so far, and the last block to finish the pass picks the
+// digit bin that holds rank k.  Nothing returns to the host between passes.
+#include "maps_internal.cuh"
+
+namespace maps {
+namespace {
+
+constexpr int kBins = 2048;
+constexpr int kPasses = 3;
+constexpr int kSelectThreads = 256;
+
+template <int PASS>
+struct Digit;
+template <>
+struct Digit<0> { static constexpr int shift = 21, bits = 11; };
+template <>
+struct Digit<1> { static constexpr int shift = 10, bits = 11; };
+template <>
+struct Digit<2> { static constexpr int shift = 0, bits = 10; };
+
+struct SelectState {
+  unsigned long long hist[kPasses][kBins];  // global digit counts per pass
+  unsigned long long k_rem;                 // rank still to find below prefix
+  uint32_t prefix;                          // digits chosen so far
+  uint32_t done[kPasses];                   // blocks finished per pass
+  int32_t q;                                // the quantile once selected
+};
+
+__device__ __forceinline__ uint32_t score(int32_t L, int32_t P) {
+  long long d = static_cast<long long>(L) - static_cast<long long>(P);
+  return d > 0 ? static_cast<uint32_t>(d) : 0u;
+}
+
+template <int PASS>
+__global__ void __launch_bounds__(kSelectThreads)
+select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
+                   int64_t n, unsigned long long k0, SelectState *st,
+                   int32_t *q_dev_out, int32_t *status) {
+  constexpr int kShift = Digit<PASS>::shift;
+  constexpr uint32_t kMask = (1u << Digit<PASS>::bits) - 1u;
+  constexpr int kPrevShift = PASS == 0 ? 0 : Digit<(PASS > 0 ? PASS - 1 : 0)>::shift;
+  __shared__ uint32_t sh[kBins];
+  __shared__ int s_last;
+  __shared__ unsigned long long s_warp[kSelectThreads / 32];
+
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
+  __syncthreads();
+  const uint32_t prefix = PASS == 0 ? 0u : *reinterpret_cast<volatile uint32_t *>(&st->prefix);
+
+  auto visit = [&](uint32_t s) {
+    if (PASS > 0 && (s >> kPrevShift) != prefix) return;
+    atomicAdd(&sh[(s >> kShift) & kMask], 1u);
+  };
+
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const bool vec = (reinterpret_cast<uintptr_t>(L) % 16 == 0) &&
+                   (reinterpret_cast<uintptr_t>(P) % 16 == 0);
+  int64_t tail_start = 0;
+  if (vec) {
+    const int64_t n4 = n / 4;
+    const int4 *L4 = reinterpret_cast<const int4 *>(L);
+    const int4 *P4 = reinterpret_cast<const int4 *>(P);
+    for (int64_t i = i0; i < n4; i += stride) {
+      const int4 a = __ldg(L4 + i), b = __ldg(P4 + i);
+      visit(score(a.x, b.x));
+      visit(score(a.y, b.y));
+      visit(score(a.z, b.z));
+      visit(score(a.w, b.w));
+    }
+    tail_start = n4 * 4;
+  }
+  for (int64_t i = tail_start + i0; i < n; i += stride) visit(score(__ldg(L + i), __ldg(P + i)));
+  __syncthreads();
+
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x)
+    if (sh[b]) atomicAdd(&st->hist[PASS][b], static_cast<unsigned long long>(sh[b]));
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(&st->done[PASS], 1u) == gridDim.x - 1);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+
+  // The last block: find the bin holding rank k among the survivors.
+  const unsigned long long k =
+      PASS == 0 ? k0 : *reinterpret_cast<volatile unsigned long long *>(&st->k_rem);
+  constexpr int kPer = kBins / kSelectThreads;  // 8 consecutive bins per thread
+  unsigned long long c[kPer], tot = 0;
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    c[j] = __ldcg(&st->hist[PASS][threadIdx.x * kPer + j]);
+    tot += c[j];
+  }
+  // exclusive scan of the per-thread totals
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  unsigned long long incl = tot;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    unsigned long long y = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += y;
+  }
+  if (lane == 31) s_warp[warp] = incl;
+  __syncthreads();
+  unsigned long long excl = incl - tot;
+  for (int w = 0; w < warp; ++w) excl += s_warp[w];
+  if (excl < k && k <= excl + tot) {
+    unsigned long long cum = excl;
+    int d = 0;
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+      if (k <= cum + c[j]) {
+        d = threadIdx.x * kPer + j;
+        break;
+      }
+      cum += c[j];
+    }
+    const uint32_t np = (prefix << Digit<PASS>::bits) | static_cast<uint32_t>(d);
+    st->prefix = np;
+    st->k_rem = k - cum;
+    if (PASS == kPasses - 1) {
+      if (np > 0x7fffffffu) {
+        flag_error(status, MAPS_E_RANGE);
+      } else {
+        st->q = static_cast<int32_t>(np);
+        if (q_dev_out) *q_dev_out = static_cast<int32_t>(np);
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256)
+bound_kernel(const int32_t *__restrict__ pred, int64_t m, const SelectState *st,
+             int32_t *__restrict__ out, int32_t *status) {
+  const long long q = *reinterpret_cast<const volatile int32_t *>(&st->q);
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  bool bad = false;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < m; i += stride) {
+    long long u = static_cast<long long>(__ldg(pred + i)) + q;  // Eq. (conformal_upper)
+    if (u > 0x7fffffffLL) {
+      bad = true;
+      u = 0x7fffffffLL;
+    }
+    out[i] = static_cast<int32_t>(u);
+  }
+  if (bad) flag_error(status, MAPS_E_RANGE);
+}
+
+inline int64_t conformal_rank(int64_t n, uint32_t alpha_ppm) {
+  const int64_t num = static_cast<int64_t>(1000000u - alpha_ppm) * (n + 1);
+  return (num + 999999) / 1000000;
+}
+
+int grid_for(int64_t work, int per_block) {
+  int64_t g = (work + per_block - 1) / per_block;
+  const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
+  if (g > cap) g = cap;
+  if (g < 1) g = 1;
+  return static_cast<int>(g);
+}
+
+}  // namespace
+}  // namespace maps
+
+extern "C" {
+
+size_t maps_calibrate_workspace_size(int64_t n, int64_t m) {
+  (void)n;
+  (void)m;
+  maps::Carve c(nullptr);
+  c.take<maps::SelectState>(1);
+  return c.bytes();
+}
+
+int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
+                   uint32_t alpha_ppm, const int32_t *query_pred, int64_t m,
+                   int32_t *bound_out, int32_t *q_dev_out, int32_t *q_host_out,
+                   void *ws, size_t ws_bytes, void *stream) {
+  using namespace maps;
+  if (n < 0 || n > (int64_t(1) << 40) || alpha_ppm == 0 || alpha_ppm >= 1000000u || m < 0)
+    return MAPS_E_INVALID;
+  if (n > 0 && (true_len == nullptr || pred_len == nullptr)) return MAPS_E_INVALID;
+  if (m > 0 && (query_pred == nullptr || bound_out == nullptr)) return MAPS_E_INVALID;
+  const int64_t k = conformal_rank(n, alpha_ppm);
+  if (k > n) return MAPS_E_UNBOUNDED;  // the quantile is +infinity
+  MAPS_TRY(check_ws(ws, ws_bytes, maps_calibrate_workspace_size(n, m)));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Carve cv(ws);
+  SelectState *st = cv.take<SelectState>(1);
+  int32_t *status = status_word(ws);
+
+  MAPS_TRY(cuda_ok(cudaMemsetAsync(st, 0, sizeof(SelectState), s)));
+  const int g = grid_for(n, kSelectThreads * 16);
+  const unsigned long long kk = static_cast<unsigned long long>(k);
+  select_pass_kernel<0><<<g, kSelectThreads, 0, s>>>(true_len, pred_len, n, kk, st, q_dev_out, status);
+  select_pass_kernel<1><<<g, kSelectThreads, 0, s>>>(true_len, pred_len, n, kk, st, q_dev_out, status);
+  select_pass_kernel<2><<<g, kSelectThreads, 0, s>>>(true_len, pred_len, n, kk, st, q_dev_out, status);
+  MAPS_TRY(launch_ok());
+  if (m > 0) {
+    bound_kernel<<<grid_for(m, 256 * 8), 256, 0, s>>>(query_pred, m, st, bound_out, status);
+    MAPS_TRY(launch_ok());
+  }
+  if (q_host_out != nullptr) {
+    MAPS_TRY(cuda_ok(cudaMemcpyAsync(q_host_out, &st->q, sizeof(int32_t), cudaMemcpyDeviceToHost, s)));
+    return maps_check(ws, stream);
+  }
+  return MAPS_OK;
+}
+
+}  // extern "C"

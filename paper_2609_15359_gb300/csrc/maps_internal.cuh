@@ -1,0 +1,99 @@
+// maps_internal.cuh -- helpers shared by the MAPS CUDA kernels (sm_103a).
+//
+// Nothing here is part of the public ABI (include/maps.h).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "maps.h"
+
+namespace maps {
+
+// ---------------------------------------------------------------------------
+// Workspace: a 256-byte control block followed by per-call scratch carved in
+// 256-byte aligned pieces.  The control block's first word is the sticky
+// device status (MAPS_OK or the first error recorded by a kernel).
+// ---------------------------------------------------------------------------
+constexpr size_t kAlign = 256;
+constexpr size_t kCtrlBytes = 256;
+
+struct Carve {
+  char *base;      // nullptr while only sizing
+  size_t off = kCtrlBytes;
+  explicit Carve(void *b) : base(static_cast<char *>(b)) {}
+  template <class T>
+  T *take(size_t count) {
+    off = (off + kAlign - 1) / kAlign * kAlign;
+    T *p = base ? reinterpret_cast<T *>(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+  size_t bytes() const { return (off + kAlign - 1) / kAlign * kAlign; }
+};
+
+inline int32_t *status_word(void *ws) { return static_cast<int32_t *>(ws); }
+
+// First error wins; later errors do not overwrite it.
+__device__ __forceinline__ void flag_error(int32_t *status, int code) {
+  atomicCAS(status, 0, code);
+}
+
+// Bounded waits: a device-side wait gives up after this many polls (each poll
+// sleeps briefly), records MAPS_E_TIMEOUT and lets the kernel finish.
+constexpr uint32_t kSpinLimit = 1u << 22;
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t *p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long *p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_u32(uint32_t *p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_release_u64(unsigned long long *p, unsigned long long v) {
+  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+void set_last_cuda_error(cudaError_t e);
+
+// Returns MAPS_OK or MAPS_E_CUDA (remembering the CUDA error).
+inline int cuda_ok(cudaError_t e) {
+  if (e == cudaSuccess) return MAPS_OK;
+  set_last_cuda_error(e);
+  return MAPS_E_CUDA;
+}
+inline int launch_ok() { return cuda_ok(cudaGetLastError()); }
+
+inline bool aligned(const void *p, size_t a) {
+  return (reinterpret_cast<uintptr_t>(p) % a) == 0;
+}
+
+// Checks a caller workspace against a required size.
+inline int check_ws(void *ws, size_t ws_bytes, size_t need) {
+  if (ws == nullptr || !aligned(ws, kAlign)) return MAPS_E_INVALID;
+  if (ws_bytes < need) return MAPS_E_WORKSPACE;
+  return MAPS_OK;
+}
+
+int sm_count();           // multiprocessors of the current device
+int max_smem_optin();     // opt-in shared memory per block, bytes
+
+#define MAPS_TRY(expr)            \
+  do {                            \
+    int maps_try_rc_ = (expr);    \
+    if (maps_try_rc_ != MAPS_OK)  \
+      return maps_try_rc_;        \
+  } while (0)
+
+}  // namespace maps

@@ -1,0 +1,457 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle.
+
+Integer work throughout, so every comparison is bit-exact (tolerance 0).
+Sizes: the hand-derived goldens, seeded random instances with ragged shapes
+that span several tiles, and the benchmark workloads at full size (whole
+outputs where the oracle finishes in seconds, sampled candidates otherwise).
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_15359_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+I32_MAX = 2**31 - 1
+
+
+@pytest.fixture(scope="module")
+def M():
+    if not torch.cuda.is_available():
+        pytest.fail("CUDA device required for -m gpu tests")
+    from paper_2609_15359_gb300 import maps
+    return maps
+
+
+@pytest.fixture(scope="module")
+def ws(M):
+    return M.Workspace()
+
+
+def dev(x, dtype=None):
+    a = np.ascontiguousarray(x if dtype is None else np.asarray(x, dtype=dtype))
+    return torch.from_numpy(a).cuda()
+
+
+def host(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+# ---------------------------------------------------------------------------
+# helpers running one op on the GPU and returning (status, outputs)
+# ---------------------------------------------------------------------------
+
+def gpu_calibrate(M, ws, L, P, a, query=None):
+    m = 0 if query is None else len(query)
+    U = torch.empty(max(m, 1), dtype=torch.int32, device="cuda")
+    qd = torch.zeros(1, dtype=torch.int32, device="cuda")
+    st, q = M.maps_calibrate(dev(L, np.int32), dev(P, np.int32), a,
+                             None if query is None else dev(query, np.int32),
+                             U[:m] if m else None, qd, q_host=True, ws=ws)
+    return st, q, int(host(qd)[0]), host(U[:m])
+
+
+def gpu_occupancy(M, ws, D, H, off, p, g, u):
+    K = torch.full((D, H), -7, dtype=torch.int32, device="cuda")
+    st = M.maps_project_occupancy(D, H, dev(off, np.int64), dev(p, np.int32), dev(g, np.int32),
+                                  dev(u, np.int32), K, ws=ws)
+    assert st == 0
+    return M.maps_check(ws), host(K)
+
+
+def gpu_dispatch(M, ws, mode, D, H, S, K, cap, Q, cp, cb, res=None):
+    J = len(cp)
+    Kd = None if K is None else dev(K, np.int32)
+    Qd = dev(Q, np.int32)
+    ch = torch.full((max(J, 1),), -9, dtype=torch.int32, device="cuda")
+    hr = torch.full((max(J, 1),), -9, dtype=torch.int64, device="cuda")
+    kw = {}
+    if res is not None:
+        kw = dict(res_off=dev(res[0], np.int64), prompt=dev(res[1], np.int32),
+                  gen=dev(res[2], np.int32), bound=dev(res[3], np.int32))
+    st = M.maps_dispatch(mode, D, H, S, Kd, dev(cap, np.int32), Qd, dev(cp, np.int32),
+                         dev(cb, np.int32), ch[:J], hr[:J], ws=ws, **kw)
+    assert st == 0, st
+    st = M.maps_check(ws)
+    return st, host(ch[:J]), host(hr[:J]), (None if Kd is None else host(Kd)), host(Qd)
+
+
+def gpu_order(M, ws, D, dec, U, wait, arr, mw):
+    N = len(dec)
+    perm = torch.full((max(N, 1),), -1, dtype=torch.int32, device="cuda")
+    seg = torch.full((D + 1,), -1, dtype=torch.int64, device="cuda")
+    st = M.maps_order_local(D, dev(dec, np.int32), dev(U, np.int32), dev(wait, np.int32),
+                            dev(arr, np.int32), mw, perm[:N], seg, ws=ws)
+    assert st == 0
+    return M.maps_check(ws), host(perm[:N]), host(seg)
+
+
+# ---------------------------------------------------------------------------
+# golden worked examples
+# ---------------------------------------------------------------------------
+
+def test_golden_worked_example(M, ws, golden):
+    c = golden["calibration"]
+    for case in c["cases"]:
+        st, q, qd, _ = gpu_calibrate(M, ws, c["true_len"], c["pred_len"], case["alpha_ppm"])
+        assert st == case["status"]
+        if st == 0:
+            assert q == qd == case["q"]
+    m = c["misround_case"]
+    assert gpu_calibrate(M, ws, m["true_len"], m["pred_len"], m["alpha_ppm"])[1] == m["q"]
+    b = c["bound"]
+    st, q, _, U = gpu_calibrate(M, ws, [9, 9, 9, 9, 9, 9, 9, 9, 13], [9] * 9, 100000, b["pred"])
+    assert st == 0 and q == 4 and U.tolist() == b["U"]
+
+    d, cd = golden["decoders"], golden["candidates"]
+    st, K = gpu_occupancy(M, ws, 2, 8, d["res_off"], d["res_prompt"], d["res_gen"], d["res_bound"])
+    assert st == 0 and K.tolist() == d["K"]
+    res = (d["res_off"], d["res_prompt"], d["res_gen"], d["res_bound"])
+    st, ch, hr, _, _ = gpu_dispatch(M, ws, 0, 2, 8, 1, d["K"], d["cap"], d["Q"], cd["prompt"], cd["bound"])
+    assert st == 0 and ch.tolist() == golden["snapshot"]["choice"]
+    assert hr.tolist() == golden["snapshot"]["headroom"]
+    s = golden["sequential"]
+    st, ch, hr, Ka, Qa = gpu_dispatch(M, ws, 1, 2, 8, 1, d["K"], d["cap"], d["Q"], cd["prompt"], cd["bound"])
+    assert st == 0 and ch.tolist() == s["choice"] and hr.tolist() == s["headroom"]
+    assert Ka.tolist() == s["K_after"] and Qa.tolist() == s["Q_after"]
+    a = golden["alg1"]
+    st, ch, hr, _, _ = gpu_dispatch(M, ws, 2, 2, 8, 1, None, d["cap"], d["Q"], cd["prompt"], cd["bound"], res)
+    assert st == 0 and ch.tolist() == a["choice"] and hr.tolist() == a["headroom"]
+    st, ch, hr, _, Qa = gpu_dispatch(M, ws, 3, 2, 8, 1, None, d["cap"], d["Q"], cd["prompt"], cd["bound"], res)
+    assert st == 0 and ch.tolist() == a["sequential_choice"]
+    assert hr.tolist() == a["sequential_headroom"] and Qa.tolist() == a["sequential_Q_after"]
+    o = golden["order"]
+    st, perm, seg = gpu_order(M, ws, 1, o["dec"], o["bound"], o["wait"], o["arrival"], o["max_wait"])
+    assert st == 0 and perm.tolist() == o["perm"] and seg.tolist() == o["seg_off"]
+
+
+# ---------------------------------------------------------------------------
+# calibration
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n", [1, 2, 3, 9, 10, 1000, 4097, 65537, 1000003])
+def test_calibrate_random(M, ws, oracle, n):
+    rng = np.random.default_rng(n)
+    L = rng.integers(-(2**31), 2**31, n, dtype=np.int64).astype(np.int32) if n % 2 else \
+        rng.integers(0, 3000, n).astype(np.int32)
+    P = rng.integers(-(2**31), 2**31, n, dtype=np.int64).astype(np.int32) if n % 3 == 0 else \
+        rng.integers(0, 3000, n).astype(np.int32)
+    if n > 10:
+        P[: n // 4] = L[: n // 4]  # exact zeros
+    query = rng.integers(0, 5000, 4099).astype(np.int32)
+    for a in (1, 50000, 100000, 200000, 900000, 999999):
+        sto, qo = oracle.calibrate(L, P, a)
+        st, q, qd, U = gpu_calibrate(M, ws, L, P, a, query)
+        assert st == sto, (n, a)
+        if st == 0:
+            assert q == qd == qo
+            assert np.array_equal(U, oracle.bound(query, qo)[1])
+
+
+def test_calibrate_unaligned_and_ranges(M, ws, oracle):
+    rng = np.random.default_rng(3)
+    L = rng.integers(0, 10**6, 10001).astype(np.int32)
+    P = rng.integers(0, 10**6, 10001).astype(np.int32)
+    Ld, Pd = dev(L), dev(P)
+    qd = torch.zeros(1, dtype=torch.int32, device="cuda")
+    st, q = M.maps_calibrate(Ld[1:], Pd[1:], 100000, q_dev_out=qd, q_host=True, ws=ws)
+    assert st == 0 and q == oracle.calibrate(L[1:], P[1:], 100000)[1]
+    # score above INT32_MAX -> range error
+    st, _ = M.maps_calibrate(dev([I32_MAX] * 3, np.int32), dev([-5] * 3, np.int32), 500000,
+                             q_host=True, ws=ws)
+    assert st == M.MAPS_E_RANGE
+    # bound above INT32_MAX -> range error
+    U = torch.empty(1, dtype=torch.int32, device="cuda")
+    st, _ = M.maps_calibrate(dev([10] * 3, np.int32), dev([0] * 3, np.int32), 500000,
+                             dev([I32_MAX - 3], np.int32), U, q_host=True, ws=ws)
+    assert st == M.MAPS_E_RANGE
+    # rank above n: unbounded, returned at once
+    assert gpu_calibrate(M, ws, [1] * 8, [0] * 8, 100000)[0] == M.MAPS_E_UNBOUNDED
+    assert gpu_calibrate(M, ws, [], [], 100000)[0] == M.MAPS_E_UNBOUNDED
+    assert M.maps_calibrate(Ld, Pd, 0, ws=ws)[0] == M.MAPS_E_INVALID
+
+
+@pytest.mark.parametrize("name", ["tiny", "d16", "d64", "large"])
+def test_calibrate_workloads(M, ws, oracle, name):
+    w = W.make(name)
+    query = np.concatenate([w["res_pred"], w["cand_pred"]])
+    for a in w["alphas_ppm"]:
+        sto, qo = oracle.calibrate(w["cal_true"], w["cal_pred"], a)
+        st, q, qd, U = gpu_calibrate(M, ws, w["cal_true"], w["cal_pred"], a, query)
+        assert st == sto == 0 and q == qd == qo
+        assert np.array_equal(U, oracle.bound(query, qo)[1])
+
+
+# ---------------------------------------------------------------------------
+# occupancy
+# ---------------------------------------------------------------------------
+
+def random_residents(rng, D, H, per_max, with_empty=True):
+    R_per = rng.integers(0 if with_empty else 1, per_max + 1, D)
+    off = np.concatenate([[0], np.cumsum(R_per)]).astype(np.int64)
+    R = int(off[-1])
+    p = rng.integers(0, 3000, R).astype(np.int32)
+    g = rng.integers(0, 2 * H + 3, R).astype(np.int32)
+    U = rng.integers(0, 3 * H + 5, R).astype(np.int32)
+    return off, p, g, U
+
+
+@pytest.mark.parametrize("D,H", [(1, 1), (3, 3), (2, 8), (5, 511), (4, 512), (3, 513), (7, 4095),
+                                 (2, 4097), (9, 4100), (3, 12289), (2, 65536)])
+def test_occupancy_random(M, ws, oracle, D, H):
+    rng = np.random.default_rng(D * 100003 + H)
+    off, p, g, U = random_residents(rng, D, H, 700)
+    sto, Ko = oracle.occupancy(D, H, off, p, g, U)
+    st, K = gpu_occupancy(M, ws, D, H, off, p, g, U)
+    assert st == sto == 0
+    assert np.array_equal(K, Ko)
+
+
+@pytest.mark.parametrize("name", ["tiny", "d16", "d64", "large"])
+def test_occupancy_workloads(M, ws, oracle, name):
+    w = W.make(name)
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    sto, Ko = oracle.occupancy(w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U)
+    st, K = gpu_occupancy(M, ws, w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U)
+    assert st == sto == 0
+    assert np.array_equal(K, Ko)
+
+
+def test_occupancy_errors(M, ws, oracle):
+    # K above INT32_MAX
+    big = I32_MAX // 2
+    st, _ = gpu_occupancy(M, ws, 1, 4, [0, 2], [big, big], [0, 0], [4, 4])
+    assert st == M.MAPS_E_RANGE == oracle.occupancy(1, 4, [0, 2], [big, big], [0, 0], [4, 4])[0]
+    st, K = gpu_occupancy(M, ws, 1, 4, [0, 1], [I32_MAX - 4], [0], [4])
+    assert st == 0 and K[0].tolist() == [I32_MAX - 3, I32_MAX - 2, I32_MAX - 1, I32_MAX]
+    st, _ = gpu_occupancy(M, ws, 1, 8, [0, 1], [-1], [0], [3])
+    assert st == M.MAPS_E_RANGE
+    st, _ = gpu_occupancy(M, ws, 2, 8, [0, 2, 1], [1, 1], [0, 0], [3, 3])
+    assert st == M.MAPS_E_RANGE
+    st, _ = gpu_occupancy(M, ws, 1, 8, [0, 5], [1, 1], [0, 0], [3, 3])  # beyond R
+    assert st == M.MAPS_E_RANGE
+    K = torch.empty((1, 8), dtype=torch.int32, device="cuda")
+    assert M.maps_project_occupancy(0, 8, dev([0], np.int64), dev([1], np.int32), dev([0], np.int32),
+                                    dev([1], np.int32), K, ws=ws) == M.MAPS_E_INVALID
+
+
+# ---------------------------------------------------------------------------
+# dispatch
+# ---------------------------------------------------------------------------
+
+def diverse_caps(rng, K, spread):
+    """Capacities straddling each decoder's occupancy so that the feasible set
+    changes from candidate to candidate (test input built from the oracle)."""
+    base = K[:, 0].astype(np.int64)
+    cap = base + rng.integers(-spread, 3 * spread, K.shape[0])
+    return np.clip(cap, 0, I32_MAX).astype(np.int32)
+
+
+def check_dispatch(M, ws, oracle, mode, D, H, K, cap, Q, cp, cb, S=1, res=None):
+    sto, co, ho, Ko, Qo = oracle.dispatch(mode, D, H, S, K, cap, Q, cp, cb,
+                                          *(res if res is not None else ()))
+    st, ch, hr, Ka, Qa = gpu_dispatch(M, ws, mode, D, H, S, K, cap, Q, cp, cb, res)
+    assert st == sto
+    if st == 0:
+        assert np.array_equal(ch, co)
+        assert np.array_equal(hr, ho)
+        if mode == 1:
+            assert np.array_equal(Ka, Ko)
+        assert np.array_equal(Qa, Qo)
+    return co, ho
+
+
+@pytest.mark.parametrize("D,H,J", [(1, 1, 1), (1, 9, 33), (2, 8, 40), (3, 100, 700), (5, 511, 1000),
+                                   (17, 4100, 3000), (64, 4096, 5000), (255, 1000, 3000),
+                                   (256, 8192, 6000), (257, 2048, 2000), (300, 777, 1500),
+                                   (1024, 1024, 2000)])
+def test_dispatch_snapshot_random(M, ws, oracle, D, H, J):
+    rng = np.random.default_rng(D * 7919 + H)
+    off, p, g, U = random_residents(rng, D, H, 40)
+    _, K = oracle.occupancy(D, H, off, p, g, U)
+    cap = diverse_caps(rng, K, 4000)
+    Q = rng.integers(0, 4, D).astype(np.int32)
+    cp = rng.integers(0, 3000, J).astype(np.int32)
+    cb = rng.integers(0, 2 * H + 2, J).astype(np.int32)
+    co, ho = check_dispatch(M, ws, oracle, 0, D, H, K, cap, Q, cp, cb)
+    if J >= 100:
+        assert (ho >= 0).any() and (ho < 0).any()  # both branches exercised
+        assert len(set(co.tolist())) > 1
+
+
+@pytest.mark.parametrize("name", ["tiny", "d16", "d64"])
+@pytest.mark.parametrize("variant", ["given", "feasible", "diverse"])
+def test_dispatch_snapshot_workloads(M, ws, oracle, name, variant):
+    w = W.make(name, feasible=(variant == "feasible"))
+    rng = np.random.default_rng(11)
+    for a in w["alphas_ppm"]:
+        q = oracle.calibrate(w["cal_true"], w["cal_pred"], a)[1]
+        U = oracle.bound(w["res_pred"], q)[1]
+        cb = oracle.bound(w["cand_pred"], q)[1]
+        _, K = oracle.occupancy(w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U)
+        cap, Q = w["cap"], w["Q"]
+        if variant == "diverse":
+            cap = diverse_caps(rng, K, 3000)
+            Q = rng.integers(0, 3, w["D"]).astype(np.int32)
+        check_dispatch(M, ws, oracle, 0, w["D"], w["H"], K, cap, Q, w["cand_prompt"], cb)
+
+
+@pytest.mark.parametrize("variant", ["given", "feasible", "diverse"])
+def test_dispatch_snapshot_large_sampled(M, ws, oracle, variant):
+    """Full-size run on the GPU in the benchmark's launch configuration;
+    the oracle scores a sample of the candidates one by one."""
+    w = W.make("large", feasible=(variant == "feasible"))
+    D, H, J = w["D"], w["H"], w["J"]
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    cb = oracle.bound(w["cand_pred"], q)[1]
+    _, K = oracle.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U)
+    cap, Q = w["cap"], w["Q"]
+    rng = np.random.default_rng(5)
+    if variant == "diverse":
+        cap = diverse_caps(rng, K, 6000)
+        Q = rng.integers(0, 3, D).astype(np.int32)
+    st, ch, hr, _, _ = gpu_dispatch(M, ws, 0, D, H, 1, K, cap, Q, w["cand_prompt"], cb)
+    assert st == 0
+    assert ch.min() >= 0 and ch.max() < D
+    idx = np.concatenate([np.argsort(cb)[-64:], rng.choice(J, 1500, replace=False)])
+    sto, co, ho, _, _ = oracle.dispatch(0, D, H, 1, K, cap, Q, w["cand_prompt"][idx], cb[idx])
+    assert sto == 0
+    assert np.array_equal(ch[idx], co)
+    assert np.array_equal(hr[idx], ho)
+
+
+@pytest.mark.parametrize("D,H,J", [(1, 5, 20), (2, 8, 50), (3, 100, 300), (7, 513, 400),
+                                   (32, 2048, 256), (100, 1000, 300), (1024, 64, 100)])
+def test_dispatch_sequential_random(M, ws, oracle, D, H, J):
+    rng = np.random.default_rng(D * 31 + H)
+    off, p, g, U = random_residents(rng, D, H, 30)
+    _, K = oracle.occupancy(D, H, off, p, g, U)
+    cap = diverse_caps(rng, K, 3000)
+    Q = rng.integers(0, 3, D).astype(np.int32)
+    cp = rng.integers(0, 500, J).astype(np.int32)
+    cb = rng.integers(0, H + 5, J).astype(np.int32)
+    check_dispatch(M, ws, oracle, 1, D, H, K, cap, Q, cp, cb)
+
+
+@pytest.mark.parametrize("name", ["tiny", "d16"])
+def test_dispatch_sequential_workloads(M, ws, oracle, name):
+    w = W.make(name, feasible=True)
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    cb = oracle.bound(w["cand_pred"], q)[1]
+    _, K = oracle.occupancy(w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U)
+    check_dispatch(M, ws, oracle, 1, w["D"], w["H"], K, w["cap"], w["Q"], w["cand_prompt"], cb)
+
+
+@pytest.mark.parametrize("S", [1, 16])
+@pytest.mark.parametrize("name", ["tiny", "d16", "d64", "large"])
+def test_dispatch_alg1_workloads(M, ws, oracle, name, S):
+    w = W.make(name, feasible=True)
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    cb = oracle.bound(w["cand_pred"], q)[1]
+    res = (w["res_off"], w["res_prompt"], w["res_gen"], U)
+    rng = np.random.default_rng(S)
+    cap = (w["cap"].astype(np.int64) // 2 + rng.integers(0, w["cap"].max() // 8, w["D"])).astype(np.int32)
+    Q = rng.integers(0, 3, w["D"]).astype(np.int32)
+    co, ho = check_dispatch(M, ws, oracle, 2, w["D"], w["H"], None, cap, Q, w["cand_prompt"], cb, S, res)
+    if name != "large":
+        J = min(w["J"], 2048)
+        check_dispatch(M, ws, oracle, 3, w["D"], w["H"], None, cap, Q, w["cand_prompt"][:J], cb[:J], S, res)
+
+
+def test_dispatch_errors(M, ws, oracle):
+    K = np.zeros((2, 8), np.int32)
+    st, ch, _, _, _ = gpu_dispatch(M, ws, 0, 2, 8, 1, K, [5, 5], [0, 0], [1, -1], [2, 2])
+    assert st == M.MAPS_E_RANGE and ch[1] == -1
+    K[1, 3] = -1
+    assert gpu_dispatch(M, ws, 0, 2, 8, 1, K, [5, 5], [0, 0], [1], [2])[0] == M.MAPS_E_RANGE
+    assert gpu_dispatch(M, ws, 1, 2, 8, 1, K, [5, 5], [0, 0], [1], [2])[0] == M.MAPS_E_RANGE
+    assert gpu_dispatch(M, ws, 0, 2, 8, 1, np.zeros((2, 8), np.int32), [5, -5], [0, 0], [1], [2])[0] \
+        == M.MAPS_E_RANGE
+    ch = torch.empty(1, dtype=torch.int32, device="cuda")
+    z = dev([0, 0], np.int32)
+    Kd = dev(np.zeros((2, 8), np.int32))
+    assert M.maps_dispatch(7, 2, 8, 1, Kd, z, z, dev([1], np.int32), dev([1], np.int32), ch,
+                           ws=ws) == M.MAPS_E_INVALID
+    assert M.maps_dispatch(0, 1025, 8, 1, Kd, z, z, dev([1], np.int32), dev([1], np.int32), ch,
+                           ws=ws) == M.MAPS_E_INVALID
+    small = M.Workspace(256)
+    assert M.lib.maps_dispatch(0, 2, 8, 1, M._ptr(Kd), M._ptr(z), M._ptr(z), None, 0, None, None,
+                               None, 1, M._ptr(dev([1], np.int32)), M._ptr(dev([1], np.int32)),
+                               M._ptr(ch), None, small.ptr, 256, M._stream(None)) == M.MAPS_E_WORKSPACE
+
+
+# ---------------------------------------------------------------------------
+# local order
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("N,D,sorted_arrival", [(0, 3, True), (1, 1, True), (2, 2, False),
+                                                (100, 3, False), (4096, 8, True), (4097, 8, False),
+                                                (50000, 64, True), (50001, 300, False),
+                                                (300000, 256, False), (1000, 70000, True)])
+def test_order_random(M, ws, oracle, N, D, sorted_arrival):
+    rng = np.random.default_rng(N + D)
+    dec = rng.integers(0, D, N).astype(np.int32)
+    U = rng.integers(0, 60 if N < 5000 else 2**31 - 1, N, dtype=np.int64).astype(np.int32)
+    wait = rng.integers(-10, 3000, N).astype(np.int32)
+    if sorted_arrival:
+        arr = np.sort(rng.integers(0, max(N // 2, 1), N)).astype(np.int32)
+    else:
+        arr = rng.integers(0, 2**31 - 1, N, dtype=np.int64).astype(np.int32)
+        arr[: N // 3] = rng.integers(0, 50, N // 3)  # ties on arrival too
+    sto, po, so = oracle.order_local(D, dec, U, wait, arr, 1000)
+    st, perm, seg = gpu_order(M, ws, D, dec, U, wait, arr, 1000)
+    assert st == sto == 0
+    assert np.array_equal(perm, po)
+    assert np.array_equal(seg, so)
+
+
+def test_order_degenerate_keys(M, ws, oracle):
+    # every key identical: all digit passes trivial -> identity order
+    N = 9000
+    z = np.zeros(N, np.int32)
+    st, perm, seg = gpu_order(M, ws, 1, z, z, z, z, 5)
+    assert st == 0 and np.array_equal(perm, np.arange(N)) and seg.tolist() == [0, N]
+    st, perm, _ = gpu_order(M, ws, 2, [3], [1], [0], [0], 5)
+    assert st == M.MAPS_E_RANGE
+
+
+@pytest.mark.parametrize("name", ["d64", "large"])
+def test_order_workload_pipeline(M, ws, oracle, name):
+    """The benchmark's order step: residents plus dispatched candidates."""
+    w = W.make(name)
+    R, J, D = w["R"], w["J"], w["D"]
+    rng = np.random.default_rng(1)
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(np.concatenate([w["res_pred"], w["cand_pred"]]), q)[1]
+    dec = np.concatenate([w["res_dec"], rng.integers(0, D, J).astype(np.int32)])
+    wait = np.concatenate([w["res_wait"], np.zeros(J, np.int32)])
+    arr = np.arange(R + J, dtype=np.int32)
+    sto, po, so = oracle.order_local(D, dec, U, wait, arr, w["max_wait"])
+    st, perm, seg = gpu_order(M, ws, D, dec, U, wait, arr, w["max_wait"])
+    assert st == sto == 0
+    assert np.array_equal(perm, po) and np.array_equal(seg, so)
+
+
+# ---------------------------------------------------------------------------
+# determinism
+# ---------------------------------------------------------------------------
+
+def test_repeat_runs_identical(M, ws, oracle):
+    w = W.make("d64")
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], 100000)[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    cb = oracle.bound(w["cand_pred"], q)[1]
+    outs = []
+    for _ in range(3):
+        _, K = gpu_occupancy(M, ws, w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U)
+        _, ch, hr, _, _ = gpu_dispatch(M, ws, 0, w["D"], w["H"], 1, K, w["cap"], w["Q"],
+                                       w["cand_prompt"], cb)
+        outs.append((K, ch, hr))
+    for o in outs[1:]:
+        assert all(np.array_equal(x, y) for x, y in zip(o, outs[0]))
