@@ -1,0 +1,493 @@
+"""Benchmark of the MAPS scheduler hot path on GB300.
+
+One step = one pass of the whole hot path over one batch of the Large
+workload (D=256 decoders x 4,096 residents, H=65,536, 65,536 candidates,
+n=1,000,000 calibration residuals, alpha=0.1):
+    maps_calibrate (q, then bounds for residents and candidates)
+    -> maps_project_occupancy (K, 256 x 65,536)
+    -> maps_dispatch SNAPSHOT (a decoder for every candidate)
+    -> maps_order_local (queue order of residents + dispatched candidates).
+The metric is dispatch decisions per second (candidates decided per step /
+step time); occupancy cells per second is reported beside it.
+
+Timing: inputs resident in HBM; before every step the L2 is flushed (a
+256 MiB memset) and the GPU is kept busy by a short sleep kernel while the
+host enqueues the step, so CUDA events on the launching stream bracket the
+device time of the step alone.  The end-to-end figure repeats the step
+through the same C-ABI calls with pinned host buffers, host-to-device copies
+of every input and device-to-host copies of every output inside the timed
+region.
+
+--impl reference runs the CPU oracle on the host cores over a bounded
+sample of the same workload and prints the same metric.
+Multi-GPU (torchrun): every rank runs an independent replica (its own
+scheduler instance with its own seed); there is no collective on the data
+path.  The value is all ranks' decisions over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "dispatch decisions/sec and occupancy cells/sec on 1 GB300; % of HBM peak"
+UNIT = "decisions/s"
+WORKLOAD = "large"
+L2_FLUSH_BYTES = 256 << 20
+
+# DRAM traffic of the occupancy kernel on this workload from an ncu capture
+# (dram__bytes_read.sum + dram__bytes_write.sum, one launch), valid only for
+# the kernel source it was taken on.
+TRAFFIC = {
+    "occupancy": {"bytes": None, "source_sha256": None,
+                  "profile": "profiles/occupancy_large.md"},
+}
+
+
+def _sha256(path: str) -> str:
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def measured_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "source": "fallback"}
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (replicas only)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def aggregate(local_seconds: float, local_units: float, dist=None):
+    """Max of the ranks' timed seconds and sum of their units (decisions)."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return local_seconds, local_units
+    import torch
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([local_seconds], dtype=torch.float64, device=dev)
+    u = torch.tensor([local_units], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines: list[str] = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.gpu)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": float(np.median(sm)) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# the GPU step
+# ---------------------------------------------------------------------------
+
+class Step:
+    """Device buffers and the four C-ABI calls of one hot-path pass."""
+
+    KERNELS_PER_STEP = None  # set in __init__
+
+    def __init__(self, w: dict, device):
+        import torch
+        from paper_2609_15359_gb300 import maps as M
+        self.M, self.torch, self.w = M, torch, w
+        self.D, self.H, self.R, self.J = w["D"], w["H"], w["R"], w["J"]
+        self.alpha = w["alphas_ppm"][0]
+        t = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(device)  # noqa: E731
+        R, J = self.R, self.J
+        # inputs (resident in HBM)
+        self.cal_true, self.cal_pred = t(w["cal_true"]), t(w["cal_pred"])
+        self.pred_all = t(np.concatenate([w["res_pred"], w["cand_pred"]]))
+        self.res_off, self.res_prompt, self.res_gen = t(w["res_off"]), t(w["res_prompt"]), t(w["res_gen"])
+        self.cap, self.Q0 = t(w["cap"]), t(w["Q"])
+        self.cand_prompt = t(w["cand_prompt"])
+        self.wait_all = t(np.concatenate([w["res_wait"], np.zeros(J, np.int32)]))
+        self.arrival = t(np.arange(R + J, dtype=np.int32))
+        # outputs / intermediates
+        self.U_all = torch.empty(R + J, dtype=torch.int32, device=device)
+        self.q = torch.empty(1, dtype=torch.int32, device=device)
+        self.K = torch.empty((self.D, self.H), dtype=torch.int32, device=device)
+        self.dec_all = t(np.concatenate([w["res_dec"], np.zeros(J, np.int32)]))
+        self.choice = self.dec_all[R:]
+        self.headroom = torch.empty(J, dtype=torch.int64, device=device)
+        self.perm = torch.empty(R + J, dtype=torch.int32, device=device)
+        self.seg = torch.empty(self.D + 1, dtype=torch.int64, device=device)
+        need = max(M.lib.maps_calibrate_workspace_size(w["n_cal"], R + J),
+                   M.lib.maps_project_occupancy_workspace_size(self.D, self.H, R),
+                   M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, self.D, self.H, J),
+                   M.lib.maps_order_local_workspace_size(R + J, self.D))
+        self.ws = M.Workspace(need, device)
+        dbits = (self.D - 1).bit_length()
+        n_hi = min(8, (32 + dbits + 7) // 8)
+        # calibrate 4, occupancy 1, dispatch 4, order 2 + 4 + n_hi + 2
+        self.kernels_per_step = 4 + 1 + 4 + (2 + 4 + n_hi + 2)
+
+    def run(self, ev=None):
+        M, R = self.M, self.R
+        st, _ = M.maps_calibrate(self.cal_true, self.cal_pred, self.alpha, self.pred_all,
+                                 self.U_all, self.q, ws=self.ws)
+        assert st == 0, st
+        if ev:
+            ev[0].record()
+        st = M.maps_project_occupancy(self.D, self.H, self.res_off, self.res_prompt,
+                                      self.res_gen, self.U_all[:R], self.K, ws=self.ws)
+        assert st == 0, st
+        if ev:
+            ev[1].record()
+        st = M.maps_dispatch(M.MODE_SNAPSHOT, self.D, self.H, 1, self.K, self.cap, self.Q0,
+                             self.cand_prompt, self.U_all[R:], self.choice, self.headroom,
+                             ws=self.ws)
+        assert st == 0, st
+        if ev:
+            ev[2].record()
+        st = M.maps_order_local(self.D, self.dec_all, self.U_all, self.wait_all, self.arrival,
+                                self.w["max_wait"], self.perm, self.seg, ws=self.ws)
+        assert st == 0, st
+
+    def check(self):
+        st = self.M.maps_check(self.ws)
+        if st != 0:
+            raise RuntimeError(f"device status {st}")
+
+
+def host_inputs(w):
+    """Pinned host copies of every per-step input and output of the e2e path."""
+    import torch
+    R, J = w["R"], w["J"]
+    pin = lambda x: torch.from_numpy(np.ascontiguousarray(x)).pin_memory()  # noqa: E731
+    ins = {
+        "cal_true": pin(w["cal_true"]), "cal_pred": pin(w["cal_pred"]),
+        "pred_all": pin(np.concatenate([w["res_pred"], w["cand_pred"]])),
+        "res_off": pin(w["res_off"]), "res_prompt": pin(w["res_prompt"]),
+        "res_gen": pin(w["res_gen"]), "cap": pin(w["cap"]), "Q0": pin(w["Q"]),
+        "cand_prompt": pin(w["cand_prompt"]),
+        "wait_all": pin(np.concatenate([w["res_wait"], np.zeros(J, np.int32)])),
+        "arrival": pin(np.arange(R + J, dtype=np.int32)),
+        "res_dec": pin(w["res_dec"]),
+    }
+    outs = {
+        "choice": torch.empty(J, dtype=torch.int32).pin_memory(),
+        "headroom": torch.empty(J, dtype=torch.int64).pin_memory(),
+        "perm": torch.empty(R + J, dtype=torch.int32).pin_memory(),
+        "seg": torch.empty(w["D"] + 1, dtype=torch.int64).pin_memory(),
+        "q": torch.empty(1, dtype=torch.int32).pin_memory(),
+    }
+    return ins, outs
+
+
+def e2e_step(step: Step, ins: dict, outs: dict):
+    s = step
+    R = s.R
+    s.cal_true.copy_(ins["cal_true"], non_blocking=True)
+    s.cal_pred.copy_(ins["cal_pred"], non_blocking=True)
+    s.pred_all.copy_(ins["pred_all"], non_blocking=True)
+    s.res_off.copy_(ins["res_off"], non_blocking=True)
+    s.res_prompt.copy_(ins["res_prompt"], non_blocking=True)
+    s.res_gen.copy_(ins["res_gen"], non_blocking=True)
+    s.cap.copy_(ins["cap"], non_blocking=True)
+    s.Q0.copy_(ins["Q0"], non_blocking=True)
+    s.cand_prompt.copy_(ins["cand_prompt"], non_blocking=True)
+    s.wait_all.copy_(ins["wait_all"], non_blocking=True)
+    s.arrival.copy_(ins["arrival"], non_blocking=True)
+    s.dec_all[:R].copy_(ins["res_dec"], non_blocking=True)
+    s.run()
+    outs["choice"].copy_(s.choice, non_blocking=True)
+    outs["headroom"].copy_(s.headroom, non_blocking=True)
+    outs["perm"].copy_(s.perm, non_blocking=True)
+    outs["seg"].copy_(s.seg, non_blocking=True)
+    outs["q"].copy_(s.q, non_blocking=True)
+
+
+def bench_gpu(args, world, rank, local, dist):
+    import torch
+    from paper_2609_15359_gb300 import workloads as W
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    w = W.make(WORKLOAD, seed=None if rank == 0 else 4 + 1000 * rank)
+    step = Step(w, device)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+    sleep_cycles = int(1.5e6)  # ~1 ms at GB300 clocks: covers host enqueue of a step
+
+    for _ in range(max(args.warmup, 3)):
+        step.run()
+    torch.cuda.synchronize()
+    step.check()
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    sampler = ClockSampler(local)
+    if dist is not None and dist.is_initialized():
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)
+    for i in range(K):
+        flush.zero_()
+        torch.cuda._sleep(sleep_cycles)
+        e = ev[i]
+        e[3].record()
+        step.run(ev=e)
+        e[4].record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    if dist is not None and dist.is_initialized():
+        dist.barrier()
+    step.check()
+    step_ms = [ev[i][3].elapsed_time(ev[i][4]) for i in range(K)]
+    occ_ms = [ev[i][0].elapsed_time(ev[i][1]) for i in range(K)]
+    disp_ms = [ev[i][1].elapsed_time(ev[i][2]) for i in range(K)]
+    cal_ms = [ev[i][3].elapsed_time(ev[i][0]) for i in range(K)]
+    order_ms = [ev[i][2].elapsed_time(ev[i][4]) for i in range(K)]
+    local_s = sum(step_ms) / 1e3
+    max_s, units = aggregate(local_s, float(K * step.J), dist)
+
+    # end to end through the public API with host buffers
+    ins, outs = host_inputs(w)
+    h2d = sum(v.numel() * v.element_size() for v in ins.values())
+    d2h = sum(v.numel() * v.element_size() for v in outs.values())
+    for _ in range(2):
+        e2e_step(step, ins, outs)
+    torch.cuda.synchronize()
+    Ke = max(5, min(K, 50))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(Ke):
+        e2e_step(step, ins, outs)
+    e1.record()
+    torch.cuda.synchronize()
+    step.check()
+    e2e_s = e0.elapsed_time(e1) / 1e3
+    e2e_max, e2e_units = aggregate(e2e_s, float(Ke * step.J), dist)
+
+    peaks = measured_peaks()
+    D, H, R, J = step.D, step.H, step.R, step.J
+    occ_bytes = 12 * R + 4 * D * H + 8 * (D + 1)  # residents in, K out, offsets
+    occ_avg = float(np.mean(occ_ms)) / 1e3
+    achieved = occ_bytes / occ_avg / 1e9
+    tr = TRAFFIC["occupancy"]
+    occ_src = os.path.join(ROOT, "paper_2609_15359_gb300", "csrc", "occupancy.cu")
+    traffic = tr["bytes"] if (tr["bytes"] and tr["source_sha256"] == _sha256(occ_src)) else None
+    disp_bytes = 4 * D * H + 8 * J + 12 * J + 8 * D  # K, candidates, choice+headroom, cap+Q
+    disp_avg = float(np.mean(disp_ms)) / 1e3
+    ms_per_step = max_s / K * 1e3
+    result = {
+        "metric": METRIC,
+        "value": units / max_s,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int32",
+        "data": "synthetic",
+        "config": {
+            "workload": "Large: D=256 decoders x 4,096 residents (1,048,576), capacity 524,288, "
+                        "H=65,536, 65,536 candidates, calibration n=1,000,000, alpha=0.1",
+            "D": D, "H": H, "residents": R, "candidates": J, "n_cal": w["n_cal"],
+            "alpha_ppm": step.alpha, "dispatch_mode": "SNAPSHOT",
+            "l2": "flushed before every step (256 MiB memset)",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+        },
+        "occupancy_cells_per_s": K * D * H * world / max_s,
+        "kernels_ms": {"calibrate": float(np.mean(cal_ms)), "occupancy": float(np.mean(occ_ms)),
+                       "dispatch": float(np.mean(disp_ms)), "order": float(np.mean(order_ms))},
+        "roofline": {"kernel": "occupancy_kernel (maps_project_occupancy)", "bound": "hbm",
+                     "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
+                     "algorithmic_bytes": occ_bytes, "peak_source": peaks["source"]},
+        "roofline_dispatch": {"scope": "whole maps_dispatch call (bucketing + main kernel)",
+                              "bound": "hbm", "achieved": disp_bytes / disp_avg / 1e9,
+                              "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                              "frac": disp_bytes / disp_avg / 1e9 / peaks["hbm_gbs"],
+                              "algorithmic_bytes": disp_bytes},
+        "e2e": {"value": e2e_units / e2e_max, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": step.kernels_per_step * K,
+        "clocks": clocks,
+    }
+    return result, w
+
+
+# ---------------------------------------------------------------------------
+# the CPU oracle as the baseline / reference arm
+# ---------------------------------------------------------------------------
+
+def oracle_step(w: dict, n_dispatch: int) -> tuple[float, int]:
+    """Runs the oracle over the whole step except that only the first
+    n_dispatch candidates are dispatched; returns (seconds extrapolated to all
+    candidates, candidates the extrapolation stands for)."""
+    import oracle as O
+    R, J, D, H = w["R"], w["J"], w["D"], w["H"]
+    a = w["alphas_ppm"][0]
+    t0 = time.perf_counter()
+    st, q = O.calibrate(w["cal_true"], w["cal_pred"], a)
+    st, U = O.bound(np.concatenate([w["res_pred"], w["cand_pred"]]), q)
+    st, K = O.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U[:R])
+    t1 = time.perf_counter()
+    st, ch, _, _, _ = O.dispatch(0, D, H, 1, K, w["cap"], w["Q"], w["cand_prompt"][:n_dispatch],
+                                 U[R:R + n_dispatch])
+    t2 = time.perf_counter()
+    dec = np.concatenate([w["res_dec"], np.resize(ch, J).astype(np.int32)])
+    wait = np.concatenate([w["res_wait"], np.zeros(J, np.int32)])
+    st, perm, seg = O.order_local(D, dec, U, wait, np.arange(R + J, dtype=np.int32), w["max_wait"])
+    t3 = time.perf_counter()
+    fixed = (t1 - t0) + (t3 - t2)
+    return fixed + (t2 - t1) * J / n_dispatch, J
+
+
+def cpu_baseline(w: dict, n_dispatch: int = 8192) -> dict:
+    secs, J = oracle_step(w, n_dispatch)
+    return {"value": J / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": (f"full calibration, bounds, occupancy and order of the Large workload; "
+                       f"dispatch of the first {n_dispatch} of {J} candidates, its time scaled "
+                       f"by {J}/{n_dispatch}; single thread")}
+
+
+def bench_reference(args, world, rank):
+    if rank != 0:
+        return None
+    from paper_2609_15359_gb300 import workloads as W
+    import oracle
+    oracle.build()
+    w = W.make(WORKLOAD)
+    budget = 150.0 / max(1, args.steps + args.warmup)  # seconds per oracle step
+    n_dispatch = int(np.clip(512 * budget / 2.0, 64, 4096))
+    for _ in range(args.warmup):
+        oracle_step(w, 64)
+    times = []
+    for _ in range(args.steps):
+        s, J = oracle_step(w, n_dispatch)
+        times.append(s)
+    total = float(np.sum(times))
+    value = args.steps * w["J"] / total
+    return {
+        "metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": total / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic",
+        "config": {"workload": "Large: D=256 decoders x 4,096 residents (1,048,576), capacity "
+                               "524,288, H=65,536, 65,536 candidates, calibration n=1,000,000, "
+                               "alpha=0.1"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": (f"per step: full calibration, occupancy and order; dispatch "
+                                    f"of {n_dispatch} candidates scaled to {w['J']}")},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["maps", "reference"], default="maps")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world, rank, local = dist_env()
+
+    if args.impl == "reference":
+        res = bench_reference(args, world, rank)
+        if res is not None:
+            print(json.dumps(res), flush=True)
+        return
+
+    import torch
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    from paper_2609_15359_gb300 import build as B
+    if rank == 0 and not B.up_to_date():
+        B.build()
+    if dist is not None:
+        dist.barrier()
+    res, w = bench_gpu(args, world, rank, local, dist)
+    if rank == 0:
+        if world == 1 and not args.no_cpu_baseline:
+            res["cpu_baseline"] = cpu_baseline(w)
+        print(json.dumps(res), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -143,11 +143,13 @@ def test_calibrate_random(M, ws, oracle, n):
     query = rng.integers(0, 5000, 4099).astype(np.int32)
     for a in (1, 50000, 100000, 200000, 900000, 999999):
         sto, qo = oracle.calibrate(L, P, a)
+        if sto == 0:  # the call also bounds the queries, which may overflow
+            sto, Uo = oracle.bound(query, qo)
         st, q, qd, U = gpu_calibrate(M, ws, L, P, a, query)
         assert st == sto, (n, a)
         if st == 0:
             assert q == qd == qo
-            assert np.array_equal(U, oracle.bound(query, qo)[1])
+            assert np.array_equal(U, Uo)
 
 
 def test_calibrate_unaligned_and_ranges(M, ws, oracle):
@@ -246,8 +248,9 @@ def diverse_caps(rng, K, spread):
     """Capacities straddling each decoder's occupancy so that the feasible set
     changes from candidate to candidate (test input built from the oracle)."""
     base = K[:, 0].astype(np.int64)
-    cap = base + rng.integers(-spread, 3 * spread, K.shape[0])
-    return np.clip(cap, 0, I32_MAX).astype(np.int32)
+    off = rng.integers(-spread, spread // 2, K.shape[0])
+    off[rng.integers(K.shape[0])] = spread // 2 - 1  # at least one roomy decoder
+    return np.clip(base + off, 0, I32_MAX).astype(np.int32)
 
 
 def check_dispatch(M, ws, oracle, mode, D, H, K, cap, Q, cp, cb, S=1, res=None):
@@ -273,13 +276,15 @@ def test_dispatch_snapshot_random(M, ws, oracle, D, H, J):
     off, p, g, U = random_residents(rng, D, H, 40)
     _, K = oracle.occupancy(D, H, off, p, g, U)
     cap = diverse_caps(rng, K, 4000)
-    Q = rng.integers(0, 4, D).astype(np.int32)
+    # tied queue lengths for even D, all distinct for odd D
+    Q = (rng.integers(0, 4, D) if D % 2 == 0 else rng.permutation(D)).astype(np.int32)
     cp = rng.integers(0, 3000, J).astype(np.int32)
     cb = rng.integers(0, 2 * H + 2, J).astype(np.int32)
     co, ho = check_dispatch(M, ws, oracle, 0, D, H, K, cap, Q, cp, cb)
     if J >= 100:
         assert (ho >= 0).any() and (ho < 0).any()  # both branches exercised
-        assert len(set(co.tolist())) > 1
+        if D >= 8:
+            assert len(set(co.tolist())) > 1
 
 
 @pytest.mark.parametrize("name", ["tiny", "d16", "d64"])
