@@ -182,6 +182,7 @@ class Step:
         self.U_all = torch.empty(R + J, dtype=torch.int32, device=device)
         self.q = torch.empty(1, dtype=torch.int32, device=device)
         self.K = torch.empty((self.D, self.H), dtype=torch.int32, device=device)
+        self.kmax = torch.empty(M.kmax_shape(self.D, self.H), dtype=torch.int32, device=device)
         self.dec_all = t(np.concatenate([w["res_dec"], np.zeros(J, np.int32)]))
         self.choice = self.dec_all[R:]
         self.headroom = torch.empty(J, dtype=torch.int64, device=device)
@@ -194,8 +195,9 @@ class Step:
         self.ws = M.Workspace(need, device)
         dbits = (self.D - 1).bit_length()
         n_hi = min(8, (32 + dbits + 7) // 8)
-        # calibrate 4, occupancy 1, dispatch 4, order 2 + 4 + n_hi + 2
-        self.kernels_per_step = 4 + 1 + 4 + (2 + 4 + n_hi + 2)
+        # calibrate 4, occupancy 1, dispatch 5 (carry scan, bin count / scan /
+        # scatter, main), order 2 + 4 + n_hi + 2
+        self.kernels_per_step = 4 + 1 + 5 + (2 + 4 + n_hi + 2)
 
     def run(self, ev=None):
         M, R = self.M, self.R
@@ -205,13 +207,14 @@ class Step:
         if ev:
             ev[0].record()
         st = M.maps_project_occupancy(self.D, self.H, self.res_off, self.res_prompt,
-                                      self.res_gen, self.U_all[:R], self.K, ws=self.ws)
+                                      self.res_gen, self.U_all[:R], self.K, self.kmax,
+                                      ws=self.ws)
         assert st == 0, st
         if ev:
             ev[1].record()
         st = M.maps_dispatch(M.MODE_SNAPSHOT, self.D, self.H, 1, self.K, self.cap, self.Q0,
                              self.cand_prompt, self.U_all[R:], self.choice, self.headroom,
-                             ws=self.ws)
+                             kmax=self.kmax, ws=self.ws)
         assert st == 0, st
         if ev:
             ev[2].record()

@@ -114,14 +114,20 @@ int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
  *   prompt, gen, bound  [R] int32 resident prompt lengths, generated tokens,
  *                       calibrated bounds.
  *   K_out               [D][H] int32 output.
+ *   kmax_out            optional [D][ceil(H/16)] uint32 output (NULL: not
+ *                       written): kmax[k][b] = max over the steps t of block
+ *                       b (t in [16b, min(16b+16, H))) of K[k][t] + t.  It
+ *                       summarises K for maps_dispatch (SNAPSHOT), which
+ *                       then need not re-read the whole of K.
  * A K value above INT32_MAX, offsets out of order or a negative length is
  * MAPS_E_RANGE (via maps_check).
  * ---------------------------------------------------------------------- */
 size_t maps_project_occupancy_workspace_size(int32_t D, int32_t H, int64_t R);
 int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
                            int64_t R, const int32_t *prompt, const int32_t *gen,
-                           const int32_t *bound, int32_t *K_out, void *ws,
-                           size_t ws_bytes, void *stream);
+                           const int32_t *bound, int32_t *K_out,
+                           uint32_t *kmax_out, void *ws, size_t ws_bytes,
+                           void *stream);
 
 /* ------------------------------------------------------------------------
  * Global memory-aware dispatch, Sec. 3.3 and Alg. 1.
@@ -148,9 +154,15 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
  * each choice.  K is not read in the ALG1 modes.
  *
  *   mode                MAPS_MODE_*.
- *   D, H, S             decoders (1 <= D <= 1024), horizon, block size (ALG1).
+ *   D, H, S             decoders (1 <= D <= 1024), horizon (1 <= H <= 2^28),
+ *                       block size (ALG1).
  *   K                   [D][H] int32 occupancy (horizon modes; updated in
  *                       place by SEQUENTIAL).
+ *   kmax                optional [D][ceil(H/16)] uint32, SNAPSHOT only: the
+ *                       summary maps_project_occupancy wrote for this same K.
+ *                       NULL makes the call derive it from K (one more pass
+ *                       over K).  A summary that does not match K gives
+ *                       unspecified results.
  *   cap, Q              [D] int32 capacities and queue lengths (Q updated in
  *                       place by the SEQUENTIAL modes).
  *   res_off, R, prompt, gen, bound   residents as in maps_project_occupancy
@@ -164,7 +176,8 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
 size_t maps_dispatch_workspace_size(int32_t mode, int32_t D, int32_t H,
                                     int64_t J);
 int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K,
-                  const int32_t *cap, int32_t *Q, const int64_t *res_off,
+                  const uint32_t *kmax, const int32_t *cap, int32_t *Q,
+                  const int64_t *res_off,
                   int64_t R, const int32_t *prompt, const int32_t *gen,
                   const int32_t *bound, int64_t J, const int32_t *cand_prompt,
                   const int32_t *cand_bound, int32_t *choice_out,

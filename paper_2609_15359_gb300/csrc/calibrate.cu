@@ -54,13 +54,20 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
   __syncthreads();
   const uint32_t prefix = PASS == 0 ? 0u : *reinterpret_cast<volatile uint32_t *>(&st->prefix);
 
-  auto visit = [&](uint32_t s) {
-    if (PASS > 0 && (s >> kPrevShift) != prefix) return;
-    atomicAdd(&sh[(s >> kShift) & kMask], 1u);
+  // Warp-aggregated histogram update: lanes holding the same digit add once
+  // (about half of all scores are 0, so single-lane atomics would pile up).
+  auto visit = [&](uint32_t s, bool valid) {
+    if (PASS > 0 && (s >> kPrevShift) != prefix) valid = false;
+    const int d = valid ? static_cast<int>((s >> kShift) & kMask) : -1;
+    const unsigned peers = __match_any_sync(0xffffffffu, d);
+    if (valid && static_cast<int>(threadIdx.x & 31) == __ffs(peers) - 1)
+      atomicAdd(&sh[d], static_cast<uint32_t>(__popc(peers)));
   };
 
+  // Grid-stride loops whose bounds depend only on the block's first index,
+  // so whole warps iterate together.
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  const int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t b0 = static_cast<int64_t>(blockIdx.x) * blockDim.x;
   const bool vec = (reinterpret_cast<uintptr_t>(L) % 16 == 0) &&
                    (reinterpret_cast<uintptr_t>(P) % 16 == 0);
   int64_t tail_start = 0;
@@ -68,20 +75,39 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
     const int64_t n4 = n / 4;
     const int4 *L4 = reinterpret_cast<const int4 *>(L);
     const int4 *P4 = reinterpret_cast<const int4 *>(P);
-    for (int64_t i = i0; i < n4; i += stride) {
-      const int4 a = __ldg(L4 + i), b = __ldg(P4 + i);
-      visit(score(a.x, b.x));
-      visit(score(a.y, b.y));
-      visit(score(a.z, b.z));
-      visit(score(a.w, b.w));
+    for (int64_t i0 = b0; i0 < n4; i0 += 4 * stride) {
+      int4 a[4], b[4];
+      bool ok[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {  // issue all loads first
+        const int64_t i = i0 + u * stride + threadIdx.x;
+        ok[u] = i < n4;
+        a[u] = ok[u] ? __ldg(L4 + i) : make_int4(0, 0, 0, 0);
+        b[u] = ok[u] ? __ldg(P4 + i) : make_int4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        visit(score(a[u].x, b[u].x), ok[u]);
+        visit(score(a[u].y, b[u].y), ok[u]);
+        visit(score(a[u].z, b[u].z), ok[u]);
+        visit(score(a[u].w, b[u].w), ok[u]);
+      }
     }
     tail_start = n4 * 4;
   }
-  for (int64_t i = tail_start + i0; i < n; i += stride) visit(score(__ldg(L + i), __ldg(P + i)));
+  for (int64_t i0 = tail_start + b0; i0 < n; i0 += stride) {
+    const int64_t i = i0 + threadIdx.x;
+    const bool ok = i < n;
+    visit(ok ? score(__ldg(L + i), __ldg(P + i)) : 0u, ok);
+  }
   __syncthreads();
 
-  for (int b = threadIdx.x; b < kBins; b += blockDim.x)
+  // start each block's flush at a different bin so blocks do not collide
+  const int rot = static_cast<int>((blockIdx.x * 97u) % kBins);
+  for (int i = threadIdx.x; i < kBins; i += blockDim.x) {
+    const int b = (i + rot) & (kBins - 1);
     if (sh[b]) atomicAdd(&st->hist[PASS][b], static_cast<unsigned long long>(sh[b]));
+  }
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) s_last = (atomicAdd(&st->done[PASS], 1u) == gridDim.x - 1);
@@ -136,19 +162,44 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
   }
 }
 
+// U = pred + q.  Four bounds per thread (one 128-bit load and store when
+// both arrays allow it), all loads issued before any store.
 __global__ void __launch_bounds__(256)
 bound_kernel(const int32_t *__restrict__ pred, int64_t m, const SelectState *st,
              int32_t *__restrict__ out, int32_t *status) {
   const long long q = *reinterpret_cast<const volatile int32_t *>(&st->q);
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t i4 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t i = i4 * 4;
+  if (i >= m) return;
+  const bool vec = (reinterpret_cast<uintptr_t>(pred) % 16 == 0) &&
+                   (reinterpret_cast<uintptr_t>(out) % 16 == 0) && i + 4 <= m;
+  int32_t v[4];
+  if (vec) {
+    const int4 x = __ldg(reinterpret_cast<const int4 *>(pred) + i4);
+    v[0] = x.x;
+    v[1] = x.y;
+    v[2] = x.z;
+    v[3] = x.w;
+  } else {
+#pragma unroll
+    for (int c = 0; c < 4; ++c) v[c] = i + c < m ? __ldg(pred + i + c) : 0;
+  }
   bool bad = false;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < m; i += stride) {
-    long long u = static_cast<long long>(__ldg(pred + i)) + q;  // Eq. (conformal_upper)
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    long long u = static_cast<long long>(v[c]) + q;  // Eq. (conformal_upper)
     if (u > 0x7fffffffLL) {
-      bad = true;
+      if (i + c < m) bad = true;
       u = 0x7fffffffLL;
     }
-    out[i] = static_cast<int32_t>(u);
+    v[c] = static_cast<int32_t>(u);
+  }
+  if (vec) {
+    *reinterpret_cast<int4 *>(out + i) = make_int4(v[0], v[1], v[2], v[3]);
+  } else {
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+      if (i + c < m) out[i + c] = v[c];
   }
   if (bad) flag_error(status, MAPS_E_RANGE);
 }
@@ -204,7 +255,9 @@ int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
   select_pass_kernel<2><<<g, kSelectThreads, 0, s>>>(true_len, pred_len, n, kk, st, q_dev_out, status);
   MAPS_TRY(launch_ok());
   if (m > 0) {
-    bound_kernel<<<grid_for(m, 256 * 8), 256, 0, s>>>(query_pred, m, st, bound_out, status);
+    const int64_t gb = (m + 1023) / 1024;
+    if (gb > 0x7fffffffLL) return MAPS_E_INVALID;
+    bound_kernel<<<static_cast<unsigned>(gb), 256, 0, s>>>(query_pred, m, st, bound_out, status);
     MAPS_TRY(launch_ok());
   }
   if (q_host_out != nullptr) {

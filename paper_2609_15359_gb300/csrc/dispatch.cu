@@ -32,7 +32,7 @@ namespace maps {
 namespace {
 
 constexpr int kMaxD = 1024;
-constexpr int kMainThreads = 512;
+constexpr int kMainThreads = 256;
 constexpr int kBoxRows = 256;  // TMA box height limit
 
 // ---------------------------------------------------------------------------
@@ -76,389 +76,553 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
 }
-__device__ __forceinline__ void fence_proxy_async() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 __device__ __forceinline__ void fence_mbar_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
 
 // ---------------------------------------------------------------------------
-// SNAPSHOT preparation: bucket candidates by the horizon tile of u_j - 1.
+// SNAPSHOT preparation.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int candidate_steps(int32_t U, int H) {
   return U < 1 ? 1 : (U > H ? H : U);
 }
 
-__global__ void bin_count_kernel(int64_t J, int H, int W2, const int32_t *__restrict__ cp,
-                                 const int32_t *__restrict__ cb, uint32_t *tcount,
-                                 int32_t *choice, int64_t *headroom, int32_t *status) {
+constexpr int kSumBlock = 16;      // steps per kmax summary entry
+constexpr int kUnitCands = 4096;   // candidates per work unit of the main kernel
+
+// kmax[k][b] = max over the 16 steps of block b of K[k][t] + t, for callers
+// that do not pass the summary from maps_project_occupancy.
+__global__ void __launch_bounds__(256)
+kmax_from_K_kernel(int D, int H, const int32_t *__restrict__ K, uint32_t *__restrict__ kmax,
+                   int32_t *status) {
+  const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
+  const int64_t total = nb * D;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  bool bad = false;
-  for (int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; j < J; j += stride) {
-    const int32_t p = cp[j], U = cb[j];
-    if ((p | U) < 0) {
-      bad = true;
-      choice[j] = -1;
-      if (headroom) headroom[j] = 0;
-      continue;
+  bool neg = false;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total; i += stride) {
+    const int64_t k = i / nb, b = i - k * nb;
+    const int32_t *row = K + k * H;
+    const int64_t t0 = b * kSumBlock;
+    uint32_t m = 0;
+    for (int c = 0; c < kSumBlock; ++c) {
+      const int64_t t = t0 + c;
+      if (t >= H) break;
+      const int32_t v = __ldg(row + t);
+      if (v < 0) neg = true;
+      const uint32_t x = static_cast<uint32_t>(v) + static_cast<uint32_t>(t);
+      m = x > m ? x : m;
     }
-    const int u = candidate_steps(U, H);
-    atomicAdd(&tcount[(u - 1) / W2], 1u);
+    kmax[i] = m;
   }
-  if (bad) flag_error(status, MAPS_E_RANGE);
+  if (neg) flag_error(status, MAPS_E_RANGE);
 }
 
-// Exclusive scan of the T2 tile counts into toff[0..T2] (single block).
-__global__ void __launch_bounds__(1024) bin_scan_kernel(int T2, const uint32_t *tcount, uint32_t *toff) {
-  __shared__ uint32_t s_warp[32];
-  __shared__ uint32_t s_carry;
+// carry[k][i] = max of K[k][t] + t over t < i*W2 (0 for i = 0): the prefix
+// maximum that horizon tile i inherits from the tiles before it.  One block
+// per decoder; each thread reads 16 consecutive summary entries at once
+// (whole tiles, as W2/16 divides 16), keeps its tiles' maxima in registers,
+// and after a block scan writes its tiles' carries contiguously.
+__global__ void __launch_bounds__(256)
+carry_scan_kernel(int D, int H, int W2, int T2, const uint32_t *__restrict__ kmax,
+                  uint32_t *__restrict__ carry) {
+  __shared__ uint32_t s_w[8];
+  constexpr int kPer = 16;
+  const int k = blockIdx.x;
+  const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
+  const int bpt = W2 / kSumBlock;  // summary blocks per tile (1..16)
+  const uint32_t *row = kmax + static_cast<int64_t>(k) * nb;
+  uint32_t *out = carry + static_cast<int64_t>(k) * T2;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) s_carry = 0;
-  __syncthreads();
-  for (int base = 0; base < T2; base += 1024) {
-    const int i = base + threadIdx.x;
-    const uint32_t v = i < T2 ? tcount[i] : 0u;
-    uint32_t incl = v;
+  const bool vec = (reinterpret_cast<uintptr_t>(row) % 16) == 0;
+  uint32_t run = 0;
+  for (int64_t c0 = 0; c0 < nb; c0 += 256 * kPer) {
+    const int64_t b0 = c0 + threadIdx.x * kPer;
+    uint32_t v[kPer];
+    if (vec && b0 + kPer <= nb) {
+#pragma unroll
+      for (int q = 0; q < kPer; q += 4) {
+        const uint4 x = __ldg(reinterpret_cast<const uint4 *>(row + b0 + q));
+        v[q] = x.x, v[q + 1] = x.y, v[q + 2] = x.z, v[q + 3] = x.w;
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < kPer; ++q) v[q] = b0 + q < nb ? __ldg(row + b0 + q) : 0u;
+    }
+    uint32_t m = 0;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) m = v[q] > m ? v[q] : m;
+    uint32_t incl = m;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
-      if (lane >= off) incl += y;
+      if (lane >= off) incl = y > incl ? y : incl;
     }
-    if (lane == 31) s_warp[warp] = incl;
+    if (lane == 31) s_w[warp] = incl;
     __syncthreads();
-    uint32_t wbase = 0;
-    for (int w = 0; w < warp; ++w) wbase += s_warp[w];
-    const uint32_t carry = s_carry;
-    if (i < T2) toff[i] = carry + wbase + incl - v;
-    __syncthreads();
-    if (threadIdx.x == 1023) s_carry = carry + wbase + incl;
+    uint32_t r = __shfl_up_sync(0xffffffffu, incl, 1);
+    if (lane == 0) r = 0;
+    uint32_t all = 0;
+    for (int w = 0; w < 8; ++w) {
+      if (w < warp) r = s_w[w] > r ? s_w[w] : r;
+      all = s_w[w] > all ? s_w[w] : all;
+    }
+    r = r > run ? r : run;
+    // this thread's tiles: [b0 / bpt, (b0 + kPer) / bpt)
+    const int64_t tile0 = b0 / bpt;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      if (q % bpt == 0) {
+        const int64_t ti = tile0 + q / bpt;
+        if (ti < T2) out[ti] = r;
+      }
+      r = v[q] > r ? v[q] : r;
+    }
+    run = all > run ? all : run;
     __syncthreads();
   }
-  if (threadIdx.x == 0) toff[T2] = s_carry;
 }
 
-__global__ void bin_scatter_kernel(int64_t J, int H, int W2, const int32_t *__restrict__ cp,
-                                   const int32_t *__restrict__ cb, const uint32_t *toff,
-                                   uint32_t *tcursor, int32_t *ord) {
+__device__ __forceinline__ unsigned lanemask_lt() {
+  unsigned m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// Candidates are bucketed by the horizon tile holding their last live step
+// u_j - 1.  When the tile count fits in shared memory each block first counts
+// its candidates per tile locally and then adds one global count per
+// non-empty tile; otherwise lanes with the same tile combine their atomic.
+// Grid-stride loops run in whole warps.
+constexpr int kBinSmem = 4096;
+
+__global__ void __launch_bounds__(1024)
+bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ cp,
+                 const int32_t *__restrict__ cb, uint32_t *tcount, int32_t *choice,
+                 int64_t *headroom, int32_t *status) {
+  __shared__ uint32_t s_h[kBinSmem];
+  const bool local = T2 <= kBinSmem;
+  if (local)
+    for (int i = threadIdx.x; i < T2; i += blockDim.x) s_h[i] = 0;
+  __syncthreads();
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; j < J; j += stride) {
-    const int32_t p = cp[j], U = cb[j];
-    if ((p | U) < 0) continue;
-    const int tile = (candidate_steps(U, H) - 1) / W2;
-    const uint32_t pos = toff[tile] + atomicAdd(&tcursor[tile], 1u);
-    ord[pos] = static_cast<int32_t>(j);
+  bool bad = false;
+  for (int64_t j0 = static_cast<int64_t>(blockIdx.x) * blockDim.x; j0 < J; j0 += stride) {
+    const int64_t j = j0 + threadIdx.x;
+    int tile = -1;
+    if (j < J) {
+      const int32_t p = cp[j], U = cb[j];
+      if ((p | U) < 0) {
+        bad = true;
+        choice[j] = -1;
+        if (headroom) headroom[j] = 0;
+      } else {
+        tile = (candidate_steps(U, H) - 1) / W2;
+      }
+    }
+    const unsigned peers = __match_any_sync(0xffffffffu, tile);
+    if (tile >= 0 && (threadIdx.x & 31) == __ffs(peers) - 1)
+      atomicAdd(local ? &s_h[tile] : &tcount[tile], static_cast<uint32_t>(__popc(peers)));
+  }
+  if (bad) flag_error(status, MAPS_E_RANGE);
+  if (local) {
+    __syncthreads();
+    // start each block's flush at a different tile so blocks do not collide
+    const int rot = static_cast<int>((static_cast<int64_t>(blockIdx.x) * 97) % T2);
+    for (int i = threadIdx.x; i < T2; i += blockDim.x) {
+      const int t = (i + rot) % T2;
+      if (s_h[t]) atomicAdd(&tcount[t], s_h[t]);
+    }
+  }
+}
+
+struct Unit {
+  int32_t tile, start, count, pad;
+};
+
+// One block: tile offsets toff[0..T2], the work units (a tile with c
+// candidates gives ceil(c / kUnitCands) units; the unit count goes to
+// *nunits), and the decoders' queue order (Q, then index): sig maps queue
+// position to decoder, rank the reverse, capq holds capacities by position.
+__global__ void __launch_bounds__(1024)
+bin_scan_kernel(int T2, const uint32_t *tcount, uint32_t *toff, Unit *units, uint32_t *nunits,
+                int D, const int32_t *__restrict__ Q, const int32_t *__restrict__ cap,
+                int32_t *sig, int32_t *rank_of, int32_t *capq, int32_t *status) {
+  __shared__ uint32_t s_w[2][32];
+  __shared__ uint32_t s_carry[2];
+  __shared__ int32_t s_q[kMaxD];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  bool bad = false;
+  for (int k = threadIdx.x; k < D; k += blockDim.x) {
+    s_q[k] = Q[k];
+    if ((s_q[k] | cap[k]) < 0) bad = true;
+  }
+  if (bad) flag_error(status, MAPS_E_RANGE);
+  if (threadIdx.x == 0) s_carry[0] = s_carry[1] = 0;
+  __syncthreads();
+  for (int k = threadIdx.x; k < D; k += blockDim.x) {
+    const int32_t qk = s_q[k];
+    int r = 0;
+    for (int k2 = 0; k2 < D; ++k2) {
+      const int32_t q2 = s_q[k2];
+      r += (q2 < qk) || (q2 == qk && k2 < k);
+    }
+    sig[r] = k;
+    rank_of[k] = r;
+    capq[r] = cap[k];
+  }
+  for (int base = 0; base < T2; base += 1024) {
+    const int i = base + threadIdx.x;
+    const uint32_t c = i < T2 ? tcount[i] : 0u;
+    const uint32_t nu = (c + kUnitCands - 1) / kUnitCands;
+    uint32_t ic = c, iu = nu;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t yc = __shfl_up_sync(0xffffffffu, ic, off);
+      const uint32_t yu = __shfl_up_sync(0xffffffffu, iu, off);
+      if (lane >= off) {
+        ic += yc;
+        iu += yu;
+      }
+    }
+    if (lane == 31) {
+      s_w[0][warp] = ic;
+      s_w[1][warp] = iu;
+    }
+    __syncthreads();
+    uint32_t bc = s_carry[0], bu = s_carry[1];
+    for (int w = 0; w < warp; ++w) {
+      bc += s_w[0][w];
+      bu += s_w[1][w];
+    }
+    if (i < T2) {
+      const uint32_t start = bc + ic - c;
+      toff[i] = start;
+      uint32_t u0 = bu + iu - nu;
+      for (uint32_t q = 0; q < nu; ++q) {
+        Unit un;
+        un.tile = i;
+        un.start = static_cast<int32_t>(start + q * kUnitCands);
+        un.count = static_cast<int32_t>(min(static_cast<uint32_t>(kUnitCands), c - q * kUnitCands));
+        un.pad = 0;
+        units[u0 + q] = un;
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 1023) {
+      s_carry[0] = bc + ic;
+      s_carry[1] = bu + iu;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    toff[T2] = s_carry[0];
+    *nunits = s_carry[1];
+  }
+}
+
+// Place every valid candidate into its tile's bucket as (index, prompt,
+// steps).  The order inside a bucket does not matter: each candidate's
+// decision depends only on itself.
+__global__ void __launch_bounds__(1024)
+bin_scatter_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ cp,
+                   const int32_t *__restrict__ cb, const uint32_t *toff, uint32_t *tcursor,
+                   int32_t *ord, int32_t *sp, int32_t *su) {
+  __shared__ uint32_t s_h[kBinSmem];  // local counts, then local cursors
+  __shared__ uint32_t s_b[kBinSmem];  // this block's base inside each bucket
+  const bool local = T2 <= kBinSmem;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t b0 = static_cast<int64_t>(blockIdx.x) * blockDim.x;
+  if (local) {
+    for (int i = threadIdx.x; i < T2; i += blockDim.x) s_h[i] = 0;
+    __syncthreads();
+    for (int64_t j0 = b0; j0 < J; j0 += stride) {
+      const int64_t j = j0 + threadIdx.x;
+      int tile = -1;
+      if (j < J) {
+        const int32_t U = cb[j];
+        if ((cp[j] | U) >= 0) tile = (candidate_steps(U, H) - 1) / W2;
+      }
+      const unsigned peers = __match_any_sync(0xffffffffu, tile);
+      if (tile >= 0 && (threadIdx.x & 31) == __ffs(peers) - 1)
+        atomicAdd(&s_h[tile], static_cast<uint32_t>(__popc(peers)));
+    }
+    __syncthreads();
+    const int rot = static_cast<int>((static_cast<int64_t>(blockIdx.x) * 97) % T2);
+    for (int i = threadIdx.x; i < T2; i += blockDim.x) {
+      const int t = (i + rot) % T2;
+      const uint32_t c = s_h[t];
+      s_b[t] = c ? toff[t] + atomicAdd(&tcursor[t], c) : 0u;
+      s_h[t] = 0;
+    }
+    __syncthreads();
+  }
+  for (int64_t j0 = b0; j0 < J; j0 += stride) {
+    const int64_t j = j0 + threadIdx.x;
+    int tile = -1, u = 0;
+    int32_t p = 0;
+    if (j < J) {
+      p = cp[j];
+      const int32_t U = cb[j];
+      if ((p | U) >= 0) {
+        u = candidate_steps(U, H);
+        tile = (u - 1) / W2;
+      }
+    }
+    const unsigned peers = __match_any_sync(0xffffffffu, tile);
+    const int leader = __ffs(peers) - 1;
+    uint32_t base = 0;
+    if (tile >= 0 && (threadIdx.x & 31) == leader) {
+      const uint32_t c = static_cast<uint32_t>(__popc(peers));
+      base = local ? s_b[tile] + atomicAdd(&s_h[tile], c) : toff[tile] + atomicAdd(&tcursor[tile], c);
+    }
+    base = __shfl_sync(0xffffffffu, base, leader);
+    if (tile >= 0) {
+      const uint32_t pos = base + __popc(peers & lanemask_lt());
+      ord[pos] = static_cast<int32_t>(j);
+      sp[pos] = p;
+      su[pos] = u;
+    }
   }
 }
 
 // ---------------------------------------------------------------------------
-// SNAPSHOT main kernel: persistent, one CTA per SM, tiles taken in ticket
-// order so that decoupled look-back always makes progress.
+// SNAPSHOT main kernel: one CTA per work unit, a unit being (tile, a slice of
+// the tile's candidates).  Tiles without candidates are never read: their
+// contribution reaches later tiles through the carry, built from the summary.
+// Several CTAs share an SM, so one CTA's TMA wait overlaps another's work.
 // ---------------------------------------------------------------------------
 struct SnapArgs {
   int D, H, W2, T2, Drows, boxes, box_rows;  // Drows = rows per staged tile (>= D)
-  int tile_stride;                           // elements per tile buffer (1 KB multiple)
+  int tile_stride;                           // elements of the tile buffer (1 KB multiple)
   bool use_tma;
   const int32_t *K;
-  const int32_t *cap, *Q, *cp, *cb;
-  const uint32_t *toff;
-  const int32_t *ord;
-  uint32_t *flags;  // per tile: 0 none, 1 aggregate, 2 inclusive
-  uint32_t *agg;    // [T2][D] tile row maxima of K + t
-  uint32_t *inc;    // [T2][D] inclusive prefix maxima through the tile
-  uint32_t *ticket;
+  const int32_t *sig, *rank_of, *capq;  // queue order
+  const uint32_t *carry;                // [D][T2]
+  const Unit *units;
+  const uint32_t *nunits;
+  const int32_t *ord, *sp, *su;
   int32_t *choice;
   int64_t *headroom;
   int32_t *status;
 };
 
-constexpr uint32_t kFlagAgg = 1, kFlagInc = 2;
-
 template <int W2>
-__global__ void __launch_bounds__(kMainThreads, 1)
+__global__ void __launch_bounds__(kMainThreads, 3)
 dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   extern __shared__ __align__(1024) unsigned char smem[];
+  const int unit = blockIdx.x;
+  if (unit >= static_cast<int>(*a.nunits)) return;
   const int D = a.D, H = a.H;
-  const int tid = threadIdx.x, lane = tid & 31;
-  const size_t tile_elems = static_cast<size_t>(a.tile_stride);
-  uint32_t *kbuf0 = reinterpret_cast<uint32_t *>(smem);
-  uint32_t *kbuf1 = kbuf0 + tile_elems;
-  int32_t *pmq = reinterpret_cast<int32_t *>(kbuf1 + tile_elems);  // [D][W2] by Q-position
-  int32_t *s_cap = pmq + static_cast<size_t>(D) * W2;
-  int32_t *s_sig = s_cap + D;  // Q-position -> decoder
-  uint32_t *s_carry = reinterpret_cast<uint32_t *>(s_sig + D);
-  uint32_t *s_agg = s_carry + D;
-  constexpr int nch = kMainThreads / W2;  // position chunks per column
-  int32_t *s_chPM = reinterpret_cast<int32_t *>(s_agg + D);  // [nch][W2]
-  int32_t *s_chK = s_chPM + nch * W2;
-  int32_t *s_argA = s_chK + nch * W2;  // [W2]
-  long long *s_chA = reinterpret_cast<long long *>(
-      (reinterpret_cast<uintptr_t>(s_argA + W2) + 15) & ~uintptr_t(15));  // [nch][W2]
-  long long *s_maxA = s_chA + nch * W2;                                   // [W2]
-  uint64_t *s_bar = reinterpret_cast<uint64_t *>(s_maxA + W2);            // [2]
-  __shared__ int s_tile, s_next, s_abort;
-  __shared__ uint32_t s_flag;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int kWarpsM = kMainThreads / 32;
+  uint32_t *kb = reinterpret_cast<uint32_t *>(smem);
+  // comp[slot][i]: M of decoder sig[i] at the slot's column, then rewritten
+  // in place into the queue-ordered prefix maximum of A (clamped at -1)
+  uint32_t *comp = kb + a.tile_stride;
+  int32_t *s_capq = reinterpret_cast<int32_t *>(comp + static_cast<size_t>(W2) * D);
+  int32_t *s_sig = s_capq + D;
+  int32_t *s_rank = s_sig + D;
+  uint32_t *s_carry = reinterpret_cast<uint32_t *>(s_rank + D);
+  int32_t *s_slot = reinterpret_cast<int32_t *>(s_carry + D);  // [W2] column -> slot (-1 none)
+  int32_t *s_argA = s_slot + W2;                               // [W2]
+  long long *s_maxA = reinterpret_cast<long long *>(
+      (reinterpret_cast<uintptr_t>(s_argA + W2) + 15) & ~uintptr_t(15));  // [W2]
+  uint64_t *s_bar = reinterpret_cast<uint64_t *>(s_maxA + W2);
+  __shared__ int s_nslots, s_abort;
 
-  // --- setup: capacities, queue order (stable by index), barriers ---------
-  bool bad = false;
-  for (int k = tid; k < D; k += kMainThreads) {
-    const int32_t c = a.cap[k], q = a.Q[k];
-    if ((c | q) < 0) bad = true;
-    s_cap[k] = c;
-  }
-  for (int k = tid; k < D; k += kMainThreads) {
-    const int32_t qk = a.Q[k];
-    int rank = 0;
-    for (int k2 = 0; k2 < D; ++k2) {
-      const int32_t q2 = a.Q[k2];
-      rank += (q2 < qk) || (q2 == qk && k2 < k);
-    }
-    s_sig[rank] = k;
-  }
-  if (bad) flag_error(a.status, MAPS_E_RANGE);
+  const Unit un = a.units[unit];
+  const int64_t t0 = static_cast<int64_t>(un.tile) * W2;
   if (tid == 0) {
     s_abort = 0;
     if (a.use_tma) {
-      mbar_init(&s_bar[0], 1);
-      mbar_init(&s_bar[1], 1);
+      mbar_init(s_bar, 1);
       fence_mbar_init();
+      // every box is credited in full, rows past D included (zero-filled)
+      mbar_expect_tx(s_bar, static_cast<uint32_t>(a.boxes) * a.box_rows * W2 * 4u);
+      for (int b = 0; b < a.boxes; ++b)
+        tma_load_2d(kb + static_cast<size_t>(b) * a.box_rows * W2, &tmap, s_bar, un.tile * W2,
+                    b * a.box_rows);
+    }
+  }
+  // queue order, capacities and this tile's carries; columns this unit needs
+  for (int k = tid; k < D; k += kMainThreads) {
+    s_sig[k] = __ldg(a.sig + k);
+    s_rank[k] = __ldg(a.rank_of + k);
+    s_capq[k] = __ldg(a.capq + k);
+    s_carry[k] = __ldg(a.carry + static_cast<int64_t>(k) * a.T2 + un.tile);
+  }
+  for (int c = tid; c < W2; c += kMainThreads) s_slot[c] = 0;
+  __syncthreads();
+  for (int q0 = 0; q0 < un.count; q0 += kMainThreads * 8) {
+    int32_t uu[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {  // issue the loads together
+      const int q = q0 + i * kMainThreads + tid;
+      uu[i] = q < un.count ? __ldg(a.su + un.start + q) : 0;
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if (uu[i] > 0) s_slot[uu[i] - 1 - t0] = 1;
+  }
+  if (!a.use_tma) {
+    for (int e = tid; e < D * W2; e += kMainThreads) {
+      const int r = e / W2, c = e - (e / W2) * W2;
+      const int64_t t = t0 + c;
+      kb[e] = t < H ? static_cast<uint32_t>(a.K[static_cast<int64_t>(r) * H + t]) : 0u;
     }
   }
   __syncthreads();
-
-  // every box is credited in full, rows past D included (zero-filled)
-  const uint32_t tile_bytes = static_cast<uint32_t>(a.boxes) * a.box_rows * W2 * 4u;
-  auto issue = [&](int tile, uint32_t *buf, uint64_t *bar) {
-    mbar_expect_tx(bar, tile_bytes);
-    for (int b = 0; b < a.boxes; ++b)
-      tma_load_2d(buf + static_cast<size_t>(b) * a.box_rows * W2, &tmap, bar, tile * W2, b * a.box_rows);
-  };
-  if (tid == 0) {
-    const int t = static_cast<int>(atomicAdd(a.ticket, 1u));
-    s_tile = t;
-    if (a.use_tma && t < a.T2) issue(t, kbuf0, &s_bar[0]);
+  if (warp == 0) {  // compact the flagged columns (W2 <= 256)
+    int run = 0;
+    for (int c0 = 0; c0 < W2; c0 += 32) {
+      const int c = c0 + lane;
+      const bool f = c < W2 && s_slot[c] != 0;
+      const unsigned bal = __ballot_sync(0xffffffffu, f);
+      if (c < W2) s_slot[c] = f ? run + __popc(bal & lanemask_lt()) : -1;
+      run += __popc(bal);
+    }
+    if (lane == 0) s_nslots = run;
+  }
+  if (a.use_tma && !mbar_wait_bounded(s_bar, 0)) {
+    if (tid == 0) flag_error(a.status, MAPS_E_TIMEOUT);
+    s_abort = 1;
   }
   __syncthreads();
+  if (s_abort) {
+    // a copy may still land: wait for it once more (bounded) before leaving
+    mbar_wait_bounded(s_bar, 0);
+    return;
+  }
+  const int nslots = s_nslots;
 
-  int cur = s_tile;
-  int buf = 0;
-  uint32_t phase[2] = {0u, 0u};
+  // --- prefix maximum of K + t along each row; keep the needed columns ----
   constexpr int seg = W2 / 16;  // cells per row segment; 16 segments per row
   const int items = ((D * 16 + kMainThreads - 1) / kMainThreads) * kMainThreads;
-
-  while (cur < a.T2) {
-    uint32_t *kb = buf ? kbuf1 : kbuf0;
-    const int64_t t0 = static_cast<int64_t>(cur) * W2;
-    // prefetch the next tile into the other buffer (it was released by the
-    // __syncthreads that ended the previous iteration)
-    if (tid == 0) {
-      const int nx = static_cast<int>(atomicAdd(a.ticket, 1u));
-      s_next = nx;
-      if (a.use_tma && nx < a.T2) {
-        fence_proxy_async();
-        issue(nx, buf ? kbuf0 : kbuf1, &s_bar[buf ^ 1]);
+  bool neg = false;
+  for (int it = tid; it < items; it += kMainThreads) {
+    const int row = it >> 4, sg = it & 15;
+    const bool live_row = row < D;
+    uint32_t v[seg];
+    uint32_t run = 0;
+#pragma unroll
+    for (int j = 0; j < seg; ++j) {
+      const int c = sg * seg + j;
+      const int64_t t = t0 + c;
+      uint32_t x = 0;
+      if (live_row && t < H) {
+        const uint32_t raw = kb[static_cast<size_t>(row) * W2 + c];
+        if (static_cast<int32_t>(raw) < 0) neg = true;
+        x = raw + static_cast<uint32_t>(t);  // K + t < 2^32
       }
+      run = x > run ? x : run;
+      v[j] = run;
     }
-    if (a.use_tma) {
-      if (!mbar_wait_bounded(&s_bar[buf], phase[buf])) {
-        if (tid == 0) flag_error(a.status, MAPS_E_TIMEOUT);
-        s_abort = 1;
-      }
-      phase[buf] ^= 1u;
-    } else {
-      for (size_t e = tid; e < static_cast<size_t>(D) * W2; e += kMainThreads) {
-        const int r = static_cast<int>(e / W2), c = static_cast<int>(e % W2);
-        const int64_t t = t0 + c;
-        kb[e] = t < H ? static_cast<uint32_t>(a.K[static_cast<int64_t>(r) * H + t]) : 0u;
-      }
+    uint32_t incl = run;
+#pragma unroll
+    for (int off = 1; off < 16; off <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off, 16);
+      if (sg >= off) incl = y > incl ? y : incl;
     }
-    __syncthreads();
-    if (s_abort) break;
-
-    // --- in-tile prefix maximum of K + t along each row ---------------------
-    bool neg = false;
-    for (int it = tid; it < items; it += kMainThreads) {
-      const int row = it >> 4, sg = it & 15;
-      const bool live_row = row < D;
-      uint32_t v[seg];
-      uint32_t run = 0;
+    uint32_t excl = __shfl_up_sync(0xffffffffu, incl, 1, 16);
+    if (sg == 0) excl = 0;
+    if (live_row) {
+      const uint32_t cr = s_carry[row];
+      const int rk = s_rank[row];
+      excl = excl > cr ? excl : cr;
 #pragma unroll
       for (int j = 0; j < seg; ++j) {
-        const int c = sg * seg + j;
-        const int64_t t = t0 + c;
-        uint32_t x = 0;
-        if (live_row && t < H) {
-          const uint32_t raw = kb[static_cast<size_t>(row) * W2 + c];
-          if (static_cast<int32_t>(raw) < 0) neg = true;
-          x = raw + static_cast<uint32_t>(t);  // K + t < 2^32
-        }
-        run = x > run ? x : run;
-        v[j] = run;
-      }
-      uint32_t incl = run;
-#pragma unroll
-      for (int off = 1; off < 16; off <<= 1) {
-        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off, 16);
-        if (sg >= off) incl = y > incl ? y : incl;
-      }
-      uint32_t excl = __shfl_up_sync(0xffffffffu, incl, 1, 16);
-      if (sg == 0) excl = 0;
-      if (live_row) {
-#pragma unroll
-        for (int j = 0; j < seg; ++j) {
-          const uint32_t y = v[j] > excl ? v[j] : excl;
-          kb[static_cast<size_t>(row) * W2 + sg * seg + j] = y;
-        }
-        if (sg == 15) s_agg[row] = incl;
+        const int sl = s_slot[sg * seg + j];
+        if (sl >= 0) comp[static_cast<size_t>(sl) * D + rk] = v[j] > excl ? v[j] : excl;
       }
     }
-    if (neg) flag_error(a.status, MAPS_E_RANGE);
-    __syncthreads();
+  }
+  if (neg) flag_error(a.status, MAPS_E_RANGE);
+  __syncthreads();
 
-    // --- carry across tiles: decoupled look-back ---------------------------
-    uint32_t *agg_row = a.agg + static_cast<size_t>(cur) * D;
-    uint32_t *inc_row = a.inc + static_cast<size_t>(cur) * D;
-    for (int k = tid; k < D; k += kMainThreads) {
-      s_carry[k] = 0;
-      if (cur == 0)
-        inc_row[k] = s_agg[k];
-      else
-        agg_row[k] = s_agg[k];
-    }
-    __syncthreads();
-    if (tid == 0) {
-      __threadfence();
-      st_release_u32(a.flags + cur, cur == 0 ? kFlagInc : kFlagAgg);
-    }
-    for (int p = cur - 1; p >= 0; --p) {
-      if (tid == 0) {
-        uint32_t f = 0, spins = 0;
-        while ((f = ld_acquire_u32(a.flags + p)) == 0) {
-          if (++spins > kSpinLimit) {
-            flag_error(a.status, MAPS_E_TIMEOUT);
-            f = kFlagInc;  // give up: use what is there
-            break;
-          }
-          __nanosleep(32);
-        }
-        s_flag = f;
-      }
-      __syncthreads();
-      const uint32_t f = s_flag;
-      const uint32_t *src = (f == kFlagInc ? a.inc : a.agg) + static_cast<size_t>(p) * D;
-      for (int k = tid; k < D; k += kMainThreads) {
-        const uint32_t y = __ldcg(src + k);
-        if (y > s_carry[k]) s_carry[k] = y;
-      }
-      __syncthreads();
-      if (f == kFlagInc) break;
-    }
-    if (cur > 0) {
-      for (int k = tid; k < D; k += kMainThreads) {
-        const uint32_t x = s_agg[k], c = s_carry[k];
-        inc_row[k] = x > c ? x : c;
-      }
-      __syncthreads();
-      if (tid == 0) {
-        __threadfence();
-        st_release_u32(a.flags + cur, kFlagInc);
-      }
-    }
-
-    // --- per column: queue-ordered prefix max of A, and arg-max of A --------
-    {
-      const int c = tid % W2, ch = tid / W2;
-      const int per = (D + nch - 1) / nch;
-      const int i_lo = ch * per, i_hi = min(D, i_lo + per);
-      int32_t run = -1;
-      long long bestA = LLONG_MIN;
-      int bestK = 0x7fffffff;
-      for (int i = i_lo; i < i_hi; ++i) {
+  // --- per needed column: prefix max of A in queue order, arg-max of A -----
+  const int P = (D + 31) / 32;  // strided queue positions per lane
+  for (int sl = warp; sl < nslots; sl += kWarpsM) {
+    uint32_t *col = comp + static_cast<size_t>(sl) * D;
+    int32_t carryq = -1;
+    long long bestA = LLONG_MIN;
+    int bestK = 0x7fffffff;
+    for (int s = 0; s < P; ++s) {
+      const int i = s * 32 + lane;
+      int32_t a32 = -1;
+      if (i < D) {
+        const long long A = static_cast<long long>(s_capq[i]) - 1 - static_cast<long long>(col[i]);
+        a32 = A < -1 ? -1 : static_cast<int32_t>(A);
         const int k = s_sig[i];
-        const uint32_t m0 = kb[static_cast<size_t>(k) * W2 + c], cr = s_carry[k];
-        const uint32_t M = m0 > cr ? m0 : cr;
-        const long long A = static_cast<long long>(s_cap[k]) - 1 - static_cast<long long>(M);
-        const int32_t a32 = A < -1 ? -1 : static_cast<int32_t>(A);
-        run = a32 > run ? a32 : run;
         if (A > bestA || (A == bestA && k < bestK)) {
           bestA = A;
           bestK = k;
         }
       }
-      s_chPM[ch * W2 + c] = run;
-      s_chA[ch * W2 + c] = bestA;
-      s_chK[ch * W2 + c] = bestK;
-      __syncthreads();
-      int32_t pre = -1;
-      for (int c2 = 0; c2 < ch; ++c2) {
-        const int32_t y = s_chPM[c2 * W2 + c];
-        pre = y > pre ? y : pre;
+      int32_t x = a32;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int32_t y = __shfl_up_sync(0xffffffffu, x, off);
+        if (lane >= off) x = y > x ? y : x;
       }
-      run = pre;
-      for (int i = i_lo; i < i_hi; ++i) {
-        const int k = s_sig[i];
-        const uint32_t m0 = kb[static_cast<size_t>(k) * W2 + c], cr = s_carry[k];
-        const uint32_t M = m0 > cr ? m0 : cr;
-        const long long A = static_cast<long long>(s_cap[k]) - 1 - static_cast<long long>(M);
-        const int32_t a32 = A < -1 ? -1 : static_cast<int32_t>(A);
-        run = a32 > run ? a32 : run;
-        pmq[static_cast<size_t>(i) * W2 + c] = run;
-      }
-      if (ch == 0) {
-        long long bA = LLONG_MIN;
-        int bK = 0x7fffffff;
-        for (int c2 = 0; c2 < nch; ++c2) {
-          const long long A = s_chA[c2 * W2 + c];
-          const int k = s_chK[c2 * W2 + c];
-          if (A > bA || (A == bA && k < bK)) {
-            bA = A;
-            bK = k;
-          }
-        }
-        s_maxA[c] = bA;
-        s_argA[c] = bK;
+      x = x > carryq ? x : carryq;
+      if (i < D) col[i] = static_cast<uint32_t>(x);
+      carryq = __shfl_sync(0xffffffffu, x, 31);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const long long yA = __shfl_xor_sync(0xffffffffu, bestA, off);
+      const int yK = __shfl_xor_sync(0xffffffffu, bestK, off);
+      if (yA > bestA || (yA == bestA && yK < bestK)) {
+        bestA = yA;
+        bestK = yK;
       }
     }
-    __syncthreads();
-
-    // --- the candidates whose last live step falls in this tile -----------
-    {
-      const uint32_t lo = a.toff[cur], hi = a.toff[cur + 1];
-      for (uint32_t pos = lo + tid; pos < hi; pos += kMainThreads) {
-        const int j = a.ord[pos];
-        const int32_t p = a.cp[j];
-        const int u = candidate_steps(a.cb[j], H);
-        const int c = static_cast<int>(u - 1 - t0);
-        int k;
-        long long h;
-        if (pmq[static_cast<size_t>(D - 1) * W2 + c] < p) {
-          k = s_argA[c];  // nothing feasible: most headroom
-          h = s_maxA[c] - p;
-        } else {
-          int l = 0, r = D - 1;  // first queue position whose prefix reaches p
-          while (l < r) {
-            const int mid = (l + r) >> 1;
-            if (pmq[static_cast<size_t>(mid) * W2 + c] >= p)
-              r = mid;
-            else
-              l = mid + 1;
-          }
-          k = s_sig[l];
-          h = static_cast<long long>(pmq[static_cast<size_t>(l) * W2 + c]) - p;
-        }
-        a.choice[j] = k;
-        if (a.headroom) a.headroom[j] = h;
-      }
+    if (lane == 0) {
+      s_maxA[sl] = bestA;
+      s_argA[sl] = bestK;
     }
-    __syncthreads();
-    cur = s_next;
-    buf ^= 1;
   }
-  (void)lane;
-  // The loop ends normally only on a ticket >= T2, for which nothing was
-  // prefetched.  After an abort, wait (bounded) for a prefetch in flight so
-  // no copy lands in shared memory after the block has exited.
-  if (a.use_tma && s_abort && s_next < a.T2) mbar_wait_bounded(&s_bar[buf ^ 1], phase[buf ^ 1]);
+  __syncthreads();
+
+  // --- this unit's candidates (loads issued together, then the searches) ----
+  for (int q0 = 0; q0 < un.count; q0 += kMainThreads * 8) {
+    int32_t pp[8], uu[8], jj[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int q = q0 + i * kMainThreads + tid;
+      const bool ok = q < un.count;
+      pp[i] = ok ? __ldg(a.sp + un.start + q) : 0;
+      uu[i] = ok ? __ldg(a.su + un.start + q) : 0;
+      jj[i] = ok ? __ldg(a.ord + un.start + q) : -1;
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if (jj[i] < 0) continue;
+      const int32_t p = pp[i];
+      const int c = static_cast<int>(uu[i] - 1 - t0);
+      const int sl = s_slot[c];
+      const int32_t *pm = reinterpret_cast<const int32_t *>(comp) + static_cast<size_t>(sl) * D;
+      int k;
+      long long h;
+      if (pm[D - 1] < p) {
+        k = s_argA[sl];  // nothing feasible: most headroom
+        h = s_maxA[sl] - p;
+      } else {
+        int l = 0, r = D - 1;  // first queue position whose prefix reaches p
+        while (l < r) {
+          const int mid = (l + r) >> 1;
+          if (pm[mid] >= p)
+            r = mid;
+          else
+            l = mid + 1;
+        }
+        k = s_sig[l];
+        h = static_cast<long long>(pm[l]) - p;
+      }
+      a.choice[jj[i]] = k;
+      if (a.headroom) a.headroom[jj[i]] = h;
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -795,36 +959,49 @@ SnapGeom snap_geom(int D, int H) {
   g.boxes = (D + g.box_rows - 1) / g.box_rows;
   g.Drows = g.boxes * g.box_rows;
   int w = 256;
-  while (w > 16 && static_cast<long long>(w) * g.Drows > 16384) w >>= 1;
+  while (w > 16 && static_cast<long long>(w) * g.Drows > 8192) w >>= 1;
   g.W2 = w;
   g.T2 = static_cast<int>((static_cast<long long>(H) + w - 1) / w);
-  const int nch = kMainThreads / w;
-  g.tile_stride = (g.Drows * w + 255) / 256 * 256;       // 1 KB-aligned buffers
-  size_t b = 2 * static_cast<size_t>(g.tile_stride) * 4; // two K tiles
-  b += static_cast<size_t>(D) * w * 4;                  // pmq
-  b += 4 * static_cast<size_t>(D) * 4;                  // cap, sig, carry, agg
-  b += 2 * static_cast<size_t>(nch) * w * 4 + w * 4;    // chPM, chK, argA
-  b += 16;                                              // alignment slack
-  b += static_cast<size_t>(nch) * w * 8 + w * 8;        // chA, maxA
-  b += 2 * 8;                                           // barriers
+  g.tile_stride = (g.Drows * w + 255) / 256 * 256;  // 1 KB-aligned buffer
+  size_t b = static_cast<size_t>(g.tile_stride) * 4;  // K tile
+  b += static_cast<size_t>(D) * w * 4;                // comp / prefix maxima
+  b += 4 * static_cast<size_t>(D) * 4;                // capq, sig, rank, carry
+  b += 2 * static_cast<size_t>(w) * 4;                // slot, argA
+  b += 16;                                            // alignment slack
+  b += static_cast<size_t>(w) * 8;                    // maxA
+  b += 8;                                             // barrier
   g.smem = b;
   return g;
 }
 
 struct SnapWs {
-  uint32_t *zero;  // tcount[T2], tcursor[T2], flags[T2], ticket
+  uint32_t *zero;  // tcount[T2], tcursor[T2], nunits (zeroed per call)
+  size_t zero_words;
   uint32_t *toff;
-  int32_t *ord;
-  uint32_t *agg, *inc;
+  Unit *units;
+  int32_t *ord, *sp, *su;
+  int32_t *sig, *rank_of, *capq;
+  uint32_t *carry;  // [D][T2]
+  uint32_t *kmax;   // [D][ceil(H/16)], used when the caller passes none
+  int64_t max_units;
 };
 
-SnapWs carve_snap(Carve &c, int D, int T2, int64_t J) {
+SnapWs carve_snap(Carve &c, int D, int H, int T2, int64_t J) {
   SnapWs w;
-  w.zero = c.take<uint32_t>(3 * static_cast<size_t>(T2) + 1);
+  w.zero_words = 2 * static_cast<size_t>(T2) + 1;
+  w.zero = c.take<uint32_t>(w.zero_words);
   w.toff = c.take<uint32_t>(static_cast<size_t>(T2) + 1);
-  w.ord = c.take<int32_t>(static_cast<size_t>(J > 0 ? J : 1));
-  w.agg = c.take<uint32_t>(static_cast<size_t>(T2) * D);
-  w.inc = c.take<uint32_t>(static_cast<size_t>(T2) * D);
+  w.max_units = static_cast<int64_t>(T2) + (J + kUnitCands - 1) / kUnitCands;
+  w.units = c.take<Unit>(static_cast<size_t>(w.max_units) + 1);
+  const size_t nj = static_cast<size_t>(J > 0 ? J : 1);
+  w.ord = c.take<int32_t>(nj);
+  w.sp = c.take<int32_t>(nj);
+  w.su = c.take<int32_t>(nj);
+  w.sig = c.take<int32_t>(static_cast<size_t>(D));
+  w.rank_of = c.take<int32_t>(static_cast<size_t>(D));
+  w.capq = c.take<int32_t>(static_cast<size_t>(D));
+  w.carry = c.take<uint32_t>(static_cast<size_t>(T2) * D);
+  w.kmax = c.take<uint32_t>(static_cast<size_t>(D) * ((static_cast<size_t>(H) + kSumBlock - 1) / kSumBlock));
   return w;
 }
 
@@ -845,30 +1022,39 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 constexpr int kMaxH = 1 << 28;
 
 template <int W2>
-int run_snapshot(int grid, size_t smem, cudaStream_t s, const CUtensorMap &tmap, const SnapArgs &a) {
+int run_snapshot(int64_t grid, size_t smem, cudaStream_t s, const CUtensorMap &tmap, const SnapArgs &a) {
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(dispatch_snapshot_kernel<W2>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));
-  dispatch_snapshot_kernel<W2><<<grid, kMainThreads, smem, s>>>(tmap, a);
+  dispatch_snapshot_kernel<W2><<<static_cast<unsigned>(grid), kMainThreads, smem, s>>>(tmap, a);
   return launch_ok();
 }
 
-int launch_snapshot(int D, int H, const int32_t *K, const int32_t *cap, const int32_t *Q, int64_t J,
-                    const int32_t *cp, const int32_t *cb, int32_t *choice, int64_t *headroom,
-                    void *ws, cudaStream_t s) {
+int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const int32_t *cap,
+                    const int32_t *Q, int64_t J, const int32_t *cp, const int32_t *cb,
+                    int32_t *choice, int64_t *headroom, void *ws, cudaStream_t s) {
   const SnapGeom g = snap_geom(D, H);
   if (g.smem + 1024 > static_cast<size_t>(max_smem_optin())) return MAPS_E_INVALID;
   Carve cv(ws);
-  const SnapWs w = carve_snap(cv, D, g.T2, J);
+  const SnapWs w = carve_snap(cv, D, H, g.T2, J);
+  if (w.max_units > 0x7fffffffLL) return MAPS_E_INVALID;
   int32_t *status = status_word(ws);
-  uint32_t *tcount = w.zero, *tcursor = w.zero + g.T2, *flags = w.zero + 2 * static_cast<size_t>(g.T2);
-  uint32_t *ticket = w.zero + 3 * static_cast<size_t>(g.T2);
-  MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zero, 0, (3 * static_cast<size_t>(g.T2) + 1) * 4, s)));
+  uint32_t *tcount = w.zero, *tcursor = w.zero + g.T2;
+  uint32_t *nunits = w.zero + 2 * static_cast<size_t>(g.T2);
+  MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zero, 0, w.zero_words * 4, s)));
   const int sms = sm_count();
-  const int gb = static_cast<int>(std::min<int64_t>((J + 255) / 256, 4LL * sms));
-  bin_count_kernel<<<gb, 256, 0, s>>>(J, H, g.W2, cp, cb, tcount, choice, headroom, status);
-  bin_scan_kernel<<<1, 1024, 0, s>>>(g.T2, tcount, w.toff);
-  bin_scatter_kernel<<<gb, 256, 0, s>>>(J, H, g.W2, cp, cb, w.toff, tcursor, w.ord);
+  if (kmax == nullptr) {
+    const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
+    const int gk = static_cast<int>(std::min<int64_t>((nb * D + 255) / 256, 8LL * sms));
+    kmax_from_K_kernel<<<gk, 256, 0, s>>>(D, H, K, w.kmax, status);
+    kmax = w.kmax;
+  }
+  carry_scan_kernel<<<D, 256, 0, s>>>(D, H, g.W2, g.T2, kmax, w.carry);
+  const int gb = static_cast<int>(std::min<int64_t>((J + 1023) / 1024, 4LL * sms));
+  bin_count_kernel<<<gb, 1024, 0, s>>>(J, H, g.W2, g.T2, cp, cb, tcount, choice, headroom, status);
+  bin_scan_kernel<<<1, 1024, 0, s>>>(g.T2, tcount, w.toff, w.units, nunits, D, Q, cap, w.sig,
+                                     w.rank_of, w.capq, status);
+  bin_scatter_kernel<<<gb, 1024, 0, s>>>(J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord, w.sp, w.su);
   MAPS_TRY(launch_ok());
 
   CUtensorMap tmap;
@@ -898,20 +1084,19 @@ int launch_snapshot(int D, int H, const int32_t *K, const int32_t *cap, const in
   a.tile_stride = g.tile_stride;
   a.use_tma = use_tma;
   a.K = K;
-  a.cap = cap;
-  a.Q = Q;
-  a.cp = cp;
-  a.cb = cb;
-  a.toff = w.toff;
+  a.sig = w.sig;
+  a.rank_of = w.rank_of;
+  a.capq = w.capq;
+  a.carry = w.carry;
+  a.units = w.units;
+  a.nunits = nunits;
   a.ord = w.ord;
-  a.flags = flags;
-  a.agg = w.agg;
-  a.inc = w.inc;
-  a.ticket = ticket;
+  a.sp = w.sp;
+  a.su = w.su;
   a.choice = choice;
   a.headroom = headroom;
   a.status = status;
-  const int grid = std::min(sms, g.T2);
+  const int64_t grid = std::max<int64_t>(1, w.max_units);  // units past *nunits return at once
   switch (g.W2) {
     case 16: return run_snapshot<16>(grid, g.smem, s, tmap, a);
     case 32: return run_snapshot<32>(grid, g.smem, s, tmap, a);
@@ -931,15 +1116,15 @@ size_t maps_dispatch_workspace_size(int32_t mode, int32_t D, int32_t H, int64_t 
   Carve c(nullptr);
   if (mode == MAPS_MODE_SNAPSHOT && D >= 1 && H >= 1 && H <= kMaxH) {
     const SnapGeom g = snap_geom(D, H);
-    carve_snap(c, D, g.T2, J);
+    carve_snap(c, D, H, g.T2, J);
   } else if ((mode == MAPS_MODE_ALG1_SNAPSHOT || mode == MAPS_MODE_ALG1_SEQUENTIAL) && D >= 1) {
     c.take<long long>(static_cast<size_t>(D));
   }
   return c.bytes();
 }
 
-int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K, const int32_t *cap,
-                  int32_t *Q, const int64_t *res_off, int64_t R, const int32_t *prompt,
+int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K, const uint32_t *kmax,
+                  const int32_t *cap, int32_t *Q, const int64_t *res_off, int64_t R, const int32_t *prompt,
                   const int32_t *gen, const int32_t *bound, int64_t J, const int32_t *cand_prompt,
                   const int32_t *cand_bound, int32_t *choice_out, int64_t *headroom_out, void *ws,
                   size_t ws_bytes, void *stream) {
@@ -960,7 +1145,8 @@ int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K, con
   if (J == 0) return MAPS_OK;
   switch (mode) {
     case MAPS_MODE_SNAPSHOT:
-      return launch_snapshot(D, H, K, cap, Q, J, cand_prompt, cand_bound, choice_out, headroom_out, ws, s);
+      return launch_snapshot(D, H, K, kmax, cap, Q, J, cand_prompt, cand_bound, choice_out,
+                             headroom_out, ws, s);
     case MAPS_MODE_SEQUENTIAL:
       dispatch_sequential_kernel<<<1, 1024, 0, s>>>(D, H, K, cap, Q, J, cand_prompt, cand_bound,
                                                     choice_out, headroom_out, status);

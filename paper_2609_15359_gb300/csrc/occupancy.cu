@@ -3,21 +3,25 @@
 // K[k][t] = sum over residents r of decoder k with t < e_r of (b_r + t),
 // b_r = p_r + g_r + 1, e_r = min(max(U_r - g_r, 1), H), which is
 //   K[k][t] = SumB_k(t) + t * Cnt_k(t)
-// with Cnt / SumB the count and b-sum of residents ending after t.
+// with Cnt / SumB the count and b-sum of residents still live at t.
 //
-// One CTA owns one (decoder, horizon tile of W steps).  It sweeps the
-// decoder's residents once: a resident ending inside the tile goes into a
-// shared-memory difference histogram at its end step; one ending at or after
-// the tile's end only adds to the carry (count, b-sum) that every cell of the
-// tile sees.  The carry is therefore computed directly by each tile and no
-// tile waits on another.  A reverse scan of the histogram then gives each
-// cell's suffix count and sum, and the tile is written with 128-bit stores.
+// Layout of the work.  One CTA owns one decoder and a chunk of up to four
+// horizon tiles of W steps.  It loads the decoder's residents once, keeps
+// each resident's footprint at t = 0 (b) and end step (e) in shared memory,
+// and walks its tiles from the highest down.  For a tile, residents ending
+// inside it go into a shared-memory end-step histogram; those ending after
+// it form the tile's carry (count, b-sum), which is the previous tile's carry
+// plus the previous tile's bin totals.  A reverse scan of the histogram
+// gives each cell's live count and b-sum, and the tile is written with
+// 128-bit stores.  Chunks of the same decoder re-read the residents from L2.
+// Optionally every group of 16 steps also yields
+// kmax[k][t/16] = max (K[k][t] + t), a summary the dispatch uses for the
+// prefix maxima of earlier horizon tiles.
 //
 // Integer range: every resident is live at t = 0, so K[k][0] = sum of b_r
-// over the decoder and every partial sum in the tile is at most K[k][0].  If
-// that total exceeds INT32_MAX the call reports MAPS_E_RANGE; otherwise the
-// 32-bit shared-memory sums cannot wrap and each cell is formed exactly in
-// 64 bits before its own range check.
+// and every partial sum is at most K[k][0]; if that total exceeds INT32_MAX
+// the call reports MAPS_E_RANGE, otherwise the 32-bit shared-memory sums
+// cannot wrap and each cell is formed exactly in 64 bits.
 #include "maps_internal.cuh"
 
 namespace maps {
@@ -25,58 +29,91 @@ namespace {
 
 constexpr int kOccThreads = 512;
 constexpr int kWarps = kOccThreads / 32;
+constexpr int kTilesPerChunk = 4;
+constexpr int kBlock = 16;    // steps per kmax summary entry
+constexpr int kStage = 4096;  // residents staged in shared memory at a time
 
 template <int CPT, bool VEC>
-__global__ void __launch_bounds__(kOccThreads)
-occupancy_kernel(int D, int H, int T, const int64_t *__restrict__ res_off, int64_t R,
+__global__ void __launch_bounds__(kOccThreads, 2)
+occupancy_kernel(int D, int H, int TPC, int G, const int64_t *__restrict__ res_off, int64_t R,
                  const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
-                 const int32_t *__restrict__ bound, int32_t *__restrict__ K, int32_t *status) {
+                 const int32_t *__restrict__ bound, int32_t *__restrict__ K,
+                 uint32_t *__restrict__ kmax, int32_t *status) {
   constexpr int W = kOccThreads * CPT;
-  __shared__ int32_t s_cnt[W + 1];  // bin m (1..W-1): residents ending at t0 + m
-  __shared__ int32_t s_sb[W + 1];   // ... and the sum of their b
+  __shared__ __align__(16) int32_t s_cnt[W];  // bin j: residents whose last live step is t0 + j
+  __shared__ __align__(16) int32_t s_sb[W];   // ... and the sum of their b
+  __shared__ int2 s_res[kStage];    // staged residents (b, e); e = 0 marks one outside the domain
   __shared__ long long s_red[3][kWarps];
   __shared__ int32_t s_scan[2][kWarps];
+  __shared__ long long s_carry[2];
 
-  const int k = blockIdx.x / T;
-  const int tile = blockIdx.x - k * T;
-  const int64_t t0 = static_cast<int64_t>(tile) * W;
+  const int k = blockIdx.x / G, chunk = blockIdx.x - (blockIdx.x / G) * G;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t tile_lo = static_cast<int64_t>(chunk) * TPC;
+  const int64_t tiles_all = (static_cast<int64_t>(H) + W - 1) / W;
+  const int ntile = static_cast<int>(min(static_cast<int64_t>(TPC), tiles_all - tile_lo));
+  const int64_t chunk_end = (tile_lo + ntile) * W;  // first step after this chunk
 
-  for (int i = tid; i <= W; i += kOccThreads) {
-    s_cnt[i] = 0;
-    s_sb[i] = 0;
-  }
   int64_t lo = res_off[k], hi = res_off[k + 1];
   if (lo < 0 || hi < lo || hi > R) {
-    if (tid == 0) flag_error(status, MAPS_E_RANGE);
+    if (tid == 0 && chunk == 0) flag_error(status, MAPS_E_RANGE);
     lo = hi = 0;
   }
-  __syncthreads();
-
-  long long carry_c = 0, carry_s = 0, total_b = 0;
+  const int64_t nres = hi - lo;
+  const bool staged_once = nres <= kStage;  // residents stay staged for all tiles
   bool bad = false;
-  for (int64_t r = lo + tid; r < hi; r += kOccThreads) {
-    const int32_t p = __ldg(prompt + r), g = __ldg(gen + r), U = __ldg(bound + r);
-    if ((p | g | U) < 0) {
-      bad = true;
-      continue;
+
+  // Stage residents [b0, b0 + n) of the decoder as (b, e); each thread
+  // issues the loads of all its residents before using any.
+  constexpr int kPer = kStage / kOccThreads;
+  auto stage = [&](int64_t b0, int n) {
+    int32_t p[kPer], gg[kPer], U[kPer];
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+      const int i = j * kOccThreads + tid;
+      const int64_t r = lo + b0 + i;
+      const bool ok = i < n;
+      p[j] = ok ? __ldg(prompt + r) : 0;
+      gg[j] = ok ? __ldg(gen + r) : 0;
+      U[j] = ok ? __ldg(bound + r) : 0;
     }
-    const long long b = static_cast<long long>(p) + g + 1;
-    long long e = static_cast<long long>(U) - g;
-    e = e < 1 ? 1 : (e > H ? H : e);
-    total_b += b;
-    if (e >= t0 + W) {
-      carry_c += 1;
-      carry_s += b;
-    } else if (e > t0) {
-      const int m = static_cast<int>(e - t0);
-      atomicAdd(&s_cnt[m], 1);
-      atomicAdd(&s_sb[m], static_cast<int32_t>(b));  // exact when total_b fits int32
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+      const int i = j * kOccThreads + tid;
+      if (i >= n) break;
+      int2 v = make_int2(0, 0);
+      if ((p[j] | gg[j] | U[j]) < 0) {
+        bad = true;
+      } else {
+        const long long b = static_cast<long long>(p[j]) + gg[j] + 1;
+        long long e = static_cast<long long>(U[j]) - gg[j];
+        e = e < 1 ? 1 : (e > H ? H : e);
+        if (b > 0x7fffffffLL) bad = true;  // K[k][0] = sum of b overflows
+        v = make_int2(static_cast<int32_t>(b > 0x7fffffffLL ? 0x7fffffffLL : b),
+                      static_cast<int32_t>(e));
+      }
+      s_res[i] = v;
+    }
+  };
+
+  // 1. Carry into the chunk's highest tile (residents live past the chunk)
+  //    and the decoder's whole sum of b.
+  long long carry_c = 0, carry_s = 0, total_b = 0;
+  for (int64_t b0 = 0; b0 < nres; b0 += kStage) {
+    const int n = static_cast<int>(min(static_cast<int64_t>(kStage), nres - b0));
+    __syncthreads();
+    stage(b0, n);
+    __syncthreads();
+    for (int i = tid; i < n; i += kOccThreads) {
+      const int2 v = s_res[i];
+      if (v.y == 0) continue;
+      total_b += v.x;
+      if (v.y > chunk_end) {
+        carry_c += 1;
+        carry_s += v.x;
+      }
     }
   }
-  if (bad) flag_error(status, MAPS_E_RANGE);
-
-  // block sums of the carry and of the decoder's total b
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     carry_c += __shfl_xor_sync(0xffffffffu, carry_c, off);
@@ -89,80 +126,172 @@ occupancy_kernel(int D, int H, int T, const int64_t *__restrict__ res_off, int64
     s_red[2][warp] = total_b;
   }
   __syncthreads();
-  carry_c = carry_s = total_b = 0;
-#pragma unroll
-  for (int w = 0; w < kWarps; ++w) {
-    carry_c += s_red[0][w];
-    carry_s += s_red[1][w];
-    total_b += s_red[2][w];
-  }
-  if (total_b > 0x7fffffffLL && tid == 0 && tile == 0) flag_error(status, MAPS_E_RANGE);
-
-  // Thread tid owns cells l = tid*CPT + c and bins m = l + 1.  Cell l needs
-  // the sums over bins m > l: its own bins above l plus every bin of the
-  // threads above it (an exclusive suffix scan of the per-thread totals).
-  int32_t own_c[CPT], own_s[CPT];
-  int32_t tot_c = 0, tot_s = 0;
-#pragma unroll
-  for (int c = 0; c < CPT; ++c) {
-    own_c[c] = s_cnt[tid * CPT + c + 1];
-    own_s[c] = s_sb[tid * CPT + c + 1];
-    tot_c += own_c[c];
-    tot_s += own_s[c];
-  }
-  int32_t suf_c = tot_c, suf_s = tot_s;  // inclusive suffix within the warp
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const int32_t yc = __shfl_down_sync(0xffffffffu, suf_c, off);
-    const int32_t ys = __shfl_down_sync(0xffffffffu, suf_s, off);
-    if (lane + off < 32) {
-      suf_c += yc;
-      suf_s += ys;
+  if (tid == 0) {
+    long long a = 0, b = 0, t = 0;
+    for (int w = 0; w < kWarps; ++w) {
+      a += s_red[0][w];
+      b += s_red[1][w];
+      t += s_red[2][w];
     }
+    s_carry[0] = a;
+    s_carry[1] = b;
+    if (chunk == 0 && t > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
   }
-  if (lane == 0) {
-    s_scan[0][warp] = suf_c;
-    s_scan[1][warp] = suf_s;
+
+  // 2. Tiles from the highest down.  The histograms start zeroed and each
+  //    thread clears its own bins right after reading them.
+  for (int i = tid; i < W; i += kOccThreads) {
+    s_cnt[i] = 0;
+    s_sb[i] = 0;
   }
   __syncthreads();
-  long long run_c = carry_c + (suf_c - tot_c);
-  long long run_s = carry_s + (suf_s - tot_s);
-  for (int w = warp + 1; w < kWarps; ++w) {
-    run_c += s_scan[0][w];
-    run_s += s_scan[1][w];
-  }
-
-  int32_t out[CPT];
   bool over = false;
-#pragma unroll
-  for (int c = CPT - 1; c >= 0; --c) {
-    run_c += own_c[c];
-    run_s += own_s[c];
-    const long long t = t0 + tid * CPT + c;
-    long long v = run_s + t * run_c;
-    if (v > 0x7fffffffLL) {
-      if (t < H) over = true;  // only cells inside the horizon count
-      v = 0x7fffffffLL;
-    }
-    out[c] = static_cast<int32_t>(v);
-  }
-
-  const int64_t cell0 = t0 + static_cast<int64_t>(tid) * CPT;
-  int32_t *row = K + static_cast<int64_t>(k) * H;
-  if (VEC) {
-    // H % 4 == 0 and CPT % 4 == 0: each group of 4 is wholly inside or outside
-#pragma unroll
-    for (int c = 0; c < CPT; c += 4) {
-      if (cell0 + c < H) {
-        *reinterpret_cast<int4 *>(row + cell0 + c) = make_int4(out[c], out[c + 1], out[c + 2], out[c + 3]);
+  for (int ti = ntile - 1; ti >= 0; --ti) {
+    const int64_t t0 = (tile_lo + ti) * W;
+    for (int64_t b0 = 0; b0 < nres; b0 += kStage) {
+      const int n = static_cast<int>(min(static_cast<int64_t>(kStage), nres - b0));
+      if (!staged_once) {
+        __syncthreads();
+        stage(b0, n);
+        __syncthreads();
+      }
+      for (int i = tid; i < n; i += kOccThreads) {
+        const int2 v = s_res[i];
+        const long long e = v.y;
+        if (e > t0 && e <= t0 + W) {
+          const int j = static_cast<int>(e - t0 - 1);  // last live cell, 0..W-1
+          atomicAdd(&s_cnt[j], 1);
+          atomicAdd(&s_sb[j], v.x);  // exact while sum b fits int32
+        }
       }
     }
-  } else {
+    __syncthreads();
+
+    // Thread tid owns cells l = tid*CPT + c and the bins with the same index
+    // (residents whose last live step is that cell).  Cell l needs every bin
+    // j >= l: its own bins from l up plus all bins of the threads above it
+    // (an exclusive suffix scan of the per-thread totals).  All sums are below
+    // K[k][0] <= INT32_MAX unless a range error is already flagged, so they
+    // are kept in 32 bits; each cell is formed with one widening multiply.
+    int32_t oc[CPT], os[CPT];
 #pragma unroll
-    for (int c = 0; c < CPT; ++c)
-      if (cell0 + c < H) row[cell0 + c] = out[c];
+    for (int c = 0; c < CPT; c += 4) {
+      const int4 x = *reinterpret_cast<const int4 *>(&s_cnt[tid * CPT + c]);
+      const int4 y = *reinterpret_cast<const int4 *>(&s_sb[tid * CPT + c]);
+      oc[c] = x.x, oc[c + 1] = x.y, oc[c + 2] = x.z, oc[c + 3] = x.w;
+      os[c] = y.x, os[c + 1] = y.y, os[c + 2] = y.z, os[c + 3] = y.w;
+      *reinterpret_cast<int4 *>(&s_cnt[tid * CPT + c]) = make_int4(0, 0, 0, 0);
+      *reinterpret_cast<int4 *>(&s_sb[tid * CPT + c]) = make_int4(0, 0, 0, 0);
+    }
+    uint32_t tot_c = 0, tot_s = 0;
+#pragma unroll
+    for (int c = 0; c < CPT; ++c) {
+      tot_c += static_cast<uint32_t>(oc[c]);
+      tot_s += static_cast<uint32_t>(os[c]);
+    }
+    uint32_t suf_c = tot_c, suf_s = tot_s;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t yc = __shfl_down_sync(0xffffffffu, suf_c, off);
+      const uint32_t ys = __shfl_down_sync(0xffffffffu, suf_s, off);
+      if (lane + off < 32) {
+        suf_c += yc;
+        suf_s += ys;
+      }
+    }
+    if (lane == 0) {
+      s_scan[0][warp] = static_cast<int32_t>(suf_c);
+      s_scan[1][warp] = static_cast<int32_t>(suf_s);
+    }
+    __syncthreads();
+    const long long cc = s_carry[0], cs = s_carry[1];
+    uint32_t run_c = static_cast<uint32_t>(cc) + (suf_c - tot_c);
+    uint32_t run_s = static_cast<uint32_t>(cs) + (suf_s - tot_s);
+    for (int w = warp + 1; w < kWarps; ++w) {
+      run_c += static_cast<uint32_t>(s_scan[0][w]);
+      run_s += static_cast<uint32_t>(s_scan[1][w]);
+    }
+
+    uint32_t bmax = 0;  // max of K + t over this thread's valid cells
+    const int64_t cell0 = t0 + static_cast<int64_t>(tid) * CPT;
+    const uint32_t tc0 = static_cast<uint32_t>(cell0);
+    int32_t *row = K + static_cast<int64_t>(k) * H;
+    int32_t out[CPT];
+#pragma unroll
+    for (int c = CPT - 1; c >= 0; --c) {
+      run_c += static_cast<uint32_t>(oc[c]);
+      run_s += static_cast<uint32_t>(os[c]);
+      const uint32_t t = tc0 + c;
+      // K = run_s + t * run_c, exact in 64 bits
+      const unsigned long long v = static_cast<unsigned long long>(t) * run_c + run_s;
+      uint32_t o = static_cast<uint32_t>(v);
+      if (v > 0x7fffffffull) {
+        if (cell0 + c < H) over = true;
+        o = 0x7fffffffu;
+      }
+      out[c] = static_cast<int32_t>(o);
+      if (cell0 + c < H) {
+        const uint32_t x = o + t;
+        bmax = x > bmax ? x : bmax;
+      }
+    }
+    if (VEC) {
+#pragma unroll
+      for (int c = 0; c < CPT; c += 4)
+        if (cell0 + c < H)
+          *reinterpret_cast<int4 *>(row + cell0 + c) = make_int4(out[c], out[c + 1], out[c + 2], out[c + 3]);
+    } else {
+#pragma unroll
+      for (int c = 0; c < CPT; ++c)
+        if (cell0 + c < H) row[cell0 + c] = out[c];
+    }
+    if (kmax != nullptr) {
+      constexpr int L = kBlock / CPT;  // lanes per 16-step block
+#pragma unroll
+      for (int off = L / 2; off > 0; off >>= 1) {
+        const uint32_t y = __shfl_xor_sync(0xffffffffu, bmax, off);
+        bmax = y > bmax ? y : bmax;
+      }
+      if ((lane % L) == 0 && cell0 < H) {
+        const int64_t nb = (static_cast<int64_t>(H) + kBlock - 1) / kBlock;
+        kmax[static_cast<int64_t>(k) * nb + cell0 / kBlock] = bmax;
+      }
+    }
+    // the next lower tile also carries this tile's residents
+    if (tid == 0) {
+      long long bc = 0, bs = 0;
+      for (int w = 0; w < kWarps; ++w) {
+        bc += static_cast<uint32_t>(s_scan[0][w]);
+        bs += static_cast<uint32_t>(s_scan[1][w]);
+      }
+      s_carry[0] = cc + bc;
+      s_carry[1] = cs + bs;
+    }
+    __syncthreads();
   }
-  if (over) flag_error(status, MAPS_E_RANGE);
+  if (bad || over) flag_error(status, MAPS_E_RANGE);
+}
+
+int launch_occ(int cpt, bool vec, int64_t blocks, cudaStream_t s, int D, int H, int TPC, int G,
+               const int64_t *res_off, int64_t R, const int32_t *prompt, const int32_t *gen,
+               const int32_t *bound, int32_t *K, uint32_t *kmax, int32_t *status) {
+  const dim3 grid(static_cast<unsigned>(blocks));
+  if (cpt == 8) {
+    if (vec)
+      occupancy_kernel<8, true><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
+                                                             bound, K, kmax, status);
+    else
+      occupancy_kernel<8, false><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
+                                                              bound, K, kmax, status);
+  } else if (cpt == 4) {
+    if (vec)
+      occupancy_kernel<4, true><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
+                                                             bound, K, kmax, status);
+    else
+      occupancy_kernel<4, false><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
+                                                              bound, K, kmax, status);
+  }
+  return launch_ok();
 }
 
 }  // namespace
@@ -179,30 +308,24 @@ size_t maps_project_occupancy_workspace_size(int32_t D, int32_t H, int64_t R) {
 
 int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off, int64_t R,
                            const int32_t *prompt, const int32_t *gen, const int32_t *bound,
-                           int32_t *K_out, void *ws, size_t ws_bytes, void *stream) {
+                           int32_t *K_out, uint32_t *kmax_out, void *ws, size_t ws_bytes,
+                           void *stream) {
   using namespace maps;
   if (D < 1 || H < 1 || R < 0 || res_off == nullptr || K_out == nullptr) return MAPS_E_INVALID;
   if (R > 0 && (prompt == nullptr || gen == nullptr || bound == nullptr)) return MAPS_E_INVALID;
   MAPS_TRY(check_ws(ws, ws_bytes, maps_project_occupancy_workspace_size(D, H, R)));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int32_t *status = status_word(ws);
-  const bool big = H > 512;
-  const int W = kOccThreads * (big ? 8 : 1);
-  const int64_t T = (static_cast<int64_t>(H) + W - 1) / W;
-  const int64_t blocks = T * D;
+  const int cpt = H <= 2048 ? 4 : 8;
+  const int64_t W = static_cast<int64_t>(kOccThreads) * cpt;
+  const int64_t tiles = (H + W - 1) / W;
+  const int TPC = static_cast<int>(tiles < kTilesPerChunk ? tiles : kTilesPerChunk);
+  const int64_t G = (tiles + TPC - 1) / TPC;
+  const int64_t blocks = static_cast<int64_t>(D) * G;
   if (blocks > 0x7fffffffLL) return MAPS_E_INVALID;
   const bool vec = (H % 4 == 0) && aligned(K_out, 16);
-  const dim3 grid(static_cast<unsigned>(blocks));
-  const int Ti = static_cast<int>(T);
-  if (big) {
-    if (vec)
-      occupancy_kernel<8, true><<<grid, kOccThreads, 0, s>>>(D, H, Ti, res_off, R, prompt, gen, bound, K_out, status);
-    else
-      occupancy_kernel<8, false><<<grid, kOccThreads, 0, s>>>(D, H, Ti, res_off, R, prompt, gen, bound, K_out, status);
-  } else {
-    occupancy_kernel<1, false><<<grid, kOccThreads, 0, s>>>(D, H, Ti, res_off, R, prompt, gen, bound, K_out, status);
-  }
-  return launch_ok();
+  return launch_occ(cpt, vec, blocks, s, D, H, TPC, static_cast<int>(G), res_off, R, prompt, gen,
+                    bound, K_out, kmax_out, status);
 }
 
 }  // extern "C"

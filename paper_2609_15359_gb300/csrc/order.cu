@@ -1,22 +1,24 @@
 // order.cu -- local SJF reordering with max-wait promotion (Sec. 3.3).
 //
 // The queue order is the lexicographic order of
-//     (decoder, not promoted, promoted ? arrival : bound, arrival, index)
-// computed as a stable least-significant-digit radix sort of 8-bit digits:
-//   * one upfront pass builds the 64-bit key (decoder << 32 | not-promoted
-//     << 31 | primary), counts every digit of it and of the arrival, counts
-//     entries per decoder, and checks whether arrival is already
-//     non-decreasing in index;
-//   * a one-block plan kernel turns the counts into digit offsets, marks a
-//     digit pass inactive when every key has the same digit, and skips the
-//     arrival passes when arrival is already in index order (stability then
-//     gives the arrival tie-break for free);
-//   * each active digit pass is a single sweep: tiles of 4096 keys are
-//     ranked in shared memory (warp match + per-warp histograms, stable),
-//     the per-digit tile offsets come from a decoupled look-back across
-//     tiles taken in ticket order, and each tile is written out bin by bin.
-// Passes that the plan marks inactive return at once, so the host never
-// waits for the plan.
+//     (decoder, not promoted, promoted ? arrival : bound, arrival, index).
+// It is computed as a stable least-significant-digit radix sort of 8-bit
+// digits over a compact key:
+//   * entries are first put in arrival order (stable), unless arrival is
+//     already non-decreasing in index, which the first pass checks;
+//   * the key is then  decoder << (1 + ub) | not_promoted << ub | (not
+//     promoted ? bound : 0), with ub the bit width of the largest bound of a
+//     non-promoted entry: promoted entries need no primary key because the
+//     arrival order is already in place and the sort is stable;
+//   * a key of at most 32 bits is sorted as 32 bits, otherwise as 64 bits.
+// Kernels: a prep pass (validation, promoted flags, largest bound, entries
+// per decoder, arrival order check), a key pass (keys and every digit
+// histogram), a one-block plan (digit offsets, which passes run, buffers,
+// decoder segment offsets), then one sweep per digit: tiles of 4096 keys are
+// ranked stably in shared memory, each tile learns its offsets from earlier
+// tiles by decoupled look-back (256 predecessors inspected per round, one
+// thread each), and writes out bin by bin.  Passes the plan marks inactive return at once,
+// so the host never waits on the device.
 #include "maps_internal.cuh"
 
 #include <algorithm>
@@ -29,25 +31,30 @@ constexpr int kPassThreads = 512;
 constexpr int kIPT = 8;
 constexpr int kTile = kPassThreads * kIPT;  // 4096 keys per tile
 constexpr int kPassWarps = kPassThreads / 32;
-constexpr int kLoPasses = 4;   // arrival digits
-constexpr int kHiPasses = 8;   // key digits (only the low ones can vary)
+constexpr int kLoPasses = 4;  // arrival digits
+constexpr int kHiPasses = 8;  // key digits
 constexpr int kPasses = kLoPasses + kHiPasses;
-constexpr unsigned long long kAgg = 1ull << 62, kInc = 2ull << 62;
-constexpr unsigned long long kValMask = 0xffffffffull;
+constexpr int kDecSmem = 8192;  // decoders counted in shared memory up to this D
+constexpr uint32_t kFlagAgg = 1, kFlagInc = 2;
+constexpr int kLookWindow = 256;  // predecessor tiles inspected per look-back round
 
 enum : int32_t { kBufA = 0, kBufB = 1, kHiIdentity = 2, kPermOut = 2 };
 
 struct OrderCounts {
   uint32_t h[kPasses][kRadix];
-  uint32_t unsorted;
+  uint32_t unsorted;   // arrival decreases somewhere along the index
+  uint32_t max_bound;  // largest bound of a non-promoted entry
 };
 
 struct OrderPlan {
   int32_t active[kPasses];
   int32_t src[kPasses];
   int32_t dst[kPasses];
+  int32_t shift[kPasses];
   int32_t gather_buf;  // -1: none
   int32_t npasses;
+  int32_t wide;        // keys need 64 bits
+  int32_t ubits;       // bit width of the primary (bound) field
   uint32_t digit_off[kPasses][kRadix];
 };
 
@@ -57,57 +64,131 @@ __device__ __forceinline__ unsigned lanemask_lt() {
   return m;
 }
 
-// Warp-aggregated shared-memory increment of bin `b` (all lanes active).
+// Warp-aggregated shared-memory increment of bin `b` (all lanes present).
 __device__ __forceinline__ void warp_count(uint32_t *hist, int b, bool valid) {
   const unsigned peers = __match_any_sync(0xffffffffu, valid ? b : -1);
-  const int lane = threadIdx.x & 31;
-  if (valid && lane == __ffs(peers) - 1) atomicAdd(&hist[b], static_cast<uint32_t>(__popc(peers)));
+  if (valid && static_cast<int>(threadIdx.x & 31) == __ffs(peers) - 1)
+    atomicAdd(&hist[b], static_cast<uint32_t>(__popc(peers)));
 }
 
+__device__ __forceinline__ int bit_width(uint32_t x) { return x ? 32 - __clz(x) : 0; }
+
+// Pass 1: validation, largest non-promoted bound, entries per decoder, and
+// whether arrival is non-decreasing.
 __global__ void __launch_bounds__(512)
-order_prep_kernel(int64_t N, int D, int n_hi, const int32_t *__restrict__ dec,
+order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
-                  const int32_t *__restrict__ arrival, int32_t max_wait,
-                  unsigned long long *hi_orig, unsigned long long *keyA, uint32_t *valA,
-                  OrderCounts *counts, uint32_t *dec_count, int32_t *status) {
+                  const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
+                  uint32_t *dec_count, int32_t *status) {
+  __shared__ uint32_t s_dec[kDecSmem];
+  const bool dec_smem = D <= kDecSmem;
+  if (dec_smem)
+    for (int i = threadIdx.x; i < D; i += blockDim.x) s_dec[i] = 0;
+  __syncthreads();
+  bool bad = false, unsorted = false;
+  uint32_t umax = 0;
+  constexpr int kU = 4;  // entries per thread per round, loads issued together
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x * kU;
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x * kU; i0 < N; i0 += stride) {
+    int32_t d[kU], u[kU], w[kU], ar[kU], an[kU];
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int64_t i = i0 + q * blockDim.x + threadIdx.x;
+      const bool ok = i < N;
+      d[q] = ok ? __ldg(dec + i) : -1;
+      u[q] = ok ? __ldg(bound + i) : 0;
+      w[q] = ok ? __ldg(wait + i) : 0;
+      ar[q] = ok ? __ldg(arrival + i) : 0;
+      an[q] = (ok && i + 1 < N) ? __ldg(arrival + i + 1) : 0x7fffffff;
+    }
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int64_t i = i0 + q * blockDim.x + threadIdx.x;
+      int dd = -1;
+      if (i < N) {
+        dd = d[q];
+        if (dd < 0 || dd >= D || u[q] < 0 || ar[q] < 0) {
+          bad = true;
+          dd = dd < 0 || dd >= D ? 0 : dd;
+        }
+        if (w[q] <= max_wait && u[q] > 0) umax = max(umax, static_cast<uint32_t>(u[q]));
+        if (an[q] < ar[q]) unsorted = true;
+      }
+      if (dec_smem) {
+        if (dd >= 0) atomicAdd(&s_dec[dd], 1u);
+      } else {
+        const unsigned peers = __match_any_sync(0xffffffffu, dd);
+        if (dd >= 0 && static_cast<int>(threadIdx.x & 31) == __ffs(peers) - 1)
+          atomicAdd(&dec_count[dd], static_cast<uint32_t>(__popc(peers)));
+      }
+    }
+  }
+  if (bad) flag_error(status, MAPS_E_RANGE);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) umax = max(umax, __shfl_xor_sync(0xffffffffu, umax, off));
+  if ((threadIdx.x & 31) == 0 && umax) atomicMax(&counts->max_bound, umax);
+  if (__syncthreads_or(unsorted) && threadIdx.x == 0) atomicOr(&counts->unsorted, 1u);
+  if (dec_smem)
+    for (int i = threadIdx.x; i < D; i += blockDim.x)
+      if (s_dec[i]) atomicAdd(&dec_count[i], s_dec[i]);
+}
+
+// Pass 2: keys in the compact layout and the histograms of every digit.
+__global__ void __launch_bounds__(512)
+order_keys_kernel(int64_t N, int D, int dbits, const int32_t *__restrict__ dec,
+                  const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
+                  const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
+                  unsigned long long *hi_orig, unsigned long long *keyA, uint32_t *valA) {
   __shared__ uint32_t sh[kPasses][kRadix];
   for (int i = threadIdx.x; i < kPasses * kRadix; i += blockDim.x) (&sh[0][0])[i] = 0;
   __syncthreads();
-  bool bad = false, unsorted = false;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  // the loop bound depends only on the block's first index, so whole warps
-  // iterate together and the warp-wide matches below see every lane
-  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x; i0 < N; i0 += stride) {
-    const int64_t i = i0 + threadIdx.x;
-    const bool valid = i < N;
-    unsigned long long hi = 0;
-    uint32_t a = 0;
-    if (valid) {
-      int32_t d = dec[i], u = bound[i], w = wait[i], ar = arrival[i];
-      if (d < 0 || d >= D || u < 0 || ar < 0) {
-        bad = true;
-        d = d < 0 || d >= D ? 0 : d;
-        u = u < 0 ? 0 : u;
-        ar = ar < 0 ? 0 : ar;
-      }
-      const bool promoted = w > max_wait;
-      const uint32_t prim = static_cast<uint32_t>(promoted ? ar : u);
-      hi = (static_cast<unsigned long long>(d) << 32) |
-           (static_cast<unsigned long long>(promoted ? 0u : 1u) << 31) | prim;
-      a = static_cast<uint32_t>(ar);
-      hi_orig[i] = hi;
-      keyA[i] = a;
-      valA[i] = static_cast<uint32_t>(i);
-      atomicAdd(&dec_count[d], 1u);
-      if (i + 1 < N && arrival[i + 1] < ar) unsorted = true;
+  const int ub = bit_width(*reinterpret_cast<volatile uint32_t *>(&counts->max_bound));
+  const bool unsorted = *reinterpret_cast<volatile uint32_t *>(&counts->unsorted) != 0;
+  const bool wide = dbits + 1 + ub > 32;
+  const int n_hi = (dbits + 1 + ub + 7) / 8;
+  constexpr int kU = 4;  // entries per thread per round, loads issued together
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x * kU;
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x * kU; i0 < N; i0 += stride) {
+    int32_t d[kU], u[kU], ar[kU], w[kU];
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int64_t i = i0 + q * blockDim.x + threadIdx.x;
+      const bool ok = i < N;
+      d[q] = ok ? __ldg(dec + i) : 0;
+      u[q] = ok ? __ldg(bound + i) : 0;
+      ar[q] = ok ? __ldg(arrival + i) : 0;
+      w[q] = ok ? __ldg(wait + i) : 0;
     }
 #pragma unroll
-    for (int p = 0; p < kLoPasses; ++p) warp_count(sh[p], (a >> (8 * p)) & 255u, valid);
-    for (int p = 0; p < n_hi; ++p)
-      warp_count(sh[kLoPasses + p], static_cast<int>((hi >> (8 * p)) & 255u), valid);
+    for (int q = 0; q < kU; ++q) {
+      const int64_t i = i0 + q * blockDim.x + threadIdx.x;
+      const bool valid = i < N;
+      unsigned long long key = 0;
+      uint32_t a = 0;
+      if (valid) {
+        const int32_t dd = d[q] < 0 || d[q] >= D ? 0 : d[q];  // out-of-domain entries were flagged
+        const int32_t uu = u[q] < 0 ? 0 : u[q];
+        const int32_t aa = ar[q] < 0 ? 0 : ar[q];
+        const bool promoted = w[q] > max_wait;
+        const unsigned long long prim = promoted ? 0ull : static_cast<unsigned long long>(uu);
+        key = (static_cast<unsigned long long>(dd) << (1 + ub)) |
+              (static_cast<unsigned long long>(promoted ? 0u : 1u) << ub) | prim;
+        a = static_cast<uint32_t>(aa);
+        hi_orig[i] = key;
+        if (unsorted) {
+          keyA[i] = a;
+          valA[i] = static_cast<uint32_t>(i);
+        }
+      }
+      if (unsorted)
+#pragma unroll
+        for (int p = 0; p < kLoPasses; ++p) warp_count(sh[p], (a >> (8 * p)) & 255u, valid);
+      for (int p = 0; p < n_hi; ++p)
+        warp_count(sh[kLoPasses + p], static_cast<int>((key >> (8 * p)) & 255u), valid);
+    }
   }
-  if (bad) flag_error(status, MAPS_E_RANGE);
-  if (__syncthreads_or(unsorted) && threadIdx.x == 0) atomicOr(&counts->unsorted, 1u);
+  (void)wide;
+  __syncthreads();
   for (int i = threadIdx.x; i < kPasses * kRadix; i += blockDim.x) {
     const uint32_t c = (&sh[0][0])[i];
     if (c) atomicAdd(&(&counts->h[0][0])[i], c);
@@ -117,7 +198,7 @@ order_prep_kernel(int64_t N, int D, int n_hi, const int32_t *__restrict__ dec,
 // One block: digit offsets, active passes, buffer assignment, and the
 // decoder segment offsets.
 __global__ void __launch_bounds__(kRadix)
-order_plan_kernel(int64_t N, int D, int n_hi, const OrderCounts *counts, OrderPlan *plan,
+order_plan_kernel(int64_t N, int D, int dbits, const OrderCounts *counts, OrderPlan *plan,
                   const uint32_t *dec_count, int64_t *seg_off) {
   __shared__ uint32_t s_warp[kRadix / 32];
   __shared__ long long s_w64[kRadix / 32];
@@ -133,7 +214,7 @@ order_plan_kernel(int64_t N, int D, int n_hi, const OrderCounts *counts, OrderPl
       if (lane >= off) incl += y;
     }
     if (lane == 31) s_warp[warp] = incl;
-    const int triv = __syncthreads_or(static_cast<int64_t>(c) == N);
+    const int triv = __syncthreads_or(static_cast<int64_t>(c) == N || N == 0);
     uint32_t base = 0;
     for (int w = 0; w < warp; ++w) base += s_warp[w];
     plan->digit_off[p][b] = base + incl - c;
@@ -142,8 +223,15 @@ order_plan_kernel(int64_t N, int D, int n_hi, const OrderCounts *counts, OrderPl
   }
   if (b == 0) {
     const bool unsorted = counts->unsorted != 0;
+    const int ub = counts->max_bound ? 32 - __clz(counts->max_bound) : 0;
+    const int n_hi = min(kHiPasses, (dbits + 1 + ub + 7) / 8);
+    plan->ubits = ub;
+    plan->wide = dbits + 1 + ub > 32;
     int last = -1, n = 0, buf = kBufA;  // buffer holding the current keys
-    for (int p = 0; p < kPasses; ++p) plan->active[p] = 0;
+    for (int p = 0; p < kPasses; ++p) {
+      plan->active[p] = 0;
+      plan->shift[p] = p < kLoPasses ? 8 * p : 8 * (p - kLoPasses);
+    }
     plan->gather_buf = -1;
     if (N > 0) {
       if (unsorted)
@@ -203,17 +291,24 @@ order_plan_kernel(int64_t N, int D, int n_hi, const OrderCounts *counts, OrderPl
   }
 }
 
-// After arrival passes: keys of the hi passes follow the arrival order.
-__global__ void order_gather_kernel(int64_t N, const OrderPlan *plan, const unsigned long long *hi_orig,
-                                    unsigned long long *keyA, unsigned long long *keyB,
-                                    const uint32_t *valA, const uint32_t *valB) {
+// After arrival passes: the keys follow the arrival order.
+__global__ void order_gather_kernel(int64_t N, const OrderPlan *plan,
+                                    const unsigned long long *hi_orig, unsigned long long *keyA,
+                                    unsigned long long *keyB, const uint32_t *valA,
+                                    const uint32_t *valB) {
   const int gb = plan->gather_buf;
   if (gb < 0) return;
+  const bool wide = plan->wide != 0;
   unsigned long long *k = gb == kBufA ? keyA : keyB;
   const uint32_t *v = gb == kBufA ? valA : valB;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < N; i += stride)
-    k[i] = hi_orig[v[i]];
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < N; i += stride) {
+    const unsigned long long x = hi_orig[v[i]];
+    if (wide)
+      k[i] = x;
+    else
+      reinterpret_cast<uint32_t *>(k)[i] = static_cast<uint32_t>(x);
+  }
 }
 
 // No active pass at all: the identity is the order.
@@ -230,22 +325,40 @@ struct PassSmem {
   uint32_t hw[kPassWarps][kRadix];  // per-warp counts, then per-warp bin bases
   uint32_t tile_cnt[kRadix];
   uint32_t bin_start[kRadix];       // tile-local start of each bin
-  uint32_t excl[kRadix];            // global offset of this tile within each bin
+  uint32_t excl[kRadix];            // offset of this tile within each bin
   uint32_t scan_w[kRadix / 32];
+  uint32_t look_flag[256];          // flags of the predecessor window
+  uint32_t look_part[2][kRadix];    // partial window sums
+  int look_inc;                     // nearest window slot with an inclusive prefix
   int tile;
 };
 
-__global__ void __launch_bounds__(kPassThreads)
-order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
-                  unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
-                  const unsigned long long *hi_orig, int32_t *perm, unsigned long long *tstatus,
-                  uint32_t *ticket, int32_t *status) {
-  if (!plan->active[p]) return;
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  PassSmem &sm = *reinterpret_cast<PassSmem *>(smem_raw);
+// Key access for a pass: lo passes read arrival as 32 bits from a 64-bit
+// slot array; narrow hi passes read 32-bit keys; wide ones 64-bit keys.
+template <bool WIDE>
+__device__ __forceinline__ unsigned long long load_key(const unsigned long long *k, int64_t i, bool lo) {
+  if (lo) return k[i];
+  if (WIDE) return k[i];
+  return reinterpret_cast<const uint32_t *>(k)[i];
+}
+template <bool WIDE>
+__device__ __forceinline__ void store_key(unsigned long long *k, int64_t i, unsigned long long v, bool lo) {
+  if (lo || WIDE)
+    k[i] = v;
+  else
+    reinterpret_cast<uint32_t *>(k)[i] = static_cast<uint32_t>(v);
+}
+
+template <bool WIDE>
+__device__ void order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
+                                unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
+                                const unsigned long long *hi_orig, int32_t *perm,
+                                uint32_t *flags, uint32_t *agg, uint32_t *inc, uint32_t *ticket,
+                                int32_t *status, PassSmem &sm) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool lo = p < kLoPasses;
   const int src = plan->src[p], dst = plan->dst[p];
-  const int shift = p < kLoPasses ? 8 * p : 8 * (p - kLoPasses);
+  const int shift = plan->shift[p];
   const bool identity = src == kHiIdentity;
   const unsigned long long *kin = src == kBufA ? keyA : (src == kBufB ? keyB : hi_orig);
   const uint32_t *vin = src == kBufA ? valA : valB;
@@ -259,7 +372,8 @@ order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *k
   const int tile = sm.tile;
   const int64_t base = static_cast<int64_t>(tile) * kTile;
 
-  // load and rank within the warp (stable: warp-major, then item, then lane)
+  // load (all loads first), then rank within the warp (stable: warp-major,
+  // then item, then lane)
   unsigned long long key[kIPT];
   uint32_t val[kIPT];
   int dig[kIPT];
@@ -268,11 +382,18 @@ order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *k
   for (int it = 0; it < kIPT; ++it) {
     const int64_t idx = base + warp * (32 * kIPT) + it * 32 + lane;
     const bool valid = idx < N;
-    key[it] = valid ? kin[idx] : 0ull;
+    // the first hi pass reads the original keys in their own width
+    key[it] = valid ? (identity ? (WIDE ? hi_orig[idx] : static_cast<uint32_t>(hi_orig[idx]))
+                                : load_key<WIDE>(kin, idx, lo))
+                    : 0ull;
     val[it] = valid ? (identity ? static_cast<uint32_t>(idx) : vin[idx]) : 0u;
     dig[it] = valid ? static_cast<int>((key[it] >> shift) & 255u) : kRadix;
+  }
+#pragma unroll
+  for (int it = 0; it < kIPT; ++it) {
     const unsigned peers = __match_any_sync(0xffffffffu, dig[it]);
     const uint32_t before = __popc(peers & lanemask_lt());
+    const bool valid = dig[it] < kRadix;
     uint32_t cur = 0;
     if (valid) cur = sm.hw[warp][dig[it]];
     __syncwarp();
@@ -281,7 +402,9 @@ order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *k
     rank[it] = cur + before;
   }
   __syncthreads();
-  // per bin: exclusive scan over warps, tile total
+  // per bin: exclusive scan over warps, tile total; publish the aggregate
+  uint32_t *my_agg = agg + static_cast<size_t>(tile) * kRadix;
+  uint32_t *my_inc = inc + static_cast<size_t>(tile) * kRadix;
   if (tid < kRadix) {
     uint32_t run = 0;
     for (int w = 0; w < kPassWarps; ++w) {
@@ -290,36 +413,80 @@ order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *k
       run += c;
     }
     sm.tile_cnt[tid] = run;
-    // publish this tile's count, then look back for the offset of the tile
-    unsigned long long *st = tstatus + static_cast<size_t>(tile) * kRadix;
-    if (tile == 0) {
-      st_release_u64(st + tid, kInc | run);
-      sm.excl[tid] = 0;
-    } else {
-      st_release_u64(st + tid, kAgg | run);
-      unsigned long long excl = 0;
-      for (int q = tile - 1; q >= 0; --q) {
-        const unsigned long long *w = tstatus + static_cast<size_t>(q) * kRadix + tid;
-        unsigned long long v;
+    sm.excl[tid] = 0;
+    if (tile == 0)
+      my_inc[tid] = run;
+    else
+      my_agg[tid] = run;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    st_release_u32(flags + tile, tile == 0 ? kFlagInc : kFlagAgg);
+  }
+  // Look back over up to 256 predecessor tiles per round, one thread per
+  // tile: wait until each has published at least its aggregate, find the
+  // nearest one that has published its inclusive prefix, and add up the
+  // aggregates above it (and its inclusive value) bin by bin.
+  for (int top = tile - 1; top >= 0;) {
+    if (tid < kLookWindow) {
+      const int q = top - tid;
+      uint32_t f = kFlagInc;  // "tile -1" is an empty inclusive prefix
+      if (q >= 0) {
         uint32_t spins = 0;
-        while (((v = ld_acquire_u64(w)) >> 62) == 0) {
+        while ((f = ld_acquire_u32(flags + q)) == 0) {
           if (++spins > kSpinLimit) {
             flag_error(status, MAPS_E_TIMEOUT);
-            v = kInc;
+            f = kFlagInc;  // give up: use what is there
             break;
           }
           __nanosleep(32);
         }
-        excl += v & kValMask;
-        if ((v >> 62) == 2) break;
       }
-      st_release_u64(st + tid, kInc | (excl + run));
-      sm.excl[tid] = static_cast<uint32_t>(excl);
+      sm.look_flag[tid] = f;
+    }
+    if (tid == 0) sm.look_inc = -1;
+    __syncthreads();
+    if (tid < kLookWindow && sm.look_flag[tid] == kFlagInc) atomicMin(reinterpret_cast<unsigned *>(&sm.look_inc), static_cast<unsigned>(tid));
+    __syncthreads();
+    // lanes 0 .. depth-1 of the window are added; depth ends at the nearest
+    // inclusive prefix (included), else covers the whole window
+    const int near = sm.look_inc;  // -1 (as unsigned max) when none
+    const int depth = (near >= 0 && near < kLookWindow) ? near + 1 : kLookWindow;
+    {
+      // thread (bin, half) adds every other group of 16 window slots, with
+      // the 16 loads of a group in flight together
+      const int bin = tid & (kRadix - 1), half = tid >> 8;
+      uint32_t add = 0;
+      for (int x0 = half * 16; x0 < depth; x0 += 32) {
+        uint32_t v[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const int x = x0 + u, q = top - x;
+          v[u] = (x < depth && q >= 0)
+                     ? __ldcg((sm.look_flag[x] == kFlagInc ? inc : agg) + static_cast<size_t>(q) * kRadix + bin)
+                     : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < 16; ++u) add += v[u];
+      }
+      sm.look_part[half][bin] = add;
+    }
+    __syncthreads();
+    if (tid < kRadix) sm.excl[tid] += sm.look_part[0][tid] + sm.look_part[1][tid];
+    __syncthreads();
+    if (near >= 0 && near < kLookWindow) break;
+    top -= kLookWindow;
+  }
+  if (tile > 0) {
+    if (tid < kRadix) my_inc[tid] = sm.excl[tid] + sm.tile_cnt[tid];
+    __syncthreads();
+    if (tid == 0) {
+      __threadfence();
+      st_release_u32(flags + tile, kFlagInc);
     }
   }
-  __syncthreads();
-  // tile-local bin starts (exclusive scan of tile counts over 256 bins; the
-  // first 8 warps hold the 256 bins, so every shuffle below has full warps)
+  // tile-local bin starts (the first 8 warps hold the 256 bins)
   uint32_t bc = 0, bincl = 0;
   if (tid < kRadix) {
     bc = sm.tile_cnt[tid];
@@ -354,32 +521,50 @@ order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *k
     const unsigned long long k = sm.keys[s];
     const int d = static_cast<int>((k >> shift) & 255u);
     const uint32_t pos = plan->digit_off[p][d] + sm.excl[d] + (s - sm.bin_start[d]);
-    if (keys_out) kout[pos] = k;
+    if (keys_out) store_key<WIDE>(kout, pos, k, lo);
     vout[pos] = sm.vals[s];
   }
+}
+
+__global__ void __launch_bounds__(kPassThreads)
+order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
+                  unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
+                  const unsigned long long *hi_orig, int32_t *perm, uint32_t *flags,
+                  uint32_t *agg, uint32_t *inc, uint32_t *ticket, int32_t *status) {
+  if (!plan->active[p]) return;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  PassSmem &sm = *reinterpret_cast<PassSmem *>(smem_raw);
+  if (plan->wide)
+    order_pass_body<true>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, flags, agg, inc,
+                          ticket, status, sm);
+  else
+    order_pass_body<false>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, flags, agg, inc,
+                           ticket, status, sm);
 }
 
 struct OrderWs {
   OrderCounts *counts;
   uint32_t *dec_count;
   uint32_t *tickets;
-  unsigned long long *tstatus;
+  uint32_t *flags;  // [kPasses][tiles]
+  size_t zero_bytes;  // counts .. flags are contiguous and zeroed per call
+  uint32_t *agg, *inc;  // [kPasses][tiles][256]
   OrderPlan *plan;
   unsigned long long *hi_orig, *keyA, *keyB;
   uint32_t *valA, *valB;
-  size_t zero_bytes;  // counts .. tstatus are contiguous and zeroed per call
 };
 
 OrderWs carve_order(Carve &c, int64_t N, int D) {
   OrderWs w;
-  const int64_t tiles = (N + kTile - 1) / kTile;
-  const size_t zero_begin = c.off;
+  const int64_t tiles = std::max<int64_t>(1, (N + kTile - 1) / kTile);
+  const size_t zero_begin = (c.off + kAlign - 1) / kAlign * kAlign;
   w.counts = c.take<OrderCounts>(1);
   w.dec_count = c.take<uint32_t>(static_cast<size_t>(D));
   w.tickets = c.take<uint32_t>(kPasses);
-  w.tstatus = c.take<unsigned long long>(static_cast<size_t>(kPasses) * (tiles > 0 ? tiles : 1) * kRadix);
-  const size_t zero_end = c.off;
-  w.zero_bytes = zero_end - ((zero_begin + kAlign - 1) / kAlign * kAlign);
+  w.flags = c.take<uint32_t>(static_cast<size_t>(kPasses) * tiles);
+  w.zero_bytes = c.off - zero_begin;
+  w.agg = c.take<uint32_t>(static_cast<size_t>(kPasses) * tiles * kRadix);
+  w.inc = c.take<uint32_t>(static_cast<size_t>(kPasses) * tiles * kRadix);
   w.plan = c.take<OrderPlan>(1);
   const size_t n = static_cast<size_t>(N > 0 ? N : 1);
   w.hi_orig = c.take<unsigned long long>(n);
@@ -416,33 +601,35 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   Carve cv(ws);
   const OrderWs w = carve_order(cv, N, D);
   MAPS_TRY(cuda_ok(cudaMemsetAsync(w.counts, 0, w.zero_bytes, s)));
-  // key digits that can differ: bits [0, 32 + bits(D - 1))
-  int dbits = 0;
+  int dbits = 0;  // bits of the largest decoder index
   while ((1ll << dbits) < D) ++dbits;
-  const int n_hi = std::min(kHiPasses, (32 + dbits + 7) / 8);
+  // hi passes that can be active: the key has at most dbits + 1 + 31 bits
+  const int n_hi = std::min(kHiPasses, (dbits + 1 + 31 + 7) / 8);
   const int sms = sm_count();
-  const int64_t tiles = (N + kTile - 1) / kTile;
+  const int64_t tiles = std::max<int64_t>(1, (N + kTile - 1) / kTile);
   if (N > 0) {
-    const int gprep = static_cast<int>(std::min<int64_t>((N + 511) / 512, 2LL * sms));
-    order_prep_kernel<<<gprep, 512, 0, s>>>(N, D, n_hi, dec, bound, wait, arrival, max_wait,
-                                            w.hi_orig, w.keyA, w.valA, w.counts, w.dec_count, status);
+    const int g = static_cast<int>(std::min<int64_t>((N + 2047) / 2048, 2LL * sms));
+    order_prep_kernel<<<g, 512, 0, s>>>(N, D, dec, bound, wait, arrival, max_wait, w.counts,
+                                        w.dec_count, status);
+    order_keys_kernel<<<g, 512, 0, s>>>(N, D, dbits, dec, bound, wait, arrival, max_wait, w.counts,
+                                        w.hi_orig, w.keyA, w.valA);
   }
-  order_plan_kernel<<<1, kRadix, 0, s>>>(N, D, n_hi, w.counts, w.plan, w.dec_count, seg_off_out);
+  order_plan_kernel<<<1, kRadix, 0, s>>>(N, D, dbits, w.counts, w.plan, w.dec_count, seg_off_out);
   MAPS_TRY(launch_ok());
   if (N == 0) return MAPS_OK;
   const size_t smem = sizeof(PassSmem);
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_pass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));
   const int gcopy = static_cast<int>(std::min<int64_t>((N + 255) / 256, 4LL * sms));
-  for (int p = 0; p < kLoPasses; ++p)
+  auto pass = [&](int p) {
     order_pass_kernel<<<static_cast<unsigned>(tiles), kPassThreads, smem, s>>>(
         p, N, w.plan, w.keyA, w.keyB, w.valA, w.valB, w.hi_orig, perm_out,
-        w.tstatus + static_cast<size_t>(p) * tiles * kRadix, w.tickets + p, status);
+        w.flags + static_cast<size_t>(p) * tiles, w.agg + static_cast<size_t>(p) * tiles * kRadix,
+        w.inc + static_cast<size_t>(p) * tiles * kRadix, w.tickets + p, status);
+  };
+  for (int p = 0; p < kLoPasses; ++p) pass(p);
   order_gather_kernel<<<gcopy, 256, 0, s>>>(N, w.plan, w.hi_orig, w.keyA, w.keyB, w.valA, w.valB);
-  for (int p = kLoPasses; p < kLoPasses + n_hi; ++p)
-    order_pass_kernel<<<static_cast<unsigned>(tiles), kPassThreads, smem, s>>>(
-        p, N, w.plan, w.keyA, w.keyB, w.valA, w.valB, w.hi_orig, perm_out,
-        w.tstatus + static_cast<size_t>(p) * tiles * kRadix, w.tickets + p, status);
+  for (int p = kLoPasses; p < kLoPasses + n_hi; ++p) pass(p);
   order_identity_kernel<<<gcopy, 256, 0, s>>>(N, w.plan, perm_out);
   return launch_ok();
 }

@@ -54,9 +54,9 @@ def _load():
         "maps_calibrate_workspace_size": ([i64, i64], sz),
         "maps_calibrate": ([vp, vp, i64, u32, vp, i64, vp, vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_project_occupancy_workspace_size": ([i32, i32, i64], sz),
-        "maps_project_occupancy": ([i32, i32, vp, i64, vp, vp, vp, vp, vp, sz, vp], ctypes.c_int),
+        "maps_project_occupancy": ([i32, i32, vp, i64, vp, vp, vp, vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_dispatch_workspace_size": ([i32, i32, i32, i64], sz),
-        "maps_dispatch": ([i32, i32, i32, i32, vp, vp, vp, vp, i64, vp, vp, vp, i64, vp, vp,
+        "maps_dispatch": ([i32, i32, i32, i32, vp, vp, vp, vp, vp, i64, vp, vp, vp, i64, vp, vp,
                            vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_order_local_workspace_size": ([i64, i32], sz),
         "maps_order_local": ([i64, i32, vp, vp, vp, vp, i32, vp, vp, vp, sz, vp], ctypes.c_int),
@@ -135,7 +135,12 @@ def maps_calibrate(true_len, pred_len, alpha_ppm: int, query_pred=None, bound_ou
     return st, (int(qh.value) if q_host else None)
 
 
-def maps_project_occupancy(D: int, H: int, res_off, prompt, gen, bound, K_out,
+def kmax_shape(D: int, H: int) -> tuple[int, int]:
+    """Shape of the 16-step summary of K (uint32 values, stored as int32)."""
+    return D, (H + 15) // 16
+
+
+def maps_project_occupancy(D: int, H: int, res_off, prompt, gen, bound, K_out, kmax_out=None,
                            ws: Workspace | None = None, stream=None) -> int:
     R = prompt.numel()
     ws = ws or Workspace()
@@ -143,17 +148,19 @@ def maps_project_occupancy(D: int, H: int, res_off, prompt, gen, bound, K_out,
     return lib.maps_project_occupancy(D, H, _ptr(res_off, torch.int64), R,
                                       _ptr(prompt, torch.int32), _ptr(gen, torch.int32),
                                       _ptr(bound, torch.int32), _ptr(K_out, torch.int32),
-                                      ws.ptr, ws.nbytes, _stream(stream))
+                                      _ptr(kmax_out, torch.int32), ws.ptr, ws.nbytes,
+                                      _stream(stream))
 
 
 def maps_dispatch(mode: int, D: int, H: int, S: int, K, cap, Q, cand_prompt, cand_bound,
                   choice_out, headroom_out=None, res_off=None, prompt=None, gen=None,
-                  bound=None, ws: Workspace | None = None, stream=None) -> int:
+                  bound=None, kmax=None, ws: Workspace | None = None, stream=None) -> int:
     J = cand_prompt.numel()
     R = 0 if prompt is None else prompt.numel()
     ws = ws or Workspace()
     ws.ensure(lib.maps_dispatch_workspace_size(mode, D, H, J))
-    return lib.maps_dispatch(mode, D, H, S, _ptr(K, torch.int32), _ptr(cap, torch.int32),
+    return lib.maps_dispatch(mode, D, H, S, _ptr(K, torch.int32), _ptr(kmax, torch.int32),
+                             _ptr(cap, torch.int32),
                              _ptr(Q, torch.int32), _ptr(res_off, torch.int64), R,
                              _ptr(prompt, torch.int32), _ptr(gen, torch.int32),
                              _ptr(bound, torch.int32), J, _ptr(cand_prompt, torch.int32),

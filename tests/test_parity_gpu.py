@@ -53,17 +53,31 @@ def gpu_calibrate(M, ws, L, P, a, query=None):
     return st, q, int(host(qd)[0]), host(U[:m])
 
 
-def gpu_occupancy(M, ws, D, H, off, p, g, u):
+def gpu_occupancy(M, ws, D, H, off, p, g, u, with_kmax=False):
     K = torch.full((D, H), -7, dtype=torch.int32, device="cuda")
+    km = torch.full(M.kmax_shape(D, H), -7, dtype=torch.int32, device="cuda") if with_kmax else None
     st = M.maps_project_occupancy(D, H, dev(off, np.int64), dev(p, np.int32), dev(g, np.int32),
-                                  dev(u, np.int32), K, ws=ws)
+                                  dev(u, np.int32), K, km, ws=ws)
     assert st == 0
+    if with_kmax:
+        return M.maps_check(ws), host(K), host(km).view(np.uint32)
     return M.maps_check(ws), host(K)
 
 
-def gpu_dispatch(M, ws, mode, D, H, S, K, cap, Q, cp, cb, res=None):
+def kmax_of(K):
+    """16-step block maxima of K + t (the summary's definition, in numpy)."""
+    D, H = K.shape
+    x = K.astype(np.int64) + np.arange(H)
+    nb = (H + 15) // 16
+    pad = np.full((D, nb * 16), -1, np.int64)
+    pad[:, :H] = x
+    return pad.reshape(D, nb, 16).max(axis=2).astype(np.uint32)
+
+
+def gpu_dispatch(M, ws, mode, D, H, S, K, cap, Q, cp, cb, res=None, kmax=None):
     J = len(cp)
     Kd = None if K is None else dev(K, np.int32)
+    kmd = None if kmax is None else dev(np.ascontiguousarray(kmax).view(np.int32))
     Qd = dev(Q, np.int32)
     ch = torch.full((max(J, 1),), -9, dtype=torch.int32, device="cuda")
     hr = torch.full((max(J, 1),), -9, dtype=torch.int64, device="cuda")
@@ -72,7 +86,7 @@ def gpu_dispatch(M, ws, mode, D, H, S, K, cap, Q, cp, cb, res=None):
         kw = dict(res_off=dev(res[0], np.int64), prompt=dev(res[1], np.int32),
                   gen=dev(res[2], np.int32), bound=dev(res[3], np.int32))
     st = M.maps_dispatch(mode, D, H, S, Kd, dev(cap, np.int32), Qd, dev(cp, np.int32),
-                         dev(cb, np.int32), ch[:J], hr[:J], ws=ws, **kw)
+                         dev(cb, np.int32), ch[:J], hr[:J], kmax=kmd, ws=ws, **kw)
     assert st == 0, st
     st = M.maps_check(ws)
     return st, host(ch[:J]), host(hr[:J]), (None if Kd is None else host(Kd)), host(Qd)
@@ -206,9 +220,10 @@ def test_occupancy_random(M, ws, oracle, D, H):
     rng = np.random.default_rng(D * 100003 + H)
     off, p, g, U = random_residents(rng, D, H, 700)
     sto, Ko = oracle.occupancy(D, H, off, p, g, U)
-    st, K = gpu_occupancy(M, ws, D, H, off, p, g, U)
+    st, K, km = gpu_occupancy(M, ws, D, H, off, p, g, U, with_kmax=True)
     assert st == sto == 0
     assert np.array_equal(K, Ko)
+    assert np.array_equal(km, kmax_of(Ko))
 
 
 @pytest.mark.parametrize("name", ["tiny", "d16", "d64", "large"])
@@ -217,9 +232,11 @@ def test_occupancy_workloads(M, ws, oracle, name):
     q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
     U = oracle.bound(w["res_pred"], q)[1]
     sto, Ko = oracle.occupancy(w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U)
-    st, K = gpu_occupancy(M, ws, w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U)
+    st, K, km = gpu_occupancy(M, ws, w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"],
+                              U, with_kmax=True)
     assert st == sto == 0
     assert np.array_equal(K, Ko)
+    assert np.array_equal(km, kmax_of(Ko))
 
 
 def test_occupancy_errors(M, ws, oracle):
@@ -256,14 +273,16 @@ def diverse_caps(rng, K, spread):
 def check_dispatch(M, ws, oracle, mode, D, H, K, cap, Q, cp, cb, S=1, res=None):
     sto, co, ho, Ko, Qo = oracle.dispatch(mode, D, H, S, K, cap, Q, cp, cb,
                                           *(res if res is not None else ()))
-    st, ch, hr, Ka, Qa = gpu_dispatch(M, ws, mode, D, H, S, K, cap, Q, cp, cb, res)
-    assert st == sto
-    if st == 0:
-        assert np.array_equal(ch, co)
-        assert np.array_equal(hr, ho)
-        if mode == 1:
-            assert np.array_equal(Ka, Ko)
-        assert np.array_equal(Qa, Qo)
+    runs = [None, kmax_of(np.asarray(K))] if mode == 0 else [None]
+    for km in runs:  # SNAPSHOT: summary derived inside, and passed in
+        st, ch, hr, Ka, Qa = gpu_dispatch(M, ws, mode, D, H, S, K, cap, Q, cp, cb, res, km)
+        assert st == sto
+        if st == 0:
+            assert np.array_equal(ch, co)
+            assert np.array_equal(hr, ho)
+            if mode == 1:
+                assert np.array_equal(Ka, Ko)
+            assert np.array_equal(Qa, Qo)
     return co, ho
 
 
@@ -319,9 +338,12 @@ def test_dispatch_snapshot_large_sampled(M, ws, oracle, variant):
     if variant == "diverse":
         cap = diverse_caps(rng, K, 6000)
         Q = rng.integers(0, 3, D).astype(np.int32)
-    st, ch, hr, _, _ = gpu_dispatch(M, ws, 0, D, H, 1, K, cap, Q, w["cand_prompt"], cb)
+    st, ch, hr, _, _ = gpu_dispatch(M, ws, 0, D, H, 1, K, cap, Q, w["cand_prompt"], cb,
+                                    kmax=kmax_of(K))
     assert st == 0
     assert ch.min() >= 0 and ch.max() < D
+    st2, ch2, hr2, _, _ = gpu_dispatch(M, ws, 0, D, H, 1, K, cap, Q, w["cand_prompt"], cb)
+    assert st2 == 0 and np.array_equal(ch, ch2) and np.array_equal(hr, hr2)
     idx = np.concatenate([np.argsort(cb)[-64:], rng.choice(J, 1500, replace=False)])
     sto, co, ho, _, _ = oracle.dispatch(0, D, H, 1, K, cap, Q, w["cand_prompt"][idx], cb[idx])
     assert sto == 0
@@ -386,7 +408,7 @@ def test_dispatch_errors(M, ws, oracle):
     assert M.maps_dispatch(0, 1025, 8, 1, Kd, z, z, dev([1], np.int32), dev([1], np.int32), ch,
                            ws=ws) == M.MAPS_E_INVALID
     small = M.Workspace(256)
-    assert M.lib.maps_dispatch(0, 2, 8, 1, M._ptr(Kd), M._ptr(z), M._ptr(z), None, 0, None, None,
+    assert M.lib.maps_dispatch(0, 2, 8, 1, M._ptr(Kd), None, M._ptr(z), M._ptr(z), None, 0, None, None,
                                None, 1, M._ptr(dev([1], np.int32)), M._ptr(dev([1], np.int32)),
                                M._ptr(ch), None, small.ptr, 256, M._stream(None)) == M.MAPS_E_WORKSPACE
 
