@@ -209,6 +209,39 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec,
                      int32_t *perm_out, int64_t *seg_off_out, void *ws,
                      size_t ws_bytes, void *stream);
 
+/* ------------------------------------------------------------------------
+ * maps_order_local without any allocation.  The paper has no counterpart:
+ * this is a deployment aid.
+ *
+ * Some callers cannot call cudaMalloc at all -- for instance a scheduler
+ * embedded in a host process whose device allocator belongs to another
+ * framework, or one that must not allocate once it is serving.  This call
+ * computes exactly what maps_order_local computes, but its scratch memory is
+ * a fixed array of 3 MiB compiled into the library (every GPU that loads the
+ * library holds it until the process exits), so it takes no workspace and
+ * allocates nothing.  The caller still provides inputs and outputs, in
+ * device memory, as for maps_order_local.
+ *
+ *   Limits              N <= 65,536 entries and D <= 4,096 decoders; larger
+ *                       sizes return MAPS_E_WORKSPACE at once.
+ *   status_host         optional host int32 (NULL: not written).  Non-NULL
+ *                       synchronises the stream and returns the full status,
+ *                       data-dependent errors included; with NULL, data errors
+ *                       are not reported.
+ *   First call          the first call on each device looks up the array's
+ *                       device address; make that call before any stream
+ *                       capture.
+ *   Concurrency         every call shares the one array: calls whose work
+ *                       overlaps on the GPU (other streams, other threads)
+ *                       race and give wrong results.  Order them on one
+ *                       stream.
+ * ---------------------------------------------------------------------- */
+int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
+                            const int32_t *bound, const int32_t *wait,
+                            const int32_t *arrival, int32_t max_wait,
+                            int32_t *perm_out, int64_t *seg_off_out,
+                            int32_t *status_host, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

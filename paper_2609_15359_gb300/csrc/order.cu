@@ -22,6 +22,7 @@
 #include "maps_internal.cuh"
 
 #include <algorithm>
+#include <mutex>
 
 namespace maps {
 namespace {
@@ -635,3 +636,70 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of maps_order_local.
+//
+// For callers that cannot allocate device memory at all -- code running
+// where cudaMalloc is unavailable or forbidden, such as a scheduler embedded
+// in a host process whose allocator is owned by someone else, or one that
+// must never allocate after start-up -- the scratch lives in this file-scope
+// device array instead of a caller workspace.  Every GPU that loads the
+// library holds it until the process exits.
+// ---------------------------------------------------------------------------
+namespace maps {
+namespace {
+
+constexpr int64_t kStaticMaxN = 65536;  // entries
+constexpr int32_t kStaticMaxD = 4096;   // decoders
+constexpr size_t kStaticBytes = size_t(3) << 20;
+static __device__ __align__(256) unsigned char g_order_scratch[kStaticBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mu;
+void *g_static_ptr[kMaxDevices] = {};
+
+// Device address of the static scratch on the current device, looked up once
+// per device (the host-side symbol is not a device address).
+int static_scratch(void **out) {
+  int dev = 0;
+  MAPS_TRY(cuda_ok(cudaGetDevice(&dev)));
+  if (dev < 0 || dev >= kMaxDevices) return MAPS_E_INVALID;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (g_static_ptr[dev] == nullptr) {
+    void *p = nullptr;
+    MAPS_TRY(cuda_ok(cudaGetSymbolAddress(&p, g_order_scratch)));
+    if (p == nullptr || !aligned(p, kAlign)) return MAPS_E_CUDA;
+    g_static_ptr[dev] = p;
+  }
+  *out = g_static_ptr[dev];
+  return MAPS_OK;
+}
+
+}  // namespace
+}  // namespace maps
+
+extern "C" int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
+                                       const int32_t *bound, const int32_t *wait,
+                                       const int32_t *arrival, int32_t max_wait,
+                                       int32_t *perm_out, int64_t *seg_off_out,
+                                       int32_t *status_host, void *stream) {
+  using namespace maps;
+  if (N < 0 || D < 1) return MAPS_E_INVALID;
+  if (N > kStaticMaxN || D > kStaticMaxD) return MAPS_E_WORKSPACE;
+  const size_t need = maps_order_local_workspace_size(N, D);
+  if (need > kStaticBytes) return MAPS_E_WORKSPACE;
+  void *ws = nullptr;
+  MAPS_TRY(static_scratch(&ws));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the array keeps the previous call's contents: start this call's status
+  // at zero (the order itself zeroes every counter it needs)
+  MAPS_TRY(cuda_ok(cudaMemsetAsync(ws, 0, kCtrlBytes, s)));
+  MAPS_TRY(maps_order_local(N, D, dec, bound, wait, arrival, max_wait, perm_out, seg_off_out, ws,
+                            kStaticBytes, stream));
+  if (status_host != nullptr) {
+    *status_host = maps_check(ws, stream);
+    return *status_host;
+  }
+  return MAPS_OK;
+}

@@ -60,6 +60,7 @@ def _load():
                            vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_order_local_workspace_size": ([i64, i32], sz),
         "maps_order_local": ([i64, i32, vp, vp, vp, vp, i32, vp, vp, vp, sz, vp], ctypes.c_int),
+        "maps_order_local_static": ([i64, i32, vp, vp, vp, vp, i32, vp, vp, vp, vp], ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -73,7 +74,7 @@ EXPORTS = ("maps_version", "maps_last_cuda_error", "maps_check",
            "maps_calibrate_workspace_size", "maps_calibrate",
            "maps_project_occupancy_workspace_size", "maps_project_occupancy",
            "maps_dispatch_workspace_size", "maps_dispatch",
-           "maps_order_local_workspace_size", "maps_order_local")
+           "maps_order_local_workspace_size", "maps_order_local", "maps_order_local_static")
 
 
 def _stream(stream) -> ctypes.c_void_p:
@@ -179,3 +180,17 @@ def maps_order_local(D: int, dec, bound, wait, arrival, max_wait: int, perm_out,
                                 int(max_wait), _ptr(perm_out, torch.int32),
                                 _ptr(seg_off_out, torch.int64), ws.ptr, ws.nbytes,
                                 _stream(stream))
+
+
+def maps_order_local_static(D: int, dec, bound, wait, arrival, max_wait: int, perm_out,
+                            seg_off_out, sync_status: bool = True, stream=None) -> int:
+    """maps_order_local with the library's fixed scratch array: no workspace,
+    no allocation.  N <= 65,536 and D <= 4,096."""
+    N = dec.numel()
+    st = ctypes.c_int32(0)
+    return lib.maps_order_local_static(N, D, _ptr(dec, torch.int32), _ptr(bound, torch.int32),
+                                       _ptr(wait, torch.int32), _ptr(arrival, torch.int32),
+                                       int(max_wait), _ptr(perm_out, torch.int32),
+                                       _ptr(seg_off_out, torch.int64),
+                                       ctypes.byref(st) if sync_status else None,
+                                       _stream(stream))
