@@ -239,6 +239,22 @@ def test_occupancy_workloads(M, ws, oracle, name):
     assert np.array_equal(km, kmax_of(Ko))
 
 
+@pytest.mark.parametrize("D,H,per", [(2, 20000, 9000), (3, 3000, 4097)])
+def test_occupancy_many_residents_per_decoder(M, ws, oracle, D, H, per):
+    """More residents on one decoder than a block stages at once."""
+    rng = np.random.default_rng(H + per)
+    off = np.arange(D + 1, dtype=np.int64) * per
+    R = D * per
+    p = rng.integers(0, 300, R).astype(np.int32)
+    g = rng.integers(0, H, R).astype(np.int32)
+    U = rng.integers(0, 2 * H, R).astype(np.int32)
+    sto, Ko = oracle.occupancy(D, H, off, p, g, U)
+    st, K, km = gpu_occupancy(M, ws, D, H, off, p, g, U, with_kmax=True)
+    assert st == sto == 0
+    assert np.array_equal(K, Ko)
+    assert np.array_equal(km, kmax_of(Ko))
+
+
 def test_occupancy_errors(M, ws, oracle):
     # K above INT32_MAX
     big = I32_MAX // 2
