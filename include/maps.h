@@ -107,7 +107,8 @@ int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
  * is kept for one step), so
  *     K[k][t] = sum over residents r of k with t < e_r of (p + g + 1 + t).
  *
- *   D, H                decoders (>= 1) and horizon steps (>= 1).
+ *   D, H                decoders (>= 1) and horizon steps (1 <= H <= 2^28;
+ *                       a larger H is MAPS_E_INVALID).
  *   res_off             [D+1] int64 CSR offsets into the resident arrays,
  *                       non-decreasing within [0, R].
  *   R                   length of prompt / gen / bound.

@@ -5,23 +5,28 @@
 //   K[k][t] = SumB_k(t) + t * Cnt_k(t)
 // with Cnt / SumB the count and b-sum of residents still live at t.
 //
-// Layout of the work.  One CTA owns one decoder and a chunk of up to four
-// horizon tiles of W steps.  It loads the decoder's residents once, keeps
-// each resident's footprint at t = 0 (b) and end step (e) in shared memory,
-// and walks its tiles from the highest down.  For a tile, residents ending
-// inside it go into a shared-memory end-step histogram; those ending after
-// it form the tile's carry (count, b-sum), which is the previous tile's carry
-// plus the previous tile's bin totals.  A reverse scan of the histogram
-// gives each cell's live count and b-sum, and the tile is written with
-// 128-bit stores.  Chunks of the same decoder re-read the residents from L2.
-// Optionally every group of 16 steps also yields
-// kmax[k][t/16] = max (K[k][t] + t), a summary the dispatch uses for the
-// prefix maxima of earlier horizon tiles.
+// Layout of the work.  A decoder's horizon is cut into tiles of W steps.
+//   1. bucket kernel, one CTA per decoder: reads the decoder's residents
+//      once, forms (b, e) and counting-sorts the pairs by the tile that holds
+//      their last live step, into the workspace, with per-tile offsets.  It
+//      also checks the inputs and that K[k][0] = sum of b fits int32.
+//   2. tile kernel, one CTA per (decoder, tile): reads the pairs of its own
+//      tile and of the later tiles (contiguous after the sort).  Its own go
+//      into a shared-memory end-step histogram; the later ones only add to the
+//      tile's carry (count, b-sum), the residents live past the tile.  A
+//      reverse scan of the histogram plus the carry gives every cell's live
+//      count and b-sum, and the tile is written with 128-bit stores.
+// For horizons of more than kMaxTiles tiles a single-kernel form is used
+// instead, in which every tile CTA streams all of its decoder's residents.
+// Optionally every group of 16 steps also yields kmax[k][t/16] =
+// max (K[k][t] + t), a summary the dispatch uses for the prefix maxima of
+// earlier horizon tiles.
 //
 // Integer range: every resident is live at t = 0, so K[k][0] = sum of b_r
 // and every partial sum is at most K[k][0]; if that total exceeds INT32_MAX
 // the call reports MAPS_E_RANGE, otherwise the 32-bit shared-memory sums
-// cannot wrap and each cell is formed exactly in 64 bits.
+// cannot wrap.  A thread forms its cells in 32 bits when a bound over its
+// cells shows that none exceeds INT32_MAX, and exactly in 64 bits otherwise.
 #include "maps_internal.cuh"
 
 namespace maps {
@@ -29,306 +34,466 @@ namespace {
 
 constexpr int kOccThreads = 512;
 constexpr int kWarps = kOccThreads / 32;
-constexpr int kTilesPerChunk = 2;
-constexpr int kBlock = 16;    // steps per kmax summary entry
-constexpr int kStage = 4096;  // residents staged in shared memory at a time
+constexpr int kBlock = 16;     // steps per kmax summary entry
+constexpr int kPerThread = 4;  // entries a thread loads per round
+constexpr int kRound = kPerThread * kOccThreads;
+constexpr int kMaxTiles = 64;  // tiles per decoder of the bucketed form
 
-template <int CPT, bool VEC>
-__global__ void __launch_bounds__(kOccThreads, 2)
-occupancy_kernel(int D, int H, int TPC, int G, const int64_t *__restrict__ res_off, int64_t R,
-                 const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
-                 const int32_t *__restrict__ bound, int32_t *__restrict__ K,
-                 uint32_t *__restrict__ kmax, int32_t *status) {
-  constexpr int W = kOccThreads * CPT;
-  // Bins are padded by 4 words after every CPT bins so that the threads'
-  // 16-byte reads of their own CPT bins fall on distinct banks.
-  constexpr int kPad = CPT == 4 ? 0 : 4;
-  constexpr int WP = W + (W / CPT) * kPad;
-  __shared__ __align__(16) int32_t s_cnt[WP];  // bin j: residents whose last live step is t0 + j
-  __shared__ __align__(16) int32_t s_sb[WP];   // ... and the sum of their b
-  __shared__ int2 s_res[kStage];              // residents ending inside the chunk: (b, e)
-  __shared__ int s_nin;                       // entries in s_res
-  __shared__ long long s_red[3][kWarps];
-  __shared__ uint32_t s_wsum[2][kWarps];      // per-warp bin totals, then exclusive suffixes
-  __shared__ long long s_carry[2][2];         // [tile parity][count, b-sum]
+// Shared-memory state of one tile.  Bins are padded by 4 words after every
+// CPT bins so that the threads' 16-byte reads of their own CPT bins fall on
+// distinct banks.
+template <int CPT>
+struct TileSmem {
+  static constexpr int W = kOccThreads * CPT;
+  static constexpr int kPad = CPT == 4 ? 0 : 4;
+  static constexpr int WP = W + (W / CPT) * kPad;
+  int32_t cnt[WP];  // bin j: residents whose last live step is t0 + j
+  int32_t sb[WP];   // ... and the sum of their b
+  uint32_t part[2][kWarps];  // per-warp carry partials (count, b-sum)
+  uint32_t wsum[2][kWarps];
+  uint32_t carry[2];
+};
 
-  const int k = blockIdx.x / G, chunk = blockIdx.x - (blockIdx.x / G) * G;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t tile_lo = static_cast<int64_t>(chunk) * TPC;
-  const int64_t tiles_all = (static_cast<int64_t>(H) + W - 1) / W;
-  const int ntile = static_cast<int>(min(static_cast<int64_t>(TPC), tiles_all - tile_lo));
-  const int64_t chunk_start = tile_lo * W;             // first step of this chunk
-  const int64_t chunk_end = (tile_lo + ntile) * W;     // first step after it
-
-  int64_t lo = res_off[k], hi = res_off[k + 1];
-  if (lo < 0 || hi < lo || hi > R) {
-    if (tid == 0 && chunk == 0) flag_error(status, MAPS_E_RANGE);
-    lo = hi = 0;
+template <int CPT>
+__device__ __forceinline__ void zero_bins(TileSmem<CPT> &sm) {
+  for (int i = threadIdx.x * 4; i < TileSmem<CPT>::WP; i += kOccThreads * 4) {
+    *reinterpret_cast<int4 *>(&sm.cnt[i]) = make_int4(0, 0, 0, 0);
+    *reinterpret_cast<int4 *>(&sm.sb[i]) = make_int4(0, 0, 0, 0);
   }
-  const int64_t nres = hi - lo;
-  bool bad = false;
-  long long carry_c = 0, carry_s = 0, total_b = 0;
+}
 
-  // Read residents [b0, b0 + n): the ones ending inside the chunk are
-  // appended to s_res (warp-aggregated), the ones live past it only add to
-  // the chunk's carry; all loads of a thread are issued before use.
-  constexpr int kPer = kStage / kOccThreads;
-  auto gather = [&](int64_t b0, int n, bool count) {
-    int32_t p[kPer], gg[kPer], U[kPer];
+template <int CPT>
+__device__ __forceinline__ void add_to_bin(TileSmem<CPT> &sm, int jj, int32_t b) {
+  const int jp = jj + (jj / CPT) * TileSmem<CPT>::kPad;
+  atomicAdd(&sm.cnt[jp], 1);
+  atomicAdd(&sm.sb[jp], b);  // exact while sum b fits int32
+}
+
+// Writes tile [t0, t0 + W) of row k from the histogram and the per-warp
+// carry partials.  Entry: bins complete, part[][warp] written by every warp,
+// and a block barrier since.  The carry partials are 32-bit: they only wrap
+// when sum b exceeds INT32_MAX, which is reported as MAPS_E_RANGE.
+template <int CPT, bool VEC>
+__device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t0, int32_t *K,
+                                          uint32_t *kmax, int32_t *status) {
+  constexpr int kPad = TileSmem<CPT>::kPad;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // Thread tid owns cells l = tid*CPT + c and the bins with the same index;
+  // cell l needs every bin j >= l: its own bins from l up plus all bins of
+  // the threads above it.
+  const int32_t *cb = &sm.cnt[tid * (CPT + kPad)], *sb = &sm.sb[tid * (CPT + kPad)];
+  uint32_t tot_c = 0, tot_s = 0;
 #pragma unroll
-    for (int j = 0; j < kPer; ++j) {
-      const int i = j * kOccThreads + tid;
-      const int64_t r = lo + b0 + i;
-      const bool ok = i < n;
-      p[j] = ok ? __ldg(prompt + r) : 0;
-      gg[j] = ok ? __ldg(gen + r) : 0;
-      U[j] = ok ? __ldg(bound + r) : 0;
+  for (int c = 0; c < CPT; c += 4) {
+    const int4 x = *reinterpret_cast<const int4 *>(cb + c);
+    const int4 y = *reinterpret_cast<const int4 *>(sb + c);
+    tot_c += static_cast<uint32_t>(x.x + x.y + x.z + x.w);
+    tot_s += static_cast<uint32_t>(y.x + y.y + y.z + y.w);
+  }
+  uint32_t suf_c = tot_c, suf_s = tot_s;  // inclusive suffix within the warp
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t yc = __shfl_down_sync(0xffffffffu, suf_c, off);
+    const uint32_t ys = __shfl_down_sync(0xffffffffu, suf_s, off);
+    if (lane + off < 32) {
+      suf_c += yc;
+      suf_s += ys;
     }
+  }
+  if (lane == 0) {
+    sm.wsum[0][warp] = suf_c;
+    sm.wsum[1][warp] = suf_s;
+  }
+  __syncthreads();
+  if (warp == 0) {  // exclusive suffix over the warps' totals; the carry
+    uint32_t wc = lane < kWarps ? sm.wsum[0][lane] : 0u;
+    uint32_t ws = lane < kWarps ? sm.wsum[1][lane] : 0u;
+    const uint32_t oc = wc, os = ws;
 #pragma unroll
-    for (int j = 0; j < kPer; ++j) {
-      const int i = j * kOccThreads + tid;
-      bool keep = false;
-      int2 v = make_int2(0, 0);
-      if (i < n) {
-        if ((p[j] | gg[j] | U[j]) < 0) {
-          bad = true;
-        } else {
-          const long long b = static_cast<long long>(p[j]) + gg[j] + 1;
-          long long e = static_cast<long long>(U[j]) - gg[j];
-          e = e < 1 ? 1 : (e > H ? H : e);
-          if (b > 0x7fffffffLL) bad = true;  // K[k][0] = sum of b overflows
-          const int32_t b32 = static_cast<int32_t>(b > 0x7fffffffLL ? 0x7fffffffLL : b);
-          if (count) {
-            total_b += b32;
-            if (e > chunk_end) {
-              carry_c += 1;
-              carry_s += b32;
-            }
-          }
-          keep = e > chunk_start && e <= chunk_end;
-          v = make_int2(b32, static_cast<int32_t>(e));
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t yc = __shfl_down_sync(0xffffffffu, wc, off);
+      const uint32_t ys = __shfl_down_sync(0xffffffffu, ws, off);
+      if (lane + off < 32) {
+        wc += yc;
+        ws += ys;
+      }
+    }
+    uint32_t cc = lane < kWarps ? sm.part[0][lane] : 0u;
+    uint32_t cs = lane < kWarps ? sm.part[1][lane] : 0u;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      cc += __shfl_xor_sync(0xffffffffu, cc, off);
+      cs += __shfl_xor_sync(0xffffffffu, cs, off);
+    }
+    __syncwarp();
+    if (lane < kWarps) {
+      sm.wsum[0][lane] = wc - oc;
+      sm.wsum[1][lane] = ws - os;
+    }
+    if (lane == 0) {
+      sm.carry[0] = cc;
+      sm.carry[1] = cs;
+    }
+  }
+  __syncthreads();
+
+  // All partial sums are below K[k][0] <= INT32_MAX unless a range error is
+  // flagged, so they are kept in 32 bits.
+  const uint32_t c_lo = sm.carry[0] + sm.wsum[0][warp] + (suf_c - tot_c);
+  const uint32_t s_lo = sm.carry[1] + sm.wsum[1][warp] + (suf_s - tot_s);
+  const int cell0 = t0 + tid * CPT;
+  const uint32_t tc0 = static_cast<uint32_t>(cell0);
+  uint32_t bmax = 0;  // max of K + t over this thread's valid cells
+  if (cell0 < H) {
+    // Both running sums only grow towards the thread's first cell, so their
+    // totals and the last cell's step bound every cell of the thread.
+    const unsigned long long bound64 =
+        static_cast<unsigned long long>(tc0 + CPT - 1) * (c_lo + tot_c) + (s_lo + tot_s);
+    int32_t *row = K + static_cast<int64_t>(k) * H;
+    uint32_t run_c = c_lo, run_s = s_lo;
+    if (VEC && bound64 <= 0x7fffffffull && cell0 + CPT <= H) {
+      // every cell valid and exact in 32 bits
+#pragma unroll
+      for (int c0 = CPT - 4; c0 >= 0; c0 -= 4) {
+        const int4 x = *reinterpret_cast<const int4 *>(cb + c0);
+        const int4 y = *reinterpret_cast<const int4 *>(sb + c0);
+        const uint32_t t = tc0 + c0;
+        uint32_t o3, o2, o1, o0;
+        run_c += static_cast<uint32_t>(x.w);
+        run_s += static_cast<uint32_t>(y.w);
+        o3 = (t + 3) * run_c + run_s;
+        run_c += static_cast<uint32_t>(x.z);
+        run_s += static_cast<uint32_t>(y.z);
+        o2 = (t + 2) * run_c + run_s;
+        run_c += static_cast<uint32_t>(x.y);
+        run_s += static_cast<uint32_t>(y.y);
+        o1 = (t + 1) * run_c + run_s;
+        run_c += static_cast<uint32_t>(x.x);
+        run_s += static_cast<uint32_t>(y.x);
+        o0 = t * run_c + run_s;
+        bmax = max(bmax, max(max(o0 + t, o1 + t + 1), max(o2 + t + 2, o3 + t + 3)));
+        *reinterpret_cast<int4 *>(row + cell0 + c0) = make_int4(o0, o1, o2, o3);
+      }
+    } else {
+      bool over = false;
+#pragma unroll
+      for (int c = CPT - 1; c >= 0; --c) {
+        run_c += static_cast<uint32_t>(cb[c]);
+        run_s += static_cast<uint32_t>(sb[c]);
+        if (cell0 + c < H) {
+          const uint32_t t = tc0 + c;
+          const unsigned long long v = static_cast<unsigned long long>(t) * run_c + run_s;
+          over |= (v >> 31) != 0;
+          const uint32_t o = static_cast<uint32_t>(v);
+          bmax = max(bmax, o + t);
+          row[cell0 + c] = static_cast<int32_t>(o);
         }
       }
-      const unsigned m = __ballot_sync(0xffffffffu, keep);
-      int base = 0;
-      if (lane == 0 && m) base = atomicAdd(&s_nin, __popc(m));
-      base = __shfl_sync(0xffffffffu, base, 0);
-      if (keep) s_res[base + __popc(m & ((1u << lane) - 1u))] = v;
+      if (over) flag_error(status, MAPS_E_RANGE);
     }
-  };
+  }
+  if (kmax != nullptr) {
+    constexpr int L = kBlock / CPT > 0 ? kBlock / CPT : 1;  // lanes per 16-step block
+#pragma unroll
+    for (int off = L / 2; off > 0; off >>= 1) bmax = max(bmax, __shfl_xor_sync(0xffffffffu, bmax, off));
+    if ((lane % L) == 0 && cell0 < H) {
+      const int64_t nb = (static_cast<int64_t>(H) + kBlock - 1) / kBlock;
+      kmax[static_cast<int64_t>(k) * nb + cell0 / kBlock] = bmax;
+    }
+  }
+}
 
-  // 1. Carry into the chunk's highest tile, the decoder's sum of b, and (when
-  //    they fit) the chunk's own residents staged once for all its tiles.
-  const bool staged_once = nres <= kStage;
-  if (tid == 0) s_nin = 0;
+// Resident terms: false for a negative length (a range error).
+__device__ __forceinline__ bool resident_terms(int32_t p, int32_t g, int32_t U, int H,
+                                               int32_t &b32, int32_t &e, bool &big) {
+  if ((p | g | U) < 0) return false;
+  const long long b = static_cast<long long>(p) + g + 1;
+  big = b > 0x7fffffffLL;  // alone already above the K[k][0] limit
+  b32 = static_cast<int32_t>(big ? 0x7fffffffLL : b);
+  e = U - g;  // both non-negative: no wrap
+  e = e < 1 ? 1 : (e > H ? H : e);
+  return true;
+}
+
+__device__ __forceinline__ long long block_sum_ll(long long v, long long *s_red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  if (lane == 0) s_red[warp] = v;
   __syncthreads();
-  for (int64_t b0 = 0; b0 < nres; b0 += kStage) {
-    const int n = static_cast<int>(min(static_cast<int64_t>(kStage), nres - b0));
-    gather(b0, n, true);
-    if (!staged_once) {
-      __syncthreads();
-      if (tid == 0) s_nin = 0;  // batches are re-read per tile below
-      __syncthreads();
+  long long t = 0;
+  for (int w = 0; w < kWarps; ++w) t += s_red[w];
+  return t;
+}
+
+// ---------------------------------------------------------------------------
+// 1. Bucket kernel: one CTA per decoder.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kOccThreads)
+occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, int64_t R,
+                  const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
+                  const int32_t *__restrict__ bound, int2 *__restrict__ bucket,
+                  int32_t *__restrict__ tile_off, int32_t *status) {
+  __shared__ int s_cnt[kMaxTiles];
+  __shared__ int s_cur[kMaxTiles];
+  __shared__ long long s_red[kWarps];
+  const int k = blockIdx.x, tid = threadIdx.x, lane = tid & 31;
+  int64_t lo = res_off[k], hi = res_off[k + 1];
+  if (lo < 0 || hi < lo || hi > R || hi - lo > 0x7fffffffLL) {
+    if (tid == 0) flag_error(status, MAPS_E_RANGE);
+    lo = hi = 0;
+  }
+  const int n = static_cast<int>(hi - lo);
+  const int32_t *pp = prompt + lo, *pg = gen + lo, *pu = bound + lo;
+  if (tid < kMaxTiles) s_cnt[tid] = 0;
+  __syncthreads();
+
+  // pass 1: residents per tile
+  for (int r0 = 0; r0 < n; r0 += kRound) {
+    int32_t p[kPerThread], g[kPerThread], U[kPerThread];
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      const int i = r0 + j * kOccThreads + tid;
+      const bool ok = i < n;
+      p[j] = ok ? __ldg(pp + i) : -1;
+      g[j] = ok ? __ldg(pg + i) : 0;
+      U[j] = ok ? __ldg(pu + i) : 0;
+    }
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      int32_t b32, e;
+      bool big;
+      const int tile = resident_terms(p[j], g[j], U[j], H, b32, e, big) ? (e - 1) >> log2W : -1;
+      const unsigned peers = __match_any_sync(0xffffffffu, tile);
+      if (tile >= 0 && lane == __ffs(peers) - 1) atomicAdd(&s_cnt[tile], __popc(peers));
+    }
+  }
+  __syncthreads();
+  if (tid == 0) {  // tile starts; T <= kMaxTiles
+    int run = 0;
+    int32_t *to = tile_off + static_cast<int64_t>(k) * (T + 1);
+    for (int y = 0; y < T; ++y) {
+      to[y] = run;
+      s_cur[y] = run;
+      run += s_cnt[y];
+    }
+    to[T] = run;
+  }
+  __syncthreads();
+
+  // pass 2: scatter the pairs (the residents come from L2 this time)
+  bool bad = false;
+  long long total = 0;
+  for (int r0 = 0; r0 < n; r0 += kRound) {
+    int32_t p[kPerThread], g[kPerThread], U[kPerThread];
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      const int i = r0 + j * kOccThreads + tid;
+      const bool ok = i < n;
+      p[j] = ok ? __ldg(pp + i) : -1;
+      g[j] = ok ? __ldg(pg + i) : 0;
+      U[j] = ok ? __ldg(pu + i) : 0;
+    }
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      const bool present = r0 + j * kOccThreads + tid < n;
+      int32_t b32 = 0, e = 0;
+      bool big = false;
+      int tile = -1;
+      if (resident_terms(p[j], g[j], U[j], H, b32, e, big)) {
+        tile = (e - 1) >> log2W;
+        total += b32;
+        bad |= big;
+      } else if (present) {
+        bad = true;
+      }
+      const unsigned peers = __match_any_sync(0xffffffffu, tile);
+      const int leader = __ffs(peers) - 1;
+      int base = 0;
+      if (tile >= 0 && lane == leader) base = atomicAdd(&s_cur[tile], __popc(peers));
+      base = __shfl_sync(0xffffffffu, base, leader);
+      if (tile >= 0) bucket[lo + base + __popc(peers & ((1u << lane) - 1u))] = make_int2(b32, e);
+    }
+  }
+  if (bad) flag_error(status, MAPS_E_RANGE);
+  const long long sum_b = block_sum_ll(total, s_red);
+  if (tid == 0 && sum_b > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
+}
+
+// ---------------------------------------------------------------------------
+// 2. Tile kernel: one CTA per (decoder, tile), reading the sorted pairs.
+// ---------------------------------------------------------------------------
+template <int CPT, bool VEC>
+__global__ void __launch_bounds__(kOccThreads, 2)
+occ_tile_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
+                const int2 *__restrict__ bucket, const int32_t *__restrict__ tile_off,
+                int32_t *__restrict__ K, uint32_t *__restrict__ kmax, int32_t *status) {
+  __shared__ __align__(16) TileSmem<CPT> sm;
+  constexpr int W = TileSmem<CPT>::W;
+  const int k = blockIdx.x / T, ti = blockIdx.x - (blockIdx.x / T) * T;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int t0 = ti * W;
+  int64_t lo = res_off[k];
+  const int32_t *to = tile_off + static_cast<int64_t>(k) * (T + 1);
+  const int a = to[ti], m = to[ti + 1], z = to[T];
+  if (lo < 0 || lo > R) lo = 0;  // reported by the bucket kernel; the range is then empty
+  const int2 *bk = bucket + lo;
+  zero_bins(sm);
+  __syncthreads();
+
+  uint32_t car_c = 0, car_s = 0;
+  for (int r0 = a; r0 < z; r0 += kRound) {
+    int2 v[kPerThread];
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      const int i = r0 + j * kOccThreads + tid;
+      v[j] = i < z ? __ldg(bk + i) : make_int2(0, 0);
+    }
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      const int i = r0 + j * kOccThreads + tid;
+      if (i < m) {
+        add_to_bin(sm, v[j].y - 1 - t0, v[j].x);
+      } else if (i < z) {
+        car_c += 1;
+        car_s += static_cast<uint32_t>(v[j].x);
+      }
     }
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
-    carry_c += __shfl_xor_sync(0xffffffffu, carry_c, off);
-    carry_s += __shfl_xor_sync(0xffffffffu, carry_s, off);
-    total_b += __shfl_xor_sync(0xffffffffu, total_b, off);
+    car_c += __shfl_xor_sync(0xffffffffu, car_c, off);
+    car_s += __shfl_xor_sync(0xffffffffu, car_s, off);
   }
   if (lane == 0) {
-    s_red[0][warp] = carry_c;
-    s_red[1][warp] = carry_s;
-    s_red[2][warp] = total_b;
-  }
-  for (int i = tid; i < WP; i += kOccThreads) {
-    s_cnt[i] = 0;
-    s_sb[i] = 0;
+    sm.part[0][warp] = car_c;
+    sm.part[1][warp] = car_s;
   }
   __syncthreads();
-  if (tid == 0) {
-    long long a = 0, b = 0, t = 0;
-    for (int w = 0; w < kWarps; ++w) {
-      a += s_red[0][w];
-      b += s_red[1][w];
-      t += s_red[2][w];
-    }
-    s_carry[(ntile - 1) & 1][0] = a;
-    s_carry[(ntile - 1) & 1][1] = b;
-    if (chunk == 0 && t > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
-  }
-
-  // 2. Tiles from the highest down; tile ti reads its carry from slot ti & 1
-  //    and leaves the next lower tile's in the other slot.  Histograms start
-  //    zeroed; each thread
-  //    clears its own bins as it reads them.
-  bool over = false;
-  for (int ti = ntile - 1; ti >= 0; --ti) {
-    const int64_t t0 = (tile_lo + ti) * W;
-    for (int64_t b0 = 0; b0 < nres; b0 += kStage) {
-      if (!staged_once) {
-        __syncthreads();
-        if (tid == 0) s_nin = 0;
-        __syncthreads();
-        gather(b0, static_cast<int>(min(static_cast<int64_t>(kStage), nres - b0)), false);
-      }
-      __syncthreads();
-      const int nin = s_nin;
-      for (int i = tid; i < nin; i += kOccThreads) {
-        const int2 v = s_res[i];
-        const long long e = v.y;
-        if (e > t0 && e <= t0 + W) {
-          const int j = static_cast<int>(e - t0 - 1);  // last live cell, 0..W-1
-          const int jp = j + (j / CPT) * kPad;
-          atomicAdd(&s_cnt[jp], 1);
-          atomicAdd(&s_sb[jp], v.x);  // exact while sum b fits int32
-        }
-      }
-      if (staged_once) break;
-    }
-    __syncthreads();
-
-    // Thread tid owns cells l = tid*CPT + c and the bins with the same index.
-    // Cell l needs every bin j >= l: its own bins from l up plus all bins of
-    // the threads above it.  All sums stay below K[k][0] <= INT32_MAX unless
-    // a range error is already flagged, so they are kept in 32 bits.
-    int32_t *cb = &s_cnt[tid * (CPT + kPad)], *sb = &s_sb[tid * (CPT + kPad)];
-    uint32_t tot_c = 0, tot_s = 0;
-#pragma unroll
-    for (int c = 0; c < CPT; c += 4) {
-      const int4 x = *reinterpret_cast<const int4 *>(cb + c);
-      const int4 y = *reinterpret_cast<const int4 *>(sb + c);
-      tot_c += static_cast<uint32_t>(x.x + x.y + x.z + x.w);
-      tot_s += static_cast<uint32_t>(y.x + y.y + y.z + y.w);
-    }
-    uint32_t suf_c = tot_c, suf_s = tot_s;  // inclusive suffix within the warp
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t yc = __shfl_down_sync(0xffffffffu, suf_c, off);
-      const uint32_t ys = __shfl_down_sync(0xffffffffu, suf_s, off);
-      if (lane + off < 32) {
-        suf_c += yc;
-        suf_s += ys;
-      }
-    }
-    if (lane == 0) {
-      s_wsum[0][warp] = suf_c;
-      s_wsum[1][warp] = suf_s;
-    }
-    __syncthreads();
-    if (warp == 0) {  // exclusive suffix over the warps' totals
-      uint32_t wc = lane < kWarps ? s_wsum[0][lane] : 0u;
-      uint32_t ws = lane < kWarps ? s_wsum[1][lane] : 0u;
-      const uint32_t oc = wc, os = ws;
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const uint32_t yc = __shfl_down_sync(0xffffffffu, wc, off);
-        const uint32_t ys = __shfl_down_sync(0xffffffffu, ws, off);
-        if (lane + off < 32) {
-          wc += yc;
-          ws += ys;
-        }
-      }
-      __syncwarp();
-      if (lane < kWarps) {
-        s_wsum[0][lane] = wc - oc;
-        s_wsum[1][lane] = ws - os;
-      }
-      if (lane == 0) {  // the next lower tile also carries this tile's residents
-        s_red[0][0] = wc;
-        s_red[1][0] = ws;
-      }
-    }
-    __syncthreads();
-    const long long cc = s_carry[ti & 1][0], cs = s_carry[ti & 1][1];
-    uint32_t run_c = static_cast<uint32_t>(cc) + s_wsum[0][warp] + (suf_c - tot_c);
-    uint32_t run_s = static_cast<uint32_t>(cs) + s_wsum[1][warp] + (suf_s - tot_s);
-
-    uint32_t bmax = 0;  // max of K + t over this thread's valid cells
-    const int64_t cell0 = t0 + static_cast<int64_t>(tid) * CPT;
-    const uint32_t tc0 = static_cast<uint32_t>(cell0);
-    int32_t *row = K + static_cast<int64_t>(k) * H;
-    const bool full = cell0 + CPT <= H;
-    bool ovf = false;
-#pragma unroll
-    for (int c0 = CPT - 4; c0 >= 0; c0 -= 4) {
-      const int4 x = *reinterpret_cast<const int4 *>(cb + c0);
-      const int4 y = *reinterpret_cast<const int4 *>(sb + c0);
-      *reinterpret_cast<int4 *>(cb + c0) = make_int4(0, 0, 0, 0);
-      *reinterpret_cast<int4 *>(sb + c0) = make_int4(0, 0, 0, 0);
-      const int32_t xc[4] = {x.x, x.y, x.z, x.w}, xs[4] = {y.x, y.y, y.z, y.w};
-      uint32_t o[4];
-#pragma unroll
-      for (int c = 3; c >= 0; --c) {
-        run_c += static_cast<uint32_t>(xc[c]);
-        run_s += static_cast<uint32_t>(xs[c]);
-        const uint32_t t = tc0 + c0 + c;
-        // K = run_s + t * run_c, exact in 64 bits
-        const unsigned long long v = static_cast<unsigned long long>(t) * run_c + run_s;
-        o[c] = static_cast<uint32_t>(v);
-        const bool valid = full || (cell0 + c0 + c < H);
-        ovf |= valid && (v >> 31) != 0;
-        const uint32_t xm = valid ? o[c] + t : 0u;
-        bmax = xm > bmax ? xm : bmax;
-      }
-      if (VEC && full) {
-        *reinterpret_cast<int4 *>(row + cell0 + c0) = make_int4(o[0], o[1], o[2], o[3]);
-      } else {
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-          if (cell0 + c0 + c < H) row[cell0 + c0 + c] = static_cast<int32_t>(o[c]);
-      }
-    }
-    over |= ovf;
-    if (kmax != nullptr) {
-      constexpr int L = kBlock / CPT > 0 ? kBlock / CPT : 1;  // lanes per 16-step block
-#pragma unroll
-      for (int off = L / 2; off > 0; off >>= 1) {
-        const uint32_t y = __shfl_xor_sync(0xffffffffu, bmax, off);
-        bmax = y > bmax ? y : bmax;
-      }
-      if ((lane % L) == 0 && cell0 < H) {
-        const int64_t nb = (static_cast<int64_t>(H) + kBlock - 1) / kBlock;
-        kmax[static_cast<int64_t>(k) * nb + cell0 / kBlock] = bmax;
-      }
-    }
-    if (tid == 0) {
-      s_carry[(ti & 1) ^ 1][0] = cc + s_red[0][0];
-      s_carry[(ti & 1) ^ 1][1] = cs + s_red[1][0];
-    }
-    __syncthreads();
-  }
-  if (bad || over) flag_error(status, MAPS_E_RANGE);
+  emit_tile<CPT, VEC>(sm, H, k, t0, K, kmax, status);
 }
 
-int launch_occ(int cpt, bool vec, int64_t blocks, cudaStream_t s, int D, int H, int TPC, int G,
-               const int64_t *res_off, int64_t R, const int32_t *prompt, const int32_t *gen,
-               const int32_t *bound, int32_t *K, uint32_t *kmax, int32_t *status) {
-  const dim3 grid(static_cast<unsigned>(blocks));
-  if (cpt == 16) {
-    if (vec)
-      occupancy_kernel<16, true><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
-                                                              bound, K, kmax, status);
-    else
-      occupancy_kernel<16, false><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
-                                                               bound, K, kmax, status);
-  } else if (cpt == 8) {
-    if (vec)
-      occupancy_kernel<8, true><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
-                                                             bound, K, kmax, status);
-    else
-      occupancy_kernel<8, false><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
-                                                              bound, K, kmax, status);
-  } else if (cpt == 4) {
-    if (vec)
-      occupancy_kernel<4, true><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
-                                                             bound, K, kmax, status);
-    else
-      occupancy_kernel<4, false><<<grid, kOccThreads, 0, s>>>(D, H, TPC, G, res_off, R, prompt, gen,
-                                                              bound, K, kmax, status);
+// ---------------------------------------------------------------------------
+// Long horizons: every tile CTA streams all of its decoder's residents.
+// ---------------------------------------------------------------------------
+template <int CPT, bool VEC>
+__global__ void __launch_bounds__(kOccThreads, 2)
+occ_direct_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
+                  const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
+                  const int32_t *__restrict__ bound, int32_t *__restrict__ K,
+                  uint32_t *__restrict__ kmax, int32_t *status) {
+  __shared__ __align__(16) TileSmem<CPT> sm;
+  __shared__ long long s_red[kWarps];
+  constexpr int W = TileSmem<CPT>::W;
+  const int k = blockIdx.x / T, ti = blockIdx.x - (blockIdx.x / T) * T;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int t0 = ti * W;
+  int64_t lo = res_off[k], hi = res_off[k + 1];
+  if (lo < 0 || hi < lo || hi > R) {
+    if (tid == 0) flag_error(status, MAPS_E_RANGE);
+    lo = hi = 0;
   }
-  return launch_ok();
+  const int64_t n = hi - lo;
+  const int32_t *pp = prompt + lo, *pg = gen + lo, *pu = bound + lo;
+  zero_bins(sm);
+  __syncthreads();
+
+  bool bad = false;
+  long long total = 0;
+  uint32_t car_c = 0, car_s = 0;
+  for (int64_t r0 = 0; r0 < n; r0 += kRound) {
+    int32_t p[kPerThread], g[kPerThread], U[kPerThread];
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      const int64_t i = r0 + j * kOccThreads + tid;
+      const bool ok = i < n;
+      p[j] = ok ? __ldg(pp + i) : -1;
+      g[j] = ok ? __ldg(pg + i) : 0;
+      U[j] = ok ? __ldg(pu + i) : 0;
+    }
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      int32_t b32, e;
+      bool big;
+      if (resident_terms(p[j], g[j], U[j], H, b32, e, big)) {
+        total += b32;
+        bad |= big;
+        const int jj = e - 1 - t0;  // last live step, relative to the tile
+        if (jj >= W) {
+          car_c += 1;
+          car_s += static_cast<uint32_t>(b32);
+        } else if (jj >= 0) {
+          add_to_bin(sm, jj, b32);
+        }
+      } else if (r0 + j * kOccThreads + tid < n) {
+        bad = true;
+      }
+    }
+  }
+  if (bad) flag_error(status, MAPS_E_RANGE);
+  const long long sum_b = block_sum_ll(total, s_red);
+  if (ti == 0 && tid == 0 && sum_b > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    car_c += __shfl_xor_sync(0xffffffffu, car_c, off);
+    car_s += __shfl_xor_sync(0xffffffffu, car_s, off);
+  }
+  if (lane == 0) {
+    sm.part[0][warp] = car_c;
+    sm.part[1][warp] = car_s;
+  }
+  __syncthreads();
+  emit_tile<CPT, VEC>(sm, H, k, t0, K, kmax, status);
+}
+
+struct OccPlan {
+  int cpt, T, log2W;
+  bool bucketed;
+};
+
+OccPlan plan_occ(int32_t H, int64_t R) {
+  OccPlan p;
+  p.cpt = H <= 2048 ? 4 : (H <= 8192 ? 8 : 16);
+  p.log2W = 9 + (p.cpt == 4 ? 2 : (p.cpt == 8 ? 3 : 4));
+  p.T = static_cast<int>((static_cast<int64_t>(H) + (1 << p.log2W) - 1) >> p.log2W);
+  p.bucketed = p.T <= kMaxTiles && R <= 0x7fffffffLL;
+  return p;
+}
+
+size_t carve_occ(Carve &c, int32_t D, int64_t R, const OccPlan &p, int2 **bucket,
+                 int32_t **tile_off) {
+  if (p.bucketed) {
+    *bucket = c.take<int2>(static_cast<size_t>(R));
+    *tile_off = c.take<int32_t>(static_cast<size_t>(D) * (p.T + 1));
+  }
+  return c.bytes();
+}
+
+template <int CPT, bool VEC>
+void launch_tiles(const OccPlan &p, int64_t blocks, cudaStream_t s, int H, const int64_t *res_off,
+                  int64_t R, const int32_t *prompt, const int32_t *gen, const int32_t *bound,
+                  const int2 *bucket, const int32_t *tile_off, int32_t *K, uint32_t *kmax,
+                  int32_t *status) {
+  const dim3 grid(static_cast<unsigned>(blocks));
+  if (p.bucketed)
+    occ_tile_kernel<CPT, VEC><<<grid, kOccThreads, 0, s>>>(H, p.T, res_off, R, bucket, tile_off, K,
+                                                          kmax, status);
+  else
+    occ_direct_kernel<CPT, VEC><<<grid, kOccThreads, 0, s>>>(H, p.T, res_off, R, prompt, gen,
+                                                            bound, K, kmax, status);
+}
+
+template <int CPT>
+void launch_cpt(bool vec, const OccPlan &p, int64_t blocks, cudaStream_t s, int H,
+                const int64_t *res_off, int64_t R, const int32_t *prompt, const int32_t *gen,
+                const int32_t *bound, const int2 *bucket, const int32_t *tile_off, int32_t *K,
+                uint32_t *kmax, int32_t *status) {
+  if (vec)
+    launch_tiles<CPT, true>(p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K,
+                            kmax, status);
+  else
+    launch_tiles<CPT, false>(p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K,
+                             kmax, status);
 }
 
 }  // namespace
@@ -337,10 +502,12 @@ int launch_occ(int cpt, bool vec, int64_t blocks, cudaStream_t s, int D, int H, 
 extern "C" {
 
 size_t maps_project_occupancy_workspace_size(int32_t D, int32_t H, int64_t R) {
-  (void)D;
-  (void)H;
-  (void)R;
-  return maps::kCtrlBytes;
+  using namespace maps;
+  if (D < 1 || H < 1 || R < 0) return kCtrlBytes;
+  Carve c(nullptr);
+  int2 *bucket = nullptr;
+  int32_t *tile_off = nullptr;
+  return carve_occ(c, D, R, plan_occ(H, R), &bucket, &tile_off);
 }
 
 int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off, int64_t R,
@@ -348,21 +515,35 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off, int64_t
                            int32_t *K_out, uint32_t *kmax_out, void *ws, size_t ws_bytes,
                            void *stream) {
   using namespace maps;
-  if (D < 1 || H < 1 || R < 0 || res_off == nullptr || K_out == nullptr) return MAPS_E_INVALID;
+  if (D < 1 || H < 1 || H > (1 << 28) || R < 0 || res_off == nullptr || K_out == nullptr)
+    return MAPS_E_INVALID;
   if (R > 0 && (prompt == nullptr || gen == nullptr || bound == nullptr)) return MAPS_E_INVALID;
   MAPS_TRY(check_ws(ws, ws_bytes, maps_project_occupancy_workspace_size(D, H, R)));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int32_t *status = status_word(ws);
-  const int cpt = H <= 2048 ? 4 : (H <= 8192 ? 8 : 16);
-  const int64_t W = static_cast<int64_t>(kOccThreads) * cpt;
-  const int64_t tiles = (H + W - 1) / W;
-  const int TPC = static_cast<int>(tiles < kTilesPerChunk ? tiles : kTilesPerChunk);
-  const int64_t G = (tiles + TPC - 1) / TPC;
-  const int64_t blocks = static_cast<int64_t>(D) * G;
+  const OccPlan p = plan_occ(H, R);
+  const int64_t blocks = static_cast<int64_t>(D) * p.T;
   if (blocks > 0x7fffffffLL) return MAPS_E_INVALID;
+  Carve c(ws);
+  int2 *bucket = nullptr;
+  int32_t *tile_off = nullptr;
+  carve_occ(c, D, R, p, &bucket, &tile_off);
+  if (p.bucketed) {
+    occ_bucket_kernel<<<D, kOccThreads, 0, s>>>(H, p.T, p.log2W, res_off, R, prompt, gen, bound,
+                                                bucket, tile_off, status);
+    MAPS_TRY(launch_ok());
+  }
   const bool vec = (H % 4 == 0) && aligned(K_out, 16);
-  return launch_occ(cpt, vec, blocks, s, D, H, TPC, static_cast<int>(G), res_off, R, prompt, gen,
-                    bound, K_out, kmax_out, status);
+  if (p.cpt == 16)
+    launch_cpt<16>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K_out,
+                   kmax_out, status);
+  else if (p.cpt == 8)
+    launch_cpt<8>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K_out,
+                  kmax_out, status);
+  else
+    launch_cpt<4>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K_out,
+                  kmax_out, status);
+  return launch_ok();
 }
 
 }  // extern "C"

@@ -215,7 +215,10 @@ def random_residents(rng, D, H, per_max, with_empty=True):
 
 
 @pytest.mark.parametrize("D,H", [(1, 1), (3, 3), (2, 8), (5, 511), (4, 512), (3, 513), (7, 4095),
-                                 (2, 4097), (9, 4100), (3, 12289), (2, 65536)])
+                                 (2, 4097), (9, 4100), (3, 12289), (2, 65536),
+                                 # 64 horizon tiles (the most the bucketed form takes), then
+                                 # more, which stream every resident per tile instead
+                                 (2, 524288), (2, 524292), (1, 600001)])
 def test_occupancy_random(M, ws, oracle, D, H):
     rng = np.random.default_rng(D * 100003 + H)
     off, p, g, U = random_residents(rng, D, H, 700)
