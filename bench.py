@@ -194,10 +194,11 @@ class Step:
                    M.lib.maps_order_local_workspace_size(R + J, self.D))
         self.ws = M.Workspace(need, device)
         dbits = (self.D - 1).bit_length()
-        n_hi = min(8, (32 + dbits + 7) // 8)
-        # calibrate 4, occupancy 1, dispatch 5 (carry scan, bin count / scan /
-        # scatter, main), order 2 + 4 + n_hi + 2
-        self.kernels_per_step = 4 + 1 + 5 + (2 + 4 + n_hi + 2)
+        n_hi = min(8, (dbits + 1 + 31 + 7) // 8)
+        # calibrate 4 (three select passes, bounds); occupancy 2 (bucket, tile);
+        # dispatch 5 (carry scan, bin count / scan / scatter, main); order
+        # prep, keys, plan, 4 arrival passes, gather, n_hi key passes, identity
+        self.kernels_per_step = 4 + 2 + 5 + (3 + 4 + 1 + n_hi + 1)
 
     def run(self, ev=None):
         M, R = self.M, self.R

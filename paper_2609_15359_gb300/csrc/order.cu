@@ -16,9 +16,10 @@
 // histogram), a one-block plan (digit offsets, which passes run, buffers,
 // decoder segment offsets), then one sweep per digit: tiles of 4096 keys are
 // ranked stably in shared memory, each tile learns its offsets from earlier
-// tiles by decoupled look-back (256 predecessors inspected per round, one
-// thread each), and writes out bin by bin.  Passes the plan marks inactive return at once,
-// so the host never waits on the device.
+// tiles by decoupled look-back (one thread per digit walks back over packed
+// flag-and-count words until it meets an inclusive prefix), and writes out
+// bin by bin.  Passes the plan marks inactive return at once, so the host
+// never waits on the device.
 #include "maps_internal.cuh"
 
 #include <algorithm>
@@ -37,7 +38,6 @@ constexpr int kHiPasses = 8;  // key digits
 constexpr int kPasses = kLoPasses + kHiPasses;
 constexpr int kDecSmem = 8192;  // decoders counted in shared memory up to this D
 constexpr uint32_t kFlagAgg = 1, kFlagInc = 2;
-constexpr int kLookWindow = 256;  // predecessor tiles inspected per look-back round
 
 enum : int32_t { kBufA = 0, kBufB = 1, kHiIdentity = 2, kPermOut = 2 };
 
@@ -56,6 +56,7 @@ struct OrderPlan {
   int32_t npasses;
   int32_t wide;        // keys need 64 bits
   int32_t ubits;       // bit width of the primary (bound) field
+  int32_t ordinal[kPasses];  // position among the active passes
   uint32_t digit_off[kPasses][kRadix];
 };
 
@@ -267,6 +268,7 @@ order_plan_kernel(int64_t N, int D, int dbits, const OrderCounts *counts, OrderP
       if (last >= 0) plan->dst[last] = kPermOut;
     }
     plan->npasses = n;
+    for (int p = 0, o = 0; p < kPasses; ++p) plan->ordinal[p] = plan->active[p] ? o++ : -1;
     s_carry = 0;
   }
   __syncthreads();
@@ -328,9 +330,6 @@ struct PassSmem {
   uint32_t bin_start[kRadix];       // tile-local start of each bin
   uint32_t excl[kRadix];            // offset of this tile within each bin
   uint32_t scan_w[kRadix / 32];
-  uint32_t look_flag[256];          // flags of the predecessor window
-  uint32_t look_part[2][kRadix];    // partial window sums
-  int look_inc;                     // nearest window slot with an inclusive prefix
   int tile;
 };
 
@@ -354,7 +353,7 @@ template <bool WIDE>
 __device__ void order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
                                 unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
                                 const unsigned long long *hi_orig, int32_t *perm,
-                                uint32_t *flags, uint32_t *agg, uint32_t *inc, uint32_t *ticket,
+                                unsigned long long *state, int64_t tiles, uint32_t *ticket,
                                 int32_t *status, PassSmem &sm) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool lo = p < kLoPasses;
@@ -403,9 +402,16 @@ __device__ void order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
     rank[it] = cur + before;
   }
   __syncthreads();
-  // per bin: exclusive scan over warps, tile total; publish the aggregate
-  uint32_t *my_agg = agg + static_cast<size_t>(tile) * kRadix;
-  uint32_t *my_inc = inc + static_cast<size_t>(tile) * kRadix;
+  // Per bin: exclusive scan over warps and the tile total.  Then decoupled
+  // look-back, one thread per bin: the tile publishes its aggregate, walks
+  // back over its predecessors' (flag, count) words until it meets an
+  // inclusive prefix, and publishes its own inclusive prefix.  Words carry the
+  // flag in their top two bits.  Active pass number o uses state buffer o & 1
+  // and clears this tile's row of the other buffer for active pass o + 1
+  // (the buffer of the first active pass is cleared with the counts).
+  const int ord = plan->ordinal[p];
+  unsigned long long *st_cur = state + static_cast<size_t>(ord & 1) * tiles * kRadix;
+  unsigned long long *st_nxt = state + static_cast<size_t>((ord + 1) & 1) * tiles * kRadix;
   if (tid < kRadix) {
     uint32_t run = 0;
     for (int w = 0; w < kPassWarps; ++w) {
@@ -414,79 +420,31 @@ __device__ void order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
       run += c;
     }
     sm.tile_cnt[tid] = run;
-    sm.excl[tid] = 0;
-    if (tile == 0)
-      my_inc[tid] = run;
-    else
-      my_agg[tid] = run;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    __threadfence();
-    st_release_u32(flags + tile, tile == 0 ? kFlagInc : kFlagAgg);
-  }
-  // Look back over up to 256 predecessor tiles per round, one thread per
-  // tile: wait until each has published at least its aggregate, find the
-  // nearest one that has published its inclusive prefix, and add up the
-  // aggregates above it (and its inclusive value) bin by bin.
-  for (int top = tile - 1; top >= 0;) {
-    if (tid < kLookWindow) {
-      const int q = top - tid;
-      uint32_t f = kFlagInc;  // "tile -1" is an empty inclusive prefix
-      if (q >= 0) {
+    const size_t me = static_cast<size_t>(tile) * kRadix + tid;
+    st_nxt[me] = 0ull;
+    st_release_u64(&st_cur[me], static_cast<unsigned long long>(run) |
+                                    (static_cast<unsigned long long>(tile == 0 ? kFlagInc : kFlagAgg) << 62));
+    unsigned long long excl = 0;
+    if (tile > 0) {
+      for (int q = tile - 1;; --q) {
+        unsigned long long v;
         uint32_t spins = 0;
-        while ((f = ld_acquire_u32(flags + q)) == 0) {
+        while (((v = ld_acquire_u64(&st_cur[static_cast<size_t>(q) * kRadix + tid])) >> 62) == 0) {
           if (++spins > kSpinLimit) {
             flag_error(status, MAPS_E_TIMEOUT);
-            f = kFlagInc;  // give up: use what is there
+            v = static_cast<unsigned long long>(kFlagInc) << 62;  // give up
             break;
           }
           __nanosleep(32);
         }
+        excl += v & ((1ull << 62) - 1);
+        if ((v >> 62) == kFlagInc || q == 0) break;
       }
-      sm.look_flag[tid] = f;
+      st_release_u64(&st_cur[me], (excl + run) | (static_cast<unsigned long long>(kFlagInc) << 62));
     }
-    if (tid == 0) sm.look_inc = -1;
-    __syncthreads();
-    if (tid < kLookWindow && sm.look_flag[tid] == kFlagInc) atomicMin(reinterpret_cast<unsigned *>(&sm.look_inc), static_cast<unsigned>(tid));
-    __syncthreads();
-    // lanes 0 .. depth-1 of the window are added; depth ends at the nearest
-    // inclusive prefix (included), else covers the whole window
-    const int near = sm.look_inc;  // -1 (as unsigned max) when none
-    const int depth = (near >= 0 && near < kLookWindow) ? near + 1 : kLookWindow;
-    {
-      // thread (bin, half) adds every other group of 16 window slots, with
-      // the 16 loads of a group in flight together
-      const int bin = tid & (kRadix - 1), half = tid >> 8;
-      uint32_t add = 0;
-      for (int x0 = half * 16; x0 < depth; x0 += 32) {
-        uint32_t v[16];
-#pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          const int x = x0 + u, q = top - x;
-          v[u] = (x < depth && q >= 0)
-                     ? __ldcg((sm.look_flag[x] == kFlagInc ? inc : agg) + static_cast<size_t>(q) * kRadix + bin)
-                     : 0u;
-        }
-#pragma unroll
-        for (int u = 0; u < 16; ++u) add += v[u];
-      }
-      sm.look_part[half][bin] = add;
-    }
-    __syncthreads();
-    if (tid < kRadix) sm.excl[tid] += sm.look_part[0][tid] + sm.look_part[1][tid];
-    __syncthreads();
-    if (near >= 0 && near < kLookWindow) break;
-    top -= kLookWindow;
+    sm.excl[tid] = static_cast<uint32_t>(excl);
   }
-  if (tile > 0) {
-    if (tid < kRadix) my_inc[tid] = sm.excl[tid] + sm.tile_cnt[tid];
-    __syncthreads();
-    if (tid == 0) {
-      __threadfence();
-      st_release_u32(flags + tile, kFlagInc);
-    }
-  }
+  __syncthreads();
   // tile-local bin starts (the first 8 warps hold the 256 bins)
   uint32_t bc = 0, bincl = 0;
   if (tid < kRadix) {
@@ -530,16 +488,16 @@ __device__ void order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
 __global__ void __launch_bounds__(kPassThreads)
 order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
                   unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
-                  const unsigned long long *hi_orig, int32_t *perm, uint32_t *flags,
-                  uint32_t *agg, uint32_t *inc, uint32_t *ticket, int32_t *status) {
+                  const unsigned long long *hi_orig, int32_t *perm, unsigned long long *state,
+                  int64_t tiles, uint32_t *ticket, int32_t *status) {
   if (!plan->active[p]) return;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PassSmem &sm = *reinterpret_cast<PassSmem *>(smem_raw);
   if (plan->wide)
-    order_pass_body<true>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, flags, agg, inc,
-                          ticket, status, sm);
+    order_pass_body<true>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, state, tiles, ticket,
+                          status, sm);
   else
-    order_pass_body<false>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, flags, agg, inc,
+    order_pass_body<false>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, state, tiles,
                            ticket, status, sm);
 }
 
@@ -547,9 +505,8 @@ struct OrderWs {
   OrderCounts *counts;
   uint32_t *dec_count;
   uint32_t *tickets;
-  uint32_t *flags;  // [kPasses][tiles]
-  size_t zero_bytes;  // counts .. flags are contiguous and zeroed per call
-  uint32_t *agg, *inc;  // [kPasses][tiles][256]
+  unsigned long long *state;  // [2][tiles][256] look-back words
+  size_t zero_bytes;  // counts .. state buffer 0 are contiguous and zeroed per call
   OrderPlan *plan;
   unsigned long long *hi_orig, *keyA, *keyB;
   uint32_t *valA, *valB;
@@ -562,10 +519,8 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.counts = c.take<OrderCounts>(1);
   w.dec_count = c.take<uint32_t>(static_cast<size_t>(D));
   w.tickets = c.take<uint32_t>(kPasses);
-  w.flags = c.take<uint32_t>(static_cast<size_t>(kPasses) * tiles);
-  w.zero_bytes = c.off - zero_begin;
-  w.agg = c.take<uint32_t>(static_cast<size_t>(kPasses) * tiles * kRadix);
-  w.inc = c.take<uint32_t>(static_cast<size_t>(kPasses) * tiles * kRadix);
+  w.state = c.take<unsigned long long>(static_cast<size_t>(2) * tiles * kRadix);
+  w.zero_bytes = c.off - zero_begin - static_cast<size_t>(tiles) * kRadix * sizeof(unsigned long long);
   w.plan = c.take<OrderPlan>(1);
   const size_t n = static_cast<size_t>(N > 0 ? N : 1);
   w.hi_orig = c.take<unsigned long long>(n);
@@ -624,9 +579,8 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   const int gcopy = static_cast<int>(std::min<int64_t>((N + 255) / 256, 4LL * sms));
   auto pass = [&](int p) {
     order_pass_kernel<<<static_cast<unsigned>(tiles), kPassThreads, smem, s>>>(
-        p, N, w.plan, w.keyA, w.keyB, w.valA, w.valB, w.hi_orig, perm_out,
-        w.flags + static_cast<size_t>(p) * tiles, w.agg + static_cast<size_t>(p) * tiles * kRadix,
-        w.inc + static_cast<size_t>(p) * tiles * kRadix, w.tickets + p, status);
+        p, N, w.plan, w.keyA, w.keyB, w.valA, w.valB, w.hi_orig, perm_out, w.state, tiles,
+        w.tickets + p, status);
   };
   for (int p = 0; p < kLoPasses; ++p) pass(p);
   order_gather_kernel<<<gcopy, 256, 0, s>>>(N, w.plan, w.hi_orig, w.keyA, w.keyB, w.valA, w.valB);
