@@ -243,6 +243,68 @@ int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
                             int32_t *perm_out, int64_t *seg_off_out,
                             int32_t *status_host, void *stream);
 
+/* ------------------------------------------------------------------------
+ * The streaming scheduler loop, run on the device end to end.
+ *
+ * Requests arrive with arrival step arrival_ms[i] (1 ms per decode step,
+ * non-decreasing in i) and are dispatched in batches of cfg->batch in index
+ * order; batch b is dispatched at the arrival step s_b of its last request.
+ * Per batch, following Sec. 3.2 (sliding calibration window), Sec. 3.3
+ * (memory-aware dispatch, local SJF order with promotion), Algorithm 1 (round
+ * robin when no bound is available) and App. A Eq. (admission):
+ *   1. every running request generates s_b - s_{b-1} tokens (one per step);
+ *      one that reaches its true length completes at the step it does;
+ *   2. completions enter a window of the last cfg->window completed
+ *      requests, ordered by (completion step, index);
+ *   3. q = the conformal quantile of the window (maps_calibrate); every
+ *      request in the system and in the batch gets U = pred + q.  If the
+ *      quantile is unbounded (too few completions) U = pred, q_out[b] = -1
+ *      and the batch is dispatched round robin: choice = index mod D;
+ *   4. otherwise occupancy is projected over the running (g generated) and
+ *      waiting (g = 0) requests and the batch is dispatched SEQUENTIALly
+ *      (maps_dispatch) with Q[k] = requests waiting at decoder k;
+ *   5. the batch joins the chosen decoders' waiting queues;
+ *   6. each waiting queue is put in local order (maps_order_local, with
+ *      wait = s_b - dispatch step) and admitted in that order while
+ *      used + p + U <= cap (used = prompt + generated tokens of the running
+ *      requests, grown by p per admission); the first misfit stops its queue.
+ * No preemption; a running request above capacity is only counted.
+ *
+ *   cfg                 host struct: N requests (1 .. INT32_MAX), D decoders
+ *                       (1 .. 1024), horizon H steps, capacity cap tokens per
+ *                       decoder, batch size, window size, alpha in parts per
+ *                       million (0 < alpha_ppm < 10^6), max_wait steps.
+ *   arrival_ms          [N] int64 arrival step.
+ *   prompt, true_len, pred   [N] int32 prompt length (>= 0), true output
+ *                       length (>= 1), predicted output length (>= 0).
+ *   choice_out          [N] int32 decoder chosen for each request.
+ *   q_out               [ceil(N / batch)] int32 quantile per batch (-1:
+ *                       unbounded, round robin).
+ *   stats_out           [ceil(N / batch)][4] int64 per batch: completions,
+ *                       admissions, requests left waiting, decoders whose
+ *                       running requests exceed capacity after advancing.
+ * The call runs the whole loop: it synchronises the stream once per batch
+ * (to read the request counts that size the next launches) and at the end,
+ * and returns the full status.  A negative length or decreasing arrival is
+ * MAPS_E_RANGE before any batch runs.
+ * ---------------------------------------------------------------------- */
+typedef struct {
+  int64_t N;
+  int32_t D, H;
+  int32_t cap;
+  int32_t batch;
+  int32_t window;
+  uint32_t alpha_ppm;
+  int32_t max_wait;
+} maps_stream_cfg;
+
+size_t maps_stream_workspace_size(const maps_stream_cfg *cfg);
+int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms,
+                    const int32_t *prompt, const int32_t *true_len,
+                    const int32_t *pred, int32_t *choice_out, int32_t *q_out,
+                    int64_t *stats_out, void *ws, size_t ws_bytes,
+                    void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -683,22 +683,25 @@ __device__ __forceinline__ Pick no_pick() {
 }
 
 // ---------------------------------------------------------------------------
-// SEQUENTIAL horizon dispatch: one block walks the candidates in order,
-// scores every decoder, commits the footprint at the chosen one.
+// SEQUENTIAL horizon dispatch: one block walks the candidates in order.
+// Scoring decoder k needs M_k(u) = max_{t<u} (K[k][t] + t); it is read from
+// the 16-step summary kmax (built from K just before) for the whole blocks
+// below u plus at most 15 cells of K.  Reserving the footprint adds
+// p + t + 1 to K[k*][t] for t < u and rebuilds the summary entries of the
+// blocks it touched, so the summary always matches K.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024, 1)
-dispatch_sequential_kernel(int D, int H, int32_t *K, const int32_t *cap, int32_t *Q, int64_t J,
-                           const int32_t *cp, const int32_t *cb, int32_t *choice,
-                           int64_t *headroom, int32_t *status) {
+dispatch_sequential_kernel(int D, int H, int32_t *K, uint32_t *kmax, const int32_t *cap,
+                           int32_t *Q, int64_t J, const int32_t *cp, const int32_t *cb,
+                           int32_t *choice, int64_t *headroom, int32_t *status) {
   __shared__ uint32_t s_M[kMaxD];
   __shared__ Pick s_w[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
+  const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
   bool bad = false;
   for (int k = tid; k < D; k += blockDim.x)
     if ((cap[k] | Q[k]) < 0) bad = true;
-  for (int64_t i = tid; i < static_cast<int64_t>(D) * H; i += blockDim.x)
-    if (K[i] < 0) bad = true;
-  if (bad) flag_error(status, MAPS_E_RANGE);
+  if (bad) flag_error(status, MAPS_E_RANGE);  // K < 0 is reported by the summary pass
   __syncthreads();
   for (int64_t j = 0; j < J; ++j) {
     const int32_t p = cp[j], U = cb[j];
@@ -711,18 +714,18 @@ dispatch_sequential_kernel(int D, int H, int32_t *K, const int32_t *cap, int32_t
       continue;
     }
     const int u = candidate_steps(U, H);
+    const int nfull = u / kSumBlock, rem = u - nfull * kSumBlock;
     for (int k = warp; k < D; k += nwarp) {
+      const uint32_t *km = kmax + static_cast<int64_t>(k) * nb;
       const int32_t *row = K + static_cast<int64_t>(k) * H;
       uint32_t m = 0;
-      for (int t = lane; t < u; t += 32) {
-        const uint32_t x = static_cast<uint32_t>(row[t]) + static_cast<uint32_t>(t);
-        m = x > m ? x : m;
+      for (int b = lane; b < nfull; b += 32) m = max(m, km[b]);
+      if (lane < rem) {
+        const int t = nfull * kSumBlock + lane;
+        m = max(m, static_cast<uint32_t>(row[t]) + static_cast<uint32_t>(t));
       }
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const uint32_t y = __shfl_xor_sync(0xffffffffu, m, off);
-        m = y > m ? y : m;
-      }
+      for (int off = 16; off > 0; off >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, off));
       if (lane == 0) s_M[k] = m;
     }
     __syncthreads();
@@ -741,16 +744,31 @@ dispatch_sequential_kernel(int D, int H, int32_t *K, const int32_t *cap, int32_t
       else
         Q[b.k] += 1;
     }
-    // reserve the candidate's footprint at the chosen decoder
+    // reserve the candidate's footprint at the chosen decoder; the blocks it
+    // touches are whole 16-lane groups of the loop, so a group's shuffle
+    // maximum is that block's new summary entry
     int32_t *row = K + static_cast<int64_t>(b.k) * H;
+    uint32_t *km = kmax + static_cast<int64_t>(b.k) * nb;
+    const int end = min(((u + kSumBlock - 1) / kSumBlock) * kSumBlock, H);
     bool over = false;
-    for (int t = tid; t < u; t += blockDim.x) {
-      long long v = static_cast<long long>(row[t]) + p + t + 1;
-      if (v > 0x7fffffffLL) {
-        over = true;
-        v = 0x7fffffffLL;
+    for (int t0 = 0; t0 < end; t0 += blockDim.x) {
+      const int t = t0 + tid;
+      uint32_t x = 0;
+      if (t < end) {
+        long long v = row[t];
+        if (t < u) {
+          v += static_cast<long long>(p) + t + 1;
+          if (v > 0x7fffffffLL) {
+            over = true;
+            v = 0x7fffffffLL;
+          }
+          row[t] = static_cast<int32_t>(v);
+        }
+        x = static_cast<uint32_t>(v) + static_cast<uint32_t>(t);
       }
-      row[t] = static_cast<int32_t>(v);
+#pragma unroll
+      for (int off = 8; off > 0; off >>= 1) x = max(x, __shfl_xor_sync(0xffffffffu, x, off));
+      if ((lane & (kSumBlock - 1)) == 0 && t < end) km[t / kSumBlock] = x;
     }
     if (over) flag_error(status, MAPS_E_RANGE);
     __syncthreads();
@@ -1117,6 +1135,8 @@ size_t maps_dispatch_workspace_size(int32_t mode, int32_t D, int32_t H, int64_t 
   if (mode == MAPS_MODE_SNAPSHOT && D >= 1 && H >= 1 && H <= kMaxH) {
     const SnapGeom g = snap_geom(D, H);
     carve_snap(c, D, H, g.T2, J);
+  } else if (mode == MAPS_MODE_SEQUENTIAL && D >= 1 && H >= 1 && H <= kMaxH) {
+    c.take<uint32_t>(static_cast<size_t>(D) * ((static_cast<size_t>(H) + kSumBlock - 1) / kSumBlock));
   } else if ((mode == MAPS_MODE_ALG1_SNAPSHOT || mode == MAPS_MODE_ALG1_SEQUENTIAL) && D >= 1) {
     c.take<long long>(static_cast<size_t>(D));
   }
@@ -1147,10 +1167,17 @@ int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K, con
     case MAPS_MODE_SNAPSHOT:
       return launch_snapshot(D, H, K, kmax, cap, Q, J, cand_prompt, cand_bound, choice_out,
                              headroom_out, ws, s);
-    case MAPS_MODE_SEQUENTIAL:
-      dispatch_sequential_kernel<<<1, 1024, 0, s>>>(D, H, K, cap, Q, J, cand_prompt, cand_bound,
-                                                    choice_out, headroom_out, status);
+    case MAPS_MODE_SEQUENTIAL: {
+      // a private summary of K (also validating K >= 0); updated in place
+      Carve cv(ws);
+      const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
+      uint32_t *km = cv.take<uint32_t>(static_cast<size_t>(D) * nb);
+      const int gk = static_cast<int>(std::min<int64_t>((nb * D + 255) / 256, 8LL * sm_count()));
+      kmax_from_K_kernel<<<gk, 256, 0, s>>>(D, H, K, km, status);
+      dispatch_sequential_kernel<<<1, 1024, 0, s>>>(D, H, K, km, cap, Q, J, cand_prompt,
+                                                    cand_bound, choice_out, headroom_out, status);
       return launch_ok();
+    }
     default: {
       Carve cv(ws);
       long long *B_eff = cv.take<long long>(static_cast<size_t>(D));

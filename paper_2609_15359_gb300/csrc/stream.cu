@@ -1,0 +1,512 @@
+// stream.cu -- the streaming scheduler loop (Sec. 3.2 sliding calibration
+// window, Sec. 3.3 dispatch and local order, Algorithm 1's round-robin
+// fallback, App. A Eq. admission) with all state resident on the device.
+//
+// Per batch of arrivals, in the paper's order:
+//   1. advance every running request by the steps since the last batch; a
+//      request completes on reaching its true length      (stream_advance)
+//   2. completions enter the calibration window in (completion step, id)
+//      order: maps_order_local sorts them, stream_window writes the ring
+//   3. calibrate on the window and bound every request in the system and the
+//      batch (maps_calibrate); an unbounded quantile sends the batch round
+//      robin                                                (stream_rr)
+//   4. group running and waiting requests by decoder      (stream_csr)
+//   5. project occupancy and dispatch the batch SEQUENTIALly with Q = the
+//      waiting counts (maps_project_occupancy, maps_dispatch)
+//   6. the batch joins its decoders' waiting queues        (stream_enqueue)
+//   7. local order of every waiting queue (stream_waitlist, maps_order_local)
+//   8. admission in queue order while used + p + U <= capacity, the first
+//      misfit blocking its queue                            (stream_admit)
+// The host issues the launches; it reads 24 bytes of loop state once per
+// batch (the request, completion and waiting counts that size the calls).
+#include <algorithm>
+
+#include "maps_internal.cuh"
+
+namespace maps {
+namespace {
+
+constexpr int kSt = 1024;  // threads of the one-block kernels
+constexpr int kStWarps = kSt / 32;
+constexpr int kStreamMaxD = 1024;
+enum : uint8_t { kNotYet = 0, kWaiting = 1, kRunning = 2, kDone = 3 };
+
+struct StreamState {
+  long long prev_s;  // dispatch step of the previous batch
+  int32_t nact;      // requests in the system (waiting or running)
+  int32_t ndone;     // completions found by the last advance
+  int32_t nwait;     // waiting requests after the last advance
+  int32_t pad;
+};
+
+// Exclusive position of a 0/1 flag across the block (kSt threads) and the
+// block's total.  Every thread must call it.
+__device__ __forceinline__ int block_flag_scan(bool f, int *s_w, int &total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const unsigned m = __ballot_sync(0xffffffffu, f);
+  if (lane == 0) s_w[warp] = __popc(m);
+  __syncthreads();
+  int base = 0, tot = 0;
+#pragma unroll 8
+  for (int w = 0; w < kStWarps; ++w) {
+    const int c = s_w[w];
+    base += w < warp ? c : 0;
+    tot += c;
+  }
+  __syncthreads();
+  total = tot;
+  return base + __popc(m & ((1u << lane) - 1u));
+}
+
+__global__ void stream_validate_kernel(int64_t N, const int64_t *arrival, const int32_t *prompt,
+                                       const int32_t *true_len, const int32_t *pred,
+                                       int32_t *status) {
+  bool bad = false;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < N; i += stride)
+    if (prompt[i] < 0 || true_len[i] < 1 || pred[i] < 0 || (i > 0 && arrival[i] < arrival[i - 1]))
+      bad = true;
+  if (bad) flag_error(status, MAPS_E_RANGE);
+}
+
+__global__ void stream_init_kernel(int64_t first_hi, int D, int32_t cap, const int64_t *arrival,
+                                   int32_t *capv, StreamState *S) {
+  for (int k = threadIdx.x; k < D; k += blockDim.x) capv[k] = cap;
+  if (threadIdx.x == 0) {
+    S->prev_s = arrival[first_hi - 1];
+    S->nact = 0;
+    S->ndone = 0;
+    S->nwait = 0;
+  }
+}
+
+// 1. Advance by delta = s - prev_s steps; keep the survivors in id order.
+__global__ void __launch_bounds__(kSt, 1)
+stream_advance_kernel(int64_t hi, int D, int32_t cap, const int64_t *arrival,
+                      const int32_t *prompt, const int32_t *true_len, uint8_t *st, int32_t *g,
+                      const int32_t *dec, const int32_t *act_in, int32_t *act_out,
+                      int32_t *done_id, int32_t *done_rem, long long *used, StreamState *S,
+                      int64_t *stats_b) {
+  __shared__ unsigned long long s_used[kStreamMaxD];
+  __shared__ int s_w[kStWarps];
+  __shared__ int s_nwait;
+  const int tid = threadIdx.x;
+  for (int k = tid; k < D; k += kSt) s_used[k] = 0;
+  if (tid == 0) s_nwait = 0;
+  const long long s = arrival[hi - 1];
+  const long long delta = s - S->prev_s;
+  const int nact = S->nact;
+  __syncthreads();
+  int nkeep = 0, ndone = 0, nwait = 0;
+  for (int c0 = 0; c0 < nact; c0 += kSt) {
+    const int x = c0 + tid;
+    int id = -1, rem32 = 0;
+    bool done = false;
+    if (x < nact) {
+      id = act_in[x];
+      const uint8_t sv = st[id];
+      if (sv == kRunning) {
+        const long long rem = static_cast<long long>(true_len[id]) - g[id];  // >= 1
+        if (rem <= delta) {
+          done = true;
+          rem32 = static_cast<int>(rem);
+          st[id] = kDone;
+        } else {
+          const int gn = g[id] + static_cast<int>(delta);  // < true_len
+          g[id] = gn;
+          atomicAdd(&s_used[dec[id]],
+                    static_cast<unsigned long long>(static_cast<long long>(prompt[id]) + gn));
+        }
+      } else if (sv == kWaiting) {
+        ++nwait;
+      }
+    }
+    int tk, td;
+    const int pk = block_flag_scan(id >= 0 && !done, s_w, tk);
+    const int pd = block_flag_scan(done, s_w, td);
+    if (id >= 0 && !done) act_out[nkeep + pk] = id;
+    if (done) {
+      done_id[ndone + pd] = id;
+      done_rem[ndone + pd] = rem32;
+    }
+    nkeep += tk;
+    ndone += td;
+  }
+  if (nwait) atomicAdd(&s_nwait, nwait);
+  const bool ov = tid < D && static_cast<long long>(s_used[tid]) > cap;  // D <= kSt
+  if (tid < D) used[tid] = static_cast<long long>(s_used[tid]);
+  const int over = __syncthreads_count(ov);
+  if (tid == 0) {
+    S->prev_s = s;
+    S->nact = nkeep;
+    S->ndone = ndone;
+    S->nwait = s_nwait;
+    stats_b[0] = ndone;
+    stats_b[3] = over;
+  }
+}
+
+// 2. Completions, sorted by (step, id), enter the ring of the last Wn; the
+//    c-th completion ever goes to slot c mod Wn.
+__global__ void stream_window_kernel(int ndone, long long c0, int Wn, const int32_t *perm,
+                                     const int32_t *done_id, const int32_t *true_len,
+                                     const int32_t *pred, int32_t *win_true, int32_t *win_pred) {
+  const int stride = gridDim.x * blockDim.x;
+  for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < ndone; x += stride) {
+    if (x < ndone - Wn) continue;  // overwritten by a later completion of this batch
+    const int id = done_id[perm[x]];
+    const int slot = static_cast<int>((c0 + x) % Wn);
+    win_true[slot] = true_len[id];
+    win_pred[slot] = pred[id];
+  }
+}
+
+// 3. Predictions of the requests in the system, then of the batch.
+__global__ void stream_gather_kernel(int nact, int nb, int64_t lo, const int32_t *act,
+                                     const int32_t *pred, int32_t *qpred) {
+  const int stride = gridDim.x * blockDim.x;
+  for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < nact + nb; x += stride)
+    qpred[x] = x < nact ? pred[act[x]] : pred[lo + (x - nact)];
+}
+
+// 3'. No bound available: U = prediction, the batch goes round robin.
+__global__ void stream_rr_kernel(int n, int nb, int64_t lo, int D, const int32_t *qpred,
+                                 int32_t *Uq, int32_t *choice) {
+  const int stride = gridDim.x * blockDim.x;
+  for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
+    Uq[x] = qpred[x];
+    if (x < nb) choice[lo + x] = static_cast<int32_t>((lo + x) % D);
+  }
+}
+
+// 4. Residents by decoder (running with g, waiting with g = 0) and the
+//    waiting count per decoder; new bounds of the requests in the system.
+__global__ void __launch_bounds__(kSt, 1)
+stream_csr_kernel(int nact, int D, int rr, const int32_t *q_dev, int32_t *q_out_b,
+                  const int32_t *act, const uint8_t *st, const int32_t *g, const int32_t *dec,
+                  const int32_t *prompt, const int32_t *Uq, int32_t *U, int64_t *res_off,
+                  int32_t *rp, int32_t *rg, int32_t *rU, int32_t *Q) {
+  __shared__ int s_cnt[kStreamMaxD], s_q[kStreamMaxD], s_cur[kStreamMaxD];
+  __shared__ int s_w[kStWarps];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int k = tid; k < D; k += kSt) s_cnt[k] = s_q[k] = 0;
+  __syncthreads();
+  for (int x = tid; x < nact; x += kSt) {
+    const int id = act[x];
+    U[id] = Uq[x];
+    atomicAdd(&s_cnt[dec[id]], 1);
+    if (st[id] == kWaiting) atomicAdd(&s_q[dec[id]], 1);
+  }
+  __syncthreads();
+  const int c = tid < D ? s_cnt[tid] : 0;  // D <= kSt
+  int incl = c;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += y;
+  }
+  if (lane == 31) s_w[warp] = incl;
+  __syncthreads();
+  int base = 0;
+  for (int w = 0; w < warp; ++w) base += s_w[w];
+  if (tid < D) {
+    const int ex = base + incl - c;
+    s_cur[tid] = ex;
+    res_off[tid] = ex;
+    Q[tid] = s_q[tid];
+    if (tid == D - 1) res_off[D] = ex + c;
+  }
+  __syncthreads();
+  for (int x = tid; x < nact; x += kSt) {
+    const int id = act[x];
+    const int pos = atomicAdd(&s_cur[dec[id]], 1);
+    rp[pos] = prompt[id];
+    rg[pos] = st[id] == kRunning ? g[id] : 0;
+    rU[pos] = Uq[x];
+  }
+  if (tid == 0) *q_out_b = rr ? -1 : q_dev[0];
+}
+
+// 6. The batch joins the waiting queues of its decoders.
+__global__ void stream_enqueue_kernel(int64_t lo, int nb, int nact, int64_t hi, int D,
+                                      const int64_t *arrival, const int32_t *choice,
+                                      const int32_t *Uq, uint8_t *st, int32_t *dec,
+                                      long long *disp, int32_t *g, int32_t *U, int32_t *act,
+                                      StreamState *S, int32_t *status) {
+  const long long s = arrival[hi - 1];
+  const int stride = gridDim.x * blockDim.x;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
+    const int64_t id = lo + i;
+    int c = choice[id];
+    if (c < 0 || c >= D) {  // only after a range error (a bound that overflowed)
+      flag_error(status, MAPS_E_RANGE);
+      c = 0;
+    }
+    st[id] = kWaiting;
+    dec[id] = c;
+    disp[id] = s;
+    g[id] = 0;
+    U[id] = Uq[nact + i];
+    act[nact + i] = static_cast<int32_t>(id);
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) S->nact = nact + nb;
+}
+
+// 7. The waiting requests with their order keys.
+__global__ void __launch_bounds__(kSt, 1)
+stream_waitlist_kernel(int n, int64_t hi, const int64_t *arrival, const int32_t *act,
+                       const uint8_t *st, const int32_t *dec, const int32_t *U,
+                       const long long *disp, int32_t *wid, int32_t *wdec, int32_t *wU,
+                       int32_t *wwait, int32_t *warr) {
+  __shared__ int s_w[kStWarps];
+  const long long s = arrival[hi - 1];
+  int nw = 0;
+  for (int c0 = 0; c0 < n; c0 += kSt) {
+    const int x = c0 + threadIdx.x;
+    const int id = x < n ? act[x] : -1;
+    const bool f = id >= 0 && st[id] == kWaiting;
+    int tot;
+    const int pos = block_flag_scan(f, s_w, tot);
+    if (f) {
+      const int o = nw + pos;
+      const long long w = s - disp[id];
+      wid[o] = id;
+      wdec[o] = dec[id];
+      wU[o] = U[id];
+      wwait[o] = static_cast<int32_t>(w > 0x7fffffffLL ? 0x7fffffffLL : w);
+      warr[o] = id;
+    }
+    nw += tot;
+  }
+}
+
+// 8. Admission, one warp per decoder: entry x of the queue is admitted while
+//    it and every entry before it satisfy used + (prompts admitted before) +
+//    p + U <= cap.
+__global__ void __launch_bounds__(kSt, 1)
+stream_admit_kernel(int D, int32_t cap, int nw, const int64_t *wseg, const int32_t *wperm,
+                    const int32_t *wid, const int32_t *prompt, const int32_t *U,
+                    const long long *used, uint8_t *st, int32_t *g, int64_t *stats_b) {
+  __shared__ int s_adm;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) s_adm = 0;
+  __syncthreads();
+  for (int k = warp; k < D; k += kStWarps) {
+    long long u = used[k];
+    const long long x1 = wseg[k + 1];
+    int adm = 0;
+    bool stop = false;
+    for (long long b0 = wseg[k]; b0 < x1 && !stop; b0 += 32) {
+      const long long x = b0 + lane;
+      const bool valid = x < x1;
+      const int id = valid ? wid[wperm[x]] : -1;
+      const long long p = valid ? prompt[id] : 0, uu = valid ? U[id] : 0;
+      long long incl = p;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const long long y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+      }
+      const bool ok = valid && u + (incl - p) + p + uu <= cap;
+      const unsigned fail = __ballot_sync(0xffffffffu, valid && !ok);
+      const unsigned vmask = __ballot_sync(0xffffffffu, valid);
+      const int nadm = fail ? __ffs(fail) - 1 : __popc(vmask);
+      if (lane < nadm) {
+        st[id] = kRunning;
+        g[id] = 0;
+      }
+      if (nadm > 0) u += __shfl_sync(0xffffffffu, incl, nadm - 1);
+      adm += nadm;
+      stop = fail != 0;
+    }
+    if (lane == 0 && adm) atomicAdd(&s_adm, adm);
+  }
+  __syncthreads();
+  if (tid == 0) {
+    stats_b[1] = s_adm;
+    stats_b[2] = nw - s_adm;
+  }
+}
+
+struct StreamWs {
+  size_t sub_bytes;  // [0, sub_bytes): workspace of the calls the loop makes
+  StreamState *S;
+  uint8_t *st;
+  int32_t *g, *dec, *U;
+  long long *disp;
+  int32_t *act[2];
+  int32_t *done_id, *done_rem, *done_perm, *zeros;
+  int64_t *done_seg;
+  int32_t *win_true, *win_pred, *qpred, *Uq;
+  int64_t *res_off;
+  int32_t *rp, *rg, *rU, *capv, *Q;
+  long long *used;
+  int32_t *K;
+  int64_t *headroom;
+  int32_t *wid, *wdec, *wU, *wwait, *warr, *wperm;
+  int64_t *wseg;
+  int32_t *q_dev;
+};
+
+size_t stream_sub_bytes(const maps_stream_cfg &c) {
+  size_t b = maps_calibrate_workspace_size(c.window, c.N);
+  b = std::max(b, maps_project_occupancy_workspace_size(c.D, c.H, c.N));
+  b = std::max(b, maps_dispatch_workspace_size(MAPS_MODE_SEQUENTIAL, c.D, c.H, c.batch));
+  b = std::max(b, maps_order_local_workspace_size(c.N, c.D));
+  b = std::max(b, maps_order_local_workspace_size(c.N, 1));
+  return (b + kAlign - 1) / kAlign * kAlign;
+}
+
+StreamWs carve_stream(Carve &c, const maps_stream_cfg &cfg) {
+  StreamWs w;
+  const size_t N = static_cast<size_t>(cfg.N), D = static_cast<size_t>(cfg.D);
+  w.sub_bytes = stream_sub_bytes(cfg);
+  c.off = w.sub_bytes;
+  w.S = c.take<StreamState>(1);
+  w.st = c.take<uint8_t>(N);
+  w.g = c.take<int32_t>(N);
+  w.dec = c.take<int32_t>(N);
+  w.U = c.take<int32_t>(N);
+  w.disp = c.take<long long>(N);
+  w.act[0] = c.take<int32_t>(N);
+  w.act[1] = c.take<int32_t>(N);
+  w.done_id = c.take<int32_t>(N);
+  w.done_rem = c.take<int32_t>(N);
+  w.done_perm = c.take<int32_t>(N);
+  w.zeros = c.take<int32_t>(N);
+  w.done_seg = c.take<int64_t>(2);
+  w.win_true = c.take<int32_t>(static_cast<size_t>(cfg.window));
+  w.win_pred = c.take<int32_t>(static_cast<size_t>(cfg.window));
+  w.qpred = c.take<int32_t>(N);
+  w.Uq = c.take<int32_t>(N);
+  w.res_off = c.take<int64_t>(D + 1);
+  w.rp = c.take<int32_t>(N);
+  w.rg = c.take<int32_t>(N);
+  w.rU = c.take<int32_t>(N);
+  w.capv = c.take<int32_t>(D);
+  w.Q = c.take<int32_t>(D);
+  w.used = c.take<long long>(D);
+  w.K = c.take<int32_t>(D * static_cast<size_t>(cfg.H));
+  w.headroom = c.take<int64_t>(static_cast<size_t>(cfg.batch));
+  w.wid = c.take<int32_t>(N);
+  w.wdec = c.take<int32_t>(N);
+  w.wU = c.take<int32_t>(N);
+  w.wwait = c.take<int32_t>(N);
+  w.warr = c.take<int32_t>(N);
+  w.wperm = c.take<int32_t>(N);
+  w.wseg = c.take<int64_t>(D + 1);
+  w.q_dev = c.take<int32_t>(1);
+  return w;
+}
+
+bool cfg_ok(const maps_stream_cfg *c) {
+  return c != nullptr && c->N >= 1 && c->N <= 0x7fffffffLL && c->D >= 1 && c->D <= kStreamMaxD &&
+         c->H >= 1 && c->H <= (1 << 28) && c->cap >= 0 && c->batch >= 1 && c->window >= 1 &&
+         c->alpha_ppm > 0 && c->alpha_ppm < 1000000u;
+}
+
+int grid_for(int64_t n, int threads = 256) {
+  return static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((n + threads - 1) / threads,
+                                                                 4LL * sm_count())));
+}
+
+}  // namespace
+}  // namespace maps
+
+extern "C" {
+
+size_t maps_stream_workspace_size(const maps_stream_cfg *cfg) {
+  using namespace maps;
+  if (!cfg_ok(cfg)) return kCtrlBytes;
+  Carve c(nullptr);
+  carve_stream(c, *cfg);
+  return c.bytes();
+}
+
+int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const int32_t *prompt,
+                    const int32_t *true_len, const int32_t *pred, int32_t *choice_out,
+                    int32_t *q_out, int64_t *stats_out, void *ws, size_t ws_bytes, void *stream) {
+  using namespace maps;
+  if (!cfg_ok(cfg) || arrival_ms == nullptr || prompt == nullptr || true_len == nullptr ||
+      pred == nullptr || choice_out == nullptr || q_out == nullptr || stats_out == nullptr)
+    return MAPS_E_INVALID;
+  MAPS_TRY(check_ws(ws, ws_bytes, maps_stream_workspace_size(cfg)));
+  const maps_stream_cfg c = *cfg;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int32_t *status = status_word(ws);
+  Carve cv(ws);
+  const StreamWs w = carve_stream(cv, c);
+  const int64_t N = c.N, B = c.batch, nbatch = (N + B - 1) / B;
+  const int D = c.D;
+
+  MAPS_TRY(cuda_ok(cudaMemsetAsync(w.st, 0, static_cast<size_t>(N), s)));
+  MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zeros, 0, static_cast<size_t>(N) * sizeof(int32_t), s)));
+  stream_init_kernel<<<1, kSt, 0, s>>>(std::min(N, B), D, c.cap, arrival_ms, w.capv, w.S);
+  stream_validate_kernel<<<grid_for(N), 256, 0, s>>>(N, arrival_ms, prompt, true_len, pred, status);
+  MAPS_TRY(launch_ok());
+  {
+    const int st0 = maps_check(ws, stream);  // a bad input stops the loop before it starts
+    if (st0 != MAPS_OK) return st0;
+  }
+
+  long long total_done = 0;
+  StreamState hs;
+  for (int64_t b = 0; b < nbatch; ++b) {
+    const int64_t lo = b * B, hi = std::min(lo + B, N);
+    const int nb = static_cast<int>(hi - lo);
+    int32_t *act_in = w.act[b & 1], *act = w.act[(b & 1) ^ 1];
+    int64_t *stats_b = stats_out + 4 * b;
+    stream_advance_kernel<<<1, kSt, 0, s>>>(hi, D, c.cap, arrival_ms, prompt, true_len, w.st, w.g,
+                                            w.dec, act_in, act, w.done_id, w.done_rem, w.used, w.S,
+                                            stats_b);
+    MAPS_TRY(launch_ok());
+    MAPS_TRY(cuda_ok(cudaMemcpyAsync(&hs, w.S, sizeof(hs), cudaMemcpyDeviceToHost, s)));
+    MAPS_TRY(cuda_ok(cudaStreamSynchronize(s)));
+    const int nact = hs.nact, ndone = hs.ndone, nwait = hs.nwait;
+
+    if (ndone > 0) {  // 2.
+      MAPS_TRY(maps_order_local(ndone, 1, w.zeros, w.done_rem, w.zeros, w.done_id, 0, w.done_perm,
+                                w.done_seg, ws, w.sub_bytes, stream));
+      stream_window_kernel<<<grid_for(ndone), 256, 0, s>>>(ndone, total_done, c.window,
+                                                           w.done_perm, w.done_id, true_len, pred,
+                                                           w.win_true, w.win_pred);
+      total_done += ndone;
+    }
+    const int64_t win_len = std::min<long long>(total_done, c.window);
+
+    stream_gather_kernel<<<grid_for(nact + nb), 256, 0, s>>>(nact, nb, lo, act, pred, w.qpred);
+    const int cs = maps_calibrate(w.win_true, w.win_pred, win_len, c.alpha_ppm, w.qpred, nact + nb,
+                                  w.Uq, w.q_dev, nullptr, ws, w.sub_bytes, stream);  // 3.
+    const bool rr = cs == MAPS_E_UNBOUNDED;
+    if (cs != MAPS_OK && !rr) return cs;
+    if (rr)
+      stream_rr_kernel<<<grid_for(nact + nb), 256, 0, s>>>(nact + nb, nb, lo, D, w.qpred, w.Uq,
+                                                           choice_out);
+    stream_csr_kernel<<<1, kSt, 0, s>>>(nact, D, rr ? 1 : 0, w.q_dev, q_out + b, act, w.st, w.g,
+                                        w.dec, prompt, w.Uq, w.U, w.res_off, w.rp, w.rg, w.rU,
+                                        w.Q);  // 4.
+    MAPS_TRY(launch_ok());
+    if (!rr) {  // 5.
+      MAPS_TRY(maps_project_occupancy(D, c.H, w.res_off, nact, w.rp, w.rg, w.rU, w.K, nullptr, ws,
+                                      w.sub_bytes, stream));
+      MAPS_TRY(maps_dispatch(MAPS_MODE_SEQUENTIAL, D, c.H, 1, w.K, nullptr, w.capv, w.Q, nullptr, 0,
+                             nullptr, nullptr, nullptr, nb, prompt + lo, w.Uq + nact,
+                             choice_out + lo, w.headroom, ws, w.sub_bytes, stream));
+    }
+    stream_enqueue_kernel<<<grid_for(nb), 256, 0, s>>>(lo, nb, nact, hi, D, arrival_ms,
+                                                       choice_out, w.Uq, w.st, w.dec, w.disp, w.g,
+                                                       w.U, act, w.S, status);  // 6.
+    const int n_all = nact + nb, nw = nwait + nb;
+    stream_waitlist_kernel<<<1, kSt, 0, s>>>(n_all, hi, arrival_ms, act, w.st, w.dec, w.U, w.disp,
+                                             w.wid, w.wdec, w.wU, w.wwait, w.warr);  // 7.
+    MAPS_TRY(launch_ok());
+    MAPS_TRY(maps_order_local(nw, D, w.wdec, w.wU, w.wwait, w.warr, c.max_wait, w.wperm, w.wseg, ws,
+                              w.sub_bytes, stream));
+    stream_admit_kernel<<<1, kSt, 0, s>>>(D, c.cap, nw, w.wseg, w.wperm, w.wid, prompt, w.U, w.used,
+                                          w.st, w.g, stats_b);  // 8.
+    MAPS_TRY(launch_ok());
+  }
+  return maps_check(ws, stream);
+}
+
+}  // extern "C"

@@ -33,6 +33,13 @@ STATUS_NAMES = {0: "MAPS_OK", -1: "MAPS_E_INVALID", -2: "MAPS_E_RANGE",
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmaps.so")
 
 
+class StreamCfg(ctypes.Structure):
+    """``maps_stream_cfg`` of include/maps.h."""
+    _fields_ = [("N", ctypes.c_int64), ("D", ctypes.c_int32), ("H", ctypes.c_int32),
+                ("cap", ctypes.c_int32), ("batch", ctypes.c_int32), ("window", ctypes.c_int32),
+                ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32)]
+
+
 class MapsError(RuntimeError):
     def __init__(self, status: int, what: str = ""):
         super().__init__(f"{what}: {STATUS_NAMES.get(status, status)}")
@@ -61,6 +68,9 @@ def _load():
         "maps_order_local_workspace_size": ([i64, i32], sz),
         "maps_order_local": ([i64, i32, vp, vp, vp, vp, i32, vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_order_local_static": ([i64, i32, vp, vp, vp, vp, i32, vp, vp, vp, vp], ctypes.c_int),
+        "maps_stream_workspace_size": ([ctypes.POINTER(StreamCfg)], sz),
+        "maps_stream_run": ([ctypes.POINTER(StreamCfg), vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
+                            ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -74,7 +84,8 @@ EXPORTS = ("maps_version", "maps_last_cuda_error", "maps_check",
            "maps_calibrate_workspace_size", "maps_calibrate",
            "maps_project_occupancy_workspace_size", "maps_project_occupancy",
            "maps_dispatch_workspace_size", "maps_dispatch",
-           "maps_order_local_workspace_size", "maps_order_local", "maps_order_local_static")
+           "maps_order_local_workspace_size", "maps_order_local", "maps_order_local_static",
+           "maps_stream_workspace_size", "maps_stream_run")
 
 
 def _stream(stream) -> ctypes.c_void_p:
@@ -194,3 +205,21 @@ def maps_order_local_static(D: int, dec, bound, wait, arrival, max_wait: int, pe
                                        _ptr(seg_off_out, torch.int64),
                                        ctypes.byref(st) if sync_status else None,
                                        _stream(stream))
+
+
+def stream_cfg(N: int, D: int, H: int, cap: int, batch: int, window: int, alpha_ppm: int,
+               max_wait: int) -> StreamCfg:
+    return StreamCfg(int(N), int(D), int(H), int(cap), int(batch), int(window), int(alpha_ppm),
+                     int(max_wait))
+
+
+def maps_stream_run(cfg: StreamCfg, arrival_ms, prompt, true_len, pred, choice_out, q_out,
+                    stats_out, ws: Workspace | None = None, stream=None) -> int:
+    """The whole streaming loop on the device; returns the full status."""
+    ws = ws or Workspace()
+    ws.ensure(lib.maps_stream_workspace_size(ctypes.byref(cfg)))
+    return lib.maps_stream_run(ctypes.byref(cfg), _ptr(arrival_ms, torch.int64),
+                               _ptr(prompt, torch.int32), _ptr(true_len, torch.int32),
+                               _ptr(pred, torch.int32), _ptr(choice_out, torch.int32),
+                               _ptr(q_out, torch.int32), _ptr(stats_out, torch.int64),
+                               ws.ptr, ws.nbytes, _stream(stream))

@@ -501,3 +501,64 @@ def test_repeat_runs_identical(M, ws, oracle):
         outs.append((K, ch, hr))
     for o in outs[1:]:
         assert all(np.array_equal(x, y) for x, y in zip(o, outs[0]))
+
+
+# ---------------------------------------------------------------------------
+# streaming loop
+# ---------------------------------------------------------------------------
+
+def gpu_stream(M, ws, N, D, H, cap, B, Wn, a, mw, arrival, prompt, true, pred):
+    nb = (N + B - 1) // B
+    ch = torch.full((N,), -9, dtype=torch.int32, device="cuda")
+    q = torch.full((nb,), -9, dtype=torch.int32, device="cuda")
+    stats = torch.full((nb, 4), -9, dtype=torch.int64, device="cuda")
+    cfg = M.stream_cfg(N, D, H, cap, B, Wn, a, mw)
+    st = M.maps_stream_run(cfg, dev(arrival[:N], np.int64), dev(prompt[:N], np.int32),
+                           dev(true[:N], np.int32), dev(pred[:N], np.int32), ch, q, stats, ws=ws)
+    return st, host(ch), host(q), host(stats)
+
+
+def check_stream(M, ws, oracle, N, D, H, cap, B, Wn, a, mw, w):
+    args = (N, D, H, cap, B, Wn, a, mw, w["arrival_ms"], w["prompt"], w["true"], w["pred"])
+    sto, cho, qo, so = oracle.stream(*args)
+    st, ch, q, s = gpu_stream(M, ws, *args)
+    assert st == sto
+    if st == 0:
+        assert np.array_equal(q, qo)
+        assert np.array_equal(s, so)
+        assert np.array_equal(ch, cho)
+    return qo, so
+
+
+def test_stream_golden(M, ws, stream_golden):
+    c, r = stream_golden["config"], stream_golden["requests"]
+    st, ch, q, s = gpu_stream(M, ws, c["N"], c["D"], c["H"], c["cap"], c["batch"], c["window"],
+                              c["alpha_ppm"], c["max_wait"], np.array(r["arrival_ms"]),
+                              np.array(r["prompt"]), np.array(r["true_len"]), np.array(r["pred"]))
+    assert st == 0
+    assert ch.tolist() == stream_golden["choice"]
+    assert q.tolist() == stream_golden["q"]
+    assert s.tolist() == stream_golden["stats"]
+
+
+@pytest.mark.parametrize("N,D,H,cap,B,Wn,a,mw", [
+    (1, 32, 16384, 262144, 256, 500, 100000, 1000),       # one request, round robin
+    (300, 32, 16384, 262144, 256, 500, 100000, 1000),     # ragged last batch
+    (20000, 32, 16384, 262144, 256, 500, 100000, 1000),   # the streaming workload's prefix
+    (20000, 4, 4096, 12000, 256, 500, 100000, 1000),      # queues back up and block
+    (20000, 3, 2048, 9000, 100, 37, 300000, 50),          # promotions, small window
+    (5000, 5, 1000, 20000, 33, 7, 500000, 0),             # horizon below many bounds
+])
+def test_stream_prefix(M, ws, oracle, N, D, H, cap, B, Wn, a, mw):
+    w = W.make_stream(n_requests=N)
+    qo, so = check_stream(M, ws, oracle, N, D, H, cap, B, Wn, a, mw, w)
+    assert (qo >= 0).any() or N < 1000
+
+
+def test_stream_full_workload(M, ws, oracle):
+    """All 1,000,000 requests of the streaming workload, bit for bit."""
+    w = W.make_stream()
+    c = W.WORKLOADS["stream"]
+    qo, so = check_stream(M, ws, oracle, w["N"], w["D"], w["H"], w["cap"], w["batch"],
+                          w["window"], w["alpha_ppm"], w["max_wait"], w)
+    assert len(qo) == (w["N"] + c["batch"] - 1) // c["batch"]
