@@ -46,13 +46,33 @@ UNIT = "decisions/s"
 WORKLOAD = "large"
 L2_FLUSH_BYTES = 256 << 20
 
-# DRAM traffic of the occupancy kernel on this workload from an ncu capture
-# (dram__bytes_read.sum + dram__bytes_write.sum, one launch), valid only for
-# the kernel source it was taken on.
+# DRAM traffic per call on this workload from an ncu capture
+# (dram__bytes_read.sum + dram__bytes_write.sum summed over the call's
+# kernels, one launch each), valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "occupancy": {"bytes": None, "source_sha256": None,
-                  "profile": "profiles/occupancy_large.md"},
+    "calibrate": {"bytes": 28_590_000, "source": "calibrate.cu", "source_sha256":
+                  "6ec8bc77c9905f1af3141b12009fd86baae3ffe17558a3c0de8269a58b9d0526"},
+    "occupancy": {"bytes": 33_340_000, "source": "occupancy.cu", "source_sha256":
+                  "3e4f278da7bdb6fe20c9cb07522c6deaaf45cda7ebeb264a7f3c2e8379339b75"},
+    "dispatch": {"bytes": 26_430_000, "source": "dispatch.cu", "source_sha256":
+                 "e14c618e37ab801c0680186b4ba30477e3352cfc88b8e4f3f499d40ba265f22c"},
+    "order": {"bytes": 72_640_000, "source": "order.cu", "source_sha256":
+              "9614d5b5eb08039bdfe4f5a1b3e6d5d7dca3b624bc9055ed51660c7d00c87040"},
 }
+KERNELS = {
+    "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
+    "occupancy": "occ_bucket_kernel + occ_tile_kernel (maps_project_occupancy)",
+    "dispatch": "carry_scan + bin_count/scan/scatter + dispatch_snapshot_kernel (maps_dispatch)",
+    "order": "order_prep/keys/plan + order_pass_kernel x active digits (maps_order_local)",
+}
+
+
+def traffic_for(call: str):
+    t = TRAFFIC[call]
+    src = os.path.join(ROOT, "paper_2609_15359_gb300", "csrc", t["source"])
+    if t["bytes"] and os.path.exists(src) and t["source_sha256"] == _sha256(src):
+        return t["bytes"]
+    return None
 
 
 def _sha256(path: str) -> str:
@@ -340,14 +360,23 @@ def bench_gpu(args, world, rank, local, dist):
 
     peaks = measured_peaks()
     D, H, R, J = step.D, step.H, step.R, step.J
-    occ_bytes = 12 * R + 4 * D * H + 8 * (D + 1)  # residents in, K out, offsets
-    occ_avg = float(np.mean(occ_ms)) / 1e3
-    achieved = occ_bytes / occ_avg / 1e9
-    tr = TRAFFIC["occupancy"]
-    occ_src = os.path.join(ROOT, "paper_2609_15359_gb300", "csrc", "occupancy.cu")
-    traffic = tr["bytes"] if (tr["bytes"] and tr["source_sha256"] == _sha256(occ_src)) else None
-    disp_bytes = 4 * D * H + 8 * J + 12 * J + 8 * D  # K, candidates, choice+headroom, cap+Q
-    disp_avg = float(np.mean(disp_ms)) / 1e3
+    # algorithmic bytes per call (what the method must move)
+    alg = {
+        "calibrate": 8 * w["n_cal"] + 8 * (R + J),     # residual pairs in; predictions in, bounds out
+        "occupancy": 12 * R + 4 * D * H + 8 * (D + 1),  # residents in, K out, offsets
+        "dispatch": 4 * D * H + 8 * J + 12 * J + 8 * D,  # K, candidates, choice + headroom, cap + Q
+        "order": 20 * (R + J) + 8 * (D + 1),           # four int32 keys in, perm out, segments
+    }
+    call_ms = {"calibrate": cal_ms, "occupancy": occ_ms, "dispatch": disp_ms, "order": order_ms}
+    rooflines = {}
+    for c in alg:
+        avg = float(np.mean(call_ms[c])) / 1e3
+        a = alg[c] / avg / 1e9
+        rooflines[c] = {"kernel": KERNELS[c], "bound": "hbm", "achieved": a,
+                        "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": a / peaks["hbm_gbs"],
+                        "traffic": traffic_for(c), "algorithmic_bytes": alg[c],
+                        "ms": avg * 1e3, "peak_source": peaks["source"]}
+    dominant = max(rooflines, key=lambda c: rooflines[c]["ms"])
     ms_per_step = max_s / K * 1e3
     result = {
         "metric": METRIC,
@@ -373,21 +402,66 @@ def bench_gpu(args, world, rank, local, dist):
         "occupancy_cells_per_s": K * D * H * world / max_s,
         "kernels_ms": {"calibrate": float(np.mean(cal_ms)), "occupancy": float(np.mean(occ_ms)),
                        "dispatch": float(np.mean(disp_ms)), "order": float(np.mean(order_ms))},
-        "roofline": {"kernel": "occupancy_kernel (maps_project_occupancy)", "bound": "hbm",
-                     "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                     "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
-                     "algorithmic_bytes": occ_bytes, "peak_source": peaks["source"]},
-        "roofline_dispatch": {"scope": "whole maps_dispatch call (bucketing + main kernel)",
-                              "bound": "hbm", "achieved": disp_bytes / disp_avg / 1e9,
-                              "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                              "frac": disp_bytes / disp_avg / 1e9 / peaks["hbm_gbs"],
-                              "algorithmic_bytes": disp_bytes},
+        "roofline": dict(rooflines[dominant], call=dominant),
+        "rooflines": rooflines,
         "e2e": {"value": e2e_units / e2e_max, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": step.kernels_per_step * K,
         "clocks": clocks,
     }
     return result, w
+
+
+# ---------------------------------------------------------------------------
+# the streaming loop (all 1,000,000 requests through maps_stream_run)
+# ---------------------------------------------------------------------------
+
+def bench_stream(device, cpu_sample: int = 0) -> dict:
+    """Wall time of the whole streaming loop on the device (it synchronises
+    once per batch, so host time is the loop's time), after one warm-up run
+    on a 20,000-request prefix.  With cpu_sample > 0 the oracle is timed on
+    that many leading requests as the CPU reference."""
+    import torch
+    from paper_2609_15359_gb300 import maps as M
+    from paper_2609_15359_gb300 import workloads as W
+    w = W.make_stream()
+    t = lambda x, d: torch.from_numpy(np.ascontiguousarray(x, dtype=d)).to(device)  # noqa: E731
+    arr, pr, tr, pd = (t(w["arrival_ms"], np.int64), t(w["prompt"], np.int32),
+                       t(w["true"], np.int32), t(w["pred"], np.int32))
+    N, B = w["N"], w["batch"]
+    nb = (N + B - 1) // B
+    ch = torch.empty(N, dtype=torch.int32, device=device)
+    q = torch.empty(nb, dtype=torch.int32, device=device)
+    stats = torch.empty((nb, 4), dtype=torch.int64, device=device)
+    ws = M.Workspace(device=device)
+
+    def run(n):
+        cfg = M.stream_cfg(n, w["D"], w["H"], w["cap"], B, w["window"], w["alpha_ppm"],
+                           w["max_wait"])
+        st = M.maps_stream_run(cfg, arr[:n], pr[:n], tr[:n], pd[:n], ch[:n], q, stats, ws=ws)
+        if st != 0:
+            raise RuntimeError(f"maps_stream_run status {st}")
+
+    run(20000)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    run(N)
+    secs = time.perf_counter() - t0
+    out = {"workload": W.DESCRIPTIONS["stream"], "requests": N, "batches": nb,
+           "value": N / secs, "unit": "decisions/s", "seconds": secs,
+           "ms_per_batch": secs / nb * 1e3, "dispatch_mode": "SEQUENTIAL",
+           "timing": "host wall clock of one maps_stream_run call (it synchronises per batch)"}
+    if cpu_sample:
+        import oracle as O
+        n = min(cpu_sample, N)
+        t0 = time.perf_counter()
+        O.stream(n, w["D"], w["H"], w["cap"], B, w["window"], w["alpha_ppm"], w["max_wait"],
+                 w["arrival_ms"], w["prompt"], w["true"], w["pred"])
+        cs = time.perf_counter() - t0
+        out["cpu_baseline"] = {"value": n / cs, "unit": "decisions/s", "cores": 1,
+                               "kind": "oracle",
+                               "sample": f"the first {n} requests of the streaming workload"}
+    return out
 
 
 # ---------------------------------------------------------------------------
@@ -464,6 +538,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["maps", "reference"], default="maps")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-stream", action="store_true",
+                    help="skip the streaming-loop measurement")
     args = ap.parse_args()
     world, rank, local = dist_env()
 
@@ -488,6 +564,9 @@ def main():
     if rank == 0:
         if world == 1 and not args.no_cpu_baseline:
             res["cpu_baseline"] = cpu_baseline(w)
+        if world == 1 and not args.no_stream:
+            res["stream"] = bench_stream(torch.device(f"cuda:{local}"),
+                                         0 if args.no_cpu_baseline else 100000)
         print(json.dumps(res), flush=True)
     if dist is not None:
         dist.destroy_process_group()
