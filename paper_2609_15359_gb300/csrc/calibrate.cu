@@ -43,6 +43,7 @@ __global__ void __launch_bounds__(kSelectThreads)
 select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
                    int64_t n, unsigned long long k0, SelectState *st,
                    int32_t *q_dev_out, int32_t *status) {
+  pdl_prologue();
   constexpr int kShift = Digit<PASS>::shift;
   constexpr uint32_t kMask = (1u << Digit<PASS>::bits) - 1u;
   constexpr int kPrevShift = PASS == 0 ? 0 : Digit<(PASS > 0 ? PASS - 1 : 0)>::shift;
@@ -167,6 +168,7 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
 __global__ void __launch_bounds__(256)
 bound_kernel(const int32_t *__restrict__ pred, int64_t m, const SelectState *st,
              int32_t *__restrict__ out, int32_t *status) {
+  pdl_prologue();
   const long long q = *reinterpret_cast<const volatile int32_t *>(&st->q);
   const int64_t i4 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   const int64_t i = i4 * 4;
@@ -250,14 +252,14 @@ int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
   MAPS_TRY(cuda_ok(cudaMemsetAsync(st, 0, sizeof(SelectState), s)));
   const int g = grid_for(n, kSelectThreads * 16);
   const unsigned long long kk = static_cast<unsigned long long>(k);
-  select_pass_kernel<0><<<g, kSelectThreads, 0, s>>>(true_len, pred_len, n, kk, st, q_dev_out, status);
-  select_pass_kernel<1><<<g, kSelectThreads, 0, s>>>(true_len, pred_len, n, kk, st, q_dev_out, status);
-  select_pass_kernel<2><<<g, kSelectThreads, 0, s>>>(true_len, pred_len, n, kk, st, q_dev_out, status);
+  launch_pdl(select_pass_kernel<0>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
+  launch_pdl(select_pass_kernel<1>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
+  launch_pdl(select_pass_kernel<2>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
   MAPS_TRY(launch_ok());
   if (m > 0) {
     const int64_t gb = (m + 1023) / 1024;
     if (gb > 0x7fffffffLL) return MAPS_E_INVALID;
-    bound_kernel<<<static_cast<unsigned>(gb), 256, 0, s>>>(query_pred, m, st, bound_out, status);
+    launch_pdl(bound_kernel, static_cast<unsigned>(gb), 256, 0, s, query_pred, m, st, bound_out, status);
     MAPS_TRY(launch_ok());
   }
   if (q_host_out != nullptr) {

@@ -95,6 +95,7 @@ constexpr int kUnitCands = 4096;   // candidates per work unit of the main kerne
 __global__ void __launch_bounds__(256)
 kmax_from_K_kernel(int D, int H, const int32_t *__restrict__ K, uint32_t *__restrict__ kmax,
                    int32_t *status) {
+  pdl_prologue();
   const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
   const int64_t total = nb * D;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -125,6 +126,7 @@ kmax_from_K_kernel(int D, int H, const int32_t *__restrict__ K, uint32_t *__rest
 __global__ void __launch_bounds__(256)
 carry_scan_kernel(int D, int H, int W2, int T2, const uint32_t *__restrict__ kmax,
                   uint32_t *__restrict__ carry) {
+  pdl_prologue();
   __shared__ uint32_t s_w[8];
   constexpr int kPer = 16;
   const int k = blockIdx.x;
@@ -199,6 +201,7 @@ __global__ void __launch_bounds__(1024)
 bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ cp,
                  const int32_t *__restrict__ cb, uint32_t *tcount, int32_t *choice,
                  int64_t *headroom, int32_t *status) {
+  pdl_prologue();
   __shared__ uint32_t s_h[kBinSmem];
   const bool local = T2 <= kBinSmem;
   if (local)
@@ -247,6 +250,7 @@ __global__ void __launch_bounds__(1024)
 bin_scan_kernel(int T2, const uint32_t *tcount, uint32_t *toff, Unit *units, uint32_t *nunits,
                 int D, const int32_t *__restrict__ Q, const int32_t *__restrict__ cap,
                 int32_t *sig, int32_t *rank_of, int32_t *capq, int32_t *status) {
+  pdl_prologue();
   __shared__ uint32_t s_w[2][32];
   __shared__ uint32_t s_carry[2];
   __shared__ int32_t s_q[kMaxD];
@@ -327,6 +331,7 @@ __global__ void __launch_bounds__(1024)
 bin_scatter_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ cp,
                    const int32_t *__restrict__ cb, const uint32_t *toff, uint32_t *tcursor,
                    int32_t *ord, int32_t *sp, int32_t *su) {
+  pdl_prologue();
   __shared__ uint32_t s_h[kBinSmem];  // local counts, then local cursors
   __shared__ uint32_t s_b[kBinSmem];  // this block's base inside each bucket
   const bool local = T2 <= kBinSmem;
@@ -409,6 +414,7 @@ struct SnapArgs {
 template <int W2>
 __global__ void __launch_bounds__(kMainThreads, 3)
 dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
+  pdl_prologue();
   extern __shared__ __align__(1024) unsigned char smem[];
   const int unit = blockIdx.x;
   if (unit >= static_cast<int>(*a.nunits)) return;
@@ -694,6 +700,7 @@ __global__ void __launch_bounds__(1024, 1)
 dispatch_sequential_kernel(int D, int H, int32_t *K, uint32_t *kmax, const int32_t *cap,
                            int32_t *Q, int64_t J, const int32_t *cp, const int32_t *cb,
                            int32_t *choice, int64_t *headroom, int32_t *status) {
+  pdl_prologue();
   __shared__ uint32_t s_M[kMaxD];
   __shared__ Pick s_w[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
@@ -783,6 +790,7 @@ __global__ void __launch_bounds__(256)
 alg1_budget_kernel(int D, int S, const int64_t *res_off, int64_t R, const int32_t *prompt,
                    const int32_t *gen, const int32_t *bound, const int32_t *cap,
                    long long *B_eff, int32_t *status) {
+  pdl_prologue();
   __shared__ long long s_red[8];
   const int k = blockIdx.x;
   int64_t lo = res_off[k], hi = res_off[k + 1];
@@ -821,6 +829,7 @@ __global__ void __launch_bounds__(256)
 alg1_snapshot_kernel(int D, int S, const long long *B_eff, const int32_t *cap, const int32_t *Q,
                      int64_t J, const int32_t *cp, const int32_t *cb, int32_t *choice,
                      int64_t *headroom, int32_t *status) {
+  pdl_prologue();
   __shared__ long long s_B[kMaxD];
   __shared__ long long s_pm[kMaxD];
   __shared__ int s_sig[kMaxD];
@@ -923,6 +932,7 @@ __global__ void __launch_bounds__(1024, 1)
 alg1_sequential_kernel(int D, int S, long long *B_eff, const int32_t *cap, int32_t *Q, int64_t J,
                        const int32_t *cp, const int32_t *cb, int32_t *choice, int64_t *headroom,
                        int32_t *status) {
+  pdl_prologue();
   __shared__ long long s_B[kMaxD];
   __shared__ Pick s_w[32];
   const int tid = threadIdx.x;
@@ -1044,7 +1054,7 @@ int run_snapshot(int64_t grid, size_t smem, cudaStream_t s, const CUtensorMap &t
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(dispatch_snapshot_kernel<W2>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));
-  dispatch_snapshot_kernel<W2><<<static_cast<unsigned>(grid), kMainThreads, smem, s>>>(tmap, a);
+  launch_pdl(dispatch_snapshot_kernel<W2>, static_cast<unsigned>(grid), kMainThreads, smem, s, tmap, a);
   return launch_ok();
 }
 
@@ -1064,15 +1074,15 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
   if (kmax == nullptr) {
     const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
     const int gk = static_cast<int>(std::min<int64_t>((nb * D + 255) / 256, 8LL * sms));
-    kmax_from_K_kernel<<<gk, 256, 0, s>>>(D, H, K, w.kmax, status);
+    launch_pdl(kmax_from_K_kernel, gk, 256, 0, s, D, H, K, w.kmax, status);
     kmax = w.kmax;
   }
-  carry_scan_kernel<<<D, 256, 0, s>>>(D, H, g.W2, g.T2, kmax, w.carry);
+  launch_pdl(carry_scan_kernel, D, 256, 0, s, D, H, g.W2, g.T2, kmax, w.carry);
   const int gb = static_cast<int>(std::min<int64_t>((J + 1023) / 1024, 4LL * sms));
-  bin_count_kernel<<<gb, 1024, 0, s>>>(J, H, g.W2, g.T2, cp, cb, tcount, choice, headroom, status);
-  bin_scan_kernel<<<1, 1024, 0, s>>>(g.T2, tcount, w.toff, w.units, nunits, D, Q, cap, w.sig,
+  launch_pdl(bin_count_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, tcount, choice, headroom, status);
+  launch_pdl(bin_scan_kernel, 1, 1024, 0, s, g.T2, tcount, w.toff, w.units, nunits, D, Q, cap, w.sig,
                                      w.rank_of, w.capq, status);
-  bin_scatter_kernel<<<gb, 1024, 0, s>>>(J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord, w.sp, w.su);
+  launch_pdl(bin_scatter_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord, w.sp, w.su);
   MAPS_TRY(launch_ok());
 
   CUtensorMap tmap;
@@ -1173,21 +1183,21 @@ int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K, con
       const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
       uint32_t *km = cv.take<uint32_t>(static_cast<size_t>(D) * nb);
       const int gk = static_cast<int>(std::min<int64_t>((nb * D + 255) / 256, 8LL * sm_count()));
-      kmax_from_K_kernel<<<gk, 256, 0, s>>>(D, H, K, km, status);
-      dispatch_sequential_kernel<<<1, 1024, 0, s>>>(D, H, K, km, cap, Q, J, cand_prompt,
+      launch_pdl(kmax_from_K_kernel, gk, 256, 0, s, D, H, K, km, status);
+      launch_pdl(dispatch_sequential_kernel, 1, 1024, 0, s, D, H, K, km, cap, Q, J, cand_prompt,
                                                     cand_bound, choice_out, headroom_out, status);
       return launch_ok();
     }
     default: {
       Carve cv(ws);
       long long *B_eff = cv.take<long long>(static_cast<size_t>(D));
-      alg1_budget_kernel<<<D, 256, 0, s>>>(D, S, res_off, R, prompt, gen, bound, cap, B_eff, status);
+      launch_pdl(alg1_budget_kernel, D, 256, 0, s, D, S, res_off, R, prompt, gen, bound, cap, B_eff, status);
       if (mode == MAPS_MODE_ALG1_SNAPSHOT) {
         const int grid = static_cast<int>(std::min<int64_t>((J + 255) / 256, 4LL * sm_count()));
-        alg1_snapshot_kernel<<<grid, 256, 0, s>>>(D, S, B_eff, cap, Q, J, cand_prompt, cand_bound,
+        launch_pdl(alg1_snapshot_kernel, grid, 256, 0, s, D, S, B_eff, cap, Q, J, cand_prompt, cand_bound,
                                                   choice_out, headroom_out, status);
       } else {
-        alg1_sequential_kernel<<<1, 1024, 0, s>>>(D, S, B_eff, cap, Q, J, cand_prompt, cand_bound,
+        launch_pdl(alg1_sequential_kernel, 1, 1024, 0, s, D, S, B_eff, cap, Q, J, cand_prompt, cand_bound,
                                                   choice_out, headroom_out, status);
       }
       return launch_ok();

@@ -62,6 +62,17 @@ __device__ __forceinline__ void st_release_u64(unsigned long long *p, unsigned l
   asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
+// Programmatic dependent launch.  Every kernel of the library is launched
+// with programmatic stream serialisation and starts with pdl_prologue():
+// griddepcontrol.wait blocks until the previous grid on the stream has
+// completed and its memory is visible (so nothing reads a predecessor's
+// output early), and launch_dependents lets the next grid be scheduled once
+// every CTA of this one has started, which hides the launch gap.
+__device__ __forceinline__ void pdl_prologue() {
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
+
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
@@ -74,6 +85,24 @@ inline int cuda_ok(cudaError_t e) {
   return MAPS_E_CUDA;
 }
 inline int launch_ok() { return cuda_ok(cudaGetLastError()); }
+
+// Launches `kernel` with programmatic stream serialisation (see pdl_prologue);
+// errors surface through launch_ok().
+template <typename... KArgs, typename... Args>
+inline void launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  (void)cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
 
 inline bool aligned(const void *p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;

@@ -32,16 +32,25 @@
 namespace maps {
 namespace {
 
-constexpr int kOccThreads = 512;
+constexpr int kOccThreads = 512;  // tile CTAs: 512 threads x CPT cells
 constexpr int kWarps = kOccThreads / 32;
+constexpr int kBucketThreads = 512;
 constexpr int kBlock = 16;     // steps per kmax summary entry
 constexpr int kPerThread = 4;  // entries a thread loads per round
 constexpr int kRound = kPerThread * kOccThreads;
+constexpr int kBucketRound = kPerThread * kBucketThreads;
 constexpr int kMaxTiles = 64;  // tiles per decoder of the bucketed form
 
-// Shared-memory state of one tile.  Bins are padded by 4 words after every
-// CPT bins so that the threads' 16-byte reads of their own CPT bins fall on
-// distinct banks.
+// Per-warp carry partials and the block scan's scratch.
+struct TileScan {
+  uint32_t part[2][kWarps];  // per-warp carry partials (count, b-sum)
+  uint32_t wsum[2][kWarps];
+  uint32_t carry[2];
+};
+
+// Shared-memory end-step histogram of one tile (the long-horizon form).  Bins
+// are padded by 4 words after every CPT bins so that the threads' 16-byte
+// reads of their own CPT bins fall on distinct banks.
 template <int CPT>
 struct TileSmem {
   static constexpr int W = kOccThreads * CPT;
@@ -49,9 +58,7 @@ struct TileSmem {
   static constexpr int WP = W + (W / CPT) * kPad;
   int32_t cnt[WP];  // bin j: residents whose last live step is t0 + j
   int32_t sb[WP];   // ... and the sum of their b
-  uint32_t part[2][kWarps];  // per-warp carry partials (count, b-sum)
-  uint32_t wsum[2][kWarps];
-  uint32_t carry[2];
+  TileScan scan;
 };
 
 template <int CPT>
@@ -69,26 +76,23 @@ __device__ __forceinline__ void add_to_bin(TileSmem<CPT> &sm, int jj, int32_t b)
   atomicAdd(&sm.sb[jp], b);  // exact while sum b fits int32
 }
 
-// Writes tile [t0, t0 + W) of row k from the histogram and the per-warp
-// carry partials.  Entry: bins complete, part[][warp] written by every warp,
-// and a block barrier since.  The carry partials are 32-bit: they only wrap
-// when sum b exceeds INT32_MAX, which is reported as MAPS_E_RANGE.
+// Writes tile [t0, t0 + W) of row k.  Thread tid owns cells tid*CPT + c,
+// c < CPT, and holds in bc[c] / bs[c] the count and b-sum of the residents
+// whose last live step is that cell.  Entry: sc.part[][warp] written by every
+// warp and a block barrier since.  Cell l needs every bin at or after l: the
+// thread's own bins from l up, all bins of the threads above it, and the
+// carry.  The 32-bit sums only wrap when sum b exceeds INT32_MAX, which is
+// reported as MAPS_E_RANGE.
 template <int CPT, bool VEC>
-__device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t0, int32_t *K,
-                                          uint32_t *kmax, int32_t *status) {
-  constexpr int kPad = TileSmem<CPT>::kPad;
+__device__ __forceinline__ void emit_cells(const uint32_t (&bc)[CPT], const uint32_t (&bs)[CPT],
+                                           TileScan &sc, int H, int k, int t0, int32_t *K,
+                                           uint32_t *kmax, int32_t *status) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // Thread tid owns cells l = tid*CPT + c and the bins with the same index;
-  // cell l needs every bin j >= l: its own bins from l up plus all bins of
-  // the threads above it.
-  const int32_t *cb = &sm.cnt[tid * (CPT + kPad)], *sb = &sm.sb[tid * (CPT + kPad)];
   uint32_t tot_c = 0, tot_s = 0;
 #pragma unroll
-  for (int c = 0; c < CPT; c += 4) {
-    const int4 x = *reinterpret_cast<const int4 *>(cb + c);
-    const int4 y = *reinterpret_cast<const int4 *>(sb + c);
-    tot_c += static_cast<uint32_t>(x.x + x.y + x.z + x.w);
-    tot_s += static_cast<uint32_t>(y.x + y.y + y.z + y.w);
+  for (int c = 0; c < CPT; ++c) {
+    tot_c += bc[c];
+    tot_s += bs[c];
   }
   uint32_t suf_c = tot_c, suf_s = tot_s;  // inclusive suffix within the warp
 #pragma unroll
@@ -101,13 +105,13 @@ __device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t
     }
   }
   if (lane == 0) {
-    sm.wsum[0][warp] = suf_c;
-    sm.wsum[1][warp] = suf_s;
+    sc.wsum[0][warp] = suf_c;
+    sc.wsum[1][warp] = suf_s;
   }
   __syncthreads();
   if (warp == 0) {  // exclusive suffix over the warps' totals; the carry
-    uint32_t wc = lane < kWarps ? sm.wsum[0][lane] : 0u;
-    uint32_t ws = lane < kWarps ? sm.wsum[1][lane] : 0u;
+    uint32_t wc = lane < kWarps ? sc.wsum[0][lane] : 0u;
+    uint32_t ws = lane < kWarps ? sc.wsum[1][lane] : 0u;
     const uint32_t oc = wc, os = ws;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
@@ -118,8 +122,8 @@ __device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t
         ws += ys;
       }
     }
-    uint32_t cc = lane < kWarps ? sm.part[0][lane] : 0u;
-    uint32_t cs = lane < kWarps ? sm.part[1][lane] : 0u;
+    uint32_t cc = lane < kWarps ? sc.part[0][lane] : 0u;
+    uint32_t cs = lane < kWarps ? sc.part[1][lane] : 0u;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
       cc += __shfl_xor_sync(0xffffffffu, cc, off);
@@ -127,20 +131,18 @@ __device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t
     }
     __syncwarp();
     if (lane < kWarps) {
-      sm.wsum[0][lane] = wc - oc;
-      sm.wsum[1][lane] = ws - os;
+      sc.wsum[0][lane] = wc - oc;
+      sc.wsum[1][lane] = ws - os;
     }
     if (lane == 0) {
-      sm.carry[0] = cc;
-      sm.carry[1] = cs;
+      sc.carry[0] = cc;
+      sc.carry[1] = cs;
     }
   }
   __syncthreads();
 
-  // All partial sums are below K[k][0] <= INT32_MAX unless a range error is
-  // flagged, so they are kept in 32 bits.
-  const uint32_t c_lo = sm.carry[0] + sm.wsum[0][warp] + (suf_c - tot_c);
-  const uint32_t s_lo = sm.carry[1] + sm.wsum[1][warp] + (suf_s - tot_s);
+  const uint32_t c_lo = sc.carry[0] + sc.wsum[0][warp] + (suf_c - tot_c);
+  const uint32_t s_lo = sc.carry[1] + sc.wsum[1][warp] + (suf_s - tot_s);
   const int cell0 = t0 + tid * CPT;
   const uint32_t tc0 = static_cast<uint32_t>(cell0);
   uint32_t bmax = 0;  // max of K + t over this thread's valid cells
@@ -153,33 +155,23 @@ __device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t
     uint32_t run_c = c_lo, run_s = s_lo;
     if (VEC && bound64 <= 0x7fffffffull && cell0 + CPT <= H) {
       // every cell valid and exact in 32 bits
+      uint32_t o[CPT];
 #pragma unroll
-      for (int c0 = CPT - 4; c0 >= 0; c0 -= 4) {
-        const int4 x = *reinterpret_cast<const int4 *>(cb + c0);
-        const int4 y = *reinterpret_cast<const int4 *>(sb + c0);
-        const uint32_t t = tc0 + c0;
-        uint32_t o3, o2, o1, o0;
-        run_c += static_cast<uint32_t>(x.w);
-        run_s += static_cast<uint32_t>(y.w);
-        o3 = (t + 3) * run_c + run_s;
-        run_c += static_cast<uint32_t>(x.z);
-        run_s += static_cast<uint32_t>(y.z);
-        o2 = (t + 2) * run_c + run_s;
-        run_c += static_cast<uint32_t>(x.y);
-        run_s += static_cast<uint32_t>(y.y);
-        o1 = (t + 1) * run_c + run_s;
-        run_c += static_cast<uint32_t>(x.x);
-        run_s += static_cast<uint32_t>(y.x);
-        o0 = t * run_c + run_s;
-        bmax = max(bmax, max(max(o0 + t, o1 + t + 1), max(o2 + t + 2, o3 + t + 3)));
-        *reinterpret_cast<int4 *>(row + cell0 + c0) = make_int4(o0, o1, o2, o3);
+      for (int c = CPT - 1; c >= 0; --c) {
+        run_c += bc[c];
+        run_s += bs[c];
+        o[c] = (tc0 + c) * run_c + run_s;
+        bmax = max(bmax, o[c] + tc0 + c);
       }
+#pragma unroll
+      for (int c = 0; c < CPT; c += 4)
+        *reinterpret_cast<int4 *>(row + cell0 + c) = make_int4(o[c], o[c + 1], o[c + 2], o[c + 3]);
     } else {
       bool over = false;
 #pragma unroll
       for (int c = CPT - 1; c >= 0; --c) {
-        run_c += static_cast<uint32_t>(cb[c]);
-        run_s += static_cast<uint32_t>(sb[c]);
+        run_c += bc[c];
+        run_s += bs[c];
         if (cell0 + c < H) {
           const uint32_t t = tc0 + c;
           const unsigned long long v = static_cast<unsigned long long>(t) * run_c + run_s;
@@ -203,6 +195,23 @@ __device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t
   }
 }
 
+// The histogram form: each thread takes its own CPT bins into registers.
+template <int CPT, bool VEC>
+__device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t0, int32_t *K,
+                                          uint32_t *kmax, int32_t *status) {
+  constexpr int kPad = TileSmem<CPT>::kPad;
+  const int32_t *cb = &sm.cnt[threadIdx.x * (CPT + kPad)], *sb = &sm.sb[threadIdx.x * (CPT + kPad)];
+  uint32_t bc[CPT], bs[CPT];
+#pragma unroll
+  for (int c = 0; c < CPT; c += 4) {
+    const int4 x = *reinterpret_cast<const int4 *>(cb + c);
+    const int4 y = *reinterpret_cast<const int4 *>(sb + c);
+    bc[c] = x.x, bc[c + 1] = x.y, bc[c + 2] = x.z, bc[c + 3] = x.w;
+    bs[c] = y.x, bs[c + 1] = y.y, bs[c + 2] = y.z, bs[c + 3] = y.w;
+  }
+  emit_cells<CPT, VEC>(bc, bs, sm.scan, H, k, t0, K, kmax, status);
+}
+
 // Resident terms: false for a negative length (a range error).
 __device__ __forceinline__ bool resident_terms(int32_t p, int32_t g, int32_t U, int H,
                                                int32_t &b32, int32_t &e, bool &big) {
@@ -215,6 +224,7 @@ __device__ __forceinline__ bool resident_terms(int32_t p, int32_t g, int32_t U, 
   return true;
 }
 
+template <int NW>
 __device__ __forceinline__ long long block_sum_ll(long long v, long long *s_red) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
@@ -222,21 +232,22 @@ __device__ __forceinline__ long long block_sum_ll(long long v, long long *s_red)
   if (lane == 0) s_red[warp] = v;
   __syncthreads();
   long long t = 0;
-  for (int w = 0; w < kWarps; ++w) t += s_red[w];
+  for (int w = 0; w < NW; ++w) t += s_red[w];
   return t;
 }
 
 // ---------------------------------------------------------------------------
 // 1. Bucket kernel: one CTA per decoder.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kOccThreads)
+__global__ void __launch_bounds__(kBucketThreads)
 occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, int64_t R,
                   const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
                   const int32_t *__restrict__ bound, int2 *__restrict__ bucket,
                   int32_t *__restrict__ tile_off, int32_t *status) {
+  pdl_prologue();
   __shared__ int s_cnt[kMaxTiles];
   __shared__ int s_cur[kMaxTiles];
-  __shared__ long long s_red[kWarps];
+  __shared__ long long s_red[kBucketThreads / 32];
   const int k = blockIdx.x, tid = threadIdx.x, lane = tid & 31;
   int64_t lo = res_off[k], hi = res_off[k + 1];
   if (lo < 0 || hi < lo || hi > R || hi - lo > 0x7fffffffLL) {
@@ -249,11 +260,11 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
   __syncthreads();
 
   // pass 1: residents per tile
-  for (int r0 = 0; r0 < n; r0 += kRound) {
+  for (int r0 = 0; r0 < n; r0 += kBucketRound) {
     int32_t p[kPerThread], g[kPerThread], U[kPerThread];
 #pragma unroll
     for (int j = 0; j < kPerThread; ++j) {
-      const int i = r0 + j * kOccThreads + tid;
+      const int i = r0 + j * kBucketThreads + tid;
       const bool ok = i < n;
       p[j] = ok ? __ldg(pp + i) : -1;
       g[j] = ok ? __ldg(pg + i) : 0;
@@ -284,11 +295,11 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
   // pass 2: scatter the pairs (the residents come from L2 this time)
   bool bad = false;
   long long total = 0;
-  for (int r0 = 0; r0 < n; r0 += kRound) {
+  for (int r0 = 0; r0 < n; r0 += kBucketRound) {
     int32_t p[kPerThread], g[kPerThread], U[kPerThread];
 #pragma unroll
     for (int j = 0; j < kPerThread; ++j) {
-      const int i = r0 + j * kOccThreads + tid;
+      const int i = r0 + j * kBucketThreads + tid;
       const bool ok = i < n;
       p[j] = ok ? __ldg(pp + i) : -1;
       g[j] = ok ? __ldg(pg + i) : 0;
@@ -296,7 +307,7 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
     }
 #pragma unroll
     for (int j = 0; j < kPerThread; ++j) {
-      const bool present = r0 + j * kOccThreads + tid < n;
+      const bool present = r0 + j * kBucketThreads + tid < n;
       int32_t b32 = 0, e = 0;
       bool big = false;
       int tile = -1;
@@ -316,7 +327,7 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
     }
   }
   if (bad) flag_error(status, MAPS_E_RANGE);
-  const long long sum_b = block_sum_ll(total, s_red);
+  const long long sum_b = block_sum_ll<kBucketThreads / 32>(total, s_red);
   if (tid == 0 && sum_b > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
 }
 
@@ -328,6 +339,7 @@ __global__ void __launch_bounds__(kOccThreads, 2)
 occ_tile_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
                 const int2 *__restrict__ bucket, const int32_t *__restrict__ tile_off,
                 int32_t *__restrict__ K, uint32_t *__restrict__ kmax, int32_t *status) {
+  pdl_prologue();
   __shared__ __align__(16) TileSmem<CPT> sm;
   constexpr int W = TileSmem<CPT>::W;
   const int k = blockIdx.x / T, ti = blockIdx.x - (blockIdx.x / T) * T;
@@ -366,8 +378,8 @@ occ_tile_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
     car_s += __shfl_xor_sync(0xffffffffu, car_s, off);
   }
   if (lane == 0) {
-    sm.part[0][warp] = car_c;
-    sm.part[1][warp] = car_s;
+    sm.scan.part[0][warp] = car_c;
+    sm.scan.part[1][warp] = car_s;
   }
   __syncthreads();
   emit_tile<CPT, VEC>(sm, H, k, t0, K, kmax, status);
@@ -382,6 +394,7 @@ occ_direct_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
                   const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
                   const int32_t *__restrict__ bound, int32_t *__restrict__ K,
                   uint32_t *__restrict__ kmax, int32_t *status) {
+  pdl_prologue();
   __shared__ __align__(16) TileSmem<CPT> sm;
   __shared__ long long s_red[kWarps];
   constexpr int W = TileSmem<CPT>::W;
@@ -431,7 +444,7 @@ occ_direct_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
     }
   }
   if (bad) flag_error(status, MAPS_E_RANGE);
-  const long long sum_b = block_sum_ll(total, s_red);
+  const long long sum_b = block_sum_ll<kWarps>(total, s_red);
   if (ti == 0 && tid == 0 && sum_b > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -439,8 +452,8 @@ occ_direct_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
     car_s += __shfl_xor_sync(0xffffffffu, car_s, off);
   }
   if (lane == 0) {
-    sm.part[0][warp] = car_c;
-    sm.part[1][warp] = car_s;
+    sm.scan.part[0][warp] = car_c;
+    sm.scan.part[1][warp] = car_s;
   }
   __syncthreads();
   emit_tile<CPT, VEC>(sm, H, k, t0, K, kmax, status);
@@ -454,7 +467,7 @@ struct OccPlan {
 OccPlan plan_occ(int32_t H, int64_t R) {
   OccPlan p;
   p.cpt = H <= 2048 ? 4 : (H <= 8192 ? 8 : 16);
-  p.log2W = 9 + (p.cpt == 4 ? 2 : (p.cpt == 8 ? 3 : 4));
+  p.log2W = 9 + (p.cpt == 4 ? 2 : (p.cpt == 8 ? 3 : 4));  // W = 512 threads x CPT
   p.T = static_cast<int>((static_cast<int64_t>(H) + (1 << p.log2W) - 1) >> p.log2W);
   p.bucketed = p.T <= kMaxTiles && R <= 0x7fffffffLL;
   return p;
@@ -476,10 +489,10 @@ void launch_tiles(const OccPlan &p, int64_t blocks, cudaStream_t s, int H, const
                   int32_t *status) {
   const dim3 grid(static_cast<unsigned>(blocks));
   if (p.bucketed)
-    occ_tile_kernel<CPT, VEC><<<grid, kOccThreads, 0, s>>>(H, p.T, res_off, R, bucket, tile_off, K,
+    launch_pdl(occ_tile_kernel<CPT, VEC>, grid, kOccThreads, 0, s, H, p.T, res_off, R, bucket, tile_off, K,
                                                           kmax, status);
   else
-    occ_direct_kernel<CPT, VEC><<<grid, kOccThreads, 0, s>>>(H, p.T, res_off, R, prompt, gen,
+    launch_pdl(occ_direct_kernel<CPT, VEC>, grid, kOccThreads, 0, s, H, p.T, res_off, R, prompt, gen,
                                                             bound, K, kmax, status);
 }
 
@@ -529,7 +542,7 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off, int64_t
   int32_t *tile_off = nullptr;
   carve_occ(c, D, R, p, &bucket, &tile_off);
   if (p.bucketed) {
-    occ_bucket_kernel<<<D, kOccThreads, 0, s>>>(H, p.T, p.log2W, res_off, R, prompt, gen, bound,
+    launch_pdl(occ_bucket_kernel, D, kBucketThreads, 0, s, H, p.T, p.log2W, res_off, R, prompt, gen, bound,
                                                 bucket, tile_off, status);
     MAPS_TRY(launch_ok());
   }

@@ -82,6 +82,7 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
                   uint32_t *dec_count, int32_t *status) {
+  pdl_prologue();
   __shared__ uint32_t s_dec[kDecSmem];
   const bool dec_smem = D <= kDecSmem;
   if (dec_smem)
@@ -141,6 +142,7 @@ order_keys_kernel(int64_t N, int D, int dbits, const int32_t *__restrict__ dec,
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
                   unsigned long long *hi_orig, unsigned long long *keyA, uint32_t *valA) {
+  pdl_prologue();
   __shared__ uint32_t sh[kPasses][kRadix];
   for (int i = threadIdx.x; i < kPasses * kRadix; i += blockDim.x) (&sh[0][0])[i] = 0;
   __syncthreads();
@@ -202,13 +204,18 @@ order_keys_kernel(int64_t N, int D, int dbits, const int32_t *__restrict__ dec,
 __global__ void __launch_bounds__(kRadix)
 order_plan_kernel(int64_t N, int D, int dbits, const OrderCounts *counts, OrderPlan *plan,
                   const uint32_t *dec_count, int64_t *seg_off) {
+  pdl_prologue();
   __shared__ uint32_t s_warp[kRadix / 32];
   __shared__ long long s_w64[kRadix / 32];
   __shared__ int s_trivial[kPasses];
   __shared__ long long s_carry;
   const int b = threadIdx.x, lane = b & 31, warp = b >> 5;
+  uint32_t cnt[kPasses];  // all loads first
+#pragma unroll
+  for (int p = 0; p < kPasses; ++p) cnt[p] = counts->h[p][b];
+#pragma unroll
   for (int p = 0; p < kPasses; ++p) {
-    const uint32_t c = counts->h[p][b];
+    const uint32_t c = cnt[p];
     uint32_t incl = c;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
@@ -299,6 +306,7 @@ __global__ void order_gather_kernel(int64_t N, const OrderPlan *plan,
                                     const unsigned long long *hi_orig, unsigned long long *keyA,
                                     unsigned long long *keyB, const uint32_t *valA,
                                     const uint32_t *valB) {
+  pdl_prologue();
   const int gb = plan->gather_buf;
   if (gb < 0) return;
   const bool wide = plan->wide != 0;
@@ -316,6 +324,7 @@ __global__ void order_gather_kernel(int64_t N, const OrderPlan *plan,
 
 // No active pass at all: the identity is the order.
 __global__ void order_identity_kernel(int64_t N, const OrderPlan *plan, int32_t *perm) {
+  pdl_prologue();
   if (plan->npasses != 0) return;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < N; i += stride)
@@ -490,6 +499,7 @@ order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *k
                   unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
                   const unsigned long long *hi_orig, int32_t *perm, unsigned long long *state,
                   int64_t tiles, uint32_t *ticket, int32_t *status) {
+  pdl_prologue();
   if (!plan->active[p]) return;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PassSmem &sm = *reinterpret_cast<PassSmem *>(smem_raw);
@@ -565,12 +575,12 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   const int64_t tiles = std::max<int64_t>(1, (N + kTile - 1) / kTile);
   if (N > 0) {
     const int g = static_cast<int>(std::min<int64_t>((N + 2047) / 2048, 2LL * sms));
-    order_prep_kernel<<<g, 512, 0, s>>>(N, D, dec, bound, wait, arrival, max_wait, w.counts,
+    launch_pdl(order_prep_kernel, g, 512, 0, s, N, D, dec, bound, wait, arrival, max_wait, w.counts,
                                         w.dec_count, status);
-    order_keys_kernel<<<g, 512, 0, s>>>(N, D, dbits, dec, bound, wait, arrival, max_wait, w.counts,
+    launch_pdl(order_keys_kernel, g, 512, 0, s, N, D, dbits, dec, bound, wait, arrival, max_wait, w.counts,
                                         w.hi_orig, w.keyA, w.valA);
   }
-  order_plan_kernel<<<1, kRadix, 0, s>>>(N, D, dbits, w.counts, w.plan, w.dec_count, seg_off_out);
+  launch_pdl(order_plan_kernel, 1, kRadix, 0, s, N, D, dbits, w.counts, w.plan, w.dec_count, seg_off_out);
   MAPS_TRY(launch_ok());
   if (N == 0) return MAPS_OK;
   const size_t smem = sizeof(PassSmem);
@@ -578,14 +588,14 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
                                         static_cast<int>(smem))));
   const int gcopy = static_cast<int>(std::min<int64_t>((N + 255) / 256, 4LL * sms));
   auto pass = [&](int p) {
-    order_pass_kernel<<<static_cast<unsigned>(tiles), kPassThreads, smem, s>>>(
+    launch_pdl(order_pass_kernel, static_cast<unsigned>(tiles), kPassThreads, smem, s, 
         p, N, w.plan, w.keyA, w.keyB, w.valA, w.valB, w.hi_orig, perm_out, w.state, tiles,
         w.tickets + p, status);
   };
   for (int p = 0; p < kLoPasses; ++p) pass(p);
-  order_gather_kernel<<<gcopy, 256, 0, s>>>(N, w.plan, w.hi_orig, w.keyA, w.keyB, w.valA, w.valB);
+  launch_pdl(order_gather_kernel, gcopy, 256, 0, s, N, w.plan, w.hi_orig, w.keyA, w.keyB, w.valA, w.valB);
   for (int p = kLoPasses; p < kLoPasses + n_hi; ++p) pass(p);
-  order_identity_kernel<<<gcopy, 256, 0, s>>>(N, w.plan, perm_out);
+  launch_pdl(order_identity_kernel, gcopy, 256, 0, s, N, w.plan, perm_out);
   return launch_ok();
 }
 

@@ -61,6 +61,7 @@ __device__ __forceinline__ int block_flag_scan(bool f, int *s_w, int &total) {
 __global__ void stream_validate_kernel(int64_t N, const int64_t *arrival, const int32_t *prompt,
                                        const int32_t *true_len, const int32_t *pred,
                                        int32_t *status) {
+  pdl_prologue();
   bool bad = false;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < N; i += stride)
@@ -71,6 +72,7 @@ __global__ void stream_validate_kernel(int64_t N, const int64_t *arrival, const 
 
 __global__ void stream_init_kernel(int64_t first_hi, int D, int32_t cap, const int64_t *arrival,
                                    int32_t *capv, StreamState *S) {
+  pdl_prologue();
   for (int k = threadIdx.x; k < D; k += blockDim.x) capv[k] = cap;
   if (threadIdx.x == 0) {
     S->prev_s = arrival[first_hi - 1];
@@ -87,6 +89,7 @@ stream_advance_kernel(int64_t hi, int D, int32_t cap, const int64_t *arrival,
                       const int32_t *dec, const int32_t *act_in, int32_t *act_out,
                       int32_t *done_id, int32_t *done_rem, long long *used, StreamState *S,
                       int64_t *stats_b) {
+  pdl_prologue();
   __shared__ unsigned long long s_used[kStreamMaxD];
   __shared__ int s_w[kStWarps];
   __shared__ int s_nwait;
@@ -151,6 +154,7 @@ stream_advance_kernel(int64_t hi, int D, int32_t cap, const int64_t *arrival,
 __global__ void stream_window_kernel(int ndone, long long c0, int Wn, const int32_t *perm,
                                      const int32_t *done_id, const int32_t *true_len,
                                      const int32_t *pred, int32_t *win_true, int32_t *win_pred) {
+  pdl_prologue();
   const int stride = gridDim.x * blockDim.x;
   for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < ndone; x += stride) {
     if (x < ndone - Wn) continue;  // overwritten by a later completion of this batch
@@ -164,6 +168,7 @@ __global__ void stream_window_kernel(int ndone, long long c0, int Wn, const int3
 // 3. Predictions of the requests in the system, then of the batch.
 __global__ void stream_gather_kernel(int nact, int nb, int64_t lo, const int32_t *act,
                                      const int32_t *pred, int32_t *qpred) {
+  pdl_prologue();
   const int stride = gridDim.x * blockDim.x;
   for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < nact + nb; x += stride)
     qpred[x] = x < nact ? pred[act[x]] : pred[lo + (x - nact)];
@@ -172,6 +177,7 @@ __global__ void stream_gather_kernel(int nact, int nb, int64_t lo, const int32_t
 // 3'. No bound available: U = prediction, the batch goes round robin.
 __global__ void stream_rr_kernel(int n, int nb, int64_t lo, int D, const int32_t *qpred,
                                  int32_t *Uq, int32_t *choice) {
+  pdl_prologue();
   const int stride = gridDim.x * blockDim.x;
   for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
     Uq[x] = qpred[x];
@@ -186,6 +192,7 @@ stream_csr_kernel(int nact, int D, int rr, const int32_t *q_dev, int32_t *q_out_
                   const int32_t *act, const uint8_t *st, const int32_t *g, const int32_t *dec,
                   const int32_t *prompt, const int32_t *Uq, int32_t *U, int64_t *res_off,
                   int32_t *rp, int32_t *rg, int32_t *rU, int32_t *Q) {
+  pdl_prologue();
   __shared__ int s_cnt[kStreamMaxD], s_q[kStreamMaxD], s_cur[kStreamMaxD];
   __shared__ int s_w[kStWarps];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -233,6 +240,7 @@ __global__ void stream_enqueue_kernel(int64_t lo, int nb, int nact, int64_t hi, 
                                       const int32_t *Uq, uint8_t *st, int32_t *dec,
                                       long long *disp, int32_t *g, int32_t *U, int32_t *act,
                                       StreamState *S, int32_t *status) {
+  pdl_prologue();
   const long long s = arrival[hi - 1];
   const int stride = gridDim.x * blockDim.x;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
@@ -258,6 +266,7 @@ stream_waitlist_kernel(int n, int64_t hi, const int64_t *arrival, const int32_t 
                        const uint8_t *st, const int32_t *dec, const int32_t *U,
                        const long long *disp, int32_t *wid, int32_t *wdec, int32_t *wU,
                        int32_t *wwait, int32_t *warr) {
+  pdl_prologue();
   __shared__ int s_w[kStWarps];
   const long long s = arrival[hi - 1];
   int nw = 0;
@@ -287,6 +296,7 @@ __global__ void __launch_bounds__(kSt, 1)
 stream_admit_kernel(int D, int32_t cap, int nw, const int64_t *wseg, const int32_t *wperm,
                     const int32_t *wid, const int32_t *prompt, const int32_t *U,
                     const long long *used, uint8_t *st, int32_t *g, int64_t *stats_b) {
+  pdl_prologue();
   __shared__ int s_adm;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) s_adm = 0;
@@ -441,8 +451,8 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
 
   MAPS_TRY(cuda_ok(cudaMemsetAsync(w.st, 0, static_cast<size_t>(N), s)));
   MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zeros, 0, static_cast<size_t>(N) * sizeof(int32_t), s)));
-  stream_init_kernel<<<1, kSt, 0, s>>>(std::min(N, B), D, c.cap, arrival_ms, w.capv, w.S);
-  stream_validate_kernel<<<grid_for(N), 256, 0, s>>>(N, arrival_ms, prompt, true_len, pred, status);
+  launch_pdl(stream_init_kernel, 1, kSt, 0, s, std::min(N, B), D, c.cap, arrival_ms, w.capv, w.S);
+  launch_pdl(stream_validate_kernel, grid_for(N), 256, 0, s, N, arrival_ms, prompt, true_len, pred, status);
   MAPS_TRY(launch_ok());
   {
     const int st0 = maps_check(ws, stream);  // a bad input stops the loop before it starts
@@ -456,7 +466,7 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
     const int nb = static_cast<int>(hi - lo);
     int32_t *act_in = w.act[b & 1], *act = w.act[(b & 1) ^ 1];
     int64_t *stats_b = stats_out + 4 * b;
-    stream_advance_kernel<<<1, kSt, 0, s>>>(hi, D, c.cap, arrival_ms, prompt, true_len, w.st, w.g,
+    launch_pdl(stream_advance_kernel, 1, kSt, 0, s, hi, D, c.cap, arrival_ms, prompt, true_len, w.st, w.g,
                                             w.dec, act_in, act, w.done_id, w.done_rem, w.used, w.S,
                                             stats_b);
     MAPS_TRY(launch_ok());
@@ -467,22 +477,22 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
     if (ndone > 0) {  // 2.
       MAPS_TRY(maps_order_local(ndone, 1, w.zeros, w.done_rem, w.zeros, w.done_id, 0, w.done_perm,
                                 w.done_seg, ws, w.sub_bytes, stream));
-      stream_window_kernel<<<grid_for(ndone), 256, 0, s>>>(ndone, total_done, c.window,
+      launch_pdl(stream_window_kernel, grid_for(ndone), 256, 0, s, ndone, total_done, c.window,
                                                            w.done_perm, w.done_id, true_len, pred,
                                                            w.win_true, w.win_pred);
       total_done += ndone;
     }
     const int64_t win_len = std::min<long long>(total_done, c.window);
 
-    stream_gather_kernel<<<grid_for(nact + nb), 256, 0, s>>>(nact, nb, lo, act, pred, w.qpred);
+    launch_pdl(stream_gather_kernel, grid_for(nact + nb), 256, 0, s, nact, nb, lo, act, pred, w.qpred);
     const int cs = maps_calibrate(w.win_true, w.win_pred, win_len, c.alpha_ppm, w.qpred, nact + nb,
                                   w.Uq, w.q_dev, nullptr, ws, w.sub_bytes, stream);  // 3.
     const bool rr = cs == MAPS_E_UNBOUNDED;
     if (cs != MAPS_OK && !rr) return cs;
     if (rr)
-      stream_rr_kernel<<<grid_for(nact + nb), 256, 0, s>>>(nact + nb, nb, lo, D, w.qpred, w.Uq,
+      launch_pdl(stream_rr_kernel, grid_for(nact + nb), 256, 0, s, nact + nb, nb, lo, D, w.qpred, w.Uq,
                                                            choice_out);
-    stream_csr_kernel<<<1, kSt, 0, s>>>(nact, D, rr ? 1 : 0, w.q_dev, q_out + b, act, w.st, w.g,
+    launch_pdl(stream_csr_kernel, 1, kSt, 0, s, nact, D, rr ? 1 : 0, w.q_dev, q_out + b, act, w.st, w.g,
                                         w.dec, prompt, w.Uq, w.U, w.res_off, w.rp, w.rg, w.rU,
                                         w.Q);  // 4.
     MAPS_TRY(launch_ok());
@@ -493,16 +503,16 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
                              nullptr, nullptr, nullptr, nb, prompt + lo, w.Uq + nact,
                              choice_out + lo, w.headroom, ws, w.sub_bytes, stream));
     }
-    stream_enqueue_kernel<<<grid_for(nb), 256, 0, s>>>(lo, nb, nact, hi, D, arrival_ms,
+    launch_pdl(stream_enqueue_kernel, grid_for(nb), 256, 0, s, lo, nb, nact, hi, D, arrival_ms,
                                                        choice_out, w.Uq, w.st, w.dec, w.disp, w.g,
                                                        w.U, act, w.S, status);  // 6.
     const int n_all = nact + nb, nw = nwait + nb;
-    stream_waitlist_kernel<<<1, kSt, 0, s>>>(n_all, hi, arrival_ms, act, w.st, w.dec, w.U, w.disp,
+    launch_pdl(stream_waitlist_kernel, 1, kSt, 0, s, n_all, hi, arrival_ms, act, w.st, w.dec, w.U, w.disp,
                                              w.wid, w.wdec, w.wU, w.wwait, w.warr);  // 7.
     MAPS_TRY(launch_ok());
     MAPS_TRY(maps_order_local(nw, D, w.wdec, w.wU, w.wwait, w.warr, c.max_wait, w.wperm, w.wseg, ws,
                               w.sub_bytes, stream));
-    stream_admit_kernel<<<1, kSt, 0, s>>>(D, c.cap, nw, w.wseg, w.wperm, w.wid, prompt, w.U, w.used,
+    launch_pdl(stream_admit_kernel, 1, kSt, 0, s, D, c.cap, nw, w.wseg, w.wperm, w.wid, prompt, w.U, w.used,
                                           w.st, w.g, stats_b);  // 8.
     MAPS_TRY(launch_ok());
   }
