@@ -32,14 +32,14 @@
 namespace maps {
 namespace {
 
-constexpr int kOccThreads = 512;  // tile CTAs: 512 threads x CPT cells
+constexpr int kOccThreads = 256;  // tile CTAs: 256 threads x CPT cells
 constexpr int kWarps = kOccThreads / 32;
 constexpr int kBucketThreads = 512;
 constexpr int kBlock = 16;     // steps per kmax summary entry
 constexpr int kPerThread = 4;  // entries a thread loads per round
 constexpr int kRound = kPerThread * kOccThreads;
 constexpr int kBucketRound = kPerThread * kBucketThreads;
-constexpr int kMaxTiles = 64;  // tiles per decoder of the bucketed form
+constexpr int kMaxTiles = 128;  // tiles per decoder of the bucketed form
 
 // Per-warp carry partials and the block scan's scratch.
 struct TileScan {
@@ -335,7 +335,7 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
 // 2. Tile kernel: one CTA per (decoder, tile), reading the sorted pairs.
 // ---------------------------------------------------------------------------
 template <int CPT, bool VEC>
-__global__ void __launch_bounds__(kOccThreads, 2)
+__global__ void __launch_bounds__(kOccThreads, 5)
 occ_tile_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
                 const int2 *__restrict__ bucket, const int32_t *__restrict__ tile_off,
                 int32_t *__restrict__ K, uint32_t *__restrict__ kmax, int32_t *status) {
@@ -389,7 +389,7 @@ occ_tile_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
 // Long horizons: every tile CTA streams all of its decoder's residents.
 // ---------------------------------------------------------------------------
 template <int CPT, bool VEC>
-__global__ void __launch_bounds__(kOccThreads, 2)
+__global__ void __launch_bounds__(kOccThreads, 5)
 occ_direct_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
                   const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
                   const int32_t *__restrict__ bound, int32_t *__restrict__ K,
@@ -466,8 +466,8 @@ struct OccPlan {
 
 OccPlan plan_occ(int32_t H, int64_t R) {
   OccPlan p;
-  p.cpt = H <= 2048 ? 4 : (H <= 8192 ? 8 : 16);
-  p.log2W = 9 + (p.cpt == 4 ? 2 : (p.cpt == 8 ? 3 : 4));  // W = 512 threads x CPT
+  p.cpt = H <= 1024 ? 4 : (H <= 2048 ? 8 : 16);
+  p.log2W = 8 + (p.cpt == 4 ? 2 : (p.cpt == 8 ? 3 : 4));  // W = 256 threads x CPT
   p.T = static_cast<int>((static_cast<int64_t>(H) + (1 << p.log2W) - 1) >> p.log2W);
   p.bucketed = p.T <= kMaxTiles && R <= 0x7fffffffLL;
   return p;
