@@ -118,7 +118,7 @@ kmax_from_K_kernel(int D, int H, const int32_t *__restrict__ K, uint32_t *__rest
   if (neg) flag_error(status, MAPS_E_RANGE);
 }
 
-// carry[k][i] = max of K[k][t] + t over t < i*W2 (0 for i = 0): the prefix
+// carry[i][k] = max of K[k][t] + t over t < i*W2 (0 for i = 0): the prefix
 // maximum that horizon tile i inherits from the tiles before it.  One block
 // per decoder; each thread reads 16 consecutive summary entries at once
 // (whole tiles, as W2/16 divides 16), keeps its tiles' maxima in registers,
@@ -133,7 +133,7 @@ carry_scan_kernel(int D, int H, int W2, int T2, const uint32_t *__restrict__ kma
   const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
   const int bpt = W2 / kSumBlock;  // summary blocks per tile (1..16)
   const uint32_t *row = kmax + static_cast<int64_t>(k) * nb;
-  uint32_t *out = carry + static_cast<int64_t>(k) * T2;
+  uint32_t *out = carry + k;  // carry[i][k], decoder-contiguous per tile
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const bool vec = (reinterpret_cast<uintptr_t>(row) % 16) == 0;
   uint32_t run = 0;
@@ -175,7 +175,7 @@ carry_scan_kernel(int D, int H, int W2, int T2, const uint32_t *__restrict__ kma
     for (int q = 0; q < kPer; ++q) {
       if (q % bpt == 0) {
         const int64_t ti = tile0 + q / bpt;
-        if (ti < T2) out[ti] = r;
+        if (ti < T2) out[ti * D] = r;
       }
       r = v[q] > r ? v[q] : r;
     }
@@ -402,7 +402,7 @@ struct SnapArgs {
   bool use_tma;
   const int32_t *K;
   const int32_t *sig, *rank_of, *capq;  // queue order
-  const uint32_t *carry;                // [D][T2]
+  const uint32_t *carry;                // [T2][D]
   const Unit *units;
   const uint32_t *nunits;
   const int32_t *ord, *sp, *su;
@@ -423,9 +423,12 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   constexpr int kWarpsM = kMainThreads / 32;
   uint32_t *kb = reinterpret_cast<uint32_t *>(smem);
   // comp[slot][i]: M of decoder sig[i] at the slot's column, then rewritten
-  // in place into the queue-ordered prefix maximum of A (clamped at -1)
+  // in place into the queue-ordered prefix maximum of A (clamped at -1).
+  // Rows are D + 1 words apart so that one row's writes to several slots fall
+  // on different banks.
+  const int Dp = D + 1;
   uint32_t *comp = kb + a.tile_stride;
-  int32_t *s_capq = reinterpret_cast<int32_t *>(comp + static_cast<size_t>(W2) * D);
+  int32_t *s_capq = reinterpret_cast<int32_t *>(comp + static_cast<size_t>(W2) * Dp);
   int32_t *s_sig = s_capq + D;
   int32_t *s_rank = s_sig + D;
   uint32_t *s_carry = reinterpret_cast<uint32_t *>(s_rank + D);
@@ -455,7 +458,7 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
     s_sig[k] = __ldg(a.sig + k);
     s_rank[k] = __ldg(a.rank_of + k);
     s_capq[k] = __ldg(a.capq + k);
-    s_carry[k] = __ldg(a.carry + static_cast<int64_t>(k) * a.T2 + un.tile);
+    s_carry[k] = __ldg(a.carry + static_cast<int64_t>(un.tile) * D + k);
   }
   for (int c = tid; c < W2; c += kMainThreads) s_slot[c] = 0;
   __syncthreads();
@@ -538,7 +541,7 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
 #pragma unroll
       for (int j = 0; j < seg; ++j) {
         const int sl = s_slot[sg * seg + j];
-        if (sl >= 0) comp[static_cast<size_t>(sl) * D + rk] = v[j] > excl ? v[j] : excl;
+        if (sl >= 0) comp[static_cast<size_t>(sl) * Dp + rk] = v[j] > excl ? v[j] : excl;
       }
     }
   }
@@ -548,7 +551,7 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   // --- per needed column: prefix max of A in queue order, arg-max of A -----
   const int P = (D + 31) / 32;  // strided queue positions per lane
   for (int sl = warp; sl < nslots; sl += kWarpsM) {
-    uint32_t *col = comp + static_cast<size_t>(sl) * D;
+    uint32_t *col = comp + static_cast<size_t>(sl) * Dp;
     int32_t carryq = -1;
     long long bestA = LLONG_MIN;
     int bestK = 0x7fffffff;
@@ -607,7 +610,7 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
       const int32_t p = pp[i];
       const int c = static_cast<int>(uu[i] - 1 - t0);
       const int sl = s_slot[c];
-      const int32_t *pm = reinterpret_cast<const int32_t *>(comp) + static_cast<size_t>(sl) * D;
+      const int32_t *pm = reinterpret_cast<const int32_t *>(comp) + static_cast<size_t>(sl) * Dp;
       int k;
       long long h;
       if (pm[D - 1] < p) {
@@ -992,7 +995,7 @@ SnapGeom snap_geom(int D, int H) {
   g.T2 = static_cast<int>((static_cast<long long>(H) + w - 1) / w);
   g.tile_stride = (g.Drows * w + 255) / 256 * 256;  // 1 KB-aligned buffer
   size_t b = static_cast<size_t>(g.tile_stride) * 4;  // K tile
-  b += static_cast<size_t>(D) * w * 4;                // comp / prefix maxima
+  b += static_cast<size_t>(D + 1) * w * 4;            // comp / prefix maxima (padded rows)
   b += 4 * static_cast<size_t>(D) * 4;                // capq, sig, rank, carry
   b += 2 * static_cast<size_t>(w) * 4;                // slot, argA
   b += 16;                                            // alignment slack
@@ -1009,7 +1012,7 @@ struct SnapWs {
   Unit *units;
   int32_t *ord, *sp, *su;
   int32_t *sig, *rank_of, *capq;
-  uint32_t *carry;  // [D][T2]
+  uint32_t *carry;  // [T2][D]
   uint32_t *kmax;   // [D][ceil(H/16)], used when the caller passes none
   int64_t max_units;
 };

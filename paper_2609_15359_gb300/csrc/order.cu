@@ -11,10 +11,15 @@
 //     non-promoted entry: promoted entries need no primary key because the
 //     arrival order is already in place and the sort is stable;
 //   * a key of at most 32 bits is sorted as 32 bits, otherwise as 64 bits.
-// Kernels: a prep pass (validation, promoted flags, largest bound, entries
-// per decoder, arrival order check), a key pass (keys and every digit
-// histogram), a one-block plan (digit offsets, which passes run, buffers,
-// decoder segment offsets), then one sweep per digit: tiles of 4096 keys are
+// Kernels: a prep pass (validation, largest bound, entries per decoder,
+// arrival order check; its last block chooses the form), a key pass, a
+// one-block plan (digit offsets, which passes run, buffers, decoder segment
+// offsets).
+// Segmented form (arrival non-decreasing along the index and every decoder's
+// queue within kSegMax entries): the key pass scatters each entry's index to
+// its decoder's segment, and one block per decoder sorts the segment in
+// shared memory on (not promoted, primary, index), a unique key.  Otherwise
+// one global sweep per digit: tiles of 4096 keys are
 // ranked stably in shared memory, each tile learns its offsets from earlier
 // tiles by decoupled look-back (one thread per digit walks back over packed
 // flag-and-count words until it meets an inclusive prefix), and writes out
@@ -45,7 +50,23 @@ struct OrderCounts {
   uint32_t h[kPasses][kRadix];
   uint32_t unsorted;   // arrival decreases somewhere along the index
   uint32_t max_bound;  // largest bound of a non-promoted entry
+  uint32_t segmented;  // decoder segments are sorted in shared memory
+  uint32_t nitems;     // segments to sort
+  uint32_t done_blocks;  // prep blocks finished
 };
+
+// Segmented form: when arrival is non-decreasing along the index (so arrival
+// order is index order) and every decoder's queue fits in shared memory, the
+// entries are scattered to their decoder's segment in any order and each
+// segment is sorted by one block on the key (not promoted, primary, index),
+// which is unique, so no pass has to be stable across blocks.
+constexpr int kSegThreads = 512;
+constexpr int kSegIPT = 11;
+constexpr int kSegMax = kSegThreads * kSegIPT;  // entries of the largest segment
+constexpr int kSegWarps = kSegThreads / 32;
+__device__ __forceinline__ int index_bits(int64_t N) {
+  return N > 1 ? 64 - __clzll(static_cast<unsigned long long>(N - 1)) : 1;
+}
 
 struct OrderPlan {
   int32_t active[kPasses];
@@ -75,15 +96,78 @@ __device__ __forceinline__ void warp_count(uint32_t *hist, int b, bool valid) {
 
 __device__ __forceinline__ int bit_width(uint32_t x) { return x ? 32 - __clz(x) : 0; }
 
+// Segmented form, step 1 (one block, run by the last prep block): decoder
+// segment offsets, one sort item per non-empty queue, and the choice of form
+// (arrival already in index order and no queue longer than kSegMax).
+__device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_count,
+                               int64_t *seg_off, int64_t *item_off, int32_t *item_n) {
+  __shared__ long long s_w[32];
+  __shared__ int s_bw[32];
+  __shared__ long long s_carry;
+  __shared__ int s_bcarry;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x;
+  if (t == 0) {
+    s_carry = 0;
+    s_bcarry = 0;
+  }
+  __syncthreads();
+  for (int base = 0; base <= D; base += nt) {
+    const int k = base + t;
+    const long long c = k < D ? __ldcg(dec_count + k) : 0;
+    const int big = c > kSegMax ? 1 : 0;
+    long long incl = c;
+    int bincl = big;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const long long y = __shfl_up_sync(0xffffffffu, incl, off);
+      const int by = __shfl_up_sync(0xffffffffu, bincl, off);
+      if (lane >= off) {
+        incl += y;
+        bincl += by;
+      }
+    }
+    if (lane == 31) {
+      s_w[warp] = incl;
+      s_bw[warp] = bincl;
+    }
+    __syncthreads();
+    long long wb = 0;
+    int bwb = 0;
+    for (int w = 0; w < warp; ++w) {
+      wb += s_w[w];
+      bwb += s_bw[w];
+    }
+    const long long carry = s_carry;
+    const int bcarry = s_bcarry;
+    const long long start = carry + wb + incl - c;
+    if (k <= D) seg_off[k] = start;
+    if (k < D && c > 0 && !big) {
+      const uint32_t it = atomicAdd(&counts->nitems, 1u);
+      item_off[it] = start;
+      item_n[it] = static_cast<int32_t>(c);
+    }
+    __syncthreads();
+    if (t == nt - 1) {
+      s_carry = carry + wb + incl;
+      s_bcarry = bcarry + bwb + bincl;
+    }
+    __syncthreads();
+  }
+  if (t == 0)
+    counts->segmented = (__ldcg(&counts->unsorted) == 0 && s_bcarry == 0) ? 1u : 0u;
+}
+
 // Pass 1: validation, largest non-promoted bound, entries per decoder, and
 // whether arrival is non-decreasing.
 __global__ void __launch_bounds__(512)
 order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
-                  uint32_t *dec_count, int32_t *status) {
+                  uint32_t *dec_count, int32_t *status, int64_t *seg_off, int64_t *item_off,
+                  int32_t *item_n) {
   pdl_prologue();
   __shared__ uint32_t s_dec[kDecSmem];
+  __shared__ bool s_last;
   const bool dec_smem = D <= kDecSmem;
   if (dec_smem)
     for (int i = threadIdx.x; i < D; i += blockDim.x) s_dec[i] = 0;
@@ -134,6 +218,15 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
   if (dec_smem)
     for (int i = threadIdx.x; i < D; i += blockDim.x)
       if (s_dec[i]) atomicAdd(&dec_count[i], s_dec[i]);
+  // the last block to finish plans the segmented form
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(&counts->done_blocks, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n);
+  }
 }
 
 // Pass 2: keys in the compact layout and the histograms of every digit.
@@ -141,8 +234,43 @@ __global__ void __launch_bounds__(512)
 order_keys_kernel(int64_t N, int D, int dbits, const int32_t *__restrict__ dec,
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
-                  unsigned long long *hi_orig, unsigned long long *keyA, uint32_t *valA) {
+                  unsigned long long *hi_orig, unsigned long long *keyA, uint32_t *valA,
+                  const int64_t *seg_off, uint32_t *dec_cursor) {
   pdl_prologue();
+  if (*reinterpret_cast<volatile uint32_t *>(&counts->segmented)) {
+    // Each entry's index goes to a free slot of its decoder's segment.  A
+    // round of kU entries per thread issues its loads and its (warp-combined)
+    // slot claims together, so the claims' latency overlaps.
+    constexpr int kU = 4;
+    const int lane = threadIdx.x & 31;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x * kU;
+    for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x * kU; i0 < N; i0 += stride) {
+      int d[kU];
+#pragma unroll
+      for (int q = 0; q < kU; ++q) {
+        const int64_t i = i0 + q * blockDim.x + threadIdx.x;
+        d[q] = i < N ? __ldg(dec + i) : -1;
+        if (i < N && (d[q] < 0 || d[q] >= D)) d[q] = 0;  // out-of-domain entries were flagged
+      }
+      uint32_t slot[kU];
+      unsigned peers[kU];
+#pragma unroll
+      for (int q = 0; q < kU; ++q) {
+        peers[q] = __match_any_sync(0xffffffffu, d[q]);
+        slot[q] = 0;
+        if (d[q] >= 0 && lane == __ffs(peers[q]) - 1)
+          slot[q] = atomicAdd(&dec_cursor[d[q]], static_cast<uint32_t>(__popc(peers[q])));
+      }
+#pragma unroll
+      for (int q = 0; q < kU; ++q) {
+        const uint32_t base = __shfl_sync(0xffffffffu, slot[q], __ffs(peers[q]) - 1);
+        const int64_t i = i0 + q * blockDim.x + threadIdx.x;
+        if (d[q] >= 0)
+          valA[seg_off[d[q]] + base + __popc(peers[q] & lanemask_lt())] = static_cast<uint32_t>(i);
+      }
+    }
+    return;
+  }
   __shared__ uint32_t sh[kPasses][kRadix];
   for (int i = threadIdx.x; i < kPasses * kRadix; i += blockDim.x) (&sh[0][0])[i] = 0;
   __syncthreads();
@@ -210,6 +338,18 @@ order_plan_kernel(int64_t N, int D, int dbits, const OrderCounts *counts, OrderP
   __shared__ int s_trivial[kPasses];
   __shared__ long long s_carry;
   const int b = threadIdx.x, lane = b & 31, warp = b >> 5;
+  if (*reinterpret_cast<const volatile uint32_t *>(&counts->segmented)) {
+    // segment offsets are already written; no global pass runs
+    if (b == 0) {
+      for (int p = 0; p < kPasses; ++p) {
+        plan->active[p] = 0;
+        plan->ordinal[p] = -1;
+      }
+      plan->gather_buf = -1;
+      plan->npasses = -1;  // neither passes nor the identity order
+    }
+    return;
+  }
   uint32_t cnt[kPasses];  // all loads first
 #pragma unroll
   for (int p = 0; p < kPasses; ++p) cnt[p] = counts->h[p][b];
@@ -298,6 +438,145 @@ order_plan_kernel(int64_t N, int D, int dbits, const OrderCounts *counts, OrderP
     __syncthreads();
     if (b == kRadix - 1) s_carry = carry + wb + incl;
     __syncthreads();
+  }
+}
+
+struct SegSmem {
+  unsigned long long key[2][kSegMax];
+  uint32_t hw[kSegWarps][kRadix];  // per-warp digit counts, then bases
+  uint32_t bin_start[kRadix];
+  uint32_t scan_w[kRadix / 32];
+  unsigned long long orv[kSegWarps], andv[kSegWarps];
+};
+
+// Segmented form, step 2: each sort item (one decoder's queue, at most
+// kSegMax entries) is sorted by one block on (not promoted,
+// promoted ? 0 : bound, index) with stable 8-bit LSD passes in shared
+// memory, skipping digits that do not vary, and its indices are written.
+// Blocks take items in turn until none is left.
+__global__ void __launch_bounds__(kSegThreads, 2)
+order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_off,
+                     const int32_t *item_n, const uint32_t *seg_idx,
+                     const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
+                     int32_t max_wait, int32_t *perm) {
+  pdl_prologue();
+  if (!counts->segmented) return;
+  extern __shared__ __align__(16) unsigned char seg_raw[];
+  SegSmem &sm = *reinterpret_cast<SegSmem *>(seg_raw);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int ub = counts->max_bound ? 32 - __clz(counts->max_bound) : 0;
+  const int ib = index_bits(N);
+  const int nbits = 1 + ub + ib;  // <= 1 + 31 + 31
+  const int nitems = static_cast<int>(counts->nitems);
+  for (int item = blockIdx.x; item < nitems; item += gridDim.x) {
+    const int64_t off = item_off[item];
+    const int n = item_n[item];
+    unsigned long long orv = 0, andv = ~0ull;
+    {
+      uint32_t idx[kSegIPT];  // every index load, then every gather, in flight together
+      int32_t u[kSegIPT], w[kSegIPT];
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it) {
+        const int x = it * kSegThreads + tid;
+        idx[it] = x < n ? seg_idx[off + x] : 0u;
+      }
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it) {
+        const int x = it * kSegThreads + tid;
+        u[it] = x < n ? __ldg(bound + idx[it]) : 0;
+        w[it] = x < n ? __ldg(wait + idx[it]) : 0;
+      }
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it) {
+        const int x = it * kSegThreads + tid;
+        if (x < n) {
+          const unsigned long long np = w[it] > max_wait ? 0ull : 1ull;
+          const unsigned long long prim = np ? static_cast<unsigned long long>(u[it] < 0 ? 0 : u[it]) : 0ull;
+          const unsigned long long key = (np << (ub + ib)) | (prim << ib) | idx[it];
+          sm.key[0][x] = key;
+          orv |= key;
+          andv &= key;
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      orv |= __shfl_xor_sync(0xffffffffu, orv, o);
+      andv &= __shfl_xor_sync(0xffffffffu, andv, o);
+    }
+    if (lane == 0) {
+      sm.orv[warp] = orv;
+      sm.andv[warp] = andv;
+    }
+    __syncthreads();
+    unsigned long long diff = 0;
+    {
+      unsigned long long o = 0, a = ~0ull;
+      for (int w = 0; w < kSegWarps; ++w) {
+        o |= sm.orv[w];
+        a &= sm.andv[w];
+      }
+      diff = o ^ a;  // bits that differ between keys of this segment
+    }
+    int cur = 0;
+    for (int shift = 0; shift < nbits; shift += 8) {
+      if (((diff >> shift) & 255ull) == 0) continue;  // same digit everywhere: order unchanged
+      for (int i = tid; i < kSegWarps * kRadix; i += kSegThreads) (&sm.hw[0][0])[i] = 0;
+      __syncthreads();
+      // rank within the warp, stable in item order (warp-major, then item, then lane)
+      uint32_t dr[kSegIPT];  // digit << 16 | rank within the warp's items of that digit
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it) {
+        const int x = warp * (32 * kSegIPT) + it * 32 + lane;
+        const bool valid = x < n;
+        const int d = valid ? static_cast<int>((sm.key[cur][x] >> shift) & 255ull) : kRadix;
+        const unsigned peers = __match_any_sync(0xffffffffu, d);
+        uint32_t c = 0;
+        if (valid) c = sm.hw[warp][d];
+        __syncwarp();
+        if (valid && lane == __ffs(peers) - 1) sm.hw[warp][d] = c + __popc(peers);
+        __syncwarp();
+        dr[it] = (static_cast<uint32_t>(d) << 16) | (c + __popc(peers & lanemask_lt()));
+      }
+      __syncthreads();
+      // per digit: exclusive scan over warps; then over digits
+      uint32_t tot = 0;
+      if (tid < kRadix) {
+        for (int w = 0; w < kSegWarps; ++w) {
+          const uint32_t c = sm.hw[w][tid];
+          sm.hw[w][tid] = tot;
+          tot += c;
+        }
+        uint32_t incl = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        if (lane == 31) sm.scan_w[warp] = incl;
+        tot = incl - tot;  // exclusive within the warp
+      }
+      __syncthreads();
+      if (tid < kRadix) {
+        uint32_t wb = 0;
+        for (int w = 0; w < warp; ++w) wb += sm.scan_w[w];
+        sm.bin_start[tid] = wb + tot;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it) {
+        const int x = warp * (32 * kSegIPT) + it * 32 + lane;
+        if (x < n) {
+          const int d = static_cast<int>(dr[it] >> 16);
+          sm.key[cur ^ 1][sm.bin_start[d] + sm.hw[warp][d] + (dr[it] & 0xffffu)] = sm.key[cur][x];
+        }
+      }
+      __syncthreads();
+      cur ^= 1;
+    }
+    const unsigned long long imask = (1ull << ib) - 1;
+    for (int x = tid; x < n; x += kSegThreads) perm[off + x] = static_cast<int32_t>(sm.key[cur][x] & imask);
+    __syncthreads();  // the next item reuses shared memory
   }
 }
 
@@ -514,10 +793,13 @@ order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *k
 struct OrderWs {
   OrderCounts *counts;
   uint32_t *dec_count;
+  uint32_t *dec_cursor;  // segmented form: slots taken per decoder
   uint32_t *tickets;
   unsigned long long *state;  // [2][tiles][256] look-back words
   size_t zero_bytes;  // counts .. state buffer 0 are contiguous and zeroed per call
   OrderPlan *plan;
+  int64_t *item_off;  // [D] sort items (non-empty queues)
+  int32_t *item_n;
   unsigned long long *hi_orig, *keyA, *keyB;
   uint32_t *valA, *valB;
 };
@@ -528,10 +810,13 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   const size_t zero_begin = (c.off + kAlign - 1) / kAlign * kAlign;
   w.counts = c.take<OrderCounts>(1);
   w.dec_count = c.take<uint32_t>(static_cast<size_t>(D));
+  w.dec_cursor = c.take<uint32_t>(static_cast<size_t>(D));
   w.tickets = c.take<uint32_t>(kPasses);
   w.state = c.take<unsigned long long>(static_cast<size_t>(2) * tiles * kRadix);
   w.zero_bytes = c.off - zero_begin - static_cast<size_t>(tiles) * kRadix * sizeof(unsigned long long);
   w.plan = c.take<OrderPlan>(1);
+  w.item_off = c.take<int64_t>(static_cast<size_t>(D));
+  w.item_n = c.take<int32_t>(static_cast<size_t>(D));
   const size_t n = static_cast<size_t>(N > 0 ? N : 1);
   w.hi_orig = c.take<unsigned long long>(n);
   w.keyA = c.take<unsigned long long>(n);
@@ -575,14 +860,22 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   const int64_t tiles = std::max<int64_t>(1, (N + kTile - 1) / kTile);
   if (N > 0) {
     const int g = static_cast<int>(std::min<int64_t>((N + 2047) / 2048, 2LL * sms));
-    launch_pdl(order_prep_kernel, g, 512, 0, s, N, D, dec, bound, wait, arrival, max_wait, w.counts,
-                                        w.dec_count, status);
-    launch_pdl(order_keys_kernel, g, 512, 0, s, N, D, dbits, dec, bound, wait, arrival, max_wait, w.counts,
-                                        w.hi_orig, w.keyA, w.valA);
+    launch_pdl(order_prep_kernel, g, 512, 0, s, N, D, dec, bound, wait, arrival, max_wait,
+               w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n);
+    launch_pdl(order_keys_kernel, g, 512, 0, s, N, D, dbits, dec, bound, wait, arrival, max_wait,
+               w.counts, w.hi_orig, w.keyA, w.valA, seg_off_out, w.dec_cursor);
   }
-  launch_pdl(order_plan_kernel, 1, kRadix, 0, s, N, D, dbits, w.counts, w.plan, w.dec_count, seg_off_out);
+  launch_pdl(order_plan_kernel, 1, kRadix, 0, s, N, D, dbits, w.counts, w.plan, w.dec_count,
+             seg_off_out);
   MAPS_TRY(launch_ok());
   if (N == 0) return MAPS_OK;
+  const size_t seg_smem = sizeof(SegSmem);
+  MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_segsort_kernel,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        static_cast<int>(seg_smem))));
+  launch_pdl(order_segsort_kernel, static_cast<unsigned>(std::min<int64_t>(D, 2LL * sms)),
+             kSegThreads, seg_smem, s, N, w.counts, w.item_off, w.item_n, w.valA, bound, wait,
+             max_wait, perm_out);
   const size_t smem = sizeof(PassSmem);
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_pass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));

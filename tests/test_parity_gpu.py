@@ -439,7 +439,11 @@ def test_dispatch_errors(M, ws, oracle):
 @pytest.mark.parametrize("N,D,sorted_arrival", [(0, 3, True), (1, 1, True), (2, 2, False),
                                                 (100, 3, False), (4096, 8, True), (4097, 8, False),
                                                 (50000, 64, True), (50001, 300, False),
-                                                (300000, 256, False), (1000, 70000, True)])
+                                                (300000, 256, False), (1000, 70000, True),
+                                                # one decoder's queue at, and past, the most a
+                                                # block sorts in shared memory
+                                                (5632, 1, True), (5633, 1, True),
+                                                (20000, 2, True), (300000, 256, True)])
 def test_order_random(M, ws, oracle, N, D, sorted_arrival):
     rng = np.random.default_rng(N + D)
     dec = rng.integers(0, D, N).astype(np.int32)
