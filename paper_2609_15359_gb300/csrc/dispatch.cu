@@ -477,7 +477,9 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
     for (int e = tid; e < D * W2; e += kMainThreads) {
       const int r = e / W2, c = e - (e / W2) * W2;
       const int64_t t = t0 + c;
-      kb[e] = t < H ? static_cast<uint32_t>(a.K[static_cast<int64_t>(r) * H + t]) : 0u;
+      // 32-column tiles use the layout of a 128-byte swizzled TMA copy
+      const int at = W2 == 32 ? r * 32 + ((((c >> 2) ^ (r & 7))) << 2) + (c & 3) : e;
+      kb[at] = t < H ? static_cast<uint32_t>(a.K[static_cast<int64_t>(r) * H + t]) : 0u;
     }
   }
   __syncthreads();
@@ -505,43 +507,72 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   const int nslots = s_nslots;
 
   // --- prefix maximum of K + t along each row; keep the needed columns ----
-  constexpr int seg = W2 / 16;  // cells per row segment; 16 segments per row
-  const int items = ((D * 16 + kMainThreads - 1) / kMainThreads) * kMainThreads;
   bool neg = false;
-  for (int it = tid; it < items; it += kMainThreads) {
-    const int row = it >> 4, sg = it & 15;
-    const bool live_row = row < D;
-    uint32_t v[seg];
-    uint32_t run = 0;
-#pragma unroll
-    for (int j = 0; j < seg; ++j) {
-      const int c = sg * seg + j;
-      const int64_t t = t0 + c;
-      uint32_t x = 0;
-      if (live_row && t < H) {
-        const uint32_t raw = kb[static_cast<size_t>(row) * W2 + c];
-        if (static_cast<int32_t>(raw) < 0) neg = true;
-        x = raw + static_cast<uint32_t>(t);  // K + t < 2^32
-      }
-      run = x > run ? x : run;
-      v[j] = run;
-    }
-    uint32_t incl = run;
-#pragma unroll
-    for (int off = 1; off < 16; off <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off, 16);
-      if (sg >= off) incl = y > incl ? y : incl;
-    }
-    uint32_t excl = __shfl_up_sync(0xffffffffu, incl, 1, 16);
-    if (sg == 0) excl = 0;
-    if (live_row) {
-      const uint32_t cr = s_carry[row];
+  if constexpr (W2 == 32) {
+    // One thread per row.  The tile is stored with 128-byte swizzling: the
+    // 16-byte chunk ch of row r sits at chunk ch ^ (r & 7) of its 128-byte
+    // row, so a warp loading one chunk of 32 rows hits every bank once per
+    // quarter-warp.  The running maximum starts from the row's carry.
+    for (int row = tid; row < D; row += kMainThreads) {
+      const uint4 *rp = reinterpret_cast<const uint4 *>(kb + static_cast<size_t>(row) * 32);
+      uint32_t run = s_carry[row];
       const int rk = s_rank[row];
-      excl = excl > cr ? excl : cr;
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) {
+        const uint4 q = rp[ch ^ (row & 7)];
+        const uint32_t raw[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int c = ch * 4 + e;
+          const int64_t t = t0 + c;
+          if (t < H) {
+            if (static_cast<int32_t>(raw[e]) < 0) neg = true;
+            const uint32_t x = raw[e] + static_cast<uint32_t>(t);  // K + t < 2^32
+            run = x > run ? x : run;
+          }
+          const int sl = s_slot[c];
+          if (sl >= 0) comp[static_cast<size_t>(sl) * Dp + rk] = run;
+        }
+      }
+    }
+  } else {
+    constexpr int seg = W2 / 16;  // cells per row segment; 16 segments per row
+    const int items = ((D * 16 + kMainThreads - 1) / kMainThreads) * kMainThreads;
+    for (int it = tid; it < items; it += kMainThreads) {
+      const int row = it >> 4, sg = it & 15;
+      const bool live_row = row < D;
+      uint32_t v[seg];
+      uint32_t run = 0;
 #pragma unroll
       for (int j = 0; j < seg; ++j) {
-        const int sl = s_slot[sg * seg + j];
-        if (sl >= 0) comp[static_cast<size_t>(sl) * Dp + rk] = v[j] > excl ? v[j] : excl;
+        const int c = sg * seg + j;
+        const int64_t t = t0 + c;
+        uint32_t x = 0;
+        if (live_row && t < H) {
+          const uint32_t raw = kb[static_cast<size_t>(row) * W2 + c];
+          if (static_cast<int32_t>(raw) < 0) neg = true;
+          x = raw + static_cast<uint32_t>(t);  // K + t < 2^32
+        }
+        run = x > run ? x : run;
+        v[j] = run;
+      }
+      uint32_t incl = run;
+#pragma unroll
+      for (int off = 1; off < 16; off <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off, 16);
+        if (sg >= off) incl = y > incl ? y : incl;
+      }
+      uint32_t excl = __shfl_up_sync(0xffffffffu, incl, 1, 16);
+      if (sg == 0) excl = 0;
+      if (live_row) {
+        const uint32_t cr = s_carry[row];
+        const int rk = s_rank[row];
+        excl = excl > cr ? excl : cr;
+#pragma unroll
+        for (int j = 0; j < seg; ++j) {
+          const int sl = s_slot[sg * seg + j];
+          if (sl >= 0) comp[static_cast<size_t>(sl) * Dp + rk] = v[j] > excl ? v[j] : excl;
+        }
       }
     }
   }
@@ -1100,7 +1131,8 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
     cuuint32_t estr[2] = {1, 1};
     const CUresult r = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_INT32, 2, const_cast<int32_t *>(K), dims,
                            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                           CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                           g.W2 == 32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) use_tma = false;
   }

@@ -308,7 +308,10 @@ def check_dispatch(M, ws, oracle, mode, D, H, K, cap, Q, cp, cb, S=1, res=None):
 @pytest.mark.parametrize("D,H,J", [(1, 1, 1), (1, 9, 33), (2, 8, 40), (3, 100, 700), (5, 511, 1000),
                                    (17, 4100, 3000), (64, 4096, 5000), (255, 1000, 3000),
                                    (256, 8192, 6000), (257, 2048, 2000), (300, 777, 1500),
-                                   (1024, 1024, 2000)])
+                                   (1024, 1024, 2000),
+                                   # 32-column tiles (129..256 decoders), copied by TMA and,
+                                   # with H not a multiple of 4, by plain loads
+                                   (129, 3000, 2000), (200, 1001, 2000)])
 def test_dispatch_snapshot_random(M, ws, oracle, D, H, J):
     rng = np.random.default_rng(D * 7919 + H)
     off, p, g, U = random_residents(rng, D, H, 40)
