@@ -217,8 +217,9 @@ class Step:
         n_hi = min(8, (dbits + 1 + 31 + 7) // 8)
         # calibrate 4 (three select passes, bounds); occupancy 2 (bucket, tile);
         # dispatch 5 (carry scan, bin count / scan / scatter, main); order
-        # prep, keys, plan, 4 arrival passes, gather, n_hi key passes, identity
-        self.kernels_per_step = 4 + 2 + 5 + (3 + 4 + 1 + n_hi + 1)
+        # prep, keys, plan, segment sort, 4 arrival passes, gather, n_hi key
+        # passes, identity
+        self.kernels_per_step = 4 + 2 + 5 + (4 + 4 + 1 + n_hi + 1)
 
     def run(self, ev=None):
         M, R = self.M, self.R
