@@ -104,6 +104,27 @@ inline void launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   (void)cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
 }
 
+// A cooperative launch (every block resident at once, so the grid may wait at
+// grid-wide barriers).  It is stream-ordered without programmatic overlap, so
+// none of its blocks is placed while an earlier grid still holds resources.
+// The caller sizes the grid within the occupancy limit; a launch the device
+// refuses is reported.
+template <typename... KArgs, typename... Args>
+inline int launch_coop(void (*kernel)(KArgs...), int64_t grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid < 1 ? 1 : grid));
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cuda_ok(cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...));
+}
+
 inline bool aligned(const void *p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;
 }

@@ -15,20 +15,25 @@
 // arrival order check; its last block chooses the form), a key pass, a
 // one-block plan (digit offsets, which passes run, buffers, decoder segment
 // offsets).
-// Segmented form (arrival non-decreasing along the index and every decoder's
-// queue within kSegMax entries): the key pass scatters each entry's index to
-// its decoder's segment, and one block per decoder sorts the segment in
-// shared memory on (not promoted, primary, index), a unique key.  Otherwise
-// one global sweep per digit: tiles of 4096 keys are
+// Segmented form (arrival non-decreasing along the index): the key pass
+// scatters each entry's index to its decoder's segment; one block sorts a
+// segment of at most kSegMax entries in shared memory on (not promoted,
+// primary, index), a unique key, and a longer segment is sorted as chunks of
+// kSegMax whose runs are merged pairwise level by level.  Otherwise one
+// global sweep per digit: tiles of 4096 keys are
 // ranked stably in shared memory, each tile learns its offsets from earlier
 // tiles by decoupled look-back (one thread per digit walks back over packed
 // flag-and-count words until it meets an inclusive prefix), and writes out
 // bin by bin.  Passes the plan marks inactive return at once, so the host
 // never waits on the device.
+#include <cooperative_groups.h>
+
 #include "maps_internal.cuh"
 
 #include <algorithm>
 #include <mutex>
+
+namespace cg = cooperative_groups;
 
 namespace maps {
 namespace {
@@ -51,7 +56,9 @@ struct OrderCounts {
   uint32_t unsorted;   // arrival decreases somewhere along the index
   uint32_t max_bound;  // largest bound of a non-promoted entry
   uint32_t segmented;  // decoder segments are sorted in shared memory
-  uint32_t nitems;     // segments to sort
+  uint32_t nitems;     // segments and chunks to sort
+  uint32_t nmtiles;    // merge tiles of the long queues
+  uint32_t max_levels; // merge levels the longest queue needs
   uint32_t done_blocks;  // prep blocks finished
 };
 
@@ -62,7 +69,21 @@ struct OrderCounts {
 // which is unique, so no pass has to be stable across blocks.
 constexpr int kSegThreads = 512;
 constexpr int kSegIPT = 11;
-constexpr int kSegMax = kSegThreads * kSegIPT;  // entries of the largest segment
+constexpr int kSegMax = kSegThreads * kSegIPT;  // entries one block sorts
+// A longer queue is sorted as chunks of kSegMax entries, whose sorted runs are
+// then merged pairwise, level by level, in tiles of kMergeTile outputs
+// (kMergeTile divides kSegMax, so no tile straddles two runs).
+constexpr int kMergeTile = 512;
+constexpr int kMergeThreads = 256;
+static_assert(kSegMax % kMergeTile == 0, "merge tiles align with runs");
+
+// Merge levels a queue of n entries needs: ceil(log2(ceil(n / kSegMax))).
+__host__ __device__ __forceinline__ int merge_levels(int64_t n) {
+  int64_t runs = (n + kSegMax - 1) / kSegMax;
+  int l = 0;
+  while ((int64_t(1) << l) < runs) ++l;
+  return l;
+}
 constexpr int kSegWarps = kSegThreads / 32;
 __device__ __forceinline__ int index_bits(int64_t N) {
   return N > 1 ? 64 - __clzll(static_cast<unsigned long long>(N - 1)) : 1;
@@ -97,10 +118,14 @@ __device__ __forceinline__ void warp_count(uint32_t *hist, int b, bool valid) {
 __device__ __forceinline__ int bit_width(uint32_t x) { return x ? 32 - __clz(x) : 0; }
 
 // Segmented form, step 1 (one block, run by the last prep block): decoder
-// segment offsets, one sort item per non-empty queue, and the choice of form
-// (arrival already in index order and no queue longer than kSegMax).
+// segment offsets, the sort items (a queue of at most kSegMax entries is one
+// item whose sort writes the order; a longer one gives one item per chunk,
+// marked by a negative count, whose sort writes keys for the merges) and the
+// merge tiles of the long queues; the form applies when arrival is already
+// in index order.
 __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_count,
-                               int64_t *seg_off, int64_t *item_off, int32_t *item_n) {
+                               int64_t *seg_off, int64_t *item_off, int32_t *item_n,
+                               int64_t *mt_off, int32_t *mt_n, int32_t *mt_t) {
   __shared__ long long s_w[32];
   __shared__ int s_bw[32];
   __shared__ long long s_carry;
@@ -145,6 +170,21 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
       const uint32_t it = atomicAdd(&counts->nitems, 1u);
       item_off[it] = start;
       item_n[it] = static_cast<int32_t>(c);
+    } else if (k < D && big) {
+      const int nch = static_cast<int>((c + kSegMax - 1) / kSegMax);
+      const uint32_t it = atomicAdd(&counts->nitems, static_cast<uint32_t>(nch));
+      for (int j = 0; j < nch; ++j) {
+        item_off[it + j] = start + static_cast<int64_t>(j) * kSegMax;
+        item_n[it + j] = -static_cast<int32_t>(min(static_cast<long long>(kSegMax), c - static_cast<long long>(j) * kSegMax));
+      }
+      atomicMax(&counts->max_levels, static_cast<uint32_t>(merge_levels(c)));
+      const int ntl = static_cast<int>((c + kMergeTile - 1) / kMergeTile);
+      const uint32_t mt = atomicAdd(&counts->nmtiles, static_cast<uint32_t>(ntl));
+      for (int j = 0; j < ntl; ++j) {
+        mt_off[mt + j] = start;
+        mt_n[mt + j] = static_cast<int32_t>(c);
+        mt_t[mt + j] = j;
+      }
     }
     __syncthreads();
     if (t == nt - 1) {
@@ -153,8 +193,8 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
     }
     __syncthreads();
   }
-  if (t == 0)
-    counts->segmented = (__ldcg(&counts->unsorted) == 0 && s_bcarry == 0) ? 1u : 0u;
+  if (t == 0) counts->segmented = __ldcg(&counts->unsorted) == 0 ? 1u : 0u;
+  (void)s_bcarry;
 }
 
 // Pass 1: validation, largest non-promoted bound, entries per decoder, and
@@ -164,7 +204,7 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
                   uint32_t *dec_count, int32_t *status, int64_t *seg_off, int64_t *item_off,
-                  int32_t *item_n) {
+                  int32_t *item_n, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t) {
   pdl_prologue();
   __shared__ uint32_t s_dec[kDecSmem];
   __shared__ bool s_last;
@@ -225,7 +265,7 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
   __syncthreads();
   if (s_last) {
     __threadfence();
-    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n);
+    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, mt_off, mt_n, mt_t);
   }
 }
 
@@ -458,7 +498,7 @@ __global__ void __launch_bounds__(kSegThreads, 2)
 order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_off,
                      const int32_t *item_n, const uint32_t *seg_idx,
                      const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
-                     int32_t max_wait, int32_t *perm) {
+                     int32_t max_wait, int32_t *perm, unsigned long long *run_keys) {
   pdl_prologue();
   if (!counts->segmented) return;
   extern __shared__ __align__(16) unsigned char seg_raw[];
@@ -470,7 +510,8 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
   const int nitems = static_cast<int>(counts->nitems);
   for (int item = blockIdx.x; item < nitems; item += gridDim.x) {
     const int64_t off = item_off[item];
-    const int n = item_n[item];
+    const bool chunk = item_n[item] < 0;  // a chunk of a long queue: keys for the merges
+    const int n = chunk ? -item_n[item] : item_n[item];
     unsigned long long orv = 0, andv = ~0ull;
     {
       uint32_t idx[kSegIPT];  // every index load, then every gather, in flight together
@@ -575,8 +616,103 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
       cur ^= 1;
     }
     const unsigned long long imask = (1ull << ib) - 1;
-    for (int x = tid; x < n; x += kSegThreads) perm[off + x] = static_cast<int32_t>(sm.key[cur][x] & imask);
+    if (chunk)
+      for (int x = tid; x < n; x += kSegThreads) run_keys[off + x] = sm.key[cur][x];
+    else
+      for (int x = tid; x < n; x += kSegThreads) perm[off + x] = static_cast<int32_t>(sm.key[cur][x] & imask);
     __syncthreads();  // the next item reuses shared memory
+  }
+}
+
+// Segmented form, step 3: merge level `level` of the long queues.  Runs of
+// L = kSegMax << level sorted keys are merged pairwise from buf[level & 1]
+// into buf[(level + 1) & 1]; a queue needing fewer levels is left alone.
+// One block writes one tile of kMergeTile outputs: a merge-path search splits
+// the two runs at the tile's ends, the tile's inputs are staged in shared
+// memory, and each thread merges kMergeTile / kMergeThreads outputs after a
+// second search.  Keys are unique, so there are no ties.
+__device__ __forceinline__ int merge_path(const unsigned long long *A, int la,
+                                          const unsigned long long *B, int lb, int d) {
+  int lo = d > lb ? d - lb : 0, hi = d < la ? d : la;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (A[mid] < B[d - 1 - mid])
+      lo = mid + 1;
+    else
+      hi = mid;
+  }
+  return lo;  // outputs before d taken from A
+}
+
+// All merge levels and the final order in one cooperative launch: the grid
+// waits at a grid-wide barrier after each level.
+__device__ void merge_level(int level, int ntiles, const int64_t *mt_off, const int32_t *mt_n,
+                            const int32_t *mt_t, unsigned long long *bufA,
+                            unsigned long long *bufB) {
+  __shared__ unsigned long long s_a[kMergeTile], s_b[kMergeTile];
+  __shared__ int s_split[2];
+  const unsigned long long *src = (level & 1) ? bufB : bufA;
+  unsigned long long *dst = (level & 1) ? bufA : bufB;
+  const int64_t L = static_cast<int64_t>(kSegMax) << level;
+  for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    const int n = mt_n[tile];
+    if (level >= merge_levels(n)) continue;  // this queue is complete (uniform per block)
+    const int64_t off = mt_off[tile];
+    const int w0 = mt_t[tile] * kMergeTile, w1 = min(w0 + kMergeTile, n);
+    const int64_t pstart = (w0 / (2 * L)) * (2 * L);
+    const int64_t rest = n - pstart;  // entries from this pair's start to the queue's end
+    const int la = static_cast<int>(rest < L ? rest : L);
+    const int lb = static_cast<int>(rest > L ? (rest < 2 * L ? rest : 2 * L) - L : 0);
+    const unsigned long long *A = src + off + pstart, *B = A + la;
+    const int d0 = static_cast<int>(w0 - pstart), d1 = static_cast<int>(w1 - pstart);
+    if (threadIdx.x < 2) s_split[threadIdx.x] = merge_path(A, la, B, lb, threadIdx.x ? d1 : d0);
+    __syncthreads();
+    const int i0 = s_split[0], i1 = s_split[1];
+    const int j0 = d0 - i0, j1 = d1 - i1;
+    const int na = i1 - i0, nbb = j1 - j0;
+    for (int x = threadIdx.x; x < na; x += kMergeThreads) s_a[x] = A[i0 + x];
+    for (int x = threadIdx.x; x < nbb; x += kMergeThreads) s_b[x] = B[j0 + x];
+    __syncthreads();
+    constexpr int kPer = kMergeTile / kMergeThreads;
+    const int dt = threadIdx.x * kPer;
+    if (dt < na + nbb) {
+      int ia = merge_path(s_a, na, s_b, nbb, dt), ib = dt - ia;
+      unsigned long long *out = dst + off + pstart + d0;
+#pragma unroll
+      for (int q = 0; q < kPer; ++q) {
+        if (dt + q >= na + nbb) break;
+        const bool takeA = ib >= nbb || (ia < na && s_a[ia] < s_b[ib]);
+        out[dt + q] = takeA ? s_a[ia++] : s_b[ib++];
+      }
+    }
+    __syncthreads();  // the next tile reuses shared memory
+  }
+}
+
+__global__ void __launch_bounds__(kMergeThreads)
+order_merge_kernel(int64_t N, const OrderCounts *counts, const int64_t *mt_off,
+                   const int32_t *mt_n, const int32_t *mt_t, unsigned long long *bufA,
+                   unsigned long long *bufB, int32_t *perm) {
+  pdl_prologue();
+  // every block takes the same branch, so no block waits at a barrier alone
+  if (!counts->segmented || counts->nmtiles == 0) return;
+  cg::grid_group grid = cg::this_grid();
+  const int ntiles = static_cast<int>(counts->nmtiles);
+  const int levels = static_cast<int>(counts->max_levels);
+  for (int level = 0; level < levels; ++level) {
+    merge_level(level, ntiles, mt_off, mt_n, mt_t, bufA, bufB);
+    grid.sync();
+  }
+  // each long queue's final run becomes its order
+  const int ib = index_bits(N);
+  const unsigned long long imask = (1ull << ib) - 1;
+  for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    const int n = mt_n[tile];
+    const unsigned long long *src = (merge_levels(n) & 1) ? bufB : bufA;
+    const int64_t off = mt_off[tile];
+    const int w0 = mt_t[tile] * kMergeTile, w1 = min(w0 + kMergeTile, n);
+    for (int x = w0 + static_cast<int>(threadIdx.x); x < w1; x += kMergeThreads)
+      perm[off + x] = static_cast<int32_t>(src[off + x] & imask);
   }
 }
 
@@ -790,6 +926,17 @@ order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *k
                            ticket, status, sm);
 }
 
+// Blocks of the merge kernel that can be resident at once (its grid limit as
+// a cooperative launch).
+int64_t merge_grid() {
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, order_merge_kernel, kMergeThreads, 0) !=
+          cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  return static_cast<int64_t>(per_sm) * sm_count();
+}
+
 struct OrderWs {
   OrderCounts *counts;
   uint32_t *dec_count;
@@ -798,8 +945,11 @@ struct OrderWs {
   unsigned long long *state;  // [2][tiles][256] look-back words
   size_t zero_bytes;  // counts .. state buffer 0 are contiguous and zeroed per call
   OrderPlan *plan;
-  int64_t *item_off;  // [D] sort items (non-empty queues)
+  int64_t *item_off;  // sort items: queues and chunks of long queues
   int32_t *item_n;
+  int64_t *mt_off;    // merge tiles of the long queues
+  int32_t *mt_n, *mt_t;
+  int64_t nitems_max, ntiles_max;
   unsigned long long *hi_orig, *keyA, *keyB;
   uint32_t *valA, *valB;
 };
@@ -815,8 +965,13 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.state = c.take<unsigned long long>(static_cast<size_t>(2) * tiles * kRadix);
   w.zero_bytes = c.off - zero_begin - static_cast<size_t>(tiles) * kRadix * sizeof(unsigned long long);
   w.plan = c.take<OrderPlan>(1);
-  w.item_off = c.take<int64_t>(static_cast<size_t>(D));
-  w.item_n = c.take<int32_t>(static_cast<size_t>(D));
+  w.nitems_max = D + N / kSegMax + 1;
+  w.ntiles_max = N / kMergeTile + D + 1;
+  w.item_off = c.take<int64_t>(static_cast<size_t>(w.nitems_max));
+  w.item_n = c.take<int32_t>(static_cast<size_t>(w.nitems_max));
+  w.mt_off = c.take<int64_t>(static_cast<size_t>(w.ntiles_max));
+  w.mt_n = c.take<int32_t>(static_cast<size_t>(w.ntiles_max));
+  w.mt_t = c.take<int32_t>(static_cast<size_t>(w.ntiles_max));
   const size_t n = static_cast<size_t>(N > 0 ? N : 1);
   w.hi_orig = c.take<unsigned long long>(n);
   w.keyA = c.take<unsigned long long>(n);
@@ -861,7 +1016,8 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   if (N > 0) {
     const int g = static_cast<int>(std::min<int64_t>((N + 2047) / 2048, 2LL * sms));
     launch_pdl(order_prep_kernel, g, 512, 0, s, N, D, dec, bound, wait, arrival, max_wait,
-               w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n);
+               w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n, w.mt_off, w.mt_n,
+               w.mt_t);
     launch_pdl(order_keys_kernel, g, 512, 0, s, N, D, dbits, dec, bound, wait, arrival, max_wait,
                w.counts, w.hi_orig, w.keyA, w.valA, seg_off_out, w.dec_cursor);
   }
@@ -873,9 +1029,14 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_segsort_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(seg_smem))));
-  launch_pdl(order_segsort_kernel, static_cast<unsigned>(std::min<int64_t>(D, 2LL * sms)),
+  launch_pdl(order_segsort_kernel, static_cast<unsigned>(std::min<int64_t>(w.nitems_max, 2LL * sms)),
              kSegThreads, seg_smem, s, N, w.counts, w.item_off, w.item_n, w.valA, bound, wait,
-             max_wait, perm_out);
+             max_wait, perm_out, w.keyA);
+  if (N > kSegMax) {  // some queue may be longer than one block sorts
+    MAPS_TRY(launch_coop(order_merge_kernel, std::min<int64_t>(w.ntiles_max, merge_grid()),
+                         kMergeThreads, 0, s, N, w.counts, w.mt_off, w.mt_n, w.mt_t, w.keyA, w.keyB,
+                         perm_out));
+  }
   const size_t smem = sizeof(PassSmem);
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_pass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));

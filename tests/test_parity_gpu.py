@@ -446,7 +446,9 @@ def test_dispatch_errors(M, ws, oracle):
                                                 # one decoder's queue at, and past, the most a
                                                 # block sorts in shared memory
                                                 (5632, 1, True), (5633, 1, True),
-                                                (20000, 2, True), (300000, 256, True)])
+                                                (20000, 2, True), (300000, 256, True),
+                                                # a queue of 18 chunks: five merge levels
+                                                (100000, 1, True)])
 def test_order_random(M, ws, oracle, N, D, sorted_arrival):
     rng = np.random.default_rng(N + D)
     dec = rng.integers(0, D, N).astype(np.int32)
