@@ -216,10 +216,11 @@ class Step:
         dbits = (self.D - 1).bit_length()
         n_hi = min(8, (dbits + 1 + 31 + 7) // 8)
         # calibrate 4 (three select passes, bounds); occupancy 2 (bucket, tile);
-        # dispatch 5 (carry scan, bin count / scan / scatter, main); order
-        # prep, keys, plan, segment sort, 4 arrival passes, gather, n_hi key
-        # passes, identity
-        self.kernels_per_step = 4 + 2 + 5 + (4 + 4 + 1 + n_hi + 1)
+        # dispatch 4 (carry scan, bin count, bin scatter, main); order prep,
+        # keys, plan, segment sort, merge (more entries than one block sorts),
+        # 4 arrival passes, gather, n_hi key passes, identity
+        merge = 1 if R + J > 5632 else 0
+        self.kernels_per_step = 4 + 2 + 4 + (4 + merge + 4 + 1 + n_hi + 1)
 
     def run(self, ev=None):
         M, R = self.M, self.R

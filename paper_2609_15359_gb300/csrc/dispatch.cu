@@ -125,9 +125,35 @@ kmax_from_K_kernel(int D, int H, const int32_t *__restrict__ K, uint32_t *__rest
 // and after a block scan writes its tiles' carries contiguously.
 __global__ void __launch_bounds__(256)
 carry_scan_kernel(int D, int H, int W2, int T2, const uint32_t *__restrict__ kmax,
-                  uint32_t *__restrict__ carry) {
+                  uint32_t *__restrict__ carry, const int32_t *__restrict__ Q,
+                  const int32_t *__restrict__ cap, int32_t *sig, int32_t *rank_of,
+                  int32_t *capq, int32_t *status) {
   pdl_prologue();
   __shared__ uint32_t s_w[8];
+  __shared__ int s_rank;
+  {
+    // this decoder's position in (Q, index) order: the decoders before it
+    const int kk = blockIdx.x;
+    const int32_t qk = __ldg(Q + kk);
+    int r = 0;
+    for (int k2 = threadIdx.x; k2 < D; k2 += blockDim.x) {
+      const int32_t q2 = __ldg(Q + k2);
+      r += (q2 < qk) || (q2 == qk && k2 < kk);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) r += __shfl_xor_sync(0xffffffffu, r, off);
+    if (threadIdx.x == 0) s_rank = 0;
+    __syncthreads();
+    if ((threadIdx.x & 31) == 0) atomicAdd(&s_rank, r);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      const int32_t ck = __ldg(cap + kk);
+      if ((qk | ck) < 0) flag_error(status, MAPS_E_RANGE);
+      sig[s_rank] = kk;
+      rank_of[kk] = s_rank;
+      capq[s_rank] = ck;
+    }
+  }
   constexpr int kPer = 16;
   const int k = blockIdx.x;
   const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
@@ -197,12 +223,21 @@ __device__ __forceinline__ unsigned lanemask_lt() {
 // Grid-stride loops run in whole warps.
 constexpr int kBinSmem = 4096;
 
+struct Unit {
+  int32_t tile, start, count, pad;
+};
+
+__device__ void bin_scan_block(int T2, const uint32_t *tcount, uint32_t *toff, Unit *units,
+                               uint32_t *nunits);
+
 __global__ void __launch_bounds__(1024)
 bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ cp,
                  const int32_t *__restrict__ cb, uint32_t *tcount, int32_t *choice,
-                 int64_t *headroom, int32_t *status) {
+                 int64_t *headroom, int32_t *status, uint32_t *ticket, uint32_t *toff,
+                 Unit *units, uint32_t *nunits) {
   pdl_prologue();
   __shared__ uint32_t s_h[kBinSmem];
+  __shared__ bool s_last;
   const bool local = T2 <= kBinSmem;
   if (local)
     for (int i = threadIdx.x; i < T2; i += blockDim.x) s_h[i] = 0;
@@ -236,47 +271,30 @@ bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ c
       if (s_h[t]) atomicAdd(&tcount[t], s_h[t]);
     }
   }
+  // the last block to finish turns the counts into offsets and work units
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    bin_scan_block(T2, tcount, toff, units, nunits);
+  }
 }
 
-struct Unit {
-  int32_t tile, start, count, pad;
-};
-
-// One block: tile offsets toff[0..T2], the work units (a tile with c
-// candidates gives ceil(c / kUnitCands) units; the unit count goes to
-// *nunits), and the decoders' queue order (Q, then index): sig maps queue
-// position to decoder, rank the reverse, capq holds capacities by position.
-__global__ void __launch_bounds__(1024)
-bin_scan_kernel(int T2, const uint32_t *tcount, uint32_t *toff, Unit *units, uint32_t *nunits,
-                int D, const int32_t *__restrict__ Q, const int32_t *__restrict__ cap,
-                int32_t *sig, int32_t *rank_of, int32_t *capq, int32_t *status) {
-  pdl_prologue();
+// Run by the last bin_count block (1024 threads): tile offsets toff[0..T2]
+// and the work units (a tile with c candidates gives ceil(c / kUnitCands)
+// units; the unit count goes to *nunits).
+__device__ void bin_scan_block(int T2, const uint32_t *tcount, uint32_t *toff, Unit *units,
+                               uint32_t *nunits) {
   __shared__ uint32_t s_w[2][32];
   __shared__ uint32_t s_carry[2];
-  __shared__ int32_t s_q[kMaxD];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  bool bad = false;
-  for (int k = threadIdx.x; k < D; k += blockDim.x) {
-    s_q[k] = Q[k];
-    if ((s_q[k] | cap[k]) < 0) bad = true;
-  }
-  if (bad) flag_error(status, MAPS_E_RANGE);
   if (threadIdx.x == 0) s_carry[0] = s_carry[1] = 0;
   __syncthreads();
-  for (int k = threadIdx.x; k < D; k += blockDim.x) {
-    const int32_t qk = s_q[k];
-    int r = 0;
-    for (int k2 = 0; k2 < D; ++k2) {
-      const int32_t q2 = s_q[k2];
-      r += (q2 < qk) || (q2 == qk && k2 < k);
-    }
-    sig[r] = k;
-    rank_of[k] = r;
-    capq[r] = cap[k];
-  }
   for (int base = 0; base < T2; base += 1024) {
     const int i = base + threadIdx.x;
-    const uint32_t c = i < T2 ? tcount[i] : 0u;
+    const uint32_t c = i < T2 ? __ldcg(tcount + i) : 0u;
     const uint32_t nu = (c + kUnitCands - 1) / kUnitCands;
     uint32_t ic = c, iu = nu;
 #pragma unroll
@@ -1037,7 +1055,7 @@ SnapGeom snap_geom(int D, int H) {
 }
 
 struct SnapWs {
-  uint32_t *zero;  // tcount[T2], tcursor[T2], nunits (zeroed per call)
+  uint32_t *zero;  // tcount[T2], tcursor[T2], nunits, ticket (zeroed per call)
   size_t zero_words;
   uint32_t *toff;
   Unit *units;
@@ -1050,7 +1068,7 @@ struct SnapWs {
 
 SnapWs carve_snap(Carve &c, int D, int H, int T2, int64_t J) {
   SnapWs w;
-  w.zero_words = 2 * static_cast<size_t>(T2) + 1;
+  w.zero_words = 2 * static_cast<size_t>(T2) + 2;  // tcount, tcursor, nunits, ticket
   w.zero = c.take<uint32_t>(w.zero_words);
   w.toff = c.take<uint32_t>(static_cast<size_t>(T2) + 1);
   w.max_units = static_cast<int64_t>(T2) + (J + kUnitCands - 1) / kUnitCands;
@@ -1103,6 +1121,7 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
   int32_t *status = status_word(ws);
   uint32_t *tcount = w.zero, *tcursor = w.zero + g.T2;
   uint32_t *nunits = w.zero + 2 * static_cast<size_t>(g.T2);
+  uint32_t *ticket = nunits + 1;  // bin_count blocks finished
   MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zero, 0, w.zero_words * 4, s)));
   const int sms = sm_count();
   if (kmax == nullptr) {
@@ -1111,12 +1130,13 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
     launch_pdl(kmax_from_K_kernel, gk, 256, 0, s, D, H, K, w.kmax, status);
     kmax = w.kmax;
   }
-  launch_pdl(carry_scan_kernel, D, 256, 0, s, D, H, g.W2, g.T2, kmax, w.carry);
+  launch_pdl(carry_scan_kernel, D, 256, 0, s, D, H, g.W2, g.T2, kmax, w.carry, Q, cap, w.sig,
+             w.rank_of, w.capq, status);
   const int gb = static_cast<int>(std::min<int64_t>((J + 1023) / 1024, 4LL * sms));
-  launch_pdl(bin_count_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, tcount, choice, headroom, status);
-  launch_pdl(bin_scan_kernel, 1, 1024, 0, s, g.T2, tcount, w.toff, w.units, nunits, D, Q, cap, w.sig,
-                                     w.rank_of, w.capq, status);
-  launch_pdl(bin_scatter_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord, w.sp, w.su);
+  launch_pdl(bin_count_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, tcount, choice, headroom,
+             status, ticket, w.toff, w.units, nunits);
+  launch_pdl(bin_scatter_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord,
+             w.sp, w.su);
   MAPS_TRY(launch_ok());
 
   CUtensorMap tmap;
