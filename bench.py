@@ -213,14 +213,12 @@ class Step:
                    M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, self.D, self.H, J),
                    M.lib.maps_order_local_workspace_size(R + J, self.D))
         self.ws = M.Workspace(need, device)
-        dbits = (self.D - 1).bit_length()
-        n_hi = min(8, (dbits + 1 + 31 + 7) // 8)
         # calibrate 4 (three select passes, bounds); occupancy 2 (bucket, tile);
-        # dispatch 4 (carry scan, bin count, bin scatter, main); order prep,
-        # keys, plan, segment sort, merge (more entries than one block sorts),
-        # 4 arrival passes, gather, n_hi key passes, identity
+        # dispatch 4 (carry scan, bin count, bin scatter, main); order 6 (prep,
+        # keys, plan, segment sort, merge when more entries than one block
+        # sorts, the global radix form)
         merge = 1 if R + J > 5632 else 0
-        self.kernels_per_step = 4 + 2 + 4 + (4 + merge + 4 + 1 + n_hi + 1)
+        self.kernels_per_step = 4 + 2 + 4 + (5 + merge)
 
     def run(self, ev=None):
         M, R = self.M, self.R

@@ -716,36 +716,6 @@ order_merge_kernel(int64_t N, const OrderCounts *counts, const int64_t *mt_off,
   }
 }
 
-// After arrival passes: the keys follow the arrival order.
-__global__ void order_gather_kernel(int64_t N, const OrderPlan *plan,
-                                    const unsigned long long *hi_orig, unsigned long long *keyA,
-                                    unsigned long long *keyB, const uint32_t *valA,
-                                    const uint32_t *valB) {
-  pdl_prologue();
-  const int gb = plan->gather_buf;
-  if (gb < 0) return;
-  const bool wide = plan->wide != 0;
-  unsigned long long *k = gb == kBufA ? keyA : keyB;
-  const uint32_t *v = gb == kBufA ? valA : valB;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < N; i += stride) {
-    const unsigned long long x = hi_orig[v[i]];
-    if (wide)
-      k[i] = x;
-    else
-      reinterpret_cast<uint32_t *>(k)[i] = static_cast<uint32_t>(x);
-  }
-}
-
-// No active pass at all: the identity is the order.
-__global__ void order_identity_kernel(int64_t N, const OrderPlan *plan, int32_t *perm) {
-  pdl_prologue();
-  if (plan->npasses != 0) return;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < N; i += stride)
-    perm[i] = static_cast<int32_t>(i);
-}
-
 struct PassSmem {
   unsigned long long keys[kTile];
   uint32_t vals[kTile];
@@ -773,8 +743,10 @@ __device__ __forceinline__ void store_key(unsigned long long *k, int64_t i, unsi
     reinterpret_cast<uint32_t *>(k)[i] = static_cast<uint32_t>(v);
 }
 
+// One tile of pass p: takes the next ticket; false when the pass has no tile
+// left (the same answer in every thread).
 template <bool WIDE>
-__device__ void order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
+__device__ bool order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
                                 unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
                                 const unsigned long long *hi_orig, int32_t *perm,
                                 unsigned long long *state, int64_t tiles, uint32_t *ticket,
@@ -794,6 +766,7 @@ __device__ void order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
   if (tid == 0) sm.tile = static_cast<int>(atomicAdd(ticket, 1u));
   __syncthreads();
   const int tile = sm.tile;
+  if (tile >= tiles) return false;
   const int64_t base = static_cast<int64_t>(tile) * kTile;
 
   // load (all loads first), then rank within the warp (stable: warp-major,
@@ -907,23 +880,69 @@ __device__ void order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
     if (keys_out) store_key<WIDE>(kout, pos, k, lo);
     vout[pos] = sm.vals[s];
   }
+  __syncthreads();  // the next tile reuses shared memory
+  return true;
 }
 
-__global__ void __launch_bounds__(kPassThreads)
-order_pass_kernel(int p, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
-                  unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
-                  const unsigned long long *hi_orig, int32_t *perm, unsigned long long *state,
-                  int64_t tiles, uint32_t *ticket, int32_t *status) {
+// The global form in one cooperative launch: the active digit passes in
+// turn (arrival digits, the key gather, key digits), with a grid-wide
+// barrier after each; blocks take tiles by ticket, so a look-back only ever
+// waits on tiles already taken by running blocks.  With no active pass the
+// identity is the order.  Nothing runs in the segmented form.
+__global__ void __launch_bounds__(kPassThreads, 2)
+order_global_kernel(int n_hi, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
+                    unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
+                    const unsigned long long *hi_orig, int32_t *perm, unsigned long long *state,
+                    int64_t tiles, uint32_t *tickets, int32_t *status) {
   pdl_prologue();
-  if (!plan->active[p]) return;
+  const int npasses = plan->npasses;
+  if (npasses < 0) return;  // segmented form (every block returns)
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PassSmem &sm = *reinterpret_cast<PassSmem *>(smem_raw);
-  if (plan->wide)
-    order_pass_body<true>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, state, tiles, ticket,
-                          status, sm);
-  else
-    order_pass_body<false>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, state, tiles,
-                           ticket, status, sm);
+  cg::grid_group grid = cg::this_grid();
+  const bool wide = plan->wide != 0;
+  auto run_pass = [&](int p) {
+    if (wide)
+      while (order_pass_body<true>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, state,
+                                   tiles, tickets + p, status, sm)) {
+      }
+    else
+      while (order_pass_body<false>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, state,
+                                    tiles, tickets + p, status, sm)) {
+      }
+    grid.sync();
+  };
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t first = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  for (int p = 0; p < kLoPasses; ++p)
+    if (plan->active[p]) run_pass(p);
+  const int gb = plan->gather_buf;
+  if (gb >= 0) {  // after arrival passes the keys follow the arrival order
+    unsigned long long *k = gb == kBufA ? keyA : keyB;
+    const uint32_t *v = gb == kBufA ? valA : valB;
+    for (int64_t i = first; i < N; i += stride) {
+      const unsigned long long x = hi_orig[v[i]];
+      if (wide)
+        k[i] = x;
+      else
+        reinterpret_cast<uint32_t *>(k)[i] = static_cast<uint32_t>(x);
+    }
+    grid.sync();
+  }
+  for (int p = kLoPasses; p < kLoPasses + n_hi; ++p)
+    if (plan->active[p]) run_pass(p);
+  if (npasses == 0)
+    for (int64_t i = first; i < N; i += stride) perm[i] = static_cast<int32_t>(i);
+}
+
+// Blocks of the global kernel that can be resident at once.
+int64_t global_grid(size_t smem) {
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, order_global_kernel, kPassThreads,
+                                                    smem) != cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  return static_cast<int64_t>(per_sm) * sm_count();
 }
 
 // Blocks of the merge kernel that can be resident at once (its grid limit as
@@ -1038,18 +1057,12 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
                          perm_out));
   }
   const size_t smem = sizeof(PassSmem);
-  MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_pass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_global_kernel,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));
-  const int gcopy = static_cast<int>(std::min<int64_t>((N + 255) / 256, 4LL * sms));
-  auto pass = [&](int p) {
-    launch_pdl(order_pass_kernel, static_cast<unsigned>(tiles), kPassThreads, smem, s, 
-        p, N, w.plan, w.keyA, w.keyB, w.valA, w.valB, w.hi_orig, perm_out, w.state, tiles,
-        w.tickets + p, status);
-  };
-  for (int p = 0; p < kLoPasses; ++p) pass(p);
-  launch_pdl(order_gather_kernel, gcopy, 256, 0, s, N, w.plan, w.hi_orig, w.keyA, w.keyB, w.valA, w.valB);
-  for (int p = kLoPasses; p < kLoPasses + n_hi; ++p) pass(p);
-  launch_pdl(order_identity_kernel, gcopy, 256, 0, s, N, w.plan, perm_out);
+  MAPS_TRY(launch_coop(order_global_kernel, std::min<int64_t>(tiles, global_grid(smem)),
+                       kPassThreads, smem, s, n_hi, N, w.plan, w.keyA, w.keyB, w.valA, w.valB,
+                       w.hi_orig, perm_out, w.state, tiles, w.tickets, status));
   return launch_ok();
 }
 
