@@ -50,14 +50,14 @@ L2_FLUSH_BYTES = 256 << 20
 # (dram__bytes_read.sum + dram__bytes_write.sum summed over the call's
 # kernels, one launch each), valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 28_590_000, "source": "calibrate.cu", "source_sha256":
-                  "6ec8bc77c9905f1af3141b12009fd86baae3ffe17558a3c0de8269a58b9d0526"},
-    "occupancy": {"bytes": 33_340_000, "source": "occupancy.cu", "source_sha256":
-                  "3e4f278da7bdb6fe20c9cb07522c6deaaf45cda7ebeb264a7f3c2e8379339b75"},
-    "dispatch": {"bytes": 26_430_000, "source": "dispatch.cu", "source_sha256":
-                 "e14c618e37ab801c0680186b4ba30477e3352cfc88b8e4f3f499d40ba265f22c"},
-    "order": {"bytes": 72_640_000, "source": "order.cu", "source_sha256":
-              "9614d5b5eb08039bdfe4f5a1b3e6d5d7dca3b624bc9055ed51660c7d00c87040"},
+    "calibrate": {"bytes": 28586560, "source": "calibrate.cu", "source_sha256":
+                  "3a6393a37ce14d09f6e338762dc0ba08c7d1a033a7873853f340c030f0209387"},
+    "occupancy": {"bytes": 34351680, "source": "occupancy.cu", "source_sha256":
+                  "379a765fc47297f3f8241bafa1256b8621eeebae9de3f96359172554405b4f3c"},
+    "dispatch": {"bytes": 25894058, "source": "dispatch.cu", "source_sha256":
+                 "cc8943377249213803429a38d9417b64bdc6bcd27ee45074c7f89c91f72d191e"},
+    "order": {"bytes": 36410730, "source": "order.cu", "source_sha256":
+              "5073063cc1a1ab6f1b07eeda41e4f4b83e37c5ca93a1a02d1f378852ab369a31"},
 }
 KERNELS = {
     "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
