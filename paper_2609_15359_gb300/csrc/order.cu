@@ -241,13 +241,11 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
         if (w[q] <= max_wait && u[q] > 0) umax = max(umax, static_cast<uint32_t>(u[q]));
         if (an[q] < ar[q]) unsorted = true;
       }
-      if (dec_smem) {
-        if (dd >= 0) atomicAdd(&s_dec[dd], 1u);
-      } else {
-        const unsigned peers = __match_any_sync(0xffffffffu, dd);
-        if (dd >= 0 && static_cast<int>(threadIdx.x & 31) == __ffs(peers) - 1)
-          atomicAdd(&dec_count[dd], static_cast<uint32_t>(__popc(peers)));
-      }
+      // lanes of one decoder combine their count (residents come grouped by
+      // decoder, so a warp is often a single decoder)
+      const unsigned peers = __match_any_sync(0xffffffffu, dd);
+      if (dd >= 0 && static_cast<int>(threadIdx.x & 31) == __ffs(peers) - 1)
+        atomicAdd(dec_smem ? &s_dec[dd] : &dec_count[dd], static_cast<uint32_t>(__popc(peers)));
     }
   }
   if (bad) flag_error(status, MAPS_E_RANGE);
@@ -255,9 +253,14 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
   for (int off = 16; off > 0; off >>= 1) umax = max(umax, __shfl_xor_sync(0xffffffffu, umax, off));
   if ((threadIdx.x & 31) == 0 && umax) atomicMax(&counts->max_bound, umax);
   if (__syncthreads_or(unsorted) && threadIdx.x == 0) atomicOr(&counts->unsorted, 1u);
-  if (dec_smem)
-    for (int i = threadIdx.x; i < D; i += blockDim.x)
-      if (s_dec[i]) atomicAdd(&dec_count[i], s_dec[i]);
+  if (dec_smem) {
+    // blocks start their flush at different decoders so they do not collide
+    const int rot = static_cast<int>((static_cast<int64_t>(blockIdx.x) * 97) % D);
+    for (int i = threadIdx.x; i < D; i += blockDim.x) {
+      const int k = (i + rot) % D;
+      if (s_dec[k]) atomicAdd(&dec_count[k], s_dec[k]);
+    }
+  }
   // the last block to finish plans the segmented form
   __threadfence();
   __syncthreads();
@@ -646,6 +649,29 @@ __device__ __forceinline__ int merge_path(const unsigned long long *A, int la,
 
 // All merge levels and the final order in one cooperative launch: the grid
 // waits at a grid-wide barrier after each level.
+// merge_path computed by one warp over global memory: each round probes 32
+// diagonal positions at once and keeps the bracket between the last probe
+// that takes from A and the first that does not, so a long run costs a few
+// rounds of loads instead of one dependent load per halving.
+__device__ __forceinline__ int merge_path_warp(const unsigned long long *A, int la,
+                                               const unsigned long long *B, int lb, int d) {
+  const int lane = threadIdx.x & 31;
+  int lo = d > lb ? d - lb : 0, hi = d < la ? d : la;  // the answer lies in [lo, hi]
+  while (hi - lo > 32) {
+    const int span = hi - lo;
+    const int pos = lo + static_cast<int>((static_cast<long long>(lane + 1) * span) / 33);
+    const unsigned t = __ballot_sync(0xffffffffu, A[pos] < B[d - 1 - pos]);
+    const int nt = __popc(t);  // probes before the answer
+    const int plo = __shfl_sync(0xffffffffu, pos, nt > 0 ? nt - 1 : 0);
+    const int phi = __shfl_sync(0xffffffffu, pos, nt < 32 ? nt : 31);
+    lo = nt > 0 ? plo + 1 : lo;
+    hi = nt < 32 ? phi : hi;
+  }
+  const int pos = lo + lane;
+  const bool take_a = pos < hi && A[pos] < B[d - 1 - pos];
+  return lo + __popc(__ballot_sync(0xffffffffu, take_a));
+}
+
 __device__ void merge_level(int level, int ntiles, const int64_t *mt_off, const int32_t *mt_n,
                             const int32_t *mt_t, unsigned long long *bufA,
                             unsigned long long *bufB) {
@@ -665,7 +691,10 @@ __device__ void merge_level(int level, int ntiles, const int64_t *mt_off, const 
     const int lb = static_cast<int>(rest > L ? (rest < 2 * L ? rest : 2 * L) - L : 0);
     const unsigned long long *A = src + off + pstart, *B = A + la;
     const int d0 = static_cast<int>(w0 - pstart), d1 = static_cast<int>(w1 - pstart);
-    if (threadIdx.x < 2) s_split[threadIdx.x] = merge_path(A, la, B, lb, threadIdx.x ? d1 : d0);
+    if (threadIdx.x < 64) {  // warp 0 splits at d0, warp 1 at d1
+      const int r = merge_path_warp(A, la, B, lb, threadIdx.x < 32 ? d0 : d1);
+      if ((threadIdx.x & 31) == 0) s_split[threadIdx.x >> 5] = r;
+    }
     __syncthreads();
     const int i0 = s_split[0], i1 = s_split[1];
     const int j0 = d0 - i0, j1 = d1 - i1;
