@@ -40,6 +40,9 @@ constexpr int kPerThread = 4;  // entries a thread loads per round
 constexpr int kRound = kPerThread * kOccThreads;
 constexpr int kBucketRound = kPerThread * kBucketThreads;
 constexpr int kMaxTiles = 128;  // tiles per decoder of the bucketed form
+// A tile holding at most this many end steps skips the histogram: its pairs
+// are kept as a list that every thread scans for its own cells.
+constexpr int kSparse = 32;
 
 // Per-warp carry partials and the block scan's scratch.
 struct TileScan {
@@ -76,13 +79,82 @@ __device__ __forceinline__ void add_to_bin(TileSmem<CPT> &sm, int jj, int32_t b)
   atomicAdd(&sm.sb[jp], b);  // exact while sum b fits int32
 }
 
-// Writes tile [t0, t0 + W) of row k.  Thread tid owns cells tid*CPT + c,
-// c < CPT, and holds in bc[c] / bs[c] the count and b-sum of the residents
-// whose last live step is that cell.  Entry: sc.part[][warp] written by every
-// warp and a block barrier since.  Cell l needs every bin at or after l: the
-// thread's own bins from l up, all bins of the threads above it, and the
-// carry.  The 32-bit sums only wrap when sum b exceeds INT32_MAX, which is
-// reported as MAPS_E_RANGE.
+// Writes the cells tid*CPT + c, c < CPT, of tile [t0, t0 + W) of row k.
+// bc[c] / bs[c] are the count and b-sum of the residents whose last live step
+// is that cell, tot_c / tot_s their sums over the thread's cells, and
+// c_hi / s_hi the count and b-sum of the residents live past the thread's
+// last cell.  The 32-bit sums only wrap when sum b exceeds INT32_MAX, which
+// is reported as MAPS_E_RANGE.  Every thread of the block calls it.
+template <int CPT, bool VEC>
+__device__ __forceinline__ void write_cells(const uint32_t (&bc)[CPT], const uint32_t (&bs)[CPT],
+                                            uint32_t tot_c, uint32_t tot_s, uint32_t c_hi,
+                                            uint32_t s_hi, int H, int k, int t0, int32_t *K,
+                                            uint32_t *kmax, int32_t *status) {
+  const int tid = threadIdx.x, lane = tid & 31;
+  const int cell0 = t0 + tid * CPT;
+  const uint32_t tc0 = static_cast<uint32_t>(cell0);
+  uint32_t bmax = 0;  // max of K + t over this thread's valid cells
+  if (cell0 < H) {
+    // Both running sums only grow towards the thread's first cell, so their
+    // totals and the last cell's step bound every cell of the thread.
+    const unsigned long long bound64 =
+        static_cast<unsigned long long>(tc0 + CPT - 1) * (c_hi + tot_c) + (s_hi + tot_s);
+    int32_t *row = K + static_cast<int64_t>(k) * H;
+    uint32_t run_c = c_hi, run_s = s_hi;
+    if (VEC && bound64 <= 0x7fffffffull && cell0 + CPT <= H) {
+      // every cell valid and exact in 32 bits
+      uint32_t o[CPT];
+      if (tot_c == 0) {
+        // no resident ends in these cells: K is affine in t over them, and
+        // K + t grows with t, so the last cell holds the maximum
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) o[c] = (tc0 + c) * run_c + run_s;
+        bmax = o[CPT - 1] + tc0 + CPT - 1;
+      } else {
+#pragma unroll
+        for (int c = CPT - 1; c >= 0; --c) {
+          run_c += bc[c];
+          run_s += bs[c];
+          o[c] = (tc0 + c) * run_c + run_s;
+          bmax = max(bmax, o[c] + tc0 + c);
+        }
+      }
+#pragma unroll
+      for (int c = 0; c < CPT; c += 4)
+        *reinterpret_cast<int4 *>(row + cell0 + c) = make_int4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+    } else {
+      bool over = false;
+#pragma unroll
+      for (int c = CPT - 1; c >= 0; --c) {
+        run_c += bc[c];
+        run_s += bs[c];
+        if (cell0 + c < H) {
+          const uint32_t t = tc0 + c;
+          const unsigned long long v = static_cast<unsigned long long>(t) * run_c + run_s;
+          over |= (v >> 31) != 0;
+          const uint32_t o = static_cast<uint32_t>(v);
+          bmax = max(bmax, o + t);
+          row[cell0 + c] = static_cast<int32_t>(o);
+        }
+      }
+      if (over) flag_error(status, MAPS_E_RANGE);
+    }
+  }
+  if (kmax != nullptr) {
+    constexpr int L = kBlock / CPT > 0 ? kBlock / CPT : 1;  // lanes per 16-step block
+#pragma unroll
+    for (int off = L / 2; off > 0; off >>= 1) bmax = max(bmax, __shfl_xor_sync(0xffffffffu, bmax, off));
+    if ((lane % L) == 0 && cell0 < H) {
+      const int64_t nb = (static_cast<int64_t>(H) + kBlock - 1) / kBlock;
+      kmax[static_cast<int64_t>(k) * nb + cell0 / kBlock] = bmax;
+    }
+  }
+}
+
+// Writes tile [t0, t0 + W) of row k from every thread's own bins.  Entry:
+// sc.part[][warp] written by every warp and a block barrier since.  Cell l
+// needs every bin at or after l: the thread's own bins from l up, all bins of
+// the threads above it (a block suffix scan), and the carry.
 template <int CPT, bool VEC>
 __device__ __forceinline__ void emit_cells(const uint32_t (&bc)[CPT], const uint32_t (&bs)[CPT],
                                            TileScan &sc, int H, int k, int t0, int32_t *K,
@@ -141,58 +213,9 @@ __device__ __forceinline__ void emit_cells(const uint32_t (&bc)[CPT], const uint
   }
   __syncthreads();
 
-  const uint32_t c_lo = sc.carry[0] + sc.wsum[0][warp] + (suf_c - tot_c);
-  const uint32_t s_lo = sc.carry[1] + sc.wsum[1][warp] + (suf_s - tot_s);
-  const int cell0 = t0 + tid * CPT;
-  const uint32_t tc0 = static_cast<uint32_t>(cell0);
-  uint32_t bmax = 0;  // max of K + t over this thread's valid cells
-  if (cell0 < H) {
-    // Both running sums only grow towards the thread's first cell, so their
-    // totals and the last cell's step bound every cell of the thread.
-    const unsigned long long bound64 =
-        static_cast<unsigned long long>(tc0 + CPT - 1) * (c_lo + tot_c) + (s_lo + tot_s);
-    int32_t *row = K + static_cast<int64_t>(k) * H;
-    uint32_t run_c = c_lo, run_s = s_lo;
-    if (VEC && bound64 <= 0x7fffffffull && cell0 + CPT <= H) {
-      // every cell valid and exact in 32 bits
-      uint32_t o[CPT];
-#pragma unroll
-      for (int c = CPT - 1; c >= 0; --c) {
-        run_c += bc[c];
-        run_s += bs[c];
-        o[c] = (tc0 + c) * run_c + run_s;
-        bmax = max(bmax, o[c] + tc0 + c);
-      }
-#pragma unroll
-      for (int c = 0; c < CPT; c += 4)
-        *reinterpret_cast<int4 *>(row + cell0 + c) = make_int4(o[c], o[c + 1], o[c + 2], o[c + 3]);
-    } else {
-      bool over = false;
-#pragma unroll
-      for (int c = CPT - 1; c >= 0; --c) {
-        run_c += bc[c];
-        run_s += bs[c];
-        if (cell0 + c < H) {
-          const uint32_t t = tc0 + c;
-          const unsigned long long v = static_cast<unsigned long long>(t) * run_c + run_s;
-          over |= (v >> 31) != 0;
-          const uint32_t o = static_cast<uint32_t>(v);
-          bmax = max(bmax, o + t);
-          row[cell0 + c] = static_cast<int32_t>(o);
-        }
-      }
-      if (over) flag_error(status, MAPS_E_RANGE);
-    }
-  }
-  if (kmax != nullptr) {
-    constexpr int L = kBlock / CPT > 0 ? kBlock / CPT : 1;  // lanes per 16-step block
-#pragma unroll
-    for (int off = L / 2; off > 0; off >>= 1) bmax = max(bmax, __shfl_xor_sync(0xffffffffu, bmax, off));
-    if ((lane % L) == 0 && cell0 < H) {
-      const int64_t nb = (static_cast<int64_t>(H) + kBlock - 1) / kBlock;
-      kmax[static_cast<int64_t>(k) * nb + cell0 / kBlock] = bmax;
-    }
-  }
+  const uint32_t c_hi = sc.carry[0] + sc.wsum[0][warp] + (suf_c - tot_c);
+  const uint32_t s_hi = sc.carry[1] + sc.wsum[1][warp] + (suf_s - tot_s);
+  write_cells<CPT, VEC>(bc, bs, tot_c, tot_s, c_hi, s_hi, H, k, t0, K, kmax, status);
 }
 
 // The histogram form: each thread takes its own CPT bins into registers.
@@ -243,9 +266,11 @@ __global__ void __launch_bounds__(kBucketThreads)
 occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, int64_t R,
                   const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
                   const int32_t *__restrict__ bound, int2 *__restrict__ bucket,
-                  int32_t *__restrict__ tile_off, int32_t *status) {
+                  int32_t *__restrict__ tile_off, uint2 *__restrict__ tile_carry,
+                  int32_t *status) {
   pdl_prologue();
   __shared__ int s_cnt[kMaxTiles];
+  __shared__ uint32_t s_sb[kMaxTiles];
   __shared__ int s_cur[kMaxTiles];
   __shared__ long long s_red[kBucketThreads / 32];
   const int k = blockIdx.x, tid = threadIdx.x, lane = tid & 31;
@@ -256,10 +281,10 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
   }
   const int n = static_cast<int>(hi - lo);
   const int32_t *pp = prompt + lo, *pg = gen + lo, *pu = bound + lo;
-  if (tid < kMaxTiles) s_cnt[tid] = 0;
+  if (tid < kMaxTiles) s_cnt[tid] = 0, s_sb[tid] = 0;
   __syncthreads();
 
-  // pass 1: residents per tile
+  // pass 1: residents per tile and the sum of their b
   for (int r0 = 0; r0 < n; r0 += kBucketRound) {
     int32_t p[kPerThread], g[kPerThread], U[kPerThread];
 #pragma unroll
@@ -276,7 +301,13 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
       bool big;
       const int tile = resident_terms(p[j], g[j], U[j], H, b32, e, big) ? (e - 1) >> log2W : -1;
       const unsigned peers = __match_any_sync(0xffffffffu, tile);
-      if (tile >= 0 && lane == __ffs(peers) - 1) atomicAdd(&s_cnt[tile], __popc(peers));
+      // every lane of a group reduces over that group only (wraps only past
+      // INT32_MAX, which is reported below)
+      const uint32_t bsum = __reduce_add_sync(peers, tile >= 0 ? static_cast<uint32_t>(b32) : 0u);
+      if (tile >= 0 && lane == __ffs(peers) - 1) {
+        atomicAdd(&s_cnt[tile], __popc(peers));
+        atomicAdd(&s_sb[tile], bsum);
+      }
     }
   }
   __syncthreads();
@@ -289,6 +320,14 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
       run += s_cnt[y];
     }
     to[T] = run;
+  } else if (tid == 32) {  // carries: residents live past each tile
+    uint32_t cc = 0, cs = 0;
+    uint2 *tc = tile_carry + static_cast<int64_t>(k) * T;
+    for (int y = T - 1; y >= 0; --y) {
+      tc[y] = make_uint2(cc, cs);
+      cc += static_cast<uint32_t>(s_cnt[y]);
+      cs += s_sb[y];
+    }
   }
   __syncthreads();
 
@@ -332,54 +371,75 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
 }
 
 // ---------------------------------------------------------------------------
-// 2. Tile kernel: one CTA per (decoder, tile), reading the sorted pairs.
+// 2. Tile kernel: one CTA per (decoder, tile), reading the sorted pairs of its
+// own tile and the tile's carry (count and b-sum of the residents live past
+// it) from the bucket kernel.
 // ---------------------------------------------------------------------------
 template <int CPT, bool VEC>
 __global__ void __launch_bounds__(kOccThreads, 5)
 occ_tile_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
                 const int2 *__restrict__ bucket, const int32_t *__restrict__ tile_off,
-                int32_t *__restrict__ K, uint32_t *__restrict__ kmax, int32_t *status) {
+                const uint2 *__restrict__ tile_carry, int32_t *__restrict__ K,
+                uint32_t *__restrict__ kmax, int32_t *status) {
   pdl_prologue();
   __shared__ __align__(16) TileSmem<CPT> sm;
-  constexpr int W = TileSmem<CPT>::W;
   const int k = blockIdx.x / T, ti = blockIdx.x - (blockIdx.x / T) * T;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int t0 = ti * W;
+  const int t0 = ti * TileSmem<CPT>::W;
   int64_t lo = res_off[k];
   const int32_t *to = tile_off + static_cast<int64_t>(k) * (T + 1);
-  const int a = to[ti], m = to[ti + 1], z = to[T];
+  const int a = to[ti], m = to[ti + 1];
+  const uint2 car = tile_carry[static_cast<int64_t>(k) * T + ti];
   if (lo < 0 || lo > R) lo = 0;  // reported by the bucket kernel; the range is then empty
   const int2 *bk = bucket + lo;
+
+  if (m - a <= kSparse) {  // the same for the whole block
+    // Sparse tile: every thread reads the tile's few pairs (one address
+    // across the warp).  A pair past the thread's last cell adds to every one
+    // of its cells, one inside from its own cell down; no block scan needed.
+    uint32_t c_hi = car.x, s_hi = car.y;
+    uint32_t bc[CPT], bs[CPT];
+#pragma unroll
+    for (int c = 0; c < CPT; ++c) bc[c] = bs[c] = 0;
+    uint32_t tot_c = 0, tot_s = 0;
+    const int c0 = tid * CPT;
+    for (int j = a; j < m; ++j) {
+      const int2 v = __ldg(bk + j);
+      const int q = v.y - 1 - t0 - c0;  // the pair's last live step, from the thread's first cell
+      if (q >= CPT) {
+        c_hi += 1;
+        s_hi += static_cast<uint32_t>(v.x);
+      } else if (q >= 0) {
+        tot_c += 1;
+        tot_s += static_cast<uint32_t>(v.x);
+#pragma unroll
+        for (int c = 0; c < CPT; ++c)
+          if (q == c) {
+            bc[c] += 1;
+            bs[c] += static_cast<uint32_t>(v.x);
+          }
+      }
+    }
+    write_cells<CPT, VEC>(bc, bs, tot_c, tot_s, c_hi, s_hi, H, k, t0, K, kmax, status);
+    return;
+  }
+
   zero_bins(sm);
   __syncthreads();
-
-  uint32_t car_c = 0, car_s = 0;
-  for (int r0 = a; r0 < z; r0 += kRound) {
+  for (int r0 = a; r0 < m; r0 += kRound) {
     int2 v[kPerThread];
 #pragma unroll
     for (int j = 0; j < kPerThread; ++j) {
       const int i = r0 + j * kOccThreads + tid;
-      v[j] = i < z ? __ldg(bk + i) : make_int2(0, 0);
+      v[j] = i < m ? __ldg(bk + i) : make_int2(0, 0);
     }
 #pragma unroll
-    for (int j = 0; j < kPerThread; ++j) {
-      const int i = r0 + j * kOccThreads + tid;
-      if (i < m) {
-        add_to_bin(sm, v[j].y - 1 - t0, v[j].x);
-      } else if (i < z) {
-        car_c += 1;
-        car_s += static_cast<uint32_t>(v[j].x);
-      }
-    }
+    for (int j = 0; j < kPerThread; ++j)
+      if (r0 + j * kOccThreads + tid < m) add_to_bin(sm, v[j].y - 1 - t0, v[j].x);
   }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    car_c += __shfl_xor_sync(0xffffffffu, car_c, off);
-    car_s += __shfl_xor_sync(0xffffffffu, car_s, off);
-  }
-  if (lane == 0) {
-    sm.scan.part[0][warp] = car_c;
-    sm.scan.part[1][warp] = car_s;
+  if (lane == 0) {  // the carry enters the scan as warp 0's partial
+    sm.scan.part[0][warp] = warp == 0 ? car.x : 0u;
+    sm.scan.part[1][warp] = warp == 0 ? car.y : 0u;
   }
   __syncthreads();
   emit_tile<CPT, VEC>(sm, H, k, t0, K, kmax, status);
@@ -474,10 +534,11 @@ OccPlan plan_occ(int32_t H, int64_t R) {
 }
 
 size_t carve_occ(Carve &c, int32_t D, int64_t R, const OccPlan &p, int2 **bucket,
-                 int32_t **tile_off) {
+                 int32_t **tile_off, uint2 **tile_carry) {
   if (p.bucketed) {
     *bucket = c.take<int2>(static_cast<size_t>(R));
     *tile_off = c.take<int32_t>(static_cast<size_t>(D) * (p.T + 1));
+    *tile_carry = c.take<uint2>(static_cast<size_t>(D) * p.T);
   }
   return c.bytes();
 }
@@ -485,12 +546,12 @@ size_t carve_occ(Carve &c, int32_t D, int64_t R, const OccPlan &p, int2 **bucket
 template <int CPT, bool VEC>
 void launch_tiles(const OccPlan &p, int64_t blocks, cudaStream_t s, int H, const int64_t *res_off,
                   int64_t R, const int32_t *prompt, const int32_t *gen, const int32_t *bound,
-                  const int2 *bucket, const int32_t *tile_off, int32_t *K, uint32_t *kmax,
-                  int32_t *status) {
+                  const int2 *bucket, const int32_t *tile_off, const uint2 *tile_carry,
+                  int32_t *K, uint32_t *kmax, int32_t *status) {
   const dim3 grid(static_cast<unsigned>(blocks));
   if (p.bucketed)
-    launch_pdl(occ_tile_kernel<CPT, VEC>, grid, kOccThreads, 0, s, H, p.T, res_off, R, bucket, tile_off, K,
-                                                          kmax, status);
+    launch_pdl(occ_tile_kernel<CPT, VEC>, grid, kOccThreads, 0, s, H, p.T, res_off, R, bucket,
+               tile_off, tile_carry, K, kmax, status);
   else
     launch_pdl(occ_direct_kernel<CPT, VEC>, grid, kOccThreads, 0, s, H, p.T, res_off, R, prompt, gen,
                                                             bound, K, kmax, status);
@@ -499,14 +560,14 @@ void launch_tiles(const OccPlan &p, int64_t blocks, cudaStream_t s, int H, const
 template <int CPT>
 void launch_cpt(bool vec, const OccPlan &p, int64_t blocks, cudaStream_t s, int H,
                 const int64_t *res_off, int64_t R, const int32_t *prompt, const int32_t *gen,
-                const int32_t *bound, const int2 *bucket, const int32_t *tile_off, int32_t *K,
-                uint32_t *kmax, int32_t *status) {
+                const int32_t *bound, const int2 *bucket, const int32_t *tile_off,
+                const uint2 *tile_carry, int32_t *K, uint32_t *kmax, int32_t *status) {
   if (vec)
-    launch_tiles<CPT, true>(p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K,
-                            kmax, status);
+    launch_tiles<CPT, true>(p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off,
+                            tile_carry, K, kmax, status);
   else
-    launch_tiles<CPT, false>(p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K,
-                             kmax, status);
+    launch_tiles<CPT, false>(p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off,
+                             tile_carry, K, kmax, status);
 }
 
 }  // namespace
@@ -520,7 +581,8 @@ size_t maps_project_occupancy_workspace_size(int32_t D, int32_t H, int64_t R) {
   Carve c(nullptr);
   int2 *bucket = nullptr;
   int32_t *tile_off = nullptr;
-  return carve_occ(c, D, R, plan_occ(H, R), &bucket, &tile_off);
+  uint2 *tile_carry = nullptr;
+  return carve_occ(c, D, R, plan_occ(H, R), &bucket, &tile_off, &tile_carry);
 }
 
 int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off, int64_t R,
@@ -540,21 +602,22 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off, int64_t
   Carve c(ws);
   int2 *bucket = nullptr;
   int32_t *tile_off = nullptr;
-  carve_occ(c, D, R, p, &bucket, &tile_off);
+  uint2 *tile_carry = nullptr;
+  carve_occ(c, D, R, p, &bucket, &tile_off, &tile_carry);
   if (p.bucketed) {
-    launch_pdl(occ_bucket_kernel, D, kBucketThreads, 0, s, H, p.T, p.log2W, res_off, R, prompt, gen, bound,
-                                                bucket, tile_off, status);
+    launch_pdl(occ_bucket_kernel, D, kBucketThreads, 0, s, H, p.T, p.log2W, res_off, R, prompt,
+               gen, bound, bucket, tile_off, tile_carry, status);
     MAPS_TRY(launch_ok());
   }
   const bool vec = (H % 4 == 0) && aligned(K_out, 16);
   if (p.cpt == 16)
-    launch_cpt<16>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K_out,
+    launch_cpt<16>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, tile_carry, K_out,
                    kmax_out, status);
   else if (p.cpt == 8)
-    launch_cpt<8>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K_out,
+    launch_cpt<8>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, tile_carry, K_out,
                   kmax_out, status);
   else
-    launch_cpt<4>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, K_out,
+    launch_cpt<4>(vec, p, blocks, s, H, res_off, R, prompt, gen, bound, bucket, tile_off, tile_carry, K_out,
                   kmax_out, status);
   return launch_ok();
 }
