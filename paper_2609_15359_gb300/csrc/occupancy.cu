@@ -40,6 +40,7 @@ constexpr int kPerThread = 4;  // entries a thread loads per round
 constexpr int kRound = kPerThread * kOccThreads;
 constexpr int kBucketRound = kPerThread * kBucketThreads;
 constexpr int kMaxTiles = 128;  // tiles per decoder of the bucketed form
+constexpr int kBHold = 8;       // residents a bucket thread keeps in registers
 // A tile holding at most this many end steps skips the histogram: its pairs
 // are kept as a list that every thread scans for its own cells.
 constexpr int kSparse = 32;
@@ -272,7 +273,7 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
   __shared__ int s_cnt[kMaxTiles];
   __shared__ uint32_t s_sb[kMaxTiles];
   __shared__ int s_cur[kMaxTiles];
-  __shared__ long long s_red[kBucketThreads / 32];
+  __shared__ unsigned long long s_total;  // sum of b over the decoder's residents
   const int k = blockIdx.x, tid = threadIdx.x, lane = tid & 31;
   int64_t lo = res_off[k], hi = res_off[k + 1];
   if (lo < 0 || hi < lo || hi > R || hi - lo > 0x7fffffffLL) {
@@ -282,9 +283,104 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
   const int n = static_cast<int>(hi - lo);
   const int32_t *pp = prompt + lo, *pg = gen + lo, *pu = bound + lo;
   if (tid < kMaxTiles) s_cnt[tid] = 0, s_sb[tid] = 0;
+  if (tid == 0) s_total = 0;
   __syncthreads();
 
-  // pass 1: residents per tile and the sum of their b
+  // tile starts and carries (the residents live past each tile); T <= kMaxTiles
+  auto publish = [&]() {
+    if (tid == 0) {
+      int run = 0;
+      int32_t *to = tile_off + static_cast<int64_t>(k) * (T + 1);
+      for (int y = 0; y < T; ++y) {
+        to[y] = run;
+        s_cur[y] = run;
+        run += s_cnt[y];
+      }
+      to[T] = run;
+    } else if (tid == 32) {
+      uint32_t cc = 0, cs = 0;
+      uint2 *tc = tile_carry + static_cast<int64_t>(k) * T;
+      for (int y = T - 1; y >= 0; --y) {
+        tc[y] = make_uint2(cc, cs);
+        cc += static_cast<uint32_t>(s_cnt[y]);
+        cs += s_sb[y];
+      }
+    } else if (tid == 64 && s_total > 0x7fffffffull) {
+      flag_error(status, MAPS_E_RANGE);
+    }
+  };
+  // a group of lanes with the same tile: count and b-sum to the tile's bins
+  // (every lane of a group reduces over that group only; the b-sum wraps
+  // only past INT32_MAX, which is reported)
+  auto count = [&](int tile, int32_t b32, unsigned peers) {
+    const uint32_t bsum = __reduce_add_sync(peers, tile >= 0 ? static_cast<uint32_t>(b32) : 0u);
+    if (tile >= 0 && lane == __ffs(peers) - 1) {
+      atomicAdd(&s_cnt[tile], __popc(peers));
+      atomicAdd(&s_sb[tile], bsum);
+    }
+  };
+  // ... and its slots in the tile's range of the bucket array
+  auto scatter = [&](int tile, int32_t b32, int32_t e, unsigned peers) {
+    const int leader = __ffs(peers) - 1;
+    int base = 0;
+    if (tile >= 0 && lane == leader) base = atomicAdd(&s_cur[tile], __popc(peers));
+    base = __shfl_sync(0xffffffffu, base, leader);
+    if (tile >= 0) bucket[lo + base + __popc(peers & ((1u << lane) - 1u))] = make_int2(b32, e);
+  };
+  auto add_total = [&](unsigned long long total) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) total += __shfl_xor_sync(0xffffffffu, total, off);
+    if (lane == 0) atomicAdd(&s_total, total);
+  };
+
+  if (n <= kBHold * kBucketThreads) {
+    // Held form: one read of the residents, kept in registers with their
+    // peer masks through both passes.
+    int32_t hb[kBHold], he[kBHold], tl[kBHold];
+    unsigned pr[kBHold];
+    bool bad = false;
+    unsigned long long total = 0;
+    {
+      int32_t p[kBHold], g[kBHold], U[kBHold];
+#pragma unroll
+      for (int j = 0; j < kBHold; ++j) {
+        const int i = j * kBucketThreads + tid;
+        const bool ok = i < n;
+        p[j] = ok ? __ldg(pp + i) : -1;
+        g[j] = ok ? __ldg(pg + i) : 0;
+        U[j] = ok ? __ldg(pu + i) : 0;
+      }
+#pragma unroll
+      for (int j = 0; j < kBHold; ++j) {
+        bool big = false;
+        hb[j] = he[j] = 0;
+        tl[j] = -1;
+        if (resident_terms(p[j], g[j], U[j], H, hb[j], he[j], big)) {
+          tl[j] = (he[j] - 1) >> log2W;
+          total += static_cast<unsigned long long>(hb[j]);
+          bad |= big;
+        } else if (j * kBucketThreads + tid < n) {
+          bad = true;
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kBHold; ++j) {
+      pr[j] = __match_any_sync(0xffffffffu, tl[j]);
+      count(tl[j], hb[j], pr[j]);
+    }
+    add_total(total);
+    if (bad) flag_error(status, MAPS_E_RANGE);
+    __syncthreads();
+    publish();
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < kBHold; ++j) scatter(tl[j], hb[j], he[j], pr[j]);
+    return;
+  }
+
+  // Streamed form (more residents than the registers hold): pass 1 counts,
+  // pass 2 reads the residents again (from L2) and scatters.
   for (int r0 = 0; r0 < n; r0 += kBucketRound) {
     int32_t p[kPerThread], g[kPerThread], U[kPerThread];
 #pragma unroll
@@ -300,40 +396,39 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
       int32_t b32, e;
       bool big;
       const int tile = resident_terms(p[j], g[j], U[j], H, b32, e, big) ? (e - 1) >> log2W : -1;
-      const unsigned peers = __match_any_sync(0xffffffffu, tile);
-      // every lane of a group reduces over that group only (wraps only past
-      // INT32_MAX, which is reported below)
-      const uint32_t bsum = __reduce_add_sync(peers, tile >= 0 ? static_cast<uint32_t>(b32) : 0u);
-      if (tile >= 0 && lane == __ffs(peers) - 1) {
-        atomicAdd(&s_cnt[tile], __popc(peers));
-        atomicAdd(&s_sb[tile], bsum);
+      count(tile, b32, __match_any_sync(0xffffffffu, tile));
+    }
+  }
+  bool bad = false;
+  unsigned long long total = 0;
+  __syncthreads();
+  for (int r0 = 0; r0 < n; r0 += kBucketRound) {  // totals and checks ride on pass 2
+    int32_t p[kPerThread], g[kPerThread], U[kPerThread];
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      const int i = r0 + j * kBucketThreads + tid;
+      const bool ok = i < n;
+      p[j] = ok ? __ldg(pp + i) : -1;
+      g[j] = ok ? __ldg(pg + i) : 0;
+      U[j] = ok ? __ldg(pu + i) : 0;
+    }
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      int32_t b32, e;
+      bool big = false;
+      if (resident_terms(p[j], g[j], U[j], H, b32, e, big)) {
+        total += static_cast<unsigned long long>(b32);
+        bad |= big;
+      } else if (r0 + j * kBucketThreads + tid < n) {
+        bad = true;
       }
     }
   }
+  add_total(total);
+  if (bad) flag_error(status, MAPS_E_RANGE);
   __syncthreads();
-  if (tid == 0) {  // tile starts; T <= kMaxTiles
-    int run = 0;
-    int32_t *to = tile_off + static_cast<int64_t>(k) * (T + 1);
-    for (int y = 0; y < T; ++y) {
-      to[y] = run;
-      s_cur[y] = run;
-      run += s_cnt[y];
-    }
-    to[T] = run;
-  } else if (tid == 32) {  // carries: residents live past each tile
-    uint32_t cc = 0, cs = 0;
-    uint2 *tc = tile_carry + static_cast<int64_t>(k) * T;
-    for (int y = T - 1; y >= 0; --y) {
-      tc[y] = make_uint2(cc, cs);
-      cc += static_cast<uint32_t>(s_cnt[y]);
-      cs += s_sb[y];
-    }
-  }
+  publish();
   __syncthreads();
-
-  // pass 2: scatter the pairs (the residents come from L2 this time)
-  bool bad = false;
-  long long total = 0;
   for (int r0 = 0; r0 < n; r0 += kBucketRound) {
     int32_t p[kPerThread], g[kPerThread], U[kPerThread];
 #pragma unroll
@@ -346,28 +441,12 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
     }
 #pragma unroll
     for (int j = 0; j < kPerThread; ++j) {
-      const bool present = r0 + j * kBucketThreads + tid < n;
       int32_t b32 = 0, e = 0;
-      bool big = false;
-      int tile = -1;
-      if (resident_terms(p[j], g[j], U[j], H, b32, e, big)) {
-        tile = (e - 1) >> log2W;
-        total += b32;
-        bad |= big;
-      } else if (present) {
-        bad = true;
-      }
-      const unsigned peers = __match_any_sync(0xffffffffu, tile);
-      const int leader = __ffs(peers) - 1;
-      int base = 0;
-      if (tile >= 0 && lane == leader) base = atomicAdd(&s_cur[tile], __popc(peers));
-      base = __shfl_sync(0xffffffffu, base, leader);
-      if (tile >= 0) bucket[lo + base + __popc(peers & ((1u << lane) - 1u))] = make_int2(b32, e);
+      bool big;
+      const int tile = resident_terms(p[j], g[j], U[j], H, b32, e, big) ? (e - 1) >> log2W : -1;
+      scatter(tile, b32, e, __match_any_sync(0xffffffffu, tile));
     }
   }
-  if (bad) flag_error(status, MAPS_E_RANGE);
-  const long long sum_b = block_sum_ll<kBucketThreads / 32>(total, s_red);
-  if (tid == 0 && sum_b > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
 }
 
 // ---------------------------------------------------------------------------
@@ -377,13 +456,14 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
 // ---------------------------------------------------------------------------
 template <int CPT, bool VEC>
 __global__ void __launch_bounds__(kOccThreads, 5)
-occ_tile_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
+occ_tile_kernel(int H, int D, int T, const int64_t *__restrict__ res_off, int64_t R,
                 const int2 *__restrict__ bucket, const int32_t *__restrict__ tile_off,
                 const uint2 *__restrict__ tile_carry, int32_t *__restrict__ K,
                 uint32_t *__restrict__ kmax, int32_t *status) {
   pdl_prologue();
   __shared__ __align__(16) TileSmem<CPT> sm;
-  const int k = blockIdx.x / T, ti = blockIdx.x - (blockIdx.x / T) * T;
+  // tile-major order: the early tiles, where most residents end, start first
+  const int ti = blockIdx.x / D, k = blockIdx.x - (blockIdx.x / D) * D;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int t0 = ti * TileSmem<CPT>::W;
   int64_t lo = res_off[k];
@@ -550,7 +630,7 @@ void launch_tiles(const OccPlan &p, int64_t blocks, cudaStream_t s, int H, const
                   int32_t *K, uint32_t *kmax, int32_t *status) {
   const dim3 grid(static_cast<unsigned>(blocks));
   if (p.bucketed)
-    launch_pdl(occ_tile_kernel<CPT, VEC>, grid, kOccThreads, 0, s, H, p.T, res_off, R, bucket,
+    launch_pdl(occ_tile_kernel<CPT, VEC>, grid, kOccThreads, 0, s, H, static_cast<int>(blocks / p.T), p.T, res_off, R, bucket,
                tile_off, tile_carry, K, kmax, status);
   else
     launch_pdl(occ_direct_kernel<CPT, VEC>, grid, kOccThreads, 0, s, H, p.T, res_off, R, prompt, gen,
