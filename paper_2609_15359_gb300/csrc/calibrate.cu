@@ -109,9 +109,13 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
     const int b = (i + rot) & (kBins - 1);
     if (sh[b]) atomicAdd(&st->hist[PASS][b], static_cast<unsigned long long>(sh[b]));
   }
-  __threadfence();
+  // one thread publishes the block's flush (the barrier orders every thread's
+  // atomics before its fence, as a grid barrier does)
   __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(&st->done[PASS], 1u) == gridDim.x - 1);
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = (atomicAdd(&st->done[PASS], 1u) == gridDim.x - 1);
+  }
   __syncthreads();
   if (!s_last) return;
   __threadfence();

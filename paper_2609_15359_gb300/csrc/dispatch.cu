@@ -272,9 +272,13 @@ bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ c
     }
   }
   // the last block to finish turns the counts into offsets and work units
-  __threadfence();
+  // (one thread publishes the block's counts: the barrier orders every
+  // thread's atomics before its fence, as a grid barrier does)
   __syncthreads();
-  if (threadIdx.x == 0) s_last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+  }
   __syncthreads();
   if (s_last) {
     __threadfence();

@@ -262,9 +262,13 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
     }
   }
   // the last block to finish plans the segmented form
-  __threadfence();
+  // (one thread publishes the block's counts: the barrier orders every
+  // thread's atomics before its fence, as a grid barrier does)
   __syncthreads();
-  if (threadIdx.x == 0) s_last = atomicAdd(&counts->done_blocks, 1u) == gridDim.x - 1;
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(&counts->done_blocks, 1u) == gridDim.x - 1;
+  }
   __syncthreads();
   if (s_last) {
     __threadfence();
