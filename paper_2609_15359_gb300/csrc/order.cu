@@ -1085,7 +1085,10 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
              kSegThreads, seg_smem, s, N, w.counts, w.item_off, w.item_n, w.valA, bound, wait,
              max_wait, perm_out, w.keyA);
   if (N > kSegMax) {  // some queue may be longer than one block sorts
-    MAPS_TRY(launch_coop(order_merge_kernel, std::min<int64_t>(w.ntiles_max, merge_grid()),
+    // one block per SM: a level has few tiles, and a smaller grid meets at its
+    // barriers sooner
+    MAPS_TRY(launch_coop(order_merge_kernel,
+                         std::min<int64_t>(w.ntiles_max, std::min<int64_t>(merge_grid(), sms)),
                          kMergeThreads, 0, s, N, w.counts, w.mt_off, w.mt_n, w.mt_t, w.keyA, w.keyB,
                          perm_out));
   }
