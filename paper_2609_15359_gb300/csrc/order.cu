@@ -12,20 +12,19 @@
 //     arrival order is already in place and the sort is stable;
 //   * a key of at most 32 bits is sorted as 32 bits, otherwise as 64 bits.
 // Kernels: a prep pass (validation, largest bound, entries per decoder,
-// arrival order check; its last block chooses the form), a key pass, a
-// one-block plan (digit offsets, which passes run, buffers, decoder segment
-// offsets).
+// arrival order check; its last block chooses the form), a key pass, the
+// segment sort, and a cooperative finishing kernel.
 // Segmented form (arrival non-decreasing along the index): the key pass
 // scatters each entry's index to its decoder's segment; one block sorts a
 // segment of at most kSegMax entries in shared memory on (not promoted,
 // primary, index), a unique key, and a longer segment is sorted as chunks of
-// kSegMax whose runs are merged pairwise level by level.  Otherwise one
-// global sweep per digit: tiles of 4096 keys are
-// ranked stably in shared memory, each tile learns its offsets from earlier
-// tiles by decoupled look-back (one thread per digit walks back over packed
-// flag-and-count words until it meets an inclusive prefix), and writes out
-// bin by bin.  Passes the plan marks inactive return at once, so the host
-// never waits on the device.
+// kSegMax whose runs the finishing kernel merges pairwise level by level.
+// Otherwise the finishing kernel plans and runs one global sweep per digit:
+// tiles of 4096 keys are ranked stably in shared memory, each tile learns its
+// offsets from earlier tiles by decoupled look-back (one thread per digit
+// walks back over packed flag-and-count words until it meets an inclusive
+// prefix), and writes out bin by bin.  Kernels of the form not taken return
+// at once, so the host never waits on the device.
 #include <cooperative_groups.h>
 
 #include "maps_internal.cuh"
@@ -74,7 +73,7 @@ constexpr int kSegMax = kSegThreads * kSegIPT;  // entries one block sorts
 // then merged pairwise, level by level, in tiles of kMergeTile outputs
 // (kMergeTile divides kSegMax, so no tile straddles two runs).
 constexpr int kMergeTile = 512;
-constexpr int kMergeThreads = 256;
+constexpr int kMergeThreads = 512;  // the finishing kernel's block
 static_assert(kSegMax % kMergeTile == 0, "merge tiles align with runs");
 
 // Merge levels a queue of n entries needs: ceil(log2(ceil(n / kSegMax))).
@@ -376,30 +375,17 @@ order_keys_kernel(int64_t N, int D, int dbits, const int32_t *__restrict__ dec,
 
 // One block: digit offsets, active passes, buffer assignment, and the
 // decoder segment offsets.
-__global__ void __launch_bounds__(kRadix)
-order_plan_kernel(int64_t N, int D, int dbits, const OrderCounts *counts, OrderPlan *plan,
-                  const uint32_t *dec_count, int64_t *seg_off) {
-  pdl_prologue();
+__device__ void plan_block(int64_t N, int D, int dbits, const OrderCounts *counts, OrderPlan *plan,
+                           const uint32_t *dec_count, int64_t *seg_off) {
   __shared__ uint32_t s_warp[kRadix / 32];
   __shared__ long long s_w64[kRadix / 32];
   __shared__ int s_trivial[kPasses];
   __shared__ long long s_carry;
   const int b = threadIdx.x, lane = b & 31, warp = b >> 5;
-  if (*reinterpret_cast<const volatile uint32_t *>(&counts->segmented)) {
-    // segment offsets are already written; no global pass runs
-    if (b == 0) {
-      for (int p = 0; p < kPasses; ++p) {
-        plan->active[p] = 0;
-        plan->ordinal[p] = -1;
-      }
-      plan->gather_buf = -1;
-      plan->npasses = -1;  // neither passes nor the identity order
-    }
-    return;
-  }
+  const bool act = b < kRadix;  // one thread per digit; the rest only meet the barriers
   uint32_t cnt[kPasses];  // all loads first
 #pragma unroll
-  for (int p = 0; p < kPasses; ++p) cnt[p] = counts->h[p][b];
+  for (int p = 0; p < kPasses; ++p) cnt[p] = act ? counts->h[p][b] : 0u;
 #pragma unroll
   for (int p = 0; p < kPasses; ++p) {
     const uint32_t c = cnt[p];
@@ -409,11 +395,13 @@ order_plan_kernel(int64_t N, int D, int dbits, const OrderCounts *counts, OrderP
       const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
       if (lane >= off) incl += y;
     }
-    if (lane == 31) s_warp[warp] = incl;
-    const int triv = __syncthreads_or(static_cast<int64_t>(c) == N || N == 0);
-    uint32_t base = 0;
-    for (int w = 0; w < warp; ++w) base += s_warp[w];
-    plan->digit_off[p][b] = base + incl - c;
+    if (act && lane == 31) s_warp[warp] = incl;
+    const int triv = __syncthreads_or(act && (static_cast<int64_t>(c) == N || N == 0));
+    if (act) {
+      uint32_t base = 0;
+      for (int w = 0; w < warp; ++w) base += s_warp[w];
+      plan->digit_off[p][b] = base + incl - c;
+    }
     if (b == 0) s_trivial[p] = triv;
     __syncthreads();
   }
@@ -469,19 +457,19 @@ order_plan_kernel(int64_t N, int D, int dbits, const OrderCounts *counts, OrderP
   // seg_off = exclusive scan of the per-decoder counts
   for (int base = 0; base <= D; base += kRadix) {
     const int k = base + b;
-    const long long c = k < D ? dec_count[k] : 0;
+    const long long c = act && k < D ? dec_count[k] : 0;
     long long incl = c;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const long long y = __shfl_up_sync(0xffffffffu, incl, off);
       if (lane >= off) incl += y;
     }
-    if (lane == 31) s_w64[warp] = incl;
+    if (act && lane == 31) s_w64[warp] = incl;
     __syncthreads();
     long long wb = 0;
-    for (int w = 0; w < warp; ++w) wb += s_w64[w];
+    for (int w = 0; w < warp && act; ++w) wb += s_w64[w];
     const long long carry = s_carry;
-    if (k <= D) seg_off[k] = carry + wb + incl - c;
+    if (act && k <= D) seg_off[k] = carry + wb + incl - c;
     __syncthreads();
     if (b == kRadix - 1) s_carry = carry + wb + incl;
     __syncthreads();
@@ -722,14 +710,9 @@ __device__ void merge_level(int level, int ntiles, const int64_t *mt_off, const 
   }
 }
 
-__global__ void __launch_bounds__(kMergeThreads)
-order_merge_kernel(int64_t N, const OrderCounts *counts, const int64_t *mt_off,
-                   const int32_t *mt_n, const int32_t *mt_t, unsigned long long *bufA,
-                   unsigned long long *bufB, int32_t *perm) {
-  pdl_prologue();
-  // every block takes the same branch, so no block waits at a barrier alone
-  if (!counts->segmented || counts->nmtiles == 0) return;
-  cg::grid_group grid = cg::this_grid();
+__device__ void merge_all(int64_t N, const OrderCounts *counts, const int64_t *mt_off,
+                          const int32_t *mt_n, const int32_t *mt_t, unsigned long long *bufA,
+                          unsigned long long *bufB, int32_t *perm, cg::grid_group &grid) {
   const int ntiles = static_cast<int>(counts->nmtiles);
   const int levels = static_cast<int>(counts->max_levels);
   for (int level = 0; level < levels; ++level) {
@@ -917,22 +900,33 @@ __device__ bool order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
   return true;
 }
 
-// The global form in one cooperative launch: the active digit passes in
-// turn (arrival digits, the key gather, key digits), with a grid-wide
-// barrier after each; blocks take tiles by ticket, so a look-back only ever
-// waits on tiles already taken by running blocks.  With no active pass the
-// identity is the order.  Nothing runs in the segmented form.
+// The last launch of every call, cooperative, so that its phases meet at grid
+// barriers:
+//   * segmented form: the merge levels of the long queues, if there are any;
+//   * otherwise block 0 plans the global passes (digit offsets, active passes,
+//     buffers, decoder segment offsets), then the passes run, one grid-wide
+//     sweep each: a block takes tiles by ticket until none is left, so a
+//     tile's look-back only waits on tiles already taken by running blocks.
+//     With no active pass the identity is the order.
 __global__ void __launch_bounds__(kPassThreads, 2)
-order_global_kernel(int n_hi, int64_t N, const OrderPlan *plan, unsigned long long *keyA,
-                    unsigned long long *keyB, uint32_t *valA, uint32_t *valB,
-                    const unsigned long long *hi_orig, int32_t *perm, unsigned long long *state,
-                    int64_t tiles, uint32_t *tickets, int32_t *status) {
+order_finish_kernel(int n_hi, int64_t N, int D, int dbits, const OrderCounts *counts,
+                    OrderPlan *plan, const uint32_t *dec_count, int64_t *seg_off,
+                    const int64_t *mt_off, const int32_t *mt_n, const int32_t *mt_t,
+                    unsigned long long *keyA, unsigned long long *keyB, uint32_t *valA,
+                    uint32_t *valB, const unsigned long long *hi_orig, int32_t *perm,
+                    unsigned long long *state, int64_t tiles, uint32_t *tickets, int32_t *status) {
   pdl_prologue();
+  cg::grid_group grid = cg::this_grid();
+  // every block takes the same branches, so no block waits at a barrier alone
+  if (*reinterpret_cast<const volatile uint32_t *>(&counts->segmented)) {
+    if (counts->nmtiles > 0) merge_all(N, counts, mt_off, mt_n, mt_t, keyA, keyB, perm, grid);
+    return;
+  }
+  if (blockIdx.x == 0) plan_block(N, D, dbits, counts, plan, dec_count, seg_off);
+  grid.sync();
   const int npasses = plan->npasses;
-  if (npasses < 0) return;  // segmented form (every block returns)
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PassSmem &sm = *reinterpret_cast<PassSmem *>(smem_raw);
-  cg::grid_group grid = cg::this_grid();
   const bool wide = plan->wide != 0;
   auto run_pass = [&](int p) {
     if (wide)
@@ -968,22 +962,12 @@ order_global_kernel(int n_hi, int64_t N, const OrderPlan *plan, unsigned long lo
     for (int64_t i = first; i < N; i += stride) perm[i] = static_cast<int32_t>(i);
 }
 
-// Blocks of the global kernel that can be resident at once.
-int64_t global_grid(size_t smem) {
+// Blocks of the finishing kernel that can be resident at once (its grid limit
+// as a cooperative launch).
+int64_t finish_grid(size_t smem) {
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, order_global_kernel, kPassThreads,
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, order_finish_kernel, kPassThreads,
                                                     smem) != cudaSuccess ||
-      per_sm < 1)
-    per_sm = 1;
-  return static_cast<int64_t>(per_sm) * sm_count();
-}
-
-// Blocks of the merge kernel that can be resident at once (its grid limit as
-// a cooperative launch).
-int64_t merge_grid() {
-  int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, order_merge_kernel, kMergeThreads, 0) !=
-          cudaSuccess ||
       per_sm < 1)
     per_sm = 1;
   return static_cast<int64_t>(per_sm) * sm_count();
@@ -1073,10 +1057,11 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
     launch_pdl(order_keys_kernel, g, 512, 0, s, N, D, dbits, dec, bound, wait, arrival, max_wait,
                w.counts, w.hi_orig, w.keyA, w.valA, seg_off_out, w.dec_cursor);
   }
-  launch_pdl(order_plan_kernel, 1, kRadix, 0, s, N, D, dbits, w.counts, w.plan, w.dec_count,
-             seg_off_out);
   MAPS_TRY(launch_ok());
-  if (N == 0) return MAPS_OK;
+  if (N == 0) {  // no entries: the segment offsets are all zero
+    MAPS_TRY(cuda_ok(cudaMemsetAsync(seg_off_out, 0, sizeof(int64_t) * (static_cast<size_t>(D) + 1), s)));
+    return MAPS_OK;
+  }
   const size_t seg_smem = sizeof(SegSmem);
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_segsort_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1084,20 +1069,14 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   launch_pdl(order_segsort_kernel, static_cast<unsigned>(std::min<int64_t>(w.nitems_max, 2LL * sms)),
              kSegThreads, seg_smem, s, N, w.counts, w.item_off, w.item_n, w.valA, bound, wait,
              max_wait, perm_out, w.keyA);
-  if (N > kSegMax) {  // some queue may be longer than one block sorts
-    // one block per SM: a level has few tiles, and a smaller grid meets at its
-    // barriers sooner
-    MAPS_TRY(launch_coop(order_merge_kernel,
-                         std::min<int64_t>(w.ntiles_max, std::min<int64_t>(merge_grid(), sms)),
-                         kMergeThreads, 0, s, N, w.counts, w.mt_off, w.mt_n, w.mt_t, w.keyA, w.keyB,
-                         perm_out));
-  }
   const size_t smem = sizeof(PassSmem);
-  MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_global_kernel,
+  MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_finish_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));
-  MAPS_TRY(launch_coop(order_global_kernel, std::min<int64_t>(tiles, global_grid(smem)),
-                       kPassThreads, smem, s, n_hi, N, w.plan, w.keyA, w.keyB, w.valA, w.valB,
+  // the global passes take tiles by ticket, so any resident grid completes them
+  MAPS_TRY(launch_coop(order_finish_kernel, std::min<int64_t>(tiles, finish_grid(smem)),
+                       kPassThreads, smem, s, n_hi, N, D, dbits, w.counts, w.plan, w.dec_count,
+                       seg_off_out, w.mt_off, w.mt_n, w.mt_t, w.keyA, w.keyB, w.valA, w.valB,
                        w.hi_orig, perm_out, w.state, tiles, w.tickets, status));
   return launch_ok();
 }
