@@ -59,6 +59,7 @@ struct OrderCounts {
   uint32_t nmtiles;    // merge tiles of the long queues
   uint32_t max_levels; // merge levels the longest queue needs
   uint32_t done_blocks;  // prep blocks finished
+  uint32_t stable;     // segmented form with the decoder scatter in index order
 };
 
 // Segmented form: when arrival is non-decreasing along the index (so arrival
@@ -66,6 +67,21 @@ struct OrderCounts {
 // entries are scattered to their decoder's segment in any order and each
 // segment is sorted by one block on the key (not promoted, primary, index),
 // which is unique, so no pass has to be stable across blocks.
+// With at most kStableD decoders the scatter keeps index order within each
+// decoder (stable): the prep and key passes split the entries into the same
+// contiguous block ranges, the prep pass counts each block's entries per
+// decoder, its last block turns the counts into each block's first slot in
+// every segment, and the key pass ranks the entries of a round in index order.
+// The segment sort then needs no index digits.
+constexpr int kStableD = 1024;
+constexpr int kPrepBlocks = 304;    // prep and key blocks at most
+constexpr int kKeysU = 4;           // entries per thread per round
+constexpr int kKeysRound = 512 * kKeysU;
+__host__ __device__ __forceinline__ int64_t prep_chunk(int64_t N) {
+  const int64_t per = (N + kPrepBlocks - 1) / kPrepBlocks;
+  const int64_t c = (per + kKeysRound - 1) / kKeysRound * kKeysRound;
+  return c > kKeysRound ? c : kKeysRound;
+}
 constexpr int kSegThreads = 512;
 constexpr int kSegIPT = 11;
 constexpr int kSegMax = kSegThreads * kSegIPT;  // entries one block sorts
@@ -124,7 +140,9 @@ __device__ __forceinline__ int bit_width(uint32_t x) { return x ? 32 - __clz(x) 
 // in index order.
 __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_count,
                                int64_t *seg_off, int64_t *item_off, int32_t *item_n,
-                               int64_t *mt_off, int32_t *mt_n, int32_t *mt_t) {
+                               int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, int G,
+                               uint32_t *blk, int Dp) {
+  __shared__ uint32_t s_part[4 * 512];
   __shared__ long long s_w[32];
   __shared__ int s_bw[32];
   __shared__ long long s_carry;
@@ -192,18 +210,56 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
     }
     __syncthreads();
   }
-  if (t == 0) counts->segmented = __ldcg(&counts->unsorted) == 0 ? 1u : 0u;
+  const bool segmented = __ldcg(&counts->unsorted) == 0;
+  const bool stable = segmented && D <= kStableD;
+  if (t == 0) {
+    counts->segmented = segmented ? 1u : 0u;
+    counts->stable = stable ? 1u : 0u;
+  }
   (void)s_bcarry;
+  if (!stable) return;
+  // Block starts, in place: blk[b][d] = seg_off[d] + sum over b' < b of
+  // blk[b'][d].  Thread (quad q of decoders, row group r) sums its rows, the
+  // row groups' sums are scanned, and the rows are walked again.
+  const int nq = Dp / 4;
+  const int rg = nt / nq > 0 ? nt / nq : 1;
+  const int q = t % nq, r = t / nq;
+  const int L = (G + rg - 1) / rg;
+  const int r0 = r * L, r1 = min(G, r0 + L);
+  uint4 sum = make_uint4(0, 0, 0, 0);
+  if (r < rg)
+    for (int b = r0; b < r1; ++b) {
+      const uint4 v = __ldcg(reinterpret_cast<const uint4 *>(blk + static_cast<int64_t>(b) * Dp) + q);
+      sum.x += v.x, sum.y += v.y, sum.z += v.z, sum.w += v.w;
+    }
+  if (r < rg) reinterpret_cast<uint4 *>(s_part)[r * nq + q] = sum;
+  __syncthreads();  // also orders this block's seg_off stores before the reads below
+  if (r < rg) {
+    uint32_t run[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int d = 4 * q + c;
+      run[c] = d < D ? static_cast<uint32_t>(seg_off[d]) : 0u;
+      for (int rr = 0; rr < r; ++rr) run[c] += s_part[rr * Dp + d];
+    }
+    for (int b = r0; b < r1; ++b) {
+      uint4 *row = reinterpret_cast<uint4 *>(blk + static_cast<int64_t>(b) * Dp) + q;
+      const uint4 v = __ldcg(row);
+      *row = make_uint4(run[0], run[1], run[2], run[3]);
+      run[0] += v.x, run[1] += v.y, run[2] += v.z, run[3] += v.w;
+    }
+  }
 }
 
 // Pass 1: validation, largest non-promoted bound, entries per decoder, and
 // whether arrival is non-decreasing.
 __global__ void __launch_bounds__(512)
-order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
+order_prep_kernel(int64_t N, int D, int64_t chunk, const int32_t *__restrict__ dec,
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
                   uint32_t *dec_count, int32_t *status, int64_t *seg_off, int64_t *item_off,
-                  int32_t *item_n, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t) {
+                  int32_t *item_n, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, uint32_t *blk,
+                  int Dp) {
   pdl_prologue();
   __shared__ uint32_t s_dec[kDecSmem];
   __shared__ bool s_last;
@@ -213,14 +269,16 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
   __syncthreads();
   bool bad = false, unsorted = false;
   uint32_t umax = 0;
-  constexpr int kU = 4;  // entries per thread per round, loads issued together
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x * kU;
-  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x * kU; i0 < N; i0 += stride) {
+  constexpr int kU = kKeysU;  // entries per thread per round, loads issued together
+  // this block's contiguous range of entries (the key pass uses the same)
+  const int64_t r_begin = static_cast<int64_t>(blockIdx.x) * chunk;
+  const int64_t r_end = r_begin + chunk < N ? r_begin + chunk : N;
+  for (int64_t i0 = r_begin; i0 < r_end; i0 += static_cast<int64_t>(blockDim.x) * kU) {
     int32_t d[kU], u[kU], w[kU], ar[kU], an[kU];
 #pragma unroll
     for (int q = 0; q < kU; ++q) {
       const int64_t i = i0 + q * blockDim.x + threadIdx.x;
-      const bool ok = i < N;
+      const bool ok = i < r_end;
       d[q] = ok ? __ldg(dec + i) : -1;
       u[q] = ok ? __ldg(bound + i) : 0;
       w[q] = ok ? __ldg(wait + i) : 0;
@@ -231,7 +289,7 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
     for (int q = 0; q < kU; ++q) {
       const int64_t i = i0 + q * blockDim.x + threadIdx.x;
       int dd = -1;
-      if (i < N) {
+      if (i < r_end) {
         dd = d[q];
         if (dd < 0 || dd >= D || u[q] < 0 || ar[q] < 0) {
           bad = true;
@@ -253,6 +311,9 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
   if ((threadIdx.x & 31) == 0 && umax) atomicMax(&counts->max_bound, umax);
   if (__syncthreads_or(unsorted) && threadIdx.x == 0) atomicOr(&counts->unsorted, 1u);
   if (dec_smem) {
+    if (D <= kStableD)  // this block's counts, for the stable scatter
+      for (int i = threadIdx.x; i < Dp; i += blockDim.x)
+        blk[static_cast<int64_t>(blockIdx.x) * Dp + i] = i < D ? s_dec[i] : 0u;
     // blocks start their flush at different decoders so they do not collide
     const int rot = static_cast<int>((static_cast<int64_t>(blockIdx.x) * 97) % D);
     for (int i = threadIdx.x; i < D; i += blockDim.x) {
@@ -271,32 +332,98 @@ order_prep_kernel(int64_t N, int D, const int32_t *__restrict__ dec,
   __syncthreads();
   if (s_last) {
     __threadfence();
-    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, mt_off, mt_n, mt_t);
+    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, mt_off, mt_n, mt_t, gridDim.x,
+                   blk, Dp);
   }
 }
 
 // Pass 2: keys in the compact layout and the histograms of every digit.
 __global__ void __launch_bounds__(512)
-order_keys_kernel(int64_t N, int D, int dbits, const int32_t *__restrict__ dec,
-                  const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
-                  const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
-                  unsigned long long *hi_orig, unsigned long long *keyA, uint32_t *valA,
-                  const int64_t *seg_off, uint32_t *dec_cursor) {
+order_keys_kernel(int64_t N, int D, int dbits, int64_t chunk, int Dp,
+                  const int32_t *__restrict__ dec, const int32_t *__restrict__ bound,
+                  const int32_t *__restrict__ wait, const int32_t *__restrict__ arrival,
+                  int32_t max_wait, OrderCounts *counts, unsigned long long *hi_orig,
+                  unsigned long long *keyA, uint32_t *valA, const int64_t *seg_off,
+                  uint32_t *dec_cursor, const uint32_t *blk) {
   pdl_prologue();
   if (*reinterpret_cast<volatile uint32_t *>(&counts->segmented)) {
-    // Each entry's index goes to a free slot of its decoder's segment.  A
-    // round of kU entries per thread issues its loads and its (warp-combined)
-    // slot claims together, so the claims' latency overlaps.
-    constexpr int kU = 4;
-    const int lane = threadIdx.x & 31;
+    // Each entry's segment key (not promoted, primary, index) goes to a slot
+    // of its decoder's segment (hi_orig holds the segments).  A round of kU
+    // entries per thread issues its loads and its slot claims together.
+    constexpr int kU = kKeysU;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int ub = bit_width(*reinterpret_cast<volatile uint32_t *>(&counts->max_bound));
+    const int ib = index_bits(N);
+    auto seg_key = [&](int64_t i, int32_t u, int32_t w) {
+      const unsigned long long np = w > max_wait ? 0ull : 1ull;
+      const unsigned long long prim = np ? static_cast<unsigned long long>(u < 0 ? 0 : u) : 0ull;
+      return (np << (ub + ib)) | (prim << ib) | static_cast<unsigned long long>(i);
+    };
+    if (*reinterpret_cast<volatile uint32_t *>(&counts->stable)) {
+      // Stable: this block's range, round by round in index order.  An entry's
+      // slot is its block's start in the segment, plus the entries of its
+      // decoder in earlier rounds and earlier warps of this round, plus its
+      // rank in its warp (item-major, then lane).
+      extern __shared__ __align__(16) uint32_t ksm[];
+      uint32_t *hw = ksm;                 // [warps][Dp] counts, then slot bases
+      uint32_t *run = ksm + kPassWarps * Dp;  // [Dp] next slot of each decoder
+      for (int k = threadIdx.x; k < Dp; k += blockDim.x) run[k] = blk[static_cast<int64_t>(blockIdx.x) * Dp + k];
+      const int64_t r_begin = static_cast<int64_t>(blockIdx.x) * chunk;
+      const int64_t r_end = r_begin + chunk < N ? r_begin + chunk : N;
+      for (int64_t i0 = r_begin; i0 < r_end; i0 += kKeysRound) {
+        for (int k = threadIdx.x; k < kPassWarps * Dp; k += blockDim.x) hw[k] = 0;
+        int d[kU];
+        unsigned long long key[kU];
+#pragma unroll
+        for (int q = 0; q < kU; ++q) {
+          const int64_t i = i0 + warp * (32 * kU) + q * 32 + lane;
+          const bool ok = i < r_end;
+          d[q] = ok ? __ldg(dec + i) : -1;
+          if (ok && (d[q] < 0 || d[q] >= D)) d[q] = 0;  // out-of-domain entries were flagged
+          key[q] = ok ? seg_key(i, __ldg(bound + i), __ldg(wait + i)) : 0ull;
+        }
+        __syncthreads();  // counts zeroed
+        uint32_t rk[kU], base[kU];  // leader lane << 8 | rank in the group; group size, then base
+#pragma unroll
+        for (int q = 0; q < kU; ++q) {
+          const unsigned pe = __match_any_sync(0xffffffffu, d[q]);
+          const int leader = __ffs(pe) - 1;
+          rk[q] = (static_cast<uint32_t>(leader) << 8) | static_cast<uint32_t>(__popc(pe & lanemask_lt()));
+          base[q] = lane == leader ? static_cast<uint32_t>(__popc(pe)) : 0u;
+        }
+#pragma unroll
+        for (int q = 0; q < kU; ++q)  // in item order, so ranks follow the index
+          if (d[q] >= 0 && base[q] != 0) base[q] = atomicAdd(&hw[warp * Dp + d[q]], base[q]);
+        __syncthreads();
+        for (int k = threadIdx.x; k < D; k += blockDim.x) {  // exclusive over the warps
+          uint32_t r = run[k];
+          for (int w = 0; w < kPassWarps; ++w) {
+            const uint32_t c = hw[w * Dp + k];
+            hw[w * Dp + k] = r;
+            r += c;
+          }
+          run[k] = r;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < kU; ++q) {
+          const uint32_t b = __shfl_sync(0xffffffffu, base[q], static_cast<int>(rk[q] >> 8));
+          if (d[q] >= 0) hi_orig[hw[warp * Dp + d[q]] + b + (rk[q] & 255u)] = key[q];
+        }
+        __syncthreads();  // the counts are zeroed again for the next round
+      }
+      return;
+    }
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x * kU;
     for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x * kU; i0 < N; i0 += stride) {
       int d[kU];
+      unsigned long long key[kU];
 #pragma unroll
       for (int q = 0; q < kU; ++q) {
         const int64_t i = i0 + q * blockDim.x + threadIdx.x;
         d[q] = i < N ? __ldg(dec + i) : -1;
         if (i < N && (d[q] < 0 || d[q] >= D)) d[q] = 0;  // out-of-domain entries were flagged
+        key[q] = i < N ? seg_key(i, __ldg(bound + i), __ldg(wait + i)) : 0ull;
       }
       uint32_t slot[kU];
       unsigned peers[kU];
@@ -310,9 +437,7 @@ order_keys_kernel(int64_t N, int D, int dbits, const int32_t *__restrict__ dec,
 #pragma unroll
       for (int q = 0; q < kU; ++q) {
         const uint32_t base = __shfl_sync(0xffffffffu, slot[q], __ffs(peers[q]) - 1);
-        const int64_t i = i0 + q * blockDim.x + threadIdx.x;
-        if (d[q] >= 0)
-          valA[seg_off[d[q]] + base + __popc(peers[q] & lanemask_lt())] = static_cast<uint32_t>(i);
+        if (d[q] >= 0) hi_orig[seg_off[d[q]] + base + __popc(peers[q] & lanemask_lt())] = key[q];
       }
     }
     return;
@@ -485,15 +610,16 @@ struct SegSmem {
 };
 
 // Segmented form, step 2: each sort item (one decoder's queue, at most
-// kSegMax entries) is sorted by one block on (not promoted,
+// kSegMax entries) is sorted by one block on its keys (not promoted,
 // promoted ? 0 : bound, index) with stable 8-bit LSD passes in shared
 // memory, skipping digits that do not vary, and its indices are written.
-// Blocks take items in turn until none is left.
+// After a stable scatter the keys of a queue are already in index order and
+// the index digits are skipped too.  Blocks take items in turn until none is
+// left.
 __global__ void __launch_bounds__(kSegThreads, 2)
 order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_off,
-                     const int32_t *item_n, const uint32_t *seg_idx,
-                     const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
-                     int32_t max_wait, int32_t *perm, unsigned long long *run_keys) {
+                     const int32_t *item_n, const unsigned long long *seg_keys, int32_t *perm,
+                     unsigned long long *run_keys) {
   pdl_prologue();
   if (!counts->segmented) return;
   extern __shared__ __align__(16) unsigned char seg_raw[];
@@ -502,37 +628,21 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
   const int ub = counts->max_bound ? 32 - __clz(counts->max_bound) : 0;
   const int ib = index_bits(N);
   const int nbits = 1 + ub + ib;  // <= 1 + 31 + 31
+  const int lo_bit = counts->stable ? ib : 0;  // first digit that needs sorting
   const int nitems = static_cast<int>(counts->nitems);
   for (int item = blockIdx.x; item < nitems; item += gridDim.x) {
     const int64_t off = item_off[item];
     const bool chunk = item_n[item] < 0;  // a chunk of a long queue: keys for the merges
     const int n = chunk ? -item_n[item] : item_n[item];
     unsigned long long orv = 0, andv = ~0ull;
-    {
-      uint32_t idx[kSegIPT];  // every index load, then every gather, in flight together
-      int32_t u[kSegIPT], w[kSegIPT];
 #pragma unroll
-      for (int it = 0; it < kSegIPT; ++it) {
-        const int x = it * kSegThreads + tid;
-        idx[it] = x < n ? seg_idx[off + x] : 0u;
-      }
-#pragma unroll
-      for (int it = 0; it < kSegIPT; ++it) {
-        const int x = it * kSegThreads + tid;
-        u[it] = x < n ? __ldg(bound + idx[it]) : 0;
-        w[it] = x < n ? __ldg(wait + idx[it]) : 0;
-      }
-#pragma unroll
-      for (int it = 0; it < kSegIPT; ++it) {
-        const int x = it * kSegThreads + tid;
-        if (x < n) {
-          const unsigned long long np = w[it] > max_wait ? 0ull : 1ull;
-          const unsigned long long prim = np ? static_cast<unsigned long long>(u[it] < 0 ? 0 : u[it]) : 0ull;
-          const unsigned long long key = (np << (ub + ib)) | (prim << ib) | idx[it];
-          sm.key[0][x] = key;
-          orv |= key;
-          andv &= key;
-        }
+    for (int it = 0; it < kSegIPT; ++it) {
+      const int x = it * kSegThreads + tid;
+      if (x < n) {
+        const unsigned long long key = seg_keys[off + x];
+        sm.key[0][x] = key;
+        orv |= key;
+        andv &= key;
       }
     }
 #pragma unroll
@@ -555,7 +665,7 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
       diff = o ^ a;  // bits that differ between keys of this segment
     }
     int cur = 0;
-    for (int shift = 0; shift < nbits; shift += 8) {
+    for (int shift = lo_bit; shift < nbits; shift += 8) {
       if (((diff >> shift) & 255ull) == 0) continue;  // same digit everywhere: order unchanged
       for (int i = tid; i < kSegWarps * kRadix; i += kSegThreads) (&sm.hw[0][0])[i] = 0;
       __syncthreads();
@@ -988,6 +1098,9 @@ struct OrderWs {
   int64_t nitems_max, ntiles_max;
   unsigned long long *hi_orig, *keyA, *keyB;
   uint32_t *valA, *valB;
+  uint32_t *blk;      // stable scatter: [blocks][Dp] counts, then block starts
+  int64_t chunk;      // entries per prep / key block
+  int blocks, Dp;
 };
 
 OrderWs carve_order(Carve &c, int64_t N, int D) {
@@ -1014,6 +1127,10 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.keyB = c.take<unsigned long long>(n);
   w.valA = c.take<uint32_t>(n);
   w.valB = c.take<uint32_t>(n);
+  w.chunk = prep_chunk(N);
+  w.blocks = static_cast<int>(std::max<int64_t>(1, (N + w.chunk - 1) / w.chunk));
+  w.Dp = (D + 3) / 4 * 4;
+  w.blk = c.take<uint32_t>(D <= kStableD ? static_cast<size_t>(w.blocks) * w.Dp : 1);
   return w;
 }
 
@@ -1050,12 +1167,19 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   const int sms = sm_count();
   const int64_t tiles = std::max<int64_t>(1, (N + kTile - 1) / kTile);
   if (N > 0) {
-    const int g = static_cast<int>(std::min<int64_t>((N + 2047) / 2048, 2LL * sms));
-    launch_pdl(order_prep_kernel, g, 512, 0, s, N, D, dec, bound, wait, arrival, max_wait,
-               w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n, w.mt_off, w.mt_n,
-               w.mt_t);
-    launch_pdl(order_keys_kernel, g, 512, 0, s, N, D, dbits, dec, bound, wait, arrival, max_wait,
-               w.counts, w.hi_orig, w.keyA, w.valA, seg_off_out, w.dec_cursor);
+    launch_pdl(order_prep_kernel, w.blocks, 512, 0, s, N, D, w.chunk, dec, bound, wait, arrival,
+               max_wait, w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n,
+               w.mt_off, w.mt_n, w.mt_t, w.blk, w.Dp);
+    // the stable scatter's per-warp counts and running slots
+    const size_t keys_smem =
+        D <= kStableD ? sizeof(uint32_t) * static_cast<size_t>(kPassWarps + 1) * w.Dp : 0;
+    if (keys_smem > 0)
+      MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_keys_kernel,
+                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            static_cast<int>(keys_smem))));
+    launch_pdl(order_keys_kernel, w.blocks, 512, keys_smem, s, N, D, dbits, w.chunk, w.Dp, dec,
+               bound, wait, arrival, max_wait, w.counts, w.hi_orig, w.keyA, w.valA, seg_off_out,
+               w.dec_cursor, w.blk);
   }
   MAPS_TRY(launch_ok());
   if (N == 0) {  // no entries: the segment offsets are all zero
@@ -1067,8 +1191,8 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(seg_smem))));
   launch_pdl(order_segsort_kernel, static_cast<unsigned>(std::min<int64_t>(w.nitems_max, 2LL * sms)),
-             kSegThreads, seg_smem, s, N, w.counts, w.item_off, w.item_n, w.valA, bound, wait,
-             max_wait, perm_out, w.keyA);
+             kSegThreads, seg_smem, s, N, w.counts, w.item_off, w.item_n, w.hi_orig, perm_out,
+             w.keyA);
   const size_t smem = sizeof(PassSmem);
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_finish_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
