@@ -601,17 +601,22 @@ __device__ void plan_block(int64_t N, int D, int dbits, const OrderCounts *count
   }
 }
 
+// The segment sort's digits are 9 bits wide.  Each per-warp counter word
+// holds two 16-bit bins (2j low, 2j + 1 high): every count and position is at
+// most kSegMax + a warp's items, so no half carries into the other.
+constexpr int kSegBits = 9;
+constexpr int kSegBins = 1 << kSegBits;
+static_assert(2 * kSegMax + 32 * kSegIPT < 65536, "16-bit bins");
 struct SegSmem {
   unsigned long long key[2][kSegMax];
-  uint32_t hw[kSegWarps][kRadix];  // per-warp digit counts, then bases
-  uint32_t bin_start[kRadix];
-  uint32_t scan_w[kRadix / 32];
+  uint32_t hw[kSegWarps][kSegBins / 2];  // per-warp bin counts, then positions (packed pairs)
+  uint32_t scan_w[kSegBins / 2 / 32];
   unsigned long long orv[kSegWarps], andv[kSegWarps];
 };
 
 // Segmented form, step 2: each sort item (one decoder's queue, at most
 // kSegMax entries) is sorted by one block on its keys (not promoted,
-// promoted ? 0 : bound, index) with stable 8-bit LSD passes in shared
+// promoted ? 0 : bound, index) with stable 9-bit LSD passes in shared
 // memory, skipping digits that do not vary, and its indices are written.
 // After a stable scatter the keys of a queue are already in index order and
 // the index digits are skipped too.  Blocks take items in turn until none is
@@ -665,48 +670,66 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
       diff = o ^ a;  // bits that differ between keys of this segment
     }
     int cur = 0;
-    for (int shift = lo_bit; shift < nbits; shift += 8) {
-      if (((diff >> shift) & 255ull) == 0) continue;  // same digit everywhere: order unchanged
-      for (int i = tid; i < kSegWarps * kRadix; i += kSegThreads) (&sm.hw[0][0])[i] = 0;
+    for (int shift = lo_bit; shift < nbits; shift += kSegBits) {
+      if (((diff >> shift) & (kSegBins - 1)) == 0) continue;  // same digit everywhere: order unchanged
+      for (int i = tid; i < kSegWarps * kSegBins / 2; i += kSegThreads) (&sm.hw[0][0])[i] = 0;
       __syncthreads();
-      // rank within the warp, stable in item order (warp-major, then item, then lane)
-      uint32_t dr[kSegIPT];  // digit << 16 | rank within the warp's items of that digit
+      // rank within the warp, stable in item order (warp-major, then item, then
+      // lane): every match first, then one shared atomic per group leader,
+      // issued in item order, whose old value gives the group's base
+      uint32_t dr[kSegIPT];    // digit << 16 | leader lane << 8 | rank in the group
+      uint32_t base[kSegIPT];  // the leader's group size, then the group's base
 #pragma unroll
       for (int it = 0; it < kSegIPT; ++it) {
         const int x = warp * (32 * kSegIPT) + it * 32 + lane;
-        const bool valid = x < n;
-        const int d = valid ? static_cast<int>((sm.key[cur][x] >> shift) & 255ull) : kRadix;
-        const unsigned peers = __match_any_sync(0xffffffffu, d);
-        uint32_t c = 0;
-        if (valid) c = sm.hw[warp][d];
-        __syncwarp();
-        if (valid && lane == __ffs(peers) - 1) sm.hw[warp][d] = c + __popc(peers);
-        __syncwarp();
-        dr[it] = (static_cast<uint32_t>(d) << 16) | (c + __popc(peers & lanemask_lt()));
+        const int d = x < n ? static_cast<int>((sm.key[cur][x] >> shift) & (kSegBins - 1)) : kSegBins;
+        const unsigned pe = __match_any_sync(0xffffffffu, d);
+        const int leader = __ffs(pe) - 1;
+        dr[it] = (static_cast<uint32_t>(d) << 16) | (static_cast<uint32_t>(leader) << 8) |
+                 static_cast<uint32_t>(__popc(pe & lanemask_lt()));
+        base[it] = lane == leader ? static_cast<uint32_t>(__popc(pe)) : 0u;
       }
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it) {
+        const int d = static_cast<int>(dr[it] >> 16);
+        if (d < kSegBins && base[it] != 0) {
+          const int h = (d & 1) * 16;
+          base[it] = (atomicAdd(&sm.hw[warp][d >> 1], base[it] << h) >> h) & 0xffffu;
+        }
+      }
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it)
+        dr[it] = (dr[it] & 0xffff0000u) +
+                 __shfl_sync(0xffffffffu, base[it], static_cast<int>((dr[it] >> 8) & 31u)) +
+                 (dr[it] & 255u);
       __syncthreads();
-      // per digit: exclusive scan over warps; then over digits
-      uint32_t tot = 0;
-      if (tid < kRadix) {
+      // per bin pair: exclusive scan over the warps (packed), then the bins'
+      // starts from a block scan of the pair totals
+      constexpr int kPairs = kSegBins / 2;
+      uint32_t run = 0, tot = 0;
+      if (tid < kPairs) {
         for (int w = 0; w < kSegWarps; ++w) {
           const uint32_t c = sm.hw[w][tid];
-          sm.hw[w][tid] = tot;
-          tot += c;
+          sm.hw[w][tid] = run;
+          run += c;
         }
-        uint32_t incl = tot;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += y;
-        }
-        if (lane == 31) sm.scan_w[warp] = incl;
-        tot = incl - tot;  // exclusive within the warp
+        tot = (run & 0xffffu) + (run >> 16);
       }
+      uint32_t incl = tot;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (tid < kPairs && lane == 31) sm.scan_w[warp] = incl;
       __syncthreads();
-      if (tid < kRadix) {
+      if (tid < kPairs) {
         uint32_t wb = 0;
         for (int w = 0; w < warp; ++w) wb += sm.scan_w[w];
-        sm.bin_start[tid] = wb + tot;
+        const uint32_t start0 = wb + incl - tot;           // bin 2j
+        const uint32_t start1 = start0 + (run & 0xffffu);  // bin 2j + 1
+        const uint32_t add = start0 | (start1 << 16);
+        for (int w = 0; w < kSegWarps; ++w) sm.hw[w][tid] += add;
       }
       __syncthreads();
 #pragma unroll
@@ -714,7 +737,8 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
         const int x = warp * (32 * kSegIPT) + it * 32 + lane;
         if (x < n) {
           const int d = static_cast<int>(dr[it] >> 16);
-          sm.key[cur ^ 1][sm.bin_start[d] + sm.hw[warp][d] + (dr[it] & 0xffffu)] = sm.key[cur][x];
+          const uint32_t pos = (sm.hw[warp][d >> 1] >> ((d & 1) * 16)) & 0xffffu;
+          sm.key[cur ^ 1][pos + (dr[it] & 0xffffu)] = sm.key[cur][x];
         }
       }
       __syncthreads();
