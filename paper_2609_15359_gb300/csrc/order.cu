@@ -140,9 +140,7 @@ __device__ __forceinline__ int bit_width(uint32_t x) { return x ? 32 - __clz(x) 
 // in index order.
 __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_count,
                                int64_t *seg_off, int64_t *item_off, int32_t *item_n,
-                               int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, int G,
-                               uint32_t *blk, int Dp) {
-  __shared__ uint32_t s_part[4 * 512];
+                               int64_t *mt_off, int32_t *mt_n, int32_t *mt_t) {
   __shared__ long long s_w[32];
   __shared__ int s_bw[32];
   __shared__ long long s_carry;
@@ -217,38 +215,6 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
     counts->stable = stable ? 1u : 0u;
   }
   (void)s_bcarry;
-  if (!stable) return;
-  // Block starts, in place: blk[b][d] = seg_off[d] + sum over b' < b of
-  // blk[b'][d].  Thread (quad q of decoders, row group r) sums its rows, the
-  // row groups' sums are scanned, and the rows are walked again.
-  const int nq = Dp / 4;
-  const int rg = nt / nq > 0 ? nt / nq : 1;
-  const int q = t % nq, r = t / nq;
-  const int L = (G + rg - 1) / rg;
-  const int r0 = r * L, r1 = min(G, r0 + L);
-  uint4 sum = make_uint4(0, 0, 0, 0);
-  if (r < rg)
-    for (int b = r0; b < r1; ++b) {
-      const uint4 v = __ldcg(reinterpret_cast<const uint4 *>(blk + static_cast<int64_t>(b) * Dp) + q);
-      sum.x += v.x, sum.y += v.y, sum.z += v.z, sum.w += v.w;
-    }
-  if (r < rg) reinterpret_cast<uint4 *>(s_part)[r * nq + q] = sum;
-  __syncthreads();  // also orders this block's seg_off stores before the reads below
-  if (r < rg) {
-    uint32_t run[4];
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int d = 4 * q + c;
-      run[c] = d < D ? static_cast<uint32_t>(seg_off[d]) : 0u;
-      for (int rr = 0; rr < r; ++rr) run[c] += s_part[rr * Dp + d];
-    }
-    for (int b = r0; b < r1; ++b) {
-      uint4 *row = reinterpret_cast<uint4 *>(blk + static_cast<int64_t>(b) * Dp) + q;
-      const uint4 v = __ldcg(row);
-      *row = make_uint4(run[0], run[1], run[2], run[3]);
-      run[0] += v.x, run[1] += v.y, run[2] += v.z, run[3] += v.w;
-    }
-  }
 }
 
 // Pass 1: validation, largest non-promoted bound, entries per decoder, and
@@ -332,8 +298,7 @@ order_prep_kernel(int64_t N, int D, int64_t chunk, const int32_t *__restrict__ d
   __syncthreads();
   if (s_last) {
     __threadfence();
-    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, mt_off, mt_n, mt_t, gridDim.x,
-                   blk, Dp);
+    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, mt_off, mt_n, mt_t);
   }
 }
 
@@ -367,7 +332,38 @@ order_keys_kernel(int64_t N, int D, int dbits, int64_t chunk, int Dp,
       extern __shared__ __align__(16) uint32_t ksm[];
       uint32_t *hw = ksm;                 // [warps][Dp] counts, then slot bases
       uint32_t *run = ksm + kPassWarps * Dp;  // [Dp] next slot of each decoder
-      for (int k = threadIdx.x; k < Dp; k += blockDim.x) run[k] = blk[static_cast<int64_t>(blockIdx.x) * Dp + k];
+      {
+        // this block's first slot in every segment: seg_off[d] plus the
+        // counts of the blocks before it.  Thread (quad q of decoders, row
+        // group r) sums rows r, r + rg, ...; the row groups meet in hw.
+        const int nq = Dp / 4;
+        // rg row groups fit in hw: rg * Dp <= kPassWarps * Dp words
+        const int rg = min(kPassWarps, max(1, static_cast<int>(blockDim.x) / nq));
+        const int qd = threadIdx.x % nq, r = threadIdx.x / nq;
+        uint4 a0 = make_uint4(0, 0, 0, 0), a1 = a0;
+        if (r < rg) {
+          const uint4 *col = reinterpret_cast<const uint4 *>(blk) + qd;
+          int b2 = r;
+          for (; b2 + rg < static_cast<int>(blockIdx.x); b2 += 2 * rg) {  // two loads in flight
+            const uint4 v = col[static_cast<int64_t>(b2) * nq], u = col[static_cast<int64_t>(b2 + rg) * nq];
+            a0.x += v.x, a0.y += v.y, a0.z += v.z, a0.w += v.w;
+            a1.x += u.x, a1.y += u.y, a1.z += u.z, a1.w += u.w;
+          }
+          if (b2 < static_cast<int>(blockIdx.x)) {
+            const uint4 v = col[static_cast<int64_t>(b2) * nq];
+            a0.x += v.x, a0.y += v.y, a0.z += v.z, a0.w += v.w;
+          }
+          reinterpret_cast<uint4 *>(hw)[r * nq + qd] =
+              make_uint4(a0.x + a1.x, a0.y + a1.y, a0.z + a1.z, a0.w + a1.w);
+        }
+        __syncthreads();
+        for (int k = threadIdx.x; k < D; k += blockDim.x) {
+          uint32_t v = static_cast<uint32_t>(seg_off[k]);
+          for (int rr = 0; rr < rg; ++rr) v += hw[rr * Dp + k];
+          run[k] = v;
+        }
+        __syncthreads();  // hw is zeroed next
+      }
       const int64_t r_begin = static_cast<int64_t>(blockIdx.x) * chunk;
       const int64_t r_end = r_begin + chunk < N ? r_begin + chunk : N;
       for (int64_t i0 = r_begin; i0 < r_end; i0 += kKeysRound) {
