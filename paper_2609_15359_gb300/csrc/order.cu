@@ -751,7 +751,8 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
 
 // Segmented form, step 3: merge level `level` of the long queues.  Runs of
 // L = kSegMax << level sorted keys are merged pairwise from buf[level & 1]
-// into buf[(level + 1) & 1]; a queue needing fewer levels is left alone.
+// into buf[(level + 1) & 1], except at a queue's last level, which writes its
+// indices to the order; a queue needing fewer levels is left alone.
 // One block writes one tile of kMergeTile outputs: a merge-path search splits
 // the two runs at the tile's ends, the tile's inputs are staged in shared
 // memory, and each thread merges kMergeTile / kMergeThreads outputs after a
@@ -796,7 +797,7 @@ __device__ __forceinline__ int merge_path_warp(const unsigned long long *A, int 
 
 __device__ void merge_level(int level, int ntiles, const int64_t *mt_off, const int32_t *mt_n,
                             const int32_t *mt_t, unsigned long long *bufA,
-                            unsigned long long *bufB) {
+                            unsigned long long *bufB, int32_t *perm, unsigned long long imask) {
   __shared__ unsigned long long s_a[kMergeTile], s_b[kMergeTile];
   __shared__ int s_split[2];
   const unsigned long long *src = (level & 1) ? bufB : bufA;
@@ -828,12 +829,19 @@ __device__ void merge_level(int level, int ntiles, const int64_t *mt_off, const 
     const int dt = threadIdx.x * kPer;
     if (dt < na + nbb) {
       int ia = merge_path(s_a, na, s_b, nbb, dt), ib = dt - ia;
+      // the queue's last level writes its order, the others the next runs
+      const bool last = level == merge_levels(n) - 1;
       unsigned long long *out = dst + off + pstart + d0;
+      int32_t *pout = perm + off + pstart + d0;
 #pragma unroll
       for (int q = 0; q < kPer; ++q) {
         if (dt + q >= na + nbb) break;
         const bool takeA = ib >= nbb || (ia < na && s_a[ia] < s_b[ib]);
-        out[dt + q] = takeA ? s_a[ia++] : s_b[ib++];
+        const unsigned long long k = takeA ? s_a[ia++] : s_b[ib++];
+        if (last)
+          pout[dt + q] = static_cast<int32_t>(k & imask);
+        else
+          out[dt + q] = k;
       }
     }
     __syncthreads();  // the next tile reuses shared memory
@@ -845,20 +853,10 @@ __device__ void merge_all(int64_t N, const OrderCounts *counts, const int64_t *m
                           unsigned long long *bufB, int32_t *perm, cg::grid_group &grid) {
   const int ntiles = static_cast<int>(counts->nmtiles);
   const int levels = static_cast<int>(counts->max_levels);
+  const unsigned long long imask = (1ull << index_bits(N)) - 1;
   for (int level = 0; level < levels; ++level) {
-    merge_level(level, ntiles, mt_off, mt_n, mt_t, bufA, bufB);
-    grid.sync();
-  }
-  // each long queue's final run becomes its order
-  const int ib = index_bits(N);
-  const unsigned long long imask = (1ull << ib) - 1;
-  for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-    const int n = mt_n[tile];
-    const unsigned long long *src = (merge_levels(n) & 1) ? bufB : bufA;
-    const int64_t off = mt_off[tile];
-    const int w0 = mt_t[tile] * kMergeTile, w1 = min(w0 + kMergeTile, n);
-    for (int x = w0 + static_cast<int>(threadIdx.x); x < w1; x += kMergeThreads)
-      perm[off + x] = static_cast<int32_t>(src[off + x] & imask);
+    merge_level(level, ntiles, mt_off, mt_n, mt_t, bufA, bufB, perm, imask);
+    if (level + 1 < levels) grid.sync();
   }
 }
 
