@@ -50,20 +50,20 @@ L2_FLUSH_BYTES = 256 << 20
 # (dram__bytes_read.sum + dram__bytes_write.sum summed over the call's
 # kernels, one launch each), valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 28586560, "source": "calibrate.cu", "source_sha256":
-                  "3a6393a37ce14d09f6e338762dc0ba08c7d1a033a7873853f340c030f0209387"},
-    "occupancy": {"bytes": 34351680, "source": "occupancy.cu", "source_sha256":
-                  "379a765fc47297f3f8241bafa1256b8621eeebae9de3f96359172554405b4f3c"},
-    "dispatch": {"bytes": 25894058, "source": "dispatch.cu", "source_sha256":
-                 "cc8943377249213803429a38d9417b64bdc6bcd27ee45074c7f89c91f72d191e"},
-    "order": {"bytes": 36410730, "source": "order.cu", "source_sha256":
-              "5073063cc1a1ab6f1b07eeda41e4f4b83e37c5ca93a1a02d1f378852ab369a31"},
+    "calibrate": {"bytes": 28586816, "source": "calibrate.cu", "source_sha256":
+                  "dd8c5172871bbabfc606a4ff99cdf1a98fafb7e4db9833dbe2e5fab2935a310f"},
+    "occupancy": {"bytes": 33504981, "source": "occupancy.cu", "source_sha256":
+                  "06173e6d7b5f25d1b4e9f8ef12b41b49833f494de66460e4a96c35ddf5c6800e"},
+    "dispatch": {"bytes": 25893504, "source": "dispatch.cu", "source_sha256":
+                 "6c98d6a4c43dac99891618ecb1e3cc8fe5399c96f7b58ba919f13bc73f21439e"},
+    "order": {"bytes": 41118080, "source": "order.cu", "source_sha256":
+              "08e654cb33fdb17daeead3569eee685985db1b0f21f4aa06a482d3873e4597a7"},
 }
 KERNELS = {
     "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
     "occupancy": "occ_bucket_kernel + occ_tile_kernel (maps_project_occupancy)",
     "dispatch": "carry_scan + bin_count/scan/scatter + dispatch_snapshot_kernel (maps_dispatch)",
-    "order": "order_prep/keys/plan + order_pass_kernel x active digits (maps_order_local)",
+    "order": "order_prep + order_keys + order_segsort + order_finish (maps_order_local)",
 }
 
 
@@ -214,11 +214,10 @@ class Step:
                    M.lib.maps_order_local_workspace_size(R + J, self.D))
         self.ws = M.Workspace(need, device)
         # calibrate 4 (three select passes, bounds); occupancy 2 (bucket, tile);
-        # dispatch 4 (carry scan, bin count, bin scatter, main); order 6 (prep,
-        # keys, plan, segment sort, merge when more entries than one block
-        # sorts, the global radix form)
-        merge = 1 if R + J > 5632 else 0
-        self.kernels_per_step = 4 + 2 + 4 + (5 + merge)
+        # dispatch 4 (carry scan, bin count, bin scatter, main); order 4 (prep,
+        # keys, segment sort, the cooperative finishing kernel: merges or the
+        # global radix form)
+        self.kernels_per_step = 4 + 2 + 4 + 4
 
     def run(self, ev=None):
         M, R = self.M, self.R
