@@ -62,7 +62,7 @@ TRAFFIC = {
 KERNELS = {
     "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
     "occupancy": "occ_bucket_kernel + occ_tile_kernel (maps_project_occupancy)",
-    "dispatch": "carry_scan + bin_count/scan/scatter + dispatch_snapshot_kernel (maps_dispatch)",
+    "dispatch": "dispatch_prep (carry scan + bin count) + bin_scatter + dispatch_snapshot_kernel (maps_dispatch)",
     "order": "order_prep + order_keys + order_segsort + order_finish (maps_order_local)",
 }
 
@@ -214,10 +214,10 @@ class Step:
                    M.lib.maps_order_local_workspace_size(R + J, self.D))
         self.ws = M.Workspace(need, device)
         # calibrate 4 (three select passes, bounds); occupancy 2 (bucket, tile);
-        # dispatch 4 (carry scan, bin count, bin scatter, main); order 4 (prep,
-        # keys, segment sort, the cooperative finishing kernel: merges or the
-        # global radix form)
-        self.kernels_per_step = 4 + 2 + 4 + 4
+        # dispatch 3 (carry scan with bin count, bin scatter, main); order 4
+        # (prep, keys, segment sort, the cooperative finishing kernel: merges or
+        # the global radix form)
+        self.kernels_per_step = 4 + 2 + 3 + 4
 
     def run(self, ev=None):
         M, R = self.M, self.R

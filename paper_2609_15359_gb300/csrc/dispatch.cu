@@ -15,6 +15,8 @@
 // maximum across tiles is resolved by decoupled look-back; and each candidate
 // costs a binary search over D instead of D scores.  Candidates are first
 // bucketed by the tile of their last live step so each tile serves its own.
+// Three launches: the carry scan and the bucket counts (independent, one
+// launch), the bucket scatter, the main kernel.
 //
 // SEQUENTIAL (reservation after each choice) and the literal Algorithm 1
 // modes are separate kernels below.
@@ -123,17 +125,14 @@ kmax_from_K_kernel(int D, int H, const int32_t *__restrict__ K, uint32_t *__rest
 // per decoder; each thread reads 16 consecutive summary entries at once
 // (whole tiles, as W2/16 divides 16), keeps its tiles' maxima in registers,
 // and after a block scan writes its tiles' carries contiguously.
-__global__ void __launch_bounds__(256)
-carry_scan_kernel(int D, int H, int W2, int T2, const uint32_t *__restrict__ kmax,
-                  uint32_t *__restrict__ carry, const int32_t *__restrict__ Q,
-                  const int32_t *__restrict__ cap, int32_t *sig, int32_t *rank_of,
-                  int32_t *capq, int32_t *status) {
-  pdl_prologue();
+__device__ void carry_scan_block(int kk, int D, int H, int W2, int T2,
+                                 const uint32_t *__restrict__ kmax, uint32_t *__restrict__ carry,
+                                 const int32_t *__restrict__ Q, const int32_t *__restrict__ cap,
+                                 int32_t *sig, int32_t *rank_of, int32_t *capq, int32_t *status) {
   __shared__ uint32_t s_w[8];
   __shared__ int s_rank;
   {
     // this decoder's position in (Q, index) order: the decoders before it
-    const int kk = blockIdx.x;
     const int32_t qk = __ldg(Q + kk);
     int r = 0;
     for (int k2 = threadIdx.x; k2 < D; k2 += blockDim.x) {
@@ -155,7 +154,7 @@ carry_scan_kernel(int D, int H, int W2, int T2, const uint32_t *__restrict__ kma
     }
   }
   constexpr int kPer = 16;
-  const int k = blockIdx.x;
+  const int k = kk;
   const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
   const int bpt = W2 / kSumBlock;  // summary blocks per tile (1..16)
   const uint32_t *row = kmax + static_cast<int64_t>(k) * nb;
@@ -230,21 +229,21 @@ struct Unit {
 __device__ void bin_scan_block(int T2, const uint32_t *tcount, uint32_t *toff, Unit *units,
                                uint32_t *nunits);
 
-__global__ void __launch_bounds__(1024)
-bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ cp,
-                 const int32_t *__restrict__ cb, uint32_t *tcount, int32_t *choice,
-                 int64_t *headroom, int32_t *status, uint32_t *ticket, uint32_t *toff,
-                 Unit *units, uint32_t *nunits) {
-  pdl_prologue();
+// Counting block b of nblk.
+__device__ void bin_count_block(int b, int nblk, int64_t J, int H, int W2, int T2,
+                                const int32_t *__restrict__ cp, const int32_t *__restrict__ cb,
+                                uint32_t *tcount, int32_t *choice, int64_t *headroom,
+                                int32_t *status, uint32_t *ticket, uint32_t *toff, Unit *units,
+                                uint32_t *nunits) {
   __shared__ uint32_t s_h[kBinSmem];
   __shared__ bool s_last;
   const bool local = T2 <= kBinSmem;
   if (local)
     for (int i = threadIdx.x; i < T2; i += blockDim.x) s_h[i] = 0;
   __syncthreads();
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t stride = static_cast<int64_t>(nblk) * blockDim.x;
   bool bad = false;
-  for (int64_t j0 = static_cast<int64_t>(blockIdx.x) * blockDim.x; j0 < J; j0 += stride) {
+  for (int64_t j0 = static_cast<int64_t>(b) * blockDim.x; j0 < J; j0 += stride) {
     const int64_t j = j0 + threadIdx.x;
     int tile = -1;
     if (j < J) {
@@ -265,7 +264,7 @@ bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ c
   if (local) {
     __syncthreads();
     // start each block's flush at a different tile so blocks do not collide
-    const int rot = static_cast<int>((static_cast<int64_t>(blockIdx.x) * 97) % T2);
+    const int rot = static_cast<int>((static_cast<int64_t>(b) * 97) % T2);
     for (int i = threadIdx.x; i < T2; i += blockDim.x) {
       const int t = (i + rot) % T2;
       if (s_h[t]) atomicAdd(&tcount[t], s_h[t]);
@@ -277,7 +276,7 @@ bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ c
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
-    s_last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+    s_last = atomicAdd(ticket, 1u) == static_cast<uint32_t>(nblk) - 1;
   }
   __syncthreads();
   if (s_last) {
@@ -286,63 +285,78 @@ bin_count_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ c
   }
 }
 
-// Run by the last bin_count block (1024 threads): tile offsets toff[0..T2]
-// and the work units (a tile with c candidates gives ceil(c / kUnitCands)
-// units; the unit count goes to *nunits).
+// The two independent first steps in one launch: blocks [0, D) scan the
+// carries of decoder blockIdx.x, the others count the candidates per tile.
+__global__ void __launch_bounds__(256)
+dispatch_prep_kernel(int D, int H, int W2, int T2, const uint32_t *__restrict__ kmax,
+                     uint32_t *__restrict__ carry, const int32_t *__restrict__ Q,
+                     const int32_t *__restrict__ cap, int32_t *sig, int32_t *rank_of,
+                     int32_t *capq, int64_t J, const int32_t *__restrict__ cp,
+                     const int32_t *__restrict__ cb, uint32_t *tcount, int32_t *choice,
+                     int64_t *headroom, int32_t *status, uint32_t *ticket, uint32_t *toff,
+                     Unit *units, uint32_t *nunits) {
+  pdl_prologue();
+  if (static_cast<int>(blockIdx.x) < D)
+    carry_scan_block(blockIdx.x, D, H, W2, T2, kmax, carry, Q, cap, sig, rank_of, capq, status);
+  else
+    bin_count_block(blockIdx.x - D, gridDim.x - D, J, H, W2, T2, cp, cb, tcount, choice, headroom,
+                    status, ticket, toff, units, nunits);
+}
+
+// Run by the last counting block (any multiple of 32 threads up to 1024):
+// tile offsets toff[0..T2] and the work units (a tile with c candidates gives
+// ceil(c / kUnitCands) units; the unit count goes to *nunits).
 __device__ void bin_scan_block(int T2, const uint32_t *tcount, uint32_t *toff, Unit *units,
                                uint32_t *nunits) {
   __shared__ uint32_t s_w[2][32];
-  __shared__ uint32_t s_carry[2];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) s_carry[0] = s_carry[1] = 0;
-  __syncthreads();
-  for (int base = 0; base < T2; base += 1024) {
-    const int i = base + threadIdx.x;
-    const uint32_t c = i < T2 ? __ldcg(tcount + i) : 0u;
-    const uint32_t nu = (c + kUnitCands - 1) / kUnitCands;
-    uint32_t ic = c, iu = nu;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t yc = __shfl_up_sync(0xffffffffu, ic, off);
-      const uint32_t yu = __shfl_up_sync(0xffffffffu, iu, off);
-      if (lane >= off) {
-        ic += yc;
-        iu += yu;
-      }
-    }
-    if (lane == 31) {
-      s_w[0][warp] = ic;
-      s_w[1][warp] = iu;
-    }
-    __syncthreads();
-    uint32_t bc = s_carry[0], bu = s_carry[1];
-    for (int w = 0; w < warp; ++w) {
-      bc += s_w[0][w];
-      bu += s_w[1][w];
-    }
-    if (i < T2) {
-      const uint32_t start = bc + ic - c;
-      toff[i] = start;
-      uint32_t u0 = bu + iu - nu;
-      for (uint32_t q = 0; q < nu; ++q) {
-        Unit un;
-        un.tile = i;
-        un.start = static_cast<int32_t>(start + q * kUnitCands);
-        un.count = static_cast<int32_t>(min(static_cast<uint32_t>(kUnitCands), c - q * kUnitCands));
-        un.pad = 0;
-        units[u0 + q] = un;
-      }
-    }
-    __syncthreads();
-    if (threadIdx.x == 1023) {
-      s_carry[0] = bc + ic;
-      s_carry[1] = bu + iu;
-    }
-    __syncthreads();
+  const int nt = blockDim.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  // each thread takes a contiguous run of tiles: one block scan in all
+  const int per = (T2 + nt - 1) / nt;
+  const int i0 = min(T2, static_cast<int>(threadIdx.x) * per), i1 = min(T2, i0 + per);
+  uint32_t sc = 0, su = 0;
+  for (int i = i0; i < i1; ++i) {
+    const uint32_t c = __ldcg(tcount + i);
+    sc += c;
+    su += (c + kUnitCands - 1) / kUnitCands;
   }
-  if (threadIdx.x == 0) {
-    toff[T2] = s_carry[0];
-    *nunits = s_carry[1];
+  uint32_t ic = sc, iu = su;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t yc = __shfl_up_sync(0xffffffffu, ic, off);
+    const uint32_t yu = __shfl_up_sync(0xffffffffu, iu, off);
+    if (lane >= off) {
+      ic += yc;
+      iu += yu;
+    }
+  }
+  if (lane == 31) {
+    s_w[0][warp] = ic;
+    s_w[1][warp] = iu;
+  }
+  __syncthreads();
+  uint32_t rc = ic - sc, ru = iu - su;  // exclusive starts of this thread's run
+  for (int w = 0; w < warp; ++w) {
+    rc += s_w[0][w];
+    ru += s_w[1][w];
+  }
+  for (int i = i0; i < i1; ++i) {
+    const uint32_t c = __ldcg(tcount + i);
+    const uint32_t nu = (c + kUnitCands - 1) / kUnitCands;
+    toff[i] = rc;
+    for (uint32_t q = 0; q < nu; ++q) {
+      Unit un;
+      un.tile = i;
+      un.start = static_cast<int32_t>(rc + q * kUnitCands);
+      un.count = static_cast<int32_t>(min(static_cast<uint32_t>(kUnitCands), c - q * kUnitCands));
+      un.pad = 0;
+      units[ru + q] = un;
+    }
+    rc += c;
+    ru += nu;
+  }
+  if (threadIdx.x == nt - 1) {  // the last thread's run ends at the totals
+    toff[T2] = rc;
+    *nunits = ru;
   }
 }
 
@@ -1134,11 +1148,12 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
     launch_pdl(kmax_from_K_kernel, gk, 256, 0, s, D, H, K, w.kmax, status);
     kmax = w.kmax;
   }
-  launch_pdl(carry_scan_kernel, D, 256, 0, s, D, H, g.W2, g.T2, kmax, w.carry, Q, cap, w.sig,
-             w.rank_of, w.capq, status);
+  // carries of D decoders, and candidate counts in blocks of 1,024 candidates
+  const int gc = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((J + 1023) / 1024, 4LL * sms)));
+  launch_pdl(dispatch_prep_kernel, D + gc, 256, 0, s, D, H, g.W2, g.T2, kmax, w.carry, Q, cap,
+             w.sig, w.rank_of, w.capq, J, cp, cb, tcount, choice, headroom, status, ticket, w.toff,
+             w.units, nunits);
   const int gb = static_cast<int>(std::min<int64_t>((J + 1023) / 1024, 4LL * sms));
-  launch_pdl(bin_count_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, tcount, choice, headroom,
-             status, ticket, w.toff, w.units, nunits);
   launch_pdl(bin_scatter_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord,
              w.sp, w.su);
   MAPS_TRY(launch_ok());
