@@ -90,7 +90,7 @@ __device__ __forceinline__ int candidate_steps(int32_t U, int H) {
 }
 
 constexpr int kSumBlock = 16;      // steps per kmax summary entry
-constexpr int kUnitCands = 4096;   // candidates per work unit of the main kernel
+constexpr int kUnitCands = 1024;   // candidates per work unit of the main kernel
 
 // kmax[k][b] = max over the 16 steps of block b of K[k][t] + t, for callers
 // that do not pass the summary from maps_project_occupancy.
