@@ -65,6 +65,14 @@ struct TileSmem {
   TileScan scan;
 };
 
+// This warp's staging rows for the stores (32 lanes x (CPT + 4) words), over
+// the count bins, which hold exactly the block's rows when CPT >= 8.
+template <int CPT>
+__device__ __forceinline__ uint32_t *stage_rows(TileSmem<CPT> &sm) {
+  static_assert(CPT < 8 || TileSmem<CPT>::WP >= kOccThreads * (CPT + 4), "staging fits the bins");
+  return reinterpret_cast<uint32_t *>(sm.cnt) + (threadIdx.x >> 5) * 32 * (CPT + 4);
+}
+
 template <int CPT>
 __device__ __forceinline__ void zero_bins(TileSmem<CPT> &sm) {
   for (int i = threadIdx.x * 4; i < TileSmem<CPT>::WP; i += kOccThreads * 4) {
@@ -90,56 +98,78 @@ template <int CPT, bool VEC>
 __device__ __forceinline__ void write_cells(const uint32_t (&bc)[CPT], const uint32_t (&bs)[CPT],
                                             uint32_t tot_c, uint32_t tot_s, uint32_t c_hi,
                                             uint32_t s_hi, int H, int k, int t0, int32_t *K,
-                                            uint32_t *kmax, int32_t *status) {
+                                            uint32_t *kmax, int32_t *status, uint32_t *stage) {
   const int tid = threadIdx.x, lane = tid & 31;
   const int cell0 = t0 + tid * CPT;
   const uint32_t tc0 = static_cast<uint32_t>(cell0);
+  int32_t *row = K + static_cast<int64_t>(k) * H;
   uint32_t bmax = 0;  // max of K + t over this thread's valid cells
-  if (cell0 < H) {
-    // Both running sums only grow towards the thread's first cell, so their
-    // totals and the last cell's step bound every cell of the thread.
-    const unsigned long long bound64 =
-        static_cast<unsigned long long>(tc0 + CPT - 1) * (c_hi + tot_c) + (s_hi + tot_s);
-    int32_t *row = K + static_cast<int64_t>(k) * H;
+  // Both running sums only grow towards the thread's first cell, so their
+  // totals and the last cell's step bound every cell of the thread.
+  const unsigned long long bound64 =
+      static_cast<unsigned long long>(tc0 + CPT - 1) * (c_hi + tot_c) + (s_hi + tot_s);
+  // every cell valid and exact in 32 bits
+  const bool fast = VEC && cell0 + CPT <= H && bound64 <= 0x7fffffffull;
+  uint32_t o[CPT];
+  if (fast) {
     uint32_t run_c = c_hi, run_s = s_hi;
-    if (VEC && bound64 <= 0x7fffffffull && cell0 + CPT <= H) {
-      // every cell valid and exact in 32 bits
-      uint32_t o[CPT];
-      if (tot_c == 0) {
-        // no resident ends in these cells: K is affine in t over them, and
-        // K + t grows with t, so the last cell holds the maximum
+    if (tot_c == 0) {
+      // no resident ends in these cells: K is affine in t over them, and
+      // K + t grows with t, so the last cell holds the maximum
 #pragma unroll
-        for (int c = 0; c < CPT; ++c) o[c] = (tc0 + c) * run_c + run_s;
-        bmax = o[CPT - 1] + tc0 + CPT - 1;
-      } else {
-#pragma unroll
-        for (int c = CPT - 1; c >= 0; --c) {
-          run_c += bc[c];
-          run_s += bs[c];
-          o[c] = (tc0 + c) * run_c + run_s;
-          bmax = max(bmax, o[c] + tc0 + c);
-        }
-      }
-#pragma unroll
-      for (int c = 0; c < CPT; c += 4)
-        *reinterpret_cast<int4 *>(row + cell0 + c) = make_int4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+      for (int c = 0; c < CPT; ++c) o[c] = (tc0 + c) * run_c + run_s;
+      bmax = o[CPT - 1] + tc0 + CPT - 1;
     } else {
-      bool over = false;
 #pragma unroll
       for (int c = CPT - 1; c >= 0; --c) {
         run_c += bc[c];
         run_s += bs[c];
-        if (cell0 + c < H) {
-          const uint32_t t = tc0 + c;
-          const unsigned long long v = static_cast<unsigned long long>(t) * run_c + run_s;
-          over |= (v >> 31) != 0;
-          const uint32_t o = static_cast<uint32_t>(v);
-          bmax = max(bmax, o + t);
-          row[cell0 + c] = static_cast<int32_t>(o);
-        }
+        o[c] = (tc0 + c) * run_c + run_s;
+        bmax = max(bmax, o[c] + tc0 + c);
       }
-      if (over) flag_error(status, MAPS_E_RANGE);
     }
+  }
+  if (CPT >= 8 && __all_sync(0xffffffffu, fast)) {
+    // The warp's 32 * CPT cells are contiguous: pass them through this warp's
+    // shared staging rows (CPT + 4 words a lane, so both the row writes and
+    // the chunk reads spread over the banks) and store 512 contiguous bytes
+    // per instruction, whole sectors instead of half sectors.
+    constexpr int kLS = CPT + 4;
+    constexpr int kChunks = CPT / 4;  // 16-byte chunks per lane
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c)
+      *reinterpret_cast<uint4 *>(stage + lane * kLS + 4 * c) =
+          make_uint4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
+    __syncwarp();
+    int32_t *wrow = row + (cell0 - lane * CPT);  // the warp's first cell
+#pragma unroll
+    for (int s2 = 0; s2 < kChunks; ++s2) {
+      const int q = s2 * 32 + lane;  // chunk of the warp's range
+      const uint4 v = *reinterpret_cast<const uint4 *>(stage + (q / kChunks) * kLS + (q % kChunks) * 4);
+      *reinterpret_cast<uint4 *>(wrow + 4 * q) = v;
+    }
+    __syncwarp();  // the staging rows are reused
+  } else if (fast) {
+#pragma unroll
+    for (int c = 0; c < CPT; c += 4)
+      *reinterpret_cast<int4 *>(row + cell0 + c) = make_int4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+  } else if (cell0 < H) {
+    uint32_t run_c = c_hi, run_s = s_hi;
+    bool over = false;
+#pragma unroll
+    for (int c = CPT - 1; c >= 0; --c) {
+      run_c += bc[c];
+      run_s += bs[c];
+      if (cell0 + c < H) {
+        const uint32_t t = tc0 + c;
+        const unsigned long long v = static_cast<unsigned long long>(t) * run_c + run_s;
+        over |= (v >> 31) != 0;
+        const uint32_t ov = static_cast<uint32_t>(v);
+        bmax = max(bmax, ov + t);
+        row[cell0 + c] = static_cast<int32_t>(ov);
+      }
+    }
+    if (over) flag_error(status, MAPS_E_RANGE);
   }
   if (kmax != nullptr) {
     constexpr int L = kBlock / CPT > 0 ? kBlock / CPT : 1;  // lanes per 16-step block
@@ -159,7 +189,7 @@ __device__ __forceinline__ void write_cells(const uint32_t (&bc)[CPT], const uin
 template <int CPT, bool VEC>
 __device__ __forceinline__ void emit_cells(const uint32_t (&bc)[CPT], const uint32_t (&bs)[CPT],
                                            TileScan &sc, int H, int k, int t0, int32_t *K,
-                                           uint32_t *kmax, int32_t *status) {
+                                           uint32_t *kmax, int32_t *status, uint32_t *stage) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   uint32_t tot_c = 0, tot_s = 0;
 #pragma unroll
@@ -216,7 +246,7 @@ __device__ __forceinline__ void emit_cells(const uint32_t (&bc)[CPT], const uint
 
   const uint32_t c_hi = sc.carry[0] + sc.wsum[0][warp] + (suf_c - tot_c);
   const uint32_t s_hi = sc.carry[1] + sc.wsum[1][warp] + (suf_s - tot_s);
-  write_cells<CPT, VEC>(bc, bs, tot_c, tot_s, c_hi, s_hi, H, k, t0, K, kmax, status);
+  write_cells<CPT, VEC>(bc, bs, tot_c, tot_s, c_hi, s_hi, H, k, t0, K, kmax, status, stage);
 }
 
 // The histogram form: each thread takes its own CPT bins into registers.
@@ -233,7 +263,9 @@ __device__ __forceinline__ void emit_tile(TileSmem<CPT> &sm, int H, int k, int t
     bc[c] = x.x, bc[c + 1] = x.y, bc[c + 2] = x.z, bc[c + 3] = x.w;
     bs[c] = y.x, bs[c + 1] = y.y, bs[c + 2] = y.z, bs[c + 3] = y.w;
   }
-  emit_cells<CPT, VEC>(bc, bs, sm.scan, H, k, t0, K, kmax, status);
+  // the staging rows reuse the count bins: every thread has read its own bins
+  // before the scan's first barrier
+  emit_cells<CPT, VEC>(bc, bs, sm.scan, H, k, t0, K, kmax, status, stage_rows(sm));
 }
 
 // Resident terms: false for a negative length (a range error).
@@ -455,7 +487,7 @@ occ_bucket_kernel(int H, int T, int log2W, const int64_t *__restrict__ res_off, 
 // it) from the bucket kernel.
 // ---------------------------------------------------------------------------
 template <int CPT, bool VEC>
-__global__ void __launch_bounds__(kOccThreads, 5)
+__global__ void __launch_bounds__(kOccThreads, 4)
 occ_tile_kernel(int H, int D, int T, const int64_t *__restrict__ res_off, int64_t R,
                 const int2 *__restrict__ bucket, const int32_t *__restrict__ tile_off,
                 const uint2 *__restrict__ tile_carry, int32_t *__restrict__ K,
@@ -500,7 +532,8 @@ occ_tile_kernel(int H, int D, int T, const int64_t *__restrict__ res_off, int64_
           }
       }
     }
-    write_cells<CPT, VEC>(bc, bs, tot_c, tot_s, c_hi, s_hi, H, k, t0, K, kmax, status);
+    write_cells<CPT, VEC>(bc, bs, tot_c, tot_s, c_hi, s_hi, H, k, t0, K, kmax, status,
+                          stage_rows(sm));
     return;
   }
 
@@ -529,7 +562,7 @@ occ_tile_kernel(int H, int D, int T, const int64_t *__restrict__ res_off, int64_
 // Long horizons: every tile CTA streams all of its decoder's residents.
 // ---------------------------------------------------------------------------
 template <int CPT, bool VEC>
-__global__ void __launch_bounds__(kOccThreads, 5)
+__global__ void __launch_bounds__(kOccThreads, 4)
 occ_direct_kernel(int H, int T, const int64_t *__restrict__ res_off, int64_t R,
                   const int32_t *__restrict__ prompt, const int32_t *__restrict__ gen,
                   const int32_t *__restrict__ bound, int32_t *__restrict__ K,
