@@ -83,7 +83,7 @@ __host__ __device__ __forceinline__ int64_t prep_chunk(int64_t N) {
   return c > kKeysRound ? c : kKeysRound;
 }
 constexpr int kSegThreads = 512;
-constexpr int kSegIPT = 11;
+constexpr int kSegIPT = 9;
 constexpr int kSegMax = kSegThreads * kSegIPT;  // entries one block sorts
 // A longer queue is sorted as chunks of kSegMax entries, whose sorted runs are
 // then merged pairwise, level by level, in tiles of kMergeTile outputs

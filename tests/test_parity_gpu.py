@@ -445,10 +445,13 @@ def test_dispatch_errors(M, ws, oracle):
                                                 (300000, 256, False), (1000, 70000, True),
                                                 # one decoder's queue at, and past, the most a
                                                 # block sorts in shared memory
+                                                (4608, 1, True), (4609, 1, True),
                                                 (5632, 1, True), (5633, 1, True),
                                                 (20000, 2, True), (300000, 256, True),
-                                                # a queue of 18 chunks: five merge levels
-                                                (100000, 1, True)])
+                                                # a queue of 22 chunks: five merge levels
+                                                (100000, 1, True),
+                                                # more decoders than the stable scatter takes
+                                                (60000, 1500, True)])
 def test_order_random(M, ws, oracle, N, D, sorted_arrival):
     rng = np.random.default_rng(N + D)
     dec = rng.integers(0, D, N).astype(np.int32)
