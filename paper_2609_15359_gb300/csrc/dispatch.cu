@@ -120,11 +120,12 @@ kmax_from_K_kernel(int D, int H, const int32_t *__restrict__ K, uint32_t *__rest
   if (neg) flag_error(status, MAPS_E_RANGE);
 }
 
-// carry[i][k] = max of K[k][t] + t over t < i*W2 (0 for i = 0): the prefix
+// carry[k][i] = max of K[k][t] + t over t < i*W2 (0 for i = 0): the prefix
 // maximum that horizon tile i inherits from the tiles before it.  One block
 // per decoder; each thread reads 16 consecutive summary entries at once
 // (whole tiles, as W2/16 divides 16), keeps its tiles' maxima in registers,
-// and after a block scan writes its tiles' carries contiguously.
+// and after a block scan writes its tiles' carries (the decoder's row of the
+// carries is contiguous; a work unit later reads one word per decoder).
 __device__ void carry_scan_block(int kk, int D, int H, int W2, int T2,
                                  const uint32_t *__restrict__ kmax, uint32_t *__restrict__ carry,
                                  const int32_t *__restrict__ Q, const int32_t *__restrict__ cap,
@@ -158,7 +159,7 @@ __device__ void carry_scan_block(int kk, int D, int H, int W2, int T2,
   const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
   const int bpt = W2 / kSumBlock;  // summary blocks per tile (1..16)
   const uint32_t *row = kmax + static_cast<int64_t>(k) * nb;
-  uint32_t *out = carry + k;  // carry[i][k], decoder-contiguous per tile
+  uint32_t *out = carry + static_cast<int64_t>(k) * T2;  // carry[k][i], tile-contiguous per decoder
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const bool vec = (reinterpret_cast<uintptr_t>(row) % 16) == 0;
   uint32_t run = 0;
@@ -200,7 +201,7 @@ __device__ void carry_scan_block(int kk, int D, int H, int W2, int T2,
     for (int q = 0; q < kPer; ++q) {
       if (q % bpt == 0) {
         const int64_t ti = tile0 + q / bpt;
-        if (ti < T2) out[ti * D] = r;
+        if (ti < T2) out[ti] = r;
       }
       r = v[q] > r ? v[q] : r;
     }
@@ -438,7 +439,7 @@ struct SnapArgs {
   bool use_tma;
   const int32_t *K;
   const int32_t *sig, *rank_of, *capq;  // queue order
-  const uint32_t *carry;                // [T2][D]
+  const uint32_t *carry;                // [D][T2]
   const Unit *units;
   const uint32_t *nunits;
   const int32_t *ord, *sp, *su;
@@ -494,7 +495,7 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
     s_sig[k] = __ldg(a.sig + k);
     s_rank[k] = __ldg(a.rank_of + k);
     s_capq[k] = __ldg(a.capq + k);
-    s_carry[k] = __ldg(a.carry + static_cast<int64_t>(un.tile) * D + k);
+    s_carry[k] = __ldg(a.carry + static_cast<int64_t>(k) * a.T2 + un.tile);
   }
   for (int c = tid; c < W2; c += kMainThreads) s_slot[c] = 0;
   __syncthreads();
@@ -1079,7 +1080,7 @@ struct SnapWs {
   Unit *units;
   int32_t *ord, *sp, *su;
   int32_t *sig, *rank_of, *capq;
-  uint32_t *carry;  // [T2][D]
+  uint32_t *carry;  // [D][T2]
   uint32_t *kmax;   // [D][ceil(H/16)], used when the caller passes none
   int64_t max_units;
 };
