@@ -364,7 +364,7 @@ __device__ void bin_scan_block(int T2, const uint32_t *tcount, uint32_t *toff, U
 // Place every valid candidate into its tile's bucket as (index, prompt,
 // steps).  The order inside a bucket does not matter: each candidate's
 // decision depends only on itself.
-__global__ void __launch_bounds__(1024)
+__global__ void __launch_bounds__(256)
 bin_scatter_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ cp,
                    const int32_t *__restrict__ cb, const uint32_t *toff, uint32_t *tcursor,
                    int32_t *ord, int32_t *sp, int32_t *su) {
@@ -1149,13 +1149,13 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
     launch_pdl(kmax_from_K_kernel, gk, 256, 0, s, D, H, K, w.kmax, status);
     kmax = w.kmax;
   }
-  // carries of D decoders, and candidate counts in blocks of 1,024 candidates
-  const int gc = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((J + 1023) / 1024, 4LL * sms)));
+  // carries of D decoders, and candidate counts in blocks of 256 candidates
+  const int gc = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((J + 255) / 256, 4LL * sms)));
   launch_pdl(dispatch_prep_kernel, D + gc, 256, 0, s, D, H, g.W2, g.T2, kmax, w.carry, Q, cap,
              w.sig, w.rank_of, w.capq, J, cp, cb, tcount, choice, headroom, status, ticket, w.toff,
              w.units, nunits);
-  const int gb = static_cast<int>(std::min<int64_t>((J + 1023) / 1024, 4LL * sms));
-  launch_pdl(bin_scatter_kernel, gb, 1024, 0, s, J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord,
+  const int gb = static_cast<int>(std::min<int64_t>((J + 255) / 256, 4LL * sms));
+  launch_pdl(bin_scatter_kernel, gb, 256, 0, s, J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord,
              w.sp, w.su);
   MAPS_TRY(launch_ok());
 
