@@ -20,6 +20,7 @@
 // The host issues the launches; it reads 24 bytes of loop state once per
 // batch (the request, completion and waiting counts that size the calls).
 #include <algorithm>
+#include <climits>
 
 #include "maps_internal.cuh"
 
@@ -232,6 +233,186 @@ stream_csr_kernel(int nact, int D, int rr, const int32_t *q_dev, int32_t *q_out_
     rU[pos] = Uq[x];
   }
   if (tid == 0) *q_out_b = rr ? -1 : q_dev[0];
+}
+
+// 5. (shared-memory form) SEQUENTIAL dispatch of the batch without a dense K.
+// Decoder k's occupancy is held as its residents' pairs (e, b), sorted by e:
+// on a step t the live residents are those with e > t, so
+//   K_k(t) + t = S(t) + t (C(t) + 1),  S / C = b-sum / count of e > t,
+// which is linear and rising between consecutive end steps.  Its maximum over
+// t < u is therefore taken at t = e_i - 1 for some e_i <= u, or at t = u - 1:
+// with the pairs sorted ascending and S_i / C_i the sums over pairs i.. n-1,
+//   M_k(u) = max( max_{e_i <= u} S_i + (e_i - 1)(C_i + 1),
+//                 S' + (u - 1)(C' + 1) ),  S' / C' over the pairs with e > u.
+// (A pair tied on e with one before it gives a value no larger than the
+// first's, so ties need no merging.)  One warp walks the batch: a lane scores
+// a decoder, the warp picks (feasible with the smallest Q, else the largest
+// headroom, ties to the lowest index) and reserves the candidate's footprint
+// by inserting (u, p + 1) into the chosen decoder's list.  The same decisions and range errors as
+// the dense projection followed by maps_dispatch SEQUENTIAL.
+// Shared memory: the pool of pairs (the residents of decoder k plus room for
+// nb reservations at base_k = res_off[k] + k nb), the unsorted pairs, and the
+// per-decoder tables.
+size_t stream_dispatch_smem(int D, int nact, int nb) {
+  const size_t pool = static_cast<size_t>(nact) + static_cast<size_t>(D) * nb;
+  return 8 * (pool + static_cast<size_t>(nact)) + 24 * static_cast<size_t>(D) +
+         8 * static_cast<size_t>(nb) + 64;
+}
+
+__global__ void __launch_bounds__(kSt, 1)
+stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32_t *rp,
+                       const int32_t *rg, const int32_t *rU, const int32_t *capv, int32_t *Q,
+                       const int32_t *cp, const int32_t *cU, int32_t *choice, int64_t *headroom,
+                       int32_t *status) {
+  pdl_prologue();
+  extern __shared__ __align__(16) unsigned char sdm[];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nact = static_cast<int>(res_off[D]);
+  const int pool = nact + D * nb;
+  long long *s_M = reinterpret_cast<long long *>(sdm);     // [D]
+  int32_t *E = reinterpret_cast<int32_t *>(s_M + D);       // [pool] sorted end steps
+  int32_t *Bv = E + pool;                                  // [pool] their b
+  int32_t *uE = Bv + pool;                                 // [nact] unsorted
+  int32_t *uB = uE + nact;
+  int32_t *s_base = uB + nact, *s_n = s_base + D, *s_q = s_n + D, *s_cap = s_q + D;
+  int32_t *s_cp = s_cap + D, *s_cu = s_cp + nb;           // [nb] the batch
+  __shared__ int s_bad;
+  if (tid == 0) s_bad = 0;
+  __syncthreads();
+  for (int k = tid; k < D; k += kSt) {
+    const int lo = static_cast<int>(res_off[k]);
+    s_base[k] = lo + k * nb;
+    s_n[k] = static_cast<int>(res_off[k + 1]) - lo;
+    s_q[k] = Q[k];
+    s_cap[k] = capv[k];
+    if ((s_q[k] | s_cap[k]) < 0) s_bad = 1;
+  }
+  for (int j = tid; j < nb; j += kSt) {
+    s_cp[j] = cp[j];
+    s_cu[j] = cU[j];
+  }
+  for (int x = tid; x < nact; x += kSt) {  // the residents' pairs, as the projection forms them
+    const int32_t p = rp[x], g = rg[x], U = rU[x];
+    int32_t e = 1, b = 0;
+    if ((p | g | U) < 0) {
+      s_bad = 1;
+    } else {
+      const long long bb = static_cast<long long>(p) + g + 1;
+      if (bb > 0x7fffffffLL) s_bad = 1;
+      b = static_cast<int32_t>(bb > 0x7fffffffLL ? 0x7fffffffLL : bb);
+      e = U - g;
+      e = e < 1 ? 1 : (e > H ? H : e);
+    }
+    uE[x] = e;
+    uB[x] = b;
+  }
+  __syncthreads();
+  // sort each decoder's pairs by e (rank among the decoder's pairs, ties by
+  // position), and check sum b <= INT32_MAX (K at step 0)
+  for (int k = warp; k < D; k += kSt / 32) {
+    const int lo = s_base[k] - k * nb, n = s_n[k], base = s_base[k];
+    long long sb = 0;
+    for (int i = lane; i < n; i += 32) {
+      const int ei = uE[lo + i];
+      int r = 0;
+      for (int j2 = 0; j2 < n; ++j2) {
+        const int ej = uE[lo + j2];
+        r += ej < ei || (ej == ei && j2 < i);
+      }
+      E[base + r] = ei;
+      Bv[base + r] = uB[lo + i];
+      sb += uB[lo + i];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sb += __shfl_xor_sync(0xffffffffu, sb, off);
+    if (lane == 0 && sb > 0x7fffffffLL) s_bad = 1;
+  }
+  __syncthreads();
+  if (tid == 0 && s_bad) flag_error(status, MAPS_E_RANGE);
+
+  // The walk: one warp, no block barrier.  Lane l scores decoders l, l + 32,
+  // ... by walking each list from its last pair (suffix sums as it goes); a
+  // packed key picks (feasible first, then Q or the largest headroom, then
+  // the lowest index); the warp inserts the footprint.
+  if (warp == 0) {
+    for (int j = 0; j < nb; ++j) {
+      const int32_t p = s_cp[j], U = s_cu[j];
+      if ((p | U) < 0) {
+        if (lane == 0) {
+          flag_error(status, MAPS_E_RANGE);
+          choice[j] = -1;
+          if (headroom) headroom[j] = 0;
+        }
+        continue;
+      }
+      const int u = U < 1 ? 1 : (U > H ? H : U);
+      unsigned long long key = ~0ull;  // inf << 63 | v << 10 | k, the smallest wins
+      for (int k = lane; k < D; k += 32) {
+        const int n = s_n[k], base = s_base[k];
+        long long sfx = 0, best = LLONG_MIN, sgt = 0;
+        int cgt = 0;
+        for (int i = n - 1; i >= 0; --i) {
+          const int e = E[base + i];
+          const long long b = Bv[base + i];
+          sfx += b;
+          if (e <= u)
+            best = max(best, sfx + static_cast<long long>(e - 1) * (n - i + 1));
+          else
+            sgt += b, ++cgt;
+        }
+        const long long M = max(best, sgt + static_cast<long long>(u - 1) * (cgt + 1));
+        s_M[k] = M;
+        const long long h = static_cast<long long>(s_cap[k]) - (static_cast<long long>(p) + 1 + M);
+        const unsigned long long kk =
+            h >= 0 ? (static_cast<unsigned long long>(s_q[k]) << 10) | static_cast<unsigned>(k)
+                   : (1ull << 63) | (static_cast<unsigned long long>(-h) << 10) | static_cast<unsigned>(k);
+        key = kk < key ? kk : key;
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const unsigned long long o = __shfl_xor_sync(0xffffffffu, key, off);
+        key = o < key ? o : key;
+      }
+      const int bk = static_cast<int>(key & 1023u);
+      __syncwarp();  // s_M of every decoder written
+      const long long Mb = s_M[bk];
+      const int n = s_n[bk], base = s_base[bk];
+      if (lane == 0) {
+        choice[j] = bk;
+        if (headroom) headroom[j] = static_cast<long long>(s_cap[bk]) - (static_cast<long long>(p) + 1 + Mb);
+        if (s_q[bk] == 0x7fffffff)
+          flag_error(status, MAPS_E_RANGE);
+        else
+          s_q[bk] += 1;
+        // every new cell K + p + t + 1 (t < u) is at most M + p + 1
+        if (static_cast<long long>(p) + 1 + Mb > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
+      }
+      // reserve: (u, p + 1) joins decoder bk's pairs after those with e <= u
+      int pos = 0;
+      for (int i = lane; i < n; i += 32) pos += E[base + i] <= u;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) pos += __shfl_xor_sync(0xffffffffu, pos, off);
+      for (int r = (n - 1) >> 5; r >= 0; --r) {  // shift [pos, n) up by one, last round first
+        const int i = r * 32 + lane;
+        const bool mv = i < n && i >= pos;
+        const int e = mv ? E[base + i] : 0, b = mv ? Bv[base + i] : 0;
+        __syncwarp();
+        if (mv) {
+          E[base + i + 1] = e;
+          Bv[base + i + 1] = b;
+        }
+        __syncwarp();
+      }
+      if (lane == 0) {
+        E[base + pos] = u;
+        Bv[base + pos] = p + 1;
+        s_n[bk] = n + 1;
+      }
+      __syncwarp();
+    }
+  }
+  __syncthreads();
+  for (int k = tid; k < D; k += kSt) Q[k] = s_q[k];
 }
 
 // 6. The batch joins the waiting queues of its decoders.
@@ -497,11 +678,22 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
                                         w.Q);  // 4.
     MAPS_TRY(launch_ok());
     if (!rr) {  // 5.
-      MAPS_TRY(maps_project_occupancy(D, c.H, w.res_off, nact, w.rp, w.rg, w.rU, w.K, nullptr, ws,
-                                      w.sub_bytes, stream));
-      MAPS_TRY(maps_dispatch(MAPS_MODE_SEQUENTIAL, D, c.H, 1, w.K, nullptr, w.capv, w.Q, nullptr, 0,
-                             nullptr, nullptr, nullptr, nb, prompt + lo, w.Uq + nact,
-                             choice_out + lo, w.headroom, ws, w.sub_bytes, stream));
+      const size_t dsm = stream_dispatch_smem(D, nact, nb);
+      if (dsm + 2048 <= static_cast<size_t>(max_smem_optin())) {
+        // the decoders' pairs fit in shared memory: no dense projection
+        MAPS_TRY(cuda_ok(cudaFuncSetAttribute(stream_dispatch_kernel,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              static_cast<int>(dsm))));
+        launch_pdl(stream_dispatch_kernel, 1, kSt, dsm, s, D, c.H, nb, w.res_off, w.rp, w.rg, w.rU,
+                   w.capv, w.Q, prompt + lo, w.Uq + nact, choice_out + lo, w.headroom, status);
+        MAPS_TRY(launch_ok());
+      } else {
+        MAPS_TRY(maps_project_occupancy(D, c.H, w.res_off, nact, w.rp, w.rg, w.rU, w.K, nullptr, ws,
+                                        w.sub_bytes, stream));
+        MAPS_TRY(maps_dispatch(MAPS_MODE_SEQUENTIAL, D, c.H, 1, w.K, nullptr, w.capv, w.Q, nullptr, 0,
+                               nullptr, nullptr, nullptr, nb, prompt + lo, w.Uq + nact,
+                               choice_out + lo, w.headroom, ws, w.sub_bytes, stream));
+      }
     }
     launch_pdl(stream_enqueue_kernel, grid_for(nb), 256, 0, s, lo, nb, nact, hi, D, arrival_ms,
                                                        choice_out, w.Uq, w.st, w.dec, w.disp, w.g,
