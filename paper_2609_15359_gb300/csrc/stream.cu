@@ -245,18 +245,65 @@ stream_csr_kernel(int nact, int D, int rr, const int32_t *q_dev, int32_t *q_out_
 //   M_k(u) = max( max_{e_i <= u} S_i + (e_i - 1)(C_i + 1),
 //                 S' + (u - 1)(C' + 1) ),  S' / C' over the pairs with e > u.
 // (A pair tied on e with one before it gives a value no larger than the
-// first's, so ties need no merging.)  One warp walks the batch: a lane scores
-// a decoder, the warp picks (feasible with the smallest Q, else the largest
-// headroom, ties to the lowest index) and reserves the candidate's footprint
-// by inserting (u, p + 1) into the chosen decoder's list.  The same decisions and range errors as
+// first's, so ties need no merging.)  Beside the sorted pairs each decoder
+// keeps the suffix sums of b and the prefix maxima of the first term, so a
+// score is a binary search for the pairs with e <= u and two reads.  One warp
+// walks the batch: a lane scores a decoder, the warp picks (feasible with the
+// smallest Q, else the largest headroom, ties to the lowest index), inserts
+// (u, p + 1) into the chosen decoder's list and rebuilds its tables.  The same decisions and range errors as
 // the dense projection followed by maps_dispatch SEQUENTIAL.
 // Shared memory: the pool of pairs (the residents of decoder k plus room for
 // nb reservations at base_k = res_off[k] + k nb), the unsorted pairs, and the
 // per-decoder tables.
 size_t stream_dispatch_smem(int D, int nact, int nb) {
   const size_t pool = static_cast<size_t>(nact) + static_cast<size_t>(D) * nb;
-  return 8 * (pool + static_cast<size_t>(nact)) + 24 * static_cast<size_t>(D) +
+  return 16 * pool + 8 * static_cast<size_t>(nact) + 28 * static_cast<size_t>(D) +
          8 * static_cast<size_t>(nb) + 64;
+}
+
+// A decoder's tables from its sorted pairs (one warp): SS[i] = sum of b over
+// pairs i.. n-1, and PM[i] = the largest V over pairs 0..i, with
+// V_i = SS[i] + (E[i] - 1)(n - i + 1) (K + t at t = E[i] - 1).  Returns
+// whether some K(t) exceeds INT32_MAX (the projection's range error); below
+// that every SS, V and PM fits 32 bits.
+__device__ bool rebuild_tables(const int32_t *E, const int32_t *Bv, uint32_t *SS, uint32_t *PM,
+                               int n) {
+  const int lane = threadIdx.x & 31;
+  unsigned long long carry = 0;
+  bool over = false;
+  for (int r = (n - 1) >> 5; r >= 0; --r) {  // suffix sums, last round first
+    const int i = r * 32 + lane;
+    const unsigned long long b = i < n ? static_cast<unsigned long long>(Bv[i]) : 0ull;
+    unsigned long long suf = b;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const unsigned long long y = __shfl_down_sync(0xffffffffu, suf, off);
+      if (lane + off < 32) suf += y;
+    }
+    if (i < n) {
+      const unsigned long long ss = suf + carry;
+      // K at the segment's last step: the pairs i.. n-1 are live there
+      over |= ss + static_cast<unsigned long long>(E[i] - 1) * (n - i) > 0x7fffffffull;
+      SS[i] = static_cast<uint32_t>(ss);
+    }
+    carry += __shfl_sync(0xffffffffu, suf, 0);
+  }
+  __syncwarp();
+  uint32_t run = 0;
+  for (int r = 0; r <= (n - 1) >> 5; ++r) {  // prefix maxima, first round first
+    const int i = r * 32 + lane;
+    uint32_t incl = i < n ? SS[i] + static_cast<uint32_t>(E[i] - 1) * static_cast<uint32_t>(n - i + 1) : 0u;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl = max(incl, y);
+    }
+    incl = max(incl, run);
+    if (i < n) PM[i] = incl;
+    run = __shfl_sync(0xffffffffu, incl, 31);
+  }
+  __syncwarp();
+  return __any_sync(0xffffffffu, over);
 }
 
 __global__ void __launch_bounds__(kSt, 1)
@@ -272,10 +319,13 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
   long long *s_M = reinterpret_cast<long long *>(sdm);     // [D]
   int32_t *E = reinterpret_cast<int32_t *>(s_M + D);       // [pool] sorted end steps
   int32_t *Bv = E + pool;                                  // [pool] their b
-  int32_t *uE = Bv + pool;                                 // [nact] unsorted
+  uint32_t *SS = reinterpret_cast<uint32_t *>(Bv + pool);  // [pool] suffix sums of b
+  uint32_t *PM = SS + pool;                                // [pool] prefix maxima of V
+  int32_t *uE = reinterpret_cast<int32_t *>(PM + pool);    // [nact] unsorted
   int32_t *uB = uE + nact;
   int32_t *s_base = uB + nact, *s_n = s_base + D, *s_q = s_n + D, *s_cap = s_q + D;
-  int32_t *s_cp = s_cap + D, *s_cu = s_cp + nb;           // [nb] the batch
+  int32_t *s_c = s_cap + D;                               // [D] pairs with e <= u
+  int32_t *s_cp = s_c + D, *s_cu = s_cp + nb;              // [nb] the batch
   __shared__ int s_bad;
   if (tid == 0) s_bad = 0;
   __syncthreads();
@@ -326,6 +376,8 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) sb += __shfl_xor_sync(0xffffffffu, sb, off);
     if (lane == 0 && sb > 0x7fffffffLL) s_bad = 1;
+    __syncwarp();  // the sorted pairs are written
+    if (rebuild_tables(E + base, Bv + base, SS + base, PM + base, n) && lane == 0) s_bad = 1;
   }
   __syncthreads();
   if (tid == 0 && s_bad) flag_error(status, MAPS_E_RANGE);
@@ -349,19 +401,21 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
       unsigned long long key = ~0ull;  // inf << 63 | v << 10 | k, the smallest wins
       for (int k = lane; k < D; k += 32) {
         const int n = s_n[k], base = s_base[k];
-        long long sfx = 0, best = LLONG_MIN, sgt = 0;
-        int cgt = 0;
-        for (int i = n - 1; i >= 0; --i) {
-          const int e = E[base + i];
-          const long long b = Bv[base + i];
-          sfx += b;
-          if (e <= u)
-            best = max(best, sfx + static_cast<long long>(e - 1) * (n - i + 1));
+        int lo = 0, hi = n;  // c = the pairs with e <= u
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (E[base + mid] <= u)
+            lo = mid + 1;
           else
-            sgt += b, ++cgt;
+            hi = mid;
         }
-        const long long M = max(best, sgt + static_cast<long long>(u - 1) * (cgt + 1));
+        const int c = lo;
+        const long long full = c > 0 ? static_cast<long long>(PM[base + c - 1]) : LLONG_MIN;
+        const long long part = static_cast<long long>(c < n ? SS[base + c] : 0u) +
+                               static_cast<long long>(u - 1) * (n - c + 1);
+        const long long M = max(full, part);
         s_M[k] = M;
+        s_c[k] = c;
         const long long h = static_cast<long long>(s_cap[k]) - (static_cast<long long>(p) + 1 + M);
         const unsigned long long kk =
             h >= 0 ? (static_cast<unsigned long long>(s_q[k]) << 10) | static_cast<unsigned>(k)
@@ -388,10 +442,7 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
         if (static_cast<long long>(p) + 1 + Mb > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
       }
       // reserve: (u, p + 1) joins decoder bk's pairs after those with e <= u
-      int pos = 0;
-      for (int i = lane; i < n; i += 32) pos += E[base + i] <= u;
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) pos += __shfl_xor_sync(0xffffffffu, pos, off);
+      const int pos = s_c[bk];
       for (int r = (n - 1) >> 5; r >= 0; --r) {  // shift [pos, n) up by one, last round first
         const int i = r * 32 + lane;
         const bool mv = i < n && i >= pos;
@@ -409,6 +460,7 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
         s_n[bk] = n + 1;
       }
       __syncwarp();
+      rebuild_tables(E + base, Bv + base, SS + base, PM + base, n + 1);
     }
   }
   __syncthreads();
