@@ -250,8 +250,9 @@ stream_csr_kernel(int nact, int D, int rr, const int32_t *q_dev, int32_t *q_out_
 // score is a binary search for the pairs with e <= u and two reads.  One warp
 // walks the batch: a lane scores a decoder, the warp picks (feasible with the
 // smallest Q, else the largest headroom, ties to the lowest index), inserts
-// (u, p + 1) into the chosen decoder's list and rebuilds its tables.  The same decisions and range errors as
-// the dense projection followed by maps_dispatch SEQUENTIAL.
+// (u, p + 1) into the chosen decoder's list and rebuilds its tables.  The
+// decisions and range errors are those of the dense projection followed by
+// maps_dispatch SEQUENTIAL.
 // Shared memory: the pool of pairs (the residents of decoder k plus room for
 // nb reservations at base_k = res_off[k] + k nb), the unsorted pairs, and the
 // per-decoder tables.
@@ -383,9 +384,10 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
   if (tid == 0 && s_bad) flag_error(status, MAPS_E_RANGE);
 
   // The walk: one warp, no block barrier.  Lane l scores decoders l, l + 32,
-  // ... by walking each list from its last pair (suffix sums as it goes); a
-  // packed key picks (feasible first, then Q or the largest headroom, then
-  // the lowest index); the warp inserts the footprint.
+  // ...: a binary search over the decoder's sorted ends gives c (the pairs with
+  // e <= u), then M = max(PM[c - 1], SS[c] + (u - 1)(n - c + 1)); a packed key
+  // picks (feasible first, then Q or the largest headroom, then the lowest
+  // index); the warp inserts the footprint and rebuilds that decoder's tables.
   if (warp == 0) {
     for (int j = 0; j < nb; ++j) {
       const int32_t p = s_cp[j], U = s_cu[j];
