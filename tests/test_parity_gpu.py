@@ -469,6 +469,29 @@ def test_order_random(M, ws, oracle, N, D, sorted_arrival):
     assert np.array_equal(seg, so)
 
 
+@pytest.mark.parametrize("N,D,blo,bhi,skew", [
+    # one queue far past a block (16 chunks), bounds of 17 bits
+    (70000, 256, 0, 70000, 0.95),
+    # several long queues with ragged last chunks, 31-bit bounds
+    (60001, 8, 0, 2**31 - 1, 0.0),
+    # bounds in [2^20, 2^20 + 200): keys share their high bits
+    (30000, 3, 2**20, 2**20 + 200, 0.5),
+    # more decoders than the stable scatter takes, one long queue
+    (40000, 1100, 0, 2**31 - 1, 0.9)])
+def test_order_long_queues(M, ws, oracle, N, D, blo, bhi, skew):
+    rng = np.random.default_rng(N + D)
+    dec = rng.integers(0, D, N).astype(np.int32)
+    dec[rng.random(N) < skew] = D // 2
+    U = rng.integers(blo, bhi, N, dtype=np.int64).astype(np.int32)
+    wait = rng.integers(-10, 3000, N).astype(np.int32)
+    arr = np.sort(rng.integers(0, N, N)).astype(np.int32)
+    sto, po, so = oracle.order_local(D, dec, U, wait, arr, 1000)
+    st, perm, seg = gpu_order(M, ws, D, dec, U, wait, arr, 1000)
+    assert st == sto == 0
+    assert np.array_equal(perm, po)
+    assert np.array_equal(seg, so)
+
+
 def test_order_degenerate_keys(M, ws, oracle):
     # every key identical: all digit passes trivial -> identity order
     N = 9000
@@ -479,15 +502,17 @@ def test_order_degenerate_keys(M, ws, oracle):
     assert st == M.MAPS_E_RANGE
 
 
-@pytest.mark.parametrize("name", ["d64", "large"])
-def test_order_workload_pipeline(M, ws, oracle, name):
-    """The benchmark's order step: residents plus dispatched candidates."""
+@pytest.mark.parametrize("name,one_queue", [("d64", False), ("large", False), ("large", True)])
+def test_order_workload_pipeline(M, ws, oracle, name, one_queue):
+    """The benchmark's order step: residents plus dispatched candidates (spread over the
+    decoders, or all on one decoder as when every candidate falls back to the same one)."""
     w = W.make(name)
     R, J, D = w["R"], w["J"], w["D"]
     rng = np.random.default_rng(1)
     q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
     U = oracle.bound(np.concatenate([w["res_pred"], w["cand_pred"]]), q)[1]
-    dec = np.concatenate([w["res_dec"], rng.integers(0, D, J).astype(np.int32)])
+    cand_dec = np.full(J, 37, np.int32) if one_queue else rng.integers(0, D, J).astype(np.int32)
+    dec = np.concatenate([w["res_dec"], cand_dec])
     wait = np.concatenate([w["res_wait"], np.zeros(J, np.int32)])
     arr = np.arange(R + J, dtype=np.int32)
     sto, po, so = oracle.order_local(D, dec, U, wait, arr, w["max_wait"])
