@@ -16,7 +16,8 @@ host enqueues the step, so CUDA events on the launching stream bracket the
 device time of the step alone.  The end-to-end figure repeats the step
 through the same C-ABI calls with pinned host buffers, host-to-device copies
 of every input and device-to-host copies of every output inside the timed
-region.
+region; steps are pipelined over two buffer sets, each stage replayed from a
+CUDA graph.
 
 --impl reference runs the CPU oracle on the host cores over a bounded
 sample of the same workload and prints the same metric.
@@ -177,6 +178,44 @@ class ClockSampler:
 # the GPU step
 # ---------------------------------------------------------------------------
 
+def input_layout(w: dict):
+    """Byte offsets of a step's inputs in one staging arena (256-byte aligned),
+    the same on the host and the device, so that a step's inputs arrive in one
+    host-to-device copy.  ``dec_all`` (resident decoders, then the dispatch's
+    choices) is last and only its first R entries are inputs: the copy ends
+    there and never touches the choices.  Returns (fields, total, copy_bytes)."""
+    R, J, D, n = w["R"], w["J"], w["D"], w["n_cal"]
+    spec = [("cal_true", n, np.int32), ("cal_pred", n, np.int32), ("pred_all", R + J, np.int32),
+            ("res_off", D + 1, np.int64), ("res_prompt", R, np.int32), ("res_gen", R, np.int32),
+            ("cap", D, np.int32), ("Q0", D, np.int32), ("cand_prompt", J, np.int32),
+            ("wait_all", R + J, np.int32), ("arrival", R + J, np.int32), ("dec_all", R + J, np.int32)]
+    fields, off = {}, 0
+    for name, count, dt in spec:
+        fields[name] = (off, count, dt)
+        off += (count * np.dtype(dt).itemsize + 255) // 256 * 256
+    return fields, off, fields["dec_all"][0] + 4 * R
+
+
+def input_arrays(w: dict) -> dict:
+    """The values of every input field (``dec_all`` holds zeros for the choices)."""
+    R, J = w["R"], w["J"]
+    return {
+        "cal_true": w["cal_true"], "cal_pred": w["cal_pred"],
+        "pred_all": np.concatenate([w["res_pred"], w["cand_pred"]]),
+        "res_off": w["res_off"], "res_prompt": w["res_prompt"], "res_gen": w["res_gen"],
+        "cap": w["cap"], "Q0": w["Q"], "cand_prompt": w["cand_prompt"],
+        "wait_all": np.concatenate([w["res_wait"], np.zeros(J, np.int32)]),
+        "arrival": np.arange(R + J, dtype=np.int32),
+        "dec_all": np.concatenate([w["res_dec"], np.zeros(J, np.int32)]),
+    }
+
+
+def arena_views(arena, fields: dict) -> dict:
+    import torch
+    tdt = {np.int32: torch.int32, np.int64: torch.int64}
+    return {k: arena[o:o + c * np.dtype(dt).itemsize].view(tdt[dt]) for k, (o, c, dt) in fields.items()}
+
+
 class Step:
     """Device buffers and the four C-ABI calls of one hot-path pass."""
 
@@ -188,22 +227,22 @@ class Step:
         self.M, self.torch, self.w = M, torch, w
         self.D, self.H, self.R, self.J = w["D"], w["H"], w["R"], w["J"]
         self.alpha = w["alphas_ppm"][0]
-        t = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(device)  # noqa: E731
         R, J = self.R, self.J
-        # inputs (resident in HBM)
-        self.cal_true, self.cal_pred = t(w["cal_true"]), t(w["cal_pred"])
-        self.pred_all = t(np.concatenate([w["res_pred"], w["cand_pred"]]))
-        self.res_off, self.res_prompt, self.res_gen = t(w["res_off"]), t(w["res_prompt"]), t(w["res_gen"])
-        self.cap, self.Q0 = t(w["cap"]), t(w["Q"])
-        self.cand_prompt = t(w["cand_prompt"])
-        self.wait_all = t(np.concatenate([w["res_wait"], np.zeros(J, np.int32)]))
-        self.arrival = t(np.arange(R + J, dtype=np.int32))
+        # inputs (resident in HBM), views of one staging arena
+        self.fields, total, self.copy_bytes = input_layout(w)
+        self.arena = torch.empty(total, dtype=torch.uint8, device=device)
+        v = arena_views(self.arena, self.fields)
+        for k, a in input_arrays(w).items():
+            v[k].copy_(torch.from_numpy(np.ascontiguousarray(a, dtype=self.fields[k][2])))
+        self.cal_true, self.cal_pred, self.pred_all = v["cal_true"], v["cal_pred"], v["pred_all"]
+        self.res_off, self.res_prompt, self.res_gen = v["res_off"], v["res_prompt"], v["res_gen"]
+        self.cap, self.Q0, self.cand_prompt = v["cap"], v["Q0"], v["cand_prompt"]
+        self.wait_all, self.arrival, self.dec_all = v["wait_all"], v["arrival"], v["dec_all"]
         # outputs / intermediates
         self.U_all = torch.empty(R + J, dtype=torch.int32, device=device)
         self.q = torch.empty(1, dtype=torch.int32, device=device)
         self.K = torch.empty((self.D, self.H), dtype=torch.int32, device=device)
         self.kmax = torch.empty(M.kmax_shape(self.D, self.H), dtype=torch.int32, device=device)
-        self.dec_all = t(np.concatenate([w["res_dec"], np.zeros(J, np.int32)]))
         self.choice = self.dec_all[R:]
         self.headroom = torch.empty(J, dtype=torch.int64, device=device)
         self.perm = torch.empty(R + J, dtype=torch.int32, device=device)
@@ -249,20 +288,15 @@ class Step:
 
 
 def host_inputs(w):
-    """Pinned host copies of every per-step input and output of the e2e path."""
+    """Pinned host staging arena of a step's inputs (the device arena's layout)
+    and pinned host buffers for its results."""
     import torch
     R, J = w["R"], w["J"]
-    pin = lambda x: torch.from_numpy(np.ascontiguousarray(x)).pin_memory()  # noqa: E731
-    ins = {
-        "cal_true": pin(w["cal_true"]), "cal_pred": pin(w["cal_pred"]),
-        "pred_all": pin(np.concatenate([w["res_pred"], w["cand_pred"]])),
-        "res_off": pin(w["res_off"]), "res_prompt": pin(w["res_prompt"]),
-        "res_gen": pin(w["res_gen"]), "cap": pin(w["cap"]), "Q0": pin(w["Q"]),
-        "cand_prompt": pin(w["cand_prompt"]),
-        "wait_all": pin(np.concatenate([w["res_wait"], np.zeros(J, np.int32)])),
-        "arrival": pin(np.arange(R + J, dtype=np.int32)),
-        "res_dec": pin(w["res_dec"]),
-    }
+    fields, total, _ = input_layout(w)
+    arena = torch.empty(total, dtype=torch.uint8).pin_memory()
+    v = arena_views(arena, fields)
+    for k, a in input_arrays(w).items():
+        v[k].copy_(torch.from_numpy(np.ascontiguousarray(a, dtype=fields[k][2])))
     outs = {
         "choice": torch.empty(J, dtype=torch.int32).pin_memory(),
         "headroom": torch.empty(J, dtype=torch.int64).pin_memory(),
@@ -270,27 +304,13 @@ def host_inputs(w):
         "seg": torch.empty(w["D"] + 1, dtype=torch.int64).pin_memory(),
         "q": torch.empty(1, dtype=torch.int32).pin_memory(),
     }
-    return ins, outs
+    return arena, outs
 
 
-def copy_inputs(s: Step, ins: dict, part: int = -1):
-    """The step's input copies, in three parts of about 11 MB (all with -1)."""
-    R = s.R
-    if part in (-1, 0):
-        s.cal_true.copy_(ins["cal_true"], non_blocking=True)
-        s.cal_pred.copy_(ins["cal_pred"], non_blocking=True)
-        s.cap.copy_(ins["cap"], non_blocking=True)
-        s.Q0.copy_(ins["Q0"], non_blocking=True)
-    if part in (-1, 1):
-        s.pred_all.copy_(ins["pred_all"], non_blocking=True)
-        s.res_off.copy_(ins["res_off"], non_blocking=True)
-        s.res_prompt.copy_(ins["res_prompt"], non_blocking=True)
-        s.res_gen.copy_(ins["res_gen"], non_blocking=True)
-        s.cand_prompt.copy_(ins["cand_prompt"], non_blocking=True)
-    if part in (-1, 2):
-        s.wait_all.copy_(ins["wait_all"], non_blocking=True)
-        s.arrival.copy_(ins["arrival"], non_blocking=True)
-        s.dec_all[:R].copy_(ins["res_dec"], non_blocking=True)
+def copy_inputs(s: Step, arena):
+    """The step's inputs: one copy of the staging arena up to the end of the
+    resident decoders."""
+    s.arena[:s.copy_bytes].copy_(arena[:s.copy_bytes], non_blocking=True)
 
 
 def copy_outputs(s: Step, outs: dict):
@@ -301,42 +321,70 @@ def copy_outputs(s: Step, outs: dict):
     outs["q"].copy_(s.q, non_blocking=True)
 
 
-def e2e_run(steps, ins: dict, outs: list, n: int):
+def e2e_stages(steps, ins: dict, outs: list):
+    """The three stages of an end-to-end step on buffer set b: the input copy
+    from the pinned staging arena (one copy: on this host-to-device link one
+    large copy runs near 208 GB/s where a dozen smaller ones reach about 160),
+    the four C-ABI calls, and the read-back of the results.  Each stage of each
+    set is captured once as a CUDA graph, so a step costs the host three graph
+    launches instead of thirteen kernel launches and six copies.
+    Returns (stages, how)."""
+    import torch
+    side = torch.cuda.Stream()
+    graphs = []
+    try:
+        for b, s in enumerate(steps):
+            gs = []
+            for fn in (lambda s=s: copy_inputs(s, ins), s.run,
+                       lambda s=s, b=b: copy_outputs(s, outs[b])):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=side, capture_error_mode="relaxed"):
+                    fn()
+                gs.append(g)
+            graphs.append(gs)
+        torch.cuda.synchronize()
+        return [tuple(g.replay for g in gs) for gs in graphs], "cuda graphs"
+    except RuntimeError as e:  # capture refused: run the stages directly
+        print(f"# e2e: CUDA graph capture failed ({e}); stages run directly", file=sys.stderr)
+        torch.cuda.synchronize()
+        return [(lambda s=s: copy_inputs(s, ins), s.run, lambda s=s, b=b: copy_outputs(s, outs[b]))
+                for b, s in enumerate(steps)], "direct launches"
+
+
+def e2e_run(stages, n: int):
     """n end-to-end steps through the public API, pipelined the way a server
     would run them: step i uses buffer set i % 2 (inputs, workspace, outputs);
     its inputs are copied from pinned host memory on a copy stream while step
-    i - 1 computes (more copy streams measured no faster: the host-to-device
-    link is the limit), and its results are read back to pinned host memory on
+    i - 1 computes, and its results are read back to pinned host memory on
     another stream once it finishes.  Every step copies all of its inputs and
     reads back all of its results."""
     import torch
     comp = torch.cuda.current_stream()
-    h2d = [torch.cuda.Stream()]
+    h2d = torch.cuda.Stream()
     d2h = torch.cuda.Stream()
     start = torch.cuda.Event()
-    ready = [[torch.cuda.Event()] for _ in range(2)]  # inputs of set b copied
+    ready = [torch.cuda.Event() for _ in range(2)]  # inputs of set b copied
     done = [torch.cuda.Event() for _ in range(2)]   # set b computed
     read = [torch.cuda.Event() for _ in range(2)]   # results of set b read back
     start.record(comp)
-    for hs in h2d:
-        hs.wait_event(start)
+    h2d.wait_event(start)
     d2h.wait_event(start)
     for i in range(n):
         b = i % 2
-        for part, hs in enumerate(h2d):
-            with torch.cuda.stream(hs):
-                if i >= 2:
-                    hs.wait_event(done[b])  # the set's previous step no longer reads its inputs
-                copy_inputs(steps[b], ins)
-                ready[b][part].record(hs)
-            comp.wait_event(ready[b][part])
+        copy_in, compute, copy_out = stages[b]
+        with torch.cuda.stream(h2d):
+            if i >= 2:
+                h2d.wait_event(done[b])  # the set's previous step no longer reads its inputs
+            copy_in()
+            ready[b].record(h2d)
+        comp.wait_event(ready[b])
         if i >= 2:
             comp.wait_event(read[b])  # the set's previous results have been read back
-        steps[b].run()
+        compute()
         done[b].record(comp)
         with torch.cuda.stream(d2h):
             d2h.wait_event(done[b])
-            copy_outputs(steps[b], outs[b])
+            copy_out()
             read[b].record(d2h)
     for b in range(2):
         comp.wait_event(read[b])
@@ -388,21 +436,34 @@ def bench_gpu(args, world, rank, local, dist):
     # end to end through the public API with host buffers
     ins, outs = host_inputs(w)
     outs2 = host_inputs(w)[1]
-    h2d = sum(v.numel() * v.element_size() for v in ins.values())
+    h2d = step.copy_bytes
     d2h = sum(v.numel() * v.element_size() for v in outs.values())
     steps = [step, Step(w, device)]
-    e2e_run(steps, ins, [outs, outs2], 4)
+    stages, how = e2e_stages(steps, ins, [outs, outs2])
+    e2e_run(stages, 4)
     torch.cuda.synchronize()
     Ke = max(5, min(K, 50))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
-    e2e_run(steps, ins, [outs, outs2], Ke)
+    e2e_run(stages, Ke)
     e1.record()
     torch.cuda.synchronize()
     for st_ in steps:
         st_.check()
     e2e_s = e0.elapsed_time(e1) / 1e3
     e2e_max, e2e_units = aggregate(e2e_s, float(Ke * step.J), dist)
+    # each stage alone, back to back on one stream (what the pipeline overlaps)
+    stage_us = {}
+    for name, k in (("h2d", 0), ("compute", 1), ("d2h", 2)):
+        fn = stages[0][k]
+        fn()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record()
+        for _ in range(10):
+            fn()
+        s1.record()
+        torch.cuda.synchronize()
+        stage_us[name] = s0.elapsed_time(s1) / 10 * 1e3
 
     peaks = measured_peaks()
     D, H, R, J = step.D, step.H, step.R, step.J
@@ -453,7 +514,9 @@ def bench_gpu(args, world, rank, local, dist):
         "e2e": {"value": e2e_units / e2e_max, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
                 "pipeline": "two buffer sets; step i+1's inputs copied while step i computes, "
-                            "results read back on another stream"},
+                            "results read back on another stream; each stage launched as "
+                            f"{how}",
+                "stage_us_alone": stage_us},
         "gpu_launches": step.kernels_per_step * K,
         "clocks": clocks,
     }

@@ -522,6 +522,79 @@ def test_order_workload_pipeline(M, ws, oracle, name, one_queue):
 
 
 # ---------------------------------------------------------------------------
+# CUDA graph capture of the whole pass
+# ---------------------------------------------------------------------------
+
+def test_graph_capture_replay(M, oracle):
+    """The four calls (calibrate + bound, occupancy, SNAPSHOT dispatch, local
+    order) captured once in a CUDA graph: every replay reads the inputs as they
+    are then and matches the oracle, including after the inputs change."""
+    w0, w1 = W.make("tiny", feasible=True), W.make("tiny", seed=11)
+    D, H, R, J = w0["D"], w0["H"], w0["R"], w0["J"]
+    assert (D, H, R, J) == (w1["D"], w1["H"], w1["R"], w1["J"])
+    a = w0["alphas_ppm"][0]
+    n = len(w0["cal_true"])
+    z = lambda k, dt=torch.int32: torch.zeros(k, dtype=dt, device="cuda")  # noqa: E731
+    x = dict(cal_true=z(n), cal_pred=z(n), pred=z(R + J), off=z(D + 1, torch.int64), prompt=z(R),
+             gen=z(R), cap=z(D), Q=z(D), cprompt=z(J), dec=z(R + J), wait=z(R + J),
+             arr=torch.arange(R + J, dtype=torch.int32, device="cuda"))
+    U, q = z(R + J), z(1)
+    K = z(D * H).view(D, H)
+    km = torch.zeros(M.kmax_shape(D, H), dtype=torch.int32, device="cuda")
+    hr, perm, seg = z(J, torch.int64), z(R + J), z(D + 1, torch.int64)
+    need = max(M.lib.maps_calibrate_workspace_size(n, R + J),
+               M.lib.maps_project_occupancy_workspace_size(D, H, R),
+               M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, D, H, J),
+               M.lib.maps_order_local_workspace_size(R + J, D))
+    gws = M.Workspace(need, torch.device("cuda"))
+
+    def load(w):
+        for k, v in dict(cal_true=w["cal_true"], cal_pred=w["cal_pred"],
+                         pred=np.concatenate([w["res_pred"], w["cand_pred"]]), off=w["res_off"],
+                         prompt=w["res_prompt"], gen=w["res_gen"], cap=w["cap"], Q=w["Q"],
+                         cprompt=w["cand_prompt"], wait=np.concatenate([w["res_wait"], np.zeros(J)]),
+                         dec=np.concatenate([w["res_dec"], np.zeros(J)])).items():
+            x[k].copy_(torch.from_numpy(np.ascontiguousarray(v).astype(x[k].cpu().numpy().dtype)))
+
+    def run():
+        assert M.maps_calibrate(x["cal_true"], x["cal_pred"], a, x["pred"], U, q, ws=gws)[0] == 0
+        assert M.maps_project_occupancy(D, H, x["off"], x["prompt"], x["gen"], U[:R], K, km,
+                                        ws=gws) == 0
+        assert M.maps_dispatch(M.MODE_SNAPSHOT, D, H, 1, K, x["cap"], x["Q"], x["cprompt"],
+                               U[R:], x["dec"][R:], hr, kmax=km, ws=gws) == 0
+        assert M.maps_order_local(D, x["dec"], U, x["wait"], x["arr"], w0["max_wait"], perm, seg,
+                                  ws=gws) == 0
+
+    load(w0)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        run()  # warm-up outside the capture
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side, capture_error_mode="relaxed"):
+        run()
+    for w in (w0, w1, w0):
+        load(w)
+        g.replay()
+        torch.cuda.synchronize()
+        assert M.maps_check(gws) == 0
+        sto, qo = oracle.calibrate(w["cal_true"], w["cal_pred"], a)
+        Uo = oracle.bound(np.concatenate([w["res_pred"], w["cand_pred"]]), qo)[1]
+        _, Ko = oracle.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], Uo[:R])
+        _, cho, hro, _, _ = oracle.dispatch(0, D, H, 1, Ko, w["cap"], w["Q"], w["cand_prompt"],
+                                            Uo[R:])
+        deco = np.concatenate([w["res_dec"], cho]).astype(np.int32)
+        _, po, so = oracle.order_local(D, deco, Uo, np.concatenate([w["res_wait"], np.zeros(J, np.int32)]),
+                                       np.arange(R + J, dtype=np.int32), w0["max_wait"])
+        assert int(host(q)[0]) == qo and np.array_equal(host(U), Uo)
+        assert np.array_equal(host(K), Ko)
+        assert np.array_equal(host(x["dec"])[R:], cho) and np.array_equal(host(hr), hro)
+        assert np.array_equal(host(perm), po) and np.array_equal(host(seg), so)
+
+
+# ---------------------------------------------------------------------------
 # determinism
 # ---------------------------------------------------------------------------
 
