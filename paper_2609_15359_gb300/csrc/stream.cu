@@ -258,7 +258,7 @@ stream_csr_kernel(int nact, int D, int rr, const int32_t *q_dev, int32_t *q_out_
 // per-decoder tables.
 size_t stream_dispatch_smem(int D, int nact, int nb) {
   const size_t pool = static_cast<size_t>(nact) + static_cast<size_t>(D) * nb;
-  return 16 * pool + 8 * static_cast<size_t>(nact) + 28 * static_cast<size_t>(D) +
+  return 16 * pool + 8 * static_cast<size_t>(nact) + 16 * static_cast<size_t>(D) +
          8 * static_cast<size_t>(nb) + 64;
 }
 
@@ -317,16 +317,14 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nact = static_cast<int>(res_off[D]);
   const int pool = nact + D * nb;
-  long long *s_M = reinterpret_cast<long long *>(sdm);     // [D]
-  int32_t *E = reinterpret_cast<int32_t *>(s_M + D);       // [pool] sorted end steps
+  int32_t *E = reinterpret_cast<int32_t *>(sdm);           // [pool] sorted end steps
   int32_t *Bv = E + pool;                                  // [pool] their b
   uint32_t *SS = reinterpret_cast<uint32_t *>(Bv + pool);  // [pool] suffix sums of b
   uint32_t *PM = SS + pool;                                // [pool] prefix maxima of V
   int32_t *uE = reinterpret_cast<int32_t *>(PM + pool);    // [nact] unsorted
   int32_t *uB = uE + nact;
   int32_t *s_base = uB + nact, *s_n = s_base + D, *s_q = s_n + D, *s_cap = s_q + D;
-  int32_t *s_c = s_cap + D;                               // [D] pairs with e <= u
-  int32_t *s_cp = s_c + D, *s_cu = s_cp + nb;              // [nb] the batch
+  int32_t *s_cp = s_cap + D, *s_cu = s_cp + nb;            // [nb] the batch
   __shared__ int s_bad;
   if (tid == 0) s_bad = 0;
   __syncthreads();
@@ -401,6 +399,8 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
       }
       const int u = U < 1 ? 1 : (U > H ? H : U);
       unsigned long long key = ~0ull;  // inf << 63 | v << 10 | k, the smallest wins
+      long long bM = 0;                // M and c of this lane's best decoder
+      int bc = 0;
       for (int k = lane; k < D; k += 32) {
         const int n = s_n[k], base = s_base[k];
         int lo = 0, hi = n;  // c = the pairs with e <= u
@@ -416,22 +416,38 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
         const long long part = static_cast<long long>(c < n ? SS[base + c] : 0u) +
                                static_cast<long long>(u - 1) * (n - c + 1);
         const long long M = max(full, part);
-        s_M[k] = M;
-        s_c[k] = c;
         const long long h = static_cast<long long>(s_cap[k]) - (static_cast<long long>(p) + 1 + M);
         const unsigned long long kk =
             h >= 0 ? (static_cast<unsigned long long>(s_q[k]) << 10) | static_cast<unsigned>(k)
                    : (1ull << 63) | (static_cast<unsigned long long>(-h) << 10) | static_cast<unsigned>(k);
-        key = kk < key ? kk : key;
+        if (kk < key) {
+          key = kk;
+          bM = M;
+          bc = c;
+        }
       }
+      // The warp's smallest key.  When every value fits 21 bits the key packs
+      // into 32 (inf << 31 | v << 10 | k, the same order) and one reduction
+      // finds it; otherwise a shuffle ladder over the 64-bit keys.
+      const unsigned long long kv = (key >> 10) & ((1ull << 53) - 1);
+      const bool none = key == ~0ull;  // a lane without decoders
+      int bk;
+      if (__all_sync(0xffffffffu, none || kv < (1ull << 21))) {
+        const uint32_t k32 = none ? 0xffffffffu
+                                  : (static_cast<uint32_t>(key >> 63) << 31) |
+                                        (static_cast<uint32_t>(kv) << 10) | static_cast<uint32_t>(key & 1023u);
+        bk = static_cast<int>(__reduce_min_sync(0xffffffffu, k32) & 1023u);
+      } else {
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const unsigned long long o = __shfl_xor_sync(0xffffffffu, key, off);
-        key = o < key ? o : key;
+        for (int off = 16; off > 0; off >>= 1) {
+          const unsigned long long o = __shfl_xor_sync(0xffffffffu, key, off);
+          key = o < key ? o : key;
+        }
+        bk = static_cast<int>(key & 1023u);
       }
-      const int bk = static_cast<int>(key & 1023u);
-      __syncwarp();  // s_M of every decoder written
-      const long long Mb = s_M[bk];
+      // the winner's lane (decoder bk is lane bk % 32's) hands over M and c
+      const long long Mb = __shfl_sync(0xffffffffu, bM, bk & 31);
+      const int pos = __shfl_sync(0xffffffffu, bc, bk & 31);
       const int n = s_n[bk], base = s_base[bk];
       if (lane == 0) {
         choice[j] = bk;
@@ -444,7 +460,38 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
         if (static_cast<long long>(p) + 1 + Mb > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
       }
       // reserve: (u, p + 1) joins decoder bk's pairs after those with e <= u
-      const int pos = s_c[bk];
+      const int m = n + 1;
+      if (m <= 32) {
+        // One round: lane i takes pair i of the new list.  The suffix sums
+        // follow from the old ones (b more before the new pair, the same
+        // after it), and the prefix maxima of V take one shuffle scan, in 32
+        // bits (the check above keeps every K + t of the new list within
+        // INT32_MAX).
+        const int src = lane <= pos ? lane : lane - 1;  // the old pair this lane keeps
+        const bool old_ok = src < n;
+        const int eo = old_ok ? E[base + src] : 0, bo = old_ok ? Bv[base + src] : 0;
+        const uint32_t so = old_ok ? SS[base + src] : 0u;
+        const uint32_t bnew = static_cast<uint32_t>(p) + 1u;
+        const int e2 = lane == pos ? u : eo;
+        const int b2 = lane == pos ? static_cast<int>(bnew) : bo;
+        const uint32_t suf = lane <= pos ? so + bnew : so;
+        uint32_t V = lane < m ? suf + static_cast<uint32_t>(e2 - 1) * static_cast<uint32_t>(m - lane + 1) : 0u;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, V, off);
+          if (lane >= off) V = max(V, y);
+        }
+        __syncwarp();  // every lane has read the old list
+        if (lane < m) {
+          E[base + lane] = e2;
+          Bv[base + lane] = b2;
+          SS[base + lane] = suf;
+          PM[base + lane] = V;
+        }
+        if (lane == 0) s_n[bk] = m;
+        __syncwarp();
+        continue;
+      }
       for (int r = (n - 1) >> 5; r >= 0; --r) {  // shift [pos, n) up by one, last round first
         const int i = r * 32 + lane;
         const bool mv = i < n && i >= pos;
