@@ -386,7 +386,138 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
   // e <= u), then M = max(PM[c - 1], SS[c] + (u - 1)(n - c + 1)); a packed key
   // picks (feasible first, then Q or the largest headroom, then the lowest
   // index); the warp inserts the footprint and rebuilds that decoder's tables.
-  if (warp == 0) {
+  if (warp == 0 && D <= 32) {
+    // One decoder per lane: its list length, base, Q and capacity stay in
+    // registers, the next candidate is read ahead, and c comes from an 8-ary
+    // search (eight independent probes per level: a list of up to 8 pairs
+    // takes one level, up to 64 two).
+    const int k = lane;
+    const bool has = k < D;
+    int n_r = has ? s_n[k] : 0, q_r = has ? s_q[k] : 0;
+    const int base_r = has ? s_base[k] : 0, cap_r = has ? s_cap[k] : 0;
+    int32_t p_nx = nb > 0 ? s_cp[0] : 0, U_nx = nb > 0 ? s_cu[0] : 0;
+    for (int j = 0; j < nb; ++j) {
+      const int32_t p = p_nx, U = U_nx;
+      if (j + 1 < nb) {
+        p_nx = s_cp[j + 1];
+        U_nx = s_cu[j + 1];
+      }
+      if ((p | U) < 0) {
+        if (lane == 0) {
+          flag_error(status, MAPS_E_RANGE);
+          choice[j] = -1;
+          if (headroom) headroom[j] = 0;
+        }
+        continue;
+      }
+      const int u = U < 1 ? 1 : (U > H ? H : U);
+      int lo = 0, hi = n_r;  // c = the pairs with e <= u lies in [lo, hi]
+      while (lo < hi) {
+        const int len = hi - lo;
+        int nlo = lo, nhi = hi;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {  // probes cover every position when len <= 8
+          const int pi = lo + (len * i) / 8;
+          if (E[base_r + pi] <= u)
+            nlo = max(nlo, pi + 1);
+          else
+            nhi = min(nhi, pi);
+        }
+        lo = nlo;
+        hi = nhi;
+      }
+      const int c = lo;
+      long long M = 0;
+      unsigned long long key = ~0ull;  // inf << 63 | v << 10 | k, the smallest wins
+      if (has) {
+        const long long full = c > 0 ? static_cast<long long>(PM[base_r + c - 1]) : LLONG_MIN;
+        const long long part = static_cast<long long>(c < n_r ? SS[base_r + c] : 0u) +
+                               static_cast<long long>(u - 1) * (n_r - c + 1);
+        M = max(full, part);
+        const long long h = static_cast<long long>(cap_r) - (static_cast<long long>(p) + 1 + M);
+        key = h >= 0 ? (static_cast<unsigned long long>(q_r) << 10) | static_cast<unsigned>(k)
+                     : (1ull << 63) | (static_cast<unsigned long long>(-h) << 10) | static_cast<unsigned>(k);
+      }
+      const unsigned long long kv = (key >> 10) & ((1ull << 53) - 1);
+      const bool none = key == ~0ull;
+      int bk;
+      if (__all_sync(0xffffffffu, none || kv < (1ull << 21))) {
+        const uint32_t k32 = none ? 0xffffffffu
+                                  : (static_cast<uint32_t>(key >> 63) << 31) |
+                                        (static_cast<uint32_t>(kv) << 10) | static_cast<uint32_t>(key & 1023u);
+        bk = static_cast<int>(__reduce_min_sync(0xffffffffu, k32) & 1023u);
+      } else {
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          const unsigned long long o = __shfl_xor_sync(0xffffffffu, key, off);
+          key = o < key ? o : key;
+        }
+        bk = static_cast<int>(key & 1023u);
+      }
+      const int pos = __shfl_sync(0xffffffffu, c, bk);
+      const int n = __shfl_sync(0xffffffffu, n_r, bk);
+      const int base = __shfl_sync(0xffffffffu, base_r, bk);
+      if (lane == bk) {  // the chosen decoder's lane books the decision
+        choice[j] = bk;
+        if (headroom) headroom[j] = static_cast<long long>(cap_r) - (static_cast<long long>(p) + 1 + M);
+        if (q_r == 0x7fffffff)
+          flag_error(status, MAPS_E_RANGE);
+        else
+          q_r += 1;
+        // every new cell K + p + t + 1 (t < u) is at most M + p + 1
+        if (static_cast<long long>(p) + 1 + M > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
+        n_r = n + 1;
+      }
+      const int m = n + 1;
+      if (m <= 32) {
+        // the insert and the table update in one round (as below)
+        const int src = lane <= pos ? lane : lane - 1;
+        const bool old_ok = src < n;
+        const int eo = old_ok ? E[base + src] : 0, bo = old_ok ? Bv[base + src] : 0;
+        const uint32_t so = old_ok ? SS[base + src] : 0u;
+        const uint32_t bnew = static_cast<uint32_t>(p) + 1u;
+        const int e2 = lane == pos ? u : eo;
+        const int b2 = lane == pos ? static_cast<int>(bnew) : bo;
+        const uint32_t suf = lane <= pos ? so + bnew : so;
+        uint32_t V = lane < m ? suf + static_cast<uint32_t>(e2 - 1) * static_cast<uint32_t>(m - lane + 1) : 0u;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, V, off);
+          if (lane >= off) V = max(V, y);
+        }
+        __syncwarp();  // every lane has read the old list
+        if (lane < m) {
+          E[base + lane] = e2;
+          Bv[base + lane] = b2;
+          SS[base + lane] = suf;
+          PM[base + lane] = V;
+        }
+        __syncwarp();
+      } else {
+        for (int r = (n - 1) >> 5; r >= 0; --r) {  // shift [pos, n) up by one, last round first
+          const int i = r * 32 + lane;
+          const bool mv = i < n && i >= pos;
+          const int e = mv ? E[base + i] : 0, b = mv ? Bv[base + i] : 0;
+          __syncwarp();
+          if (mv) {
+            E[base + i + 1] = e;
+            Bv[base + i + 1] = b;
+          }
+          __syncwarp();
+        }
+        if (lane == 0) {
+          E[base + pos] = u;
+          Bv[base + pos] = p + 1;
+        }
+        __syncwarp();
+        rebuild_tables(E + base, Bv + base, SS + base, PM + base, m);
+      }
+    }
+    if (has) {
+      s_n[k] = n_r;
+      s_q[k] = q_r;
+    }
+  } else if (warp == 0) {
     for (int j = 0; j < nb; ++j) {
       const int32_t p = s_cp[j], U = s_cu[j];
       if ((p | U) < 0) {

@@ -658,6 +658,9 @@ def test_stream_golden(M, ws, stream_golden):
     (20000, 4, 4096, 12000, 256, 500, 100000, 1000),      # queues back up and block
     (20000, 3, 2048, 9000, 100, 37, 300000, 50),          # promotions, small window
     (5000, 5, 1000, 20000, 33, 7, 500000, 0),             # horizon below many bounds
+    # capacity far below demand: waiting queues push M, and the deficits,
+    # past 2^21 (the dispatch's 64-bit key comparison)
+    (3000, 8, 16384, 3000, 256, 500, 100000, 1000),
     # 200 decoders x batches of 256: the end-step tables would need about 800 KB of
     # shared memory, so the loop dispatches through the dense projection instead
     (3000, 200, 2048, 60000, 256, 300, 100000, 1000),
