@@ -610,6 +610,179 @@ struct SegSmem {
   unsigned long long orv[kSegWarps], andv[kSegWarps];
 };
 
+// Stable LSD passes over the keys sm.key[cur][0, n) on the 9-bit digits of
+// bits [lo_bit, nbits), skipping digits that are the same in every key (diff
+// holds the bits that differ between the keys); returns the buffer holding
+// the sorted keys.  All threads of the block take part.
+__device__ int seg_lsd(SegSmem &sm, int n, unsigned long long diff, int lo_bit, int nbits, int cur) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int shift = lo_bit; shift < nbits; shift += kSegBits) {
+    if (((diff >> shift) & (kSegBins - 1)) == 0) continue;  // same digit everywhere: order unchanged
+    for (int i = tid; i < kSegWarps * kSegBins / 2; i += kSegThreads) (&sm.hw[0][0])[i] = 0;
+    __syncthreads();
+    // rank within the warp, stable in item order (warp-major, then item, then
+    // lane): every match first, then one shared atomic per group leader,
+    // issued in item order, whose old value gives the group's base
+    uint32_t dr[kSegIPT];    // digit << 16 | leader lane << 8 | rank in the group
+    uint32_t base[kSegIPT];  // the leader's group size, then the group's base
+#pragma unroll
+    for (int it = 0; it < kSegIPT; ++it) {
+      const int x = warp * (32 * kSegIPT) + it * 32 + lane;
+      const int d = x < n ? static_cast<int>((sm.key[cur][x] >> shift) & (kSegBins - 1)) : kSegBins;
+      const unsigned pe = __match_any_sync(0xffffffffu, d);
+      const int leader = __ffs(pe) - 1;
+      dr[it] = (static_cast<uint32_t>(d) << 16) | (static_cast<uint32_t>(leader) << 8) |
+               static_cast<uint32_t>(__popc(pe & lanemask_lt()));
+      base[it] = lane == leader ? static_cast<uint32_t>(__popc(pe)) : 0u;
+    }
+#pragma unroll
+    for (int it = 0; it < kSegIPT; ++it) {
+      const int d = static_cast<int>(dr[it] >> 16);
+      if (d < kSegBins && base[it] != 0) {
+        const int h = (d & 1) * 16;
+        base[it] = (atomicAdd(&sm.hw[warp][d >> 1], base[it] << h) >> h) & 0xffffu;
+      }
+    }
+#pragma unroll
+    for (int it = 0; it < kSegIPT; ++it)
+      dr[it] = (dr[it] & 0xffff0000u) +
+               __shfl_sync(0xffffffffu, base[it], static_cast<int>((dr[it] >> 8) & 31u)) +
+               (dr[it] & 255u);
+    __syncthreads();
+    // per bin pair: exclusive scan over the warps (packed), then the bins'
+    // starts from a block scan of the pair totals
+    constexpr int kPairs = kSegBins / 2;
+    uint32_t run = 0, tot = 0;
+    if (tid < kPairs) {
+      for (int w = 0; w < kSegWarps; ++w) {
+        const uint32_t c = sm.hw[w][tid];
+        sm.hw[w][tid] = run;
+        run += c;
+      }
+      tot = (run & 0xffffu) + (run >> 16);
+    }
+    uint32_t incl = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (tid < kPairs && lane == 31) sm.scan_w[warp] = incl;
+    __syncthreads();
+    if (tid < kPairs) {
+      uint32_t wb = 0;
+      for (int w = 0; w < warp; ++w) wb += sm.scan_w[w];
+      const uint32_t start0 = wb + incl - tot;           // bin 2j
+      const uint32_t start1 = start0 + (run & 0xffffu);  // bin 2j + 1
+      const uint32_t add = start0 | (start1 << 16);
+      for (int w = 0; w < kSegWarps; ++w) sm.hw[w][tid] += add;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int it = 0; it < kSegIPT; ++it) {
+      const int x = warp * (32 * kSegIPT) + it * 32 + lane;
+      if (x < n) {
+        const int d = static_cast<int>(dr[it] >> 16);
+        const uint32_t pos = (sm.hw[warp][d >> 1] >> ((d & 1) * 16)) & 0xffffu;
+        sm.key[cur ^ 1][pos + (dr[it] & 0xffffu)] = sm.key[cur][x];
+      }
+    }
+    __syncthreads();
+    cur ^= 1;
+  }
+  return cur;
+}
+
+// The bits that differ between the keys sm.key[cur][0, n).
+__device__ unsigned long long seg_diff(SegSmem &sm, int n, int cur) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  unsigned long long orv = 0, andv = ~0ull;
+  for (int x = tid; x < n; x += kSegThreads) {
+    orv |= sm.key[cur][x];
+    andv &= sm.key[cur][x];
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    orv |= __shfl_xor_sync(0xffffffffu, orv, o);
+    andv &= __shfl_xor_sync(0xffffffffu, andv, o);
+  }
+  __syncthreads();  // orv / andv of an earlier call have been read
+  if (lane == 0) {
+    sm.orv[warp] = orv;
+    sm.andv[warp] = andv;
+  }
+  __syncthreads();
+  unsigned long long o = 0, a = ~0ull;
+  for (int w = 0; w < kSegWarps; ++w) {
+    o |= sm.orv[w];
+    a &= sm.andv[w];
+  }
+  return o ^ a;
+}
+
+// Small calls (1 <= N <= kSegMax entries, D <= kSmallOrderD): the whole
+// order in one block.  The entries are put in arrival order first unless
+// arrival is already non-decreasing along the index (a stable LSD sort of
+// (arrival, index)); then a stable LSD sort of (decoder, not promoted,
+// promoted ? 0 : bound) in that order gives the queue order (promoted
+// entries keep their arrival order).  Keys carry the index in their low
+// bits.  The segment offsets come from binary searches over the sorted
+// decoders.  One launch instead of a memset and four.
+constexpr int kSmallOrderD = 4096;
+
+__global__ void __launch_bounds__(kSegThreads, 1)
+order_small_kernel(int N, int D, int dbits, const int32_t *__restrict__ dec,
+                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
+                   const int32_t *__restrict__ arrival, int32_t max_wait, int32_t *perm,
+                   int64_t *seg_off, int32_t *status) {
+  pdl_prologue();
+  extern __shared__ __align__(16) unsigned char small_raw[];
+  SegSmem &sm = *reinterpret_cast<SegSmem *>(small_raw);
+  const int tid = threadIdx.x;
+  const int ib = index_bits(N);
+  const unsigned long long imask = (1ull << ib) - 1;
+  bool bad = false, unsorted = false;
+  for (int x = tid; x < N; x += kSegThreads) {
+    const int32_t a = __ldg(arrival + x);
+    if (a < 0) bad = true;
+    if (x + 1 < N && __ldg(arrival + x + 1) < a) unsorted = true;
+    sm.key[0][x] = (static_cast<unsigned long long>(a < 0 ? 0 : a) << ib) | static_cast<unsigned>(x);
+  }
+  unsorted = __syncthreads_or(unsorted) != 0;
+  int cur = 0;
+  if (unsorted) cur = seg_lsd(sm, N, seg_diff(sm, N, 0), ib, ib + 31, 0);
+  for (int t = tid; t < N; t += kSegThreads) {  // the queue keys, in arrival order
+    const int x = static_cast<int>(sm.key[cur][t] & imask);
+    int32_t d = __ldg(dec + x);
+    const int32_t u = __ldg(bound + x), w = __ldg(wait + x);
+    if (d < 0 || d >= D) {
+      bad = true;
+      d = 0;
+    }
+    if (u < 0) bad = true;
+    const unsigned long long np = w > max_wait ? 0ull : 1ull;
+    const unsigned long long prim = np ? static_cast<unsigned long long>(u < 0 ? 0 : u) : 0ull;
+    sm.key[cur ^ 1][t] =
+        (((static_cast<unsigned long long>(d) << 32) | (np << 31) | prim) << ib) | static_cast<unsigned>(x);
+  }
+  __syncthreads();
+  cur ^= 1;
+  cur = seg_lsd(sm, N, seg_diff(sm, N, cur), ib, ib + 32 + dbits, cur);
+  for (int t = tid; t < N; t += kSegThreads) perm[t] = static_cast<int32_t>(sm.key[cur][t] & imask);
+  for (int d = tid; d <= D; d += kSegThreads) {  // entries of decoders below d
+    int lo = 0, hi = N;
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (static_cast<long long>(sm.key[cur][mid] >> (ib + 32)) < d)
+        lo = mid + 1;
+      else
+        hi = mid;
+    }
+    seg_off[d] = lo;
+  }
+  if (__syncthreads_or(bad) && tid == 0) flag_error(status, MAPS_E_RANGE);
+}
+
 // Segmented form, step 2: each sort item (one decoder's queue, at most
 // kSegMax entries) is sorted by one block on its keys (not promoted,
 // promoted ? 0 : bound, index) with stable 9-bit LSD passes in shared
@@ -665,81 +838,7 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
       }
       diff = o ^ a;  // bits that differ between keys of this segment
     }
-    int cur = 0;
-    for (int shift = lo_bit; shift < nbits; shift += kSegBits) {
-      if (((diff >> shift) & (kSegBins - 1)) == 0) continue;  // same digit everywhere: order unchanged
-      for (int i = tid; i < kSegWarps * kSegBins / 2; i += kSegThreads) (&sm.hw[0][0])[i] = 0;
-      __syncthreads();
-      // rank within the warp, stable in item order (warp-major, then item, then
-      // lane): every match first, then one shared atomic per group leader,
-      // issued in item order, whose old value gives the group's base
-      uint32_t dr[kSegIPT];    // digit << 16 | leader lane << 8 | rank in the group
-      uint32_t base[kSegIPT];  // the leader's group size, then the group's base
-#pragma unroll
-      for (int it = 0; it < kSegIPT; ++it) {
-        const int x = warp * (32 * kSegIPT) + it * 32 + lane;
-        const int d = x < n ? static_cast<int>((sm.key[cur][x] >> shift) & (kSegBins - 1)) : kSegBins;
-        const unsigned pe = __match_any_sync(0xffffffffu, d);
-        const int leader = __ffs(pe) - 1;
-        dr[it] = (static_cast<uint32_t>(d) << 16) | (static_cast<uint32_t>(leader) << 8) |
-                 static_cast<uint32_t>(__popc(pe & lanemask_lt()));
-        base[it] = lane == leader ? static_cast<uint32_t>(__popc(pe)) : 0u;
-      }
-#pragma unroll
-      for (int it = 0; it < kSegIPT; ++it) {
-        const int d = static_cast<int>(dr[it] >> 16);
-        if (d < kSegBins && base[it] != 0) {
-          const int h = (d & 1) * 16;
-          base[it] = (atomicAdd(&sm.hw[warp][d >> 1], base[it] << h) >> h) & 0xffffu;
-        }
-      }
-#pragma unroll
-      for (int it = 0; it < kSegIPT; ++it)
-        dr[it] = (dr[it] & 0xffff0000u) +
-                 __shfl_sync(0xffffffffu, base[it], static_cast<int>((dr[it] >> 8) & 31u)) +
-                 (dr[it] & 255u);
-      __syncthreads();
-      // per bin pair: exclusive scan over the warps (packed), then the bins'
-      // starts from a block scan of the pair totals
-      constexpr int kPairs = kSegBins / 2;
-      uint32_t run = 0, tot = 0;
-      if (tid < kPairs) {
-        for (int w = 0; w < kSegWarps; ++w) {
-          const uint32_t c = sm.hw[w][tid];
-          sm.hw[w][tid] = run;
-          run += c;
-        }
-        tot = (run & 0xffffu) + (run >> 16);
-      }
-      uint32_t incl = tot;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      if (tid < kPairs && lane == 31) sm.scan_w[warp] = incl;
-      __syncthreads();
-      if (tid < kPairs) {
-        uint32_t wb = 0;
-        for (int w = 0; w < warp; ++w) wb += sm.scan_w[w];
-        const uint32_t start0 = wb + incl - tot;           // bin 2j
-        const uint32_t start1 = start0 + (run & 0xffffu);  // bin 2j + 1
-        const uint32_t add = start0 | (start1 << 16);
-        for (int w = 0; w < kSegWarps; ++w) sm.hw[w][tid] += add;
-      }
-      __syncthreads();
-#pragma unroll
-      for (int it = 0; it < kSegIPT; ++it) {
-        const int x = warp * (32 * kSegIPT) + it * 32 + lane;
-        if (x < n) {
-          const int d = static_cast<int>(dr[it] >> 16);
-          const uint32_t pos = (sm.hw[warp][d >> 1] >> ((d & 1) * 16)) & 0xffffu;
-          sm.key[cur ^ 1][pos + (dr[it] & 0xffffu)] = sm.key[cur][x];
-        }
-      }
-      __syncthreads();
-      cur ^= 1;
-    }
+    const int cur = seg_lsd(sm, n, diff, lo_bit, nbits, 0);
     const unsigned long long imask = (1ull << ib) - 1;
     if (chunk)
       for (int x = tid; x < n; x += kSegThreads) run_keys[off + x] = sm.key[cur][x];
@@ -1177,9 +1276,18 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   int32_t *status = status_word(ws);
   Carve cv(ws);
   const OrderWs w = carve_order(cv, N, D);
-  MAPS_TRY(cuda_ok(cudaMemsetAsync(w.counts, 0, w.zero_bytes, s)));
   int dbits = 0;  // bits of the largest decoder index
   while ((1ll << dbits) < D) ++dbits;
+  if (N >= 1 && N <= kSegMax && D <= kSmallOrderD) {
+    const size_t small_smem = sizeof(SegSmem);
+    MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_small_kernel,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          static_cast<int>(small_smem))));
+    launch_pdl(order_small_kernel, 1, kSegThreads, small_smem, s, static_cast<int>(N), D, dbits, dec,
+               bound, wait, arrival, max_wait, perm_out, seg_off_out, status);
+    return launch_ok();
+  }
+  MAPS_TRY(cuda_ok(cudaMemsetAsync(w.counts, 0, w.zero_bytes, s)));
   // hi passes that can be active: the key has at most dbits + 1 + 31 bits
   const int n_hi = std::min(kHiPasses, (dbits + 1 + 31 + 7) / 8);
   const int sms = sm_count();
