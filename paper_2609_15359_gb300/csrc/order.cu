@@ -75,6 +75,7 @@ struct OrderCounts {
 // The segment sort then needs no index digits.
 constexpr int kStableD = 1024;
 constexpr int kPrepBlocks = 304;    // prep and key blocks at most
+constexpr int kGroupBlocks = 16;    // prep blocks whose counts are also summed per group
 constexpr int kKeysU = 4;           // entries per thread per round
 constexpr int kKeysRound = 512 * kKeysU;
 __host__ __device__ __forceinline__ int64_t prep_chunk(int64_t N) {
@@ -225,7 +226,7 @@ order_prep_kernel(int64_t N, int D, int64_t chunk, const int32_t *__restrict__ d
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
                   uint32_t *dec_count, int32_t *status, int64_t *seg_off, int64_t *item_off,
                   int32_t *item_n, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, uint32_t *blk,
-                  int Dp) {
+                  uint32_t *grp, int Dp) {
   pdl_prologue();
   __shared__ uint32_t s_dec[kDecSmem];
   __shared__ bool s_last;
@@ -277,9 +278,12 @@ order_prep_kernel(int64_t N, int D, int64_t chunk, const int32_t *__restrict__ d
   if ((threadIdx.x & 31) == 0 && umax) atomicMax(&counts->max_bound, umax);
   if (__syncthreads_or(unsorted) && threadIdx.x == 0) atomicOr(&counts->unsorted, 1u);
   if (dec_smem) {
-    if (D <= kStableD)  // this block's counts, for the stable scatter
-      for (int i = threadIdx.x; i < Dp; i += blockDim.x)
-        blk[static_cast<int64_t>(blockIdx.x) * Dp + i] = i < D ? s_dec[i] : 0u;
+    if (D <= kStableD)  // this block's counts, and its group's, for the stable scatter
+      for (int i = threadIdx.x; i < Dp; i += blockDim.x) {
+        const uint32_t v = i < D ? s_dec[i] : 0u;
+        blk[static_cast<int64_t>(blockIdx.x) * Dp + i] = v;
+        if (v) atomicAdd(&grp[static_cast<int64_t>(blockIdx.x / kGroupBlocks) * Dp + i], v);
+      }
     // blocks start their flush at different decoders so they do not collide
     const int rot = static_cast<int>((static_cast<int64_t>(blockIdx.x) * 97) % D);
     for (int i = threadIdx.x; i < D; i += blockDim.x) {
@@ -309,7 +313,7 @@ order_keys_kernel(int64_t N, int D, int dbits, int64_t chunk, int Dp,
                   const int32_t *__restrict__ wait, const int32_t *__restrict__ arrival,
                   int32_t max_wait, OrderCounts *counts, unsigned long long *hi_orig,
                   unsigned long long *keyA, uint32_t *valA, const int64_t *seg_off,
-                  uint32_t *dec_cursor, const uint32_t *blk) {
+                  uint32_t *dec_cursor, const uint32_t *blk, const uint32_t *grp) {
   pdl_prologue();
   if (*reinterpret_cast<volatile uint32_t *>(&counts->segmented)) {
     // Each entry's segment key (not promoted, primary, index) goes to a slot
@@ -334,23 +338,29 @@ order_keys_kernel(int64_t N, int D, int dbits, int64_t chunk, int Dp,
       uint32_t *run = ksm + kPassWarps * Dp;  // [Dp] next slot of each decoder
       {
         // this block's first slot in every segment: seg_off[d] plus the
-        // counts of the blocks before it.  Thread (quad q of decoders, row
-        // group r) sums rows r, r + rg, ...; the row groups meet in hw.
+        // counts of the blocks before it, as the totals of the earlier groups
+        // of kGroupBlocks blocks plus the rows of the earlier blocks of its
+        // own group.  Thread (quad q of decoders, row group r) sums rows r,
+        // r + rg, ... of that list; the row groups meet in hw.
         const int nq = Dp / 4;
         // rg row groups fit in hw: rg * Dp <= kPassWarps * Dp words
         const int rg = min(kPassWarps, max(1, static_cast<int>(blockDim.x) / nq));
         const int qd = threadIdx.x % nq, r = threadIdx.x / nq;
+        const int g = static_cast<int>(blockIdx.x) / kGroupBlocks, b0 = g * kGroupBlocks;
+        const int nrows = g + static_cast<int>(blockIdx.x) - b0;
         uint4 a0 = make_uint4(0, 0, 0, 0), a1 = a0;
         if (r < rg) {
-          const uint4 *col = reinterpret_cast<const uint4 *>(blk) + qd;
+          const uint4 *gcol = reinterpret_cast<const uint4 *>(grp) + qd;
+          const uint4 *bcol = reinterpret_cast<const uint4 *>(blk) + static_cast<int64_t>(b0 - g) * nq + qd;
+          auto row = [&](int i) { return i < g ? gcol[static_cast<int64_t>(i) * nq] : bcol[static_cast<int64_t>(i) * nq]; };
           int b2 = r;
-          for (; b2 + rg < static_cast<int>(blockIdx.x); b2 += 2 * rg) {  // two loads in flight
-            const uint4 v = col[static_cast<int64_t>(b2) * nq], u = col[static_cast<int64_t>(b2 + rg) * nq];
+          for (; b2 + rg < nrows; b2 += 2 * rg) {  // two loads in flight
+            const uint4 v = row(b2), u = row(b2 + rg);
             a0.x += v.x, a0.y += v.y, a0.z += v.z, a0.w += v.w;
             a1.x += u.x, a1.y += u.y, a1.z += u.z, a1.w += u.w;
           }
-          if (b2 < static_cast<int>(blockIdx.x)) {
-            const uint4 v = col[static_cast<int64_t>(b2) * nq];
+          if (b2 < nrows) {
+            const uint4 v = row(b2);
             a0.x += v.x, a0.y += v.y, a0.z += v.z, a0.w += v.w;
           }
           reinterpret_cast<uint4 *>(hw)[r * nq + qd] =
@@ -1215,7 +1225,8 @@ struct OrderWs {
   int64_t nitems_max, ntiles_max;
   unsigned long long *hi_orig, *keyA, *keyB;
   uint32_t *valA, *valB;
-  uint32_t *blk;      // stable scatter: [blocks][Dp] counts, then block starts
+  uint32_t *blk;      // stable scatter: [blocks][Dp] counts per prep block
+  uint32_t *grp;      // stable scatter: [groups][Dp] counts per kGroupBlocks prep blocks (zeroed)
   int64_t chunk;      // entries per prep / key block
   int blocks, Dp;
 };
@@ -1227,6 +1238,11 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.counts = c.take<OrderCounts>(1);
   w.dec_count = c.take<uint32_t>(static_cast<size_t>(D));
   w.dec_cursor = c.take<uint32_t>(static_cast<size_t>(D));
+  w.chunk = prep_chunk(N);
+  w.blocks = static_cast<int>(std::max<int64_t>(1, (N + w.chunk - 1) / w.chunk));
+  w.Dp = (D + 3) / 4 * 4;
+  w.grp = c.take<uint32_t>(D <= kStableD ? static_cast<size_t>((w.blocks + kGroupBlocks - 1) / kGroupBlocks) * w.Dp
+                                         : 1);
   w.tickets = c.take<uint32_t>(kPasses);
   w.state = c.take<unsigned long long>(static_cast<size_t>(2) * tiles * kRadix);
   w.zero_bytes = c.off - zero_begin - static_cast<size_t>(tiles) * kRadix * sizeof(unsigned long long);
@@ -1244,9 +1260,6 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.keyB = c.take<unsigned long long>(n);
   w.valA = c.take<uint32_t>(n);
   w.valB = c.take<uint32_t>(n);
-  w.chunk = prep_chunk(N);
-  w.blocks = static_cast<int>(std::max<int64_t>(1, (N + w.chunk - 1) / w.chunk));
-  w.Dp = (D + 3) / 4 * 4;
   w.blk = c.take<uint32_t>(D <= kStableD ? static_cast<size_t>(w.blocks) * w.Dp : 1);
   return w;
 }
@@ -1295,7 +1308,7 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   if (N > 0) {
     launch_pdl(order_prep_kernel, w.blocks, 512, 0, s, N, D, w.chunk, dec, bound, wait, arrival,
                max_wait, w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n,
-               w.mt_off, w.mt_n, w.mt_t, w.blk, w.Dp);
+               w.mt_off, w.mt_n, w.mt_t, w.blk, w.grp, w.Dp);
     // the stable scatter's per-warp counts and running slots
     const size_t keys_smem =
         D <= kStableD ? sizeof(uint32_t) * static_cast<size_t>(kPassWarps + 1) * w.Dp : 0;
@@ -1305,7 +1318,7 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
                                             static_cast<int>(keys_smem))));
     launch_pdl(order_keys_kernel, w.blocks, 512, keys_smem, s, N, D, dbits, w.chunk, w.Dp, dec,
                bound, wait, arrival, max_wait, w.counts, w.hi_orig, w.keyA, w.valA, seg_off_out,
-               w.dec_cursor, w.blk);
+               w.dec_cursor, w.blk, w.grp);
   }
   MAPS_TRY(launch_ok());
   if (N == 0) {  // no entries: the segment offsets are all zero
