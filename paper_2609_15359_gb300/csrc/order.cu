@@ -1058,7 +1058,7 @@ __device__ bool order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
   // inclusive prefix, and publishes its own inclusive prefix.  Words carry the
   // flag in their top two bits.  Active pass number o uses state buffer o & 1
   // and clears this tile's row of the other buffer for active pass o + 1
-  // (the buffer of the first active pass is cleared with the counts).
+  // (the buffer of the first active pass is cleared before the passes).
   const int ord = plan->ordinal[p];
   unsigned long long *st_cur = state + static_cast<size_t>(ord & 1) * tiles * kRadix;
   unsigned long long *st_nxt = state + static_cast<size_t>((ord + 1) & 1) * tiles * kRadix;
@@ -1160,6 +1160,11 @@ order_finish_kernel(int n_hi, int64_t N, int D, int dbits, const OrderCounts *co
     return;
   }
   if (blockIdx.x == 0) plan_block(N, D, dbits, counts, plan, dec_count, seg_off);
+  // the look-back words of the first active pass start at zero (the passes
+  // clear the other buffer as they go)
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < tiles * kRadix;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    state[i] = 0ull;
   grid.sync();
   const int npasses = plan->npasses;
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -1215,8 +1220,8 @@ struct OrderWs {
   uint32_t *dec_count;
   uint32_t *dec_cursor;  // segmented form: slots taken per decoder
   uint32_t *tickets;
-  unsigned long long *state;  // [2][tiles][256] look-back words
-  size_t zero_bytes;  // counts .. state buffer 0 are contiguous and zeroed per call
+  unsigned long long *state;  // [2][tiles][256] look-back words (buffer 0 zeroed by the finishing kernel)
+  size_t zero_bytes;  // counts .. tickets are contiguous and zeroed per call
   OrderPlan *plan;
   int64_t *item_off;  // sort items: queues and chunks of long queues
   int32_t *item_n;
@@ -1244,8 +1249,8 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.grp = c.take<uint32_t>(D <= kStableD ? static_cast<size_t>((w.blocks + kGroupBlocks - 1) / kGroupBlocks) * w.Dp
                                          : 1);
   w.tickets = c.take<uint32_t>(kPasses);
+  w.zero_bytes = c.off - zero_begin;
   w.state = c.take<unsigned long long>(static_cast<size_t>(2) * tiles * kRadix);
-  w.zero_bytes = c.off - zero_begin - static_cast<size_t>(tiles) * kRadix * sizeof(unsigned long long);
   w.plan = c.take<OrderPlan>(1);
   w.nitems_max = D + N / kSegMax + 1;
   w.ntiles_max = N / kMergeTile + D + 1;
