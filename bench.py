@@ -53,14 +53,14 @@ L2_FLUSH_BYTES = 256 << 20
 # (dram__bytes_read.sum + dram__bytes_write.sum summed over the call's
 # kernels, one launch each), valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 28587867, "source": "calibrate.cu", "source_sha256":
-                  "dd8c5172871bbabfc606a4ff99cdf1a98fafb7e4db9833dbe2e5fab2935a310f"},
-    "occupancy": {"bytes": 29152146, "source": "occupancy.cu", "source_sha256":
+    "calibrate": {"bytes": 28587178, "source": "calibrate.cu", "source_sha256":
+                  "2c0fe40e5d298e3c515db9c08484268cf10628d6eb822f828c92844c85072ce7"},
+    "occupancy": {"bytes": 29682403, "source": "occupancy.cu", "source_sha256":
                   "66b707f592bb0a8213b6e9f096669a70fc63cfc05bb2a93d1b822468b7656371"},
-    "dispatch": {"bytes": 26419291, "source": "dispatch.cu", "source_sha256":
+    "dispatch": {"bytes": 26421162, "source": "dispatch.cu", "source_sha256":
                  "365bda252b944d4fd3ee47eaca89b1159348ef48bfa86216548008b835726227"},
-    "order": {"bytes": 41114788, "source": "order.cu", "source_sha256":
-              "abd3213d1312229467ff2f47ef27e22bafd54c8ea5c2ed9dc4d4e10e07eda13b"},
+    "order": {"bytes": 41124736, "source": "order.cu", "source_sha256":
+              "325b2629ec7702d5da8b005c28c4a4b65147d7ef9c7770900a4c134be4068abd"},
 }
 KERNELS = {
     "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
