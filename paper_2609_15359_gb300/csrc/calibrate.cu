@@ -217,6 +217,7 @@ bound_kernel(const int32_t *__restrict__ pred, int64_t m, const SelectState *st,
 constexpr int kSmallN = 8192;
 constexpr int kSmallM = 8192;
 constexpr int kSmallThreads = 1024;
+constexpr int kBitonicN = 2048;  // up to this many scores are sorted outright
 
 __global__ void __launch_bounds__(kSmallThreads)
 select_small_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P, int n,
@@ -224,47 +225,71 @@ select_small_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P
                     int32_t *__restrict__ out, SelectState *st, int32_t *q_dev_out,
                     int32_t *status) {
   pdl_prologue();
-  __shared__ uint32_t s[kSmallN];
+  extern __shared__ uint32_t s[];  // the scores (kBitonicN or kSmallN words, as launched)
   __shared__ uint32_t hist[kBins];
   __shared__ uint32_t s_warp[kSmallThreads / 32];
   __shared__ uint32_t s_pick[2];  // the chosen bin, the rank left inside it
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int i = tid; i < n; i += kSmallThreads) s[i] = score(__ldg(L + i), __ldg(P + i));
   uint32_t prefix = 0;
-  unsigned long long kr = k;  // rank still to find among the scores matching prefix
-  for (int pass = 0; pass < kPasses; ++pass) {
-    const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
-    const int bits = pass == 2 ? 10 : 11;
-    const int prev = pass == 0 ? 32 : (pass == 1 ? 21 : 10);  // bits above this digit
-    for (int b = tid; b < kBins; b += kSmallThreads) hist[b] = 0;
+  if (n <= kBitonicN) {
+    // few scores: sort them (bitonic network, padded to a power of two with
+    // the largest value) and take the k-th smallest
+    int Pn = 1;
+    while (Pn < n) Pn <<= 1;
+    for (int i = n + tid; i < Pn; i += kSmallThreads) s[i] = 0xffffffffu;
     __syncthreads();
-    for (int i = tid; i < n; i += kSmallThreads) {
-      const uint32_t v = s[i];
-      if (prev == 32 || (v >> prev) == prefix) atomicAdd(&hist[(v >> shift) & ((1u << bits) - 1)], 1u);
+    for (int kk = 2; kk <= Pn; kk <<= 1)
+      for (int j = kk >> 1; j > 0; j >>= 1) {
+        for (int i = tid; i < Pn; i += kSmallThreads) {
+          const int l = i ^ j;
+          if (l > i) {
+            const uint32_t x = s[i], y = s[l];
+            if ((x > y) == ((i & kk) == 0)) {
+              s[i] = y;
+              s[l] = x;
+            }
+          }
+        }
+        __syncthreads();
+      }
+    prefix = s[k - 1];
+  } else {
+    unsigned long long kr = k;  // rank still to find among the scores matching prefix
+    for (int pass = 0; pass < kPasses; ++pass) {
+      const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
+      const int bits = pass == 2 ? 10 : 11;
+      const int prev = pass == 0 ? 32 : (pass == 1 ? 21 : 10);  // bits above this digit
+      for (int b = tid; b < kBins; b += kSmallThreads) hist[b] = 0;
+      __syncthreads();
+      for (int i = tid; i < n; i += kSmallThreads) {
+        const uint32_t v = s[i];
+        if (prev == 32 || (v >> prev) == prefix) atomicAdd(&hist[(v >> shift) & ((1u << bits) - 1)], 1u);
+      }
+      __syncthreads();
+      // exclusive scan of the bins (two per thread), then the bin holding rank kr
+      const uint32_t c0 = hist[2 * tid], c1 = hist[2 * tid + 1];
+      const uint32_t tot = c0 + c1;
+      uint32_t incl = tot;
+  #pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+      }
+      if (lane == 31) s_warp[warp] = incl;
+      __syncthreads();
+      uint32_t excl = incl - tot;
+      for (int w = 0; w < warp; ++w) excl += s_warp[w];
+      if (excl < kr && kr <= static_cast<unsigned long long>(excl) + tot) {
+        const bool first = kr <= static_cast<unsigned long long>(excl) + c0;
+        s_pick[0] = 2 * tid + (first ? 0 : 1);
+        s_pick[1] = static_cast<uint32_t>(kr - excl - (first ? 0 : c0));
+      }
+      __syncthreads();
+      prefix = (prefix << bits) | s_pick[0];
+      kr = s_pick[1];
+      __syncthreads();  // hist and s_pick are reused by the next pass
     }
-    __syncthreads();
-    // exclusive scan of the bins (two per thread), then the bin holding rank kr
-    const uint32_t c0 = hist[2 * tid], c1 = hist[2 * tid + 1];
-    const uint32_t tot = c0 + c1;
-    uint32_t incl = tot;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
-      if (lane >= off) incl += y;
-    }
-    if (lane == 31) s_warp[warp] = incl;
-    __syncthreads();
-    uint32_t excl = incl - tot;
-    for (int w = 0; w < warp; ++w) excl += s_warp[w];
-    if (excl < kr && kr <= static_cast<unsigned long long>(excl) + tot) {
-      const bool first = kr <= static_cast<unsigned long long>(excl) + c0;
-      s_pick[0] = 2 * tid + (first ? 0 : 1);
-      s_pick[1] = static_cast<uint32_t>(kr - excl - (first ? 0 : c0));
-    }
-    __syncthreads();
-    prefix = (prefix << bits) | s_pick[0];
-    kr = s_pick[1];
-    __syncthreads();  // hist and s_pick are reused by the next pass
   }
   if (prefix > 0x7fffffffu) {
     if (tid == 0) flag_error(status, MAPS_E_RANGE);
@@ -330,7 +355,9 @@ int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
   const unsigned long long kk = static_cast<unsigned long long>(k);
   if (n <= kSmallN) {
     const int mi = m <= kSmallM ? static_cast<int>(m) : 0;  // bounds in the same block
-    launch_pdl(select_small_kernel, 1, kSmallThreads, 0, s, true_len, pred_len, static_cast<int>(n),
+    launch_pdl(select_small_kernel, 1, kSmallThreads,
+               (n <= kBitonicN ? kBitonicN : kSmallN) * sizeof(uint32_t), s, true_len, pred_len,
+               static_cast<int>(n),
                kk, query_pred, mi, bound_out, st, q_dev_out, status);
     MAPS_TRY(launch_ok());
     if (m <= kSmallM) m = 0;

@@ -732,13 +732,36 @@ __device__ unsigned long long seg_diff(SegSmem &sm, int n, int cur) {
 
 // Small calls (1 <= N <= kSegMax entries, D <= kSmallOrderD): the whole
 // order in one block.  The entries are put in arrival order first unless
-// arrival is already non-decreasing along the index (a stable LSD sort of
-// (arrival, index)); then a stable LSD sort of (decoder, not promoted,
-// promoted ? 0 : bound) in that order gives the queue order (promoted
-// entries keep their arrival order).  Keys carry the index in their low
-// bits.  The segment offsets come from binary searches over the sorted
-// decoders.  One launch instead of a memset and four.
+// arrival is already non-decreasing along the index (a sort of (arrival,
+// index)); then a sort of (decoder, not promoted, promoted ? 0 : bound,
+// arrival position) gives the queue order (promoted entries keep their
+// arrival order).  Up to kBitonicN entries both sorts are bitonic networks
+// over unique keys (a few dozen barrier-separated stages); larger calls take
+// stable 9-bit LSD passes with the index in the keys' low bits.  The segment
+// offsets come from binary searches over the sorted decoders.  One launch
+// instead of a memset and four.
 constexpr int kSmallOrderD = 4096;
+constexpr int kBitonicN = 1024;
+
+// Ascending bitonic sort of a[0, P) in shared memory, P a power of two (the
+// block's threads take the compare-exchanges of each stage in turn).
+template <typename T>
+__device__ void block_bitonic(T *a, int P) {
+  for (int k = 2; k <= P; k <<= 1)
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = threadIdx.x; i < P; i += blockDim.x) {
+        const int l = i ^ j;
+        if (l > i) {
+          const T x = a[i], y = a[l];
+          if ((x > y) == ((i & k) == 0)) {
+            a[i] = y;
+            a[l] = x;
+          }
+        }
+      }
+      __syncthreads();
+    }
+}
 
 __global__ void __launch_bounds__(kSegThreads, 1)
 order_small_kernel(int N, int D, int dbits, const int32_t *__restrict__ dec,
@@ -752,17 +775,35 @@ order_small_kernel(int N, int D, int dbits, const int32_t *__restrict__ dec,
   const int ib = index_bits(N);
   const unsigned long long imask = (1ull << ib) - 1;
   bool bad = false, unsorted = false;
+  const bool bit = N <= kBitonicN;
+  unsigned long long *k0 = bit ? reinterpret_cast<unsigned long long *>(small_raw) : sm.key[0];
   for (int x = tid; x < N; x += kSegThreads) {
     const int32_t a = __ldg(arrival + x);
     if (a < 0) bad = true;
     if (x + 1 < N && __ldg(arrival + x + 1) < a) unsorted = true;
-    sm.key[0][x] = (static_cast<unsigned long long>(a < 0 ? 0 : a) << ib) | static_cast<unsigned>(x);
+    k0[x] = (static_cast<unsigned long long>(a < 0 ? 0 : a) << ib) | static_cast<unsigned>(x);
   }
+  int P = 1;
+  while (P < N) P <<= 1;
   unsorted = __syncthreads_or(unsorted) != 0;
   int cur = 0;
-  if (unsorted) cur = seg_lsd(sm, N, seg_diff(sm, N, 0), ib, ib + 31, 0);
+  // the bitonic path's two key arrays sit back to back (the launch asks for
+  // only 2 kBitonicN keys of shared memory then)
+  unsigned long long *kb[2] = {reinterpret_cast<unsigned long long *>(small_raw),
+                               reinterpret_cast<unsigned long long *>(small_raw) + kBitonicN};
+  if (unsorted) {
+    if (bit) {
+      for (int x = N + tid; x < P; x += kSegThreads) kb[0][x] = ~0ull;
+      __syncthreads();
+      block_bitonic(kb[0], P);
+    } else {
+      cur = seg_lsd(sm, N, seg_diff(sm, N, 0), ib, ib + 31, 0);
+    }
+  }
+  unsigned long long *kin = bit ? kb[0] : sm.key[cur];
+  unsigned long long *kout = bit ? kb[1] : sm.key[cur ^ 1];
   for (int t = tid; t < N; t += kSegThreads) {  // the queue keys, in arrival order
-    const int x = static_cast<int>(sm.key[cur][t] & imask);
+    const int x = static_cast<int>(kin[t] & imask);
     int32_t d = __ldg(dec + x);
     const int32_t u = __ldg(bound + x), w = __ldg(wait + x);
     if (d < 0 || d >= D) {
@@ -772,18 +813,31 @@ order_small_kernel(int N, int D, int dbits, const int32_t *__restrict__ dec,
     if (u < 0) bad = true;
     const unsigned long long np = w > max_wait ? 0ull : 1ull;
     const unsigned long long prim = np ? static_cast<unsigned long long>(u < 0 ? 0 : u) : 0ull;
-    sm.key[cur ^ 1][t] =
-        (((static_cast<unsigned long long>(d) << 32) | (np << 31) | prim) << ib) | static_cast<unsigned>(x);
+    // low bits: the arrival position for the bitonic sort (unique keys), the
+    // index for the stable passes
+    kout[t] = (((static_cast<unsigned long long>(d) << 32) | (np << 31) | prim) << ib) |
+              static_cast<unsigned>(bit ? t : x);
   }
-  __syncthreads();
-  cur ^= 1;
-  cur = seg_lsd(sm, N, seg_diff(sm, N, cur), ib, ib + 32 + dbits, cur);
-  for (int t = tid; t < N; t += kSegThreads) perm[t] = static_cast<int32_t>(sm.key[cur][t] & imask);
+  const unsigned long long *ks;  // the sorted queue keys
+  if (bit) {
+    for (int t = N + tid; t < P; t += kSegThreads) kout[t] = ~0ull;
+    __syncthreads();
+    block_bitonic(kout, P);
+    for (int t = tid; t < N; t += kSegThreads)  // arrival position -> index
+      perm[t] = static_cast<int32_t>(kin[kout[t] & imask] & imask);
+    ks = kout;
+  } else {
+    __syncthreads();
+    cur ^= 1;
+    cur = seg_lsd(sm, N, seg_diff(sm, N, cur), ib, ib + 32 + dbits, cur);
+    for (int t = tid; t < N; t += kSegThreads) perm[t] = static_cast<int32_t>(sm.key[cur][t] & imask);
+    ks = sm.key[cur];
+  }
   for (int d = tid; d <= D; d += kSegThreads) {  // entries of decoders below d
     int lo = 0, hi = N;
     while (lo < hi) {
       const int mid = (lo + hi) >> 1;
-      if (static_cast<long long>(sm.key[cur][mid] >> (ib + 32)) < d)
+      if (static_cast<long long>(ks[mid] >> (ib + 32)) < d)
         lo = mid + 1;
       else
         hi = mid;
@@ -1297,10 +1351,11 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   int dbits = 0;  // bits of the largest decoder index
   while ((1ll << dbits) < D) ++dbits;
   if (N >= 1 && N <= kSegMax && D <= kSmallOrderD) {
-    const size_t small_smem = sizeof(SegSmem);
+    const size_t small_smem =
+        N <= kBitonicN ? 2 * kBitonicN * sizeof(unsigned long long) : sizeof(SegSmem);
     MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_small_kernel,
                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          static_cast<int>(small_smem))));
+                                          static_cast<int>(sizeof(SegSmem)))));
     launch_pdl(order_small_kernel, 1, kSegThreads, small_smem, s, static_cast<int>(N), D, dbits, dec,
                bound, wait, arrival, max_wait, perm_out, seg_off_out, status);
     return launch_ok();

@@ -443,6 +443,10 @@ def test_dispatch_errors(M, ws, oracle):
                                                 (100, 3, False), (4096, 8, True), (4097, 8, False),
                                                 (50000, 64, True), (50001, 300, False),
                                                 (300000, 256, False), (1000, 70000, True),
+                                                # one-block calls: bitonic up to 1,024
+                                                # entries, then stable passes
+                                                (700, 5, True), (1024, 16, False),
+                                                (1025, 16, True), (3000, 40, False),
                                                 # one decoder's queue at, and past, the most a
                                                 # block sorts in shared memory
                                                 (4608, 1, True), (4609, 1, True),
