@@ -267,6 +267,11 @@ size_t stream_dispatch_smem(int D, int nact, int nb) {
 // V_i = SS[i] + (E[i] - 1)(n - i + 1) (K + t at t = E[i] - 1).  Returns
 // whether some K(t) exceeds INT32_MAX (the projection's range error); below
 // that every SS, V and PM fits 32 bits.
+// Barrier `id` over the first `count` threads (whole warps) of the block.
+__device__ __forceinline__ void named_bar(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 __device__ bool rebuild_tables(const int32_t *E, const int32_t *Bv, uint32_t *SS, uint32_t *PM,
                                int n) {
   const int lane = threadIdx.x & 31;
@@ -386,39 +391,32 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
   // e <= u), then M = max(PM[c - 1], SS[c] + (u - 1)(n - c + 1)); a packed key
   // picks (feasible first, then Q or the largest headroom, then the lowest
   // index); the warp inserts the footprint and rebuilds that decoder's tables.
-  if (warp == 0 && D <= 32) {
-    // One decoder per lane: its list length, base, Q and capacity stay in
-    // registers, the next candidate is read ahead, and c comes from an 8-ary
-    // search (eight independent probes per level: a list of up to 8 pairs
-    // takes one level, up to 64 two).
-    const int k = lane;
-    const bool has = k < D;
-    int n_r = has ? s_n[k] : 0, q_r = has ? s_q[k] : 0;
-    const int base_r = has ? s_base[k] : 0, cap_r = has ? s_cap[k] : 0;
-    int32_t p_nx = nb > 0 ? s_cp[0] : 0, U_nx = nb > 0 ? s_cu[0] : 0;
-    for (int j = 0; j < nb; ++j) {
-      const int32_t p = p_nx, U = U_nx;
-      if (j + 1 < nb) {
-        p_nx = s_cp[j + 1];
-        U_nx = s_cu[j + 1];
-      }
-      if ((p | U) < 0) {
-        if (lane == 0) {
-          flag_error(status, MAPS_E_RANGE);
-          choice[j] = -1;
-          if (headroom) headroom[j] = 0;
-        }
-        continue;
-      }
-      const int u = U < 1 ? 1 : (U > H ? H : U);
-      int lo = 0, hi = n_r;  // c = the pairs with e <= u lies in [lo, hi]
+  if (D <= 32) {
+    // Two warps, one decoder per lane.  Warp 0 holds each decoder's list
+    // length, base, Q and capacity in registers, scores the candidates, picks
+    // and books each decision and hands it to warp 1 through shared memory
+    // (named barrier 1); warp 1 inserts the reservation into the chosen
+    // decoder's list and scores that decoder again for the next candidate
+    // (named barrier 2).  Meanwhile warp 0 scores the next candidate on the
+    // lists as they stand: a reservation only raises the chosen decoder's Q
+    // and occupancy, so every other decoder's key is already final and the
+    // chosen one's is replaced by warp 1's.  Keys: inf << 63 | v << 10 | k,
+    // the smallest wins.
+    __shared__ int h_bk, h_pos, h_n, h_base, h_q, h_cap, h_c;
+    __shared__ long long h_M;
+    __shared__ unsigned long long h_key;
+    auto clampu = [&](int32_t U) { return U < 1 ? 1 : (U > H ? H : U); };
+    // c = the pairs with e <= u of a sorted list (8-ary search: eight
+    // independent probes per level, one level for up to 8 pairs)
+    auto count_le = [&](const int32_t *Ek, int n, int u) {
+      int lo = 0, hi = n;
       while (lo < hi) {
         const int len = hi - lo;
         int nlo = lo, nhi = hi;
 #pragma unroll
         for (int i = 0; i < 8; ++i) {  // probes cover every position when len <= 8
           const int pi = lo + (len * i) / 8;
-          if (E[base_r + pi] <= u)
+          if (Ek[pi] <= u)
             nlo = max(nlo, pi + 1);
           else
             nhi = min(nhi, pi);
@@ -426,96 +424,178 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
         lo = nlo;
         hi = nhi;
       }
-      const int c = lo;
+      return lo;
+    };
+    auto key_of = [](int k, int q, int cap, int32_t p, long long M) {
+      const long long h = static_cast<long long>(cap) - (static_cast<long long>(p) + 1 + M);
+      return h >= 0 ? (static_cast<unsigned long long>(q) << 10) | static_cast<unsigned>(k)
+                    : (1ull << 63) | (static_cast<unsigned long long>(-h) << 10) | static_cast<unsigned>(k);
+    };
+    if (warp == 0) {
+      const int k = lane;
+      const bool has = k < D;
+      int n_r = has ? s_n[k] : 0, q_r = has ? s_q[k] : 0;
+      const int base_r = has ? s_base[k] : 0, cap_r = has ? s_cap[k] : 0;
+      bool bad = false, have = false;  // have: key, c and M are the current candidate's
+      unsigned long long key = ~0ull;
       long long M = 0;
-      unsigned long long key = ~0ull;  // inf << 63 | v << 10 | k, the smallest wins
-      if (has) {
+      int c = 0;
+      auto score = [&](int32_t pp, int uu) {
+        key = ~0ull;
+        if (!has) return;
+        c = count_le(E + base_r, n_r, uu);
         const long long full = c > 0 ? static_cast<long long>(PM[base_r + c - 1]) : LLONG_MIN;
         const long long part = static_cast<long long>(c < n_r ? SS[base_r + c] : 0u) +
-                               static_cast<long long>(u - 1) * (n_r - c + 1);
+                               static_cast<long long>(uu - 1) * (n_r - c + 1);
         M = max(full, part);
-        const long long h = static_cast<long long>(cap_r) - (static_cast<long long>(p) + 1 + M);
-        key = h >= 0 ? (static_cast<unsigned long long>(q_r) << 10) | static_cast<unsigned>(k)
-                     : (1ull << 63) | (static_cast<unsigned long long>(-h) << 10) | static_cast<unsigned>(k);
-      }
-      const unsigned long long kv = (key >> 10) & ((1ull << 53) - 1);
-      const bool none = key == ~0ull;
-      int bk;
-      if (__all_sync(0xffffffffu, none || kv < (1ull << 21))) {
-        const uint32_t k32 = none ? 0xffffffffu
-                                  : (static_cast<uint32_t>(key >> 63) << 31) |
-                                        (static_cast<uint32_t>(kv) << 10) | static_cast<uint32_t>(key & 1023u);
-        bk = static_cast<int>(__reduce_min_sync(0xffffffffu, k32) & 1023u);
-      } else {
+        key = key_of(k, q_r, cap_r, pp, M);
+      };
+      for (int j = 0; j < nb; ++j) {
+        const int32_t p = s_cp[j], U = s_cu[j];
+        int bk = -1;
+        if ((p | U) >= 0) {
+          if (!have) score(p, clampu(U));
+          // the warp's smallest key: one 32-bit reduction when every value
+          // fits 21 bits (inf << 31 | v << 10 | k, the same order), else a ladder
+          const unsigned long long kv = (key >> 10) & ((1ull << 53) - 1);
+          const bool none = key == ~0ull;
+          if (__all_sync(0xffffffffu, none || kv < (1ull << 21))) {
+            const uint32_t k32 = none ? 0xffffffffu
+                                      : (static_cast<uint32_t>(key >> 63) << 31) |
+                                            (static_cast<uint32_t>(kv) << 10) | static_cast<uint32_t>(key & 1023u);
+            bk = static_cast<int>(__reduce_min_sync(0xffffffffu, k32) & 1023u);
+          } else {
+            unsigned long long kk = key;
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
-          const unsigned long long o = __shfl_xor_sync(0xffffffffu, key, off);
-          key = o < key ? o : key;
-        }
-        bk = static_cast<int>(key & 1023u);
-      }
-      const int pos = __shfl_sync(0xffffffffu, c, bk);
-      const int n = __shfl_sync(0xffffffffu, n_r, bk);
-      const int base = __shfl_sync(0xffffffffu, base_r, bk);
-      if (lane == bk) {  // the chosen decoder's lane books the decision
-        choice[j] = bk;
-        if (headroom) headroom[j] = static_cast<long long>(cap_r) - (static_cast<long long>(p) + 1 + M);
-        if (q_r == 0x7fffffff)
-          flag_error(status, MAPS_E_RANGE);
-        else
-          q_r += 1;
-        // every new cell K + p + t + 1 (t < u) is at most M + p + 1
-        if (static_cast<long long>(p) + 1 + M > 0x7fffffffLL) flag_error(status, MAPS_E_RANGE);
-        n_r = n + 1;
-      }
-      const int m = n + 1;
-      if (m <= 32) {
-        // the insert and the table update in one round (as below)
-        const int src = lane <= pos ? lane : lane - 1;
-        const bool old_ok = src < n;
-        const int eo = old_ok ? E[base + src] : 0, bo = old_ok ? Bv[base + src] : 0;
-        const uint32_t so = old_ok ? SS[base + src] : 0u;
-        const uint32_t bnew = static_cast<uint32_t>(p) + 1u;
-        const int e2 = lane == pos ? u : eo;
-        const int b2 = lane == pos ? static_cast<int>(bnew) : bo;
-        const uint32_t suf = lane <= pos ? so + bnew : so;
-        uint32_t V = lane < m ? suf + static_cast<uint32_t>(e2 - 1) * static_cast<uint32_t>(m - lane + 1) : 0u;
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-          const uint32_t y = __shfl_up_sync(0xffffffffu, V, off);
-          if (lane >= off) V = max(V, y);
-        }
-        __syncwarp();  // every lane has read the old list
-        if (lane < m) {
-          E[base + lane] = e2;
-          Bv[base + lane] = b2;
-          SS[base + lane] = suf;
-          PM[base + lane] = V;
-        }
-        __syncwarp();
-      } else {
-        for (int r = (n - 1) >> 5; r >= 0; --r) {  // shift [pos, n) up by one, last round first
-          const int i = r * 32 + lane;
-          const bool mv = i < n && i >= pos;
-          const int e = mv ? E[base + i] : 0, b = mv ? Bv[base + i] : 0;
-          __syncwarp();
-          if (mv) {
-            E[base + i + 1] = e;
-            Bv[base + i + 1] = b;
+            for (int off = 16; off > 0; off >>= 1) {
+              const unsigned long long o = __shfl_xor_sync(0xffffffffu, kk, off);
+              kk = o < kk ? o : kk;
+            }
+            bk = static_cast<int>(kk & 1023u);
           }
-          __syncwarp();
+          if (lane == bk) {  // the chosen decoder's lane books the decision
+            choice[j] = bk;
+            if (headroom) headroom[j] = static_cast<long long>(cap_r) - (static_cast<long long>(p) + 1 + M);
+            bad |= q_r == 0x7fffffff;
+            q_r += q_r == 0x7fffffff ? 0 : 1;
+            // every new cell K + p + t + 1 (t < u) is at most M + p + 1
+            bad |= static_cast<long long>(p) + 1 + M > 0x7fffffffLL;
+            h_bk = bk;
+            h_pos = c;
+            h_n = n_r;
+            h_base = base_r;
+            h_q = q_r;
+            h_cap = cap_r;
+            n_r += 1;
+          }
+        } else if (lane == 0) {
+          bad = true;
+          choice[j] = -1;
+          if (headroom) headroom[j] = 0;
+          h_bk = -1;
         }
-        if (lane == 0) {
-          E[base + pos] = u;
-          Bv[base + pos] = p + 1;
+        named_bar(1, 64);  // the decision goes to warp 1
+        const bool nxt = j + 1 < nb;
+        const int32_t p1 = nxt ? s_cp[j + 1] : 0, U1 = nxt ? s_cu[j + 1] : 0;
+        const bool ok1 = nxt && (p1 | U1) >= 0;
+        if (ok1) score(p1, clampu(U1));  // the chosen decoder's key is replaced below
+        named_bar(2, 64);  // warp 1 has updated the list and scored it again
+        if (ok1 && lane == bk) {
+          key = h_key;
+          c = h_c;
+          M = h_M;
         }
-        __syncwarp();
-        rebuild_tables(E + base, Bv + base, SS + base, PM + base, m);
+        have = ok1;
       }
-    }
-    if (has) {
-      s_n[k] = n_r;
-      s_q[k] = q_r;
+      if (__any_sync(0xffffffffu, bad) && lane == 0) flag_error(status, MAPS_E_RANGE);
+      if (has) {
+        s_n[k] = n_r;
+        s_q[k] = q_r;
+      }
+    } else if (warp == 1) {
+      for (int j = 0; j < nb; ++j) {
+        named_bar(1, 64);
+        const int bk = h_bk;
+        if (bk >= 0) {
+          const int pos = h_pos, n = h_n, base = h_base, m = n + 1;
+          const int32_t p = s_cp[j];
+          const int u = clampu(s_cu[j]);
+          const bool nxt = j + 1 < nb;
+          const int32_t p1 = nxt ? s_cp[j + 1] : 0, U1 = nxt ? s_cu[j + 1] : 0;
+          const bool ok1 = nxt && (p1 | U1) >= 0;
+          const int u1 = clampu(U1);
+          int c1 = 0;
+          long long M1 = 0;
+          if (m <= 32) {
+            // one round: lane i takes pair i of the new list; the suffix sums
+            // follow from the old ones (b more before the new pair, the same
+            // after it) and one shuffle scan gives the prefix maxima of V, in
+            // 32 bits (the booking's check keeps every K + t within INT32_MAX)
+            const int src = lane <= pos ? lane : lane - 1;
+            const bool old_ok = src < n;
+            const int eo = old_ok ? E[base + src] : 0, bo = old_ok ? Bv[base + src] : 0;
+            const uint32_t so = old_ok ? SS[base + src] : 0u;
+            const uint32_t bnew = static_cast<uint32_t>(p) + 1u;
+            const int e2 = lane == pos ? u : eo;
+            const int b2 = lane == pos ? static_cast<int>(bnew) : bo;
+            const uint32_t suf = lane <= pos ? so + bnew : so;
+            uint32_t V = lane < m ? suf + static_cast<uint32_t>(e2 - 1) * static_cast<uint32_t>(m - lane + 1) : 0u;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+              const uint32_t y = __shfl_up_sync(0xffffffffu, V, off);
+              if (lane >= off) V = max(V, y);
+            }
+            __syncwarp();  // every lane has read the old list
+            if (lane < m) {
+              E[base + lane] = e2;
+              Bv[base + lane] = b2;
+              SS[base + lane] = suf;
+              PM[base + lane] = V;
+            }
+            // the new list's count and table values at the next candidate's u
+            c1 = __popc(__ballot_sync(0xffffffffu, lane < m && e2 <= u1));
+            const uint32_t pmb = __shfl_sync(0xffffffffu, V, c1 > 0 ? c1 - 1 : 0);
+            const uint32_t ssb = __shfl_sync(0xffffffffu, suf, c1 < m ? c1 : 0);
+            const long long full = c1 > 0 ? static_cast<long long>(pmb) : LLONG_MIN;
+            const long long part = static_cast<long long>(c1 < m ? ssb : 0u) +
+                                   static_cast<long long>(u1 - 1) * (m - c1 + 1);
+            M1 = max(full, part);
+          } else {
+            // a list past 32 pairs: shift [pos, n) up by one (last round
+            // first), place the new pair, rebuild the tables
+            for (int r = (n - 1) >> 5; r >= 0; --r) {
+              const int i = r * 32 + lane;
+              const bool mv = i < n && i >= pos;
+              const int e = mv ? E[base + i] : 0, b = mv ? Bv[base + i] : 0;
+              __syncwarp();
+              if (mv) {
+                E[base + i + 1] = e;
+                Bv[base + i + 1] = b;
+              }
+              __syncwarp();
+            }
+            if (lane == 0) {
+              E[base + pos] = u;
+              Bv[base + pos] = p + 1;
+            }
+            __syncwarp();
+            rebuild_tables(E + base, Bv + base, SS + base, PM + base, m);
+            if (ok1) {
+              c1 = count_le(E + base, m, u1);
+              const long long full = c1 > 0 ? static_cast<long long>(PM[base + c1 - 1]) : LLONG_MIN;
+              const long long part = static_cast<long long>(c1 < m ? SS[base + c1] : 0u) +
+                                     static_cast<long long>(u1 - 1) * (m - c1 + 1);
+              M1 = max(full, part);
+            }
+          }
+          if (ok1 && lane == 0) {
+            h_key = key_of(bk, h_q, h_cap, p1, M1);
+            h_c = c1;
+            h_M = M1;
+          }
+        }
+        named_bar(2, 64);
+      }
     }
   } else if (warp == 0) {
     for (int j = 0; j < nb; ++j) {
