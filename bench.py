@@ -53,14 +53,14 @@ L2_FLUSH_BYTES = 256 << 20
 # (dram__bytes_read.sum + dram__bytes_write.sum summed over the call's
 # kernels, one launch each), valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 28587178, "source": "calibrate.cu", "source_sha256":
-                  "2c0fe40e5d298e3c515db9c08484268cf10628d6eb822f828c92844c85072ce7"},
-    "occupancy": {"bytes": 29682403, "source": "occupancy.cu", "source_sha256":
+    "calibrate": {"bytes": 28585216, "source": "calibrate.cu", "source_sha256":
+                  "16385f686731a11d81b2c01d813292cfe4b95130e9c4e2af1a78e2a682738e07"},
+    "occupancy": {"bytes": 29674695, "source": "occupancy.cu", "source_sha256":
                   "66b707f592bb0a8213b6e9f096669a70fc63cfc05bb2a93d1b822468b7656371"},
-    "dispatch": {"bytes": 26421162, "source": "dispatch.cu", "source_sha256":
+    "dispatch": {"bytes": 26419854, "source": "dispatch.cu", "source_sha256":
                  "365bda252b944d4fd3ee47eaca89b1159348ef48bfa86216548008b835726227"},
-    "order": {"bytes": 41124736, "source": "order.cu", "source_sha256":
-              "325b2629ec7702d5da8b005c28c4a4b65147d7ef9c7770900a4c134be4068abd"},
+    "order": {"bytes": 41117564, "source": "order.cu", "source_sha256":
+              "47710cf71f15241ffda0f21d330c997d5f56c4eff43e1872756c4a475a55d0ae"},
 }
 KERNELS = {
     "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
