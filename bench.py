@@ -15,7 +15,8 @@ Timing: inputs resident in HBM; before every step the L2 is flushed (a
 host enqueues the step, so CUDA events on the launching stream bracket the
 device time of the step alone.  Each timed step replays one CUDA graph of the
 four calls; a second pass of direct launches with an event between calls
-gives the per-call split (and the rooflines).  The end-to-end figure repeats the step
+gives the per-call split (and the rooflines), and a third times the
+dispatch's scoring kernel alone (events recorded by maps_dispatch around it).  The end-to-end figure repeats the step
 through the same C-ABI calls with pinned host buffers, host-to-device copies
 of every input and device-to-host copies of every output inside the timed
 region; steps are pipelined over two buffer sets, each stage replayed from a
@@ -51,15 +52,18 @@ L2_FLUSH_BYTES = 256 << 20
 
 # DRAM traffic per call on this workload from an ncu capture
 # (dram__bytes_read.sum + dram__bytes_write.sum summed over the call's
-# kernels, one launch each), valid only for the kernel source it was taken on.
+# kernels, one launch each; dispatch_scoring is the scoring kernel alone),
+# valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 28585216, "source": "calibrate.cu", "source_sha256":
+    "calibrate": {"bytes": 28585472, "source": "calibrate.cu", "source_sha256":
                   "16385f686731a11d81b2c01d813292cfe4b95130e9c4e2af1a78e2a682738e07"},
-    "occupancy": {"bytes": 29674695, "source": "occupancy.cu", "source_sha256":
+    "occupancy": {"bytes": 29646023, "source": "occupancy.cu", "source_sha256":
                   "66b707f592bb0a8213b6e9f096669a70fc63cfc05bb2a93d1b822468b7656371"},
-    "dispatch": {"bytes": 26419854, "source": "dispatch.cu", "source_sha256":
-                 "365bda252b944d4fd3ee47eaca89b1159348ef48bfa86216548008b835726227"},
-    "order": {"bytes": 41117564, "source": "order.cu", "source_sha256":
+    "dispatch": {"bytes": 26419911, "source": "dispatch.cu", "source_sha256":
+                 "9a0669b4c3b6a98229e1f3de3d355bb4f1ca14d1b808ae269b98701bb59cde8c"},
+    "dispatch_scoring": {"bytes": 21100600, "source": "dispatch.cu", "source_sha256":
+                         "9a0669b4c3b6a98229e1f3de3d355bb4f1ca14d1b808ae269b98701bb59cde8c"},
+    "order": {"bytes": 41119096, "source": "order.cu", "source_sha256":
               "47710cf71f15241ffda0f21d330c997d5f56c4eff43e1872756c4a475a55d0ae"},
 }
 KERNELS = {
@@ -67,6 +71,8 @@ KERNELS = {
     "occupancy": "occ_bucket_kernel + occ_tile_kernel (maps_project_occupancy)",
     "dispatch": "dispatch_prep (carry scan + bin count) + bin_scatter + dispatch_snapshot_kernel (maps_dispatch)",
     "order": "order_prep + order_keys + order_segsort + order_finish (maps_order_local)",
+    "dispatch_scoring": "dispatch_snapshot_kernel alone (maps_dispatch's scoring kernel, after "
+                        "the candidates are bucketed by horizon tile)",
 }
 
 
@@ -419,6 +425,11 @@ def bench_gpu(args, world, rank, local, dist):
     Kb = max(5, min(K, 50))
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
     evb = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(Kb)]
+    # around the dispatch's scoring kernel alone (after its candidate bucketing)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(Kb)]
+    for pair in evs:
+        for e in pair:
+            e.record()  # the CUDA events exist from here on
     sampler = ClockSampler(local)
     if dist is not None and dist.is_initialized():
         dist.barrier()
@@ -443,6 +454,14 @@ def bench_gpu(args, world, rank, local, dist):
         e[3].record()
         step.run(ev=e)
         e[4].record()
+    # pass C (the dispatch's scoring kernel alone): direct launches with events
+    # recorded by maps_dispatch right around its scoring kernel
+    for i in range(Kb):
+        flush.zero_()
+        torch.cuda._sleep(sleep_cycles)
+        step.M.maps_set_dispatch_events(evs[i][0], evs[i][1])
+        step.run()
+    step.M.maps_set_dispatch_events(None, None)
     torch.cuda.synchronize()
     clocks = sampler.stop()
     if dist is not None and dist.is_initialized():
@@ -454,6 +473,7 @@ def bench_gpu(args, world, rank, local, dist):
     disp_ms = [evb[i][1].elapsed_time(evb[i][2]) for i in range(Kb)]
     cal_ms = [evb[i][3].elapsed_time(evb[i][0]) for i in range(Kb)]
     order_ms = [evb[i][2].elapsed_time(evb[i][4]) for i in range(Kb)]
+    score_ms = [evs[i][0].elapsed_time(evs[i][1]) for i in range(Kb)]
     local_s = sum(step_ms) / 1e3
     max_s, units = aggregate(local_s, float(K * step.J), dist)
 
@@ -499,6 +519,11 @@ def bench_gpu(args, world, rank, local, dist):
         "order": 20 * (R + J) + 8 * (D + 1),           # four int32 keys in, perm out, segments
     }
     call_ms = {"calibrate": cal_ms, "occupancy": occ_ms, "dispatch": disp_ms, "order": order_ms}
+    # the dispatch's scoring kernel alone: K in, candidates in, choice and
+    # headroom out; the candidate bucketing by horizon tile is left out, as the
+    # kernel roofline of the scoring step is defined
+    alg["dispatch_scoring"] = alg["dispatch"]
+    call_ms["dispatch_scoring"] = score_ms
     rooflines = {}
     for c in alg:
         avg = float(np.mean(call_ms[c])) / 1e3
@@ -546,7 +571,7 @@ def bench_gpu(args, world, rank, local, dist):
                             "results read back on another stream; each stage launched as "
                             f"{how}",
                 "stage_us_alone": stage_us},
-        "gpu_launches": step.kernels_per_step * (K + Kb),  # both passes of the timed region
+        "gpu_launches": step.kernels_per_step * (K + 2 * Kb),  # the three passes of the timed region
         "clocks": clocks,
     }
     return result, w

@@ -70,6 +70,15 @@ int maps_last_cuda_error(void);
  * (MAPS_OK or the first error any kernel recorded in it) and clears it. */
 int maps_check(void *ws, void *stream);
 
+/* Benchmarking aid.  `before` and `after` are CUDA events (cudaEvent_t,
+ * created by the caller, passed as void *).  Every later SNAPSHOT
+ * maps_dispatch call made by this thread records them on its stream right
+ * before and right after its scoring kernel (after the candidates have been
+ * bucketed by horizon tile), so a caller can time the scoring kernel alone.
+ * An event between two launches costs the programmatic overlap there.
+ * NULL, NULL turns it off.  Results are unaffected.  Returns MAPS_OK. */
+int maps_set_dispatch_events(void *before, void *after);
+
 /* ------------------------------------------------------------------------
  * Uncertainty-aware calibration, Sec. 3.2.
  *

@@ -1120,13 +1120,19 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 
 constexpr int kMaxH = 1 << 28;
 
+// Events recorded around the scoring kernel (maps_set_dispatch_events).
+thread_local cudaEvent_t g_score_ev[2] = {nullptr, nullptr};
+
 template <int W2>
 int run_snapshot(int64_t grid, size_t smem, cudaStream_t s, const CUtensorMap &tmap, const SnapArgs &a) {
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(dispatch_snapshot_kernel<W2>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));
+  if (g_score_ev[0]) MAPS_TRY(cuda_ok(cudaEventRecord(g_score_ev[0], s)));
   launch_pdl(dispatch_snapshot_kernel<W2>, static_cast<unsigned>(grid), kMainThreads, smem, s, tmap, a);
-  return launch_ok();
+  MAPS_TRY(launch_ok());
+  if (g_score_ev[1]) MAPS_TRY(cuda_ok(cudaEventRecord(g_score_ev[1], s)));
+  return MAPS_OK;
 }
 
 int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const int32_t *cap,
@@ -1213,6 +1219,12 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
 }  // namespace maps
 
 extern "C" {
+
+int maps_set_dispatch_events(void *before, void *after) {
+  maps::g_score_ev[0] = static_cast<cudaEvent_t>(before);
+  maps::g_score_ev[1] = static_cast<cudaEvent_t>(after);
+  return MAPS_OK;
+}
 
 size_t maps_dispatch_workspace_size(int32_t mode, int32_t D, int32_t H, int64_t J) {
   using namespace maps;

@@ -58,6 +58,7 @@ def _load():
         "maps_version": ([], ctypes.c_int),
         "maps_last_cuda_error": ([], ctypes.c_int),
         "maps_check": ([vp, vp], ctypes.c_int),
+        "maps_set_dispatch_events": ([vp, vp], ctypes.c_int),
         "maps_calibrate_workspace_size": ([i64, i64], sz),
         "maps_calibrate": ([vp, vp, i64, u32, vp, i64, vp, vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_project_occupancy_workspace_size": ([i32, i32, i64], sz),
@@ -80,7 +81,7 @@ def _load():
 
 
 lib = _load()
-EXPORTS = ("maps_version", "maps_last_cuda_error", "maps_check",
+EXPORTS = ("maps_version", "maps_last_cuda_error", "maps_check", "maps_set_dispatch_events",
            "maps_calibrate_workspace_size", "maps_calibrate",
            "maps_project_occupancy_workspace_size", "maps_project_occupancy",
            "maps_dispatch_workspace_size", "maps_dispatch",
@@ -128,6 +129,15 @@ class Workspace:
 
 def maps_check(ws: Workspace, stream=None) -> int:
     return lib.maps_check(ws.ptr, _stream(stream))
+
+
+def maps_set_dispatch_events(before=None, after=None) -> int:
+    """Benchmarking aid: torch.cuda.Event objects that later SNAPSHOT
+    maps_dispatch calls of this thread record around their scoring kernel
+    (None, None turns it off).  The events must already exist on the device:
+    record each once first."""
+    h = lambda e: None if e is None else ctypes.c_void_p(e.cuda_event)  # noqa: E731
+    return lib.maps_set_dispatch_events(h(before), h(after))
 
 
 def maps_calibrate(true_len, pred_len, alpha_ppm: int, query_pred=None, bound_out=None,

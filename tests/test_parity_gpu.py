@@ -525,6 +525,30 @@ def test_order_workload_pipeline(M, ws, oracle, name, one_queue):
     assert np.array_equal(perm, po) and np.array_equal(seg, so)
 
 
+def test_dispatch_scoring_events(M, ws, oracle):
+    """The benchmarking hook records its events around the scoring kernel and
+    leaves the decisions unchanged."""
+    w = W.make("tiny", feasible=True)
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    cb = oracle.bound(w["cand_pred"], q)[1]
+    _, K = oracle.occupancy(w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    e1.record()
+    assert M.maps_set_dispatch_events(e0, e1) == 0
+    try:
+        st, ch, hr, _, _ = gpu_dispatch(M, ws, 0, w["D"], w["H"], 1, K, w["cap"], w["Q"],
+                                        w["cand_prompt"], cb)
+    finally:
+        M.maps_set_dispatch_events(None, None)
+    torch.cuda.synchronize()
+    _, cho, hro, _, _ = oracle.dispatch(0, w["D"], w["H"], 1, K, w["cap"], w["Q"],
+                                        w["cand_prompt"], cb)
+    assert st == 0 and np.array_equal(ch, cho) and np.array_equal(hr, hro)
+    assert e0.elapsed_time(e1) > 0.0
+
+
 # ---------------------------------------------------------------------------
 # CUDA graph capture of the whole pass
 # ---------------------------------------------------------------------------
