@@ -474,6 +474,9 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   long long *s_maxA = reinterpret_cast<long long *>(
       (reinterpret_cast<uintptr_t>(s_argA + W2) + 15) & ~uintptr_t(15));  // [W2]
   uint64_t *s_bar = reinterpret_cast<uint64_t *>(s_maxA + W2);
+  long long *s_segA = reinterpret_cast<long long *>(s_bar + 1);      // [8][32]
+  int32_t *s_segrun = reinterpret_cast<int32_t *>(s_segA + kWarpsM * 32);  // [8][32]
+  int32_t *s_segK = s_segrun + kWarpsM * 32;                          // [8][32]
   __shared__ int s_nslots, s_abort;
 
   const Unit un = a.units[unit];
@@ -617,49 +620,63 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   __syncthreads();
 
   // --- per needed column: prefix max of A in queue order, arg-max of A -----
-  const int P = (D + 31) / 32;  // strided queue positions per lane
-  for (int sl = warp; sl < nslots; sl += kWarpsM) {
-    uint32_t *col = comp + static_cast<size_t>(sl) * Dp;
-    int32_t carryq = -1;
-    long long bestA = LLONG_MIN;
-    int bestK = 0x7fffffff;
-    for (int s = 0; s < P; ++s) {
-      const int i = s * 32 + lane;
-      int32_t a32 = -1;
-      if (i < D) {
-        const long long A = static_cast<long long>(s_capq[i]) - 1 - static_cast<long long>(col[i]);
-        a32 = A < -1 ? -1 : static_cast<int32_t>(A);
-        const int k = s_sig[i];
-        if (A > bestA || (A == bestA && k < bestK)) {
-          bestA = A;
-          bestK = k;
+  // Columns go 32 at a time, lane c taking column cb + c; warp w takes the
+  // w-th eighth of the queue positions, in order: a running maximum of A
+  // (clamped at -1) written in place, and the segment's maximum and best
+  // (A, decoder) kept.  After a barrier each segment raises its entries to
+  // the maximum of the segments before it, and warp 0 combines the best
+  // (A, decoder) of the eight.  Rows are D + 1 words apart, so a warp's 32
+  // columns fall on 32 banks.
+  {
+    const int L = (D + kWarpsM - 1) / kWarpsM;
+    const int i0 = warp * L, i1 = min(D, i0 + L);
+    for (int cb = 0; cb < nslots; cb += 32) {
+      const int sl = cb + lane;
+      const bool live = sl < nslots;
+      uint32_t *col = comp + static_cast<size_t>(live ? sl : 0) * Dp;
+      int32_t run = -1;
+      long long bA = LLONG_MIN;
+      int bK = 0x7fffffff;
+      if (live)
+        for (int i = i0; i < i1; ++i) {
+          const long long A = static_cast<long long>(s_capq[i]) - 1 - static_cast<long long>(col[i]);
+          const int k = s_sig[i];
+          if (A > bA || (A == bA && k < bK)) {
+            bA = A;
+            bK = k;
+          }
+          const int32_t a32 = A < -1 ? -1 : static_cast<int32_t>(A);
+          run = a32 > run ? a32 : run;
+          col[i] = static_cast<uint32_t>(run);
+        }
+      s_segrun[warp * 32 + lane] = run;
+      s_segA[warp * 32 + lane] = bA;
+      s_segK[warp * 32 + lane] = bK;
+      __syncthreads();
+      if (live) {
+        int32_t ex = -1;
+        for (int w = 0; w < warp; ++w) ex = max(ex, s_segrun[w * 32 + lane]);
+        if (ex > -1)
+          for (int i = i0; i < i1; ++i) {
+            const int32_t v = static_cast<int32_t>(col[i]);
+            if (v < ex) col[i] = static_cast<uint32_t>(ex);
+          }
+        if (warp == 0) {
+          for (int w = 1; w < kWarpsM; ++w) {
+            const long long yA = s_segA[w * 32 + lane];
+            const int yK = s_segK[w * 32 + lane];
+            if (yA > bA || (yA == bA && yK < bK)) {
+              bA = yA;
+              bK = yK;
+            }
+          }
+          s_maxA[sl] = bA;
+          s_argA[sl] = bK;
         }
       }
-      int32_t x = a32;
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const int32_t y = __shfl_up_sync(0xffffffffu, x, off);
-        if (lane >= off) x = y > x ? y : x;
-      }
-      x = x > carryq ? x : carryq;
-      if (i < D) col[i] = static_cast<uint32_t>(x);
-      carryq = __shfl_sync(0xffffffffu, x, 31);
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const long long yA = __shfl_xor_sync(0xffffffffu, bestA, off);
-      const int yK = __shfl_xor_sync(0xffffffffu, bestK, off);
-      if (yA > bestA || (yA == bestA && yK < bestK)) {
-        bestA = yA;
-        bestK = yK;
-      }
-    }
-    if (lane == 0) {
-      s_maxA[sl] = bestA;
-      s_argA[sl] = bestK;
+      __syncthreads();  // the segment arrays serve the next 32 columns
     }
   }
-  __syncthreads();
 
   // --- this unit's candidates (loads issued together, then the searches) ----
   for (int q0 = 0; q0 < un.count; q0 += kMainThreads * 8) {
@@ -1069,6 +1086,7 @@ SnapGeom snap_geom(int D, int H) {
   b += 16;                                            // alignment slack
   b += static_cast<size_t>(w) * 8;                    // maxA
   b += 8;                                             // barrier
+  b += static_cast<size_t>(kMainThreads) * (8 + 4 + 4);  // per-segment partials [8][32]
   g.smem = b;
   return g;
 }
