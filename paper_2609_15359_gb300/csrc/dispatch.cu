@@ -436,6 +436,9 @@ bin_scatter_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__
 struct SnapArgs {
   int D, H, W2, T2, Drows, boxes, box_rows;  // Drows = rows per staged tile (>= D)
   int tile_stride;                           // elements of the tile buffer (1 KB multiple)
+  int comp_off;                              // words from the tile buffer to comp
+  int region;                                // words from the tile buffer to the small arrays
+  bool alias;                                // comp overwrites the tile (one row per thread)
   bool use_tma;
   const int32_t *K;
   const int32_t *sig, *rank_of, *capq;  // queue order
@@ -449,7 +452,7 @@ struct SnapArgs {
 };
 
 template <int W2>
-__global__ void __launch_bounds__(kMainThreads, 3)
+__global__ void __launch_bounds__(kMainThreads, 4)
 dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   pdl_prologue();
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -464,8 +467,8 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   // Rows are D + 1 words apart so that one row's writes to several slots fall
   // on different banks.
   const int Dp = D + 1;
-  uint32_t *comp = kb + a.tile_stride;
-  int32_t *s_capq = reinterpret_cast<int32_t *>(comp + static_cast<size_t>(W2) * Dp);
+  uint32_t *comp = kb + a.comp_off;
+  int32_t *s_capq = reinterpret_cast<int32_t *>(kb + a.region);
   int32_t *s_sig = s_capq + D;
   int32_t *s_rank = s_sig + D;
   uint32_t *s_carry = reinterpret_cast<uint32_t *>(s_rank + D);
@@ -548,7 +551,39 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
 
   // --- prefix maximum of K + t along each row; keep the needed columns ----
   bool neg = false;
-  if constexpr (W2 == 32) {
+  if (W2 == 32 && a.alias) {
+    // One row per thread (D <= kMainThreads): every row is read into registers
+    // first, then, after a barrier, comp is written over the tile.
+    const int row = tid;
+    const bool live = row < D;
+    uint4 q[8];
+    if (live) {
+      const uint4 *rp = reinterpret_cast<const uint4 *>(kb + static_cast<size_t>(row) * 32);
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) q[ch] = rp[ch ^ (row & 7)];
+    }
+    __syncthreads();  // the tile has been read: its space becomes comp
+    if (live) {
+      uint32_t run = s_carry[row];
+      const int rk = s_rank[row];
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) {
+        const uint32_t raw[4] = {q[ch].x, q[ch].y, q[ch].z, q[ch].w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int c = ch * 4 + e;
+          const int64_t t = t0 + c;
+          if (t < H) {
+            if (static_cast<int32_t>(raw[e]) < 0) neg = true;
+            const uint32_t x = raw[e] + static_cast<uint32_t>(t);  // K + t < 2^32
+            run = x > run ? x : run;
+          }
+          const int sl = s_slot[c];
+          if (sl >= 0) comp[static_cast<size_t>(sl) * Dp + rk] = run;
+        }
+      }
+    }
+  } else if constexpr (W2 == 32) {
     // One thread per row.  The tile is stored with 128-byte swizzling: the
     // 16-byte chunk ch of row r sits at chunk ch ^ (r & 7) of its 128-byte
     // row, so a warp loading one chunk of 32 rows hits every bank once per
@@ -1065,7 +1100,8 @@ alg1_sequential_kernel(int D, int S, long long *B_eff, const int32_t *cap, int32
 // Host side
 // ---------------------------------------------------------------------------
 struct SnapGeom {
-  int box_rows, boxes, Drows, W2, T2, tile_stride;
+  int box_rows, boxes, Drows, W2, T2, tile_stride, comp_off, region;
+  bool alias;
   size_t smem;
 };
 
@@ -1079,8 +1115,13 @@ SnapGeom snap_geom(int D, int H) {
   g.W2 = w;
   g.T2 = static_cast<int>((static_cast<long long>(H) + w - 1) / w);
   g.tile_stride = (g.Drows * w + 255) / 256 * 256;  // 1 KB-aligned buffer
-  size_t b = static_cast<size_t>(g.tile_stride) * 4;  // K tile
-  b += static_cast<size_t>(D + 1) * w * 4;            // comp / prefix maxima (padded rows)
+  // with 32-column tiles and at most one row per thread, comp (the prefix
+  // maxima, padded rows) overwrites the tile once every row is in registers
+  const int comp_words = (D + 1) * w;
+  g.alias = w == 32 && D <= kMainThreads;
+  g.comp_off = g.alias ? 0 : g.tile_stride;
+  g.region = g.alias ? std::max(g.tile_stride, comp_words) : g.tile_stride + comp_words;
+  size_t b = static_cast<size_t>(g.region) * 4;       // K tile and comp
   b += 4 * static_cast<size_t>(D) * 4;                // capq, sig, rank, carry
   b += 2 * static_cast<size_t>(w) * 4;                // slot, argA
   b += 16;                                            // alignment slack
@@ -1209,6 +1250,9 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
   a.boxes = g.boxes;
   a.box_rows = g.box_rows;
   a.tile_stride = g.tile_stride;
+  a.comp_off = g.comp_off;
+  a.region = g.region;
+  a.alias = g.alias;
   a.use_tma = use_tma;
   a.K = K;
   a.sig = w.sig;
