@@ -480,7 +480,9 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   long long *s_segA = reinterpret_cast<long long *>(s_bar + 1);      // [8][32]
   int32_t *s_segrun = reinterpret_cast<int32_t *>(s_segA + kWarpsM * 32);  // [8][32]
   int32_t *s_segK = s_segrun + kWarpsM * 32;                          // [8][32]
-  __shared__ int s_nslots, s_abort;
+  int32_t *s_need = s_segK + kWarpsM * 32;                            // [W2] column needs PMq
+  int32_t *s_needlist = s_need + W2;                                  // [W2]
+  __shared__ int s_nslots, s_abort, s_nneed;
 
   const Unit un = a.units[unit];
   const int64_t t0 = static_cast<int64_t>(un.tile) * W2;
@@ -654,22 +656,20 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   if (neg) flag_error(a.status, MAPS_E_RANGE);
   __syncthreads();
 
-  // --- per needed column: prefix max of A in queue order, arg-max of A -----
+  // --- per needed column: arg-max of A, then (where some candidate can be
+  // placed) the prefix maximum of A in queue order ---------------------------
   // Columns go 32 at a time, lane c taking column cb + c; warp w takes the
-  // w-th eighth of the queue positions, in order: a running maximum of A
-  // (clamped at -1) written in place, and the segment's maximum and best
-  // (A, decoder) kept.  After a barrier each segment raises its entries to
-  // the maximum of the segments before it, and warp 0 combines the best
-  // (A, decoder) of the eight.  Rows are D + 1 words apart, so a warp's 32
-  // columns fall on 32 banks.
+  // w-th eighth of the queue positions, in order.  Rows are D + 1 words apart,
+  // so a warp's 32 columns fall on 32 banks.
   {
     const int L = (D + kWarpsM - 1) / kWarpsM;
     const int i0 = warp * L, i1 = min(D, i0 + L);
+    // (1) the best (A, decoder) of each column: each segment's, then warp 0
+    // combines the eight
     for (int cb = 0; cb < nslots; cb += 32) {
       const int sl = cb + lane;
       const bool live = sl < nslots;
-      uint32_t *col = comp + static_cast<size_t>(live ? sl : 0) * Dp;
-      int32_t run = -1;
+      const uint32_t *col = comp + static_cast<size_t>(live ? sl : 0) * Dp;
       long long bA = LLONG_MIN;
       int bK = 0x7fffffff;
       if (live)
@@ -680,13 +680,68 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
             bA = A;
             bK = k;
           }
+        }
+      s_segA[warp * 32 + lane] = bA;
+      s_segK[warp * 32 + lane] = bK;
+      __syncthreads();
+      if (live && warp == 0) {
+        for (int w = 1; w < kWarpsM; ++w) {
+          const long long yA = s_segA[w * 32 + lane];
+          const int yK = s_segK[w * 32 + lane];
+          if (yA > bA || (yA == bA && yK < bK)) {
+            bA = yA;
+            bK = yK;
+          }
+        }
+        s_maxA[sl] = bA;
+        s_argA[sl] = bK;
+        s_need[sl] = 0;
+      }
+      __syncthreads();  // the segment arrays serve the next 32 columns
+    }
+    // (2) a candidate that fits no decoder (p above its column's best A) is
+    // decided here (most headroom); the others mark their column
+    for (int q = tid; q < un.count; q += kMainThreads) {
+      const int32_t p = __ldg(a.sp + un.start + q);
+      const int sl = s_slot[__ldg(a.su + un.start + q) - 1 - t0];
+      if (static_cast<long long>(p) <= s_maxA[sl]) {
+        s_need[sl] = 1;
+      } else {
+        const int j = __ldg(a.ord + un.start + q);
+        a.choice[j] = s_argA[sl];
+        if (a.headroom) a.headroom[j] = s_maxA[sl] - p;
+      }
+    }
+    __syncthreads();
+    if (warp == 0) {  // compact them
+      int run = 0;
+      for (int c0 = 0; c0 < nslots; c0 += 32) {
+        const int sl = c0 + lane;
+        const bool f = sl < nslots && s_need[sl] != 0;
+        const unsigned bal = __ballot_sync(0xffffffffu, f);
+        if (f) s_needlist[run + __popc(bal & lanemask_lt())] = sl;
+        run += __popc(bal);
+      }
+      if (lane == 0) s_nneed = run;
+    }
+    __syncthreads();
+    // (3) for those: a running maximum of A (clamped at -1) per segment,
+    // written in place, then each segment raised to the maximum of the
+    // segments before it
+    const int nneed = s_nneed;
+    for (int cb = 0; cb < nneed; cb += 32) {
+      const bool live = cb + lane < nneed;
+      const int sl = live ? s_needlist[cb + lane] : 0;
+      uint32_t *col = comp + static_cast<size_t>(sl) * Dp;
+      int32_t run = -1;
+      if (live)
+        for (int i = i0; i < i1; ++i) {
+          const long long A = static_cast<long long>(s_capq[i]) - 1 - static_cast<long long>(col[i]);
           const int32_t a32 = A < -1 ? -1 : static_cast<int32_t>(A);
           run = a32 > run ? a32 : run;
           col[i] = static_cast<uint32_t>(run);
         }
       s_segrun[warp * 32 + lane] = run;
-      s_segA[warp * 32 + lane] = bA;
-      s_segK[warp * 32 + lane] = bK;
       __syncthreads();
       if (live) {
         int32_t ex = -1;
@@ -696,25 +751,14 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
             const int32_t v = static_cast<int32_t>(col[i]);
             if (v < ex) col[i] = static_cast<uint32_t>(ex);
           }
-        if (warp == 0) {
-          for (int w = 1; w < kWarpsM; ++w) {
-            const long long yA = s_segA[w * 32 + lane];
-            const int yK = s_segK[w * 32 + lane];
-            if (yA > bA || (yA == bA && yK < bK)) {
-              bA = yA;
-              bK = yK;
-            }
-          }
-          s_maxA[sl] = bA;
-          s_argA[sl] = bK;
-        }
       }
-      __syncthreads();  // the segment arrays serve the next 32 columns
+      __syncthreads();
     }
   }
 
-  // --- this unit's candidates (loads issued together, then the searches) ----
-  for (int q0 = 0; q0 < un.count; q0 += kMainThreads * 8) {
+  // --- the candidates that fit some decoder (loads issued together, then the
+  // searches); the others were decided above ----------------------------------
+  for (int q0 = 0; s_nneed > 0 && q0 < un.count; q0 += kMainThreads * 8) {
     int32_t pp[8], uu[8], jj[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
@@ -730,26 +774,18 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
       const int32_t p = pp[i];
       const int c = static_cast<int>(uu[i] - 1 - t0);
       const int sl = s_slot[c];
+      if (s_maxA[sl] < p) continue;  // nothing feasible: decided above
       const int32_t *pm = reinterpret_cast<const int32_t *>(comp) + static_cast<size_t>(sl) * Dp;
-      int k;
-      long long h;
-      if (pm[D - 1] < p) {
-        k = s_argA[sl];  // nothing feasible: most headroom
-        h = s_maxA[sl] - p;
-      } else {
-        int l = 0, r = D - 1;  // first queue position whose prefix reaches p
-        while (l < r) {
-          const int mid = (l + r) >> 1;
-          if (pm[mid] >= p)
-            r = mid;
-          else
-            l = mid + 1;
-        }
-        k = s_sig[l];
-        h = static_cast<long long>(pm[l]) - p;
+      int l = 0, r = D - 1;  // first queue position whose prefix reaches p
+      while (l < r) {
+        const int mid = (l + r) >> 1;
+        if (pm[mid] >= p)
+          r = mid;
+        else
+          l = mid + 1;
       }
-      a.choice[jj[i]] = k;
-      if (a.headroom) a.headroom[jj[i]] = h;
+      a.choice[jj[i]] = s_sig[l];
+      if (a.headroom) a.headroom[jj[i]] = static_cast<long long>(pm[l]) - p;
     }
   }
 }
@@ -1128,6 +1164,7 @@ SnapGeom snap_geom(int D, int H) {
   b += static_cast<size_t>(w) * 8;                    // maxA
   b += 8;                                             // barrier
   b += static_cast<size_t>(kMainThreads) * (8 + 4 + 4);  // per-segment partials [8][32]
+  b += 2 * static_cast<size_t>(w) * 4;                    // columns needing PMq, their list
   g.smem = b;
   return g;
 }
