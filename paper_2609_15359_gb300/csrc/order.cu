@@ -60,6 +60,8 @@ struct OrderCounts {
   uint32_t max_levels; // merge levels the longest queue needs
   uint32_t done_blocks;  // prep blocks finished
   uint32_t stable;     // segmented form with the decoder scatter in index order
+  uint32_t npairs;     // run pairs reserved by the pairwise-ranked long queues
+  uint32_t npairq;     // pairwise-ranked long queues
 };
 
 // Segmented form: when arrival is non-decreasing along the index (so arrival
@@ -92,6 +94,25 @@ constexpr int kSegMax = kSegThreads * kSegIPT;  // entries one block sorts
 constexpr int kMergeTile = 512;
 constexpr int kMergeThreads = 512;  // the finishing kernel's block
 static_assert(kSegMax % kMergeTile == 0, "merge tiles align with runs");
+
+// A long queue of at most kPairRuns chunks is ranked pairwise instead: for
+// every ordered pair of its sorted runs (A, B) one block counts, for each key
+// of A, the keys of B below it (the keys are unique); after one grid barrier
+// a key's place in the queue is its place in A plus those counts.  The counts
+// are 16-bit, [pair][position in A]; the pairs a call may use are capped by
+// pair_budget(N), and a queue past the cap or past kPairRuns is merged.
+constexpr int kPairRuns = 16;
+__host__ __device__ __forceinline__ int64_t pair_budget(int64_t N) {
+  const int64_t b = 4 * (N / kSegMax);
+  return b < 1024 ? b : 1024;
+}
+struct PairQueues {
+  int64_t *off;    // [queue] first slot of the queue
+  int32_t *n;      // [queue] entries
+  int32_t *pair0;  // [queue] first pair id
+  uint16_t *cnt;   // [pair][kSegMax] keys of B below each key of A
+  int64_t budget;  // pairs the workspace holds
+};
 
 // Merge levels a queue of n entries needs: ceil(log2(ceil(n / kSegMax))).
 __host__ __device__ __forceinline__ int merge_levels(int64_t n) {
@@ -141,7 +162,7 @@ __device__ __forceinline__ int bit_width(uint32_t x) { return x ? 32 - __clz(x) 
 // in index order.
 __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_count,
                                int64_t *seg_off, int64_t *item_off, int32_t *item_n,
-                               int64_t *mt_off, int32_t *mt_n, int32_t *mt_t) {
+                               int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, PairQueues pq) {
   __shared__ long long s_w[32];
   __shared__ int s_bw[32];
   __shared__ long long s_carry;
@@ -193,13 +214,27 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
         item_off[it + j] = start + static_cast<int64_t>(j) * kSegMax;
         item_n[it + j] = -static_cast<int32_t>(min(static_cast<long long>(kSegMax), c - static_cast<long long>(j) * kSegMax));
       }
-      atomicMax(&counts->max_levels, static_cast<uint32_t>(merge_levels(c)));
-      const int ntl = static_cast<int>((c + kMergeTile - 1) / kMergeTile);
-      const uint32_t mt = atomicAdd(&counts->nmtiles, static_cast<uint32_t>(ntl));
-      for (int j = 0; j < ntl; ++j) {
-        mt_off[mt + j] = start;
-        mt_n[mt + j] = static_cast<int32_t>(c);
-        mt_t[mt + j] = j;
+      bool paired = false;
+      if (nch <= kPairRuns) {  // rank the runs pairwise when the budget allows
+        const uint32_t np2 = static_cast<uint32_t>(nch * (nch - 1));
+        const uint32_t p0 = atomicAdd(&counts->npairs, np2);
+        if (static_cast<int64_t>(p0) + np2 <= pq.budget) {
+          const uint32_t q = atomicAdd(&counts->npairq, 1u);
+          pq.off[q] = start;
+          pq.n[q] = static_cast<int32_t>(c);
+          pq.pair0[q] = static_cast<int32_t>(p0);
+          paired = true;
+        }
+      }
+      if (!paired) {  // pairwise merges, level by level
+        atomicMax(&counts->max_levels, static_cast<uint32_t>(merge_levels(c)));
+        const int ntl = static_cast<int>((c + kMergeTile - 1) / kMergeTile);
+        const uint32_t mt = atomicAdd(&counts->nmtiles, static_cast<uint32_t>(ntl));
+        for (int j = 0; j < ntl; ++j) {
+          mt_off[mt + j] = start;
+          mt_n[mt + j] = static_cast<int32_t>(c);
+          mt_t[mt + j] = j;
+        }
       }
     }
     __syncthreads();
@@ -225,8 +260,8 @@ order_prep_kernel(int64_t N, int D, int64_t chunk, const int32_t *__restrict__ d
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
                   uint32_t *dec_count, int32_t *status, int64_t *seg_off, int64_t *item_off,
-                  int32_t *item_n, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, uint32_t *blk,
-                  uint32_t *grp, int Dp) {
+                  int32_t *item_n, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, PairQueues pq,
+                  uint32_t *blk, uint32_t *grp, int Dp) {
   pdl_prologue();
   __shared__ uint32_t s_dec[kDecSmem];
   __shared__ bool s_last;
@@ -302,7 +337,7 @@ order_prep_kernel(int64_t N, int D, int64_t chunk, const int32_t *__restrict__ d
   __syncthreads();
   if (s_last) {
     __threadfence();
-    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, mt_off, mt_n, mt_t);
+    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, mt_off, mt_n, mt_t, pq);
   }
 }
 
@@ -1011,6 +1046,66 @@ __device__ void merge_level(int level, int ntiles, const int64_t *mt_off, const 
   }
 }
 
+// The pairwise-ranked long queues: pair counts, a grid barrier, then every
+// key to its place.  Runs are the segment sort's sorted chunks in keys.
+__device__ void pair_rank_all(int64_t N, const OrderCounts *counts, const PairQueues &pq,
+                              const unsigned long long *keys, int32_t *perm,
+                              unsigned long long *sB, cg::grid_group &grid) {
+  const int nq = static_cast<int>(counts->npairq);
+  const int64_t npairs = min(static_cast<int64_t>(counts->npairs), pq.budget);
+  // (1) pair p = (queue q, runs A != B): for each key of A, the keys of B below it
+  for (int64_t p = blockIdx.x; p < npairs; p += gridDim.x) {
+    int q = -1;
+    for (int i = 0; i < nq; ++i) {  // the queue holding pair p (few queues)
+      const int C = static_cast<int>((pq.n[i] + kSegMax - 1) / kSegMax);
+      if (p >= pq.pair0[i] && p < pq.pair0[i] + static_cast<int64_t>(C) * (C - 1)) q = i;
+    }
+    if (q < 0) continue;  // a reservation no queue kept (uniform per block)
+    const int64_t off = pq.off[q];
+    const int n = pq.n[q], C = (n + kSegMax - 1) / kSegMax;
+    const int l = static_cast<int>(p - pq.pair0[q]);
+    const int A = l / (C - 1), b = l % (C - 1), B = b < A ? b : b + 1;
+    const int nA = min(kSegMax, n - A * kSegMax), nB = min(kSegMax, n - B * kSegMax);
+    const unsigned long long *rA = keys + off + static_cast<int64_t>(A) * kSegMax;
+    const unsigned long long *rB = keys + off + static_cast<int64_t>(B) * kSegMax;
+    for (int x = threadIdx.x; x < nB; x += blockDim.x) sB[x] = rB[x];
+    __syncthreads();
+    uint16_t *out = pq.cnt + p * kSegMax;
+    for (int x = threadIdx.x; x < nA; x += blockDim.x) {
+      const unsigned long long key = rA[x];
+      int lo = 0, hi = nB;  // keys of B below key
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (sB[mid] < key)
+          lo = mid + 1;
+        else
+          hi = mid;
+      }
+      out[x] = static_cast<uint16_t>(lo);
+    }
+    __syncthreads();  // sB serves the next pair
+  }
+  grid.sync();
+  // (2) each key's place: its place in its run plus its counts in the others
+  const unsigned long long imask = (1ull << index_bits(N)) - 1;
+  const int64_t gstride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int q = 0; q < nq; ++q) {
+    const int64_t off = pq.off[q];
+    const int n = pq.n[q], C = (n + kSegMax - 1) / kSegMax;
+    const int64_t pair0 = pq.pair0[q];
+    for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < n; e += gstride) {
+      const int A = static_cast<int>(e / kSegMax), x = static_cast<int>(e - static_cast<int64_t>(A) * kSegMax);
+      int64_t pos = x;
+      for (int B = 0; B < C; ++B) {
+        if (B == A) continue;
+        const int64_t pid = pair0 + static_cast<int64_t>(A) * (C - 1) + (B < A ? B : B - 1);
+        pos += pq.cnt[pid * kSegMax + x];
+      }
+      perm[off + pos] = static_cast<int32_t>(keys[off + e] & imask);
+    }
+  }
+}
+
 __device__ void merge_all(int64_t N, const OrderCounts *counts, const int64_t *mt_off,
                           const int32_t *mt_n, const int32_t *mt_t, unsigned long long *bufA,
                           unsigned long long *bufB, int32_t *perm, cg::grid_group &grid) {
@@ -1203,13 +1298,17 @@ __global__ void __launch_bounds__(kPassThreads, 2)
 order_finish_kernel(int n_hi, int64_t N, int D, int dbits, const OrderCounts *counts,
                     OrderPlan *plan, const uint32_t *dec_count, int64_t *seg_off,
                     const int64_t *mt_off, const int32_t *mt_n, const int32_t *mt_t,
-                    unsigned long long *keyA, unsigned long long *keyB, uint32_t *valA,
+                    PairQueues pq, unsigned long long *keyA, unsigned long long *keyB, uint32_t *valA,
                     uint32_t *valB, const unsigned long long *hi_orig, int32_t *perm,
                     unsigned long long *state, int64_t tiles, uint32_t *tickets, int32_t *status) {
   pdl_prologue();
   cg::grid_group grid = cg::this_grid();
   // every block takes the same branches, so no block waits at a barrier alone
   if (*reinterpret_cast<const volatile uint32_t *>(&counts->segmented)) {
+    if (counts->npairq > 0) {
+      extern __shared__ __align__(16) unsigned char pair_raw[];
+      pair_rank_all(N, counts, pq, keyA, perm, reinterpret_cast<unsigned long long *>(pair_raw), grid);
+    }
     if (counts->nmtiles > 0) merge_all(N, counts, mt_off, mt_n, mt_t, keyA, keyB, perm, grid);
     return;
   }
@@ -1258,6 +1357,9 @@ order_finish_kernel(int n_hi, int64_t N, int D, int dbits, const OrderCounts *co
     for (int64_t i = first; i < N; i += stride) perm[i] = static_cast<int32_t>(i);
 }
 
+static_assert(sizeof(PassSmem) >= kSegMax * sizeof(unsigned long long),
+              "one sorted run fits the finishing kernel's shared memory");
+
 // Blocks of the finishing kernel that can be resident at once (its grid limit
 // as a cooperative launch).
 int64_t finish_grid(size_t smem) {
@@ -1282,6 +1384,7 @@ struct OrderWs {
   int64_t *mt_off;    // merge tiles of the long queues
   int32_t *mt_n, *mt_t;
   int64_t nitems_max, ntiles_max;
+  PairQueues pq;      // pairwise-ranked long queues
   unsigned long long *hi_orig, *keyA, *keyB;
   uint32_t *valA, *valB;
   uint32_t *blk;      // stable scatter: [blocks][Dp] counts per prep block
@@ -1313,6 +1416,12 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.mt_off = c.take<int64_t>(static_cast<size_t>(w.ntiles_max));
   w.mt_n = c.take<int32_t>(static_cast<size_t>(w.ntiles_max));
   w.mt_t = c.take<int32_t>(static_cast<size_t>(w.ntiles_max));
+  w.pq.budget = pair_budget(N);
+  const size_t nq_max = static_cast<size_t>(w.pq.budget / 2 + 1);  // a queue has >= 2 pairs
+  w.pq.off = c.take<int64_t>(nq_max);
+  w.pq.n = c.take<int32_t>(nq_max);
+  w.pq.pair0 = c.take<int32_t>(nq_max);
+  w.pq.cnt = c.take<uint16_t>(static_cast<size_t>(w.pq.budget) * kSegMax + 1);
   const size_t n = static_cast<size_t>(N > 0 ? N : 1);
   w.hi_orig = c.take<unsigned long long>(n);
   w.keyA = c.take<unsigned long long>(n);
@@ -1368,7 +1477,7 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   if (N > 0) {
     launch_pdl(order_prep_kernel, w.blocks, 512, 0, s, N, D, w.chunk, dec, bound, wait, arrival,
                max_wait, w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n,
-               w.mt_off, w.mt_n, w.mt_t, w.blk, w.grp, w.Dp);
+               w.mt_off, w.mt_n, w.mt_t, w.pq, w.blk, w.grp, w.Dp);
     // the stable scatter's per-warp counts and running slots
     const size_t keys_smem =
         D <= kStableD ? sizeof(uint32_t) * static_cast<size_t>(kPassWarps + 1) * w.Dp : 0;
@@ -1399,7 +1508,7 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   // the global passes take tiles by ticket, so any resident grid completes them
   MAPS_TRY(launch_coop(order_finish_kernel, std::min<int64_t>(tiles, finish_grid(smem)),
                        kPassThreads, smem, s, n_hi, N, D, dbits, w.counts, w.plan, w.dec_count,
-                       seg_off_out, w.mt_off, w.mt_n, w.mt_t, w.keyA, w.keyB, w.valA, w.valB,
+                       seg_off_out, w.mt_off, w.mt_n, w.mt_t, w.pq, w.keyA, w.keyB, w.valA, w.valB,
                        w.hi_orig, perm_out, w.state, tiles, w.tickets, status));
   return launch_ok();
 }
