@@ -59,6 +59,7 @@ extern "C" {
 #define MAPS_MODE_SEQUENTIAL 1
 #define MAPS_MODE_ALG1_SNAPSHOT 2
 #define MAPS_MODE_ALG1_SEQUENTIAL 3
+#define MAPS_MODE_SNAPSHOT_BINNED 4  /* SNAPSHOT of candidates bucketed by maps_dispatch_bin */
 
 /* Library version, major*10000 + minor*100 + patch. */
 int maps_version(void);
@@ -163,7 +164,8 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
  * ALG1_SEQUENTIAL subtracts B_need from B_eff[k*] and adds 1 to Q[k*] after
  * each choice.  K is not read in the ALG1 modes.
  *
- *   mode                MAPS_MODE_*.
+ *   mode                MAPS_MODE_* (MAPS_MODE_SNAPSHOT_BINNED: see
+ *                       maps_dispatch_bin below).
  *   D, H, S             decoders (1 <= D <= 1024), horizon (1 <= H <= 2^28),
  *                       block size (ALG1).
  *   K                   [D][H] int32 occupancy (horizon modes; updated in
@@ -185,6 +187,21 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
  * ---------------------------------------------------------------------- */
 size_t maps_dispatch_workspace_size(int32_t mode, int32_t D, int32_t H,
                                     int64_t J);
+
+/* SNAPSHOT in two calls.  The candidates' bucketing by horizon tile depends
+ * on the candidates alone, not on K, so a caller may issue it earlier (for
+ * instance on a second stream while maps_project_occupancy computes K):
+ * maps_dispatch_bin buckets them into `ws` (a SNAPSHOT workspace for D, H, J)
+ * and writes choice_out = -1, headroom_out = 0 for candidates with a negative
+ * prompt or bound (MAPS_E_RANGE, as in SNAPSHOT).  A later maps_dispatch with
+ * mode MAPS_MODE_SNAPSHOT_BINNED, the same D, H, J, candidates, outputs and
+ * workspace, and no other call on that workspace in between, then scores them
+ * and gives the SNAPSHOT result.  If the workspace holds no buckets of this
+ * D, H and J, the binned call reads none of them and records MAPS_E_INVALID
+ * (read with maps_check).  Returns MAPS_OK or a host-detected error. */
+int maps_dispatch_bin(int32_t D, int32_t H, int64_t J, const int32_t *cand_prompt,
+                      const int32_t *cand_bound, int32_t *choice_out,
+                      int64_t *headroom_out, void *ws, size_t ws_bytes, void *stream);
 int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K,
                   const uint32_t *kmax, const int32_t *cap, int32_t *Q,
                   const int64_t *res_off,

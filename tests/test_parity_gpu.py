@@ -525,6 +525,52 @@ def test_order_workload_pipeline(M, ws, oracle, name, one_queue):
     assert np.array_equal(perm, po) and np.array_equal(seg, so)
 
 
+@pytest.mark.parametrize("name,feasible", [("tiny", True), ("tiny", False), ("d16", True),
+                                           ("d16", False)])
+def test_dispatch_binned(M, oracle, name, feasible):
+    """maps_dispatch_bin, then the binned SNAPSHOT on the same workspace, equals
+    SNAPSHOT."""
+    w = W.make(name, feasible=feasible)
+    D, H = w["D"], w["H"]
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    cb = oracle.bound(w["cand_pred"], q)[1]
+    _, K = oracle.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U)
+    J = len(cb)
+    dws = M.Workspace(M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, D, H, J),
+                      torch.device("cuda"))
+    cp_d, cb_d = dev(w["cand_prompt"], np.int32), dev(cb, np.int32)
+    ch = torch.full((J,), -9, dtype=torch.int32, device="cuda")
+    hr = torch.full((J,), -9, dtype=torch.int64, device="cuda")
+    assert M.maps_dispatch_bin(D, H, cp_d, cb_d, ch, hr, ws=dws) == 0
+    st = M.maps_dispatch(M.MODE_SNAPSHOT_BINNED, D, H, 1, dev(K, np.int32), dev(w["cap"], np.int32),
+                         dev(w["Q"], np.int32), cp_d, cb_d, ch, hr, ws=dws)
+    assert st == 0 and M.maps_check(dws) == 0
+    _, cho, hro, _, _ = oracle.dispatch(0, D, H, 1, K, w["cap"], w["Q"], w["cand_prompt"], cb)
+    assert np.array_equal(host(ch), cho) and np.array_equal(host(hr), hro)
+
+
+def test_dispatch_binned_without_buckets(M):
+    """A binned call on a workspace that holds no buckets of its candidates reads
+    none of them and records MAPS_E_INVALID."""
+    D, H, J = 8, 4096, 300
+    dws = M.Workspace(M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, D, H, J),
+                      torch.device("cuda"))
+    rng = np.random.default_rng(3)
+    K = dev(rng.integers(0, 1000, (D, H)), np.int32)
+    cap, Q = dev(np.full(D, 10**6), np.int32), dev(np.zeros(D), np.int32)
+    cp, cb = dev(rng.integers(1, 100, J), np.int32), dev(rng.integers(1, H, J), np.int32)
+    ch = torch.full((J,), -9, dtype=torch.int32, device="cuda")
+    # never bucketed (a zeroed workspace)
+    assert M.maps_dispatch(M.MODE_SNAPSHOT_BINNED, D, H, 1, K, cap, Q, cp, cb, ch, ws=dws) == 0
+    assert M.maps_check(dws) == M.MAPS_E_INVALID
+    assert (host(ch) == -9).all()
+    # bucketed for other candidates (J differs)
+    assert M.maps_dispatch_bin(D, H, cp[:200], cb[:200], ch[:200], ws=dws) == 0
+    assert M.maps_dispatch(M.MODE_SNAPSHOT_BINNED, D, H, 1, K, cap, Q, cp, cb, ch, ws=dws) == 0
+    assert M.maps_check(dws) == M.MAPS_E_INVALID
+
+
 def test_dispatch_scoring_events(M, ws, oracle):
     """The benchmarking hook records its events around the scoring kernel and
     leaves the decisions unchanged."""
