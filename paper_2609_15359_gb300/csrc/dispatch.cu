@@ -10,13 +10,17 @@
 //   * PMq_u[i] = max over the first i+1 decoders in (Q, index) order of
 //     A_k(u): the first position where it reaches p_j is the chosen decoder;
 //   * max_k A_k(u) and its lowest arg-max for the fallback.
-// So K is read exactly once, tile by tile over the horizon, with all D rows of
-// a tile staged in shared memory by one TMA copy; the carry of the prefix
-// maximum across tiles is resolved by decoupled look-back; and each candidate
-// costs a binary search over D instead of D scores.  Candidates are first
-// bucketed by the tile of their last live step so each tile serves its own.
-// Three launches: the carry scan and the bucket counts (independent, one
-// launch), the bucket scatter, the main kernel.
+// So K is read at most once, tile by tile over the horizon (only the tiles
+// holding some candidate's last live step), with all D rows of a tile staged
+// in shared memory by one TMA copy; the carry of the prefix maximum into a
+// tile comes from a per-decoder scan of the 16-step summary; per column the
+// arg-max comes first, a candidate above every A_k is decided at once, and
+// PMq is built only where some candidate fits, each of those then costing a
+// binary search over D instead of D scores.  Candidates are first bucketed by
+// the tile of their last live step so each tile serves its own.  Three
+// launches: the carry scan and the bucket counts (independent, one launch),
+// the bucket scatter, the scoring kernel; or the bucketing alone
+// (maps_dispatch_bin) and later the carry scan and scoring (the binned mode).
 //
 // SEQUENTIAL (reservation after each choice) and the literal Algorithm 1
 // modes are separate kernels below.

@@ -8,14 +8,16 @@
 // Layout of the work.  A decoder's horizon is cut into tiles of W steps.
 //   1. bucket kernel, one CTA per decoder: reads the decoder's residents
 //      once, forms (b, e) and counting-sorts the pairs by the tile that holds
-//      their last live step, into the workspace, with per-tile offsets.  It
-//      also checks the inputs and that K[k][0] = sum of b fits int32.
-//   2. tile kernel, one CTA per (decoder, tile): reads the pairs of its own
-//      tile and of the later tiles (contiguous after the sort).  Its own go
-//      into a shared-memory end-step histogram; the later ones only add to the
-//      tile's carry (count, b-sum), the residents live past the tile.  A
-//      reverse scan of the histogram plus the carry gives every cell's live
-//      count and b-sum, and the tile is written with 128-bit stores.
+//      their last live step, into the workspace, with per-tile offsets and
+//      per-tile carries (count and b-sum of the residents live past the
+//      tile).  It also checks the inputs and that K[k][0] = sum of b fits
+//      int32.
+//   2. tile kernel, one CTA per (decoder, tile), launched tile-major: reads
+//      its carry and the pairs of its own tile.  A tile with few pairs sums
+//      them directly; a denser one bins them into a shared-memory end-step
+//      histogram whose reverse scan, plus the carry, gives every cell's live
+//      count and b-sum.  Cells are written through shared staging rows as
+//      whole 128-byte lines.
 // For horizons of more than kMaxTiles tiles a single-kernel form is used
 // instead, in which every tile CTA streams all of its decoder's residents.
 // Optionally every group of 16 steps also yields kmax[k][t/16] =

@@ -11,14 +11,17 @@
 //     non-promoted entry: promoted entries need no primary key because the
 //     arrival order is already in place and the sort is stable;
 //   * a key of at most 32 bits is sorted as 32 bits, otherwise as 64 bits.
-// Kernels: a prep pass (validation, largest bound, entries per decoder,
-// arrival order check; its last block chooses the form), a key pass, the
-// segment sort, and a cooperative finishing kernel.
+// Small calls (at most kSegMax entries and kSmallOrderD decoders) take one
+// block, order_small_kernel, with the whole order in shared memory.
+// Otherwise the kernels are a prep pass (validation, largest bound, entries
+// per decoder, arrival order check; its last block chooses the form), a key
+// pass, the segment sort, and a cooperative finishing kernel.
 // Segmented form (arrival non-decreasing along the index): the key pass
 // scatters each entry's index to its decoder's segment; one block sorts a
 // segment of at most kSegMax entries in shared memory on (not promoted,
 // primary, index), a unique key, and a longer segment is sorted as chunks of
-// kSegMax whose runs the finishing kernel merges pairwise level by level.
+// kSegMax whose runs the finishing kernel ranks pairwise (up to kPairRuns
+// chunks) or merges pairwise level by level.
 // Otherwise the finishing kernel plans and runs one global sweep per digit:
 // tiles of 4096 keys are ranked stably in shared memory, each tile learns its
 // offsets from earlier tiles by decoupled look-back (one thread per digit

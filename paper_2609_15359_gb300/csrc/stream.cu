@@ -11,8 +11,10 @@
 //      batch (maps_calibrate); an unbounded quantile sends the batch round
 //      robin                                                (stream_rr)
 //   4. group running and waiting requests by decoder      (stream_csr)
-//   5. project occupancy and dispatch the batch SEQUENTIALly with Q = the
-//      waiting counts (maps_project_occupancy, maps_dispatch)
+//   5. dispatch the batch SEQUENTIALly with Q = the waiting counts: a walk
+//      over each decoder's sorted end steps in shared memory (stream_dispatch),
+//      or, where those lists do not fit, maps_project_occupancy and
+//      maps_dispatch
 //   6. the batch joins its decoders' waiting queues        (stream_enqueue)
 //   7. local order of every waiting queue (stream_waitlist, maps_order_local)
 //   8. admission in queue order while used + p + U <= capacity, the first
