@@ -55,16 +55,16 @@ L2_FLUSH_BYTES = 256 << 20
 # kernels, one launch each; dispatch_scoring is the scoring kernel alone),
 # valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 28586410, "source": "calibrate.cu", "source_sha256":
+    "calibrate": {"bytes": 28585841, "source": "calibrate.cu", "source_sha256":
                   "16385f686731a11d81b2c01d813292cfe4b95130e9c4e2af1a78e2a682738e07"},
-    "occupancy": {"bytes": 29676544, "source": "occupancy.cu", "source_sha256":
-                  "66b707f592bb0a8213b6e9f096669a70fc63cfc05bb2a93d1b822468b7656371"},
-    "dispatch": {"bytes": 26433450, "source": "dispatch.cu", "source_sha256":
-                 "bec1efa25018815fd56104d64e90a26d2735a1d668a189f91456d6fca10655ee"},
-    "dispatch_scoring": {"bytes": 21114652, "source": "dispatch.cu", "source_sha256":
-                         "bec1efa25018815fd56104d64e90a26d2735a1d668a189f91456d6fca10655ee"},
-    "order": {"bytes": 41117155, "source": "order.cu", "source_sha256":
-              "47710cf71f15241ffda0f21d330c997d5f56c4eff43e1872756c4a475a55d0ae"},
+    "occupancy": {"bytes": 29742791, "source": "occupancy.cu", "source_sha256":
+                  "fd537e3019c8991f53d529abba17e1a23b2664a7f4477b0936c6a78e22aa0746"},
+    "dispatch": {"bytes": 26431544, "source": "dispatch.cu", "source_sha256":
+                 "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
+    "dispatch_scoring": {"bytes": 21112917, "source": "dispatch.cu", "source_sha256":
+                         "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
+    "order": {"bytes": 41117450, "source": "order.cu", "source_sha256":
+              "2aae9099a88207fe058f683410602dc85706e042756c58459f064ae821ab87da"},
 }
 KERNELS = {
     "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
