@@ -447,6 +447,9 @@ def test_dispatch_errors(M, ws, oracle):
                                                 # entries, then stable passes
                                                 (700, 5, True), (1024, 16, False),
                                                 (1025, 16, True), (3000, 40, False),
+                                                # the one-block form at its decoder limit,
+                                                # then past it
+                                                (2000, 4096, True), (2000, 4097, True),
                                                 # one decoder's queue at, and past, the most a
                                                 # block sorts in shared memory
                                                 (4608, 1, True), (4609, 1, True),
@@ -547,6 +550,32 @@ def test_dispatch_binned(M, oracle, name, feasible):
                          dev(w["Q"], np.int32), cp_d, cb_d, ch, hr, ws=dws)
     assert st == 0 and M.maps_check(dws) == 0
     _, cho, hro, _, _ = oracle.dispatch(0, D, H, 1, K, w["cap"], w["Q"], w["cand_prompt"], cb)
+    assert np.array_equal(host(ch), cho) and np.array_equal(host(hr), hro)
+
+
+def test_dispatch_binned_invalid_candidates(M, oracle):
+    """Candidates with a negative prompt or bound: the bucketing call writes -1 and
+    records MAPS_E_RANGE, as SNAPSHOT does; the others are still decided."""
+    w = W.make("tiny", feasible=True)
+    D, H = w["D"], w["H"]
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    cb = oracle.bound(w["cand_pred"], q)[1].copy()
+    cp = w["cand_prompt"].copy()
+    cp[3], cb[7] = -1, -5
+    _, K = oracle.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U)
+    J = len(cb)
+    dws = M.Workspace(M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, D, H, J),
+                      torch.device("cuda"))
+    ch = torch.full((J,), -9, dtype=torch.int32, device="cuda")
+    hr = torch.full((J,), -9, dtype=torch.int64, device="cuda")
+    cp_d, cb_d = dev(cp, np.int32), dev(cb, np.int32)
+    assert M.maps_dispatch_bin(D, H, cp_d, cb_d, ch, hr, ws=dws) == 0
+    assert M.maps_dispatch(M.MODE_SNAPSHOT_BINNED, D, H, 1, dev(K, np.int32), dev(w["cap"], np.int32),
+                           dev(w["Q"], np.int32), cp_d, cb_d, ch, hr, ws=dws) == 0
+    assert M.maps_check(dws) == M.MAPS_E_RANGE
+    sto, cho, hro, _, _ = oracle.dispatch(0, D, H, 1, K, w["cap"], w["Q"], cp, cb)
+    assert sto == M.MAPS_E_RANGE
     assert np.array_equal(host(ch), cho) and np.array_equal(host(hr), hro)
 
 
