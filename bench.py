@@ -55,15 +55,15 @@ L2_FLUSH_BYTES = 256 << 20
 # kernels, one launch each; dispatch_scoring is the scoring kernel alone),
 # valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 28585841, "source": "calibrate.cu", "source_sha256":
-                  "16385f686731a11d81b2c01d813292cfe4b95130e9c4e2af1a78e2a682738e07"},
-    "occupancy": {"bytes": 29742791, "source": "occupancy.cu", "source_sha256":
+    "calibrate": {"bytes": 12580892, "source": "calibrate.cu", "source_sha256":
+                  "2f8167c0989dce1257fabfa3dbf11839b4df88b68af313fa12b2e3614f92179e"},
+    "occupancy": {"bytes": 29785344, "source": "occupancy.cu", "source_sha256":
                   "fd537e3019c8991f53d529abba17e1a23b2664a7f4477b0936c6a78e22aa0746"},
-    "dispatch": {"bytes": 26431544, "source": "dispatch.cu", "source_sha256":
+    "dispatch": {"bytes": 26432142, "source": "dispatch.cu", "source_sha256":
                  "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
-    "dispatch_scoring": {"bytes": 21112917, "source": "dispatch.cu", "source_sha256":
+    "dispatch_scoring": {"bytes": 21113656, "source": "dispatch.cu", "source_sha256":
                          "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
-    "order": {"bytes": 41117450, "source": "order.cu", "source_sha256":
+    "order": {"bytes": 41116672, "source": "order.cu", "source_sha256":
               "2aae9099a88207fe058f683410602dc85706e042756c58459f064ae821ab87da"},
 }
 KERNELS = {

@@ -2,33 +2,36 @@
 //
 // q is the k-th smallest one-sided score s_i = max(0, L_i - Lhat_i) with
 // k = ceil((1 - alpha)(n + 1)).  The scores are unsigned 32-bit (the
-// difference of two int32 values clamped at 0 fits), so q is found by a
-// most-significant-digit radix select over three digits (11, 11, 10 bits):
-// each pass histograms the digit of the scores whose higher digits match the
-// prefix chosen so far, and the last block to finish the pass picks the
-// digit bin that holds rank k.  Nothing returns to the host between passes.
+// difference of two int32 values clamped at 0 fits), so q is found by a radix
+// select whose passes narrow a range [lo, lo + 2^w) known to hold rank k:
+//   - the first pass histograms a monotone bucket of every score: scores below
+//     1,024 have a bin each, larger ones a bin per (leading-bit position, next
+//     7 bits), so a bin covers 1 value below 1,024 and 2^(e-7) values at
+//     leading bit e;
+//   - each later pass histograms the next (up to) 12 bits of s - lo for the
+//     scores inside the range.
+// A range of one value is q, so a quantile below 1,024 takes one pass and any
+// quantile at most three.  The last block to finish a pass picks the bin that
+// holds rank k; passes after the range has closed return at once.  Nothing
+// returns to the host between passes.
 #include "maps_internal.cuh"
 
 namespace maps {
 namespace {
 
-constexpr int kBins = 2048;
+constexpr int kBins = 4096;
 constexpr int kPasses = 3;
 constexpr int kSelectThreads = 256;
-
-template <int PASS>
-struct Digit;
-template <>
-struct Digit<0> { static constexpr int shift = 21, bits = 11; };
-template <>
-struct Digit<1> { static constexpr int shift = 10, bits = 11; };
-template <>
-struct Digit<2> { static constexpr int shift = 0, bits = 10; };
+constexpr uint32_t kExactBins = 1024;  // scores below this have a bin each
+constexpr int kMantBits = 7;           // bits after the leading one, first pass
+constexpr int kStepBits = 12;          // bits per later pass
 
 struct SelectState {
-  unsigned long long hist[kPasses][kBins];  // global digit counts per pass
-  unsigned long long k_rem;                 // rank still to find below prefix
-  uint32_t prefix;                          // digits chosen so far
+  unsigned long long hist[kPasses][kBins];  // global bin counts per pass
+  unsigned long long k_rem;                 // rank still to find inside the range
+  uint32_t lo;                              // the range [lo, lo + 2^wlog) holding q
+  int32_t wlog;
+  uint32_t resolved;                        // set once the range is one value
   uint32_t done[kPasses];                   // blocks finished per pass
   int32_t q;                                // the quantile once selected
 };
@@ -38,28 +41,44 @@ __device__ __forceinline__ uint32_t score(int32_t L, int32_t P) {
   return d > 0 ? static_cast<uint32_t>(d) : 0u;
 }
 
+// First-pass bin: non-decreasing in s, at most 1024 + 22 * 128 = 3,840 bins.
+__device__ __forceinline__ int first_bin(uint32_t s) {
+  if (s < kExactBins) return static_cast<int>(s);
+  const int e = 31 - __clz(s);  // leading bit, 10..31
+  return static_cast<int>(kExactBins) + ((e - 10) << kMantBits) +
+         static_cast<int>((s >> (e - kMantBits)) & ((1u << kMantBits) - 1u));
+}
+
 template <int PASS>
 __global__ void __launch_bounds__(kSelectThreads)
 select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
                    int64_t n, unsigned long long k0, SelectState *st,
                    int32_t *q_dev_out, int32_t *status) {
   pdl_prologue();
-  constexpr int kShift = Digit<PASS>::shift;
-  constexpr uint32_t kMask = (1u << Digit<PASS>::bits) - 1u;
-  constexpr int kPrevShift = PASS == 0 ? 0 : Digit<(PASS > 0 ? PASS - 1 : 0)>::shift;
+  if (PASS > 0 && *reinterpret_cast<volatile uint32_t *>(&st->resolved)) return;
   __shared__ uint32_t sh[kBins];
   __shared__ int s_last;
   __shared__ unsigned long long s_warp[kSelectThreads / 32];
 
   for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
   __syncthreads();
-  const uint32_t prefix = PASS == 0 ? 0u : *reinterpret_cast<volatile uint32_t *>(&st->prefix);
+  // the range chosen so far and this pass's digit of s - lo
+  const uint32_t lo = PASS == 0 ? 0u : *reinterpret_cast<volatile uint32_t *>(&st->lo);
+  const int wlog = PASS == 0 ? 32 : *reinterpret_cast<volatile int32_t *>(&st->wlog);
+  const int shift = wlog > kStepBits ? wlog - kStepBits : 0;
 
-  // Warp-aggregated histogram update: lanes holding the same digit add once
+  // Warp-aggregated histogram update: lanes holding the same bin add once
   // (about half of all scores are 0, so single-lane atomics would pile up).
   auto visit = [&](uint32_t s, bool valid) {
-    if (PASS > 0 && (s >> kPrevShift) != prefix) valid = false;
-    const int d = valid ? static_cast<int>((s >> kShift) & kMask) : -1;
+    int d;
+    if constexpr (PASS == 0) {
+      d = first_bin(s);
+    } else {
+      const uint32_t r = s - lo;  // wlog <= 24 here
+      if (s < lo || r >= (1u << wlog)) valid = false;
+      d = static_cast<int>(r >> shift);
+    }
+    if (!valid) d = -1;
     const unsigned peers = __match_any_sync(0xffffffffu, d);
     if (valid && static_cast<int>(threadIdx.x & 31) == __ffs(peers) - 1)
       atomicAdd(&sh[d], static_cast<uint32_t>(__popc(peers)));
@@ -120,10 +139,10 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
   if (!s_last) return;
   __threadfence();
 
-  // The last block: find the bin holding rank k among the survivors.
+  // The last block: find the bin holding rank k inside the range.
   const unsigned long long k =
       PASS == 0 ? k0 : *reinterpret_cast<volatile unsigned long long *>(&st->k_rem);
-  constexpr int kPer = kBins / kSelectThreads;  // 8 consecutive bins per thread
+  constexpr int kPer = kBins / kSelectThreads;  // 16 consecutive bins per thread
   unsigned long long c[kPer], tot = 0;
 #pragma unroll
   for (int j = 0; j < kPer; ++j) {
@@ -153,15 +172,35 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
       }
       cum += c[j];
     }
-    const uint32_t np = (prefix << Digit<PASS>::bits) | static_cast<uint32_t>(d);
-    st->prefix = np;
+    // the new range: the bin's values
+    uint32_t nlo;
+    int nw;
+    if constexpr (PASS == 0) {
+      if (d < static_cast<int>(kExactBins)) {
+        nlo = static_cast<uint32_t>(d);
+        nw = 0;
+      } else {
+        const int e = 10 + ((d - static_cast<int>(kExactBins)) >> kMantBits);
+        const uint32_t top = (1u << kMantBits) |
+                             static_cast<uint32_t>((d - static_cast<int>(kExactBins)) &
+                                                   ((1 << kMantBits) - 1));
+        nlo = top << (e - kMantBits);
+        nw = e - kMantBits;
+      }
+    } else {
+      nlo = lo + (static_cast<uint32_t>(d) << shift);
+      nw = shift;
+    }
+    st->lo = nlo;
+    st->wlog = nw;
     st->k_rem = k - cum;
-    if (PASS == kPasses - 1) {
-      if (np > 0x7fffffffu) {
+    if (nw == 0) {
+      st->resolved = 1u;
+      if (nlo > 0x7fffffffu) {
         flag_error(status, MAPS_E_RANGE);
       } else {
-        st->q = static_cast<int32_t>(np);
-        if (q_dev_out) *q_dev_out = static_cast<int32_t>(np);
+        st->q = static_cast<int32_t>(nlo);
+        if (q_dev_out) *q_dev_out = static_cast<int32_t>(nlo);
       }
     }
   }
@@ -210,7 +249,7 @@ bound_kernel(const int32_t *__restrict__ pred, int64_t m, const SelectState *st,
   if (bad) flag_error(status, MAPS_E_RANGE);
 }
 
-// Small calibration sets (n <= kSmallN): the same three-digit radix select,
+// Small calibration sets (n <= kSmallN): a three-digit (11, 11, 10 bits) radix select,
 // run by one block over the scores held in shared memory, then the bounds of
 // up to kSmallM queries by the same block: one launch instead of a memset and
 // four.
@@ -218,6 +257,7 @@ constexpr int kSmallN = 8192;
 constexpr int kSmallM = 8192;
 constexpr int kSmallThreads = 1024;
 constexpr int kBitonicN = 2048;  // up to this many scores are sorted outright
+constexpr int kSmallBins = 2 * kSmallThreads;  // 11-bit digits, two bins per thread
 
 __global__ void __launch_bounds__(kSmallThreads)
 select_small_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P, int n,
@@ -226,7 +266,7 @@ select_small_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P
                     int32_t *status) {
   pdl_prologue();
   extern __shared__ uint32_t s[];  // the scores (kBitonicN or kSmallN words, as launched)
-  __shared__ uint32_t hist[kBins];
+  __shared__ uint32_t hist[kSmallBins];
   __shared__ uint32_t s_warp[kSmallThreads / 32];
   __shared__ uint32_t s_pick[2];  // the chosen bin, the rank left inside it
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -260,7 +300,7 @@ select_small_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P
       const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
       const int bits = pass == 2 ? 10 : 11;
       const int prev = pass == 0 ? 32 : (pass == 1 ? 21 : 10);  // bits above this digit
-      for (int b = tid; b < kBins; b += kSmallThreads) hist[b] = 0;
+      for (int b = tid; b < kSmallBins; b += kSmallThreads) hist[b] = 0;
       __syncthreads();
       for (int i = tid; i < n; i += kSmallThreads) {
         const uint32_t v = s[i];

@@ -189,6 +189,37 @@ def test_calibrate_unaligned_and_ranges(M, ws, oracle):
     assert M.maps_calibrate(Ld, Pd, 0, ws=ws)[0] == M.MAPS_E_INVALID
 
 
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_calibrate_grid_bucket_edges(M, ws, oracle, seed):
+    """Grid form (n above the one-block limit): scores on the first pass's bin
+    edges (the last exact bin, each leading-bit boundary, each 7-bit step) and
+    up to 2^32 - 1, so that quantiles resolve after one, two or three passes and
+    some lie above INT32_MAX (range error)."""
+    rng = np.random.default_rng(seed)
+    edges = {0, 1, 1022, 1023, 1024, 1025, 2**32 - 1}
+    for e in range(10, 32):
+        step = 1 << (e - 7)
+        edges |= {(1 << e) - 1, 1 << e, (1 << e) + 1, (1 << e) + step - 1, (1 << e) + step}
+    edges = np.array(sorted(edges), dtype=np.int64)
+    n = 20011
+    s = rng.choice(edges, n)
+    s[: n // 3] = rng.integers(0, 2**32, n // 3, dtype=np.int64)  # full range
+    P = np.full(n, -(2**31), dtype=np.int64)
+    small = s < 2**31 - 5000
+    P[small] = rng.integers(-2000, 2000, int(small.sum()))
+    L, P = (P + s).astype(np.int32), P.astype(np.int32)
+    assert np.array_equal(np.maximum(L.astype(np.int64) - P, 0), s)
+    seen = set()
+    for a in (1, 30, 1000, 100000, 333333, 500000, 700000, 900000, 999000, 999999):
+        sto, qo = oracle.calibrate(L, P, a)
+        st, q, qd, _ = gpu_calibrate(M, ws, L, P, a)
+        assert st == sto, (seed, a)
+        seen.add(st)
+        if st == 0:
+            assert q == qd == qo, (seed, a)
+    assert {0, M.MAPS_E_RANGE} <= seen
+
+
 @pytest.mark.parametrize("name", ["tiny", "d16", "d64", "large"])
 def test_calibrate_workloads(M, ws, oracle, name):
     w = W.make(name)
