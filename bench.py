@@ -55,15 +55,15 @@ L2_FLUSH_BYTES = 256 << 20
 # kernels, one launch each; dispatch_scoring is the scoring kernel alone),
 # valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 12580892, "source": "calibrate.cu", "source_sha256":
-                  "2f8167c0989dce1257fabfa3dbf11839b4df88b68af313fa12b2e3614f92179e"},
-    "occupancy": {"bytes": 29785344, "source": "occupancy.cu", "source_sha256":
+    "calibrate": {"bytes": 12579441, "source": "calibrate.cu", "source_sha256":
+                  "6eaf388c3ed23fe6b5f9589eb32227a9602f2f0cca9895ac790ef8bc13e73a84"},
+    "occupancy": {"bytes": 29774734, "source": "occupancy.cu", "source_sha256":
                   "fd537e3019c8991f53d529abba17e1a23b2664a7f4477b0936c6a78e22aa0746"},
-    "dispatch": {"bytes": 26432142, "source": "dispatch.cu", "source_sha256":
+    "dispatch": {"bytes": 26432085, "source": "dispatch.cu", "source_sha256":
                  "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
-    "dispatch_scoring": {"bytes": 21113656, "source": "dispatch.cu", "source_sha256":
+    "dispatch_scoring": {"bytes": 21113543, "source": "dispatch.cu", "source_sha256":
                          "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
-    "order": {"bytes": 41116672, "source": "order.cu", "source_sha256":
+    "order": {"bytes": 41117710, "source": "order.cu", "source_sha256":
               "2aae9099a88207fe058f683410602dc85706e042756c58459f064ae821ab87da"},
 }
 KERNELS = {

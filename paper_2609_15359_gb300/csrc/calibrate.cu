@@ -21,7 +21,7 @@ namespace {
 
 constexpr int kBins = 4096;
 constexpr int kPasses = 3;
-constexpr int kSelectThreads = 256;
+constexpr int kSelectThreads = 1024;
 constexpr uint32_t kExactBins = 1024;  // scores below this have a bin each
 constexpr int kMantBits = 7;           // bits after the leading one, first pass
 constexpr int kStepBits = 12;          // bits per later pass
@@ -67,21 +67,26 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
   const int wlog = PASS == 0 ? 32 : *reinterpret_cast<volatile int32_t *>(&st->wlog);
   const int shift = wlog > kStepBits ? wlog - kStepBits : 0;
 
-  // Warp-aggregated histogram update: lanes holding the same bin add once
-  // (about half of all scores are 0, so single-lane atomics would pile up).
+  // Histogram update.  First pass: the zero scores (about half of a length
+  // residual's scores) are counted by one ballot per warp and every other lane
+  // adds alone, since its bin is a single value or a narrow range.  Later
+  // passes aggregate the lanes of each bin with a match, as no bin of a range
+  // is known to be hot.
+  const int lane = static_cast<int>(threadIdx.x & 31);
   auto visit = [&](uint32_t s, bool valid) {
-    int d;
     if constexpr (PASS == 0) {
-      d = first_bin(s);
+      const int d = first_bin(s);
+      const unsigned zeros = __ballot_sync(0xffffffffu, valid && d == 0);
+      if (zeros && lane == __ffs(zeros) - 1) atomicAdd(&sh[0], static_cast<uint32_t>(__popc(zeros)));
+      if (valid && d > 0) atomicAdd(&sh[d], 1u);
     } else {
       const uint32_t r = s - lo;  // wlog <= 24 here
       if (s < lo || r >= (1u << wlog)) valid = false;
-      d = static_cast<int>(r >> shift);
+      const int d = valid ? static_cast<int>(r >> shift) : -1;
+      const unsigned peers = __match_any_sync(0xffffffffu, d);
+      if (valid && lane == __ffs(peers) - 1)
+        atomicAdd(&sh[d], static_cast<uint32_t>(__popc(peers)));
     }
-    if (!valid) d = -1;
-    const unsigned peers = __match_any_sync(0xffffffffu, d);
-    if (valid && static_cast<int>(threadIdx.x & 31) == __ffs(peers) - 1)
-      atomicAdd(&sh[d], static_cast<uint32_t>(__popc(peers)));
   };
 
   // Grid-stride loops whose bounds depend only on the block's first index,
@@ -142,7 +147,7 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
   // The last block: find the bin holding rank k inside the range.
   const unsigned long long k =
       PASS == 0 ? k0 : *reinterpret_cast<volatile unsigned long long *>(&st->k_rem);
-  constexpr int kPer = kBins / kSelectThreads;  // 16 consecutive bins per thread
+  constexpr int kPer = kBins / kSelectThreads;  // 4 consecutive bins per thread
   unsigned long long c[kPer], tot = 0;
 #pragma unroll
   for (int j = 0; j < kPer; ++j) {
@@ -150,7 +155,7 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
     tot += c[j];
   }
   // exclusive scan of the per-thread totals
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int warp = threadIdx.x >> 5;
   unsigned long long incl = tot;
 #pragma unroll
   for (int off = 1; off < 32; off <<= 1) {
