@@ -55,15 +55,15 @@ L2_FLUSH_BYTES = 256 << 20
 # kernels, one launch each; dispatch_scoring is the scoring kernel alone),
 # valid only for the kernel source it was taken on.
 TRAFFIC = {
-    "calibrate": {"bytes": 12579441, "source": "calibrate.cu", "source_sha256":
-                  "6eaf388c3ed23fe6b5f9589eb32227a9602f2f0cca9895ac790ef8bc13e73a84"},
-    "occupancy": {"bytes": 29774734, "source": "occupancy.cu", "source_sha256":
+    "calibrate": {"bytes": 12578673, "source": "calibrate.cu", "source_sha256":
+                  "2c2d7dd3d182439cc27caeb6ae856327284afa160f2de0b32e84a119acd45be6"},
+    "occupancy": {"bytes": 29642638, "source": "occupancy.cu", "source_sha256":
                   "fd537e3019c8991f53d529abba17e1a23b2664a7f4477b0936c6a78e22aa0746"},
-    "dispatch": {"bytes": 26432085, "source": "dispatch.cu", "source_sha256":
+    "dispatch": {"bytes": 26430862, "source": "dispatch.cu", "source_sha256":
                  "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
-    "dispatch_scoring": {"bytes": 21113543, "source": "dispatch.cu", "source_sha256":
+    "dispatch_scoring": {"bytes": 21113031, "source": "dispatch.cu", "source_sha256":
                          "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
-    "order": {"bytes": 41117710, "source": "order.cu", "source_sha256":
+    "order": {"bytes": 41115687, "source": "order.cu", "source_sha256":
               "2aae9099a88207fe058f683410602dc85706e042756c58459f064ae821ab87da"},
 }
 KERNELS = {

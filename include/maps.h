@@ -36,6 +36,8 @@
  * Domain.   Lengths (prompt p, generated g, bounds U), capacities, queue
  *           lengths and K values must be >= 0; a negative one is reported as
  *           MAPS_E_RANGE.
+ * Aliasing. An output array overlaps no input array, no other output and no
+ *           workspace of the same call.
  */
 #ifndef MAPS_H
 #define MAPS_H

@@ -212,18 +212,19 @@ select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
 }
 
 // U = pred + q.  Four bounds per thread (one 128-bit load and store when
-// both arrays allow it), all loads issued before any store.
+// both arrays allow it).  The predictions are the caller's input: the grid
+// before this one is a select kernel of the same call, which writes only the
+// select state, and it starts only once every earlier grid has completed.  So
+// the loads are issued before the wait on that grid and overlap its tail;
+// only the quantile is read after it.
 __global__ void __launch_bounds__(256)
 bound_kernel(const int32_t *__restrict__ pred, int64_t m, const SelectState *st,
              int32_t *__restrict__ out, int32_t *status) {
-  pdl_prologue();
-  const long long q = *reinterpret_cast<const volatile int32_t *>(&st->q);
   const int64_t i4 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   const int64_t i = i4 * 4;
-  if (i >= m) return;
   const bool vec = (reinterpret_cast<uintptr_t>(pred) % 16 == 0) &&
                    (reinterpret_cast<uintptr_t>(out) % 16 == 0) && i + 4 <= m;
-  int32_t v[4];
+  int32_t v[4] = {0, 0, 0, 0};
   if (vec) {
     const int4 x = __ldg(reinterpret_cast<const int4 *>(pred) + i4);
     v[0] = x.x;
@@ -234,6 +235,9 @@ bound_kernel(const int32_t *__restrict__ pred, int64_t m, const SelectState *st,
 #pragma unroll
     for (int c = 0; c < 4; ++c) v[c] = i + c < m ? __ldg(pred + i + c) : 0;
   }
+  pdl_prologue();
+  if (i >= m) return;
+  const long long q = *reinterpret_cast<const volatile int32_t *>(&st->q);
   bool bad = false;
 #pragma unroll
   for (int c = 0; c < 4; ++c) {
