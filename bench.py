@@ -59,10 +59,10 @@ TRAFFIC = {
                   "2c2d7dd3d182439cc27caeb6ae856327284afa160f2de0b32e84a119acd45be6"},
     "occupancy": {"bytes": 29642638, "source": "occupancy.cu", "source_sha256":
                   "fd537e3019c8991f53d529abba17e1a23b2664a7f4477b0936c6a78e22aa0746"},
-    "dispatch": {"bytes": 26430862, "source": "dispatch.cu", "source_sha256":
-                 "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
-    "dispatch_scoring": {"bytes": 21113031, "source": "dispatch.cu", "source_sha256":
-                         "974df773e052876e3be2c90316cc3615adaffcb2dd6fd029a4d83ddaf5e3e2b1"},
+    "dispatch": {"bytes": 26433052, "source": "dispatch.cu", "source_sha256":
+                 "7f665bf0eb59ac1b91fcd226e1e8dff0185ef058ce89b7c99f27a3e2179185ed"},
+    "dispatch_scoring": {"bytes": 21114424, "source": "dispatch.cu", "source_sha256":
+                         "7f665bf0eb59ac1b91fcd226e1e8dff0185ef058ce89b7c99f27a3e2179185ed"},
     "order": {"bytes": 41115687, "source": "order.cu", "source_sha256":
               "2aae9099a88207fe058f683410602dc85706e042756c58459f064ae821ab87da"},
 }

@@ -376,12 +376,19 @@ __global__ void __launch_bounds__(256)
 bin_scatter_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__ cp,
                    const int32_t *__restrict__ cb, const uint32_t *toff, uint32_t *tcursor,
                    int32_t *ord, int32_t *sp, int32_t *su) {
+  // The candidates are the caller's input and the grid before this one (the
+  // counting kernel of the same call) writes only the workspace and the
+  // call's outputs; it starts only once every earlier grid has completed.  So
+  // this thread's first candidate is loaded before the wait on it.
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t b0 = static_cast<int64_t>(blockIdx.x) * blockDim.x;
+  const int64_t j_first = b0 + threadIdx.x;
+  const int32_t p_first = j_first < J ? cp[j_first] : -1;
+  const int32_t u_first = j_first < J ? cb[j_first] : -1;
   pdl_prologue();
   __shared__ uint32_t s_h[kBinSmem];  // local counts, then local cursors
   __shared__ uint32_t s_b[kBinSmem];  // this block's base inside each bucket
   const bool local = T2 <= kBinSmem;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  const int64_t b0 = static_cast<int64_t>(blockIdx.x) * blockDim.x;
   if (local) {
     for (int i = threadIdx.x; i < T2; i += blockDim.x) s_h[i] = 0;
     __syncthreads();
@@ -389,8 +396,8 @@ bin_scatter_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__
       const int64_t j = j0 + threadIdx.x;
       int tile = -1;
       if (j < J) {
-        const int32_t U = cb[j];
-        if ((cp[j] | U) >= 0) tile = (candidate_steps(U, H) - 1) / W2;
+        const int32_t U = j0 == b0 ? u_first : cb[j];
+        if (((j0 == b0 ? p_first : cp[j]) | U) >= 0) tile = (candidate_steps(U, H) - 1) / W2;
       }
       const unsigned peers = __match_any_sync(0xffffffffu, tile);
       if (tile >= 0 && (threadIdx.x & 31) == __ffs(peers) - 1)
@@ -411,8 +418,8 @@ bin_scatter_kernel(int64_t J, int H, int W2, int T2, const int32_t *__restrict__
     int tile = -1, u = 0;
     int32_t p = 0;
     if (j < J) {
-      p = cp[j];
-      const int32_t U = cb[j];
+      p = j0 == b0 ? p_first : cp[j];
+      const int32_t U = j0 == b0 ? u_first : cb[j];
       if ((p | U) >= 0) {
         u = candidate_steps(U, H);
         tile = (u - 1) / W2;
