@@ -76,6 +76,36 @@ def test_quantile_is_sorted_order_statistic(oracle, n):
         assert np.count_nonzero(s < q) < k
 
 
+@pytest.mark.parametrize("seed", [0, 1])
+def test_quantile_full_int32_range(oracle, seed):
+    """Scores of full-range int32 lengths reach 2^32 - 1 (the difference of two
+    int32 values clamped at 0).  The quantile is still the k-th smallest of them
+    (numpy's sort in int64), and a quantile above INT32_MAX cannot be an int32
+    bound: MAPS_E_RANGE."""
+    rng = np.random.default_rng(100 + seed)
+    n = 3001
+    L = rng.integers(-(2**31), 2**31, n, dtype=np.int64)
+    P = rng.integers(-(2**31), 2**31, n, dtype=np.int64)
+    # powers of two and their neighbours among the scores
+    e = rng.integers(0, 32, n // 3)
+    P[: n // 3] = -(2**31)
+    L[: n // 3] = np.minimum(P[: n // 3] + (1 << e) + rng.integers(-1, 2, n // 3), 2**31 - 1)
+    L, P = L.astype(np.int32), P.astype(np.int32)
+    s = np.maximum(0, L.astype(np.int64) - P)
+    assert s.max() > 2**31  # some scores above INT32_MAX
+    seen = set()
+    for a in (1000, 100000, 300000, 500000, 700000, 900000, 999000):
+        k = exact_rank(n, a)
+        st, q = oracle.calibrate(L, P, a)
+        want = np.sort(s)[k - 1]
+        if want > 2**31 - 1:
+            assert st == -2, a
+        else:
+            assert st == 0 and q == want, a
+        seen.add(st)
+    assert seen == {0, -2}
+
+
 def test_calibration_unbounded_and_invalid(oracle):
     e = np.zeros(0, np.int32)
     assert oracle.calibrate(e, e, 100000)[0] == -3  # n = 0: rank 1 > 0
