@@ -1,5 +1,7 @@
 """Host-side logic of bench.py that needs no GPU: the staging arena of the
-end-to-end path and the traffic table's source keys."""
+end-to-end path, the traffic table's source keys and the reference arm (the
+oracle, timed on the host)."""
+import argparse
 import os
 
 import numpy as np
@@ -42,3 +44,29 @@ def test_traffic_table_keys_existing_sources():
         assert call in bench.KERNELS
         # a figure is only reported for the source it was measured on
         assert bench.traffic_for(call) in (None, t["bytes"])
+
+
+def test_oracle_step_sampling_scales_to_the_workload():
+    w = W.make("d16")
+    full, J = bench.oracle_step(w, w["J"])
+    assert J == w["J"] and full > 0
+    # a sample of decoders and candidates still stands for the whole step
+    part, J2 = bench.oracle_step(w, 64, 4)
+    assert J2 == J and part > 0
+    # more candidates than exist are clamped, not extrapolated
+    assert bench.oracle_step(w, 10 * w["J"], 4)[0] > 0
+
+
+def test_reference_arm_json_line(monkeypatch):
+    monkeypatch.setattr(bench, "WORKLOAD", "d16")
+    args = argparse.Namespace(steps=2, warmup=3, gpus=1, impl="reference")
+    assert bench.bench_reference(args, 2, 1) is None  # other ranks do no work
+    r = bench.bench_reference(args, 1, 0)
+    assert r["impl"] == "reference" and r["value"] > 0 and r["unit"] == bench.UNIT
+    assert r["steps"] == 2 and r["warmup"] == 3 and r["higher_is_better"] is True
+    assert r["ms_per_step"] > 0 and r["metric"] == bench.METRIC
+    cb = r["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] == r["value"]
+    assert cb["sample"]
+    assert r["e2e"] == {"value": r["value"], "unit": r["unit"], "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}
