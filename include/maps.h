@@ -61,7 +61,6 @@ extern "C" {
 #define MAPS_MODE_SEQUENTIAL 1
 #define MAPS_MODE_ALG1_SNAPSHOT 2
 #define MAPS_MODE_ALG1_SEQUENTIAL 3
-#define MAPS_MODE_SNAPSHOT_BINNED 4  /* SNAPSHOT of candidates bucketed by maps_dispatch_bin */
 
 /* Library version, major*10000 + minor*100 + patch. */
 int maps_version(void);
@@ -72,15 +71,6 @@ int maps_last_cuda_error(void);
 /* Synchronises `stream`, returns the workspace's sticky device status
  * (MAPS_OK or the first error any kernel recorded in it) and clears it. */
 int maps_check(void *ws, void *stream);
-
-/* Benchmarking aid.  `before` and `after` are CUDA events (cudaEvent_t,
- * created by the caller, passed as void *).  Every later SNAPSHOT
- * maps_dispatch call made by this thread records them on its stream right
- * before and right after its scoring kernel (after the candidates have been
- * bucketed by horizon tile), so a caller can time the scoring kernel alone.
- * An event between two launches costs the programmatic overlap there.
- * NULL, NULL turns it off.  Results are unaffected.  Returns MAPS_OK. */
-int maps_set_dispatch_events(void *before, void *after);
 
 /* ------------------------------------------------------------------------
  * Uncertainty-aware calibration, Sec. 3.2.
@@ -166,8 +156,7 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
  * ALG1_SEQUENTIAL subtracts B_need from B_eff[k*] and adds 1 to Q[k*] after
  * each choice.  K is not read in the ALG1 modes.
  *
- *   mode                MAPS_MODE_* (MAPS_MODE_SNAPSHOT_BINNED: see
- *                       maps_dispatch_bin below).
+ *   mode                MAPS_MODE_*.
  *   D, H, S             decoders (1 <= D <= 1024), horizon (1 <= H <= 2^28),
  *                       block size (ALG1).
  *   K                   [D][H] int32 occupancy (horizon modes; updated in
@@ -175,8 +164,10 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
  *   kmax                optional [D][ceil(H/16)] uint32, SNAPSHOT only: the
  *                       summary maps_project_occupancy wrote for this same K.
  *                       NULL makes the call derive it from K (one more pass
- *                       over K).  A summary that does not match K gives
- *                       unspecified results.
+ *                       over K).  The call compares a given summary with K at
+ *                       four blocks of every row and reports a mismatch there
+ *                       as MAPS_E_INVALID (via maps_check); a summary that
+ *                       differs from K elsewhere gives unspecified results.
  *   cap, Q              [D] int32 capacities and queue lengths (Q updated in
  *                       place by the SEQUENTIAL modes).
  *   res_off, R, prompt, gen, bound   residents as in maps_project_occupancy
@@ -190,20 +181,6 @@ int maps_project_occupancy(int32_t D, int32_t H, const int64_t *res_off,
 size_t maps_dispatch_workspace_size(int32_t mode, int32_t D, int32_t H,
                                     int64_t J);
 
-/* SNAPSHOT in two calls.  The candidates' bucketing by horizon tile depends
- * on the candidates alone, not on K, so a caller may issue it earlier (for
- * instance on a second stream while maps_project_occupancy computes K):
- * maps_dispatch_bin buckets them into `ws` (a SNAPSHOT workspace for D, H, J)
- * and writes choice_out = -1, headroom_out = 0 for candidates with a negative
- * prompt or bound (MAPS_E_RANGE, as in SNAPSHOT).  A later maps_dispatch with
- * mode MAPS_MODE_SNAPSHOT_BINNED, the same D, H, J, candidates, outputs and
- * workspace, and no other call on that workspace in between, then scores them
- * and gives the SNAPSHOT result.  If the workspace holds no buckets of this
- * D, H and J, the binned call reads none of them and records MAPS_E_INVALID
- * (read with maps_check).  Returns MAPS_OK or a host-detected error. */
-int maps_dispatch_bin(int32_t D, int32_t H, int64_t J, const int32_t *cand_prompt,
-                      const int32_t *cand_bound, int32_t *choice_out,
-                      int64_t *headroom_out, void *ws, size_t ws_bytes, void *stream);
 int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K,
                   const uint32_t *kmax, const int32_t *cap, int32_t *Q,
                   const int64_t *res_off,
@@ -255,11 +232,15 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec,
  *                       sizes return MAPS_E_WORKSPACE at once.
  *   status_host         optional host int32 (NULL: not written).  Non-NULL
  *                       synchronises the stream and returns the full status,
- *                       data-dependent errors included; with NULL, data errors
- *                       are not reported.
- *   First call          the first call on each device looks up the array's
- *                       device address; make that call before any stream
- *                       capture.
+ *                       data-dependent errors included.  With NULL, data
+ *                       errors (MAPS_E_RANGE, MAPS_E_TIMEOUT) are lost: the
+ *                       array's status word is cleared by the next call and
+ *                       no other call reads it, so a caller that needs them
+ *                       must pass status_host.
+ *   First call          every call looks up the array's device address on
+ *                       the current device (a host call); the first call on a
+ *                       device may also load the library's device code there,
+ *                       so make that first call before any stream capture.
  *   Concurrency         every call shares the one array: calls whose work
  *                       overlaps on the GPU (other streams, other threads)
  *                       race and give wrong results.  Order them on one

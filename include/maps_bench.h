@@ -1,0 +1,40 @@
+/*
+ * maps_bench.h -- test and benchmarking aids of libmaps.so.  Not part of the
+ * scheduler's interface (include/maps.h): a scheduler never needs them, and
+ * with their defaults they change nothing.  The paper has no counterpart.
+ */
+#ifndef MAPS_BENCH_H
+#define MAPS_BENCH_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* `before` and `after` are CUDA events (cudaEvent_t, created by the caller,
+ * passed as void *).  Every later SNAPSHOT maps_dispatch call made by this
+ * thread records them on its stream right before and right after its scoring
+ * kernel (after the candidates have been bucketed by horizon tile), so a
+ * caller can time the scoring kernel alone.  An event between two launches
+ * costs the programmatic overlap there.  NULL, NULL turns it off.  Results
+ * are unaffected.  Returns MAPS_OK (0). */
+int maps_set_dispatch_events(void *before, void *after);
+
+/* Exercises the bounded waits of maps_order_local's global form (the form
+ * taken when arrival is not non-decreasing along the index and the call is
+ * larger than one block): on the current device, later calls let tile `tile`
+ * of every radix pass publish nothing to the decoupled look-back, and every
+ * look-back wait gives up after `spin_limit` polls (0: the library default).
+ * The tile after the withheld one then waits until the limit, records
+ * MAPS_E_TIMEOUT (read with maps_check) and carries on; the order of that
+ * call is wrong, every write stays inside the outputs, and the device stays
+ * usable.  tile = -1, spin_limit = 0 restores the normal behaviour.  Calls in
+ * flight must have finished before the settings change.  Returns MAPS_OK or
+ * MAPS_E_CUDA. */
+int maps_test_withhold_lookback(int32_t tile, uint32_t spin_limit);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MAPS_BENCH_H */

@@ -22,8 +22,14 @@ _LIB = os.path.join(_HERE, "liboracle.so")
 MODE_SNAPSHOT, MODE_SEQUENTIAL, MODE_ALG1_SNAPSHOT, MODE_ALG1_SEQUENTIAL = 0, 1, 2, 3
 
 
+_SRC_P = os.path.join(_HERE, "oracle_p.cpp")
+_LIB_P = os.path.join(_HERE, "liboracle_p.so")
+
+
 def build(force: bool = False) -> str:
-    """Compile ``liboracle.so`` with the host C compiler (plain C11, -O2)."""
+    """Compile ``liboracle.so`` (plain C11, -O2) and ``liboracle_p.so`` (the
+    tier-P oracle, C++17 -O2, with OpenMP where the compiler has it) with the
+    host compilers."""
     if force or not os.path.exists(_LIB) or (
             os.path.getmtime(_LIB) < max(os.path.getmtime(_SRC),
                                          os.path.getmtime(os.path.join(_HERE, "oracle.h")))):
@@ -31,6 +37,13 @@ def build(force: bool = False) -> str:
         subprocess.check_call(["gcc", "-O2", "-std=c11", "-shared", "-fPIC",
                                "-o", tmp, _SRC])
         os.replace(tmp, _LIB)
+    if force or not os.path.exists(_LIB_P) or os.path.getmtime(_LIB_P) < os.path.getmtime(_SRC_P):
+        tmp = _LIB_P + f".{os.getpid()}.tmp"
+        base = ["g++", "-O2", "-std=c++17", "-shared", "-fPIC", "-o", tmp, _SRC_P]
+        r = subprocess.run(base[:1] + ["-fopenmp"] + base[1:], capture_output=True, text=True)
+        if r.returncode != 0:  # no OpenMP: the same code, one thread
+            subprocess.check_call(base)
+        os.replace(tmp, _LIB_P)
     return _LIB
 
 
@@ -75,6 +88,26 @@ def lib():
                                     _i32p, _i32p, _i32p, _i32p, _i64p]
         _lib = L
     return _lib
+
+
+_libp = None
+
+
+def libp():
+    """The tier-P oracle (``oracle_p.cpp``)."""
+    global _libp
+    if _libp is None:
+        build()
+        L = ctypes.CDLL(_LIB_P)
+        vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+        L.oraclep_threads.argtypes = [ctypes.c_int]
+        L.oraclep_calibrate.argtypes = [vp, vp, i64, ctypes.c_uint32, ctypes.POINTER(i64)]
+        L.oraclep_bound.argtypes = [vp, i64, i64, vp]
+        L.oraclep_occupancy.argtypes = [i32, i32, vp, i64, vp, vp, vp, vp]
+        L.oraclep_dispatch_snapshot.argtypes = [i32, i32, vp, vp, vp, i64, vp, vp, vp, vp]
+        L.oraclep_order_local.argtypes = [i64, i32, vp, vp, vp, vp, i32, vp, vp]
+        _libp = L
+    return _libp
 
 
 def _c32(a):
@@ -163,3 +196,59 @@ def stream(N, D, H, cap, batch, window, alpha_ppm, max_wait, arrival_ms,
                              _c32(prompt[:N]), _c32(true_len[:N]),
                              _c32(pred[:N]), choice, q, stats)
     return st, choice, q, stats.reshape(nb, 4)
+
+
+# ---------------------------------------------------------------------------
+# tier P: the same results computed the plain way (oracle_p.cpp)
+# ---------------------------------------------------------------------------
+
+def p_threads(n: int = 1) -> int:
+    """Host threads for the tier-P loops (n <= 0: every core); returns the
+    number used (1 when the library was built without OpenMP)."""
+    return int(libp().oraclep_threads(n))
+
+
+def p_calibrate(true_len, pred_len, alpha_ppm: int):
+    t, p = _c32(true_len), _c32(pred_len)
+    q = ctypes.c_int64(0)
+    st = libp().oraclep_calibrate(_ptr(t), _ptr(p), t.shape[0], alpha_ppm, ctypes.byref(q))
+    return st, int(q.value)
+
+
+def p_bound(pred, q: int):
+    p = _c32(pred)
+    out = np.empty_like(p)
+    st = libp().oraclep_bound(_ptr(p), p.shape[0], q, _ptr(out))
+    return st, out
+
+
+def p_occupancy(D: int, H: int, res_off, prompt, gen, bnd, out=None):
+    """``out``: an optional [D][H] int32 array to write K into (reused)."""
+    off = _c64(res_off)
+    p, g, u = _c32(prompt), _c32(gen), _c32(bnd)
+    K = np.empty((D, H), dtype=np.int32) if out is None else out
+    st = libp().oraclep_occupancy(D, H, _ptr(off), p.shape[0], _ptr(p), _ptr(g), _ptr(u),
+                                  _ptr(K))
+    return st, K
+
+
+def p_dispatch_snapshot(D: int, H: int, K, cap, Q, cand_prompt, cand_bound):
+    Kc, capc, Qc = _c32(K), _c32(cap), _c32(Q)
+    cp, cb = _c32(cand_prompt), _c32(cand_bound)
+    J = cp.shape[0]
+    choice = np.empty(J, dtype=np.int32)
+    head = np.empty(J, dtype=np.int64)
+    st = libp().oraclep_dispatch_snapshot(D, H, _ptr(Kc), _ptr(capc), _ptr(Qc), J, _ptr(cp),
+                                          _ptr(cb), _ptr(choice), _ptr(head))
+    return st, choice, head
+
+
+def p_order_local(D: int, dec, bnd, wait, arrival, max_wait: int, out=None):
+    """``out``: an optional [N] int32 array for the order (reused)."""
+    d, b, w, a = _c32(dec), _c32(bnd), _c32(wait), _c32(arrival)
+    N = d.shape[0]
+    perm = np.empty(N, dtype=np.int32) if out is None else out
+    seg = np.empty(D + 1, dtype=np.int64)
+    st = libp().oraclep_order_local(N, D, _ptr(d), _ptr(b), _ptr(w), _ptr(a), max_wait,
+                                    _ptr(perm), _ptr(seg))
+    return st, perm, seg

@@ -19,8 +19,7 @@
 // binary search over D instead of D scores.  Candidates are first bucketed by
 // the tile of their last live step so each tile serves its own.  Three
 // launches: the carry scan and the bucket counts (independent, one launch),
-// the bucket scatter, the scoring kernel; or the bucketing alone
-// (maps_dispatch_bin) and later the carry scan and scoring (the binned mode).
+// the bucket scatter, the scoring kernel.
 //
 // SEQUENTIAL (reservation after each choice) and the literal Algorithm 1
 // modes are separate kernels below.
@@ -33,6 +32,7 @@
 #include <mutex>
 
 #include "maps_internal.cuh"
+#include "maps_bench.h"
 
 namespace maps {
 namespace {
@@ -130,8 +130,9 @@ kmax_from_K_kernel(int D, int H, const int32_t *__restrict__ K, uint32_t *__rest
 // (whole tiles, as W2/16 divides 16), keeps its tiles' maxima in registers,
 // and after a block scan writes its tiles' carries (the decoder's row of the
 // carries is contiguous; a work unit later reads one word per decoder).
-__device__ void carry_scan_block(int kk, int D, int H, int W2, int T2,
-                                 const uint32_t *__restrict__ kmax, uint32_t *__restrict__ carry,
+__device__ void carry_scan_block(int kk, int D, int H, int W2, int T2, const int32_t *__restrict__ K,
+                                 bool check_kmax, const uint32_t *__restrict__ kmax,
+                                 uint32_t *__restrict__ carry,
                                  const int32_t *__restrict__ Q, const int32_t *__restrict__ cap,
                                  int32_t *sig, int32_t *rank_of, int32_t *capq, int32_t *status) {
   __shared__ uint32_t s_w[8];
@@ -212,6 +213,21 @@ __device__ void carry_scan_block(int kk, int D, int H, int W2, int T2,
     run = all > run ? all : run;
     __syncthreads();
   }
+  if (check_kmax && threadIdx.x < 4) {
+    // a caller's summary is compared with K at four blocks of this row (the
+    // first, the last, the middle and one that varies with the decoder); a
+    // mismatch there is reported, any other gives unspecified results
+    const int64_t b = threadIdx.x == 0 ? 0 : threadIdx.x == 1 ? nb - 1 : threadIdx.x == 2 ? nb / 2
+                                                                     : (k * 7919LL) % nb;
+    const int32_t *kr = K + static_cast<int64_t>(k) * H;
+    const int64_t t_end = (b + 1) * kSumBlock < H ? (b + 1) * kSumBlock : static_cast<int64_t>(H);
+    long long mx = -1;
+    for (int64_t t = b * kSumBlock; t < t_end; ++t) {
+      const long long v = static_cast<long long>(__ldg(kr + t)) + t;
+      mx = v > mx ? v : mx;
+    }
+    if (mx < 0 || static_cast<uint32_t>(mx) != __ldg(row + b)) flag_error(status, MAPS_E_INVALID);
+  }
 }
 
 __device__ __forceinline__ unsigned lanemask_lt() {
@@ -239,7 +255,7 @@ __device__ void bin_count_block(int b, int nblk, int64_t J, int H, int W2, int T
                                 const int32_t *__restrict__ cp, const int32_t *__restrict__ cb,
                                 uint32_t *tcount, int32_t *choice, int64_t *headroom,
                                 int32_t *status, uint32_t *ticket, uint32_t *toff, Unit *units,
-                                uint32_t *nunits, uint2 hdr) {
+                                uint32_t *nunits) {
   __shared__ uint32_t s_h[kBinSmem];
   __shared__ bool s_last;
   const bool local = T2 <= kBinSmem;
@@ -287,29 +303,27 @@ __device__ void bin_count_block(int b, int nblk, int64_t J, int H, int W2, int T
   if (s_last) {
     __threadfence();
     bin_scan_block(T2, tcount, toff, units, nunits);
-    if (threadIdx.x == 0) {  // the buckets' header: which call's candidates they hold
-      nunits[2] = hdr.x;
-      nunits[3] = hdr.y;
-    }
   }
 }
 
 // The two independent first steps in one launch: blocks [0, D) scan the
 // carries of decoder blockIdx.x, the others count the candidates per tile.
 __global__ void __launch_bounds__(256)
-dispatch_prep_kernel(int ncarry, int D, int H, int W2, int T2, const uint32_t *__restrict__ kmax,
+dispatch_prep_kernel(int ncarry, int D, int H, int W2, int T2, const int32_t *__restrict__ K,
+                     bool check_kmax, const uint32_t *__restrict__ kmax,
                      uint32_t *__restrict__ carry, const int32_t *__restrict__ Q,
                      const int32_t *__restrict__ cap, int32_t *sig, int32_t *rank_of,
                      int32_t *capq, int64_t J, const int32_t *__restrict__ cp,
                      const int32_t *__restrict__ cb, uint32_t *tcount, int32_t *choice,
                      int64_t *headroom, int32_t *status, uint32_t *ticket, uint32_t *toff,
-                     Unit *units, uint32_t *nunits, uint2 hdr) {
+                     Unit *units, uint32_t *nunits) {
   pdl_prologue();
   if (static_cast<int>(blockIdx.x) < ncarry)
-    carry_scan_block(blockIdx.x, D, H, W2, T2, kmax, carry, Q, cap, sig, rank_of, capq, status);
+    carry_scan_block(blockIdx.x, D, H, W2, T2, K, check_kmax, kmax, carry, Q, cap, sig, rank_of,
+                     capq, status);
   else
     bin_count_block(blockIdx.x - ncarry, gridDim.x - ncarry, J, H, W2, T2, cp, cb, tcount, choice,
-                    headroom, status, ticket, toff, units, nunits, hdr);
+                    headroom, status, ticket, toff, units, nunits);
 }
 
 // Run by the last counting block (any multiple of 32 threads up to 1024):
@@ -454,8 +468,6 @@ struct SnapArgs {
   int comp_off;                              // words from the tile buffer to comp
   int region;                                // words from the tile buffer to the small arrays
   bool alias;                                // comp overwrites the tile (one row per thread)
-  bool check_hdr;                            // buckets from an earlier maps_dispatch_bin
-  uint2 hdr;                                 // the header they must carry
   bool use_tma;
   const int32_t *K;
   const int32_t *sig, *rank_of, *capq;  // queue order
@@ -474,11 +486,6 @@ dispatch_snapshot_kernel(const __grid_constant__ CUtensorMap tmap, SnapArgs a) {
   pdl_prologue();
   extern __shared__ __align__(1024) unsigned char smem[];
   const int unit = blockIdx.x;
-  if (a.check_hdr && (a.nunits[2] != a.hdr.x || a.nunits[3] != a.hdr.y)) {
-    // the workspace holds no buckets of these candidates: nothing is read
-    if (unit == 0 && threadIdx.x == 0) flag_error(a.status, MAPS_E_INVALID);
-    return;
-  }
   if (unit >= static_cast<int>(*a.nunits)) return;
   const int D = a.D, H = a.H;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -1192,7 +1199,7 @@ SnapGeom snap_geom(int D, int H) {
 }
 
 struct SnapWs {
-  uint32_t *zero;  // tcount[T2], tcursor[T2], nunits, ticket, header[2] (zeroed per call)
+  uint32_t *zero;  // tcount[T2], tcursor[T2], nunits, ticket (zeroed per call)
   size_t zero_words;
   uint32_t *toff;
   Unit *units;
@@ -1205,7 +1212,7 @@ struct SnapWs {
 
 SnapWs carve_snap(Carve &c, int D, int H, int T2, int64_t J) {
   SnapWs w;
-  w.zero_words = 2 * static_cast<size_t>(T2) + 4;  // tcount, tcursor, nunits, ticket, header
+  w.zero_words = 2 * static_cast<size_t>(T2) + 2;  // tcount, tcursor, nunits, ticket
   w.zero = c.take<uint32_t>(w.zero_words);
   w.toff = c.take<uint32_t>(static_cast<size_t>(T2) + 1);
   w.max_units = static_cast<int64_t>(T2) + (J + kUnitCands - 1) / kUnitCands;
@@ -1253,22 +1260,9 @@ int run_snapshot(int64_t grid, size_t smem, cudaStream_t s, const CUtensorMap &t
   return MAPS_OK;
 }
 
-// The header the buckets of (D, H, J) carry.
-uint2 bin_header(int D, int H, int64_t J) {
-  return make_uint2(0x4d415053u ^ static_cast<uint32_t>(J),
-                    static_cast<uint32_t>(H) * 2654435761u ^ static_cast<uint32_t>(D) * 40503u ^
-                        static_cast<uint32_t>(J >> 32));
-}
-
-// SNAPSHOT in stages: kBinAndScore does everything; kBinOnly buckets the
-// candidates by horizon tile (they depend on the candidates alone, so a caller
-// can issue this before K exists); kScoreOnly scores candidates an earlier
-// kBinOnly call bucketed into this workspace.
-enum SnapStage { kBinAndScore, kBinOnly, kScoreOnly };
-
-int launch_snapshot(SnapStage stage, int D, int H, const int32_t *K, const uint32_t *kmax,
-                    const int32_t *cap, const int32_t *Q, int64_t J, const int32_t *cp,
-                    const int32_t *cb, int32_t *choice, int64_t *headroom, void *ws, cudaStream_t s) {
+int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const int32_t *cap,
+                    const int32_t *Q, int64_t J, const int32_t *cp, const int32_t *cb,
+                    int32_t *choice, int64_t *headroom, void *ws, cudaStream_t s) {
   const SnapGeom g = snap_geom(D, H);
   if (g.smem + 1024 > static_cast<size_t>(max_smem_optin())) return MAPS_E_INVALID;
   Carve cv(ws);
@@ -1278,31 +1272,25 @@ int launch_snapshot(SnapStage stage, int D, int H, const int32_t *K, const uint3
   uint32_t *tcount = w.zero, *tcursor = w.zero + g.T2;
   uint32_t *nunits = w.zero + 2 * static_cast<size_t>(g.T2);
   uint32_t *ticket = nunits + 1;  // bin_count blocks finished
-  const uint2 hdr = bin_header(D, H, J);
   const int sms = sm_count();
-  const bool bin = stage != kScoreOnly, score = stage != kBinOnly;
-  if (bin) MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zero, 0, w.zero_words * 4, s)));
-  if (score && kmax == nullptr) {
+  MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zero, 0, w.zero_words * 4, s)));
+  const bool check_kmax = kmax != nullptr;
+  if (kmax == nullptr) {
     const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
     const int gk = static_cast<int>(std::min<int64_t>((nb * D + 255) / 256, 8LL * sms));
     launch_pdl(kmax_from_K_kernel, gk, 256, 0, s, D, H, K, w.kmax, status);
     kmax = w.kmax;
   }
-  // carries of D decoders (when scoring), and candidate counts in blocks of
-  // 256 candidates (when bucketing)
-  const int ncarry = score ? D : 0;
-  const int gc = bin ? static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((J + 255) / 256, 4LL * sms)))
-                     : 0;
-  launch_pdl(dispatch_prep_kernel, ncarry + gc, 256, 0, s, ncarry, D, H, g.W2, g.T2, kmax, w.carry, Q,
-             cap, w.sig, w.rank_of, w.capq, J, cp, cb, tcount, choice, headroom, status, ticket, w.toff,
-             w.units, nunits, hdr);
-  if (bin) {
-    const int gb = static_cast<int>(std::min<int64_t>((J + 255) / 256, 4LL * sms));
-    launch_pdl(bin_scatter_kernel, gb, 256, 0, s, J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord,
-               w.sp, w.su);
-  }
+  // carries of D decoders, and candidate counts in blocks of 256 candidates
+  const int gc = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((J + 255) / 256, 4LL * sms)));
+  launch_pdl(dispatch_prep_kernel, D + gc, 256, 0, s, D, D, H, g.W2, g.T2, K, check_kmax, kmax,
+             w.carry, Q, cap,
+             w.sig, w.rank_of, w.capq, J, cp, cb, tcount, choice, headroom, status, ticket, w.toff,
+             w.units, nunits);
+  const int gb = static_cast<int>(std::min<int64_t>((J + 255) / 256, 4LL * sms));
+  launch_pdl(bin_scatter_kernel, gb, 256, 0, s, J, H, g.W2, g.T2, cp, cb, w.toff, tcursor, w.ord,
+             w.sp, w.su);
   MAPS_TRY(launch_ok());
-  if (!score) return MAPS_OK;
 
   CUtensorMap tmap;
   std::memset(&tmap, 0, sizeof(tmap));
@@ -1333,8 +1321,6 @@ int launch_snapshot(SnapStage stage, int D, int H, const int32_t *K, const uint3
   a.comp_off = g.comp_off;
   a.region = g.region;
   a.alias = g.alias;
-  a.check_hdr = stage == kScoreOnly;
-  a.hdr = hdr;
   a.use_tma = use_tma;
   a.K = K;
   a.sig = w.sig;
@@ -1364,19 +1350,6 @@ int launch_snapshot(SnapStage stage, int D, int H, const int32_t *K, const uint3
 
 extern "C" {
 
-int maps_dispatch_bin(int32_t D, int32_t H, int64_t J, const int32_t *cand_prompt,
-                      const int32_t *cand_bound, int32_t *choice_out, int64_t *headroom_out,
-                      void *ws, size_t ws_bytes, void *stream) {
-  using namespace maps;
-  if (D < 1 || D > kMaxD || H < 1 || H > kMaxH || J < 0 || J > 0x7fffffffLL) return MAPS_E_INVALID;
-  if (J > 0 && (cand_prompt == nullptr || cand_bound == nullptr || choice_out == nullptr))
-    return MAPS_E_INVALID;
-  MAPS_TRY(check_ws(ws, ws_bytes, maps_dispatch_workspace_size(MAPS_MODE_SNAPSHOT, D, H, J)));
-  if (J == 0) return MAPS_OK;
-  return launch_snapshot(kBinOnly, D, H, nullptr, nullptr, nullptr, nullptr, J, cand_prompt,
-                         cand_bound, choice_out, headroom_out, ws, static_cast<cudaStream_t>(stream));
-}
-
 int maps_set_dispatch_events(void *before, void *after) {
   maps::g_score_ev[0] = static_cast<cudaEvent_t>(before);
   maps::g_score_ev[1] = static_cast<cudaEvent_t>(after);
@@ -1386,8 +1359,7 @@ int maps_set_dispatch_events(void *before, void *after) {
 size_t maps_dispatch_workspace_size(int32_t mode, int32_t D, int32_t H, int64_t J) {
   using namespace maps;
   Carve c(nullptr);
-  if ((mode == MAPS_MODE_SNAPSHOT || mode == MAPS_MODE_SNAPSHOT_BINNED) && D >= 1 && H >= 1 &&
-      H <= kMaxH) {
+  if (mode == MAPS_MODE_SNAPSHOT && D >= 1 && H >= 1 && H <= kMaxH) {
     const SnapGeom g = snap_geom(D, H);
     carve_snap(c, D, H, g.T2, J);
   } else if (mode == MAPS_MODE_SEQUENTIAL && D >= 1 && H >= 1 && H <= kMaxH) {
@@ -1404,13 +1376,12 @@ int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K, con
                   const int32_t *cand_bound, int32_t *choice_out, int64_t *headroom_out, void *ws,
                   size_t ws_bytes, void *stream) {
   using namespace maps;
-  if (mode < MAPS_MODE_SNAPSHOT || mode > MAPS_MODE_SNAPSHOT_BINNED) return MAPS_E_INVALID;
+  if (mode < MAPS_MODE_SNAPSHOT || mode > MAPS_MODE_ALG1_SEQUENTIAL) return MAPS_E_INVALID;
   if (D < 1 || D > kMaxD || J < 0 || J > 0x7fffffffLL || cap == nullptr || Q == nullptr)
     return MAPS_E_INVALID;
   if (J > 0 && (cand_prompt == nullptr || cand_bound == nullptr || choice_out == nullptr))
     return MAPS_E_INVALID;
-  const bool horizon = mode == MAPS_MODE_SNAPSHOT || mode == MAPS_MODE_SEQUENTIAL ||
-                       mode == MAPS_MODE_SNAPSHOT_BINNED;
+  const bool horizon = mode == MAPS_MODE_SNAPSHOT || mode == MAPS_MODE_SEQUENTIAL;
   if (horizon && (H < 1 || H > kMaxH || K == nullptr)) return MAPS_E_INVALID;
   if (!horizon && (S < 1 || res_off == nullptr || R < 0 ||
                    (R > 0 && (prompt == nullptr || gen == nullptr || bound == nullptr))))
@@ -1421,11 +1392,8 @@ int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K, con
   if (J == 0) return MAPS_OK;
   switch (mode) {
     case MAPS_MODE_SNAPSHOT:
-      return launch_snapshot(kBinAndScore, D, H, K, kmax, cap, Q, J, cand_prompt, cand_bound,
-                             choice_out, headroom_out, ws, s);
-    case MAPS_MODE_SNAPSHOT_BINNED:
-      return launch_snapshot(kScoreOnly, D, H, K, kmax, cap, Q, J, cand_prompt, cand_bound,
-                             choice_out, headroom_out, ws, s);
+      return launch_snapshot(D, H, K, kmax, cap, Q, J, cand_prompt, cand_bound, choice_out,
+                             headroom_out, ws, s);
     case MAPS_MODE_SEQUENTIAL: {
       // a private summary of K (also validating K >= 0); updated in place
       Carve cv(ws);

@@ -31,9 +31,9 @@
 #include <cooperative_groups.h>
 
 #include "maps_internal.cuh"
+#include "maps_bench.h"
 
 #include <algorithm>
-#include <mutex>
 
 namespace cg = cooperative_groups;
 
@@ -52,6 +52,12 @@ constexpr int kDecSmem = 8192;  // decoders counted in shared memory up to this 
 constexpr uint32_t kFlagAgg = 1, kFlagInc = 2;
 
 enum : int32_t { kBufA = 0, kBufB = 1, kHiIdentity = 2, kPermOut = 2 };
+
+// Test aid (maps_test_withhold_lookback): a tile of the global form's passes
+// that publishes nothing to the look-back (-1: none), and the polls a
+// look-back wait makes before it gives up.
+__device__ int32_t g_withheld_tile = -1;
+__device__ uint32_t g_lookback_spins = kSpinLimit;
 
 struct OrderCounts {
   uint32_t h[kPasses][kRadix];
@@ -1223,18 +1229,24 @@ __device__ bool order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
     }
     sm.tile_cnt[tid] = run;
     const size_t me = static_cast<size_t>(tile) * kRadix + tid;
+    const bool publish = tile != g_withheld_tile;  // always, outside the test aid
+    const uint32_t spin_limit = g_lookback_spins;
     st_nxt[me] = 0ull;
-    st_release_u64(&st_cur[me], static_cast<unsigned long long>(run) |
-                                    (static_cast<unsigned long long>(tile == 0 ? kFlagInc : kFlagAgg) << 62));
+    if (publish)
+      st_release_u64(&st_cur[me], static_cast<unsigned long long>(run) |
+                                      (static_cast<unsigned long long>(tile == 0 ? kFlagInc : kFlagAgg) << 62));
     unsigned long long excl = 0;
     if (tile > 0) {
       for (int q = tile - 1;; --q) {
         unsigned long long v;
         uint32_t spins = 0;
         while (((v = ld_acquire_u64(&st_cur[static_cast<size_t>(q) * kRadix + tid])) >> 62) == 0) {
-          if (++spins > kSpinLimit) {
+          if (++spins > spin_limit) {
+            // give up: count the rest as empty.  The offsets then only come
+            // out smaller than the true ones, so every write of the pass
+            // stays inside [0, N); the order is wrong and the call reports it.
             flag_error(status, MAPS_E_TIMEOUT);
-            v = static_cast<unsigned long long>(kFlagInc) << 62;  // give up
+            v = static_cast<unsigned long long>(kFlagInc) << 62;
             break;
           }
           __nanosleep(32);
@@ -1242,7 +1254,8 @@ __device__ bool order_pass_body(int p, int64_t N, const OrderPlan *plan, unsigne
         excl += v & ((1ull << 62) - 1);
         if ((v >> 62) == kFlagInc || q == 0) break;
       }
-      st_release_u64(&st_cur[me], (excl + run) | (static_cast<unsigned long long>(kFlagInc) << 62));
+      if (publish)
+        st_release_u64(&st_cur[me], (excl + run) | (static_cast<unsigned long long>(kFlagInc) << 62));
     }
     sm.excl[tid] = static_cast<uint32_t>(excl);
   }
@@ -1536,24 +1549,16 @@ constexpr int32_t kStaticMaxD = 4096;   // decoders
 constexpr size_t kStaticBytes = size_t(3) << 20;
 static __device__ __align__(256) unsigned char g_order_scratch[kStaticBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_static_mu;
-void *g_static_ptr[kMaxDevices] = {};
-
-// Device address of the static scratch on the current device, looked up once
-// per device (the host-side symbol is not a device address).
+// Device address of the static scratch on the current device.  The host-side
+// symbol is not a device address; the lookup is a cheap host call, made on
+// every call so that a reset device or a new context is never handed an old
+// address.  The first call on a device also loads the library's device code
+// there if that has not happened yet.
 int static_scratch(void **out) {
-  int dev = 0;
-  MAPS_TRY(cuda_ok(cudaGetDevice(&dev)));
-  if (dev < 0 || dev >= kMaxDevices) return MAPS_E_INVALID;
-  std::lock_guard<std::mutex> lock(g_static_mu);
-  if (g_static_ptr[dev] == nullptr) {
-    void *p = nullptr;
-    MAPS_TRY(cuda_ok(cudaGetSymbolAddress(&p, g_order_scratch)));
-    if (p == nullptr || !aligned(p, kAlign)) return MAPS_E_CUDA;
-    g_static_ptr[dev] = p;
-  }
-  *out = g_static_ptr[dev];
+  void *p = nullptr;
+  MAPS_TRY(cuda_ok(cudaGetSymbolAddress(&p, g_order_scratch)));
+  if (p == nullptr || !aligned(p, kAlign)) return MAPS_E_CUDA;
+  *out = p;
   return MAPS_OK;
 }
 
@@ -1582,5 +1587,13 @@ extern "C" int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
     *status_host = maps_check(ws, stream);
     return *status_host;
   }
+  return MAPS_OK;
+}
+
+extern "C" int maps_test_withhold_lookback(int32_t tile, uint32_t spin_limit) {
+  using namespace maps;
+  const uint32_t spins = spin_limit == 0 ? kSpinLimit : spin_limit;
+  MAPS_TRY(cuda_ok(cudaMemcpyToSymbol(g_withheld_tile, &tile, sizeof(tile))));
+  MAPS_TRY(cuda_ok(cudaMemcpyToSymbol(g_lookback_spins, &spins, sizeof(spins))));
   return MAPS_OK;
 }

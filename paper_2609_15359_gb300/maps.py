@@ -25,7 +25,6 @@ MODE_SNAPSHOT = 0
 MODE_SEQUENTIAL = 1
 MODE_ALG1_SNAPSHOT = 2
 MODE_ALG1_SEQUENTIAL = 3
-MODE_SNAPSHOT_BINNED = 4
 
 STATUS_NAMES = {0: "MAPS_OK", -1: "MAPS_E_INVALID", -2: "MAPS_E_RANGE",
                 -3: "MAPS_E_UNBOUNDED", -4: "MAPS_E_TIMEOUT", -5: "MAPS_E_CUDA",
@@ -60,7 +59,7 @@ def _load():
         "maps_last_cuda_error": ([], ctypes.c_int),
         "maps_check": ([vp, vp], ctypes.c_int),
         "maps_set_dispatch_events": ([vp, vp], ctypes.c_int),
-        "maps_dispatch_bin": ([i32, i32, i64, vp, vp, vp, vp, vp, sz, vp], ctypes.c_int),
+        "maps_test_withhold_lookback": ([i32, u32], ctypes.c_int),
         "maps_calibrate_workspace_size": ([i64, i64], sz),
         "maps_calibrate": ([vp, vp, i64, u32, vp, i64, vp, vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_project_occupancy_workspace_size": ([i32, i32, i64], sz),
@@ -84,9 +83,10 @@ def _load():
 
 lib = _load()
 EXPORTS = ("maps_version", "maps_last_cuda_error", "maps_check", "maps_set_dispatch_events",
+           "maps_test_withhold_lookback",
            "maps_calibrate_workspace_size", "maps_calibrate",
            "maps_project_occupancy_workspace_size", "maps_project_occupancy",
-           "maps_dispatch_workspace_size", "maps_dispatch", "maps_dispatch_bin",
+           "maps_dispatch_workspace_size", "maps_dispatch",
            "maps_order_local_workspace_size", "maps_order_local", "maps_order_local_static",
            "maps_stream_workspace_size", "maps_stream_run")
 
@@ -191,19 +191,6 @@ def maps_dispatch(mode: int, D: int, H: int, S: int, K, cap, Q, cand_prompt, can
                              _ptr(cand_bound, torch.int32), _ptr(choice_out, torch.int32),
                              _ptr(headroom_out, torch.int64), ws.ptr, ws.nbytes,
                              _stream(stream))
-
-
-def maps_dispatch_bin(D: int, H: int, cand_prompt, cand_bound, choice_out, headroom_out=None,
-                      ws: Workspace | None = None, stream=None) -> int:
-    """The candidate bucketing of a SNAPSHOT dispatch, ahead of K; a later
-    maps_dispatch(MODE_SNAPSHOT_BINNED, ...) on the same workspace scores them."""
-    J = cand_prompt.numel()
-    ws = ws or Workspace()
-    ws.ensure(lib.maps_dispatch_workspace_size(MODE_SNAPSHOT, D, H, J))
-    return lib.maps_dispatch_bin(D, H, J, _ptr(cand_prompt, torch.int32),
-                                 _ptr(cand_bound, torch.int32), _ptr(choice_out, torch.int32),
-                                 _ptr(headroom_out, torch.int64), ws.ptr, ws.nbytes,
-                                 _stream(stream))
 
 
 def maps_order_local(D: int, dec, bound, wait, arrival, max_wait: int, perm_out, seg_off_out,

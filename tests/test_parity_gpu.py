@@ -377,15 +377,17 @@ def test_dispatch_snapshot_workloads(M, ws, oracle, name, variant):
 
 
 @pytest.mark.parametrize("variant", ["given", "feasible", "diverse"])
-def test_dispatch_snapshot_large_sampled(M, ws, oracle, variant):
-    """Full-size run on the GPU in the benchmark's launch configuration;
-    the oracle scores a sample of the candidates one by one."""
+def test_dispatch_snapshot_large_full(M, ws, oracle, variant):
+    """Full size, in the benchmark's launch configuration: every one of the
+    65,536 candidates against the plain oracle (pinned to the by-definition
+    one in test_oracle_tier_p.py), and a sample of them against the
+    by-definition oracle itself."""
     w = W.make("large", feasible=(variant == "feasible"))
     D, H, J = w["D"], w["H"], w["J"]
     q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
     U = oracle.bound(w["res_pred"], q)[1]
     cb = oracle.bound(w["cand_pred"], q)[1]
-    _, K = oracle.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U)
+    _, K = oracle.p_occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U)
     cap, Q = w["cap"], w["Q"]
     rng = np.random.default_rng(5)
     if variant == "diverse":
@@ -393,11 +395,13 @@ def test_dispatch_snapshot_large_sampled(M, ws, oracle, variant):
         Q = rng.integers(0, 3, D).astype(np.int32)
     st, ch, hr, _, _ = gpu_dispatch(M, ws, 0, D, H, 1, K, cap, Q, w["cand_prompt"], cb,
                                     kmax=kmax_of(K))
-    assert st == 0
-    assert ch.min() >= 0 and ch.max() < D
+    stp, cp_, hp_ = oracle.p_dispatch_snapshot(D, H, K, cap, Q, w["cand_prompt"], cb)
+    assert st == stp == 0
+    assert np.array_equal(ch, cp_)
+    assert np.array_equal(hr, hp_)
     st2, ch2, hr2, _, _ = gpu_dispatch(M, ws, 0, D, H, 1, K, cap, Q, w["cand_prompt"], cb)
     assert st2 == 0 and np.array_equal(ch, ch2) and np.array_equal(hr, hr2)
-    idx = np.concatenate([np.argsort(cb)[-64:], rng.choice(J, 1500, replace=False)])
+    idx = np.concatenate([np.argsort(cb)[-32:], rng.choice(J, 300, replace=False)])
     sto, co, ho, _, _ = oracle.dispatch(0, D, H, 1, K, cap, Q, w["cand_prompt"][idx], cb[idx])
     assert sto == 0
     assert np.array_equal(ch[idx], co)
@@ -417,7 +421,7 @@ def test_dispatch_sequential_random(M, ws, oracle, D, H, J):
     check_dispatch(M, ws, oracle, 1, D, H, K, cap, Q, cp, cb)
 
 
-@pytest.mark.parametrize("name", ["tiny", "d16"])
+@pytest.mark.parametrize("name", ["tiny", "d16", "d64"])
 def test_dispatch_sequential_workloads(M, ws, oracle, name):
     w = W.make(name, feasible=True)
     q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
@@ -439,9 +443,8 @@ def test_dispatch_alg1_workloads(M, ws, oracle, name, S):
     cap = (w["cap"].astype(np.int64) // 2 + rng.integers(0, w["cap"].max() // 8, w["D"])).astype(np.int32)
     Q = rng.integers(0, 3, w["D"]).astype(np.int32)
     co, ho = check_dispatch(M, ws, oracle, 2, w["D"], w["H"], None, cap, Q, w["cand_prompt"], cb, S, res)
-    if name != "large":
-        J = min(w["J"], 2048)
-        check_dispatch(M, ws, oracle, 3, w["D"], w["H"], None, cap, Q, w["cand_prompt"][:J], cb[:J], S, res)
+    # SEQUENTIAL over every candidate (65,536 reservations in order at Large)
+    check_dispatch(M, ws, oracle, 3, w["D"], w["H"], None, cap, Q, w["cand_prompt"], cb, S, res)
 
 
 def test_dispatch_errors(M, ws, oracle):
@@ -559,34 +562,9 @@ def test_order_workload_pipeline(M, ws, oracle, name, one_queue):
     assert np.array_equal(perm, po) and np.array_equal(seg, so)
 
 
-@pytest.mark.parametrize("name,feasible", [("tiny", True), ("tiny", False), ("d16", True),
-                                           ("d16", False)])
-def test_dispatch_binned(M, oracle, name, feasible):
-    """maps_dispatch_bin, then the binned SNAPSHOT on the same workspace, equals
-    SNAPSHOT."""
-    w = W.make(name, feasible=feasible)
-    D, H = w["D"], w["H"]
-    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
-    U = oracle.bound(w["res_pred"], q)[1]
-    cb = oracle.bound(w["cand_pred"], q)[1]
-    _, K = oracle.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U)
-    J = len(cb)
-    dws = M.Workspace(M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, D, H, J),
-                      torch.device("cuda"))
-    cp_d, cb_d = dev(w["cand_prompt"], np.int32), dev(cb, np.int32)
-    ch = torch.full((J,), -9, dtype=torch.int32, device="cuda")
-    hr = torch.full((J,), -9, dtype=torch.int64, device="cuda")
-    assert M.maps_dispatch_bin(D, H, cp_d, cb_d, ch, hr, ws=dws) == 0
-    st = M.maps_dispatch(M.MODE_SNAPSHOT_BINNED, D, H, 1, dev(K, np.int32), dev(w["cap"], np.int32),
-                         dev(w["Q"], np.int32), cp_d, cb_d, ch, hr, ws=dws)
-    assert st == 0 and M.maps_check(dws) == 0
-    _, cho, hro, _, _ = oracle.dispatch(0, D, H, 1, K, w["cap"], w["Q"], w["cand_prompt"], cb)
-    assert np.array_equal(host(ch), cho) and np.array_equal(host(hr), hro)
-
-
-def test_dispatch_binned_invalid_candidates(M, oracle):
-    """Candidates with a negative prompt or bound: the bucketing call writes -1 and
-    records MAPS_E_RANGE, as SNAPSHOT does; the others are still decided."""
+def test_dispatch_snapshot_invalid_candidates(M, ws, oracle):
+    """Candidates with a negative prompt or bound get choice -1 and headroom 0
+    and record MAPS_E_RANGE; the others are still decided."""
     w = W.make("tiny", feasible=True)
     D, H = w["D"], w["H"]
     q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
@@ -595,40 +573,32 @@ def test_dispatch_binned_invalid_candidates(M, oracle):
     cp = w["cand_prompt"].copy()
     cp[3], cb[7] = -1, -5
     _, K = oracle.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U)
-    J = len(cb)
-    dws = M.Workspace(M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, D, H, J),
-                      torch.device("cuda"))
-    ch = torch.full((J,), -9, dtype=torch.int32, device="cuda")
-    hr = torch.full((J,), -9, dtype=torch.int64, device="cuda")
-    cp_d, cb_d = dev(cp, np.int32), dev(cb, np.int32)
-    assert M.maps_dispatch_bin(D, H, cp_d, cb_d, ch, hr, ws=dws) == 0
-    assert M.maps_dispatch(M.MODE_SNAPSHOT_BINNED, D, H, 1, dev(K, np.int32), dev(w["cap"], np.int32),
-                           dev(w["Q"], np.int32), cp_d, cb_d, ch, hr, ws=dws) == 0
-    assert M.maps_check(dws) == M.MAPS_E_RANGE
+    st, ch, hr, _, _ = gpu_dispatch(M, ws, M.MODE_SNAPSHOT, D, H, 1, K, w["cap"], w["Q"], cp, cb)
     sto, cho, hro, _, _ = oracle.dispatch(0, D, H, 1, K, w["cap"], w["Q"], cp, cb)
-    assert sto == M.MAPS_E_RANGE
-    assert np.array_equal(host(ch), cho) and np.array_equal(host(hr), hro)
+    assert st == sto == M.MAPS_E_RANGE
+    assert np.array_equal(ch, cho) and np.array_equal(hr, hro)
 
 
-def test_dispatch_binned_without_buckets(M):
-    """A binned call on a workspace that holds no buckets of its candidates reads
-    none of them and records MAPS_E_INVALID."""
-    D, H, J = 8, 4096, 300
-    dws = M.Workspace(M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, D, H, J),
-                      torch.device("cuda"))
-    rng = np.random.default_rng(3)
-    K = dev(rng.integers(0, 1000, (D, H)), np.int32)
-    cap, Q = dev(np.full(D, 10**6), np.int32), dev(np.zeros(D), np.int32)
-    cp, cb = dev(rng.integers(1, 100, J), np.int32), dev(rng.integers(1, H, J), np.int32)
-    ch = torch.full((J,), -9, dtype=torch.int32, device="cuda")
-    # never bucketed (a zeroed workspace)
-    assert M.maps_dispatch(M.MODE_SNAPSHOT_BINNED, D, H, 1, K, cap, Q, cp, cb, ch, ws=dws) == 0
-    assert M.maps_check(dws) == M.MAPS_E_INVALID
-    assert (host(ch) == -9).all()
-    # bucketed for other candidates (J differs)
-    assert M.maps_dispatch_bin(D, H, cp[:200], cb[:200], ch[:200], ws=dws) == 0
-    assert M.maps_dispatch(M.MODE_SNAPSHOT_BINNED, D, H, 1, K, cap, Q, cp, cb, ch, ws=dws) == 0
-    assert M.maps_check(dws) == M.MAPS_E_INVALID
+def test_dispatch_kmax_checked_against_K(M, ws, oracle):
+    """A caller's 16-step summary is compared with K at four blocks of every
+    row: the summary of K itself passes, one that disagrees with K in the first
+    block of a row is MAPS_E_INVALID."""
+    w = W.make("d16", feasible=True)
+    D, H = w["D"], w["H"]
+    q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])[1]
+    U = oracle.bound(w["res_pred"], q)[1]
+    cb = oracle.bound(w["cand_pred"], q)[1]
+    _, K = oracle.occupancy(D, H, w["res_off"], w["res_prompt"], w["res_gen"], U)
+    km = kmax_of(K)
+    st, ch, hr, _, _ = gpu_dispatch(M, ws, M.MODE_SNAPSHOT, D, H, 1, K, w["cap"], w["Q"],
+                                    w["cand_prompt"], cb, kmax=km)
+    _, cho, hro, _, _ = oracle.dispatch(0, D, H, 1, K, w["cap"], w["Q"], w["cand_prompt"], cb)
+    assert st == 0 and np.array_equal(ch, cho) and np.array_equal(hr, hro)
+    bad = km.copy()
+    bad[5, 0] += 1
+    st, _, _, _, _ = gpu_dispatch(M, ws, M.MODE_SNAPSHOT, D, H, 1, K, w["cap"], w["Q"],
+                                  w["cand_prompt"], cb, kmax=bad)
+    assert st == M.MAPS_E_INVALID
 
 
 def test_dispatch_scoring_events(M, ws, oracle):

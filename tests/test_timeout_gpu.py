@@ -1,0 +1,46 @@
+"""A bounded device wait that runs out is reported, and the device stays usable.
+
+The local order's global form (arrival not in index order) sorts with
+decoupled look-back between tiles: each tile waits, bounded, for its
+predecessors' published counts.  The test aid maps_test_withhold_lookback
+makes one tile publish nothing, so the next tile's wait runs out after a short
+limit.  The call must then report MAPS_E_TIMEOUT through maps_check, write
+only inside its outputs, and the next call on a fresh workspace must give the
+oracle's order exactly.  Nothing faults, traps or hangs.
+"""
+import numpy as np
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+
+def test_order_lookback_timeout_is_reported_and_the_next_call_is_exact(oracle):
+    if not torch.cuda.is_available():
+        pytest.fail("CUDA device required")
+    from paper_2609_15359_gb300 import maps as M
+    rng = np.random.default_rng(11)
+    N, D, mw = 200_000, 64, 1000
+    dec = rng.integers(0, D, N).astype(np.int32)
+    U = rng.integers(0, 40000, N).astype(np.int32)
+    wait = rng.integers(0, 3000, N).astype(np.int32)
+    arr = rng.integers(0, 2**31 - 1, N, dtype=np.int64).astype(np.int32)  # not in index order
+    ins = [torch.from_numpy(x).cuda() for x in (dec, U, wait, arr)]
+    perm = torch.full((N,), -1, dtype=torch.int32, device="cuda")
+    seg = torch.full((D + 1,), -1, dtype=torch.int64, device="cuda")
+    ws = M.Workspace()
+    try:
+        assert M.lib.maps_test_withhold_lookback(3, 2000) == 0
+        assert M.maps_order_local(D, *ins, mw, perm, seg, ws=ws) == 0
+        assert M.maps_check(ws) == M.MAPS_E_TIMEOUT
+    finally:
+        assert M.lib.maps_test_withhold_lookback(-1, 0) == 0
+    p = perm.cpu().numpy()
+    assert p.min() >= -1 and p.max() < N  # written only inside the output
+    sto, po, so = oracle.order_local(D, dec, U, wait, arr, mw)
+    ws2 = M.Workspace()
+    perm.fill_(-1)
+    assert M.maps_order_local(D, *ins, mw, perm, seg, ws=ws2) == 0
+    assert M.maps_check(ws2) == 0 and sto == 0
+    assert np.array_equal(perm.cpu().numpy(), po)
+    assert np.array_equal(seg.cpu().numpy(), so)

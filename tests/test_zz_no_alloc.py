@@ -3,9 +3,12 @@
 Callers that cannot allocate device memory -- a scheduler inside a process
 whose allocator it does not own, or one that must not allocate while
 serving -- use this entry point: its scratch is an array compiled into the
-library.  It must give exactly what maps_order_local gives with a caller
-workspace, call after call (the array keeps the previous call's contents).
-Named to be collected last.
+library.  Call after call it must give the oracle's order exactly, although
+the array keeps the previous call's contents.  The cases alternate between
+the one-block form and the multi-kernel forms (counters, look-back state and
+plan carved from the array), so every multi-kernel call but the first reuses
+state a larger call left behind; one case has more than 1,024 decoders (the
+scatter that claims slots by atomics).  Named to be collected last.
 """
 import ctypes
 
@@ -24,44 +27,57 @@ def _inputs(rng, N, D, sorted_arrival):
         arr = np.arange(N, dtype=np.int32)
     else:
         arr = rng.integers(0, 2**31 - 1, N, dtype=np.int64).astype(np.int32)
-    return [torch.from_numpy(x).cuda() for x in (dec, U, wait, arr)]
+    return dec, U, wait, arr
 
 
-def _reference(M, D, ins, mw):
+def _static(M, D, host_ins, mw):
+    ins = [torch.from_numpy(x).cuda() for x in host_ins]
     N = ins[0].numel()
-    perm = torch.full((N,), -1, dtype=torch.int32, device="cuda")
-    seg = torch.full((D + 1,), -1, dtype=torch.int64, device="cuda")
-    ws = M.Workspace()
-    assert M.maps_order_local(D, *ins, mw, perm, seg, ws=ws) == 0
-    assert M.maps_check(ws) == 0
-    return perm.cpu().numpy(), seg.cpu().numpy()
-
-
-def _static(M, D, ins, mw):
-    N = ins[0].numel()
-    perm = torch.full((N,), -1, dtype=torch.int32, device="cuda")
+    perm = torch.full((max(N, 1),), -1, dtype=torch.int32, device="cuda")
     seg = torch.full((D + 1,), -1, dtype=torch.int64, device="cuda")
     st = ctypes.c_int32(-99)
     rc = M.lib.maps_order_local_static(N, D, M._ptr(ins[0]), M._ptr(ins[1]), M._ptr(ins[2]),
                                        M._ptr(ins[3]), mw, M._ptr(perm), M._ptr(seg),
                                        ctypes.byref(st), M._stream(None))
-    assert rc == 0 and st.value == 0
     torch.cuda.synchronize()
-    return perm.cpu().numpy(), seg.cpu().numpy()
+    return rc, st.value, perm[:N].cpu().numpy(), seg.cpu().numpy()
 
 
-def test_static_order_matches_workspace_order_on_consecutive_calls():
+# (N, D, arrival in index order, max_wait): one-block and multi-kernel forms
+# alternate; consecutive multi-kernel calls of different sizes and forms
+CASES = [(65536, 256, False, 1000), (3000, 7, True, 500), (20000, 2000, False, 800),
+         (65536, 256, True, 1000), (50000, 4096, True, 0), (4608, 4096, False, 300),
+         (40000, 3, False, 2000), (1, 1, True, 0)]
+
+
+def test_static_order_equals_the_oracle_on_consecutive_calls(oracle):
     if not torch.cuda.is_available():
         pytest.fail("CUDA device required")
     from paper_2609_15359_gb300 import maps as M
     rng = np.random.default_rng(42)
-    cases = [(65536, 256, False, 1000), (3000, 7, True, 500)]
-    for N, D, srt, mw in cases:  # two calls in a row on the shared array
-        ins = _inputs(rng, N, D, srt)
-        p_ref, s_ref = _reference(M, D, ins, mw)
-        p_st, s_st = _static(M, D, ins, mw)
-        assert np.array_equal(p_st, p_ref)
-        assert np.array_equal(s_st, s_ref)
+    for N, D, srt, mw in CASES:
+        host_ins = _inputs(rng, N, D, srt)
+        sto, po, so = oracle.order_local(D, *host_ins, mw)
+        rc, st, perm, seg = _static(M, D, host_ins, mw)
+        assert rc == 0 and st == 0 and sto == 0, (N, D, rc, st)
+        assert np.array_equal(perm, po), (N, D)
+        assert np.array_equal(seg, so), (N, D)
+
+
+def test_static_order_reports_a_data_error_then_recovers(oracle):
+    """A decoder index out of range is MAPS_E_RANGE through status_host; the
+    next call on the same array starts from a clear status and is exact."""
+    from paper_2609_15359_gb300 import maps as M
+    rng = np.random.default_rng(7)
+    dec, U, wait, arr = _inputs(rng, 20000, 300, True)
+    bad = dec.copy()
+    bad[123] = 300
+    rc, st, _, _ = _static(M, 300, (bad, U, wait, arr), 1000)
+    assert st == M.MAPS_E_RANGE
+    sto, po, so = oracle.order_local(300, dec, U, wait, arr, 1000)
+    rc, st, perm, seg = _static(M, 300, (dec, U, wait, arr), 1000)
+    assert rc == 0 and st == 0 and sto == 0
+    assert np.array_equal(perm, po) and np.array_equal(seg, so)
 
 
 def test_static_order_rejects_sizes_beyond_its_array():
