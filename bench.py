@@ -15,15 +15,19 @@ Timing: inputs resident in HBM; before every step the L2 is flushed (a
 host enqueues the step, so CUDA events on the launching stream bracket the
 device time of the step alone.  Each timed step replays one CUDA graph of the
 four calls; a second pass of direct launches with an event between calls
-gives the per-call split (and the rooflines), and a third times the
-dispatch's scoring kernel alone (events recorded by maps_dispatch around it).  The end-to-end figure repeats the step
-through the same C-ABI calls with pinned host buffers, host-to-device copies
-of every input and device-to-host copies of every output inside the timed
-region; steps are pipelined over two buffer sets, each stage replayed from a
-CUDA graph.
+gives the per-call split (and the rooflines), a third times the dispatch's
+scoring kernel alone (events recorded by maps_dispatch around it), a fourth
+the dispatch call on the feasible-regime capacities (x64, so that candidates
+fit and its min-Q branch runs), and a fifth a plain write of K, the floor
+of the occupancy call under this protocol.  The end-to-end figure repeats the
+step through the same C-ABI calls with pinned host buffers, host-to-device
+copies of every input and device-to-host copies of every output inside the
+timed region; steps are pipelined over two buffer sets, each stage replayed
+from a CUDA graph.
 
---impl reference runs the CPU oracle on the host cores over a bounded
-sample of the same workload and prints the same metric.
+The CPU baseline is the plain (tier-P) oracle on whole steps of the same
+workload, on every host core and on one.  --impl reference times it the
+same way (whole steps, every host core) and prints the same metric.
 Multi-GPU (torchrun): every rank runs an independent replica (its own
 scheduler instance with its own seed); there is no collective on the data
 path.  The value is all ranks' decisions over the slowest rank's time.
@@ -55,6 +59,7 @@ L2_FLUSH_BYTES = 256 << 20
 # kernels, one launch each; dispatch_scoring is the scoring kernel alone),
 # valid only for the kernel source it was taken on.
 TRAFFIC = {
+    "dispatch_feasible": {"bytes": 0, "source": "dispatch.cu", "source_sha256": ""},
     "calibrate": {"bytes": 12578673, "source": "calibrate.cu", "source_sha256":
                   "2c2d7dd3d182439cc27caeb6ae856327284afa160f2de0b32e84a119acd45be6"},
     "occupancy": {"bytes": 29642638, "source": "occupancy.cu", "source_sha256":
@@ -73,6 +78,8 @@ KERNELS = {
     "order": "order_prep + order_keys + order_segsort + order_finish (maps_order_local)",
     "dispatch_scoring": "dispatch_snapshot_kernel alone (maps_dispatch's scoring kernel, after "
                         "the candidates are bucketed by horizon tile)",
+    "dispatch_feasible": "maps_dispatch SNAPSHOT on the feasible-regime capacities (x64): carry "
+                         "scan + bin count, bin scatter, scoring with queue-ordered prefix maxima",
 }
 
 
@@ -245,6 +252,10 @@ class Step:
         self.cal_true, self.cal_pred, self.pred_all = v["cal_true"], v["cal_pred"], v["pred_all"]
         self.res_off, self.res_prompt, self.res_gen = v["res_off"], v["res_prompt"], v["res_gen"]
         self.cap, self.Q0, self.cand_prompt = v["cap"], v["Q0"], v["cand_prompt"]
+        # the feasible regime: the same workload with every capacity x64, so
+        # that candidates fit and the dispatch takes its min-Q branch
+        factor = W_CONFIG_FACTOR(w)
+        self.cap_feasible = (self.cap.to(torch.int64) * factor).to(torch.int32)
         self.wait_all, self.arrival, self.dec_all = v["wait_all"], v["arrival"], v["dec_all"]
         # outputs / intermediates
         self.U_all = torch.empty(R + J, dtype=torch.int32, device=device)
@@ -289,10 +300,23 @@ class Step:
                                 self.w["max_wait"], self.perm, self.seg, ws=self.ws)
         assert st == 0, st
 
+    def dispatch_feasible(self):
+        """The step's SNAPSHOT dispatch alone, on the feasible-regime capacities."""
+        M = self.M
+        st = M.maps_dispatch(M.MODE_SNAPSHOT, self.D, self.H, 1, self.K, self.cap_feasible, self.Q0,
+                             self.cand_prompt, self.U_all[self.R:], self.choice, self.headroom,
+                             kmax=self.kmax, ws=self.ws)
+        assert st == 0, st
+
     def check(self):
         st = self.M.maps_check(self.ws)
         if st != 0:
             raise RuntimeError(f"device status {st}")
+
+
+def W_CONFIG_FACTOR(w: dict) -> int:
+    from paper_2609_15359_gb300 import workloads as W
+    return int(W.WORKLOADS[WORKLOAD]["feasible_factor"])
 
 
 def host_inputs(w):
@@ -462,6 +486,25 @@ def bench_gpu(args, world, rank, local, dist):
         step.M.maps_set_dispatch_events(evs[i][0], evs[i][1])
         step.run()
     step.M.maps_set_dispatch_events(None, None)
+    # pass D (the feasible regime): the dispatch call alone, after a full step
+    # (so that K, the summary and the bounds are the step's), capacities x64
+    step.run()
+    evf = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(Kb)]
+    for i in range(Kb):
+        flush.zero_()
+        torch.cuda._sleep(sleep_cycles)
+        evf[i][0].record()
+        step.dispatch_feasible()
+        evf[i][1].record()
+    # pass E (the floor of the occupancy call): a plain write of K alone after
+    # the same flush, timed the same way
+    evk = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(Kb)]
+    for i in range(Kb):
+        flush.zero_()
+        torch.cuda._sleep(sleep_cycles)
+        evk[i][0].record()
+        step.K.zero_()
+        evk[i][1].record()
     torch.cuda.synchronize()
     clocks = sampler.stop()
     if dist is not None and dist.is_initialized():
@@ -474,6 +517,8 @@ def bench_gpu(args, world, rank, local, dist):
     cal_ms = [evb[i][3].elapsed_time(evb[i][0]) for i in range(Kb)]
     order_ms = [evb[i][2].elapsed_time(evb[i][4]) for i in range(Kb)]
     score_ms = [evs[i][0].elapsed_time(evs[i][1]) for i in range(Kb)]
+    feas_ms = [evf[i][0].elapsed_time(evf[i][1]) for i in range(Kb)]
+    kwrite_ms = [evk[i][0].elapsed_time(evk[i][1]) for i in range(Kb)]
     local_s = sum(step_ms) / 1e3
     max_s, units = aggregate(local_s, float(K * step.J), dist)
 
@@ -524,6 +569,8 @@ def bench_gpu(args, world, rank, local, dist):
     # kernel roofline of the scoring step is defined
     alg["dispatch_scoring"] = alg["dispatch"]
     call_ms["dispatch_scoring"] = score_ms
+    alg["dispatch_feasible"] = alg["dispatch"]
+    call_ms["dispatch_feasible"] = feas_ms
     rooflines = {}
     for c in alg:
         avg = float(np.mean(call_ms[c])) / 1e3
@@ -571,7 +618,16 @@ def bench_gpu(args, world, rank, local, dist):
                             "results read back on another stream; each stage launched as "
                             f"{how}",
                 "stage_us_alone": stage_us},
-        "gpu_launches": step.kernels_per_step * (K + 2 * Kb),  # the three passes of the timed region
+        # our kernels in the timed region: passes A-C and the step before pass
+        # D run the whole path; pass D runs the dispatch's three kernels
+        "gpu_launches": step.kernels_per_step * (K + 2 * Kb + 1) + 3 * Kb,
+        "occupancy_floor": {
+            "K_write_us": float(np.mean(kwrite_ms)) * 1e3,
+            "what": "a plain write of K alone (67.1 MB, one fill kernel) after the same flush, "
+                    "event-timed like the calls; the occupancy call writes K (and the 4.2 MB "
+                    "summary) and also reads the residents (12.6 MB)",
+            "frac_if_the_call_took_only_this": alg["occupancy"] / (float(np.mean(kwrite_ms)) / 1e3)
+                                               / 1e9 / peaks["hbm_gbs"]},
         "clocks": clocks,
     }
     return result, w
@@ -633,68 +689,98 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
 # the CPU oracle as the baseline / reference arm
 # ---------------------------------------------------------------------------
 
-def oracle_step(w: dict, n_dispatch: int, n_dec: int | None = None) -> tuple[float, int]:
-    """Runs the oracle over one step of the workload, sampled: only the first
-    n_dispatch candidates are dispatched and, with n_dec, only the first n_dec
-    decoders (and their residents) are projected and scored.  Calibration,
-    bounds and the local order run in full.  The projection grows linearly with
-    the decoders and the scoring with the decoders and the candidates, so their
-    times are scaled by D / n_dec and J / n_dispatch.  Returns (seconds
-    extrapolated to the whole step, candidates the extrapolation stands for)."""
-    import oracle as O
-    R, J, D, H = w["R"], w["J"], w["D"], w["H"]
-    Ds = D if n_dec is None else max(1, min(int(n_dec), D))
-    n_dispatch = max(1, min(int(n_dispatch), J))
-    Rs = int(w["res_off"][Ds])
-    a = w["alphas_ppm"][0]
-    t0 = time.perf_counter()
-    st, q = O.calibrate(w["cal_true"], w["cal_pred"], a)
-    st, U = O.bound(np.concatenate([w["res_pred"], w["cand_pred"]]), q)
-    t1 = time.perf_counter()
-    st, K = O.occupancy(Ds, H, w["res_off"][:Ds + 1], w["res_prompt"][:Rs], w["res_gen"][:Rs],
-                        U[:Rs])
-    t2 = time.perf_counter()
-    st, ch, _, _, _ = O.dispatch(0, Ds, H, 1, K, w["cap"][:Ds], w["Q"][:Ds],
-                                 w["cand_prompt"][:n_dispatch], U[R:R + n_dispatch])
-    t3 = time.perf_counter()
-    dec = np.concatenate([w["res_dec"], np.resize(ch, J).astype(np.int32)])
-    wait = np.concatenate([w["res_wait"], np.zeros(J, np.int32)])
-    st, perm, seg = O.order_local(D, dec, U, wait, np.arange(R + J, dtype=np.int32), w["max_wait"])
-    t4 = time.perf_counter()
-    scaled = ((t2 - t1) + (t3 - t2) * J / n_dispatch) * D / Ds
-    return (t1 - t0) + (t4 - t3) + scaled, J
+def cpu_info() -> dict:
+    """Host core count and CPU model (as lscpu reports them)."""
+    info = {"nproc": os.cpu_count()}
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            k, _, v = line.partition(":")
+            if k.strip() in ("Model name", "Vendor ID", "Architecture") and v.strip():
+                info[k.strip().lower().replace(" ", "_")] = v.strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return info
 
 
-def cpu_baseline(w: dict, n_dispatch: int = 8192) -> dict:
-    secs, J = oracle_step(w, n_dispatch)
-    return {"value": J / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": (f"full calibration, bounds, occupancy and order of the Large workload; "
-                       f"dispatch of the first {n_dispatch} of {J} candidates, its time scaled "
-                       f"by {J}/{n_dispatch}; single thread")}
+class OracleStep:
+    """One whole step of the Large workload through the plain (tier-P) CPU
+    oracle: calibration over all residuals, bounds of every resident and
+    candidate, occupancy of every decoder, SNAPSHOT dispatch of every
+    candidate, local order of every entry.  Output buffers are allocated once
+    and reused, as a scheduler keeps its buffers."""
+
+    def __init__(self, w: dict):
+        import oracle as O
+        self.O, self.w = O, w
+        self.K = np.empty((w["D"], w["H"]), dtype=np.int32)
+        self.perm = np.empty(w["R"] + w["J"], dtype=np.int32)
+        self.pred = np.concatenate([w["res_pred"], w["cand_pred"]])
+        self.wait = np.concatenate([w["res_wait"], np.zeros(w["J"], np.int32)])
+        self.arr = np.arange(w["R"] + w["J"], dtype=np.int32)
+
+    def run(self) -> float:
+        O, w, R = self.O, self.w, self.w["R"]
+        t0 = time.perf_counter()
+        st, q = O.p_calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])
+        st, U = O.p_bound(self.pred, q)
+        st, _ = O.p_occupancy(w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U[:R],
+                              out=self.K)
+        st, ch, _ = O.p_dispatch_snapshot(w["D"], w["H"], self.K, w["cap"], w["Q"],
+                                          w["cand_prompt"], U[R:])
+        dec = np.concatenate([w["res_dec"], ch])
+        st, _, _ = O.p_order_local(w["D"], dec, U, self.wait, self.arr, w["max_wait"],
+                                   out=self.perm)
+        return time.perf_counter() - t0
+
+
+def time_oracle(step: OracleStep, threads: int, n: int, warm: int = 1) -> tuple[float, int]:
+    """Mean seconds of n whole oracle steps on `threads` host threads (0: all
+    cores) after `warm` untimed ones; returns (seconds, threads used)."""
+    used = step.O.p_threads(threads)
+    for _ in range(warm):
+        step.run()
+    secs = [step.run() for _ in range(n)]
+    return float(np.mean(secs)), used
+
+
+def cpu_baseline(w: dict) -> dict:
+    """The plain CPU oracle timed on whole steps of the same workload, on every
+    host core and on one (a few steps each, about 10 s of CPU in all)."""
+    step = OracleStep(w)
+    s_all, cores = time_oracle(step, 0, 8)
+    s_one, _ = time_oracle(step, 1, 3)
+    step.O.p_threads(1)
+    J = w["J"]
+    return {"value": J / s_all, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": ("whole steps of the Large workload through the plain (tier-P) oracle: "
+                       "calibration of 1,000,000 residuals, bounds, occupancy of 256 decoders, "
+                       "SNAPSHOT dispatch of all 65,536 candidates, order of 1,114,112 entries; "
+                       f"mean of 8 steps on {cores} threads"),
+            "ms_per_step": s_all * 1e3,
+            "single_thread": {"value": J / s_one, "unit": UNIT, "cores": 1,
+                              "ms_per_step": s_one * 1e3, "steps": 3},
+            "host": cpu_info()}
 
 
 def bench_reference(args, world, rank):
+    """The reference arm: the plain CPU oracle on whole steps of the same
+    workload, every host core, exactly K timed steps after W untimed ones."""
     if rank != 0:
         return None
     from paper_2609_15359_gb300 import workloads as W
     import oracle
     oracle.build()
     w = W.make(WORKLOAD)
-    # Each step is a sample sized so that the whole run takes about 150 s of
-    # CPU: the calibration and order (about 0.4 s) run in full, the projection
-    # (about 1.2 s for all decoders) and the scoring (about 1.5 ms per
-    # candidate for all decoders) on the first n_dec decoders.
-    budget = 150.0 / max(1, args.steps + args.warmup)  # seconds per oracle step
-    n_dec = int(np.clip(w["D"] * budget / 10.0, 8, w["D"]))
-    n_dispatch = int(np.clip(512 * budget / 2.0, 64, 4096)) if n_dec == w["D"] else 256
+    step = OracleStep(w)
+    cores = oracle.p_threads(0)
     for _ in range(args.warmup):
-        oracle_step(w, 64, n_dec)
-    times = []
-    for _ in range(args.steps):
-        s, J = oracle_step(w, n_dispatch, n_dec)
-        times.append(s)
-    total = float(np.sum(times))
+        step.run()
+    total = float(np.sum([step.run() for _ in range(args.steps)]))
+    oracle.p_threads(1)
     value = args.steps * w["J"] / total
+    sample = (f"{args.steps} whole steps of the Large workload through the plain (tier-P) oracle "
+              f"on {cores} host threads, after {args.warmup} untimed ones")
     return {
         "metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": total / args.steps * 1e3,
@@ -703,11 +789,8 @@ def bench_reference(args, world, rank):
         "config": {"workload": "Large: D=256 decoders x 4,096 residents (1,048,576), capacity "
                                "524,288, H=65,536, 65,536 candidates, calibration n=1,000,000, "
                                "alpha=0.1"},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": (f"per step: full calibration, bounds and order; occupancy "
-                                    f"of the first {n_dec} of {w['D']} decoders and dispatch of "
-                                    f"{n_dispatch} of {w['J']} candidates to them, their times "
-                                    f"scaled to the whole workload")},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": sample, "host": cpu_info()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
