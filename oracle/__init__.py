@@ -17,6 +17,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.c")
+_SRC_RR = os.path.join(_HERE, "oracle_rr.c")
 _LIB = os.path.join(_HERE, "liboracle.so")
 
 MODE_SNAPSHOT, MODE_SEQUENTIAL, MODE_ALG1_SNAPSHOT, MODE_ALG1_SEQUENTIAL = 0, 1, 2, 3
@@ -31,11 +32,11 @@ def build(force: bool = False) -> str:
     tier-P oracle, C++17 -O2, with OpenMP where the compiler has it) with the
     host compilers."""
     if force or not os.path.exists(_LIB) or (
-            os.path.getmtime(_LIB) < max(os.path.getmtime(_SRC),
+            os.path.getmtime(_LIB) < max(os.path.getmtime(_SRC), os.path.getmtime(_SRC_RR),
                                          os.path.getmtime(os.path.join(_HERE, "oracle.h")))):
         tmp = _LIB + f".{os.getpid()}.tmp"
         subprocess.check_call(["gcc", "-O2", "-std=c11", "-shared", "-fPIC",
-                               "-o", tmp, _SRC])
+                               "-o", tmp, _SRC, _SRC_RR])
         os.replace(tmp, _LIB)
     if force or not os.path.exists(_LIB_P) or os.path.getmtime(_LIB_P) < os.path.getmtime(_SRC_P):
         tmp = _LIB_P + f".{os.getpid()}.tmp"
@@ -58,6 +59,11 @@ class StreamCfg(ctypes.Structure):
                 ("H", ctypes.c_int32), ("cap", ctypes.c_int32),
                 ("batch", ctypes.c_int32), ("window", ctypes.c_int32),
                 ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32)]
+
+
+class RRCfg(ctypes.Structure):
+    _fields_ = [("n_req", ctypes.c_int64), ("N", ctypes.c_int32), ("C", ctypes.c_int32),
+                ("t_tok_us", ctypes.c_int32), ("theta_ppm", ctypes.c_uint32)]
 
 
 def lib():
@@ -86,6 +92,8 @@ def lib():
                                          vp, vp, ctypes.c_int32, vp, vp]
         L.oracle_stream.argtypes = [ctypes.POINTER(StreamCfg), _i64p, _i32p,
                                     _i32p, _i32p, _i32p, _i32p, _i64p]
+        L.oracle_rr_pressure.argtypes = [ctypes.POINTER(RRCfg), _i64p, _i32p, _i32p,
+                                         _i64p, _i64p, _i64p, ctypes.POINTER(ctypes.c_int64)]
         _lib = L
     return _lib
 
@@ -196,6 +204,22 @@ def stream(N, D, H, cap, batch, window, alpha_ppm, max_wait, arrival_ms,
                              _c32(prompt[:N]), _c32(true_len[:N]),
                              _c32(pred[:N]), choice, q, stats)
     return st, choice, q, stats.reshape(nb, 4)
+
+
+def rr_pressure(N: int, C: int, t_tok_us: int, theta_ppm: int, arrival_us, prompt, out_len):
+    """The App. A round-robin simulation of one realisation.  Returns (status,
+    admit_us, done_us, stats [N][6] = T_hp, B_hp, C_hp, completed, longest
+    queue, total wait (times in microseconds), t_sim)."""
+    a, p, o = _c64(arrival_us), _c32(prompt), _c32(out_len)
+    n = a.shape[0]
+    cfg = RRCfg(n, N, C, t_tok_us, theta_ppm)
+    admit = np.zeros(n, dtype=np.int64)
+    done = np.zeros(n, dtype=np.int64)
+    stats = np.zeros(6 * N, dtype=np.int64)
+    tsim = ctypes.c_int64(0)
+    st = lib().oracle_rr_pressure(ctypes.byref(cfg), a, p, o, admit, done, stats,
+                                  ctypes.byref(tsim))
+    return st, admit, done, stats.reshape(N, 6), int(tsim.value)
 
 
 # ---------------------------------------------------------------------------

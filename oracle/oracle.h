@@ -91,6 +91,22 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                   const int32_t *pred, int32_t *choice_out, int32_t *q_out,
                   int64_t *stats_out);
 
+/* Round-robin KV-pressure simulation of App. A (oracle_rr.c). */
+typedef struct {
+    int64_t n_req;       /* requests, in arrival order */
+    int32_t N;           /* decoders (round robin over them) */
+    int32_t C;           /* KV-token capacity per decoder */
+    int32_t t_tok_us;    /* decode time per token, microseconds */
+    uint32_t theta_ppm;  /* high-pressure threshold * 1e6 */
+} oracle_rr_cfg;
+
+/* Outputs: admit_us[n_req], done_us[n_req]; stats[6d .. 6d+5] = T_hp,
+ * B_hp, C_hp, completed, longest queue, total wait of decoder d; *t_sim. */
+int oracle_rr_pressure(const oracle_rr_cfg *cfg, const int64_t *arrival_us,
+                       const int32_t *prompt, const int32_t *out_len,
+                       int64_t *admit_us, int64_t *done_us, int64_t *stats,
+                       int64_t *t_sim);
+
 #ifdef __cplusplus
 }
 #endif
