@@ -314,6 +314,53 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms,
                     int64_t *stats_out, void *ws, size_t ws_bytes,
                     void *stream);
 
+/* ------------------------------------------------------------------------
+ * Round-robin KV-pressure simulation and high-pressure interval metrics,
+ * App. A (Eq. kv_demand, the routing equation, Eq. admission, Definition
+ * of the high-pressure interval), for many workload realisations at once.
+ *
+ * Each realisation is n_req requests in arrival order.  Round robin sends
+ * request i to decoder i mod N.  A request holds M = prompt + out_len KV
+ * tokens while admitted; a decoder admits the head of its FIFO queue while
+ * K + M(head) <= C.  Service is processor sharing at one token per t_tok,
+ * taken at token granularity: a round gives each of the n admitted requests
+ * one token and lasts n * t_tok; completions and then admissions happen at
+ * round boundaries, and an idle decoder admits a request when it arrives.
+ * A decoder is under high pressure while K * 1e6 >= theta_ppm * C.  Times
+ * are integer microseconds.
+ *
+ *   cfg                 host struct (below).
+ *   n_real              realisations (>= 1).
+ *   arrival_us          [n_real][n_req] int64 arrival times, non-decreasing
+ *                       within a realisation.
+ *   prompt, out_len     [n_real][n_req] int32, prompt >= 0, out_len >= 1,
+ *                       prompt + out_len <= C.
+ *   admit_us, done_us   [n_real][n_req] int64 output: admission and
+ *                       completion time of every request.
+ *   stats               [n_real][N][6] int64 output per decoder: total time
+ *                       under high pressure T_hp, longest high-pressure
+ *                       interval B_hp, number of intervals C_hp, completed
+ *                       requests, longest waiting queue at an arrival, total
+ *                       waiting time (arrival to admission).
+ *   t_sim               [n_real] int64 output: first arrival to last
+ *                       completion (f_hp = T_hp / t_sim).
+ * Inputs outside the domain, or more than 1,536 requests admitted at once on
+ * one decoder, are MAPS_E_RANGE (via maps_check).
+ * ---------------------------------------------------------------------- */
+typedef struct {
+  int64_t n_req;       /* requests per realisation */
+  int32_t N;           /* decoders */
+  int32_t C;           /* KV-token capacity per decoder */
+  int32_t t_tok_us;    /* decode time per token, microseconds (>= 1) */
+  uint32_t theta_ppm;  /* high-pressure threshold, parts per million of C (1 .. 1e6) */
+} maps_rr_cfg;
+
+size_t maps_rr_pressure_workspace_size(const maps_rr_cfg *cfg, int64_t n_real);
+int maps_rr_pressure(const maps_rr_cfg *cfg, int64_t n_real, const int64_t *arrival_us,
+                     const int32_t *prompt, const int32_t *out_len, int64_t *admit_us,
+                     int64_t *done_us, int64_t *stats, int64_t *t_sim, void *ws,
+                     size_t ws_bytes, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

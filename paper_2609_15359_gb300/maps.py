@@ -40,6 +40,12 @@ class StreamCfg(ctypes.Structure):
                 ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32)]
 
 
+class RRCfg(ctypes.Structure):
+    """``maps_rr_cfg`` of include/maps.h."""
+    _fields_ = [("n_req", ctypes.c_int64), ("N", ctypes.c_int32), ("C", ctypes.c_int32),
+                ("t_tok_us", ctypes.c_int32), ("theta_ppm", ctypes.c_uint32)]
+
+
 class MapsError(RuntimeError):
     def __init__(self, status: int, what: str = ""):
         super().__init__(f"{what}: {STATUS_NAMES.get(status, status)}")
@@ -70,6 +76,9 @@ def _load():
         "maps_order_local_workspace_size": ([i64, i32], sz),
         "maps_order_local": ([i64, i32, vp, vp, vp, vp, i32, vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_order_local_static": ([i64, i32, vp, vp, vp, vp, i32, vp, vp, vp, vp], ctypes.c_int),
+        "maps_rr_pressure_workspace_size": ([ctypes.POINTER(RRCfg), i64], sz),
+        "maps_rr_pressure": ([ctypes.POINTER(RRCfg), i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
+                             ctypes.c_int),
         "maps_stream_workspace_size": ([ctypes.POINTER(StreamCfg)], sz),
         "maps_stream_run": ([ctypes.POINTER(StreamCfg), vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
                             ctypes.c_int),
@@ -88,7 +97,8 @@ EXPORTS = ("maps_version", "maps_last_cuda_error", "maps_check", "maps_set_dispa
            "maps_project_occupancy_workspace_size", "maps_project_occupancy",
            "maps_dispatch_workspace_size", "maps_dispatch",
            "maps_order_local_workspace_size", "maps_order_local", "maps_order_local_static",
-           "maps_stream_workspace_size", "maps_stream_run")
+           "maps_stream_workspace_size", "maps_stream_run",
+           "maps_rr_pressure_workspace_size", "maps_rr_pressure")
 
 
 def _stream(stream) -> ctypes.c_void_p:
@@ -235,3 +245,21 @@ def maps_stream_run(cfg: StreamCfg, arrival_ms, prompt, true_len, pred, choice_o
                                _ptr(pred, torch.int32), _ptr(choice_out, torch.int32),
                                _ptr(q_out, torch.int32), _ptr(stats_out, torch.int64),
                                ws.ptr, ws.nbytes, _stream(stream))
+
+
+def maps_rr_pressure(N: int, C: int, t_tok_us: int, theta_ppm: int, arrival_us, prompt, out_len,
+                     admit_out, done_out, stats_out, t_sim_out, ws: Workspace | None = None,
+                     stream=None) -> int:
+    """The App. A round-robin simulation of n_real realisations at once.
+    arrival_us [n_real][n_req] int64, prompt / out_len [n_real][n_req] int32;
+    outputs admit / done [n_real][n_req] int64, stats [n_real][N][6] int64,
+    t_sim [n_real] int64."""
+    n_real, n_req = arrival_us.shape
+    cfg = RRCfg(int(n_req), int(N), int(C), int(t_tok_us), int(theta_ppm))
+    ws = ws or Workspace()
+    ws.ensure(lib.maps_rr_pressure_workspace_size(ctypes.byref(cfg), n_real))
+    return lib.maps_rr_pressure(ctypes.byref(cfg), n_real, _ptr(arrival_us, torch.int64),
+                                _ptr(prompt, torch.int32), _ptr(out_len, torch.int32),
+                                _ptr(admit_out, torch.int64), _ptr(done_out, torch.int64),
+                                _ptr(stats_out, torch.int64), _ptr(t_sim_out, torch.int64),
+                                ws.ptr, ws.nbytes, _stream(stream))

@@ -45,6 +45,12 @@ WORKLOADS = {
                    rate=200.0, burst_prob=0.1, burst_mult=5.0,
                    prompt=(32, 2048), out="lognormal", out_params=(5.5, 1.0),
                    clip=8192, sigma=0.4),
+    # App. A simulation setup: N decoders of C tokens, t_tok = 1 ms, theta =
+    # 0.85, 10,000 requests; the trace's empirical length bins are not
+    # available, tiny's prompt and output distributions stand in for them
+    "rr": dict(index=5, N=4, C=50000, t_tok_us=1000, theta_ppm=850000, n_req=10000,
+               prompt=(32, 2048), out="lognormal", out_params=(5.5, 1.0), clip=8192,
+               rhos=(0.80, 0.90, 0.96, 1.00, 1.05, 1.10)),
     "large": dict(index=4, D=256, R_per=4096, H=65536, J=65536, n_cal=1000000,
                   alphas_ppm=(100000,), caps=(524288,), prompt=(64, 8192),
                   out="bimodal", out_params=(0.7, 4.5, 0.8, 7.5, 0.7),
@@ -181,3 +187,35 @@ def make_stream(seed: int | None = None, n_requests: int | None = None) -> dict:
                 batch=cfg["batch"], window=cfg["window"],
                 alpha_ppm=cfg["alpha_ppm"], max_wait=MAX_WAIT_STEPS,
                 arrival_ms=arrival_ms, prompt=prompt, true=true, pred=pred)
+
+
+def make_rr(n_seeds: int = 1, rhos=None, n_req: int | None = None, seed0: int = 0) -> dict:
+    """Realisations of the round-robin KV-pressure simulation (App. A).
+
+    Per seed one workload is drawn -- prompts, output lengths and a unit-rate
+    Poisson arrival sequence -- and, as in App. A, only the load intensity
+    varies across the utilisations rho: the arrival rate is
+    lambda = rho * N / (mean output length * t_tok), and arrival times are the
+    unit-rate arrival instants divided by lambda, in integer microseconds.
+    Realisation r = seed * len(rhos) + rho index.  Returns arrays
+    [n_real][n_req] (arrival_us int64, prompt and out_len int32) and the
+    simulation constants.
+    """
+    cfg = WORKLOADS["rr"]
+    rhos = tuple(cfg["rhos"] if rhos is None else rhos)
+    n = cfg["n_req"] if n_req is None else int(n_req)
+    arr, prm, out = [], [], []
+    for sd in range(n_seeds):
+        ss = np.random.SeedSequence([cfg["index"], seed0 + sd])
+        s_p, s_o, s_a = [np.random.default_rng(c) for c in ss.spawn(3)]
+        prompt = _prompts(s_p, cfg, n)
+        out_len = _lengths(s_o, cfg, n)
+        unit = np.cumsum(s_a.exponential(1.0, n))  # unit-rate arrival instants
+        for rho in rhos:
+            lam = rho * cfg["N"] / (float(out_len.mean()) * cfg["t_tok_us"] * 1e-6)
+            arr.append(np.rint(unit * 1e6 / lam).astype(np.int64))
+            prm.append(prompt)
+            out.append(out_len)
+    return dict(name="rr", N=cfg["N"], C=cfg["C"], t_tok_us=cfg["t_tok_us"],
+                theta_ppm=cfg["theta_ppm"], n_req=n, rhos=rhos, n_seeds=n_seeds,
+                arrival_us=np.stack(arr), prompt=np.stack(prm), out_len=np.stack(out))
