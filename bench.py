@@ -25,6 +25,10 @@ copies of every input and device-to-host copies of every output inside the
 timed region; steps are pipelined over two buffer sets, each stage replayed
 from a CUDA graph.
 
+Beside the step, the streaming loop (all 10^6 requests through
+maps_stream_run) and the App. A round-robin KV-pressure simulation
+(maps_rr_pressure, 384 realisations) are timed.
+
 The CPU baseline is the plain (tier-P) oracle on whole steps of the same
 workload, on every host core and on one.  --impl reference times it the
 same way (whole steps, every host core) and prints the same metric.
@@ -686,6 +690,73 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
 
 
 # ---------------------------------------------------------------------------
+# the App. A round-robin KV-pressure simulation (maps_rr_pressure)
+# ---------------------------------------------------------------------------
+
+def bench_rr(device, cpu_sample: int = 0, n_seeds: int = 64) -> dict:
+    """Device time of maps_rr_pressure over n_seeds workload draws x the six
+    utilisations of the App. A setup (inputs resident in HBM; CUDA events
+    around 10 calls after 3 warm-up ones).  With cpu_sample > 0 the oracle
+    simulates that many of the realisations, one after the other, as the CPU
+    reference."""
+    import torch
+    from paper_2609_15359_gb300 import maps as M
+    from paper_2609_15359_gb300 import workloads as W
+    w = W.make_rr(n_seeds)
+    t = lambda x, dt: torch.from_numpy(np.ascontiguousarray(x, dtype=dt)).to(device)  # noqa: E731
+    arr, pr, out = t(w["arrival_us"], np.int64), t(w["prompt"], np.int32), t(w["out_len"], np.int32)
+    n_real, n = w["arrival_us"].shape
+    adm = torch.empty((n_real, n), dtype=torch.int64, device=device)
+    dn = torch.empty_like(adm)
+    st = torch.empty((n_real, w["N"], 6), dtype=torch.int64, device=device)
+    ts = torch.empty(n_real, dtype=torch.int64, device=device)
+    ws = M.Workspace(device=device)
+
+    def run():
+        rc = M.maps_rr_pressure(w["N"], w["C"], w["t_tok_us"], w["theta_ppm"], arr, pr, out, adm,
+                                dn, st, ts, ws=ws)
+        if rc != 0:
+            raise RuntimeError(f"maps_rr_pressure status {rc}")
+
+    for _ in range(3):
+        run()
+    torch.cuda.synchronize()
+    reps = 10
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        run()
+    e1.record()
+    torch.cuda.synchronize()
+    if M.maps_check(ws) != 0:
+        raise RuntimeError("maps_rr_pressure reported a device error")
+    secs = e0.elapsed_time(e1) / 1e3 / reps
+    stats = st.cpu().numpy()
+    tsim = ts.cpu().numpy()
+    f_hp = stats[:, :, 0] / tsim[:, None]
+    res = {"workload": (f"App. A: N={w['N']} decoders, C={w['C']:,} tokens, t_tok=1 ms, "
+                        f"theta=0.85, {n:,} requests per realisation; {n_seeds} draws x "
+                        f"{len(w['rhos'])} utilisations rho={list(w['rhos'])}"),
+           "realisations": n_real, "value": n_real * n / secs, "unit": "simulated requests/s",
+           "ms_per_call": secs * 1e3,
+           "timing": "CUDA events around 10 calls (inputs resident), after 3 warm-up calls",
+           "max_f_hp_by_rho": {str(rho): float(f_hp[i::len(w["rhos"])].max())
+                               for i, rho in enumerate(w["rhos"])}}
+    if cpu_sample:
+        import oracle as O
+        m = min(cpu_sample, n_real)
+        t0 = time.perf_counter()
+        for r in range(m):
+            O.rr_pressure(w["N"], w["C"], w["t_tok_us"], w["theta_ppm"], w["arrival_us"][r],
+                          w["prompt"][r], w["out_len"][r])
+        cs = time.perf_counter() - t0
+        res["cpu_baseline"] = {"value": m * n / cs, "unit": "simulated requests/s", "cores": 1,
+                               "kind": "oracle",
+                               "sample": f"the first {m} realisations, one after the other"}
+    return res
+
+
+# ---------------------------------------------------------------------------
 # the CPU oracle as the baseline / reference arm
 # ---------------------------------------------------------------------------
 
@@ -803,7 +874,7 @@ def main():
     ap.add_argument("--impl", choices=["maps", "reference"], default="maps")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-stream", action="store_true",
-                    help="skip the streaming-loop measurement")
+                    help="skip the streaming-loop and round-robin simulation measurements")
     args = ap.parse_args()
     world, rank, local = dist_env()
 
@@ -831,6 +902,8 @@ def main():
         if world == 1 and not args.no_stream:
             res["stream"] = bench_stream(torch.device(f"cuda:{local}"),
                                          0 if args.no_cpu_baseline else 100000)
+            res["rr_pressure"] = bench_rr(torch.device(f"cuda:{local}"),
+                                          0 if args.no_cpu_baseline else 24)
         print(json.dumps(res), flush=True)
     if dist is not None:
         dist.destroy_process_group()
