@@ -58,7 +58,15 @@ class StreamCfg(ctypes.Structure):
     _fields_ = [("N", ctypes.c_int64), ("D", ctypes.c_int32),
                 ("H", ctypes.c_int32), ("cap", ctypes.c_int32),
                 ("batch", ctypes.c_int32), ("window", ctypes.c_int32),
-                ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32)]
+                ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32),
+                ("dispatch", ctypes.c_int32), ("local", ctypes.c_int32),
+                ("accounting", ctypes.c_int32)]
+
+
+# streaming-loop policies (the Sec. 4 ablations, the baselines, App. C)
+DISPATCH_MAPS, DISPATCH_MC, DISPATCH_RR, DISPATCH_LR = 0, 1, 2, 3
+LOCAL_SJF, LOCAL_FCFS = 0, 1
+ACCOUNT_OCCUPANCY, ACCOUNT_STAGED, ACCOUNT_HELD = 0, 1, 2
 
 
 class RRCfg(ctypes.Structure):
@@ -91,7 +99,7 @@ def lib():
         L.oracle_order_local.argtypes = [ctypes.c_int64, ctypes.c_int32, vp, vp,
                                          vp, vp, ctypes.c_int32, vp, vp]
         L.oracle_stream.argtypes = [ctypes.POINTER(StreamCfg), _i64p, _i32p,
-                                    _i32p, _i32p, _i32p, _i32p, _i64p]
+                                    _i32p, _i32p, _i32p, _i32p, _i64p, _i64p]
         L.oracle_rr_pressure.argtypes = [ctypes.POINTER(RRCfg), _i64p, _i32p, _i32p,
                                          _i64p, _i64p, _i64p, ctypes.POINTER(ctypes.c_int64)]
         _lib = L
@@ -194,15 +202,22 @@ def order_local(D: int, dec, bnd, wait, arrival, max_wait: int):
 
 
 def stream(N, D, H, cap, batch, window, alpha_ppm, max_wait, arrival_ms,
-           prompt, true_len, pred):
-    cfg = StreamCfg(N, D, H, cap, batch, window, alpha_ppm, max_wait)
+           prompt, true_len, pred, dispatch=DISPATCH_MAPS, local=LOCAL_SJF,
+           accounting=ACCOUNT_OCCUPANCY, with_dec_stats=False):
+    """Returns (status, choice, q, stats [nb][4]) and, with with_dec_stats,
+    the per-decoder statistics [D][3] as a fifth item."""
+    cfg = StreamCfg(N, D, H, cap, batch, window, alpha_ppm, max_wait, dispatch, local,
+                    accounting)
     nb = (N + batch - 1) // batch
     choice = np.empty(N, dtype=np.int32)
     q = np.empty(nb, dtype=np.int32)
     stats = np.empty(4 * nb, dtype=np.int64)
+    dstats = np.zeros(3 * D, dtype=np.int64)
     st = lib().oracle_stream(ctypes.byref(cfg), _c64(arrival_ms[:N]),
                              _c32(prompt[:N]), _c32(true_len[:N]),
-                             _c32(pred[:N]), choice, q, stats)
+                             _c32(pred[:N]), choice, q, stats, dstats)
+    if with_dec_stats:
+        return st, choice, q, stats.reshape(nb, 4), dstats.reshape(D, 3)
     return st, choice, q, stats.reshape(nb, 4)
 
 

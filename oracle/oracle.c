@@ -200,7 +200,7 @@ static int64_t candidate_peak(const int32_t *Krow, int64_t p, int64_t u)
     return m;
 }
 
-static int dispatch_horizon(int sequential, int32_t D, int32_t H, int32_t *K,
+static int dispatch_horizon(int sequential, int mc, int32_t D, int32_t H, int32_t *K,
                             const int32_t *cap, int32_t *Q, int64_t J,
                             const int32_t *cand_prompt,
                             const int32_t *cand_bound, int32_t *choice_out,
@@ -226,8 +226,9 @@ static int dispatch_horizon(int sequential, int32_t D, int32_t H, int32_t *K,
             int64_t peak = candidate_peak(K + (int64_t)k * H, p, u);
             int64_t h = (int64_t)cap[k] - peak;
             /* Feasible decoders compete on queue length (min Q); only when
-             * none is feasible does the most headroom win. */
-            int64_t key = h >= 0 ? (int64_t)Q[k] : KEY_INFEASIBLE_BASE - h;
+             * none is feasible does the most headroom win.  The MC variant
+             * (Sec. 4 ablation MQ->MC) ranks every decoder by headroom. */
+            int64_t key = h >= 0 && !mc ? (int64_t)Q[k] : KEY_INFEASIBLE_BASE - h;
             if (best < 0 || key < best_key) {
                 best = k;
                 best_key = key;
@@ -336,7 +337,7 @@ int oracle_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S,
     if (mode == ORACLE_MODE_SNAPSHOT || mode == ORACLE_MODE_SEQUENTIAL) {
         if (H < 1 || K == NULL)
             return ORACLE_E_INVALID;
-        return dispatch_horizon(mode == ORACLE_MODE_SEQUENTIAL, D, H, K, cap, Q,
+        return dispatch_horizon(mode == ORACLE_MODE_SEQUENTIAL, 0, D, H, K, cap, Q,
                                 J, cand_prompt, cand_bound, choice_out,
                                 headroom_out);
     }
@@ -440,11 +441,13 @@ static int cmp_completion(const void *a, const void *b)
 int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                   const int32_t *prompt, const int32_t *true_len,
                   const int32_t *pred, int32_t *choice_out, int32_t *q_out,
-                  int64_t *stats_out)
+                  int64_t *stats_out, int64_t *dec_stats_out)
 {
     if (cfg == NULL || cfg->N < 1 || cfg->N > I32_MAX || cfg->D < 1 ||
         cfg->H < 1 || cfg->cap < 0 || cfg->batch < 1 || cfg->window < 1 ||
-        cfg->alpha_ppm == 0 || cfg->alpha_ppm >= 1000000u)
+        cfg->alpha_ppm == 0 || cfg->alpha_ppm >= 1000000u ||
+        cfg->dispatch < 0 || cfg->dispatch > 3 || cfg->local < 0 || cfg->local > 1 ||
+        cfg->accounting < 0 || cfg->accounting > 2)
         return ORACLE_E_INVALID;
     const int64_t N = cfg->N;
     const int32_t D = cfg->D, H = cfg->H, Bsz = cfg->batch, Wn = cfg->window;
@@ -482,9 +485,14 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
     int32_t *wperm = (int32_t *)malloc((size_t)N * sizeof(int32_t));
     int32_t *cU = (int32_t *)malloc((size_t)Bsz * sizeof(int32_t));
     int64_t *hr = (int64_t *)malloc((size_t)Bsz * sizeof(int64_t));
+    int32_t *res_u = (int32_t *)calloc((size_t)N, sizeof(int32_t)); /* bound reserved at admission */
+    int64_t *occ = (int64_t *)malloc((size_t)D * sizeof(int64_t));
+    int64_t *nreq = (int64_t *)malloc((size_t)D * sizeof(int64_t));
+    int64_t *dst = (int64_t *)calloc((size_t)D * 3, sizeof(int64_t));
     if (!st || !g || !dec || !U || !disp || !act || !done || !win_true ||
         !win_pred || !K || !capv || !Q || !off || !used || !seg || !rp || !rg ||
-        !rU || !wid || !wdec || !wU || !wwait || !warr || !wperm || !cU || !hr) {
+        !rU || !wid || !wdec || !wU || !wwait || !warr || !wperm || !cU || !hr ||
+        !res_u || !occ || !nreq || !dst) {
         status = ORACLE_E_INVALID;
         goto out;
     }
@@ -515,8 +523,11 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                 g[id] += (int32_t)delta;
             }
         }
-        for (int32_t k = 0; k < D; ++k)
+        for (int32_t k = 0; k < D; ++k) {
             used[k] = 0;
+            occ[k] = 0;
+            nreq[k] = 0;
+        }
         {
             int64_t w = 0;
             for (int64_t a = 0; a < nact; ++a) {
@@ -524,14 +535,28 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                 if (st[id] == ST_DONE)
                     continue;
                 act[w++] = id;
-                if (st[id] == ST_RUNNING)
-                    used[dec[id]] += (int64_t)prompt[id] + g[id];
+                nreq[dec[id]] += 1; /* requests in the system (least requests) */
+                if (st[id] == ST_RUNNING) {
+                    /* tokens held; and what admission counts for the request
+                     * (App. C: the prompt's KV once transferred, plus the
+                     * output reserved at its bound until generation ends --
+                     * or, without the staged release, the prompt's
+                     * reservation as well) */
+                    int64_t p = prompt[id], gg = g[id], r = res_u[id];
+                    int64_t out_part = r > gg ? r : gg;
+                    occ[dec[id]] += p + gg;
+                    used[dec[id]] += cfg->accounting == 0 ? p + gg
+                                   : cfg->accounting == 1 ? p + out_part
+                                                          : 2 * p + out_part;
+                }
             }
             nact = w;
         }
         int64_t overflow = 0;
-        for (int32_t k = 0; k < D; ++k)
-            overflow += used[k] > capv[k];
+        for (int32_t k = 0; k < D; ++k) {
+            overflow += occ[k] > capv[k];
+            dst[3 * k + 1] += occ[k] > capv[k];
+        }
 
         /* 2. Sliding calibration window: the most recent completions,
          *    ordered by (completion step, request id) (Sec. 3.2). */
@@ -575,7 +600,18 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
             status = ORACLE_E_RANGE;
 
         /* 5. Dispatch the batch. */
-        if (!rr) {
+        if (!rr && cfg->dispatch == 3) {
+            /* least requests: the decoder with the fewest requests in the
+             * system, the batch counted as it is dispatched */
+            for (int64_t i = lo; i < hi; ++i) {
+                int32_t best = 0;
+                for (int32_t k = 1; k < D; ++k)
+                    if (nreq[k] < nreq[best])
+                        best = k;
+                choice_out[i] = best;
+                nreq[best] += 1;
+            }
+        } else if (!rr && cfg->dispatch != 2) {
             /* residents of each decoder: running (g) and waiting (g = 0) */
             int64_t R = 0;
             for (int32_t k = 0; k < D; ++k) {
@@ -596,9 +632,8 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
             int os = oracle_occupancy(D, H, off, R, rp, rg, rU, K);
             if (os != ORACLE_OK)
                 status = os;
-            int ds = oracle_dispatch(ORACLE_MODE_SEQUENTIAL, D, H, 1, K, capv, Q,
-                                     NULL, 0, NULL, NULL, NULL, hi - lo,
-                                     &prompt[lo], cU, &choice_out[lo], hr);
+            int ds = dispatch_horizon(1, cfg->dispatch == 1, D, H, K, capv, Q,
+                                      hi - lo, &prompt[lo], cU, &choice_out[lo], hr);
             if (ds != ORACLE_OK)
                 status = ds;
         } else {
@@ -630,8 +665,9 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
             warr[nw] = (int32_t)id;
             ++nw;
         }
-        int ls = oracle_order_local(nw, D, wdec, wU, wwait, warr, cfg->max_wait,
-                                    wperm, seg);
+        /* FCFS promotes every entry: arrival order alone */
+        int ls = oracle_order_local(nw, D, wdec, wU, wwait, warr,
+                                    cfg->local == 1 ? -1 : cfg->max_wait, wperm, seg);
         if (ls != ORACLE_OK) {
             status = ls;
             goto out;
@@ -650,9 +686,19 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                     break;
                 st[id] = ST_RUNNING;
                 g[id] = 0;
-                used[k] += prompt[id];
+                res_u[id] = U[id];
+                used[k] += cfg->accounting == 0 ? (int64_t)prompt[id]
+                         : cfg->accounting == 1 ? demand
+                                                : (int64_t)prompt[id] + demand;
                 ++admitted;
+                dst[3 * k + 2] += 1;
             }
+            /* the waiting queue holds until the next batch's dispatch step */
+            int64_t adm_k = 0;
+            for (int64_t x = seg[k]; x < seg[k + 1]; ++x)
+                adm_k += st[wid[wperm[x]]] == ST_RUNNING;
+            int64_t s_next = b + 1 < nb ? arrival_ms[((b + 2) * Bsz < N ? (b + 2) * Bsz : N) - 1] : s;
+            dst[3 * k] += (seg[k + 1] - seg[k] - adm_k) * (s_next - s);
         }
         stats_out[4 * b + 0] = ndone;
         stats_out[4 * b + 1] = admitted;
@@ -660,11 +706,15 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
         stats_out[4 * b + 3] = overflow;
         prev_s = s;
     }
+    if (dec_stats_out != NULL)
+        for (int64_t i = 0; i < (int64_t)D * 3; ++i)
+            dec_stats_out[i] = dst[i];
 
 out:
     free(st); free(g); free(dec); free(U); free(disp); free(act); free(done);
     free(win_true); free(win_pred); free(K); free(capv); free(Q); free(off);
     free(used); free(seg); free(rp); free(rg); free(rU); free(wid); free(wdec);
     free(wU); free(wwait); free(warr); free(wperm); free(cU); free(hr);
+    free(res_u); free(occ); free(nreq); free(dst);
     return status;
 }

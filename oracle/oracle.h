@@ -81,15 +81,24 @@ typedef struct {
     int32_t window;     /* calibration window (completed requests) */
     uint32_t alpha_ppm; /* miscoverage * 1e6 */
     int32_t max_wait;   /* promotion threshold, steps */
+    int32_t dispatch;   /* 0 MAPS (min Q among feasible, else most headroom),
+                           1 MC (most headroom), 2 round robin, 3 least requests */
+    int32_t local;      /* 0 SJF with max-wait promotion, 1 FCFS */
+    int32_t accounting; /* admission counts running requests at 0 their tokens,
+                           1 prompt + reserved output (staged release),
+                           2 reserved prompt + prompt + reserved output */
 } oracle_stream_cfg;
 
 /* Outputs: choice[N]; per batch b: q[b] (-1 if unbounded -> round robin),
  * stats[4b..4b+3] = completed, admitted, waiting after admission,
- * decoders over capacity after advancing. */
+ * decoders over capacity after advancing; per decoder k (dec_stats may be
+ * NULL): dec_stats[3k..3k+2] = waiting requests x steps summed over the
+ * batches (the time-weighted queue length times the span), batches in which
+ * it was over capacity after advancing, admissions. */
 int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                   const int32_t *prompt, const int32_t *true_len,
                   const int32_t *pred, int32_t *choice_out, int32_t *q_out,
-                  int64_t *stats_out);
+                  int64_t *stats_out, int64_t *dec_stats_out);
 
 /* Round-robin KV-pressure simulation of App. A (oracle_rr.c). */
 typedef struct {
