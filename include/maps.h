@@ -279,10 +279,36 @@ int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
  *      requests, grown by p per admission); the first misfit stops its queue.
  * No preemption; a running request above capacity is only counted.
  *
+ * Policy variants (the Sec. 4 ablations and the baselines of the App. C
+ * studies), chosen in cfg; the defaults (all 0) are the loop above:
+ *   dispatch_policy  MAPS_STREAM_MAPS: SEQUENTIAL dispatch as in 4;
+ *                    MAPS_STREAM_MC: the same projection, every candidate to
+ *                    the decoder of largest headroom cap - (p + 1 + M), ties
+ *                    to the lowest index (memory-only, no queue term);
+ *                    MAPS_STREAM_RR: round robin, choice = index mod D;
+ *                    MAPS_STREAM_LR: least requests, the decoder with the
+ *                    fewest requests in the system (running and waiting),
+ *                    the batch counted as it is dispatched, ties to the
+ *                    lowest index.  An unbounded quantile still sends the
+ *                    batch round robin under every policy.
+ *   local_order      MAPS_STREAM_SJF: as in 6; MAPS_STREAM_FCFS: every queue
+ *                    in arrival (index) order.
+ *   accounting       what a running request counts for in `used`, with
+ *                    g generated and U* its bound at admission:
+ *                    MAPS_STREAM_OCCUPANCY  p + g (grown by p per admission);
+ *                    MAPS_STREAM_STAGED     p + max(U*, g) (the output stays
+ *                      reserved at its bound; grown by p + U);
+ *                    MAPS_STREAM_HELD       2p + max(U*, g) (the prompt is
+ *                      held twice, at the prefill and decode sides, as when
+ *                      the staged release is off; grown by 2p + U).
+ *                    Admission is always used + p + U <= cap; the over-
+ *                    capacity count compares p + g with cap in every mode.
+ *
  *   cfg                 host struct: N requests (1 .. INT32_MAX), D decoders
  *                       (1 .. 1024), horizon H steps, capacity cap tokens per
  *                       decoder, batch size, window size, alpha in parts per
- *                       million (0 < alpha_ppm < 10^6), max_wait steps.
+ *                       million (0 < alpha_ppm < 10^6), max_wait steps,
+ *                       and the three policy fields above.
  *   arrival_ms          [N] int64 arrival step.
  *   prompt, true_len, pred   [N] int32 prompt length (>= 0), true output
  *                       length (>= 1), predicted output length (>= 0).
@@ -292,6 +318,11 @@ int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
  *   stats_out           [ceil(N / batch)][4] int64 per batch: completions,
  *                       admissions, requests left waiting, decoders whose
  *                       running requests exceed capacity after advancing.
+ *   dec_stats_out       [D][3] int64 per decoder, or NULL: the waiting-queue
+ *                       integral (requests left waiting after batch b's
+ *                       admission times s_{b+1} - s_b, the last batch
+ *                       counting 0), the batches after whose advance its
+ *                       running requests exceed capacity, its admissions.
  * The call runs the whole loop: it synchronises the stream once per batch
  * (to read the request counts that size the next launches) and at the end,
  * and returns the full status.  A negative length or decreasing arrival is
@@ -305,14 +336,27 @@ typedef struct {
   int32_t window;
   uint32_t alpha_ppm;
   int32_t max_wait;
+  int32_t dispatch_policy; /* MAPS_STREAM_MAPS / _MC / _RR / _LR */
+  int32_t local_order;     /* MAPS_STREAM_SJF / _FCFS */
+  int32_t accounting;      /* MAPS_STREAM_OCCUPANCY / _STAGED / _HELD */
 } maps_stream_cfg;
+
+#define MAPS_STREAM_MAPS 0
+#define MAPS_STREAM_MC 1
+#define MAPS_STREAM_RR 2
+#define MAPS_STREAM_LR 3
+#define MAPS_STREAM_SJF 0
+#define MAPS_STREAM_FCFS 1
+#define MAPS_STREAM_OCCUPANCY 0
+#define MAPS_STREAM_STAGED 1
+#define MAPS_STREAM_HELD 2
 
 size_t maps_stream_workspace_size(const maps_stream_cfg *cfg);
 int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms,
                     const int32_t *prompt, const int32_t *true_len,
                     const int32_t *pred, int32_t *choice_out, int32_t *q_out,
-                    int64_t *stats_out, void *ws, size_t ws_bytes,
-                    void *stream);
+                    int64_t *stats_out, int64_t *dec_stats_out, void *ws,
+                    size_t ws_bytes, void *stream);
 
 /* ------------------------------------------------------------------------
  * Round-robin KV-pressure simulation and high-pressure interval metrics,

@@ -835,10 +835,13 @@ __device__ __forceinline__ bool better(const Pick &x, const Pick &y) {
   if (x.v != y.v) return x.v < y.v;
   return x.k < y.k;
 }
-__device__ __forceinline__ Pick make_pick(long long h, int32_t q, int k) {
+// mc: rank every decoder by headroom alone (the memory-only ablation): all
+// picks take the infeasible class, whose order is the largest headroom first.
+__device__ __forceinline__ Pick make_pick(long long h, int32_t q, int k, bool mc = false) {
   Pick p;
-  p.inf = h >= 0 ? 0 : 1;
-  p.v = h >= 0 ? static_cast<long long>(q) : -h;
+  const bool feas = h >= 0 && !mc;
+  p.inf = feas ? 0 : 1;
+  p.v = feas ? static_cast<long long>(q) : -h;
   p.k = k;
   p.h = h;
   return p;
@@ -887,7 +890,7 @@ __device__ __forceinline__ Pick no_pick() {
 __global__ void __launch_bounds__(1024, 1)
 dispatch_sequential_kernel(int D, int H, int32_t *K, uint32_t *kmax, const int32_t *cap,
                            int32_t *Q, int64_t J, const int32_t *cp, const int32_t *cb,
-                           int32_t *choice, int64_t *headroom, int32_t *status) {
+                           int32_t *choice, int64_t *headroom, int mc, int32_t *status) {
   pdl_prologue();
   __shared__ uint32_t s_M[kMaxD];
   __shared__ Pick s_w[32];
@@ -927,7 +930,7 @@ dispatch_sequential_kernel(int D, int H, int32_t *K, uint32_t *kmax, const int32
     Pick mine = no_pick();
     for (int k = tid; k < D; k += blockDim.x) {
       const long long h = static_cast<long long>(cap[k]) - (static_cast<long long>(p) + 1 + s_M[k]);
-      const Pick c = make_pick(h, Q[k], k);
+      const Pick c = make_pick(h, Q[k], k, mc != 0);
       if (better(c, mine)) mine = c;
     }
     const Pick b = block_best(mine, s_w);
@@ -1348,6 +1351,23 @@ int launch_snapshot(int D, int H, const int32_t *K, const uint32_t *kmax, const 
 }  // namespace
 }  // namespace maps
 
+namespace maps {
+int dispatch_sequential(int D, int H, int32_t *K, const int32_t *cap, int32_t *Q, int64_t J,
+                        const int32_t *cp, const int32_t *cb, int32_t *choice, int64_t *headroom,
+                        bool mc, void *ws, cudaStream_t s) {
+  // a private summary of K (also validating K >= 0); updated in place
+  int32_t *status = status_word(ws);
+  Carve cv(ws);
+  const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
+  uint32_t *km = cv.take<uint32_t>(static_cast<size_t>(D) * nb);
+  const int gk = static_cast<int>(std::min<int64_t>((nb * D + 255) / 256, 8LL * sm_count()));
+  launch_pdl(kmax_from_K_kernel, gk, 256, 0, s, D, H, K, km, status);
+  launch_pdl(dispatch_sequential_kernel, 1, 1024, 0, s, D, H, K, km, cap, Q, J, cp, cb, choice,
+             headroom, mc ? 1 : 0, status);
+  return launch_ok();
+}
+}  // namespace maps
+
 extern "C" {
 
 int maps_set_dispatch_events(void *before, void *after) {
@@ -1394,17 +1414,9 @@ int maps_dispatch(int32_t mode, int32_t D, int32_t H, int32_t S, int32_t *K, con
     case MAPS_MODE_SNAPSHOT:
       return launch_snapshot(D, H, K, kmax, cap, Q, J, cand_prompt, cand_bound, choice_out,
                              headroom_out, ws, s);
-    case MAPS_MODE_SEQUENTIAL: {
-      // a private summary of K (also validating K >= 0); updated in place
-      Carve cv(ws);
-      const int64_t nb = (static_cast<int64_t>(H) + kSumBlock - 1) / kSumBlock;
-      uint32_t *km = cv.take<uint32_t>(static_cast<size_t>(D) * nb);
-      const int gk = static_cast<int>(std::min<int64_t>((nb * D + 255) / 256, 8LL * sm_count()));
-      launch_pdl(kmax_from_K_kernel, gk, 256, 0, s, D, H, K, km, status);
-      launch_pdl(dispatch_sequential_kernel, 1, 1024, 0, s, D, H, K, km, cap, Q, J, cand_prompt,
-                                                    cand_bound, choice_out, headroom_out, status);
-      return launch_ok();
-    }
+    case MAPS_MODE_SEQUENTIAL:
+      return dispatch_sequential(D, H, K, cap, Q, J, cand_prompt, cand_bound, choice_out,
+                                 headroom_out, false, ws, s);
     default: {
       Carve cv(ws);
       long long *B_eff = cv.take<long long>(static_cast<size_t>(D));

@@ -128,6 +128,13 @@ inline int check_ws(void *ws, size_t ws_bytes, size_t need) {
   return MAPS_OK;
 }
 
+// SEQUENTIAL horizon dispatch of J candidates on a dense K (the body of
+// maps_dispatch's SEQUENTIAL mode, arguments already checked); mc ranks the
+// decoders by headroom alone.  Uses the workspace past its control block.
+int dispatch_sequential(int D, int H, int32_t *K, const int32_t *cap, int32_t *Q, int64_t J,
+                        const int32_t *cp, const int32_t *cb, int32_t *choice, int64_t *headroom,
+                        bool mc, void *ws, cudaStream_t s);
+
 int sm_count();           // multiprocessors of the current device
 int max_smem_optin();     // opt-in shared memory per block, bytes
 

@@ -19,6 +19,10 @@
 //   7. local order of every waiting queue (stream_waitlist, maps_order_local)
 //   8. admission in queue order while used + p + U <= capacity, the first
 //      misfit blocking its queue                            (stream_admit)
+// Policy variants replace step 5 (max-headroom, round-robin or least-requests
+// dispatch: stream_dispatch with mc, stream_rr, stream_lr), the order of step 7
+// (FCFS: every entry promoted, so arrival order alone) and what a running
+// request counts for in step 8 (occupancy, staged or held reservation).
 // The host issues the launches; it reads 24 bytes of loop state once per
 // batch (the request, completion and waiting counts that size the calls).
 #include <algorithm>
@@ -86,18 +90,21 @@ __global__ void stream_init_kernel(int64_t first_hi, int D, int32_t cap, const i
 }
 
 // 1. Advance by delta = s - prev_s steps; keep the survivors in id order.
+//    occupancy = p + g of the running requests (the over-capacity count);
+//    used = what admission counts for them: p + g, p + max(U*, g) (staged)
+//    or 2p + max(U*, g) (held), U* the bound reserved at admission.
 __global__ void __launch_bounds__(kSt, 1)
-stream_advance_kernel(int64_t hi, int D, int32_t cap, const int64_t *arrival,
-                      const int32_t *prompt, const int32_t *true_len, uint8_t *st, int32_t *g,
-                      const int32_t *dec, const int32_t *act_in, int32_t *act_out,
-                      int32_t *done_id, int32_t *done_rem, long long *used, StreamState *S,
-                      int64_t *stats_b) {
+stream_advance_kernel(int64_t hi, int D, int32_t cap, int acct, const int64_t *arrival,
+                      const int32_t *prompt, const int32_t *true_len, const int32_t *res_u,
+                      uint8_t *st, int32_t *g, const int32_t *dec, const int32_t *act_in,
+                      int32_t *act_out, int32_t *done_id, int32_t *done_rem, long long *used,
+                      StreamState *S, int64_t *stats_b, int64_t *dst) {
   pdl_prologue();
-  __shared__ unsigned long long s_used[kStreamMaxD];
+  __shared__ unsigned long long s_occ[kStreamMaxD], s_used[kStreamMaxD];
   __shared__ int s_w[kStWarps];
   __shared__ int s_nwait;
   const int tid = threadIdx.x;
-  for (int k = tid; k < D; k += kSt) s_used[k] = 0;
+  for (int k = tid; k < D; k += kSt) s_occ[k] = s_used[k] = 0;
   if (tid == 0) s_nwait = 0;
   const long long s = arrival[hi - 1];
   const long long delta = s - S->prev_s;
@@ -120,8 +127,13 @@ stream_advance_kernel(int64_t hi, int D, int32_t cap, const int64_t *arrival,
         } else {
           const int gn = g[id] + static_cast<int>(delta);  // < true_len
           g[id] = gn;
-          atomicAdd(&s_used[dec[id]],
-                    static_cast<unsigned long long>(static_cast<long long>(prompt[id]) + gn));
+          const long long p = prompt[id];
+          atomicAdd(&s_occ[dec[id]], static_cast<unsigned long long>(p + gn));
+          if (acct != MAPS_STREAM_OCCUPANCY) {
+            const long long out = max(static_cast<long long>(res_u[id]), static_cast<long long>(gn));
+            atomicAdd(&s_used[dec[id]], static_cast<unsigned long long>(
+                                            (acct == MAPS_STREAM_HELD ? 2 * p : p) + out));
+          }
         }
       } else if (sv == kWaiting) {
         ++nwait;
@@ -139,8 +151,11 @@ stream_advance_kernel(int64_t hi, int D, int32_t cap, const int64_t *arrival,
     ndone += td;
   }
   if (nwait) atomicAdd(&s_nwait, nwait);
-  const bool ov = tid < D && static_cast<long long>(s_used[tid]) > cap;  // D <= kSt
-  if (tid < D) used[tid] = static_cast<long long>(s_used[tid]);
+  const bool ov = tid < D && static_cast<long long>(s_occ[tid]) > cap;  // D <= kSt
+  if (tid < D) {
+    used[tid] = static_cast<long long>(acct == MAPS_STREAM_OCCUPANCY ? s_occ[tid] : s_used[tid]);
+    if (dst != nullptr && ov) dst[3 * tid + 1] += 1;
+  }
   const int over = __syncthreads_count(ov);
   if (tid == 0) {
     S->prev_s = s;
@@ -177,14 +192,43 @@ __global__ void stream_gather_kernel(int nact, int nb, int64_t lo, const int32_t
     qpred[x] = x < nact ? pred[act[x]] : pred[lo + (x - nact)];
 }
 
-// 3'. No bound available: U = prediction, the batch goes round robin.
-__global__ void stream_rr_kernel(int n, int nb, int64_t lo, int D, const int32_t *qpred,
+// 3'. No bound available: U = prediction, the batch goes round robin.  With
+//     set_u = 0 only the choices (the round-robin dispatch policy).
+__global__ void stream_rr_kernel(int n, int nb, int64_t lo, int D, int set_u, const int32_t *qpred,
                                  int32_t *Uq, int32_t *choice) {
   pdl_prologue();
   const int stride = gridDim.x * blockDim.x;
   for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
-    Uq[x] = qpred[x];
+    if (set_u) Uq[x] = qpred[x];
     if (x < nb) choice[lo + x] = static_cast<int32_t>((lo + x) % D);
+  }
+}
+
+// 5'. Least requests (one warp): candidate j goes to the decoder with the
+//     fewest requests in the system, counting the batch's earlier choices;
+//     ties to the lowest index.  Lane l keeps the counts of decoders l, l + 32,
+//     ... in shared memory; per candidate two warp minima give the smallest
+//     count and then the lowest decoder holding it.
+__global__ void stream_lr_kernel(int D, int nb, const int64_t *res_off, int32_t *choice) {
+  pdl_prologue();
+  __shared__ uint32_t s_c[kStreamMaxD];
+  const int lane = threadIdx.x;
+  for (int k = lane; k < D; k += 32) s_c[k] = static_cast<uint32_t>(res_off[k + 1] - res_off[k]);
+  __syncwarp();
+  for (int j = 0; j < nb; ++j) {
+    uint32_t c = 0xffffffffu, ck = 0xffffffffu;  // this lane's smallest count, its lowest decoder
+    for (int k = lane; k < D; k += 32)
+      if (s_c[k] < c) {
+        c = s_c[k];
+        ck = static_cast<uint32_t>(k);
+      }
+    const uint32_t cmin = __reduce_min_sync(0xffffffffu, c);
+    const uint32_t bk = __reduce_min_sync(0xffffffffu, c == cmin ? ck : 0xffffffffu);
+    if (lane == 0) {
+      choice[j] = static_cast<int32_t>(bk);
+      s_c[bk] = cmin + 1;
+    }
+    __syncwarp();
   }
 }
 
@@ -258,6 +302,20 @@ stream_csr_kernel(int nact, int D, int rr, const int32_t *q_dev, int32_t *q_out_
 // Shared memory: the pool of pairs (the residents of decoder k plus room for
 // nb reservations at base_k = res_off[k] + k nb), the unsorted pairs, and the
 // per-decoder tables.
+// The packed decision key, the smallest wins: a feasible decoder (h >= 0)
+// ranks by Q, an infeasible one after every feasible one by the deficit -h,
+// each then by index: inf << 63 | v << 10 | k.  mc (the max-headroom rule)
+// ranks every decoder as the infeasible class does, by -h: v = 2^33 - h is
+// positive (h <= cap < 2^31) and, like the deficit, below 2^53 for any M the
+// walk forms.
+__device__ __forceinline__ unsigned long long dispatch_key(long long h, int q, int k, int mc) {
+  const bool feas = h >= 0 && !mc;
+  const unsigned long long v = feas ? static_cast<unsigned long long>(q)
+                               : mc ? static_cast<unsigned long long>((1ll << 33) - h)
+                                    : static_cast<unsigned long long>(-h);
+  return (feas ? 0ull : 1ull << 63) | (v << 10) | static_cast<unsigned>(k);
+}
+
 size_t stream_dispatch_smem(int D, int nact, int nb) {
   const size_t pool = static_cast<size_t>(nact) + static_cast<size_t>(D) * nb;
   return 16 * pool + 8 * static_cast<size_t>(nact) + 16 * static_cast<size_t>(D) +
@@ -315,7 +373,7 @@ __device__ bool rebuild_tables(const int32_t *E, const int32_t *Bv, uint32_t *SS
 }
 
 __global__ void __launch_bounds__(kSt, 1)
-stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32_t *rp,
+stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, const int32_t *rp,
                        const int32_t *rg, const int32_t *rU, const int32_t *capv, int32_t *Q,
                        const int32_t *cp, const int32_t *cU, int32_t *choice, int64_t *headroom,
                        int32_t *status) {
@@ -428,10 +486,9 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
       }
       return lo;
     };
-    auto key_of = [](int k, int q, int cap, int32_t p, long long M) {
+    auto key_of = [mc](int k, int q, int cap, int32_t p, long long M) {
       const long long h = static_cast<long long>(cap) - (static_cast<long long>(p) + 1 + M);
-      return h >= 0 ? (static_cast<unsigned long long>(q) << 10) | static_cast<unsigned>(k)
-                    : (1ull << 63) | (static_cast<unsigned long long>(-h) << 10) | static_cast<unsigned>(k);
+      return dispatch_key(h, q, k, mc);
     };
     if (warp == 0) {
       const int k = lane;
@@ -630,9 +687,7 @@ stream_dispatch_kernel(int D, int H, int nb, const int64_t *res_off, const int32
                                static_cast<long long>(u - 1) * (n - c + 1);
         const long long M = max(full, part);
         const long long h = static_cast<long long>(s_cap[k]) - (static_cast<long long>(p) + 1 + M);
-        const unsigned long long kk =
-            h >= 0 ? (static_cast<unsigned long long>(s_q[k]) << 10) | static_cast<unsigned>(k)
-                   : (1ull << 63) | (static_cast<unsigned long long>(-h) << 10) | static_cast<unsigned>(k);
+        const unsigned long long kk = dispatch_key(h, s_q[k], k, mc);
         if (kk < key) {
           key = kk;
           bM = M;
@@ -785,15 +840,20 @@ stream_waitlist_kernel(int n, int64_t hi, const int64_t *arrival, const int32_t 
 }
 
 // 8. Admission, one warp per decoder: entry x of the queue is admitted while
-//    it and every entry before it satisfy used + (prompts admitted before) +
-//    p + U <= cap.
+//    it and every entry before it satisfy used + (the increments of the
+//    entries admitted before) + p + U <= cap, the increment being p, p + U
+//    (staged) or 2p + U (held).  Each decoder's statistics gain its queue
+//    left waiting times the steps to the next batch, and its admissions.
 __global__ void __launch_bounds__(kSt, 1)
-stream_admit_kernel(int D, int32_t cap, int nw, const int64_t *wseg, const int32_t *wperm,
+stream_admit_kernel(int D, int32_t cap, int acct, int nw, int64_t hi, int64_t hi_next,
+                    const int64_t *arrival, const int64_t *wseg, const int32_t *wperm,
                     const int32_t *wid, const int32_t *prompt, const int32_t *U,
-                    const long long *used, uint8_t *st, int32_t *g, int64_t *stats_b) {
+                    const long long *used, uint8_t *st, int32_t *g, int32_t *res_u,
+                    int64_t *stats_b, int64_t *dst) {
   pdl_prologue();
   __shared__ int s_adm;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const long long span = arrival[hi_next - 1] - arrival[hi - 1];
   if (tid == 0) s_adm = 0;
   __syncthreads();
   for (int k = warp; k < D; k += kStWarps) {
@@ -806,25 +866,33 @@ stream_admit_kernel(int D, int32_t cap, int nw, const int64_t *wseg, const int32
       const bool valid = x < x1;
       const int id = valid ? wid[wperm[x]] : -1;
       const long long p = valid ? prompt[id] : 0, uu = valid ? U[id] : 0;
-      long long incl = p;
+      const long long inc = acct == MAPS_STREAM_OCCUPANCY ? p
+                            : acct == MAPS_STREAM_STAGED  ? p + uu
+                                                          : 2 * p + uu;
+      long long incl = inc;
 #pragma unroll
       for (int off = 1; off < 32; off <<= 1) {
         const long long y = __shfl_up_sync(0xffffffffu, incl, off);
         if (lane >= off) incl += y;
       }
-      const bool ok = valid && u + (incl - p) + p + uu <= cap;
+      const bool ok = valid && u + (incl - inc) + p + uu <= cap;
       const unsigned fail = __ballot_sync(0xffffffffu, valid && !ok);
       const unsigned vmask = __ballot_sync(0xffffffffu, valid);
       const int nadm = fail ? __ffs(fail) - 1 : __popc(vmask);
       if (lane < nadm) {
         st[id] = kRunning;
         g[id] = 0;
+        res_u[id] = static_cast<int32_t>(uu);
       }
       if (nadm > 0) u += __shfl_sync(0xffffffffu, incl, nadm - 1);
       adm += nadm;
       stop = fail != 0;
     }
     if (lane == 0 && adm) atomicAdd(&s_adm, adm);
+    if (lane == 0 && dst != nullptr) {  // decoder k is this warp's alone
+      dst[3 * k] += (x1 - wseg[k] - adm) * span;
+      dst[3 * k + 2] += adm;
+    }
   }
   __syncthreads();
   if (tid == 0) {
@@ -837,7 +905,7 @@ struct StreamWs {
   size_t sub_bytes;  // [0, sub_bytes): workspace of the calls the loop makes
   StreamState *S;
   uint8_t *st;
-  int32_t *g, *dec, *U;
+  int32_t *g, *dec, *U, *res_u;
   long long *disp;
   int32_t *act[2];
   int32_t *done_id, *done_rem, *done_perm, *zeros;
@@ -872,6 +940,7 @@ StreamWs carve_stream(Carve &c, const maps_stream_cfg &cfg) {
   w.g = c.take<int32_t>(N);
   w.dec = c.take<int32_t>(N);
   w.U = c.take<int32_t>(N);
+  w.res_u = c.take<int32_t>(N);
   w.disp = c.take<long long>(N);
   w.act[0] = c.take<int32_t>(N);
   w.act[1] = c.take<int32_t>(N);
@@ -907,7 +976,10 @@ StreamWs carve_stream(Carve &c, const maps_stream_cfg &cfg) {
 bool cfg_ok(const maps_stream_cfg *c) {
   return c != nullptr && c->N >= 1 && c->N <= 0x7fffffffLL && c->D >= 1 && c->D <= kStreamMaxD &&
          c->H >= 1 && c->H <= (1 << 28) && c->cap >= 0 && c->batch >= 1 && c->window >= 1 &&
-         c->alpha_ppm > 0 && c->alpha_ppm < 1000000u;
+         c->alpha_ppm > 0 && c->alpha_ppm < 1000000u && c->dispatch_policy >= MAPS_STREAM_MAPS &&
+         c->dispatch_policy <= MAPS_STREAM_LR && c->local_order >= MAPS_STREAM_SJF &&
+         c->local_order <= MAPS_STREAM_FCFS && c->accounting >= MAPS_STREAM_OCCUPANCY &&
+         c->accounting <= MAPS_STREAM_HELD;
 }
 
 int grid_for(int64_t n, int threads = 256) {
@@ -930,7 +1002,8 @@ size_t maps_stream_workspace_size(const maps_stream_cfg *cfg) {
 
 int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const int32_t *prompt,
                     const int32_t *true_len, const int32_t *pred, int32_t *choice_out,
-                    int32_t *q_out, int64_t *stats_out, void *ws, size_t ws_bytes, void *stream) {
+                    int32_t *q_out, int64_t *stats_out, int64_t *dec_stats_out, void *ws,
+                    size_t ws_bytes, void *stream) {
   using namespace maps;
   if (!cfg_ok(cfg) || arrival_ms == nullptr || prompt == nullptr || true_len == nullptr ||
       pred == nullptr || choice_out == nullptr || q_out == nullptr || stats_out == nullptr)
@@ -946,6 +1019,8 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
 
   MAPS_TRY(cuda_ok(cudaMemsetAsync(w.st, 0, static_cast<size_t>(N), s)));
   MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zeros, 0, static_cast<size_t>(N) * sizeof(int32_t), s)));
+  if (dec_stats_out != nullptr)
+    MAPS_TRY(cuda_ok(cudaMemsetAsync(dec_stats_out, 0, static_cast<size_t>(c.D) * 3 * sizeof(int64_t), s)));
   launch_pdl(stream_init_kernel, 1, kSt, 0, s, std::min(N, B), D, c.cap, arrival_ms, w.capv, w.S);
   launch_pdl(stream_validate_kernel, grid_for(N), 256, 0, s, N, arrival_ms, prompt, true_len, pred, status);
   MAPS_TRY(launch_ok());
@@ -961,9 +1036,9 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
     const int nb = static_cast<int>(hi - lo);
     int32_t *act_in = w.act[b & 1], *act = w.act[(b & 1) ^ 1];
     int64_t *stats_b = stats_out + 4 * b;
-    launch_pdl(stream_advance_kernel, 1, kSt, 0, s, hi, D, c.cap, arrival_ms, prompt, true_len, w.st, w.g,
-                                            w.dec, act_in, act, w.done_id, w.done_rem, w.used, w.S,
-                                            stats_b);
+    launch_pdl(stream_advance_kernel, 1, kSt, 0, s, hi, D, c.cap, c.accounting, arrival_ms, prompt,
+               true_len, w.res_u, w.st, w.g, w.dec, act_in, act, w.done_id, w.done_rem, w.used, w.S,
+               stats_b, dec_stats_out);
     MAPS_TRY(launch_ok());
     MAPS_TRY(cuda_ok(cudaMemcpyAsync(&hs, w.S, sizeof(hs), cudaMemcpyDeviceToHost, s)));
     MAPS_TRY(cuda_ok(cudaStreamSynchronize(s)));
@@ -985,28 +1060,34 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
     const bool rr = cs == MAPS_E_UNBOUNDED;
     if (cs != MAPS_OK && !rr) return cs;
     if (rr)
-      launch_pdl(stream_rr_kernel, grid_for(nact + nb), 256, 0, s, nact + nb, nb, lo, D, w.qpred, w.Uq,
-                                                           choice_out);
+      launch_pdl(stream_rr_kernel, grid_for(nact + nb), 256, 0, s, nact + nb, nb, lo, D, 1, w.qpred,
+                 w.Uq, choice_out);
     launch_pdl(stream_csr_kernel, 1, kSt, 0, s, nact, D, rr ? 1 : 0, w.q_dev, q_out + b, act, w.st, w.g,
                                         w.dec, prompt, w.Uq, w.U, w.res_off, w.rp, w.rg, w.rU,
                                         w.Q);  // 4.
     MAPS_TRY(launch_ok());
-    if (!rr) {  // 5.
+    const int mc = c.dispatch_policy == MAPS_STREAM_MC ? 1 : 0;
+    if (!rr && c.dispatch_policy == MAPS_STREAM_RR) {  // 5'.
+      launch_pdl(stream_rr_kernel, grid_for(nb), 256, 0, s, nb, nb, lo, D, 0, w.qpred, w.Uq, choice_out);
+      MAPS_TRY(launch_ok());
+    } else if (!rr && c.dispatch_policy == MAPS_STREAM_LR) {
+      launch_pdl(stream_lr_kernel, 1, 32, 0, s, D, nb, w.res_off, choice_out + lo);
+      MAPS_TRY(launch_ok());
+    } else if (!rr) {  // 5.
       const size_t dsm = stream_dispatch_smem(D, nact, nb);
       if (dsm + 2048 <= static_cast<size_t>(max_smem_optin())) {
         // the decoders' pairs fit in shared memory: no dense projection
         MAPS_TRY(cuda_ok(cudaFuncSetAttribute(stream_dispatch_kernel,
                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               static_cast<int>(dsm))));
-        launch_pdl(stream_dispatch_kernel, 1, kSt, dsm, s, D, c.H, nb, w.res_off, w.rp, w.rg, w.rU,
-                   w.capv, w.Q, prompt + lo, w.Uq + nact, choice_out + lo, w.headroom, status);
+        launch_pdl(stream_dispatch_kernel, 1, kSt, dsm, s, D, c.H, nb, mc, w.res_off, w.rp, w.rg,
+                   w.rU, w.capv, w.Q, prompt + lo, w.Uq + nact, choice_out + lo, w.headroom, status);
         MAPS_TRY(launch_ok());
       } else {
         MAPS_TRY(maps_project_occupancy(D, c.H, w.res_off, nact, w.rp, w.rg, w.rU, w.K, nullptr, ws,
                                         w.sub_bytes, stream));
-        MAPS_TRY(maps_dispatch(MAPS_MODE_SEQUENTIAL, D, c.H, 1, w.K, nullptr, w.capv, w.Q, nullptr, 0,
-                               nullptr, nullptr, nullptr, nb, prompt + lo, w.Uq + nact,
-                               choice_out + lo, w.headroom, ws, w.sub_bytes, stream));
+        MAPS_TRY(dispatch_sequential(D, c.H, w.K, w.capv, w.Q, nb, prompt + lo, w.Uq + nact,
+                                     choice_out + lo, w.headroom, mc != 0, ws, s));
       }
     }
     launch_pdl(stream_enqueue_kernel, grid_for(nb), 256, 0, s, lo, nb, nact, hi, D, arrival_ms,
@@ -1016,10 +1097,14 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
     launch_pdl(stream_waitlist_kernel, 1, kSt, 0, s, n_all, hi, arrival_ms, act, w.st, w.dec, w.U, w.disp,
                                              w.wid, w.wdec, w.wU, w.wwait, w.warr);  // 7.
     MAPS_TRY(launch_ok());
-    MAPS_TRY(maps_order_local(nw, D, w.wdec, w.wU, w.wwait, w.warr, c.max_wait, w.wperm, w.wseg, ws,
+    // FCFS: every wait is >= 0 > -1, so every entry is promoted: arrival order
+    const int32_t mw = c.local_order == MAPS_STREAM_FCFS ? -1 : c.max_wait;
+    MAPS_TRY(maps_order_local(nw, D, w.wdec, w.wU, w.wwait, w.warr, mw, w.wperm, w.wseg, ws,
                               w.sub_bytes, stream));
-    launch_pdl(stream_admit_kernel, 1, kSt, 0, s, D, c.cap, nw, w.wseg, w.wperm, w.wid, prompt, w.U, w.used,
-                                          w.st, w.g, stats_b);  // 8.
+    const int64_t hi_next = b + 1 < nbatch ? std::min(hi + B, N) : hi;
+    launch_pdl(stream_admit_kernel, 1, kSt, 0, s, D, c.cap, c.accounting, nw, hi, hi_next, arrival_ms,
+               w.wseg, w.wperm, w.wid, prompt, w.U, w.used, w.st, w.g, w.res_u, stats_b,
+               dec_stats_out);  // 8.
     MAPS_TRY(launch_ok());
   }
   return maps_check(ws, stream);

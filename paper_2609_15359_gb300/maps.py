@@ -37,7 +37,15 @@ class StreamCfg(ctypes.Structure):
     """``maps_stream_cfg`` of include/maps.h."""
     _fields_ = [("N", ctypes.c_int64), ("D", ctypes.c_int32), ("H", ctypes.c_int32),
                 ("cap", ctypes.c_int32), ("batch", ctypes.c_int32), ("window", ctypes.c_int32),
-                ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32)]
+                ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32),
+                ("dispatch_policy", ctypes.c_int32), ("local_order", ctypes.c_int32),
+                ("accounting", ctypes.c_int32)]
+
+
+# maps_stream_cfg policy fields
+STREAM_MAPS, STREAM_MC, STREAM_RR, STREAM_LR = 0, 1, 2, 3
+STREAM_SJF, STREAM_FCFS = 0, 1
+STREAM_OCCUPANCY, STREAM_STAGED, STREAM_HELD = 0, 1, 2
 
 
 class RRCfg(ctypes.Structure):
@@ -80,7 +88,7 @@ def _load():
         "maps_rr_pressure": ([ctypes.POINTER(RRCfg), i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
                              ctypes.c_int),
         "maps_stream_workspace_size": ([ctypes.POINTER(StreamCfg)], sz),
-        "maps_stream_run": ([ctypes.POINTER(StreamCfg), vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
+        "maps_stream_run": ([ctypes.POINTER(StreamCfg), vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
                             ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
@@ -230,21 +238,25 @@ def maps_order_local_static(D: int, dec, bound, wait, arrival, max_wait: int, pe
 
 
 def stream_cfg(N: int, D: int, H: int, cap: int, batch: int, window: int, alpha_ppm: int,
-               max_wait: int) -> StreamCfg:
+               max_wait: int, dispatch_policy: int = STREAM_MAPS, local_order: int = STREAM_SJF,
+               accounting: int = STREAM_OCCUPANCY) -> StreamCfg:
     return StreamCfg(int(N), int(D), int(H), int(cap), int(batch), int(window), int(alpha_ppm),
-                     int(max_wait))
+                     int(max_wait), int(dispatch_policy), int(local_order), int(accounting))
 
 
 def maps_stream_run(cfg: StreamCfg, arrival_ms, prompt, true_len, pred, choice_out, q_out,
-                    stats_out, ws: Workspace | None = None, stream=None) -> int:
-    """The whole streaming loop on the device; returns the full status."""
+                    stats_out, dec_stats_out=None, ws: Workspace | None = None,
+                    stream=None) -> int:
+    """The whole streaming loop on the device; returns the full status.
+    dec_stats_out: optional [D][3] int64 per-decoder statistics."""
     ws = ws or Workspace()
     ws.ensure(lib.maps_stream_workspace_size(ctypes.byref(cfg)))
     return lib.maps_stream_run(ctypes.byref(cfg), _ptr(arrival_ms, torch.int64),
                                _ptr(prompt, torch.int32), _ptr(true_len, torch.int32),
                                _ptr(pred, torch.int32), _ptr(choice_out, torch.int32),
                                _ptr(q_out, torch.int32), _ptr(stats_out, torch.int64),
-                               ws.ptr, ws.nbytes, _stream(stream))
+                               _ptr(dec_stats_out, torch.int64), ws.ptr, ws.nbytes,
+                               _stream(stream))
 
 
 def maps_rr_pressure(N: int, C: int, t_tok_us: int, theta_ppm: int, arrival_us, prompt, out_len,
