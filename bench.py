@@ -660,10 +660,12 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
     stats = torch.empty((nb, 4), dtype=torch.int64, device=device)
     ws = M.Workspace(device=device)
 
-    def run(n):
+    ds = torch.empty((w["D"], 3), dtype=torch.int64, device=device)
+
+    def run(n, pol=(0, 0, 0)):
         cfg = M.stream_cfg(n, w["D"], w["H"], w["cap"], B, w["window"], w["alpha_ppm"],
-                           w["max_wait"])
-        st = M.maps_stream_run(cfg, arr[:n], pr[:n], tr[:n], pd[:n], ch[:n], q, stats, ws=ws)
+                           w["max_wait"], *pol)
+        st = M.maps_stream_run(cfg, arr[:n], pr[:n], tr[:n], pd[:n], ch[:n], q, stats, ds, ws=ws)
         if st != 0:
             raise RuntimeError(f"maps_stream_run status {st}")
 
@@ -676,6 +678,25 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
            "value": N / secs, "unit": "decisions/s", "seconds": secs,
            "ms_per_batch": secs / nb * 1e3, "dispatch_mode": "SEQUENTIAL",
            "timing": "host wall clock of one maps_stream_run call (it synchronises per batch)"}
+    # the policy variants on the same workload: loop throughput and outcome
+    # (waiting-queue integral in request-steps, over-capacity events, admissions)
+    variants = {}
+    span = int(w["arrival_ms"][N - 1] - w["arrival_ms"][min(B, N) - 1])  # first to last dispatch
+    for name, pol in [("maps", (0, 0, 0)), ("mc", (1, 0, 0)), ("round_robin", (2, 0, 0)),
+                      ("least_requests", (3, 0, 0)), ("fcfs", (0, 1, 0)),
+                      ("staged", (0, 0, 1)), ("held", (0, 0, 2))]:
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        run(N, pol)
+        sv = time.perf_counter() - t0
+        per = ds.cpu().numpy()
+        d = per.sum(axis=0).tolist()
+        tw = per[:, 0] / max(span, 1)  # time-weighted average queue length per decoder
+        variants[name] = {"value": N / sv, "seconds": sv, "queue_integral": d[0],
+                          "time_weighted_queue_mean": float(tw.mean()),
+                          "time_weighted_queue_max": float(tw.max()),
+                          "overflow_events": d[1], "admissions": d[2]}
+    out["variants"] = variants
     if cpu_sample:
         import oracle as O
         n = min(cpu_sample, N)
