@@ -235,6 +235,17 @@ def arena_views(arena, fields: dict) -> dict:
     return {k: arena[o:o + c * np.dtype(dt).itemsize].view(tdt[dt]) for k, (o, c, dt) in fields.items()}
 
 
+def algorithmic_bytes(w: dict) -> dict:
+    """Algorithmic bytes per call: what the method must move."""
+    D, H, R, J = w["D"], w["H"], w["R"], w["J"]
+    return {
+        "calibrate": 8 * w["n_cal"] + 8 * (R + J),     # residual pairs in; predictions in, bounds out
+        "occupancy": 12 * R + 4 * D * H + 8 * (D + 1),  # residents in, K out, offsets
+        "dispatch": 4 * D * H + 8 * J + 12 * J + 8 * D,  # K, candidates, choice + headroom, cap + Q
+        "order": 20 * (R + J) + 8 * (D + 1),           # four int32 keys in, perm out, segments
+    }
+
+
 class Step:
     """Device buffers and the four C-ABI calls of one hot-path pass."""
 
@@ -320,7 +331,7 @@ class Step:
 
 def W_CONFIG_FACTOR(w: dict) -> int:
     from paper_2609_15359_gb300 import workloads as W
-    return int(W.WORKLOADS[WORKLOAD]["feasible_factor"])
+    return int(W.WORKLOADS[w.get("name", WORKLOAD)]["feasible_factor"])
 
 
 def host_inputs(w):
@@ -560,13 +571,7 @@ def bench_gpu(args, world, rank, local, dist):
 
     peaks = measured_peaks()
     D, H, R, J = step.D, step.H, step.R, step.J
-    # algorithmic bytes per call (what the method must move)
-    alg = {
-        "calibrate": 8 * w["n_cal"] + 8 * (R + J),     # residual pairs in; predictions in, bounds out
-        "occupancy": 12 * R + 4 * D * H + 8 * (D + 1),  # residents in, K out, offsets
-        "dispatch": 4 * D * H + 8 * J + 12 * J + 8 * D,  # K, candidates, choice + headroom, cap + Q
-        "order": 20 * (R + J) + 8 * (D + 1),           # four int32 keys in, perm out, segments
-    }
+    alg = algorithmic_bytes(w)
     call_ms = {"calibrate": cal_ms, "occupancy": occ_ms, "dispatch": disp_ms, "order": order_ms}
     # the dispatch's scoring kernel alone: K in, candidates in, choice and
     # headroom out; the candidate bucketing by horizon tile is left out, as the
@@ -638,6 +643,70 @@ def bench_gpu(args, world, rank, local, dist):
 
 
 # ---------------------------------------------------------------------------
+# the smaller configurations: Tiny, D16 and D64 (each of its three bound sets)
+# ---------------------------------------------------------------------------
+
+def bench_configs(device, steps: int = 20) -> dict:
+    """The same four calls on each smaller configuration: per step a CUDA-graph
+    replay after an L2 flush (event-timed), then a pass of direct launches with
+    an event between calls for the per-call split and its HBM fractions."""
+    import torch
+    from paper_2609_15359_gb300 import workloads as W
+    peaks = measured_peaks()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+    out = {}
+    for name in ("tiny", "d16", "d64"):
+        w = W.make(name)
+        for alpha in w["alphas_ppm"]:
+            step = Step(w, device)
+            step.alpha = alpha
+            for _ in range(3):
+                step.run()
+            torch.cuda.synchronize()
+            step.check()
+            side = torch.cuda.Stream()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
+                step.run()
+            torch.cuda.synchronize()
+            ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+            for i in range(steps):
+                flush.zero_()
+                ev[i][3].record()
+                graph.replay()
+                ev[i][4].record()
+            torch.cuda.synchronize()
+            step_ms = float(np.mean([e[3].elapsed_time(e[4]) for e in ev]))
+            for i in range(steps):
+                flush.zero_()
+                ev[i][3].record()
+                step.run(ev=ev[i])
+                ev[i][4].record()
+            torch.cuda.synchronize()
+            step.check()
+            call_ms = {"calibrate": [e[3].elapsed_time(e[0]) for e in ev],
+                       "occupancy": [e[0].elapsed_time(e[1]) for e in ev],
+                       "dispatch": [e[1].elapsed_time(e[2]) for e in ev],
+                       "order": [e[2].elapsed_time(e[4]) for e in ev]}
+            alg = algorithmic_bytes(w)
+            calls = {}
+            for c in alg:
+                us = float(np.mean(call_ms[c])) * 1e3
+                calls[c] = {"us": us, "algorithmic_bytes": alg[c],
+                            "frac_of_measured_hbm": alg[c] / (us / 1e6) / 1e9 / peaks["hbm_gbs"]}
+            key = name if len(w["alphas_ppm"]) == 1 else f"{name}_alpha{alpha / 1e6:g}"
+            out[key] = {"workload": W.DESCRIPTIONS[name], "alpha_ppm": alpha,
+                        "D": w["D"], "H": w["H"], "residents": w["R"], "candidates": w["J"],
+                        "ms_per_step": step_ms, "decisions_per_s": w["J"] / (step_ms / 1e3),
+                        "occupancy_cells_per_s": w["D"] * w["H"] / (step_ms / 1e3),
+                        "calls": calls, "steps": steps,
+                        "timing": "graph replay per step after a 256 MiB L2 flush; calls split "
+                                  "by events between direct launches"}
+            del step, graph
+    return out
+
+
+# ---------------------------------------------------------------------------
 # the streaming loop (all 1,000,000 requests through maps_stream_run)
 # ---------------------------------------------------------------------------
 
@@ -662,9 +731,9 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
 
     ds = torch.empty((w["D"], 3), dtype=torch.int64, device=device)
 
-    def run(n, pol=(0, 0, 0)):
-        cfg = M.stream_cfg(n, w["D"], w["H"], w["cap"], B, w["window"], w["alpha_ppm"],
-                           w["max_wait"], *pol)
+    def run(n, pol=(0, 0, 0), cap=None):
+        cfg = M.stream_cfg(n, w["D"], w["H"], w["cap"] if cap is None else cap, B, w["window"],
+                           w["alpha_ppm"], w["max_wait"], *pol)
         st = M.maps_stream_run(cfg, arr[:n], pr[:n], tr[:n], pd[:n], ch[:n], q, stats, ds, ws=ws)
         if st != 0:
             raise RuntimeError(f"maps_stream_run status {st}")
@@ -678,25 +747,28 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
            "value": N / secs, "unit": "decisions/s", "seconds": secs,
            "ms_per_batch": secs / nb * 1e3, "dispatch_mode": "SEQUENTIAL",
            "timing": "host wall clock of one maps_stream_run call (it synchronises per batch)"}
-    # the policy variants on the same workload: loop throughput and outcome
-    # (waiting-queue integral in request-steps, over-capacity events, admissions)
-    variants = {}
+    # the policy variants on the same arrivals: loop throughput and outcome
+    # (waiting-queue integral in request-steps, over-capacity events,
+    # admissions), at the workload's capacity (where no queue forms) and at a
+    # tight capacity of 16,000 tokens per decoder (loaded, still stable)
     span = int(w["arrival_ms"][N - 1] - w["arrival_ms"][min(B, N) - 1])  # first to last dispatch
-    for name, pol in [("maps", (0, 0, 0)), ("mc", (1, 0, 0)), ("round_robin", (2, 0, 0)),
-                      ("least_requests", (3, 0, 0)), ("fcfs", (0, 1, 0)),
-                      ("staged", (0, 0, 1)), ("held", (0, 0, 2))]:
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        run(N, pol)
-        sv = time.perf_counter() - t0
-        per = ds.cpu().numpy()
-        d = per.sum(axis=0).tolist()
-        tw = per[:, 0] / max(span, 1)  # time-weighted average queue length per decoder
-        variants[name] = {"value": N / sv, "seconds": sv, "queue_integral": d[0],
-                          "time_weighted_queue_mean": float(tw.mean()),
-                          "time_weighted_queue_max": float(tw.max()),
-                          "overflow_events": d[1], "admissions": d[2]}
-    out["variants"] = variants
+    for label, cap in (("variants", None), ("variants_cap16000", 16000)):
+        variants = {}
+        for name, pol in [("maps", (0, 0, 0)), ("mc", (1, 0, 0)), ("round_robin", (2, 0, 0)),
+                          ("least_requests", (3, 0, 0)), ("fcfs", (0, 1, 0)),
+                          ("staged", (0, 0, 1)), ("held", (0, 0, 2))]:
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            run(N, pol, cap)
+            sv = time.perf_counter() - t0
+            per = ds.cpu().numpy()
+            d = per.sum(axis=0).tolist()
+            tw = per[:, 0] / max(span, 1)  # time-weighted average queue length per decoder
+            variants[name] = {"value": N / sv, "seconds": sv, "queue_integral": d[0],
+                              "time_weighted_queue_mean": float(tw.mean()),
+                              "time_weighted_queue_max": float(tw.max()),
+                              "overflow_events": d[1], "admissions": d[2]}
+        out[label] = variants
     if cpu_sample:
         import oracle as O
         n = min(cpu_sample, N)
@@ -925,6 +997,7 @@ def main():
                                          0 if args.no_cpu_baseline else 100000)
             res["rr_pressure"] = bench_rr(torch.device(f"cuda:{local}"),
                                           0 if args.no_cpu_baseline else 24)
+            res["configs"] = bench_configs(torch.device(f"cuda:{local}"))
         print(json.dumps(res), flush=True)
     if dist is not None:
         dist.destroy_process_group()
