@@ -60,7 +60,8 @@ class StreamCfg(ctypes.Structure):
                 ("batch", ctypes.c_int32), ("window", ctypes.c_int32),
                 ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32),
                 ("dispatch", ctypes.c_int32), ("local", ctypes.c_int32),
-                ("accounting", ctypes.c_int32)]
+                ("accounting", ctypes.c_int32), ("per_step", ctypes.c_int32),
+                ("beta", ctypes.c_int32)]
 
 
 # streaming-loop policies (the Sec. 4 ablations, the baselines, App. C)
@@ -99,7 +100,8 @@ def lib():
         L.oracle_order_local.argtypes = [ctypes.c_int64, ctypes.c_int32, vp, vp,
                                          vp, vp, ctypes.c_int32, vp, vp]
         L.oracle_stream.argtypes = [ctypes.POINTER(StreamCfg), _i64p, _i32p,
-                                    _i32p, _i32p, _i32p, _i32p, _i64p, _i64p]
+                                    _i32p, _i32p, ctypes.c_void_p, _i32p, _i32p, _i64p,
+                                    _i64p]
         L.oracle_rr_pressure.argtypes = [ctypes.POINTER(RRCfg), _i64p, _i32p, _i32p,
                                          _i64p, _i64p, _i64p, ctypes.POINTER(ctypes.c_int64)]
         _lib = L
@@ -203,21 +205,27 @@ def order_local(D: int, dec, bnd, wait, arrival, max_wait: int):
 
 def stream(N, D, H, cap, batch, window, alpha_ppm, max_wait, arrival_ms,
            prompt, true_len, pred, dispatch=DISPATCH_MAPS, local=LOCAL_SJF,
-           accounting=ACCOUNT_OCCUPANCY, with_dec_stats=False):
+           accounting=ACCOUNT_OCCUPANCY, with_dec_stats=False, per_step=0, beta=-1,
+           pred_delay=None):
     """Returns (status, choice, q, stats [nb][4]) and, with with_dec_stats,
-    the per-decoder statistics [D][3] as a fifth item."""
+    the per-decoder statistics [D][4] as a fifth item.  per_step=1 admits on
+    every step with preemption; beta >= 0 with pred_delay [N] defers a
+    request until its bound is available, round robin after beta steps."""
     cfg = StreamCfg(N, D, H, cap, batch, window, alpha_ppm, max_wait, dispatch, local,
-                    accounting)
+                    accounting, per_step, beta)
     nb = (N + batch - 1) // batch
     choice = np.empty(N, dtype=np.int32)
     q = np.empty(nb, dtype=np.int32)
     stats = np.empty(4 * nb, dtype=np.int64)
-    dstats = np.zeros(3 * D, dtype=np.int64)
+    dstats = np.zeros(4 * D, dtype=np.int64)
+    pdl = None if pred_delay is None else _c32(pred_delay[:N])
     st = lib().oracle_stream(ctypes.byref(cfg), _c64(arrival_ms[:N]),
                              _c32(prompt[:N]), _c32(true_len[:N]),
-                             _c32(pred[:N]), choice, q, stats, dstats)
+                             _c32(pred[:N]),
+                             None if pdl is None else pdl.ctypes.data_as(ctypes.c_void_p),
+                             choice, q, stats, dstats)
     if with_dec_stats:
-        return st, choice, q, stats.reshape(nb, 4), dstats.reshape(D, 3)
+        return st, choice, q, stats.reshape(nb, 4), dstats.reshape(D, 4)
     return st, choice, q, stats.reshape(nb, 4)
 
 

@@ -438,22 +438,76 @@ static int cmp_completion(const void *a, const void *b)
     return (x->id > y->id) - (x->id < y->id);
 }
 
+/* Per-step mode: each decoder's running requests in admission order (a
+ * doubly linked list; the tail is the most recently admitted), the requests
+ * preempted since the last dispatch step (a stack: the latest on top, the
+ * head of the waiting queue), and the waiting queue as ordered at the last
+ * dispatch step (positions [qhead, qend) of that order). */
+typedef struct {
+    int64_t *next, *prev;   /* [N] running-list links, -1 at the ends */
+    int64_t *head, *tail;   /* [D] */
+    int64_t *pnext;         /* [N] preempted-stack links */
+    int64_t *ptop;          /* [D] */
+    int64_t *qhead, *qend;  /* [D] */
+} step_lists;
+
+static void run_append(step_lists *L, int32_t k, int64_t id)
+{
+    L->next[id] = -1;
+    L->prev[id] = L->tail[k];
+    if (L->tail[k] >= 0)
+        L->next[L->tail[k]] = id;
+    else
+        L->head[k] = id;
+    L->tail[k] = id;
+}
+
+static void run_unlink(step_lists *L, int32_t k, int64_t id)
+{
+    if (L->prev[id] >= 0)
+        L->next[L->prev[id]] = L->next[id];
+    else
+        L->head[k] = L->next[id];
+    if (L->next[id] >= 0)
+        L->prev[L->next[id]] = L->prev[id];
+    else
+        L->tail[k] = L->prev[id];
+}
+
+/* What admission counts a running request for (cfg->accounting). */
+static int64_t held_tokens(int32_t accounting, int64_t p, int64_t g, int64_t r)
+{
+    int64_t out_part = r > g ? r : g;
+    return accounting == 0 ? p + g : accounting == 1 ? p + out_part : 2 * p + out_part;
+}
+
+/* What an admission adds to that count. */
+static int64_t admit_tokens(int32_t accounting, int64_t p, int64_t u)
+{
+    return accounting == 0 ? p : accounting == 1 ? p + u : 2 * p + u;
+}
+
 int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                   const int32_t *prompt, const int32_t *true_len,
-                  const int32_t *pred, int32_t *choice_out, int32_t *q_out,
+                  const int32_t *pred, const int32_t *pred_delay,
+                  int32_t *choice_out, int32_t *q_out,
                   int64_t *stats_out, int64_t *dec_stats_out)
 {
     if (cfg == NULL || cfg->N < 1 || cfg->N > I32_MAX || cfg->D < 1 ||
         cfg->H < 1 || cfg->cap < 0 || cfg->batch < 1 || cfg->window < 1 ||
         cfg->alpha_ppm == 0 || cfg->alpha_ppm >= 1000000u ||
         cfg->dispatch < 0 || cfg->dispatch > 3 || cfg->local < 0 || cfg->local > 1 ||
-        cfg->accounting < 0 || cfg->accounting > 2)
+        cfg->accounting < 0 || cfg->accounting > 2 || cfg->per_step < 0 ||
+        cfg->per_step > 1)
         return ORACLE_E_INVALID;
     const int64_t N = cfg->N;
     const int32_t D = cfg->D, H = cfg->H, Bsz = cfg->batch, Wn = cfg->window;
     const int64_t nb = (N + Bsz - 1) / Bsz;
+    /* deferral: a bound becomes available pred_delay steps after arrival */
+    const int defer = cfg->beta >= 0 && pred_delay != NULL;
     for (int64_t i = 0; i < N; ++i)
         if (prompt[i] < 0 || true_len[i] < 1 || pred[i] < 0 ||
+            (pred_delay != NULL && pred_delay[i] < 0) ||
             (i > 0 && arrival_ms[i] < arrival_ms[i - 1]))
             return ORACLE_E_RANGE;
 
@@ -483,44 +537,133 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
     int32_t *wwait = (int32_t *)malloc((size_t)N * sizeof(int32_t));
     int32_t *warr = (int32_t *)malloc((size_t)N * sizeof(int32_t));
     int32_t *wperm = (int32_t *)malloc((size_t)N * sizeof(int32_t));
-    int32_t *cU = (int32_t *)malloc((size_t)Bsz * sizeof(int32_t));
-    int64_t *hr = (int64_t *)malloc((size_t)Bsz * sizeof(int64_t));
+    int64_t *cid = (int64_t *)malloc((size_t)N * sizeof(int64_t));  /* dispatched by the policy */
+    int32_t *cp = (int32_t *)malloc((size_t)N * sizeof(int32_t));
+    int32_t *cU = (int32_t *)malloc((size_t)N * sizeof(int32_t));
+    int32_t *cch = (int32_t *)malloc((size_t)N * sizeof(int32_t));
+    int64_t *hr = (int64_t *)malloc((size_t)N * sizeof(int64_t));
+    int64_t *pend = (int64_t *)malloc((size_t)N * sizeof(int64_t)); /* arrived, not dispatched */
     int32_t *res_u = (int32_t *)calloc((size_t)N, sizeof(int32_t)); /* bound reserved at admission */
     int64_t *occ = (int64_t *)malloc((size_t)D * sizeof(int64_t));
     int64_t *nreq = (int64_t *)malloc((size_t)D * sizeof(int64_t));
-    int64_t *dst = (int64_t *)calloc((size_t)D * 3, sizeof(int64_t));
+    int64_t *dst = (int64_t *)calloc((size_t)D * 4, sizeof(int64_t));
+    step_lists L;
+    L.next = (int64_t *)malloc((size_t)N * sizeof(int64_t));
+    L.prev = (int64_t *)malloc((size_t)N * sizeof(int64_t));
+    L.pnext = (int64_t *)malloc((size_t)N * sizeof(int64_t));
+    L.head = (int64_t *)malloc((size_t)D * sizeof(int64_t));
+    L.tail = (int64_t *)malloc((size_t)D * sizeof(int64_t));
+    L.ptop = (int64_t *)malloc((size_t)D * sizeof(int64_t));
+    L.qhead = (int64_t *)calloc((size_t)D, sizeof(int64_t));
+    L.qend = (int64_t *)calloc((size_t)D, sizeof(int64_t));
     if (!st || !g || !dec || !U || !disp || !act || !done || !win_true ||
         !win_pred || !K || !capv || !Q || !off || !used || !seg || !rp || !rg ||
-        !rU || !wid || !wdec || !wU || !wwait || !warr || !wperm || !cU || !hr ||
-        !res_u || !occ || !nreq || !dst) {
+        !rU || !wid || !wdec || !wU || !wwait || !warr || !wperm || !cid || !cp ||
+        !cU || !cch || !hr || !pend || !res_u || !occ || !nreq || !dst ||
+        !L.next || !L.prev || !L.pnext || !L.head || !L.tail || !L.ptop ||
+        !L.qhead || !L.qend) {
         status = ORACLE_E_INVALID;
         goto out;
     }
-    for (int32_t k = 0; k < D; ++k)
+    for (int32_t k = 0; k < D; ++k) {
         capv[k] = cfg->cap;
+        L.head[k] = L.tail[k] = L.ptop[k] = -1;
+    }
 
-    int64_t nact = 0, win_len = 0, win_head = 0;
+    int64_t nact = 0, npend = 0, win_len = 0, win_head = 0;
     int64_t prev_s = arrival_ms[(N < Bsz ? N : Bsz) - 1];
     for (int64_t b = 0; b < nb; ++b) {
         const int64_t lo = b * Bsz, hi = (lo + Bsz < N) ? lo + Bsz : N;
         const int64_t s = arrival_ms[hi - 1]; /* dispatch step of batch b */
         const int64_t delta = s - prev_s;
+        int64_t ndone = 0, admitted = 0;
 
         /* 1. Advance every running request by delta decode steps (one token
          *    per step); a request finishes when it reaches its true length. */
-        int64_t ndone = 0;
-        for (int64_t a = 0; a < nact; ++a) {
-            int64_t id = act[a];
-            if (st[id] != ST_RUNNING)
-                continue;
-            int64_t rem = (int64_t)true_len[id] - g[id];
-            if (rem <= delta) {
-                st[id] = ST_DONE;
-                done[ndone].step = prev_s + rem;
-                done[ndone].id = id;
-                ++ndone;
-            } else {
-                g[id] += (int32_t)delta;
+        if (!cfg->per_step) {
+            for (int64_t a = 0; a < nact; ++a) {
+                int64_t id = act[a];
+                if (st[id] != ST_RUNNING)
+                    continue;
+                int64_t rem = (int64_t)true_len[id] - g[id];
+                if (rem <= delta) {
+                    st[id] = ST_DONE;
+                    done[ndone].step = prev_s + rem;
+                    done[ndone].id = id;
+                    ++ndone;
+                } else {
+                    g[id] += (int32_t)delta;
+                }
+            }
+        } else {
+            /* Per-step mode: steps prev_s + 1 .. s one at a time, each
+             * decoder on its own.  Before its running requests take a token,
+             * a decoder whose tokens would pass its capacity preempts its
+             * most recently admitted request (which loses its tokens and
+             * goes to the head of the waiting queue) until they fit, but
+             * never its last one.  Requests reaching their true length
+             * complete.  On every step but the dispatch step s the queue
+             * admits in order (preempted requests first, the latest on top)
+             * while used + p + U <= capacity, the first misfit blocking. */
+            for (int64_t t = prev_s + 1; t <= s; ++t) {
+                for (int32_t k = 0; k < D; ++k) {
+                    int64_t tok = 0, n = 0;
+                    for (int64_t r = L.head[k]; r >= 0; r = L.next[r]) {
+                        tok += (int64_t)prompt[r] + g[r];
+                        ++n;
+                    }
+                    while (n > 1 && tok + n > capv[k]) {
+                        int64_t r = L.tail[k];
+                        run_unlink(&L, k, r);
+                        tok -= (int64_t)prompt[r] + g[r];
+                        --n;
+                        st[r] = ST_WAITING;
+                        g[r] = 0;
+                        L.pnext[r] = L.ptop[k];
+                        L.ptop[k] = r;
+                        dst[4 * k + 3] += 1;
+                    }
+                    for (int64_t r = L.head[k], nx; r >= 0; r = nx) {
+                        nx = L.next[r];
+                        g[r] += 1;
+                        if (g[r] == true_len[r]) {
+                            run_unlink(&L, k, r);
+                            st[r] = ST_DONE;
+                            done[ndone].step = t;
+                            done[ndone].id = r;
+                            ++ndone;
+                        }
+                    }
+                    if (t == s)
+                        continue;
+                    int64_t u = 0;
+                    for (int64_t r = L.head[k]; r >= 0; r = L.next[r])
+                        u += held_tokens(cfg->accounting, prompt[r], g[r], res_u[r]);
+                    for (;;) {
+                        int from_stack = L.ptop[k] >= 0;
+                        if (!from_stack && L.qhead[k] >= L.qend[k])
+                            break;
+                        int64_t r = from_stack ? L.ptop[k] : wid[wperm[L.qhead[k]]];
+                        if (u + prompt[r] + (int64_t)U[r] > capv[k])
+                            break;
+                        if (from_stack)
+                            L.ptop[k] = L.pnext[r];
+                        else
+                            L.qhead[k] += 1;
+                        st[r] = ST_RUNNING;
+                        g[r] = 0;
+                        res_u[r] = U[r];
+                        u += admit_tokens(cfg->accounting, prompt[r], U[r]);
+                        run_append(&L, k, r);
+                        ++admitted;
+                        dst[4 * k + 2] += 1;
+                    }
+                    /* requests waiting at decoder k through step t */
+                    int64_t wq = L.qend[k] - L.qhead[k];
+                    for (int64_t r = L.ptop[k]; r >= 0; r = L.pnext[r])
+                        ++wq;
+                    dst[4 * k] += wq;
+                }
             }
         }
         for (int32_t k = 0; k < D; ++k) {
@@ -542,12 +685,8 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                      * output reserved at its bound until generation ends --
                      * or, without the staged release, the prompt's
                      * reservation as well) */
-                    int64_t p = prompt[id], gg = g[id], r = res_u[id];
-                    int64_t out_part = r > gg ? r : gg;
-                    occ[dec[id]] += p + gg;
-                    used[dec[id]] += cfg->accounting == 0 ? p + gg
-                                   : cfg->accounting == 1 ? p + out_part
-                                                          : 2 * p + out_part;
+                    occ[dec[id]] += (int64_t)prompt[id] + g[id];
+                    used[dec[id]] += held_tokens(cfg->accounting, prompt[id], g[id], res_u[id]);
                 }
             }
             nact = w;
@@ -555,7 +694,7 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
         int64_t overflow = 0;
         for (int32_t k = 0; k < D; ++k) {
             overflow += occ[k] > capv[k];
-            dst[3 * k + 1] += occ[k] > capv[k];
+            dst[4 * k + 1] += occ[k] > capv[k];
         }
 
         /* 2. Sliding calibration window: the most recent completions,
@@ -588,27 +727,64 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
         }
         q_out[b] = rr ? -1 : (int32_t)q;
 
-        /* 4. Bounds for every request still in the system and the batch. */
+        /* 4. The requests dispatched at s: the batch joins the arrived ones
+         *    not yet dispatched; those whose bound is available go to the
+         *    dispatch policy, those that waited beta steps past arrival
+         *    without one (or are left at the last dispatch step) go round
+         *    robin (Sec. 3.3, the timeout; App. D), the rest wait. */
+        for (int64_t i = lo; i < hi; ++i)
+            pend[npend++] = i;
+        int64_t nc = 0, keep = 0, nto = 0;
+        for (int64_t x = 0; x < npend; ++x) {
+            int64_t id = pend[x];
+            int avail = !defer || arrival_ms[id] + pred_delay[id] <= s;
+            int timed_out = !avail && (arrival_ms[id] + cfg->beta <= s || b == nb - 1);
+            if (avail) {
+                cid[nc++] = id;
+            } else if (timed_out) {
+                /* round robin without a bound: projected to the horizon
+                 * until its prediction arrives */
+                choice_out[id] = (int32_t)(id % D);
+                st[id] = ST_WAITING;
+                dec[id] = (int32_t)(id % D);
+                disp[id] = s;
+                g[id] = 0;
+                U[id] = H;
+                act[nact++] = id;
+                nreq[id % D] += 1;
+                ++nto;
+            } else {
+                pend[keep++] = id;
+            }
+        }
+        npend = keep;
+
+        /*    Bounds for every request in the system (the horizon while its
+         *    prediction is not in yet) and for the policy's candidates. */
         for (int64_t a = 0; a < nact; ++a) {
             int64_t id = act[a];
-            int32_t u;
-            if (oracle_bound(&pred[id], 1, q, &u) != ORACLE_OK)
+            int32_t u = H;
+            if ((!defer || arrival_ms[id] + pred_delay[id] <= s) &&
+                oracle_bound(&pred[id], 1, q, &u) != ORACLE_OK)
                 status = ORACLE_E_RANGE;
             U[id] = u;
         }
-        if (oracle_bound(&pred[lo], hi - lo, q, cU) != ORACLE_OK)
-            status = ORACLE_E_RANGE;
+        for (int64_t c = 0; c < nc; ++c) {
+            cp[c] = prompt[cid[c]];
+            if (oracle_bound(&pred[cid[c]], 1, q, &cU[c]) != ORACLE_OK)
+                status = ORACLE_E_RANGE;
+        }
 
-        /* 5. Dispatch the batch. */
+        /* 5. Dispatch the candidates. */
         if (!rr && cfg->dispatch == 3) {
             /* least requests: the decoder with the fewest requests in the
-             * system, the batch counted as it is dispatched */
-            for (int64_t i = lo; i < hi; ++i) {
+             * system, the candidates counted as they are dispatched */
+            for (int64_t c = 0; c < nc; ++c) {
                 int32_t best = 0;
                 for (int32_t k = 1; k < D; ++k)
                     if (nreq[k] < nreq[best])
                         best = k;
-                choice_out[i] = best;
+                cch[c] = best;
                 nreq[best] += 1;
             }
         } else if (!rr && cfg->dispatch != 2) {
@@ -633,23 +809,26 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
             if (os != ORACLE_OK)
                 status = os;
             int ds = dispatch_horizon(1, cfg->dispatch == 1, D, H, K, capv, Q,
-                                      hi - lo, &prompt[lo], cU, &choice_out[lo], hr);
+                                      nc, cp, cU, cch, hr);
             if (ds != ORACLE_OK)
                 status = ds;
         } else {
-            for (int64_t i = lo; i < hi; ++i)
-                choice_out[i] = (int32_t)(i % D);
+            for (int64_t c = 0; c < nc; ++c)
+                cch[c] = (int32_t)(cid[c] % D);
         }
 
-        /* 6. The batch joins the chosen decoders' waiting queues. */
-        for (int64_t i = lo; i < hi; ++i) {
+        /* 6. The candidates join the chosen decoders' waiting queues. */
+        for (int64_t c = 0; c < nc; ++c) {
+            int64_t i = cid[c];
+            choice_out[i] = cch[c];
             st[i] = ST_WAITING;
-            dec[i] = choice_out[i];
+            dec[i] = cch[c];
             disp[i] = s;
             g[i] = 0;
-            U[i] = cU[i - lo];
+            U[i] = cU[c];
             act[nact++] = i;
         }
+        (void)nto;
 
         /* 7. Local order of every waiting queue. */
         int64_t nw = 0;
@@ -677,9 +856,10 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
          *    request's bounded demand fits, Eq. (admission) with the
          *    calibrated bound standing in for the unknown output length;
          *    the first misfit blocks the rest of its queue. */
-        int64_t admitted = 0;
+        int64_t admitted8 = 0;
         for (int32_t k = 0; k < D; ++k) {
-            for (int64_t x = seg[k]; x < seg[k + 1]; ++x) {
+            int64_t x = seg[k];
+            for (; x < seg[k + 1]; ++x) {
                 int64_t id = wid[wperm[x]];
                 int64_t demand = (int64_t)prompt[id] + U[id];
                 if (used[k] + demand > capv[k])
@@ -687,34 +867,44 @@ int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                 st[id] = ST_RUNNING;
                 g[id] = 0;
                 res_u[id] = U[id];
-                used[k] += cfg->accounting == 0 ? (int64_t)prompt[id]
-                         : cfg->accounting == 1 ? demand
-                                                : (int64_t)prompt[id] + demand;
-                ++admitted;
-                dst[3 * k + 2] += 1;
+                used[k] += admit_tokens(cfg->accounting, prompt[id], U[id]);
+                ++admitted8;
+                dst[4 * k + 2] += 1;
+                if (cfg->per_step)
+                    run_append(&L, k, id);
             }
-            /* the waiting queue holds until the next batch's dispatch step */
-            int64_t adm_k = 0;
-            for (int64_t x = seg[k]; x < seg[k + 1]; ++x)
-                adm_k += st[wid[wperm[x]]] == ST_RUNNING;
-            int64_t s_next = b + 1 < nb ? arrival_ms[((b + 2) * Bsz < N ? (b + 2) * Bsz : N) - 1] : s;
-            dst[3 * k] += (seg[k + 1] - seg[k] - adm_k) * (s_next - s);
+            int64_t left = seg[k + 1] - x;
+            if (cfg->per_step) {
+                /* the rest of the queue, in this order, until the next
+                 * dispatch step; preempted requests have all been ordered */
+                L.qhead[k] = x;
+                L.qend[k] = seg[k + 1];
+                L.ptop[k] = -1;
+                if (b + 1 < nb)
+                    dst[4 * k] += left; /* waiting through step s */
+            } else {
+                /* the waiting queue holds until the next batch's dispatch step */
+                int64_t s_next = b + 1 < nb ? arrival_ms[((b + 2) * Bsz < N ? (b + 2) * Bsz : N) - 1] : s;
+                dst[4 * k] += left * (s_next - s);
+            }
         }
         stats_out[4 * b + 0] = ndone;
-        stats_out[4 * b + 1] = admitted;
-        stats_out[4 * b + 2] = nw - admitted;
+        stats_out[4 * b + 1] = admitted + admitted8;
+        stats_out[4 * b + 2] = nw - admitted8;
         stats_out[4 * b + 3] = overflow;
         prev_s = s;
     }
     if (dec_stats_out != NULL)
-        for (int64_t i = 0; i < (int64_t)D * 3; ++i)
+        for (int64_t i = 0; i < (int64_t)D * 4; ++i)
             dec_stats_out[i] = dst[i];
 
 out:
     free(st); free(g); free(dec); free(U); free(disp); free(act); free(done);
     free(win_true); free(win_pred); free(K); free(capv); free(Q); free(off);
     free(used); free(seg); free(rp); free(rg); free(rU); free(wid); free(wdec);
-    free(wU); free(wwait); free(warr); free(wperm); free(cU); free(hr);
-    free(res_u); free(occ); free(nreq); free(dst);
+    free(wU); free(wwait); free(warr); free(wperm); free(cid); free(cp); free(cU);
+    free(cch); free(hr); free(pend); free(res_u); free(occ); free(nreq); free(dst);
+    free(L.next); free(L.prev); free(L.pnext); free(L.head); free(L.tail);
+    free(L.ptop); free(L.qhead); free(L.qend);
     return status;
 }

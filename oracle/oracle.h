@@ -87,17 +87,24 @@ typedef struct {
     int32_t accounting; /* admission counts running requests at 0 their tokens,
                            1 prompt + reserved output (staged release),
                            2 reserved prompt + prompt + reserved output */
+    int32_t per_step;   /* 0 admission at dispatch steps only; 1 every step,
+                           with preemption of the latest admitted request */
+    int32_t beta;       /* timeout (steps) for a bound not yet available;
+                           < 0: every bound is available at dispatch */
 } oracle_stream_cfg;
 
-/* Outputs: choice[N]; per batch b: q[b] (-1 if unbounded -> round robin),
+/* pred_delay[N] (may be NULL: 0): steps from arrival until the request's
+ * prediction, and so its bound, is available (used when beta >= 0).
+ * Outputs: choice[N]; per batch b: q[b] (-1 if unbounded -> round robin),
  * stats[4b..4b+3] = completed, admitted, waiting after admission,
  * decoders over capacity after advancing; per decoder k (dec_stats may be
- * NULL): dec_stats[3k..3k+2] = waiting requests x steps summed over the
+ * NULL): dec_stats[4k..4k+3] = waiting requests x steps summed over the
  * batches (the time-weighted queue length times the span), batches in which
- * it was over capacity after advancing, admissions. */
+ * it was over capacity after advancing, admissions, preemptions. */
 int oracle_stream(const oracle_stream_cfg *cfg, const int64_t *arrival_ms,
                   const int32_t *prompt, const int32_t *true_len,
-                  const int32_t *pred, int32_t *choice_out, int32_t *q_out,
+                  const int32_t *pred, const int32_t *pred_delay,
+                  int32_t *choice_out, int32_t *q_out,
                   int64_t *stats_out, int64_t *dec_stats_out);
 
 /* Round-robin KV-pressure simulation of App. A (oracle_rr.c). */
