@@ -729,7 +729,7 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
     stats = torch.empty((nb, 4), dtype=torch.int64, device=device)
     ws = M.Workspace(device=device)
 
-    ds = torch.empty((w["D"], 3), dtype=torch.int64, device=device)
+    ds = torch.empty((w["D"], 4), dtype=torch.int64, device=device)
 
     def run(n, pol=(0, 0, 0), cap=None):
         cfg = M.stream_cfg(n, w["D"], w["H"], w["cap"] if cap is None else cap, B, w["window"],

@@ -304,6 +304,30 @@ int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
  *                    Admission is always used + p + U <= cap; the over-
  *                    capacity count compares p + g with cap in every mode.
  *
+ * Fidelity modes (Sec. 3.3 memory-aware scheduler and App. D):
+ *   per_step = 1     between dispatch steps the loop runs step by step: on
+ *                    each step a decoder whose running requests would pass
+ *                    its capacity by taking one token each preempts its most
+ *                    recently admitted request (never its last one), which
+ *                    loses its tokens and goes to the head of the waiting
+ *                    queue; each running request takes a token and those
+ *                    reaching their true length complete; on every step
+ *                    but a dispatch step the queue (preempted requests
+ *                    first, the latest on top, then the order computed at
+ *                    the last dispatch step) admits while used + p + U <=
+ *                    cap, the first misfit blocking.
+ *   beta >= 0        deferral: a request is dispatched at the first dispatch
+ *                    step s at or after its arrival with arrival +
+ *                    pred_delay <= s (its bound is available), by the
+ *                    dispatch policy; one still without a bound beta steps
+ *                    after arrival (or at the last dispatch step) goes round
+ *                    robin (index mod D) with the horizon H as its bound
+ *                    until its prediction arrives; at a dispatch step the
+ *                    timed-out requests join their queues before the policy
+ *                    dispatches the rest, in index order.  Every request in
+ *                    the system whose prediction is not in yet is bounded
+ *                    by H.
+ *
  *   cfg                 host struct: N requests (1 .. INT32_MAX), D decoders
  *                       (1 .. 1024), horizon H steps, capacity cap tokens per
  *                       decoder, batch size, window size, alpha in parts per
@@ -318,11 +342,16 @@ int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
  *   stats_out           [ceil(N / batch)][4] int64 per batch: completions,
  *                       admissions, requests left waiting, decoders whose
  *                       running requests exceed capacity after advancing.
- *   dec_stats_out       [D][3] int64 per decoder, or NULL: the waiting-queue
- *                       integral (requests left waiting after batch b's
- *                       admission times s_{b+1} - s_b, the last batch
- *                       counting 0), the batches after whose advance its
- *                       running requests exceed capacity, its admissions.
+ *   pred_delay          [N] int32 steps from arrival until the request's
+ *                       prediction (so its bound) is available, >= 0; read
+ *                       only when cfg->beta >= 0 (then required).
+ *   dec_stats_out       [D][4] int64 per decoder, or NULL: the waiting-queue
+ *                       integral (requests waiting through each step from
+ *                       the first dispatch step to the last, exclusive:
+ *                       after batch b's admission times s_{b+1} - s_b when
+ *                       admission happens at dispatch steps only), the
+ *                       batches after whose advance its running requests
+ *                       exceed capacity, its admissions, its preemptions.
  * The call runs the whole loop: it synchronises the stream once per batch
  * (to read the request counts that size the next launches) and at the end,
  * and returns the full status.  A negative length or decreasing arrival is
@@ -339,6 +368,8 @@ typedef struct {
   int32_t dispatch_policy; /* MAPS_STREAM_MAPS / _MC / _RR / _LR */
   int32_t local_order;     /* MAPS_STREAM_SJF / _FCFS */
   int32_t accounting;      /* MAPS_STREAM_OCCUPANCY / _STAGED / _HELD */
+  int32_t per_step;        /* 0: admission at dispatch steps; 1: every step, with preemption */
+  int32_t beta;            /* < 0: bounds always available; >= 0: deferral timeout, steps */
 } maps_stream_cfg;
 
 #define MAPS_STREAM_MAPS 0
@@ -354,9 +385,10 @@ typedef struct {
 size_t maps_stream_workspace_size(const maps_stream_cfg *cfg);
 int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms,
                     const int32_t *prompt, const int32_t *true_len,
-                    const int32_t *pred, int32_t *choice_out, int32_t *q_out,
-                    int64_t *stats_out, int64_t *dec_stats_out, void *ws,
-                    size_t ws_bytes, void *stream);
+                    const int32_t *pred, const int32_t *pred_delay,
+                    int32_t *choice_out, int32_t *q_out, int64_t *stats_out,
+                    int64_t *dec_stats_out, void *ws, size_t ws_bytes,
+                    void *stream);
 
 /* ------------------------------------------------------------------------
  * Round-robin KV-pressure simulation and high-pressure interval metrics,

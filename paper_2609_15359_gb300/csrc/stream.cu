@@ -43,6 +43,10 @@ struct StreamState {
   int32_t nact;      // requests in the system (waiting or running)
   int32_t ndone;     // completions found by the last advance
   int32_t nwait;     // waiting requests after the last advance
+  int32_t npend;     // deferral: arrived requests not yet dispatched
+  int32_t nc;        // deferral: requests for the dispatch policy at this step
+  int32_t nto;       // deferral: requests timed out to round robin at this step
+  int32_t adm_i;     // per-step mode: admissions between the dispatch steps
   int32_t pad;
 };
 
@@ -67,12 +71,13 @@ __device__ __forceinline__ int block_flag_scan(bool f, int *s_w, int &total) {
 
 __global__ void stream_validate_kernel(int64_t N, const int64_t *arrival, const int32_t *prompt,
                                        const int32_t *true_len, const int32_t *pred,
-                                       int32_t *status) {
+                                       const int32_t *pred_delay, int32_t *status) {
   pdl_prologue();
   bool bad = false;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < N; i += stride)
-    if (prompt[i] < 0 || true_len[i] < 1 || pred[i] < 0 || (i > 0 && arrival[i] < arrival[i - 1]))
+    if (prompt[i] < 0 || true_len[i] < 1 || pred[i] < 0 || (i > 0 && arrival[i] < arrival[i - 1]) ||
+        (pred_delay != nullptr && pred_delay[i] < 0))
       bad = true;
   if (bad) flag_error(status, MAPS_E_RANGE);
 }
@@ -86,6 +91,10 @@ __global__ void stream_init_kernel(int64_t first_hi, int D, int32_t cap, const i
     S->nact = 0;
     S->ndone = 0;
     S->nwait = 0;
+    S->npend = 0;
+    S->nc = 0;
+    S->nto = 0;
+    S->adm_i = 0;
   }
 }
 
@@ -94,7 +103,7 @@ __global__ void stream_init_kernel(int64_t first_hi, int D, int32_t cap, const i
 //    used = what admission counts for them: p + g, p + max(U*, g) (staged)
 //    or 2p + max(U*, g) (held), U* the bound reserved at admission.
 __global__ void __launch_bounds__(kSt, 1)
-stream_advance_kernel(int64_t hi, int D, int32_t cap, int acct, const int64_t *arrival,
+stream_advance_kernel(int64_t hi, int D, int32_t cap, int acct, int per_step, const int64_t *arrival,
                       const int32_t *prompt, const int32_t *true_len, const int32_t *res_u,
                       uint8_t *st, int32_t *g, const int32_t *dec, const int32_t *act_in,
                       int32_t *act_out, int32_t *done_id, int32_t *done_rem, long long *used,
@@ -107,17 +116,19 @@ stream_advance_kernel(int64_t hi, int D, int32_t cap, int acct, const int64_t *a
   for (int k = tid; k < D; k += kSt) s_occ[k] = s_used[k] = 0;
   if (tid == 0) s_nwait = 0;
   const long long s = arrival[hi - 1];
-  const long long delta = s - S->prev_s;
+  const long long delta = s - S->prev_s;  // 0 after the per-step interval
   const int nact = S->nact;
+  // per-step mode: the interval kernel's completions come first
+  int nkeep = 0, ndone = per_step ? S->ndone : 0, nwait = 0;
   __syncthreads();
-  int nkeep = 0, ndone = 0, nwait = 0;
   for (int c0 = 0; c0 < nact; c0 += kSt) {
     const int x = c0 + tid;
     int id = -1, rem32 = 0;
-    bool done = false;
+    bool done = false, gone = false;
     if (x < nact) {
       id = act_in[x];
       const uint8_t sv = st[id];
+      gone = sv == kDone;  // completed in the per-step interval
       if (sv == kRunning) {
         const long long rem = static_cast<long long>(true_len[id]) - g[id];  // >= 1
         if (rem <= delta) {
@@ -140,9 +151,9 @@ stream_advance_kernel(int64_t hi, int D, int32_t cap, int acct, const int64_t *a
       }
     }
     int tk, td;
-    const int pk = block_flag_scan(id >= 0 && !done, s_w, tk);
+    const int pk = block_flag_scan(id >= 0 && !done && !gone, s_w, tk);
     const int pd = block_flag_scan(done, s_w, td);
-    if (id >= 0 && !done) act_out[nkeep + pk] = id;
+    if (id >= 0 && !done && !gone) act_out[nkeep + pk] = id;
     if (done) {
       done_id[ndone + pd] = id;
       done_rem[ndone + pd] = rem32;
@@ -154,7 +165,7 @@ stream_advance_kernel(int64_t hi, int D, int32_t cap, int acct, const int64_t *a
   const bool ov = tid < D && static_cast<long long>(s_occ[tid]) > cap;  // D <= kSt
   if (tid < D) {
     used[tid] = static_cast<long long>(acct == MAPS_STREAM_OCCUPANCY ? s_occ[tid] : s_used[tid]);
-    if (dst != nullptr && ov) dst[3 * tid + 1] += 1;
+    if (dst != nullptr && ov) dst[4 * tid + 1] += 1;
   }
   const int over = __syncthreads_count(ov);
   if (tid == 0) {
@@ -164,6 +175,268 @@ stream_advance_kernel(int64_t hi, int D, int32_t cap, int acct, const int64_t *a
     S->nwait = s_nwait;
     stats_b[0] = ndone;
     stats_b[3] = over;
+  }
+}
+
+// 1'. Per-step mode: the steps prev_s + 1 .. s, one warp per decoder
+//     (decoders do not interact between dispatch steps).  Each decoder holds
+//     its running requests (in rbuf, unordered; the admission order is aseq)
+//     and the requests it preempted since the last dispatch step (sbuf, a
+//     stack, the latest on top); its waiting queue is the order computed at
+//     the last dispatch step past the requests admitted then.  A step: while
+//     the running requests would pass the capacity by taking one token each,
+//     the most recently admitted one (never the last) is preempted, losing
+//     its tokens; each takes a token, and those reaching their true length
+//     complete; then, except on the dispatch step s, the stack top or the
+//     queue head is admitted while used + p + U <= capacity.  Between events
+//     nothing but the growth happens: no admission can succeed (used only
+//     grows and nothing is freed since the head last failed), so the warp
+//     jumps to the next step with a completion or a preemption, or to s.
+//     Every iteration advances the step, so the loop ends.
+__global__ void __launch_bounds__(kSt, 1)
+stream_interval_kernel(int64_t hi, int D, int32_t cap, int acct, const int64_t *arrival,
+                       const int32_t *prompt, const int32_t *true_len, const int32_t *U,
+                       int32_t *res_u, uint8_t *st, int32_t *g, const int32_t *dec,
+                       const int32_t *act, const int32_t *wid, const int32_t *wperm,
+                       const int64_t *wseg, const int64_t *qhead, long long *aseq,
+                       long long *dseq, int32_t *rbuf, int32_t *sbuf, int32_t *done_id,
+                       int32_t *done_rem, StreamState *S, int64_t *dst) {
+  pdl_prologue();
+  __shared__ int s_cnt[kStreamMaxD], s_run[kStreamMaxD], s_cur[kStreamMaxD];
+  __shared__ int s_w[kStWarps];
+  __shared__ int s_done, s_adm;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const long long s = arrival[hi - 1];
+  const long long s0 = S->prev_s;
+  const int nact = S->nact;
+  for (int k = tid; k < D; k += kSt) s_cnt[k] = s_run[k] = 0;
+  if (tid == 0) s_done = s_adm = 0;
+  __syncthreads();
+  // each decoder's region: room for all its requests in the system
+  for (int x = tid; x < nact; x += kSt) {
+    const int id = act[x];
+    atomicAdd(&s_cnt[dec[id]], 1);
+    if (st[id] == kRunning) atomicAdd(&s_run[dec[id]], 1);
+  }
+  __syncthreads();
+  {
+    const int c = tid < D ? s_cnt[tid] : 0;  // D <= kSt
+    int incl = c;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_w[warp] = incl;
+    __syncthreads();
+    int base = 0;
+    for (int w = 0; w < warp; ++w) base += s_w[w];
+    if (tid < D) {
+      s_cnt[tid] = base + incl - c;  // now the region's start
+      s_cur[tid] = 0;
+    }
+  }
+  __syncthreads();
+  for (int x = tid; x < nact; x += kSt) {
+    const int id = act[x];
+    if (st[id] == kRunning) {
+      const int k = dec[id];
+      rbuf[s_cnt[k] + atomicAdd(&s_cur[k], 1)] = id;
+    }
+  }
+  __syncthreads();
+  for (int k = warp; k < D; k += kStWarps) {
+    const int base = s_cnt[k];
+    int n = s_run[k], ns = 0;
+    long long qh = qhead[k];
+    const long long qe = wseg[k + 1];
+    long long seq = dseq[k], integ = 0;
+    int npre = 0, nadm = 0;
+    long long t = s0;
+    while (t < s) {
+      long long tok = 0;
+      int jc = INT_MAX;
+      for (int i = lane; i < n; i += 32) {
+        const int id = rbuf[base + i];
+        const int gi = g[id];
+        tok += static_cast<long long>(prompt[id]) + gi;
+        jc = min(jc, true_len[id] - gi);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        tok += __shfl_xor_sync(0xffffffffu, tok, off);
+        jc = min(jc, __shfl_xor_sync(0xffffffffu, jc, off));
+      }
+      // steps to the next completion (jc) and to the next preemption (jp)
+      long long je = LLONG_MAX;
+      if (n > 0) {
+        je = jc;
+        if (n > 1) je = min(je, tok + n > cap ? 1LL : (cap - tok) / n + 1);
+      }
+      const long long te = je >= s - t ? s : t + je;
+      const long long quiet = te - t - 1;  // steps of growth alone
+      if (quiet > 0) {
+        for (int i = lane; i < n; i += 32) g[rbuf[base + i]] += static_cast<int>(quiet);
+        integ += (static_cast<long long>(ns) + (qe - qh)) * quiet;
+        tok += static_cast<long long>(n) * quiet;
+      }
+      t = te;
+      __syncwarp();
+      // step t: preempt the latest admitted while the next tokens do not fit
+      while (n > 1 && tok + n > cap) {
+        long long best = -1;
+        int bi = 0;
+        for (int i = lane; i < n; i += 32) {
+          const long long a = aseq[rbuf[base + i]];
+          if (a > best) {
+            best = a;
+            bi = i;
+          }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          const long long ob = __shfl_xor_sync(0xffffffffu, best, off);
+          const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+          if (ob > best) {
+            best = ob;
+            bi = oi;
+          }
+        }
+        const int v = rbuf[base + bi];
+        tok -= static_cast<long long>(prompt[v]) + g[v];
+        __syncwarp();
+        if (lane == 0) {
+          rbuf[base + bi] = rbuf[base + n - 1];
+          sbuf[base + ns] = v;
+          st[v] = kWaiting;
+          g[v] = 0;
+        }
+        --n;
+        ++ns;
+        ++npre;
+        __syncwarp();
+      }
+      // one token each; completions leave the running set (in-place compaction)
+      int kept = 0;
+      for (int r0 = 0; r0 < n; r0 += 32) {
+        const int i = r0 + lane;
+        const int id = i < n ? rbuf[base + i] : -1;
+        bool fin = false;
+        if (id >= 0) {
+          const int gi = g[id] + 1;
+          g[id] = gi;
+          fin = gi == true_len[id];
+          if (fin) {
+            st[id] = kDone;
+            const int o = atomicAdd(&s_done, 1);
+            done_id[o] = id;
+            done_rem[o] = static_cast<int>(t - s0);
+          }
+        }
+        const unsigned km = __ballot_sync(0xffffffffu, id >= 0 && !fin);
+        if (id >= 0 && !fin) rbuf[base + kept + __popc(km & ((1u << lane) - 1u))] = id;
+        kept += __popc(km);
+        __syncwarp();
+      }
+      n = kept;
+      if (t == s) break;
+      // admission in queue order (the stack first)
+      long long used = 0;
+      for (int i = lane; i < n; i += 32) {
+        const int id = rbuf[base + i];
+        const long long p = prompt[id], gi = g[id];
+        const long long out = max(static_cast<long long>(res_u[id]), gi);
+        used += acct == MAPS_STREAM_OCCUPANCY ? p + gi
+                : acct == MAPS_STREAM_STAGED  ? p + out
+                                              : 2 * p + out;
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) used += __shfl_xor_sync(0xffffffffu, used, off);
+      if (lane == 0) {
+        for (;;) {
+          const bool from_stack = ns > 0;
+          if (!from_stack && qh >= qe) break;
+          const int c = from_stack ? sbuf[base + ns - 1] : wid[wperm[qh]];
+          const long long p = prompt[c], uu = U[c];
+          if (used + p + uu > cap) break;
+          if (from_stack)
+            --ns;
+          else
+            ++qh;
+          rbuf[base + n] = c;
+          ++n;
+          st[c] = kRunning;
+          g[c] = 0;
+          res_u[c] = static_cast<int32_t>(uu);
+          aseq[c] = seq++;
+          used += acct == MAPS_STREAM_OCCUPANCY ? p : acct == MAPS_STREAM_STAGED ? p + uu : 2 * p + uu;
+          ++nadm;
+        }
+      }
+      n = __shfl_sync(0xffffffffu, n, 0);
+      ns = __shfl_sync(0xffffffffu, ns, 0);
+      qh = __shfl_sync(0xffffffffu, qh, 0);
+      seq = __shfl_sync(0xffffffffu, seq, 0);
+      __syncwarp();
+      integ += static_cast<long long>(ns) + (qe - qh);  // waiting through step t
+    }
+    if (lane == 0) {
+      dseq[k] = seq;
+      if (dst != nullptr) {
+        dst[4 * k] += integ;
+        dst[4 * k + 2] += nadm;
+        dst[4 * k + 3] += npre;
+      }
+      if (nadm) atomicAdd(&s_adm, nadm);
+    }
+  }
+  __syncthreads();
+  if (tid == 0) {
+    S->ndone = s_done;
+    S->adm_i = s_adm;
+    S->prev_s = s;  // the advance that follows moves nobody
+  }
+}
+
+// Deferral: the requests arrived but not dispatched, then the batch, in index
+// order, split three ways (stable): a bound available by s (the arrival plus
+// the prediction delay) -> the dispatch policy; waited beta steps past
+// arrival without one, or the last dispatch step -> round robin; otherwise
+// they keep waiting for the next dispatch step.
+__global__ void __launch_bounds__(kSt, 1)
+stream_select_kernel(int64_t lo, int nb, int64_t hi, int32_t beta, int last, const int64_t *arrival,
+                     const int32_t *pred_delay, const int32_t *pend_in, int32_t *pend_out,
+                     int32_t *cid, int32_t *tout, StreamState *S) {
+  pdl_prologue();
+  __shared__ int s_w[kStWarps];
+  const long long s = arrival[hi - 1];
+  const int np = S->npend, n = np + nb;
+  int nc = 0, nt = 0, nk = 0;
+  for (int c0 = 0; c0 < n; c0 += kSt) {
+    const int x = c0 + static_cast<int>(threadIdx.x);
+    int id = -1;
+    bool av = false, to = false, kp = false;
+    if (x < n) {
+      id = x < np ? pend_in[x] : static_cast<int>(lo + (x - np));
+      av = arrival[id] + pred_delay[id] <= s;
+      to = !av && (arrival[id] + beta <= s || last);
+      kp = !av && !to;
+    }
+    int tc, tt, tk;
+    const int pc = block_flag_scan(av, s_w, tc);
+    const int pt = block_flag_scan(to, s_w, tt);
+    const int pk = block_flag_scan(kp, s_w, tk);
+    if (av) cid[nc + pc] = id;
+    if (to) tout[nt + pt] = id;
+    if (kp) pend_out[nk + pk] = id;
+    nc += tc;
+    nt += tt;
+    nk += tk;
+  }
+  if (threadIdx.x == 0) {
+    S->nc = nc;
+    S->nto = nt;
+    S->npend = nk;
   }
 }
 
@@ -183,24 +456,34 @@ __global__ void stream_window_kernel(int ndone, long long c0, int Wn, const int3
   }
 }
 
-// 3. Predictions of the requests in the system, then of the batch.
+// 3. Predictions of the requests in the system, then of the candidates
+//    (the batch lo.., or the listed ids, whose prompts are gathered too).
 __global__ void stream_gather_kernel(int nact, int nb, int64_t lo, const int32_t *act,
-                                     const int32_t *pred, int32_t *qpred) {
+                                     const int32_t *cid, const int32_t *pred,
+                                     const int32_t *prompt, int32_t *qpred, int32_t *cp) {
   pdl_prologue();
   const int stride = gridDim.x * blockDim.x;
-  for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < nact + nb; x += stride)
-    qpred[x] = x < nact ? pred[act[x]] : pred[lo + (x - nact)];
+  for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < nact + nb; x += stride) {
+    if (x < nact) {
+      qpred[x] = pred[act[x]];
+    } else {
+      const int id = cid ? cid[x - nact] : static_cast<int>(lo + (x - nact));
+      qpred[x] = pred[id];
+      if (cid) cp[x - nact] = prompt[id];
+    }
+  }
 }
 
 // 3'. No bound available: U = prediction, the batch goes round robin.  With
 //     set_u = 0 only the choices (the round-robin dispatch policy).
+//     choice[x] is candidate x's: lo + x, or the listed cid[x].
 __global__ void stream_rr_kernel(int n, int nb, int64_t lo, int D, int set_u, const int32_t *qpred,
-                                 int32_t *Uq, int32_t *choice) {
+                                 int32_t *Uq, const int32_t *cid, int32_t *choice) {
   pdl_prologue();
   const int stride = gridDim.x * blockDim.x;
   for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
     if (set_u) Uq[x] = qpred[x];
-    if (x < nb) choice[lo + x] = static_cast<int32_t>((lo + x) % D);
+    if (x < nb) choice[x] = static_cast<int32_t>((cid ? static_cast<int64_t>(cid[x]) : lo + x) % D);
   }
 }
 
@@ -235,11 +518,22 @@ __global__ void stream_lr_kernel(int D, int nb, const int64_t *res_off, int32_t 
 // 4. Residents by decoder (running with g, waiting with g = 0) and the
 //    waiting count per decoder; new bounds of the requests in the system.
 __global__ void __launch_bounds__(kSt, 1)
+//    Under deferral a request whose prediction is not in by s (arrival +
+//    delay > s) is bounded by the horizon H.
 stream_csr_kernel(int nact, int D, int rr, const int32_t *q_dev, int32_t *q_out_b,
                   const int32_t *act, const uint8_t *st, const int32_t *g, const int32_t *dec,
-                  const int32_t *prompt, const int32_t *Uq, int32_t *U, int64_t *res_off,
-                  int32_t *rp, int32_t *rg, int32_t *rU, int32_t *Q) {
+                  const int32_t *prompt, int32_t *Uq, int32_t *U, int64_t *res_off,
+                  int32_t *rp, int32_t *rg, int32_t *rU, int32_t *Q, const int64_t *arrival,
+                  const int32_t *pred_delay, int64_t hi, int32_t H) {
   pdl_prologue();
+  if (pred_delay != nullptr) {  // before anything reads Uq
+    const long long s = arrival[hi - 1];
+    for (int x = threadIdx.x; x < nact; x += kSt) {
+      const int id = act[x];
+      if (arrival[id] + pred_delay[id] > s) Uq[x] = H;
+    }
+    __syncthreads();
+  }
   __shared__ int s_cnt[kStreamMaxD], s_q[kStreamMaxD], s_cur[kStreamMaxD];
   __shared__ int s_w[kStWarps];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -784,6 +1078,36 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
   for (int k = tid; k < D; k += kSt) Q[k] = s_q[k];
 }
 
+// 5''. Deferral: the listed requests join the waiting queues at act[nact..]:
+//      with choices cch (and bounds Uq[nact + i]), or, with cch null, round
+//      robin with the horizon as their bound (timed out without one).
+__global__ void stream_enqueue_list_kernel(int n, int nact, int D, int32_t H, int64_t hi,
+                                           const int64_t *arrival, const int32_t *ids,
+                                           const int32_t *cch, const int32_t *Uq,
+                                           int32_t *choice_out, uint8_t *st, int32_t *dec,
+                                           long long *disp, int32_t *g, int32_t *U, int32_t *act,
+                                           StreamState *S, int32_t *status) {
+  pdl_prologue();
+  const long long s = arrival[hi - 1];
+  const int stride = gridDim.x * blockDim.x;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const int id = ids[i];
+    int c = cch ? cch[i] : id % D;
+    if (c < 0 || c >= D) {  // only after a range error (a bound that overflowed)
+      flag_error(status, MAPS_E_RANGE);
+      c = 0;
+    }
+    choice_out[id] = c;
+    st[id] = kWaiting;
+    dec[id] = c;
+    disp[id] = s;
+    g[id] = 0;
+    U[id] = cch ? Uq[nact + i] : H;
+    act[nact + i] = id;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) S->nact = nact + n;
+}
+
 // 6. The batch joins the waiting queues of its decoders.
 __global__ void stream_enqueue_kernel(int64_t lo, int nb, int nact, int64_t hi, int D,
                                       const int64_t *arrival, const int32_t *choice,
@@ -845,15 +1169,19 @@ stream_waitlist_kernel(int n, int64_t hi, const int64_t *arrival, const int32_t 
 //    (staged) or 2p + U (held).  Each decoder's statistics gain its queue
 //    left waiting times the steps to the next batch, and its admissions.
 __global__ void __launch_bounds__(kSt, 1)
-stream_admit_kernel(int D, int32_t cap, int acct, int nw, int64_t hi, int64_t hi_next,
+//    Per-step mode: each admission's sequence number (aseq), the queue's
+//    first entry left (qhead), and the waiting requests count for the
+//    dispatch step alone (the steps after it are the next interval's).
+stream_admit_kernel(int D, int32_t cap, int acct, int per_step, int nw, int64_t hi, int64_t hi_next,
                     const int64_t *arrival, const int64_t *wseg, const int32_t *wperm,
                     const int32_t *wid, const int32_t *prompt, const int32_t *U,
                     const long long *used, uint8_t *st, int32_t *g, int32_t *res_u,
+                    long long *aseq, long long *dseq, int64_t *qhead, const StreamState *S,
                     int64_t *stats_b, int64_t *dst) {
   pdl_prologue();
   __shared__ int s_adm;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const long long span = arrival[hi_next - 1] - arrival[hi - 1];
+  const long long span = per_step ? (hi_next != hi ? 1 : 0) : arrival[hi_next - 1] - arrival[hi - 1];
   if (tid == 0) s_adm = 0;
   __syncthreads();
   for (int k = warp; k < D; k += kStWarps) {
@@ -883,20 +1211,27 @@ stream_admit_kernel(int D, int32_t cap, int acct, int nw, int64_t hi, int64_t hi
         st[id] = kRunning;
         g[id] = 0;
         res_u[id] = static_cast<int32_t>(uu);
+        if (per_step) aseq[id] = dseq[k] + adm + lane;
       }
       if (nadm > 0) u += __shfl_sync(0xffffffffu, incl, nadm - 1);
       adm += nadm;
       stop = fail != 0;
     }
     if (lane == 0 && adm) atomicAdd(&s_adm, adm);
-    if (lane == 0 && dst != nullptr) {  // decoder k is this warp's alone
-      dst[3 * k] += (x1 - wseg[k] - adm) * span;
-      dst[3 * k + 2] += adm;
+    if (lane == 0) {  // decoder k is this warp's alone
+      if (per_step) {
+        dseq[k] += adm;
+        qhead[k] = wseg[k] + adm;
+      }
+      if (dst != nullptr) {
+        dst[4 * k] += (x1 - wseg[k] - adm) * span;
+        dst[4 * k + 2] += adm;
+      }
     }
   }
   __syncthreads();
   if (tid == 0) {
-    stats_b[1] = s_adm;
+    stats_b[1] = s_adm + (per_step ? S->adm_i : 0);
     stats_b[2] = nw - s_adm;
   }
 }
@@ -919,6 +1254,12 @@ struct StreamWs {
   int32_t *wid, *wdec, *wU, *wwait, *warr, *wperm;
   int64_t *wseg;
   int32_t *q_dev;
+  // deferral
+  int32_t *pend[2], *cid, *tout, *cp, *cch;
+  // per-step mode
+  long long *aseq, *dseq;
+  int32_t *rbuf, *sbuf;
+  int64_t *qhead;
 };
 
 size_t stream_sub_bytes(const maps_stream_cfg &c) {
@@ -970,6 +1311,19 @@ StreamWs carve_stream(Carve &c, const maps_stream_cfg &cfg) {
   w.wperm = c.take<int32_t>(N);
   w.wseg = c.take<int64_t>(D + 1);
   w.q_dev = c.take<int32_t>(1);
+  const bool defer = cfg.beta >= 0;
+  w.pend[0] = c.take<int32_t>(defer ? N : 0);
+  w.pend[1] = c.take<int32_t>(defer ? N : 0);
+  w.cid = c.take<int32_t>(defer ? N : 0);
+  w.tout = c.take<int32_t>(defer ? N : 0);
+  w.cp = c.take<int32_t>(defer ? N : 0);
+  w.cch = c.take<int32_t>(defer ? N : 0);
+  const bool ps = cfg.per_step != 0;
+  w.aseq = c.take<long long>(ps ? N : 0);
+  w.dseq = c.take<long long>(ps ? D : 0);
+  w.rbuf = c.take<int32_t>(ps ? N : 0);
+  w.sbuf = c.take<int32_t>(ps ? N : 0);
+  w.qhead = c.take<int64_t>(ps ? D : 0);
   return w;
 }
 
@@ -979,7 +1333,7 @@ bool cfg_ok(const maps_stream_cfg *c) {
          c->alpha_ppm > 0 && c->alpha_ppm < 1000000u && c->dispatch_policy >= MAPS_STREAM_MAPS &&
          c->dispatch_policy <= MAPS_STREAM_LR && c->local_order >= MAPS_STREAM_SJF &&
          c->local_order <= MAPS_STREAM_FCFS && c->accounting >= MAPS_STREAM_OCCUPANCY &&
-         c->accounting <= MAPS_STREAM_HELD;
+         c->accounting <= MAPS_STREAM_HELD && (c->per_step == 0 || c->per_step == 1);
 }
 
 int grid_for(int64_t n, int threads = 256) {
@@ -1001,12 +1355,13 @@ size_t maps_stream_workspace_size(const maps_stream_cfg *cfg) {
 }
 
 int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const int32_t *prompt,
-                    const int32_t *true_len, const int32_t *pred, int32_t *choice_out,
-                    int32_t *q_out, int64_t *stats_out, int64_t *dec_stats_out, void *ws,
-                    size_t ws_bytes, void *stream) {
+                    const int32_t *true_len, const int32_t *pred, const int32_t *pred_delay,
+                    int32_t *choice_out, int32_t *q_out, int64_t *stats_out,
+                    int64_t *dec_stats_out, void *ws, size_t ws_bytes, void *stream) {
   using namespace maps;
   if (!cfg_ok(cfg) || arrival_ms == nullptr || prompt == nullptr || true_len == nullptr ||
-      pred == nullptr || choice_out == nullptr || q_out == nullptr || stats_out == nullptr)
+      pred == nullptr || choice_out == nullptr || q_out == nullptr || stats_out == nullptr ||
+      (cfg->beta >= 0 && pred_delay == nullptr))
     return MAPS_E_INVALID;
   MAPS_TRY(check_ws(ws, ws_bytes, maps_stream_workspace_size(cfg)));
   const maps_stream_cfg c = *cfg;
@@ -1016,13 +1371,22 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
   const StreamWs w = carve_stream(cv, c);
   const int64_t N = c.N, B = c.batch, nbatch = (N + B - 1) / B;
   const int D = c.D;
+  const bool defer = c.beta >= 0;
+  const int per_step = c.per_step;
+  const int32_t *pdl = defer ? pred_delay : nullptr;
 
   MAPS_TRY(cuda_ok(cudaMemsetAsync(w.st, 0, static_cast<size_t>(N), s)));
   MAPS_TRY(cuda_ok(cudaMemsetAsync(w.zeros, 0, static_cast<size_t>(N) * sizeof(int32_t), s)));
   if (dec_stats_out != nullptr)
-    MAPS_TRY(cuda_ok(cudaMemsetAsync(dec_stats_out, 0, static_cast<size_t>(c.D) * 3 * sizeof(int64_t), s)));
+    MAPS_TRY(cuda_ok(cudaMemsetAsync(dec_stats_out, 0, static_cast<size_t>(c.D) * 4 * sizeof(int64_t), s)));
+  if (per_step) {
+    MAPS_TRY(cuda_ok(cudaMemsetAsync(w.dseq, 0, static_cast<size_t>(D) * sizeof(long long), s)));
+    MAPS_TRY(cuda_ok(cudaMemsetAsync(w.qhead, 0, static_cast<size_t>(D) * sizeof(int64_t), s)));
+    MAPS_TRY(cuda_ok(cudaMemsetAsync(w.wseg, 0, static_cast<size_t>(D + 1) * sizeof(int64_t), s)));
+  }
   launch_pdl(stream_init_kernel, 1, kSt, 0, s, std::min(N, B), D, c.cap, arrival_ms, w.capv, w.S);
-  launch_pdl(stream_validate_kernel, grid_for(N), 256, 0, s, N, arrival_ms, prompt, true_len, pred, status);
+  launch_pdl(stream_validate_kernel, grid_for(N), 256, 0, s, N, arrival_ms, prompt, true_len, pred,
+             pdl, status);
   MAPS_TRY(launch_ok());
   {
     const int st0 = maps_check(ws, stream);  // a bad input stops the loop before it starts
@@ -1036,13 +1400,26 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
     const int nb = static_cast<int>(hi - lo);
     int32_t *act_in = w.act[b & 1], *act = w.act[(b & 1) ^ 1];
     int64_t *stats_b = stats_out + 4 * b;
-    launch_pdl(stream_advance_kernel, 1, kSt, 0, s, hi, D, c.cap, c.accounting, arrival_ms, prompt,
-               true_len, w.res_u, w.st, w.g, w.dec, act_in, act, w.done_id, w.done_rem, w.used, w.S,
-               stats_b, dec_stats_out);
+    if (defer)  // 4 (first half): who is dispatched at this step
+      launch_pdl(stream_select_kernel, 1, kSt, 0, s, lo, nb, hi, c.beta, b + 1 == nbatch ? 1 : 0,
+                 arrival_ms, pred_delay, w.pend[b & 1], w.pend[(b & 1) ^ 1], w.cid, w.tout, w.S);
+    if (per_step)  // 1'.
+      launch_pdl(stream_interval_kernel, 1, kSt, 0, s, hi, D, c.cap, c.accounting, arrival_ms,
+                 prompt, true_len, w.U, w.res_u, w.st, w.g, w.dec, act_in, w.wid, w.wperm, w.wseg,
+                 w.qhead, w.aseq, w.dseq, w.rbuf, w.sbuf, w.done_id, w.done_rem, w.S, dec_stats_out);
+    launch_pdl(stream_advance_kernel, 1, kSt, 0, s, hi, D, c.cap, c.accounting, per_step, arrival_ms,
+               prompt, true_len, w.res_u, w.st, w.g, w.dec, act_in, act, w.done_id, w.done_rem,
+               w.used, w.S, stats_b, dec_stats_out);
     MAPS_TRY(launch_ok());
     MAPS_TRY(cuda_ok(cudaMemcpyAsync(&hs, w.S, sizeof(hs), cudaMemcpyDeviceToHost, s)));
     MAPS_TRY(cuda_ok(cudaStreamSynchronize(s)));
-    const int nact = hs.nact, ndone = hs.ndone, nwait = hs.nwait;
+    int nact = hs.nact;
+    const int ndone = hs.ndone, nwait = hs.nwait;
+    // the policy's candidates: the batch, or (deferral) the listed ids
+    const int nc = defer ? hs.nc : nb, nto = defer ? hs.nto : 0;
+    const int32_t *cids = defer ? w.cid : nullptr;
+    const int32_t *cpr = defer ? w.cp : prompt + lo;
+    int32_t *cch = defer ? w.cch : choice_out + lo;
 
     if (ndone > 0) {  // 2.
       MAPS_TRY(maps_order_local(ndone, 1, w.zeros, w.done_rem, w.zeros, w.done_id, 0, w.done_perm,
@@ -1053,47 +1430,62 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
       total_done += ndone;
     }
     const int64_t win_len = std::min<long long>(total_done, c.window);
+    if (nto > 0) {  // 4 (second half): timed out, round robin with the horizon as bound
+      launch_pdl(stream_enqueue_list_kernel, grid_for(nto), 256, 0, s, nto, nact, D, c.H, hi,
+                 arrival_ms, w.tout, nullptr, w.Uq, choice_out, w.st, w.dec, w.disp, w.g, w.U, act,
+                 w.S, status);
+      nact += nto;
+    }
 
-    launch_pdl(stream_gather_kernel, grid_for(nact + nb), 256, 0, s, nact, nb, lo, act, pred, w.qpred);
-    const int cs = maps_calibrate(w.win_true, w.win_pred, win_len, c.alpha_ppm, w.qpred, nact + nb,
+    launch_pdl(stream_gather_kernel, grid_for(nact + nc), 256, 0, s, nact, nc, lo, act, cids, pred,
+               prompt, w.qpred, w.cp);
+    const int cs = maps_calibrate(w.win_true, w.win_pred, win_len, c.alpha_ppm, w.qpred, nact + nc,
                                   w.Uq, w.q_dev, nullptr, ws, w.sub_bytes, stream);  // 3.
     const bool rr = cs == MAPS_E_UNBOUNDED;
     if (cs != MAPS_OK && !rr) return cs;
     if (rr)
-      launch_pdl(stream_rr_kernel, grid_for(nact + nb), 256, 0, s, nact + nb, nb, lo, D, 1, w.qpred,
-                 w.Uq, choice_out);
+      launch_pdl(stream_rr_kernel, grid_for(nact + nc), 256, 0, s, nact + nc, nc, lo, D, 1, w.qpred,
+                 w.Uq, cids, cch);
     launch_pdl(stream_csr_kernel, 1, kSt, 0, s, nact, D, rr ? 1 : 0, w.q_dev, q_out + b, act, w.st, w.g,
-                                        w.dec, prompt, w.Uq, w.U, w.res_off, w.rp, w.rg, w.rU,
-                                        w.Q);  // 4.
+               w.dec, prompt, w.Uq, w.U, w.res_off, w.rp, w.rg, w.rU, w.Q, arrival_ms, pdl, hi,
+               c.H);  // 4.
     MAPS_TRY(launch_ok());
     const int mc = c.dispatch_policy == MAPS_STREAM_MC ? 1 : 0;
-    if (!rr && c.dispatch_policy == MAPS_STREAM_RR) {  // 5'.
-      launch_pdl(stream_rr_kernel, grid_for(nb), 256, 0, s, nb, nb, lo, D, 0, w.qpred, w.Uq, choice_out);
+    if (nc == 0) {
+      // nobody to dispatch at this step
+    } else if (!rr && c.dispatch_policy == MAPS_STREAM_RR) {  // 5'.
+      launch_pdl(stream_rr_kernel, grid_for(nc), 256, 0, s, nc, nc, lo, D, 0, w.qpred, w.Uq, cids, cch);
       MAPS_TRY(launch_ok());
     } else if (!rr && c.dispatch_policy == MAPS_STREAM_LR) {
-      launch_pdl(stream_lr_kernel, 1, 32, 0, s, D, nb, w.res_off, choice_out + lo);
+      launch_pdl(stream_lr_kernel, 1, 32, 0, s, D, nc, w.res_off, cch);
       MAPS_TRY(launch_ok());
     } else if (!rr) {  // 5.
-      const size_t dsm = stream_dispatch_smem(D, nact, nb);
+      const size_t dsm = stream_dispatch_smem(D, nact, nc);
       if (dsm + 2048 <= static_cast<size_t>(max_smem_optin())) {
         // the decoders' pairs fit in shared memory: no dense projection
         MAPS_TRY(cuda_ok(cudaFuncSetAttribute(stream_dispatch_kernel,
                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               static_cast<int>(dsm))));
-        launch_pdl(stream_dispatch_kernel, 1, kSt, dsm, s, D, c.H, nb, mc, w.res_off, w.rp, w.rg,
-                   w.rU, w.capv, w.Q, prompt + lo, w.Uq + nact, choice_out + lo, w.headroom, status);
+        launch_pdl(stream_dispatch_kernel, 1, kSt, dsm, s, D, c.H, nc, mc, w.res_off, w.rp, w.rg,
+                   w.rU, w.capv, w.Q, cpr, w.Uq + nact, cch, w.headroom, status);
         MAPS_TRY(launch_ok());
       } else {
         MAPS_TRY(maps_project_occupancy(D, c.H, w.res_off, nact, w.rp, w.rg, w.rU, w.K, nullptr, ws,
                                         w.sub_bytes, stream));
-        MAPS_TRY(dispatch_sequential(D, c.H, w.K, w.capv, w.Q, nb, prompt + lo, w.Uq + nact,
-                                     choice_out + lo, w.headroom, mc != 0, ws, s));
+        MAPS_TRY(dispatch_sequential(D, c.H, w.K, w.capv, w.Q, nc, cpr, w.Uq + nact, cch,
+                                     w.headroom, mc != 0, ws, s));
       }
     }
-    launch_pdl(stream_enqueue_kernel, grid_for(nb), 256, 0, s, lo, nb, nact, hi, D, arrival_ms,
-                                                       choice_out, w.Uq, w.st, w.dec, w.disp, w.g,
-                                                       w.U, act, w.S, status);  // 6.
-    const int n_all = nact + nb, nw = nwait + nb;
+    if (defer) {
+      if (nc > 0)
+        launch_pdl(stream_enqueue_list_kernel, grid_for(nc), 256, 0, s, nc, nact, D, c.H, hi,
+                   arrival_ms, w.cid, w.cch, w.Uq, choice_out, w.st, w.dec, w.disp, w.g, w.U, act,
+                   w.S, status);  // 6.
+    } else {
+      launch_pdl(stream_enqueue_kernel, grid_for(nb), 256, 0, s, lo, nb, nact, hi, D, arrival_ms,
+                 choice_out, w.Uq, w.st, w.dec, w.disp, w.g, w.U, act, w.S, status);  // 6.
+    }
+    const int n_all = nact + nc, nw = nwait + nto + nc;
     launch_pdl(stream_waitlist_kernel, 1, kSt, 0, s, n_all, hi, arrival_ms, act, w.st, w.dec, w.U, w.disp,
                                              w.wid, w.wdec, w.wU, w.wwait, w.warr);  // 7.
     MAPS_TRY(launch_ok());
@@ -1102,9 +1494,9 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
     MAPS_TRY(maps_order_local(nw, D, w.wdec, w.wU, w.wwait, w.warr, mw, w.wperm, w.wseg, ws,
                               w.sub_bytes, stream));
     const int64_t hi_next = b + 1 < nbatch ? std::min(hi + B, N) : hi;
-    launch_pdl(stream_admit_kernel, 1, kSt, 0, s, D, c.cap, c.accounting, nw, hi, hi_next, arrival_ms,
-               w.wseg, w.wperm, w.wid, prompt, w.U, w.used, w.st, w.g, w.res_u, stats_b,
-               dec_stats_out);  // 8.
+    launch_pdl(stream_admit_kernel, 1, kSt, 0, s, D, c.cap, c.accounting, per_step, nw, hi, hi_next,
+               arrival_ms, w.wseg, w.wperm, w.wid, prompt, w.U, w.used, w.st, w.g, w.res_u, w.aseq,
+               w.dseq, w.qhead, w.S, stats_b, dec_stats_out);  // 8.
     MAPS_TRY(launch_ok());
   }
   return maps_check(ws, stream);

@@ -39,7 +39,8 @@ class StreamCfg(ctypes.Structure):
                 ("cap", ctypes.c_int32), ("batch", ctypes.c_int32), ("window", ctypes.c_int32),
                 ("alpha_ppm", ctypes.c_uint32), ("max_wait", ctypes.c_int32),
                 ("dispatch_policy", ctypes.c_int32), ("local_order", ctypes.c_int32),
-                ("accounting", ctypes.c_int32)]
+                ("accounting", ctypes.c_int32), ("per_step", ctypes.c_int32),
+                ("beta", ctypes.c_int32)]
 
 
 # maps_stream_cfg policy fields
@@ -88,7 +89,8 @@ def _load():
         "maps_rr_pressure": ([ctypes.POINTER(RRCfg), i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
                              ctypes.c_int),
         "maps_stream_workspace_size": ([ctypes.POINTER(StreamCfg)], sz),
-        "maps_stream_run": ([ctypes.POINTER(StreamCfg), vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
+        "maps_stream_run": ([ctypes.POINTER(StreamCfg), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz,
+                             vp],
                             ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
@@ -239,21 +241,25 @@ def maps_order_local_static(D: int, dec, bound, wait, arrival, max_wait: int, pe
 
 def stream_cfg(N: int, D: int, H: int, cap: int, batch: int, window: int, alpha_ppm: int,
                max_wait: int, dispatch_policy: int = STREAM_MAPS, local_order: int = STREAM_SJF,
-               accounting: int = STREAM_OCCUPANCY) -> StreamCfg:
+               accounting: int = STREAM_OCCUPANCY, per_step: int = 0,
+               beta: int = -1) -> StreamCfg:
     return StreamCfg(int(N), int(D), int(H), int(cap), int(batch), int(window), int(alpha_ppm),
-                     int(max_wait), int(dispatch_policy), int(local_order), int(accounting))
+                     int(max_wait), int(dispatch_policy), int(local_order), int(accounting),
+                     int(per_step), int(beta))
 
 
 def maps_stream_run(cfg: StreamCfg, arrival_ms, prompt, true_len, pred, choice_out, q_out,
                     stats_out, dec_stats_out=None, ws: Workspace | None = None,
-                    stream=None) -> int:
+                    stream=None, pred_delay=None) -> int:
     """The whole streaming loop on the device; returns the full status.
-    dec_stats_out: optional [D][3] int64 per-decoder statistics."""
+    dec_stats_out: optional [D][4] int64 per-decoder statistics; pred_delay:
+    [N] int32 prediction delays (required when cfg.beta >= 0)."""
     ws = ws or Workspace()
     ws.ensure(lib.maps_stream_workspace_size(ctypes.byref(cfg)))
     return lib.maps_stream_run(ctypes.byref(cfg), _ptr(arrival_ms, torch.int64),
                                _ptr(prompt, torch.int32), _ptr(true_len, torch.int32),
-                               _ptr(pred, torch.int32), _ptr(choice_out, torch.int32),
+                               _ptr(pred, torch.int32), _ptr(pred_delay, torch.int32),
+                               _ptr(choice_out, torch.int32),
                                _ptr(q_out, torch.int32), _ptr(stats_out, torch.int64),
                                _ptr(dec_stats_out, torch.int64), ws.ptr, ws.nbytes,
                                _stream(stream))

@@ -35,7 +35,7 @@ def run_both(M, ws, oracle, w, N, D, H, cap, B, Wn, a, mw, pol, loc, acc):
     ch = torch.full((N,), -9, dtype=torch.int32, device="cuda")
     q = torch.full((nb,), -9, dtype=torch.int32, device="cuda")
     stats = torch.full((nb, 4), -9, dtype=torch.int64, device="cuda")
-    ds = torch.full((D, 3), -9, dtype=torch.int64, device="cuda")
+    ds = torch.full((D, 4), -9, dtype=torch.int64, device="cuda")
     cfg = M.stream_cfg(N, D, H, cap, B, Wn, a, mw, pol, loc, acc)
     st = M.maps_stream_run(cfg, dev(w["arrival_ms"][:N], np.int64), dev(w["prompt"][:N], np.int32),
                            dev(w["true"][:N], np.int32), dev(w["pred"][:N], np.int32), ch, q, stats,
