@@ -731,10 +731,13 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
 
     ds = torch.empty((w["D"], 4), dtype=torch.int64, device=device)
 
-    def run(n, pol=(0, 0, 0), cap=None):
+    dl = t(w["pred_delay_ms"], np.int32)
+
+    def run(n, pol=(0, 0, 0), cap=None, per_step=0, beta=-1):
         cfg = M.stream_cfg(n, w["D"], w["H"], w["cap"] if cap is None else cap, B, w["window"],
-                           w["alpha_ppm"], w["max_wait"], *pol)
-        st = M.maps_stream_run(cfg, arr[:n], pr[:n], tr[:n], pd[:n], ch[:n], q, stats, ds, ws=ws)
+                           w["alpha_ppm"], w["max_wait"], *pol, per_step=per_step, beta=beta)
+        st = M.maps_stream_run(cfg, arr[:n], pr[:n], tr[:n], pd[:n], ch[:n], q, stats, ds, ws=ws,
+                               pred_delay=dl[:n] if beta >= 0 else None)
         if st != 0:
             raise RuntimeError(f"maps_stream_run status {st}")
 
@@ -769,6 +772,29 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
                               "time_weighted_queue_max": float(tw.max()),
                               "overflow_events": d[1], "admissions": d[2]}
         out[label] = variants
+    # the fidelity modes: per-step admission with preemption, and deferral
+    # until the bound is available (prediction delays of the workload, beta
+    # = 1 s), at the workload's capacity and at 16,000
+    fidelity = {}
+    for label, cap in (("cap262144", None), ("cap16000", 16000)):
+        for name, kw in (("per_step", dict(per_step=1)),
+                         ("deferral", dict(beta=int(w["beta_ms"]))),
+                         ("per_step_deferral", dict(per_step=1, beta=int(w["beta_ms"])))):
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            run(N, cap=cap, **kw)
+            sv = time.perf_counter() - t0
+            per = ds.cpu().numpy()
+            d = per.sum(axis=0).tolist()
+            fidelity[f"{name}_{label}"] = {
+                "value": N / sv, "seconds": sv,
+                "time_weighted_queue_mean": float((per[:, 0] / max(span, 1)).mean()),
+                "overflow_events": d[1], "admissions": d[2], "preemptions": d[3]}
+    out["fidelity"] = fidelity
+    out["pred_delay"] = {"median_ms": float(np.median(w["pred_delay_ms"])),
+                         "p95_ms": float(np.percentile(w["pred_delay_ms"], 95)),
+                         "over_beta": float((w["pred_delay_ms"] > w["beta_ms"]).mean()),
+                         "beta_ms": int(w["beta_ms"])}
     if cpu_sample:
         import oracle as O
         n = min(cpu_sample, N)

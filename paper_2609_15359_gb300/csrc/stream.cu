@@ -23,8 +23,13 @@
 // dispatch: stream_dispatch with mc, stream_rr, stream_lr), the order of step 7
 // (FCFS: every entry promoted, so arrival order alone) and what a running
 // request counts for in step 8 (occupancy, staged or held reservation).
-// The host issues the launches; it reads 24 bytes of loop state once per
-// batch (the request, completion and waiting counts that size the calls).
+// Fidelity modes: per-step admission with preemption replaces step 1 by a
+// step-by-step simulation of each decoder (stream_interval); deferral splits
+// the arrived requests at each dispatch step into those with a bound, those
+// timed out to round robin and those that keep waiting (stream_select).
+// The host issues the launches; it reads 40 bytes of loop state once per
+// batch (the request, completion and waiting counts, and the deferral's list
+// lengths, that size the calls).
 #include <algorithm>
 #include <climits>
 

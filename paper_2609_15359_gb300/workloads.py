@@ -44,7 +44,7 @@ WORKLOADS = {
                    cap=262144, H=16384, window=500, alpha_ppm=100000,
                    rate=200.0, burst_prob=0.1, burst_mult=5.0,
                    prompt=(32, 2048), out="lognormal", out_params=(5.5, 1.0),
-                   clip=8192, sigma=0.4),
+                   clip=8192, sigma=0.4, pred_delay=(30.0, 0.25, 0.5), beta=1000),
     # App. A simulation setup: N decoders of C tokens, t_tok = 1 ms, theta =
     # 0.85, 10,000 requests; the trace's empirical length bins are not
     # available, tiny's prompt and output distributions stand in for them
@@ -166,7 +166,7 @@ def make_stream(seed: int | None = None, n_requests: int | None = None) -> dict:
     cfg = WORKLOADS["stream"]
     N = cfg["n_requests"] if n_requests is None else int(n_requests)
     ss = np.random.SeedSequence(cfg["index"] if seed is None else seed)
-    s_b, s_n, s_t, s_p, s_l, s_e = [np.random.default_rng(c) for c in ss.spawn(6)]
+    s_b, s_n, s_t, s_p, s_l, s_e, s_d = [np.random.default_rng(c) for c in ss.spawn(7)]
     times = []
     total = 0
     w = 0
@@ -183,10 +183,18 @@ def make_stream(seed: int | None = None, n_requests: int | None = None) -> dict:
     prompt = _prompts(s_p, cfg, N)
     true = _lengths(s_l, cfg, N)
     pred = _predict(s_e, cfg, true)
+    # prediction latency (steps from arrival until the bound is available):
+    # grows with the prompt, tens of ms for short prompts to several hundred
+    # for the longest (App. D), with a log-normal spread; a few percent pass
+    # the 1 s timeout
+    a, b_, sd = cfg["pred_delay"]
+    delay = (a + b_ * prompt) * np.exp(s_d.normal(0.0, sd, N))
+    pred_delay_ms = np.minimum(np.rint(delay), 60000).astype(np.int32)
     return dict(name="stream", N=N, D=cfg["D"], H=cfg["H"], cap=cfg["cap"],
                 batch=cfg["batch"], window=cfg["window"],
                 alpha_ppm=cfg["alpha_ppm"], max_wait=MAX_WAIT_STEPS,
-                arrival_ms=arrival_ms, prompt=prompt, true=true, pred=pred)
+                arrival_ms=arrival_ms, prompt=prompt, true=true, pred=pred,
+                pred_delay_ms=pred_delay_ms, beta_ms=cfg["beta"])
 
 
 def make_rr(n_seeds: int = 1, rhos=None, n_req: int | None = None, seed0: int = 0) -> dict:
