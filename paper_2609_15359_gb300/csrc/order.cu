@@ -94,6 +94,15 @@ __host__ __device__ __forceinline__ int64_t prep_chunk(int64_t N) {
   const int64_t c = (per + kKeysRound - 1) / kKeysRound * kKeysRound;
   return c > kKeysRound ? c : kKeysRound;
 }
+// The bucketed form (order_bucket_kernel): entries per thread per round, and
+// its blocks' ranges (whole rounds, at most kPrepBlocks blocks).
+constexpr int kBucketU = 8;
+constexpr int kBucketRound = 512 * kBucketU;
+__host__ __device__ __forceinline__ int64_t bucket_chunk(int64_t N) {
+  const int64_t per = (N + kPrepBlocks - 1) / kPrepBlocks;
+  const int64_t c = (per + kBucketRound - 1) / kBucketRound * kBucketRound;
+  return c > kBucketRound ? c : kBucketRound;
+}
 constexpr int kSegThreads = 512;
 constexpr int kSegIPT = 9;
 constexpr int kSegMax = kSegThreads * kSegIPT;  // entries one block sorts
@@ -171,7 +180,8 @@ __device__ __forceinline__ int bit_width(uint32_t x) { return x ? 32 - __clz(x) 
 // in index order.
 __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_count,
                                int64_t *seg_off, int64_t *item_off, int32_t *item_n,
-                               int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, PairQueues pq) {
+                               int32_t *item_dec, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t,
+                               PairQueues pq) {
   __shared__ long long s_w[32];
   __shared__ int s_bw[32];
   __shared__ long long s_carry;
@@ -216,10 +226,12 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
       const uint32_t it = atomicAdd(&counts->nitems, 1u);
       item_off[it] = start;
       item_n[it] = static_cast<int32_t>(c);
+      item_dec[it] = k;
     } else if (k < D && big) {
       const int nch = static_cast<int>((c + kSegMax - 1) / kSegMax);
       const uint32_t it = atomicAdd(&counts->nitems, static_cast<uint32_t>(nch));
       for (int j = 0; j < nch; ++j) {
+        item_dec[it + j] = k;
         item_off[it + j] = start + static_cast<int64_t>(j) * kSegMax;
         item_n[it + j] = -static_cast<int32_t>(min(static_cast<long long>(kSegMax), c - static_cast<long long>(j) * kSegMax));
       }
@@ -269,8 +281,8 @@ order_prep_kernel(int64_t N, int D, int64_t chunk, const int32_t *__restrict__ d
                   const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
                   const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
                   uint32_t *dec_count, int32_t *status, int64_t *seg_off, int64_t *item_off,
-                  int32_t *item_n, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t, PairQueues pq,
-                  uint32_t *blk, uint32_t *grp, int Dp) {
+                  int32_t *item_n, int32_t *item_dec, int64_t *mt_off, int32_t *mt_n, int32_t *mt_t,
+                  PairQueues pq, uint32_t *blk, uint32_t *grp, int Dp) {
   pdl_prologue();
   __shared__ uint32_t s_dec[kDecSmem];
   __shared__ bool s_last;
@@ -346,7 +358,244 @@ order_prep_kernel(int64_t N, int D, int64_t chunk, const int32_t *__restrict__ d
   __syncthreads();
   if (s_last) {
     __threadfence();
-    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, mt_off, mt_n, mt_t, pq);
+    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, item_dec, mt_off, mt_n, mt_t, pq);
+  }
+}
+
+// Stable segmented form, first pass (D <= kStableD), in place of the prep
+// and key passes: one read of the four inputs.  Block b takes the contiguous
+// entries [b chunk, (b + 1) chunk) and
+//   1. counts them per decoder: blk[b][d], added to the totals dec_count[d];
+//   2. writes each entry's raw key (not promoted << 63 | primary << 32 |
+//      index, the primary being the bound of a non-promoted entry, else 0)
+//      to raw[b chunk + bst[b][d] + its rank among the block's entries of
+//      decoder d in index order], bst[b][d] being the block's exclusive
+//      prefix of its counts over the decoders: the block's entries bucketed
+//      by decoder, stably;
+//   3. validates, takes the largest non-promoted bound and checks that
+//      arrival is non-decreasing along the index, as the prep pass does.
+// The last block to finish plans the segments (seg_plan_block).  The segment
+// sort then gathers decoder d's entries block by block, which is index order.
+__global__ void __launch_bounds__(512, 2)
+order_bucket_kernel(int64_t N, int D, int64_t chunk, int Dp, const int32_t *__restrict__ dec,
+                    const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
+                    const int32_t *__restrict__ arrival, int32_t max_wait, OrderCounts *counts,
+                    uint32_t *dec_count, int32_t *status, int64_t *seg_off, int64_t *item_off,
+                    int32_t *item_n, int32_t *item_dec, int64_t *mt_off, int32_t *mt_n,
+                    int32_t *mt_t, PairQueues pq, uint32_t *blk, uint32_t *bst,
+                    unsigned long long *raw) {
+  pdl_prologue();
+  extern __shared__ __align__(16) uint32_t bsm[];
+  uint32_t *hw = bsm;                     // [kPassWarps][Dp] per-warp counts, then slot bases
+  uint32_t *run = bsm + kPassWarps * Dp;  // [Dp] counts, then the next slot of each bucket
+  __shared__ uint32_t s_w[kPassWarps];
+  __shared__ bool s_last;
+  constexpr int kU = kBucketU;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t r_begin = static_cast<int64_t>(blockIdx.x) * chunk;
+  const int64_t r_end = r_begin + chunk < N ? r_begin + chunk : N;
+  // a range of one round keeps its loads in registers from the count to the
+  // scatter (all of them issued together); longer ranges load twice
+  const bool one = r_end - r_begin <= kBucketRound;
+  // per entry only its decoder and raw key stay live: validation, the largest
+  // bound and the arrival check are taken as the loads land
+  int32_t d[kU];
+  uint32_t kp[kU];  // not promoted << 31 | primary (the index follows from the position)
+  bool bad = false, unsorted = false;
+  uint32_t umax = 0;
+  auto load = [&](int64_t i0, bool all) {
+    int32_t u[kU], w[kU], ar[kU], an[kU], dr[kU];
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int64_t i = i0 + warp * (32 * kU) + q * 32 + lane;
+      const bool ok = i < r_end;
+      dr[q] = ok ? __ldg(dec + i) : 0;
+      // an entry of the range always has a decoder in [0, D): one out of the
+      // domain is counted and placed at 0 (and flagged)
+      d[q] = !ok ? -1 : (dr[q] < 0 || dr[q] >= D ? 0 : dr[q]);
+      if (all) {
+        u[q] = ok ? __ldg(bound + i) : 0;
+        w[q] = ok ? __ldg(wait + i) : 0;
+        ar[q] = ok ? __ldg(arrival + i) : 0;
+        an[q] = (ok && i + 1 < N) ? __ldg(arrival + i + 1) : 0x7fffffff;
+      }
+    }
+    if (!all) return;
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int64_t i = i0 + warp * (32 * kU) + q * 32 + lane;
+      if (i < r_end) {
+        if (dr[q] < 0 || dr[q] >= D || u[q] < 0 || ar[q] < 0) bad = true;
+        if (w[q] <= max_wait && u[q] > 0) umax = max(umax, static_cast<uint32_t>(u[q]));
+        if (an[q] < ar[q]) unsorted = true;
+      }
+      const uint32_t np = w[q] > max_wait ? 0u : 1u;
+      kp[q] = np ? (1u << 31) | static_cast<uint32_t>(u[q] < 0 ? 0 : u[q]) : 0u;
+    }
+  };
+  for (int k = tid; k < Dp; k += blockDim.x) run[k] = 0;
+  __syncthreads();
+  // 1. counts
+  for (int64_t i0 = r_begin; i0 < r_end; i0 += kBucketRound) {
+    load(i0, one);
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const unsigned pe = __match_any_sync(0xffffffffu, d[q]);
+      if (d[q] >= 0 && lane == __ffs(pe) - 1) atomicAdd(&run[d[q]], static_cast<uint32_t>(__popc(pe)));
+    }
+  }
+  __syncthreads();
+  {
+    // block exclusive scan of the counts over the decoders (two per thread;
+    // Dp <= 2 * blockDim.x), published with the counts
+    const int k0 = 2 * tid;
+    const uint32_t v0 = k0 < Dp ? run[k0] : 0u, v1 = k0 + 1 < Dp ? run[k0 + 1] : 0u;
+    uint32_t incl = v0 + v1;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_w[warp] = incl;
+    __syncthreads();
+    uint32_t base = 0;
+    for (int ww2 = 0; ww2 < warp; ++ww2) base += s_w[ww2];
+    const uint32_t e0 = base + incl - v0 - v1;
+    uint32_t *brow = blk + static_cast<int64_t>(blockIdx.x) * Dp;
+    uint32_t *srow = bst + static_cast<int64_t>(blockIdx.x) * Dp;
+    if (k0 < Dp) {
+      brow[k0] = v0;
+      srow[k0] = e0;
+      run[k0] = e0;
+      if (v0) atomicAdd(&dec_count[k0], v0);
+    }
+    if (k0 + 1 < Dp) {
+      brow[k0 + 1] = v1;
+      srow[k0 + 1] = e0 + v0;
+      run[k0 + 1] = e0 + v0;
+      if (v1) atomicAdd(&dec_count[k0 + 1], v1);
+    }
+  }
+  __syncthreads();
+  // 2. and 3., round by round in index order
+  unsigned long long *out = raw + r_begin;
+  for (int64_t i0 = r_begin; i0 < r_end; i0 += kBucketRound) {
+    for (int k = tid; k < kPassWarps * Dp; k += blockDim.x) hw[k] = 0;
+    if (!one) load(i0, true);
+    __syncthreads();  // counts zeroed
+    uint32_t rk[kU], base[kU];  // leader lane << 8 | rank in the group; group size, then base
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const unsigned pe = __match_any_sync(0xffffffffu, d[q]);
+      const int leader = __ffs(pe) - 1;
+      rk[q] = (static_cast<uint32_t>(leader) << 8) | static_cast<uint32_t>(__popc(pe & lanemask_lt()));
+      base[q] = lane == leader ? static_cast<uint32_t>(__popc(pe)) : 0u;
+    }
+#pragma unroll
+    for (int q = 0; q < kU; ++q)  // in item order, so ranks follow the index
+      if (d[q] >= 0 && base[q] != 0) base[q] = atomicAdd(&hw[warp * Dp + d[q]], base[q]);
+    __syncthreads();
+    for (int k = tid; k < D; k += blockDim.x) {  // exclusive over the warps
+      uint32_t r = run[k];
+      for (int ww2 = 0; ww2 < kPassWarps; ++ww2) {
+        const uint32_t c = hw[ww2 * Dp + k];
+        hw[ww2 * Dp + k] = r;
+        r += c;
+      }
+      run[k] = r;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const uint32_t b = __shfl_sync(0xffffffffu, base[q], static_cast<int>(rk[q] >> 8));
+      const int64_t i = i0 + warp * (32 * kU) + q * 32 + lane;
+      if (d[q] >= 0)
+        out[hw[warp * Dp + d[q]] + b + (rk[q] & 255u)] =
+            (static_cast<unsigned long long>(kp[q]) << 32) | static_cast<unsigned long long>(i & 0xffffffff);
+    }
+    __syncthreads();  // the counts are zeroed again for the next round
+  }
+  if (bad) flag_error(status, MAPS_E_RANGE);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) umax = max(umax, __shfl_xor_sync(0xffffffffu, umax, off));
+  if (lane == 0 && umax) atomicMax(&counts->max_bound, umax);
+  if (__syncthreads_or(unsorted) && tid == 0) atomicOr(&counts->unsorted, 1u);
+  // the last block to finish plans the segmented form (one thread publishes
+  // the block's results: the barrier orders every thread's atomics before
+  // its fence, as a grid barrier does)
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    s_last = atomicAdd(&counts->done_blocks, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    seg_plan_block(D, counts, dec_count, seg_off, item_off, item_n, item_dec, mt_off, mt_n, mt_t, pq);
+  }
+}
+
+// The global form's key pass: each entry's key (decoder, not promoted,
+// primary) in index order, its arrival digits where arrival is out of index
+// order, and the histograms of every digit (sh: kPasses x kRadix words of
+// shared memory).  Any grid; every thread of the block takes part.
+__device__ void global_key_pass(int64_t N, int D, int dbits, const int32_t *__restrict__ dec,
+                                const int32_t *__restrict__ bound, const int32_t *__restrict__ wait,
+                                const int32_t *__restrict__ arrival, int32_t max_wait,
+                                OrderCounts *counts, unsigned long long *hi_orig,
+                                unsigned long long *keyA, uint32_t *valA, uint32_t *sh) {
+  for (int i = threadIdx.x; i < kPasses * kRadix; i += blockDim.x) sh[i] = 0;
+  __syncthreads();
+  const int ub = bit_width(*reinterpret_cast<volatile uint32_t *>(&counts->max_bound));
+  const bool unsorted = *reinterpret_cast<volatile uint32_t *>(&counts->unsorted) != 0;
+  const bool wide = dbits + 1 + ub > 32;
+  const int n_hi = (dbits + 1 + ub + 7) / 8;
+  constexpr int kU = 4;  // entries per thread per round, loads issued together
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x * kU;
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x * kU; i0 < N; i0 += stride) {
+    int32_t d[kU], u[kU], ar[kU], w[kU];
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int64_t i = i0 + q * blockDim.x + threadIdx.x;
+      const bool ok = i < N;
+      d[q] = ok ? __ldg(dec + i) : 0;
+      u[q] = ok ? __ldg(bound + i) : 0;
+      ar[q] = ok ? __ldg(arrival + i) : 0;
+      w[q] = ok ? __ldg(wait + i) : 0;
+    }
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int64_t i = i0 + q * blockDim.x + threadIdx.x;
+      const bool valid = i < N;
+      unsigned long long key = 0;
+      uint32_t a = 0;
+      if (valid) {
+        const int32_t dd = d[q] < 0 || d[q] >= D ? 0 : d[q];  // out-of-domain entries were flagged
+        const int32_t uu = u[q] < 0 ? 0 : u[q];
+        const int32_t aa = ar[q] < 0 ? 0 : ar[q];
+        const bool promoted = w[q] > max_wait;
+        const unsigned long long prim = promoted ? 0ull : static_cast<unsigned long long>(uu);
+        key = (static_cast<unsigned long long>(dd) << (1 + ub)) |
+              (static_cast<unsigned long long>(promoted ? 0u : 1u) << ub) | prim;
+        a = static_cast<uint32_t>(aa);
+        hi_orig[i] = key;
+        if (unsorted) {
+          keyA[i] = a;
+          valA[i] = static_cast<uint32_t>(i);
+        }
+      }
+      if (unsorted)
+#pragma unroll
+        for (int p = 0; p < kLoPasses; ++p) warp_count(sh + p * kRadix, (a >> (8 * p)) & 255u, valid);
+      for (int p = 0; p < n_hi; ++p)
+        warp_count(sh + (kLoPasses + p) * kRadix, static_cast<int>((key >> (8 * p)) & 255u), valid);
+    }
+  }
+  (void)wide;
+  __syncthreads();
+  for (int i = threadIdx.x; i < kPasses * kRadix; i += blockDim.x) {
+    const uint32_t c = sh[i];
+    if (c) atomicAdd(&(&counts->h[0][0])[i], c);
   }
 }
 
@@ -492,60 +741,8 @@ order_keys_kernel(int64_t N, int D, int dbits, int64_t chunk, int Dp,
     }
     return;
   }
-  __shared__ uint32_t sh[kPasses][kRadix];
-  for (int i = threadIdx.x; i < kPasses * kRadix; i += blockDim.x) (&sh[0][0])[i] = 0;
-  __syncthreads();
-  const int ub = bit_width(*reinterpret_cast<volatile uint32_t *>(&counts->max_bound));
-  const bool unsorted = *reinterpret_cast<volatile uint32_t *>(&counts->unsorted) != 0;
-  const bool wide = dbits + 1 + ub > 32;
-  const int n_hi = (dbits + 1 + ub + 7) / 8;
-  constexpr int kU = 4;  // entries per thread per round, loads issued together
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x * kU;
-  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x * kU; i0 < N; i0 += stride) {
-    int32_t d[kU], u[kU], ar[kU], w[kU];
-#pragma unroll
-    for (int q = 0; q < kU; ++q) {
-      const int64_t i = i0 + q * blockDim.x + threadIdx.x;
-      const bool ok = i < N;
-      d[q] = ok ? __ldg(dec + i) : 0;
-      u[q] = ok ? __ldg(bound + i) : 0;
-      ar[q] = ok ? __ldg(arrival + i) : 0;
-      w[q] = ok ? __ldg(wait + i) : 0;
-    }
-#pragma unroll
-    for (int q = 0; q < kU; ++q) {
-      const int64_t i = i0 + q * blockDim.x + threadIdx.x;
-      const bool valid = i < N;
-      unsigned long long key = 0;
-      uint32_t a = 0;
-      if (valid) {
-        const int32_t dd = d[q] < 0 || d[q] >= D ? 0 : d[q];  // out-of-domain entries were flagged
-        const int32_t uu = u[q] < 0 ? 0 : u[q];
-        const int32_t aa = ar[q] < 0 ? 0 : ar[q];
-        const bool promoted = w[q] > max_wait;
-        const unsigned long long prim = promoted ? 0ull : static_cast<unsigned long long>(uu);
-        key = (static_cast<unsigned long long>(dd) << (1 + ub)) |
-              (static_cast<unsigned long long>(promoted ? 0u : 1u) << ub) | prim;
-        a = static_cast<uint32_t>(aa);
-        hi_orig[i] = key;
-        if (unsorted) {
-          keyA[i] = a;
-          valA[i] = static_cast<uint32_t>(i);
-        }
-      }
-      if (unsorted)
-#pragma unroll
-        for (int p = 0; p < kLoPasses; ++p) warp_count(sh[p], (a >> (8 * p)) & 255u, valid);
-      for (int p = 0; p < n_hi; ++p)
-        warp_count(sh[kLoPasses + p], static_cast<int>((key >> (8 * p)) & 255u), valid);
-    }
-  }
-  (void)wide;
-  __syncthreads();
-  for (int i = threadIdx.x; i < kPasses * kRadix; i += blockDim.x) {
-    const uint32_t c = (&sh[0][0])[i];
-    if (c) atomicAdd(&(&counts->h[0][0])[i], c);
-  }
+  __shared__ uint32_t sh[kPasses * kRadix];
+  global_key_pass(N, D, dbits, dec, bound, wait, arrival, max_wait, counts, hi_orig, keyA, valA, sh);
 }
 
 // One block: digit offsets, active passes, buffer assignment, and the
@@ -891,21 +1088,50 @@ order_small_kernel(int N, int D, int dbits, const int32_t *__restrict__ dec,
   if (__syncthreads_or(bad) && tid == 0) flag_error(status, MAPS_E_RANGE);
 }
 
+// The bucketed form's inputs to the segment sort (on = 0: the entries are
+// already in their segments).
+struct BucketView {
+  int on;
+  const int32_t *item_dec;   // [item] decoder
+  const int64_t *seg_off;    // [D + 1] segment offsets
+  const uint32_t *blk, *bst; // [nblk][Dp] counts and bucket starts per bucketing block
+  int64_t chunk;             // entries per bucketing block
+  int Dp, nblk;
+  // the global form's key pass, when arrival is out of index order
+  int D, dbits;
+  const int32_t *dec, *bound, *wait, *arrival;
+  int32_t max_wait;
+  unsigned long long *keyA;
+  uint32_t *valA;
+};
+
 // Segmented form, step 2: each sort item (one decoder's queue, at most
 // kSegMax entries) is sorted by one block on its keys (not promoted,
 // promoted ? 0 : bound, index) with stable 9-bit LSD passes in shared
 // memory, skipping digits that do not vary, and its indices are written.
 // After a stable scatter the keys of a queue are already in index order and
-// the index digits are skipped too.  Blocks take items in turn until none is
-// left.
+// the index digits are skipped too.  In the bucketed form the item's entries
+// are gathered from the bucketing blocks' buckets, in index order as well.
+// Blocks take items in turn until none is left.
 __global__ void __launch_bounds__(kSegThreads, 2)
-order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_off,
-                     const int32_t *item_n, const unsigned long long *seg_keys, int32_t *perm,
-                     unsigned long long *run_keys) {
+order_segsort_kernel(int64_t N, OrderCounts *counts, const int64_t *item_off,
+                     const int32_t *item_n, unsigned long long *seg_keys, int32_t *perm,
+                     unsigned long long *run_keys, BucketView bv) {
   pdl_prologue();
-  if (!counts->segmented) return;
   extern __shared__ __align__(16) unsigned char seg_raw[];
+  if (bv.on && !counts->segmented) {
+    // arrival is out of index order: the global form's key pass runs here
+    global_key_pass(N, bv.D, bv.dbits, bv.dec, bv.bound, bv.wait, bv.arrival, bv.max_wait, counts,
+                    seg_keys, bv.keyA, bv.valA, reinterpret_cast<uint32_t *>(seg_raw));
+    return;
+  }
+  if (!counts->segmented) return;
   SegSmem &sm = *reinterpret_cast<SegSmem *>(seg_raw);
+  // bucketed: the item's decoder's non-empty buckets, in block order: the
+  // entries before each, and where it starts
+  __shared__ uint32_t s_P[kPrepBlocks];
+  __shared__ long long s_src[kPrepBlocks];
+  __shared__ uint32_t s_pw[kSegWarps], s_nw[kSegWarps];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int ub = counts->max_bound ? 32 - __clz(counts->max_bound) : 0;
   const int ib = index_bits(N);
@@ -917,14 +1143,72 @@ order_segsort_kernel(int64_t N, const OrderCounts *counts, const int64_t *item_o
     const bool chunk = item_n[item] < 0;  // a chunk of a long queue: keys for the merges
     const int n = chunk ? -item_n[item] : item_n[item];
     unsigned long long orv = 0, andv = ~0ull;
+    if (bv.on) {
+      // Gather: the item is positions [o0, o0 + n) of its decoder's entries,
+      // which the bucketing blocks hold in turn (block b: P[b] of them come
+      // before it, in its bucket at bst[b][d]).
+      const int d = bv.item_dec[item];
+      const uint32_t o0 = static_cast<uint32_t>(off - bv.seg_off[d]);
+      const bool blk_ok = tid < bv.nblk;
+      const uint32_t c = blk_ok ? bv.blk[static_cast<int64_t>(tid) * bv.Dp + d] : 0u;
+      const uint32_t st0 = blk_ok ? bv.bst[static_cast<int64_t>(tid) * bv.Dp + d] : 0u;
+      // exclusive scans of the counts and of the non-empty flags over the blocks
+      uint32_t incl = c;
+      const unsigned ne = __ballot_sync(0xffffffffu, c > 0);
 #pragma unroll
-    for (int it = 0; it < kSegIPT; ++it) {
-      const int x = it * kSegThreads + tid;
-      if (x < n) {
-        const unsigned long long key = seg_keys[off + x];
-        sm.key[0][x] = key;
-        orv |= key;
-        andv &= key;
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (lane == 31) {
+        s_pw[warp] = incl;
+        s_nw[warp] = __popc(ne);
+      }
+      __syncthreads();
+      uint32_t wb = 0, nb0 = 0, nruns = 0;
+      for (int w = 0; w < kSegWarps; ++w) {
+        wb += w < warp ? s_pw[w] : 0u;
+        nb0 += w < warp ? s_nw[w] : 0u;
+        nruns += s_nw[w];
+      }
+      if (c > 0) {
+        const uint32_t r = nb0 + __popc(ne & lanemask_lt());
+        s_P[r] = wb + incl - c;
+        s_src[r] = static_cast<long long>(tid) * bv.chunk + st0;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it) {
+        const int x = it * kSegThreads + tid;
+        if (x < n) {
+          const uint32_t pos = o0 + static_cast<uint32_t>(x);
+          int lo = 0, hi = static_cast<int>(nruns) - 1;  // the last run with P <= pos
+          while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_P[mid] <= pos)
+              lo = mid;
+            else
+              hi = mid - 1;
+          }
+          const unsigned long long r = seg_keys[s_src[lo] + (pos - s_P[lo])];
+          // r = not promoted << 63 | primary << 32 | index
+          const unsigned long long key = ((r >> 63) << (ub + ib)) | (((r >> 32) & 0x7fffffffull) << ib) |
+                                         (r & 0xffffffffull);
+          sm.key[0][x] = key;
+          orv |= key;
+          andv &= key;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int it = 0; it < kSegIPT; ++it) {
+        const int x = it * kSegThreads + tid;
+        if (x < n) {
+          const unsigned long long key = seg_keys[off + x];
+          sm.key[0][x] = key;
+          orv |= key;
+          andv &= key;
+        }
       }
     }
 #pragma unroll
@@ -1397,6 +1681,7 @@ struct OrderWs {
   OrderPlan *plan;
   int64_t *item_off;  // sort items: queues and chunks of long queues
   int32_t *item_n;
+  int32_t *item_dec;
   int64_t *mt_off;    // merge tiles of the long queues
   int32_t *mt_n, *mt_t;
   int64_t nitems_max, ntiles_max;
@@ -1404,6 +1689,7 @@ struct OrderWs {
   unsigned long long *hi_orig, *keyA, *keyB;
   uint32_t *valA, *valB;
   uint32_t *blk;      // stable scatter: [blocks][Dp] counts per prep block
+  uint32_t *bst;      // bucketed form: [blocks][Dp] each block's bucket starts
   uint32_t *grp;      // stable scatter: [groups][Dp] counts per kGroupBlocks prep blocks (zeroed)
   int64_t chunk;      // entries per prep / key block
   int blocks, Dp;
@@ -1416,7 +1702,7 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.counts = c.take<OrderCounts>(1);
   w.dec_count = c.take<uint32_t>(static_cast<size_t>(D));
   w.dec_cursor = c.take<uint32_t>(static_cast<size_t>(D));
-  w.chunk = prep_chunk(N);
+  w.chunk = D <= kStableD ? bucket_chunk(N) : prep_chunk(N);  // bucketed form: whole rounds
   w.blocks = static_cast<int>(std::max<int64_t>(1, (N + w.chunk - 1) / w.chunk));
   w.Dp = (D + 3) / 4 * 4;
   w.grp = c.take<uint32_t>(D <= kStableD ? static_cast<size_t>((w.blocks + kGroupBlocks - 1) / kGroupBlocks) * w.Dp
@@ -1429,6 +1715,7 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.ntiles_max = N / kMergeTile + D + 1;
   w.item_off = c.take<int64_t>(static_cast<size_t>(w.nitems_max));
   w.item_n = c.take<int32_t>(static_cast<size_t>(w.nitems_max));
+  w.item_dec = c.take<int32_t>(static_cast<size_t>(w.nitems_max));
   w.mt_off = c.take<int64_t>(static_cast<size_t>(w.ntiles_max));
   w.mt_n = c.take<int32_t>(static_cast<size_t>(w.ntiles_max));
   w.mt_t = c.take<int32_t>(static_cast<size_t>(w.ntiles_max));
@@ -1445,6 +1732,7 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.valA = c.take<uint32_t>(n);
   w.valB = c.take<uint32_t>(n);
   w.blk = c.take<uint32_t>(D <= kStableD ? static_cast<size_t>(w.blocks) * w.Dp : 1);
+  w.bst = c.take<uint32_t>(D <= kStableD ? static_cast<size_t>(w.blocks) * w.Dp : 1);
   return w;
 }
 
@@ -1490,10 +1778,38 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   const int n_hi = std::min(kHiPasses, (dbits + 1 + 31 + 7) / 8);
   const int sms = sm_count();
   const int64_t tiles = std::max<int64_t>(1, (N + kTile - 1) / kTile);
-  if (N > 0) {
+  // D <= kStableD: one bucketing pass replaces the prep and key passes
+  const bool bucketed = N > 0 && D <= kStableD;
+  BucketView bv = {};
+  if (bucketed) {
+    const size_t bsmem = sizeof(uint32_t) * static_cast<size_t>(kPassWarps + 1) * w.Dp;
+    MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_bucket_kernel,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          static_cast<int>(bsmem))));
+    launch_pdl(order_bucket_kernel, w.blocks, 512, bsmem, s, N, D, w.chunk, w.Dp, dec, bound, wait,
+               arrival, max_wait, w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n,
+               w.item_dec, w.mt_off, w.mt_n, w.mt_t, w.pq, w.blk, w.bst, w.hi_orig);
+    bv.on = 1;
+    bv.item_dec = w.item_dec;
+    bv.seg_off = seg_off_out;
+    bv.blk = w.blk;
+    bv.bst = w.bst;
+    bv.chunk = w.chunk;
+    bv.Dp = w.Dp;
+    bv.nblk = w.blocks;
+    bv.D = D;
+    bv.dbits = dbits;
+    bv.dec = dec;
+    bv.bound = bound;
+    bv.wait = wait;
+    bv.arrival = arrival;
+    bv.max_wait = max_wait;
+    bv.keyA = w.keyA;
+    bv.valA = w.valA;
+  } else if (N > 0) {
     launch_pdl(order_prep_kernel, w.blocks, 512, 0, s, N, D, w.chunk, dec, bound, wait, arrival,
                max_wait, w.counts, w.dec_count, status, seg_off_out, w.item_off, w.item_n,
-               w.mt_off, w.mt_n, w.mt_t, w.pq, w.blk, w.grp, w.Dp);
+               w.item_dec, w.mt_off, w.mt_n, w.mt_t, w.pq, w.blk, w.grp, w.Dp);
     // the stable scatter's per-warp counts and running slots
     const size_t keys_smem =
         D <= kStableD ? sizeof(uint32_t) * static_cast<size_t>(kPassWarps + 1) * w.Dp : 0;
@@ -1514,9 +1830,13 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_segsort_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(seg_smem))));
-  launch_pdl(order_segsort_kernel, static_cast<unsigned>(std::min<int64_t>(w.nitems_max, 2LL * sms)),
-             kSegThreads, seg_smem, s, N, w.counts, w.item_off, w.item_n, w.hi_orig, perm_out,
-             w.keyA);
+  // (the bucketed form's segment sort may run the global key pass: at least
+  // as many blocks as the bucketing pass)
+  const int64_t seg_grid = std::min<int64_t>(bucketed ? std::max<int64_t>(w.nitems_max, w.blocks)
+                                                      : w.nitems_max,
+                                             2LL * sms);
+  launch_pdl(order_segsort_kernel, static_cast<unsigned>(seg_grid), kSegThreads, seg_smem, s, N,
+             w.counts, w.item_off, w.item_n, w.hi_orig, perm_out, w.keyA, bv);
   const size_t smem = sizeof(PassSmem);
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_finish_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
