@@ -14,6 +14,8 @@
 // quantile at most three.  The last block to finish a pass picks the bin that
 // holds rank k; passes after the range has closed return at once.  Nothing
 // returns to the host between passes.
+#include <algorithm>
+
 #include "maps_internal.cuh"
 
 namespace maps {
@@ -363,14 +365,6 @@ inline int64_t conformal_rank(int64_t n, uint32_t alpha_ppm) {
   return (num + 999999) / 1000000;
 }
 
-int grid_for(int64_t work, int per_block) {
-  int64_t g = (work + per_block - 1) / per_block;
-  const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
-  if (g > cap) g = cap;
-  if (g < 1) g = 1;
-  return static_cast<int>(g);
-}
-
 }  // namespace
 }  // namespace maps
 
@@ -412,7 +406,11 @@ int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
     if (m <= kSmallM) m = 0;
   } else {
     MAPS_TRY(cuda_ok(cudaMemsetAsync(st, 0, sizeof(SelectState), s)));
-    const int g = grid_for(n, kSelectThreads * 16);
+    // one block of 1,024 threads per multiprocessor (its registers allow one),
+    // each reading at least a 128-bit word of both arrays per thread
+    const int g = static_cast<int>(std::min<int64_t>(std::max<int64_t>(1, (n + 4 * kSelectThreads - 1) /
+                                                                          (4 * kSelectThreads)),
+                                                     sm_count()));
     launch_pdl(select_pass_kernel<0>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
     launch_pdl(select_pass_kernel<1>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
     launch_pdl(select_pass_kernel<2>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
