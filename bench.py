@@ -64,22 +64,22 @@ L2_FLUSH_BYTES = 256 << 20
 # valid only for the kernel source it was taken on.
 TRAFFIC = {
     "dispatch_feasible": {"bytes": 0, "source": "dispatch.cu", "source_sha256": ""},
-    "calibrate": {"bytes": 12578673, "source": "calibrate.cu", "source_sha256":
-                  "2c2d7dd3d182439cc27caeb6ae856327284afa160f2de0b32e84a119acd45be6"},
-    "occupancy": {"bytes": 29642638, "source": "occupancy.cu", "source_sha256":
-                  "fd537e3019c8991f53d529abba17e1a23b2664a7f4477b0936c6a78e22aa0746"},
-    "dispatch": {"bytes": 26433052, "source": "dispatch.cu", "source_sha256":
-                 "7f665bf0eb59ac1b91fcd226e1e8dff0185ef058ce89b7c99f27a3e2179185ed"},
-    "dispatch_scoring": {"bytes": 21114424, "source": "dispatch.cu", "source_sha256":
-                         "7f665bf0eb59ac1b91fcd226e1e8dff0185ef058ce89b7c99f27a3e2179185ed"},
-    "order": {"bytes": 41115687, "source": "order.cu", "source_sha256":
-              "2aae9099a88207fe058f683410602dc85706e042756c58459f064ae821ab87da"},
+    "calibrate": {"bytes": 12582144, "source": "calibrate.cu", "source_sha256":
+        "02d8553297d735ede33d44784c9fc87d5305bf8758c41aa243e861f6e64b93ef"},
+    "occupancy": {"bytes": 31169536, "source": "occupancy.cu", "source_sha256":
+        "fd537e3019c8991f53d529abba17e1a23b2664a7f4477b0936c6a78e22aa0746"},
+    "dispatch": {"bytes": 26562560, "source": "dispatch.cu", "source_sha256":
+        "bc228a45bdc7bb49327bd4b8871778b2d0a6aa7e4c877112d9afa425f6628241"},
+    "dispatch_scoring": {"bytes": 21107968, "source": "dispatch.cu", "source_sha256":
+        "bc228a45bdc7bb49327bd4b8871778b2d0a6aa7e4c877112d9afa425f6628241"},
+    "order": {"bytes": 28046336, "source": "order.cu", "source_sha256":
+        "8916c704cd39734b0eed9bd2314a7d66308ef2586300643c1d3512f2d6baba5d"},
 }
 KERNELS = {
     "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
     "occupancy": "occ_bucket_kernel + occ_tile_kernel (maps_project_occupancy)",
     "dispatch": "dispatch_prep (carry scan + bin count) + bin_scatter + dispatch_snapshot_kernel (maps_dispatch)",
-    "order": "order_prep + order_keys + order_segsort + order_finish (maps_order_local)",
+    "order": "order_bucket + order_segsort + order_finish (maps_order_local)",
     "dispatch_scoring": "dispatch_snapshot_kernel alone (maps_dispatch's scoring kernel, after "
                         "the candidates are bucketed by horizon tile)",
     "dispatch_feasible": "maps_dispatch SNAPSHOT on the feasible-regime capacities (x64): carry "
@@ -287,10 +287,10 @@ class Step:
                    M.lib.maps_order_local_workspace_size(R + J, self.D))
         self.ws = M.Workspace(need, device)
         # calibrate 4 (three select passes, bounds); occupancy 2 (bucket, tile);
-        # dispatch 3 (carry scan with bin count, bin scatter, main); order 4
-        # (prep, keys, segment sort, the cooperative finishing kernel: merges or
-        # the global radix form)
-        self.kernels_per_step = 4 + 2 + 3 + 4
+        # dispatch 3 (carry scan with bin count, bin scatter, main); order 3
+        # (bucketing, segment sort, the cooperative finishing kernel: pairwise
+        # ranks or merges of the long queues, or the global radix form)
+        self.kernels_per_step = 4 + 2 + 3 + (3 if self.D <= 1024 else 4)
 
     def run(self, ev=None):
         M, R = self.M, self.R
@@ -374,7 +374,7 @@ def e2e_stages(steps, ins: dict, outs: list):
     large copy runs near 208 GB/s where a dozen smaller ones reach about 160),
     the four C-ABI calls, and the read-back of the results.  Each stage of each
     set is captured once as a CUDA graph, so a step costs the host three graph
-    launches instead of thirteen kernel launches and six copies.
+    launches instead of twelve kernel launches and six copies.
     Returns (stages, how)."""
     import torch
     side = torch.cuda.Stream()
@@ -453,7 +453,7 @@ def bench_gpu(args, world, rank, local, dist):
     step.check()
 
     # the step's four calls captured once as a CUDA graph: a replay launches
-    # the same 13 kernels with their programmatic (PDL) edges intact
+    # the same 12 kernels with their programmatic (PDL) edges intact
     side = torch.cuda.Stream()
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
