@@ -646,63 +646,77 @@ def bench_gpu(args, world, rank, local, dist):
 # the smaller configurations: Tiny, D16 and D64 (each of its three bound sets)
 # ---------------------------------------------------------------------------
 
+def time_workload(w: dict, alpha: int, device, flush, steps: int = 20) -> dict:
+    """One workload's four calls: per step a CUDA-graph replay after an L2 flush
+    (event-timed), then a pass of direct launches with an event between calls
+    for the per-call split and its HBM fractions."""
+    import torch
+    peaks = measured_peaks()
+    step = Step(w, device)
+    step.alpha = alpha
+    for _ in range(3):
+        step.run()
+    torch.cuda.synchronize()
+    step.check()
+    side = torch.cuda.Stream()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
+        step.run()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+    for i in range(steps):
+        flush.zero_()
+        ev[i][3].record()
+        graph.replay()
+        ev[i][4].record()
+    torch.cuda.synchronize()
+    step_ms = float(np.mean([e[3].elapsed_time(e[4]) for e in ev]))
+    for i in range(steps):
+        flush.zero_()
+        ev[i][3].record()
+        step.run(ev=ev[i])
+        ev[i][4].record()
+    torch.cuda.synchronize()
+    step.check()
+    call_ms = {"calibrate": [e[3].elapsed_time(e[0]) for e in ev],
+               "occupancy": [e[0].elapsed_time(e[1]) for e in ev],
+               "dispatch": [e[1].elapsed_time(e[2]) for e in ev],
+               "order": [e[2].elapsed_time(e[4]) for e in ev]}
+    alg = algorithmic_bytes(w)
+    calls = {}
+    for c in alg:
+        us = float(np.mean(call_ms[c])) * 1e3
+        calls[c] = {"us": us, "algorithmic_bytes": alg[c],
+                    "frac_of_measured_hbm": alg[c] / (us / 1e6) / 1e9 / peaks["hbm_gbs"]}
+    del step, graph
+    return {"alpha_ppm": alpha, "D": w["D"], "H": w["H"], "residents": w["R"],
+            "candidates": w["J"], "ms_per_step": step_ms,
+            "decisions_per_s": w["J"] / (step_ms / 1e3),
+            "occupancy_cells_per_s": w["D"] * w["H"] / (step_ms / 1e3),
+            "calls": calls, "steps": steps,
+            "timing": "graph replay per step after a 256 MiB L2 flush; calls split by events "
+                      "between direct launches"}
+
+
 def bench_configs(device, steps: int = 20) -> dict:
-    """The same four calls on each smaller configuration: per step a CUDA-graph
-    replay after an L2 flush (event-timed), then a pass of direct launches with
-    an event between calls for the per-call split and its HBM fractions."""
+    """The smaller configurations (Tiny, D16, D64 with each of its bound sets),
+    and the Large workload on two more draws (seeds 1 and 2) beside the timed
+    draw, so that no figure rests on one draw."""
     import torch
     from paper_2609_15359_gb300 import workloads as W
-    peaks = measured_peaks()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
     out = {}
     for name in ("tiny", "d16", "d64"):
         w = W.make(name)
         for alpha in w["alphas_ppm"]:
-            step = Step(w, device)
-            step.alpha = alpha
-            for _ in range(3):
-                step.run()
-            torch.cuda.synchronize()
-            step.check()
-            side = torch.cuda.Stream()
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
-                step.run()
-            torch.cuda.synchronize()
-            ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
-            for i in range(steps):
-                flush.zero_()
-                ev[i][3].record()
-                graph.replay()
-                ev[i][4].record()
-            torch.cuda.synchronize()
-            step_ms = float(np.mean([e[3].elapsed_time(e[4]) for e in ev]))
-            for i in range(steps):
-                flush.zero_()
-                ev[i][3].record()
-                step.run(ev=ev[i])
-                ev[i][4].record()
-            torch.cuda.synchronize()
-            step.check()
-            call_ms = {"calibrate": [e[3].elapsed_time(e[0]) for e in ev],
-                       "occupancy": [e[0].elapsed_time(e[1]) for e in ev],
-                       "dispatch": [e[1].elapsed_time(e[2]) for e in ev],
-                       "order": [e[2].elapsed_time(e[4]) for e in ev]}
-            alg = algorithmic_bytes(w)
-            calls = {}
-            for c in alg:
-                us = float(np.mean(call_ms[c])) * 1e3
-                calls[c] = {"us": us, "algorithmic_bytes": alg[c],
-                            "frac_of_measured_hbm": alg[c] / (us / 1e6) / 1e9 / peaks["hbm_gbs"]}
             key = name if len(w["alphas_ppm"]) == 1 else f"{name}_alpha{alpha / 1e6:g}"
-            out[key] = {"workload": W.DESCRIPTIONS[name], "alpha_ppm": alpha,
-                        "D": w["D"], "H": w["H"], "residents": w["R"], "candidates": w["J"],
-                        "ms_per_step": step_ms, "decisions_per_s": w["J"] / (step_ms / 1e3),
-                        "occupancy_cells_per_s": w["D"] * w["H"] / (step_ms / 1e3),
-                        "calls": calls, "steps": steps,
-                        "timing": "graph replay per step after a 256 MiB L2 flush; calls split "
-                                  "by events between direct launches"}
-            del step, graph
+            out[key] = dict(workload=W.DESCRIPTIONS[name],
+                            **time_workload(w, alpha, device, flush, steps))
+    for seed in (1, 2):
+        w = W.make(WORKLOAD, seed=seed)
+        out[f"{WORKLOAD}_seed{seed}"] = dict(workload=W.DESCRIPTIONS[WORKLOAD] + f", seed {seed}",
+                                             **time_workload(w, w["alphas_ppm"][0], device,
+                                                             flush, steps))
     return out
 
 

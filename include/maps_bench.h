@@ -34,6 +34,18 @@ int maps_set_dispatch_events(void *before, void *after);
  * MAPS_E_CUDA. */
 int maps_test_withhold_lookback(int32_t tile, uint32_t spin_limit);
 
+/* Exercises the bounded grid barriers of maps_order_local's finishing kernel
+ * (the cooperative kernel that ranks or merges the long queues, or runs the
+ * global form's passes): on the current device, later calls make block
+ * `block` of that kernel return at once, so the other blocks' first barrier
+ * waits until the limit maps_test_withhold_lookback sets (0 there: the
+ * library default), records MAPS_E_TIMEOUT and ends each block without
+ * another write.  The order of that call is wrong; what it wrote before the
+ * barrier stays inside its outputs and workspace.  block = -1 restores the
+ * normal behaviour.  Calls in flight must have finished before the setting
+ * changes.  Returns MAPS_OK or MAPS_E_CUDA. */
+int maps_test_absent_block(int32_t block);
+
 #ifdef __cplusplus
 }
 #endif

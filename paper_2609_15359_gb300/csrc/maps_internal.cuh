@@ -53,6 +53,57 @@ __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long
 __device__ __forceinline__ void st_release_u64(unsigned long long *p, unsigned long long v) {
   asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t *p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_u32(uint32_t *p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// A grid-wide barrier with a bounded wait, for kernels launched cooperatively
+// (every block resident).  The words start at zero.  A block arrives with an
+// acquire-release add (the block barrier before it orders every thread's
+// writes before the release); the last to arrive resets the count and
+// publishes the next generation with a release store; the others poll the
+// generation with acquire loads.  After spin_limit polls a block records
+// MAPS_E_TIMEOUT and the barrier returns false: the caller then returns at
+// once, writing nothing more, so the kernel ends rather than hangs and no
+// block works on data the barrier did not order.
+struct GridBar {
+  uint32_t arrived;
+  uint32_t gen;
+};
+__device__ __forceinline__ uint32_t atom_add_acq_rel_u32(uint32_t *p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+__device__ __forceinline__ bool grid_barrier(GridBar *b, int32_t *status, uint32_t spin_limit) {
+  __shared__ int s_ok;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    const uint32_t g = ld_acquire_u32(&b->gen);
+    if (atom_add_acq_rel_u32(&b->arrived, 1u) == gridDim.x - 1) {
+      b->arrived = 0u;  // before the release below; nobody arrives until it
+      st_release_u32(&b->gen, g + 1u);
+    } else {
+      uint32_t spins = 0;
+      while (ld_acquire_u32(&b->gen) == g) {
+        if (++spins > spin_limit) {
+          atomicCAS(status, 0, MAPS_E_TIMEOUT);
+          ok = 0;
+          break;
+        }
+      }
+    }
+    s_ok = ok;
+  }
+  __syncthreads();
+  return s_ok != 0;
+}
 
 // Programmatic dependent launch.  Every kernel of the library is launched
 // with programmatic stream serialisation and starts with pdl_prologue():

@@ -28,14 +28,11 @@
 // walks back over packed flag-and-count words until it meets an inclusive
 // prefix), and writes out bin by bin.  Kernels of the form not taken return
 // at once, so the host never waits on the device.
-#include <cooperative_groups.h>
-
 #include "maps_internal.cuh"
 #include "maps_bench.h"
 
 #include <algorithm>
 
-namespace cg = cooperative_groups;
 
 namespace maps {
 namespace {
@@ -58,6 +55,10 @@ enum : int32_t { kBufA = 0, kBufB = 1, kHiIdentity = 2, kPermOut = 2 };
 // look-back wait makes before it gives up.
 __device__ int32_t g_withheld_tile = -1;
 __device__ uint32_t g_lookback_spins = kSpinLimit;
+// Test aid (maps_test_absent_block): a block of the finishing kernel that
+// returns at once, so that the others' grid barrier runs out (-1: none).  The
+// barrier waits also give up after g_lookback_spins polls.
+__device__ int32_t g_absent_block = -1;
 
 struct OrderCounts {
   uint32_t h[kPasses][kRadix];
@@ -1343,7 +1344,7 @@ __device__ void merge_level(int level, int ntiles, const int64_t *mt_off, const 
 // key to its place.  Runs are the segment sort's sorted chunks in keys.
 __device__ void pair_rank_all(int64_t N, const OrderCounts *counts, const PairQueues &pq,
                               const unsigned long long *keys, int32_t *perm,
-                              unsigned long long *sB, cg::grid_group &grid) {
+                              unsigned long long *sB, GridBar *bar, int32_t *status) {
   const int nq = static_cast<int>(counts->npairq);
   const int64_t npairs = min(static_cast<int64_t>(counts->npairs), pq.budget);
   // (1) pair p = (queue q, runs A != B): for each key of A, the keys of B below it
@@ -1378,7 +1379,7 @@ __device__ void pair_rank_all(int64_t N, const OrderCounts *counts, const PairQu
     }
     __syncthreads();  // sB serves the next pair
   }
-  grid.sync();
+  if (!grid_barrier(bar, status, g_lookback_spins)) return;
   // (2) each key's place: its place in its run plus its counts in the others
   const unsigned long long imask = (1ull << index_bits(N)) - 1;
   const int64_t gstride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -1401,13 +1402,14 @@ __device__ void pair_rank_all(int64_t N, const OrderCounts *counts, const PairQu
 
 __device__ void merge_all(int64_t N, const OrderCounts *counts, const int64_t *mt_off,
                           const int32_t *mt_n, const int32_t *mt_t, unsigned long long *bufA,
-                          unsigned long long *bufB, int32_t *perm, cg::grid_group &grid) {
+                          unsigned long long *bufB, int32_t *perm, GridBar *bar,
+                          int32_t *status) {
   const int ntiles = static_cast<int>(counts->nmtiles);
   const int levels = static_cast<int>(counts->max_levels);
   const unsigned long long imask = (1ull << index_bits(N)) - 1;
   for (int level = 0; level < levels; ++level) {
     merge_level(level, ntiles, mt_off, mt_n, mt_t, bufA, bufB, perm, imask);
-    if (level + 1 < levels) grid.sync();
+    if (level + 1 < levels && !grid_barrier(bar, status, g_lookback_spins)) return;
   }
 }
 
@@ -1600,16 +1602,18 @@ order_finish_kernel(int n_hi, int64_t N, int D, int dbits, const OrderCounts *co
                     const int64_t *mt_off, const int32_t *mt_n, const int32_t *mt_t,
                     PairQueues pq, unsigned long long *keyA, unsigned long long *keyB, uint32_t *valA,
                     uint32_t *valB, const unsigned long long *hi_orig, int32_t *perm,
-                    unsigned long long *state, int64_t tiles, uint32_t *tickets, int32_t *status) {
+                    unsigned long long *state, int64_t tiles, uint32_t *tickets, GridBar *bar,
+                    int32_t *status) {
   pdl_prologue();
-  cg::grid_group grid = cg::this_grid();
-  // every block takes the same branches, so no block waits at a barrier alone
+  if (static_cast<int>(blockIdx.x) == g_absent_block) return;  // test aid, normally -1
+  // every block takes the same branches, so no block waits at a barrier alone;
+  // a barrier that ran out (MAPS_E_TIMEOUT) ends the block at once
   if (*reinterpret_cast<const volatile uint32_t *>(&counts->segmented)) {
     if (counts->npairq > 0) {
       extern __shared__ __align__(16) unsigned char pair_raw[];
-      pair_rank_all(N, counts, pq, keyA, perm, reinterpret_cast<unsigned long long *>(pair_raw), grid);
+      pair_rank_all(N, counts, pq, keyA, perm, reinterpret_cast<unsigned long long *>(pair_raw), bar, status);
     }
-    if (counts->nmtiles > 0) merge_all(N, counts, mt_off, mt_n, mt_t, keyA, keyB, perm, grid);
+    if (counts->nmtiles > 0) merge_all(N, counts, mt_off, mt_n, mt_t, keyA, keyB, perm, bar, status);
     return;
   }
   if (blockIdx.x == 0) plan_block(N, D, dbits, counts, plan, dec_count, seg_off);
@@ -1618,7 +1622,7 @@ order_finish_kernel(int n_hi, int64_t N, int D, int dbits, const OrderCounts *co
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < tiles * kRadix;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x)
     state[i] = 0ull;
-  grid.sync();
+  if (!grid_barrier(bar, status, g_lookback_spins)) return;
   const int npasses = plan->npasses;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PassSmem &sm = *reinterpret_cast<PassSmem *>(smem_raw);
@@ -1632,12 +1636,12 @@ order_finish_kernel(int n_hi, int64_t N, int D, int dbits, const OrderCounts *co
       while (order_pass_body<false>(p, N, plan, keyA, keyB, valA, valB, hi_orig, perm, state,
                                     tiles, tickets + p, status, sm)) {
       }
-    grid.sync();
+    return grid_barrier(bar, status, g_lookback_spins);
   };
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   const int64_t first = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   for (int p = 0; p < kLoPasses; ++p)
-    if (plan->active[p]) run_pass(p);
+    if (plan->active[p] && !run_pass(p)) return;
   const int gb = plan->gather_buf;
   if (gb >= 0) {  // after arrival passes the keys follow the arrival order
     unsigned long long *k = gb == kBufA ? keyA : keyB;
@@ -1649,10 +1653,10 @@ order_finish_kernel(int n_hi, int64_t N, int D, int dbits, const OrderCounts *co
       else
         reinterpret_cast<uint32_t *>(k)[i] = static_cast<uint32_t>(x);
     }
-    grid.sync();
+    if (!grid_barrier(bar, status, g_lookback_spins)) return;
   }
   for (int p = kLoPasses; p < kLoPasses + n_hi; ++p)
-    if (plan->active[p]) run_pass(p);
+    if (plan->active[p] && !run_pass(p)) return;
   if (npasses == 0)
     for (int64_t i = first; i < N; i += stride) perm[i] = static_cast<int32_t>(i);
 }
@@ -1676,6 +1680,7 @@ struct OrderWs {
   uint32_t *dec_count;
   uint32_t *dec_cursor;  // segmented form: slots taken per decoder
   uint32_t *tickets;
+  GridBar *bar;  // the finishing kernel's grid barrier
   unsigned long long *state;  // [2][tiles][256] look-back words (buffer 0 zeroed by the finishing kernel)
   size_t zero_bytes;  // counts .. tickets are contiguous and zeroed per call
   OrderPlan *plan;
@@ -1708,6 +1713,7 @@ OrderWs carve_order(Carve &c, int64_t N, int D) {
   w.grp = c.take<uint32_t>(D <= kStableD ? static_cast<size_t>((w.blocks + kGroupBlocks - 1) / kGroupBlocks) * w.Dp
                                          : 1);
   w.tickets = c.take<uint32_t>(kPasses);
+  w.bar = c.take<GridBar>(1);
   w.zero_bytes = c.off - zero_begin;
   w.state = c.take<unsigned long long>(static_cast<size_t>(2) * tiles * kRadix);
   w.plan = c.take<OrderPlan>(1);
@@ -1845,7 +1851,7 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   MAPS_TRY(launch_coop(order_finish_kernel, std::min<int64_t>(tiles, finish_grid(smem)),
                        kPassThreads, smem, s, n_hi, N, D, dbits, w.counts, w.plan, w.dec_count,
                        seg_off_out, w.mt_off, w.mt_n, w.mt_t, w.pq, w.keyA, w.keyB, w.valA, w.valB,
-                       w.hi_orig, perm_out, w.state, tiles, w.tickets, status));
+                       w.hi_orig, perm_out, w.state, tiles, w.tickets, w.bar, status));
   return launch_ok();
 }
 
@@ -1907,6 +1913,12 @@ extern "C" int maps_order_local_static(int64_t N, int32_t D, const int32_t *dec,
     *status_host = maps_check(ws, stream);
     return *status_host;
   }
+  return MAPS_OK;
+}
+
+extern "C" int maps_test_absent_block(int32_t block) {
+  using namespace maps;
+  MAPS_TRY(cuda_ok(cudaMemcpyToSymbol(g_absent_block, &block, sizeof(block))));
   return MAPS_OK;
 }
 
