@@ -492,7 +492,14 @@ def test_dispatch_errors(M, ws, oracle):
                                                 # a queue of 22 chunks: five merge levels
                                                 (100000, 1, True),
                                                 # more decoders than the stable scatter takes
-                                                (60000, 1500, True)])
+                                                (60000, 1500, True),
+                                                # the bucketing pass at its decoder limit, and
+                                                # with a count not a multiple of four
+                                                (200000, 1024, True), (200000, 1023, False),
+                                                # past 304 x 4,096 entries the bucketing blocks
+                                                # take several rounds (loads issued twice);
+                                                # arrival out of order: the global key pass
+                                                (1500000, 256, True), (1500000, 1024, False)])
 def test_order_random(M, ws, oracle, N, D, sorted_arrival):
     rng = np.random.default_rng(N + D)
     dec = rng.integers(0, D, N).astype(np.int32)
@@ -508,6 +515,24 @@ def test_order_random(M, ws, oracle, N, D, sorted_arrival):
     assert st == sto == 0
     assert np.array_equal(perm, po)
     assert np.array_equal(seg, so)
+
+
+def test_order_bucketing_rounds_range_error(M, ws, oracle):
+    """An entry outside the decoder domain in a call whose bucketing blocks
+    take several rounds: counted and placed at decoder 0 in both of its
+    passes, reported as MAPS_E_RANGE, every write inside the outputs."""
+    rng = np.random.default_rng(5)
+    N, D = 1300000, 64
+    dec = rng.integers(0, D, N).astype(np.int32)
+    dec[777777] = -3
+    dec[1299999] = D + 5
+    U = rng.integers(0, 5000, N).astype(np.int32)
+    wait = rng.integers(0, 3000, N).astype(np.int32)
+    arr = np.arange(N, dtype=np.int32)
+    assert oracle.order_local(D, dec, U, wait, arr, 1000)[0] == -2
+    st, perm, seg = gpu_order(M, ws, D, dec, U, wait, arr, 1000)
+    assert st == M.MAPS_E_RANGE
+    assert perm.min() >= -1 and perm.max() < N
 
 
 @pytest.mark.parametrize("N,D,blo,bhi,skew", [
