@@ -618,7 +618,7 @@ __device__ __forceinline__ unsigned long long dispatch_key(long long h, int q, i
 size_t stream_dispatch_smem(int D, int nact, int nb) {
   const size_t pool = static_cast<size_t>(nact) + static_cast<size_t>(D) * nb;
   return 16 * pool + 8 * static_cast<size_t>(nact) + 16 * static_cast<size_t>(D) +
-         8 * static_cast<size_t>(nb) + 64;
+         12 * static_cast<size_t>(nb) + 64;
 }
 
 // A decoder's tables from its sorted pairs (one warp): SS[i] = sum of b over
@@ -689,7 +689,8 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
   int32_t *uB = uE + nact;
   int32_t *s_base = uB + nact, *s_n = s_base + D, *s_q = s_n + D, *s_cap = s_q + D;
   int32_t *s_cp = s_cap + D, *s_cu = s_cp + nb;            // [nb] the batch
-  __shared__ int s_bad;
+  int32_t *s_ch = s_cu + nb;                               // [nb] choices (fast path)
+  __shared__ int s_bad, s_fast;
   if (tid == 0) s_bad = 0;
   __syncthreads();
   for (int k = tid; k < D; k += kSt) {
@@ -744,13 +745,74 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
   }
   __syncthreads();
   if (tid == 0 && s_bad) flag_error(status, MAPS_E_RANGE);
+  // Without a headroom output and with the Q-first rule, a decoder whose
+  // peak bound max(PM[n - 1], SS[0] + (u - 1)(n + 1)) >= M already fits is
+  // decided by (Q, index) alone: no search (M <= that bound, as
+  // PM[c - 1] <= PM[n - 1], SS[c] <= SS[0] and n - c + 1 <= n + 1).  Its
+  // position in the list is then found when the reservation is inserted.
+  const bool quick = headroom == nullptr && mc == 0;
+  // Fast path (at most 32 decoders, no headroom output, Q-first rule): take
+  // each candidate's choice by (Q, index) alone while checking that every
+  // decoder is feasible at that step.  Decoder k's peak for a candidate of
+  // horizon u, after the batch's earlier reservations on k, is at most
+  //   max(PM[n - 1], SS[0] + (u - 1)(n + 1)) (u - 1 when k has no pairs)
+  //   + the sum of p + u over those reservations
+  // (each adds p + t + 1 for t < u).  While p + 1 + that bound <= cap for
+  // every decoder, every decoder is feasible, so the rule picks the smallest
+  // (Q, index), which is the choice taken: the decisions are the walk's.  At
+  // the first step where some decoder might not fit, the fast path stops and
+  // the walk decides the whole batch (Q is written only on success).
+  if (tid == 0) s_fast = 0;
+  __syncthreads();
+  if (quick && D <= 32 && warp == 0) {
+    const int k = lane;
+    const bool has = k < D;
+    const int n = has ? s_n[k] : 0, base = has ? s_base[k] : 0;
+    const long long pm = has && n > 0 ? static_cast<long long>(PM[base + n - 1]) : 0;
+    const long long ss0 = has && n > 0 ? static_cast<long long>(SS[base]) : 0;
+    const long long cap = has ? s_cap[k] : 0;
+    int q = has ? s_q[k] : 0;
+    long long add = 0;
+    bool fits = true;
+    for (int j = 0; j < nb; ++j) {
+      const int32_t p = s_cp[j], U = s_cu[j];
+      // (an invalid candidate, or Q past 21 bits: the walk handles it)
+      if ((p | U) < 0 || __any_sync(0xffffffffu, has && q >= (1 << 21))) {
+        fits = false;
+        break;
+      }
+      const int u = U < 1 ? 1 : (U > H ? H : U);
+      const long long b0 = n > 0 ? max(pm, ss0 + static_cast<long long>(u - 1) * (n + 1))
+                                 : static_cast<long long>(u - 1);
+      if (!__all_sync(0xffffffffu, !has || static_cast<long long>(p) + 1 + b0 + add <= cap)) {
+        fits = false;
+        break;
+      }
+      const uint32_t key = has ? (static_cast<uint32_t>(q) << 10) | static_cast<uint32_t>(k) : 0xffffffffu;
+      const int bk = static_cast<int>(__reduce_min_sync(0xffffffffu, key) & 1023u);
+      if (lane == 0) s_ch[j] = bk;
+      if (lane == bk) {
+        q += 1;
+        add += static_cast<long long>(p) + u;
+      }
+    }
+    if (fits) {
+      __syncwarp();
+      for (int j = lane; j < nb; j += 32) choice[j] = s_ch[j];
+      if (has) s_q[k] = q;
+    }
+    if (lane == 0) s_fast = fits ? 1 : 0;
+  }
+  __syncthreads();
 
   // The walk: one warp, no block barrier.  Lane l scores decoders l, l + 32,
   // ...: a binary search over the decoder's sorted ends gives c (the pairs with
   // e <= u), then M = max(PM[c - 1], SS[c] + (u - 1)(n - c + 1)); a packed key
   // picks (feasible first, then Q or the largest headroom, then the lowest
   // index); the warp inserts the footprint and rebuilds that decoder's tables.
-  if (D <= 32) {
+  if (s_fast) {
+    // decided by the fast path
+  } else if (D <= 32) {
     // Two warps, one decoder per lane.  Warp 0 holds each decoder's list
     // length, base, Q and capacity in registers, scores the candidates, picks
     // and books each decision and hands it to warp 1 through shared memory
@@ -801,6 +863,17 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
       auto score = [&](int32_t pp, int uu) {
         key = ~0ull;
         if (!has) return;
+        if (quick && n_r > 0) {
+          const long long mub = max(static_cast<long long>(PM[base_r + n_r - 1]),
+                                    static_cast<long long>(SS[base_r]) +
+                                        static_cast<long long>(uu - 1) * (n_r + 1));
+          if (static_cast<long long>(pp) + 1 + mub <= cap_r) {
+            key = (static_cast<unsigned long long>(q_r) << 10) | static_cast<unsigned>(k);
+            c = -1;   // found at insertion
+            M = mub;  // bounds every new cell: no range error (cap <= INT32_MAX)
+            return;
+          }
+        }
         c = count_le(E + base_r, n_r, uu);
         const long long full = c > 0 ? static_cast<long long>(PM[base_r + c - 1]) : LLONG_MIN;
         const long long part = static_cast<long long>(c < n_r ? SS[base_r + c] : 0u) +
@@ -875,9 +948,16 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
         named_bar(1, 64);
         const int bk = h_bk;
         if (bk >= 0) {
-          const int pos = h_pos, n = h_n, base = h_base, m = n + 1;
+          const int n = h_n, base = h_base, m = n + 1;
           const int32_t p = s_cp[j];
           const int u = clampu(s_cu[j]);
+          int pos = h_pos;  // -1: the scoring took the bound, count the pairs with e <= u here
+          if (pos < 0) {
+            if (n < 32)
+              pos = __popc(__ballot_sync(0xffffffffu, lane < n && E[base + lane] <= u));
+            else
+              pos = count_le(E + base, n, u);
+          }
           const bool nxt = j + 1 < nb;
           const int32_t p1 = nxt ? s_cp[j + 1] : 0, U1 = nxt ? s_cu[j + 1] : 0;
           const bool ok1 = nxt && (p1 | U1) >= 0;
@@ -972,6 +1052,21 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
       int bc = 0;
       for (int k = lane; k < D; k += 32) {
         const int n = s_n[k], base = s_base[k];
+        if (quick && n > 0) {  // a sure fit is decided by (Q, index) alone
+          const long long mub = max(static_cast<long long>(PM[base + n - 1]),
+                                    static_cast<long long>(SS[base]) +
+                                        static_cast<long long>(u - 1) * (n + 1));
+          if (static_cast<long long>(p) + 1 + mub <= s_cap[k]) {
+            const unsigned long long kk = (static_cast<unsigned long long>(s_q[k]) << 10) |
+                                          static_cast<unsigned>(k);
+            if (kk < key) {
+              key = kk;
+              bM = mub;
+              bc = -1;
+            }
+            continue;
+          }
+        }
         int lo = 0, hi = n;  // c = the pairs with e <= u
         while (lo < hi) {
           const int mid = (lo + hi) >> 1;
@@ -1014,8 +1109,19 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
       }
       // the winner's lane (decoder bk is lane bk % 32's) hands over M and c
       const long long Mb = __shfl_sync(0xffffffffu, bM, bk & 31);
-      const int pos = __shfl_sync(0xffffffffu, bc, bk & 31);
+      int pos = __shfl_sync(0xffffffffu, bc, bk & 31);
       const int n = s_n[bk], base = s_base[bk];
+      if (pos < 0) {  // the bound decided it: the pairs with e <= u place the new one
+        int lo = 0, hi = n;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (E[base + mid] <= u)
+            lo = mid + 1;
+          else
+            hi = mid;
+        }
+        pos = lo;
+      }
       if (lane == 0) {
         choice[j] = bk;
         if (headroom) headroom[j] = static_cast<long long>(s_cap[bk]) - (static_cast<long long>(p) + 1 + Mb);
@@ -1472,7 +1578,7 @@ int maps_stream_run(const maps_stream_cfg *cfg, const int64_t *arrival_ms, const
                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               static_cast<int>(dsm))));
         launch_pdl(stream_dispatch_kernel, 1, kSt, dsm, s, D, c.H, nc, mc, w.res_off, w.rp, w.rg,
-                   w.rU, w.capv, w.Q, cpr, w.Uq + nact, cch, w.headroom, status);
+                   w.rU, w.capv, w.Q, cpr, w.Uq + nact, cch, nullptr, status);  // no headroom out
         MAPS_TRY(launch_ok());
       } else {
         MAPS_TRY(maps_project_occupancy(D, c.H, w.res_off, nact, w.rp, w.rg, w.rU, w.K, nullptr, ws,
