@@ -772,29 +772,30 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
     const long long ss0 = has && n > 0 ? static_cast<long long>(SS[base]) : 0;
     const long long cap = has ? s_cap[k] : 0;
     int q = has ? s_q[k] : 0;
+    // checked once: every candidate valid, and every Q stays within 21 bits
+    // (a Q grows by at most nb); otherwise the walk handles the batch
+    bool invalid = has && static_cast<long long>(q) + nb >= (1 << 21);
+    for (int j = lane; j < nb; j += 32) invalid |= (s_cp[j] | s_cu[j]) < 0;
+    bool fits = !__any_sync(0xffffffffu, invalid);
     long long add = 0;
-    bool fits = true;
-    for (int j = 0; j < nb; ++j) {
-      const int32_t p = s_cp[j], U = s_cu[j];
-      // (an invalid candidate, or Q past 21 bits: the walk handles it)
-      if ((p | U) < 0 || __any_sync(0xffffffffu, has && q >= (1 << 21))) {
-        fits = false;
-        break;
+    bool miss = false;  // some step where this lane's decoder might not fit
+    for (int j0 = 0; j0 < nb && fits; j0 += 32) {
+      const int j1 = min(nb, j0 + 32);
+      for (int j = j0; j < j1; ++j) {
+        const int32_t p = s_cp[j], U = s_cu[j];
+        const int u = U < 1 ? 1 : (U > H ? H : U);
+        const long long b0 = n > 0 ? max(pm, ss0 + static_cast<long long>(u - 1) * (n + 1))
+                                   : static_cast<long long>(u - 1);
+        miss |= has && static_cast<long long>(p) + 1 + b0 + add > cap;
+        const uint32_t key = has ? (static_cast<uint32_t>(q) << 10) | static_cast<uint32_t>(k) : 0xffffffffu;
+        const int bk = static_cast<int>(__reduce_min_sync(0xffffffffu, key) & 1023u);
+        if (lane == 0) s_ch[j] = bk;
+        if (lane == bk) {
+          q += 1;
+          add += static_cast<long long>(p) + u;
+        }
       }
-      const int u = U < 1 ? 1 : (U > H ? H : U);
-      const long long b0 = n > 0 ? max(pm, ss0 + static_cast<long long>(u - 1) * (n + 1))
-                                 : static_cast<long long>(u - 1);
-      if (!__all_sync(0xffffffffu, !has || static_cast<long long>(p) + 1 + b0 + add <= cap)) {
-        fits = false;
-        break;
-      }
-      const uint32_t key = has ? (static_cast<uint32_t>(q) << 10) | static_cast<uint32_t>(k) : 0xffffffffu;
-      const int bk = static_cast<int>(__reduce_min_sync(0xffffffffu, key) & 1023u);
-      if (lane == 0) s_ch[j] = bk;
-      if (lane == bk) {
-        q += 1;
-        add += static_cast<long long>(p) + u;
-      }
+      fits = !__any_sync(0xffffffffu, miss);  // a miss anywhere: the walk decides the batch
     }
     if (fits) {
       __syncwarp();
