@@ -691,7 +691,10 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
   int32_t *s_cp = s_cap + D, *s_cu = s_cp + nb;            // [nb] the batch
   int32_t *s_ch = s_cu + nb;                               // [nb] choices (fast path)
   __shared__ int s_bad, s_fast;
-  if (tid == 0) s_bad = 0;
+  if (tid == 0) {
+    s_bad = 0;
+    s_fast = 0;
+  }
   __syncthreads();
   for (int k = tid; k < D; k += kSt) {
     const int lo = static_cast<int>(res_off[k]);
@@ -721,60 +724,41 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
     uB[x] = b;
   }
   __syncthreads();
-  // sort each decoder's pairs by e (rank among the decoder's pairs, ties by
-  // position), and check sum b <= INT32_MAX (K at step 0)
-  for (int k = warp; k < D; k += kSt / 32) {
-    const int lo = s_base[k] - k * nb, n = s_n[k], base = s_base[k];
-    long long sb = 0;
-    for (int i = lane; i < n; i += 32) {
-      const int ei = uE[lo + i];
-      int r = 0;
-      for (int j2 = 0; j2 < n; ++j2) {
-        const int ej = uE[lo + j2];
-        r += ej < ei || (ej == ei && j2 < i);
-      }
-      E[base + r] = ei;
-      Bv[base + r] = uB[lo + i];
-      sb += uB[lo + i];
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) sb += __shfl_xor_sync(0xffffffffu, sb, off);
-    if (lane == 0 && sb > 0x7fffffffLL) s_bad = 1;
-    __syncwarp();  // the sorted pairs are written
-    if (rebuild_tables(E + base, Bv + base, SS + base, PM + base, n) && lane == 0) s_bad = 1;
-  }
-  __syncthreads();
-  if (tid == 0 && s_bad) flag_error(status, MAPS_E_RANGE);
-  // Without a headroom output and with the Q-first rule, a decoder whose
-  // peak bound max(PM[n - 1], SS[0] + (u - 1)(n + 1)) >= M already fits is
-  // decided by (Q, index) alone: no search (M <= that bound, as
-  // PM[c - 1] <= PM[n - 1], SS[c] <= SS[0] and n - c + 1 <= n + 1).  Its
-  // position in the list is then found when the reservation is inserted.
+  // Without a headroom output and with the Q-first rule, a decoder whose peak
+  // is provably within its capacity is decided by (Q, index) alone.
   const bool quick = headroom == nullptr && mc == 0;
   // Fast path (at most 32 decoders, no headroom output, Q-first rule): take
   // each candidate's choice by (Q, index) alone while checking that every
-  // decoder is feasible at that step.  Decoder k's peak for a candidate of
-  // horizon u, after the batch's earlier reservations on k, is at most
-  //   max(PM[n - 1], SS[0] + (u - 1)(n + 1)) (u - 1 when k has no pairs)
+  // decoder is feasible at that step, before any list is sorted.  For t < u,
+  // K(t) + t = S(t) + t (C(t) + 1) with S <= the decoder's b-sum and C <= n
+  // while t < e_max, and K(t) + t = t after e_max, so decoder k's peak for a
+  // candidate of horizon u, after the batch's earlier reservations on k, is
+  // at most
+  //   max(b-sum + (min(u, e_max) - 1)(n + 1), u - 1)
   //   + the sum of p + u over those reservations
   // (each adds p + t + 1 for t < u).  While p + 1 + that bound <= cap for
   // every decoder, every decoder is feasible, so the rule picks the smallest
-  // (Q, index), which is the choice taken: the decisions are the walk's.  At
-  // the first step where some decoder might not fit, the fast path stops and
-  // the walk decides the whole batch (Q is written only on success).
-  if (tid == 0) s_fast = 0;
-  __syncthreads();
+  // (Q, index), which is the choice taken: the decisions are the walk's, and
+  // the lists need no sorting.  A step where some decoder might not fit sends
+  // the whole batch to the walk (Q is written only on success).
   if (quick && D <= 32 && warp == 0) {
     const int k = lane;
     const bool has = k < D;
-    const int n = has ? s_n[k] : 0, base = has ? s_base[k] : 0;
-    const long long pm = has && n > 0 ? static_cast<long long>(PM[base + n - 1]) : 0;
-    const long long ss0 = has && n > 0 ? static_cast<long long>(SS[base]) : 0;
+    const int n = has ? s_n[k] : 0, lo = has ? s_base[k] - k * nb : 0;
+    long long sb = 0;  // this decoder's b-sum and largest end step
+    int em = 1;
+    for (int i = 0; i < n; ++i) {
+      sb += uB[lo + i];
+      em = max(em, uE[lo + i]);
+    }
     const long long cap = has ? s_cap[k] : 0;
     int q = has ? s_q[k] : 0;
-    // checked once: every candidate valid, and every Q stays within 21 bits
-    // (a Q grows by at most nb); otherwise the walk handles the batch
-    bool invalid = has && static_cast<long long>(q) + nb >= (1 << 21);
+    // checked once: every candidate valid, every Q stays within 21 bits (a Q
+    // grows by at most nb), and no K of the residents reaches INT32_MAX (so
+    // the tables' range checks could not fire); otherwise the walk handles
+    // the batch
+    bool invalid = has && (static_cast<long long>(q) + nb >= (1 << 21) ||
+                           sb + static_cast<long long>(em - 1) * (n + 1) > 0x7fffffffLL);
     for (int j = lane; j < nb; j += 32) invalid |= (s_cp[j] | s_cu[j]) < 0;
     bool fits = !__any_sync(0xffffffffu, invalid);
     long long add = 0;
@@ -784,8 +768,8 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
       for (int j = j0; j < j1; ++j) {
         const int32_t p = s_cp[j], U = s_cu[j];
         const int u = U < 1 ? 1 : (U > H ? H : U);
-        const long long b0 = n > 0 ? max(pm, ss0 + static_cast<long long>(u - 1) * (n + 1))
-                                   : static_cast<long long>(u - 1);
+        const long long b0 = max(sb + static_cast<long long>(min(u, em) - 1) * (n + 1),
+                                 static_cast<long long>(u - 1));
         miss |= has && static_cast<long long>(p) + 1 + b0 + add > cap;
         const uint32_t key = has ? (static_cast<uint32_t>(q) << 10) | static_cast<uint32_t>(k) : 0xffffffffu;
         const int bk = static_cast<int>(__reduce_min_sync(0xffffffffu, key) & 1023u);
@@ -805,6 +789,33 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
     if (lane == 0) s_fast = fits ? 1 : 0;
   }
   __syncthreads();
+
+  if (!s_fast) {
+    // sort each decoder's pairs by e (rank among the decoder's pairs, ties by
+    // position), and check sum b <= INT32_MAX (K at step 0)
+    for (int k = warp; k < D; k += kSt / 32) {
+      const int lo = s_base[k] - k * nb, n = s_n[k], base = s_base[k];
+      long long sb = 0;
+      for (int i = lane; i < n; i += 32) {
+        const int ei = uE[lo + i];
+        int r = 0;
+        for (int j2 = 0; j2 < n; ++j2) {
+          const int ej = uE[lo + j2];
+          r += ej < ei || (ej == ei && j2 < i);
+        }
+        E[base + r] = ei;
+        Bv[base + r] = uB[lo + i];
+        sb += uB[lo + i];
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) sb += __shfl_xor_sync(0xffffffffu, sb, off);
+      if (lane == 0 && sb > 0x7fffffffLL) s_bad = 1;
+      __syncwarp();  // the sorted pairs are written
+      if (rebuild_tables(E + base, Bv + base, SS + base, PM + base, n) && lane == 0) s_bad = 1;
+    }
+    __syncthreads();
+  }
+  if (tid == 0 && s_bad) flag_error(status, MAPS_E_RANGE);
 
   // The walk: one warp, no block barrier.  Lane l scores decoders l, l + 32,
   // ...: a binary search over the decoder's sorted ends gives c (the pairs with
