@@ -197,8 +197,12 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
     const int k = base + t;
     const long long c = k < D ? __ldcg(dec_count + k) : 0;
     const int big = c > kSegMax ? 1 : 0;
+    // sort items of decoder k: its queue, or its chunks; item indices follow
+    // from a scan, in decoder order
+    const int nch = big ? static_cast<int>((c + kSegMax - 1) / kSegMax) : 0;
+    const int nit = c > 0 ? (big ? nch : 1) : 0;
     long long incl = c;
-    int bincl = big;
+    int bincl = nit;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const long long y = __shfl_up_sync(0xffffffffu, incl, off);
@@ -223,14 +227,12 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
     const int bcarry = s_bcarry;
     const long long start = carry + wb + incl - c;
     if (k <= D) seg_off[k] = start;
+    const uint32_t it = static_cast<uint32_t>(bcarry + bwb + bincl - nit);
     if (k < D && c > 0 && !big) {
-      const uint32_t it = atomicAdd(&counts->nitems, 1u);
       item_off[it] = start;
       item_n[it] = static_cast<int32_t>(c);
       item_dec[it] = k;
     } else if (k < D && big) {
-      const int nch = static_cast<int>((c + kSegMax - 1) / kSegMax);
-      const uint32_t it = atomicAdd(&counts->nitems, static_cast<uint32_t>(nch));
       for (int j = 0; j < nch; ++j) {
         item_dec[it + j] = k;
         item_off[it + j] = start + static_cast<int64_t>(j) * kSegMax;
@@ -271,8 +273,8 @@ __device__ void seg_plan_block(int D, OrderCounts *counts, const uint32_t *dec_c
   if (t == 0) {
     counts->segmented = segmented ? 1u : 0u;
     counts->stable = stable ? 1u : 0u;
+    counts->nitems = static_cast<uint32_t>(s_bcarry);
   }
-  (void)s_bcarry;
 }
 
 // Pass 1: validation, largest non-promoted bound, entries per decoder, and
