@@ -613,6 +613,11 @@ def bench_gpu(args, world, rank, local, dist):
         },
         "occupancy_cells_per_s": K * D * H * world / max_s,
         "launch": "each timed step replays one CUDA graph of the four C-ABI calls",
+        "kernels_ms_median": {"calibrate": float(np.median(cal_ms)),
+                              "occupancy": float(np.median(occ_ms)),
+                              "dispatch": float(np.median(disp_ms)),
+                              "order": float(np.median(order_ms))},
+        "calibration": calibration_report(w, int(step.q.item())),
         "kernels_ms": {"calibrate": float(np.mean(cal_ms)), "occupancy": float(np.mean(occ_ms)),
                        "dispatch": float(np.mean(disp_ms)), "order": float(np.mean(order_ms))},
         "kernels_ms_pass": {"steps": Kb, "ms_per_step": float(np.mean(split_ms)),
@@ -645,6 +650,19 @@ def bench_gpu(args, world, rank, local, dist):
 # ---------------------------------------------------------------------------
 # the smaller configurations: Tiny, D16 and D64 (each of its three bound sets)
 # ---------------------------------------------------------------------------
+
+def calibration_report(w: dict, q: int) -> dict:
+    """A synthetic analogue of the paper's underestimation table: on the
+    workload's candidates (held out from the calibration set), the share whose
+    true length exceeds the raw prediction, the prediction x 1.1, and the
+    calibrated bound pred + q from the GPU's quantile (target <= alpha)."""
+    t = w["cand_true"].astype(np.int64)
+    p = w["cand_pred"].astype(np.int64)
+    return {"alpha": w["alphas_ppm"][0] / 1e6, "q": q, "held_out": int(t.size),
+            "under_raw": float(np.mean(t > p)),
+            "under_pred_x1.1": float(np.mean(t > np.floor(1.1 * p))),
+            "under_calibrated": float(np.mean(t > p + q))}
+
 
 def time_workload(w: dict, alpha: int, device, flush, steps: int = 20) -> dict:
     """One workload's four calls: per step a CUDA-graph replay after an L2 flush
@@ -760,7 +778,18 @@ def bench_stream(device, cpu_sample: int = 0) -> dict:
     t0 = time.perf_counter()
     run(N)
     secs = time.perf_counter() - t0
+    # realised coverage: the requests whose true length is within the bound
+    # their batch was dispatched with (pred + the batch's q), over the
+    # batches with a bounded quantile
+    qh = q.cpu().numpy()
+    b_of = np.arange(N) // B
+    bounded = qh[b_of] >= 0
+    covered = w["true"][:N] <= w["pred"][:N].astype(np.int64) + np.maximum(qh[b_of], 0)
+    coverage = {"realised": float(covered[bounded].mean()) if bounded.any() else None,
+                "target": 1 - w["alpha_ppm"] / 1e6,
+                "batches_round_robin": int((qh < 0).sum())}
     out = {"workload": W.DESCRIPTIONS["stream"], "requests": N, "batches": nb,
+           "coverage": coverage,
            "value": N / secs, "unit": "decisions/s", "seconds": secs,
            "ms_per_batch": secs / nb * 1e3, "dispatch_mode": "SEQUENTIAL",
            "timing": "host wall clock of one maps_stream_run call (it synchronises per batch)"}

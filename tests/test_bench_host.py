@@ -77,3 +77,19 @@ def test_reference_arm_json_line(monkeypatch):
     assert cb["sample"] and "whole steps" in cb["sample"]
     assert r["e2e"] == {"value": r["value"], "unit": r["unit"], "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}
+
+
+def test_calibration_report_reaches_the_coverage_target(oracle):
+    """The bench's underestimation report on Large's held-out candidates, with
+    the oracle's quantile: the calibrated bound underestimates at most about
+    alpha of them (three standard errors of slack), the raw prediction far
+    more."""
+    import bench
+    from paper_2609_15359_gb300 import workloads as W
+    w = W.make("large")
+    st, q = oracle.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])
+    assert st == 0
+    r = bench.calibration_report(w, int(q))
+    a, n = r["alpha"], r["held_out"]
+    assert r["under_calibrated"] <= a + 3 * (a * (1 - a) / n) ** 0.5
+    assert r["under_raw"] > 2 * a and r["under_pred_x1.1"] > r["under_calibrated"]
