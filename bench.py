@@ -968,31 +968,32 @@ class OracleStep:
 
 
 def time_oracle(step: OracleStep, threads: int, n: int, warm: int = 1) -> tuple[float, int]:
-    """Mean seconds of n whole oracle steps on `threads` host threads (0: all
+    """Median seconds of n whole oracle steps on `threads` host threads (0: all
     cores) after `warm` untimed ones; returns (seconds, threads used)."""
     used = step.O.p_threads(threads)
     for _ in range(warm):
         step.run()
     secs = [step.run() for _ in range(n)]
-    return float(np.mean(secs)), used
+    return float(np.median(secs)), used
 
 
 def cpu_baseline(w: dict) -> dict:
     """The plain CPU oracle timed on whole steps of the same workload, on every
     host core and on one (a few steps each, about 10 s of CPU in all)."""
     step = OracleStep(w)
-    s_all, cores = time_oracle(step, 0, 8)
-    s_one, _ = time_oracle(step, 1, 3)
+    s_all, cores = time_oracle(step, 0, 5)
+    s_one, _ = time_oracle(step, 1, 5)
     step.O.p_threads(1)
     J = w["J"]
     return {"value": J / s_all, "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": ("whole steps of the Large workload through the plain (tier-P) oracle: "
                        "calibration of 1,000,000 residuals, bounds, occupancy of 256 decoders, "
                        "SNAPSHOT dispatch of all 65,536 candidates, order of 1,114,112 entries; "
-                       f"mean of 8 steps on {cores} threads"),
+                       f"median of 5 steps on {cores} threads"),
             "ms_per_step": s_all * 1e3,
             "single_thread": {"value": J / s_one, "unit": UNIT, "cores": 1,
-                              "ms_per_step": s_one * 1e3, "steps": 3},
+                              "ms_per_step": s_one * 1e3, "steps": 5,
+                              "sample": "median of 5 whole steps on one thread"},
             "host": cpu_info()}
 
 
