@@ -967,6 +967,28 @@ class OracleStep:
         return time.perf_counter() - t0
 
 
+def tier_b_step_ms(name: str) -> float:
+    """One whole step of a small workload through the by-definition (tier-B)
+    oracle, single-threaded, for information: the same four calls as the
+    GPU step (SNAPSHOT dispatch), each cell and score formed step by step."""
+    import oracle as O
+    from paper_2609_15359_gb300 import workloads as W
+    w = W.make(name)
+    R = w["R"]
+    pred = np.concatenate([w["res_pred"], w["cand_pred"]])
+    wait = np.concatenate([w["res_wait"], np.zeros(w["J"], np.int32)])
+    arr = np.arange(R + w["J"], dtype=np.int32)
+    t0 = time.perf_counter()
+    st, q = O.calibrate(w["cal_true"], w["cal_pred"], w["alphas_ppm"][0])
+    st, U = O.bound(pred, q)
+    st, K = O.occupancy(w["D"], w["H"], w["res_off"], w["res_prompt"], w["res_gen"], U[:R])
+    st, ch, _, _, _ = O.dispatch(0, w["D"], w["H"], 1, K, w["cap"], w["Q"], w["cand_prompt"],
+                                 U[R:])
+    dec = np.concatenate([w["res_dec"], ch])
+    O.order_local(w["D"], dec, U, wait, arr, w["max_wait"])
+    return (time.perf_counter() - t0) * 1e3
+
+
 def time_oracle(step: OracleStep, threads: int, n: int, warm: int = 1) -> tuple[float, int]:
     """Median seconds of n whole oracle steps on `threads` host threads (0: all
     cores) after `warm` untimed ones; returns (seconds, threads used)."""
@@ -994,6 +1016,9 @@ def cpu_baseline(w: dict) -> dict:
             "single_thread": {"value": J / s_one, "unit": UNIT, "cores": 1,
                               "ms_per_step": s_one * 1e3, "steps": 5,
                               "sample": "median of 5 whole steps on one thread"},
+            "tier_b_ms_per_step": {"tiny": tier_b_step_ms("tiny"), "d16": tier_b_step_ms("d16"),
+                                   "what": "the by-definition oracle, one step, one thread "
+                                           "(for information)"},
             "host": cpu_info()}
 
 
