@@ -76,7 +76,8 @@ TRAFFIC = {
         "8916c704cd39734b0eed9bd2314a7d66308ef2586300643c1d3512f2d6baba5d"},
 }
 KERNELS = {
-    "calibrate": "select_pass_kernel<0..2> + bound_kernel (maps_calibrate)",
+    "calibrate": "calibrate_fused_kernel (maps_calibrate: select passes and bounds in one "
+                 "cooperative launch)",
     "occupancy": "occ_bucket_kernel + occ_tile_kernel (maps_project_occupancy)",
     "dispatch": "dispatch_prep (carry scan + bin count) + bin_scatter + dispatch_snapshot_kernel (maps_dispatch)",
     "order": "order_bucket + order_segsort + order_finish (maps_order_local)",
@@ -286,11 +287,12 @@ class Step:
                    M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, self.D, self.H, J),
                    M.lib.maps_order_local_workspace_size(R + J, self.D))
         self.ws = M.Workspace(need, device)
-        # calibrate 4 (three select passes, bounds); occupancy 2 (bucket, tile);
+        # calibrate 1 (select passes and bounds, one cooperative kernel);
+        # occupancy 2 (bucket, tile);
         # dispatch 3 (carry scan with bin count, bin scatter, main); order 3
         # (bucketing, segment sort, the cooperative finishing kernel: pairwise
         # ranks or merges of the long queues, or the global radix form)
-        self.kernels_per_step = 4 + 2 + 3 + (3 if self.D <= 1024 else 4)
+        self.kernels_per_step = 1 + 2 + 3 + (3 if self.D <= 1024 else 4)
 
     def run(self, ev=None):
         M, R = self.M, self.R

@@ -223,7 +223,7 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec,
  * embedded in a host process whose device allocator belongs to another
  * framework, or one that must not allocate once it is serving.  This call
  * computes exactly what maps_order_local computes, but its scratch memory is
- * a fixed array of 3 MiB compiled into the library (every GPU that loads the
+ * a fixed array of 5 MiB compiled into the library (every GPU that loads the
  * library holds it until the process exits), so it takes no workspace and
  * allocates nothing.  The caller still provides inputs and outputs, in
  * device memory, as for maps_order_local.

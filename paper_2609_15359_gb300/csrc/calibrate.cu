@@ -11,9 +11,15 @@
 //   - each later pass histograms the next (up to) 12 bits of s - lo for the
 //     scores inside the range.
 // A range of one value is q, so a quantile below 1,024 takes one pass and any
-// quantile at most three.  The last block to finish a pass picks the bin that
-// holds rank k; passes after the range has closed return at once.  Nothing
-// returns to the host between passes.
+// quantile at most three.
+// Calibration sets above 8,192 scores take one cooperative kernel: one block
+// of 1,024 threads per multiprocessor, each thread holding up to eight scores
+// and eight of the queries' predictions in registers.  A pass adds the
+// blocks' shared histograms into a global one and waits at a bounded grid
+// barrier; every block then scans the global counts and picks the same bin,
+// so the next pass needs no other exchange.  Once the range is one value each
+// thread writes its queries' bounds U = pred + q.  Smaller sets take one block
+// (select_small_kernel).
 #include <algorithm>
 
 #include "maps_internal.cuh"
@@ -27,15 +33,12 @@ constexpr int kSelectThreads = 1024;
 constexpr uint32_t kExactBins = 1024;  // scores below this have a bin each
 constexpr int kMantBits = 7;           // bits after the leading one, first pass
 constexpr int kStepBits = 12;          // bits per later pass
+constexpr int kRegItems = 8;           // scores, and predictions, a thread keeps in registers
 
 struct SelectState {
   unsigned long long hist[kPasses][kBins];  // global bin counts per pass
-  unsigned long long k_rem;                 // rank still to find inside the range
-  uint32_t lo;                              // the range [lo, lo + 2^wlog) holding q
-  int32_t wlog;
-  uint32_t resolved;                        // set once the range is one value
-  uint32_t done[kPasses];                   // blocks finished per pass
-  int32_t q;                                // the quantile once selected
+  GridBar bar;                              // the fused kernel's grid barrier
+  int32_t q;                                // the quantile once selected (0 before)
 };
 
 __device__ __forceinline__ uint32_t score(int32_t L, int32_t P) {
@@ -51,166 +54,217 @@ __device__ __forceinline__ int first_bin(uint32_t s) {
          static_cast<int>((s >> (e - kMantBits)) & ((1u << kMantBits) - 1u));
 }
 
-template <int PASS>
-__global__ void __launch_bounds__(kSelectThreads)
-select_pass_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P,
-                   int64_t n, unsigned long long k0, SelectState *st,
-                   int32_t *q_dev_out, int32_t *status) {
-  pdl_prologue();
-  if (PASS > 0 && *reinterpret_cast<volatile uint32_t *>(&st->resolved)) return;
-  __shared__ uint32_t sh[kBins];
-  __shared__ int s_last;
-  __shared__ unsigned long long s_warp[kSelectThreads / 32];
-
-  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
-  __syncthreads();
-  // the range chosen so far and this pass's digit of s - lo
-  const uint32_t lo = PASS == 0 ? 0u : *reinterpret_cast<volatile uint32_t *>(&st->lo);
-  const int wlog = PASS == 0 ? 32 : *reinterpret_cast<volatile int32_t *>(&st->wlog);
-  const int shift = wlog > kStepBits ? wlog - kStepBits : 0;
-
-  // Histogram update.  First pass: the zero scores (about half of a length
-  // residual's scores) are counted by one ballot per warp and every other lane
-  // adds alone, since its bin is a single value or a narrow range.  Later
-  // passes aggregate the lanes of each bin with a match, as no bin of a range
-  // is known to be hot.
-  const int lane = static_cast<int>(threadIdx.x & 31);
-  auto visit = [&](uint32_t s, bool valid) {
-    if constexpr (PASS == 0) {
-      const int d = first_bin(s);
-      const unsigned zeros = __ballot_sync(0xffffffffu, valid && d == 0);
-      if (zeros && lane == __ffs(zeros) - 1) atomicAdd(&sh[0], static_cast<uint32_t>(__popc(zeros)));
-      if (valid && d > 0) atomicAdd(&sh[d], 1u);
+// Item u * 4 + c of thread t (of T in the grid) is element 4 (t + u T) + c:
+// two 128-bit words per array when both pointers allow it.
+__device__ __forceinline__ void load_items(const int32_t *__restrict__ a, int64_t cnt, int64_t t,
+                                           int64_t T, bool vec, int32_t v[kRegItems]) {
+#pragma unroll
+  for (int u = 0; u < kRegItems / 4; ++u) {
+    const int64_t i4 = t + u * T, e0 = 4 * i4;
+    if (vec && e0 + 4 <= cnt) {
+      const int4 x = __ldg(reinterpret_cast<const int4 *>(a) + i4);
+      v[4 * u] = x.x, v[4 * u + 1] = x.y, v[4 * u + 2] = x.z, v[4 * u + 3] = x.w;
     } else {
-      const uint32_t r = s - lo;  // wlog <= 24 here
-      if (s < lo || r >= (1u << wlog)) valid = false;
-      const int d = valid ? static_cast<int>(r >> shift) : -1;
-      const unsigned peers = __match_any_sync(0xffffffffu, d);
-      if (valid && lane == __ffs(peers) - 1)
-        atomicAdd(&sh[d], static_cast<uint32_t>(__popc(peers)));
+#pragma unroll
+      for (int c = 0; c < 4; ++c) v[4 * u + c] = e0 + c < cnt ? __ldg(a + e0 + c) : 0;
     }
-  };
+  }
+}
 
-  // Grid-stride loops whose bounds depend only on the block's first index,
-  // so whole warps iterate together.
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  const int64_t b0 = static_cast<int64_t>(blockIdx.x) * blockDim.x;
-  const bool vec = (reinterpret_cast<uintptr_t>(L) % 16 == 0) &&
-                   (reinterpret_cast<uintptr_t>(P) % 16 == 0);
-  int64_t tail_start = 0;
-  if (vec) {
-    const int64_t n4 = n / 4;
-    const int4 *L4 = reinterpret_cast<const int4 *>(L);
-    const int4 *P4 = reinterpret_cast<const int4 *>(P);
-    for (int64_t i0 = b0; i0 < n4; i0 += 4 * stride) {
-      int4 a[4], b[4];
-      bool ok[4];
+// The fused select and bounds (n > kSmallN).  in_regs: n <= kRegItems x the
+// grid's threads, so each thread's scores stay in registers across passes;
+// otherwise every pass reads them again.  pred_in_regs likewise for the m
+// predictions.
+__global__ void __launch_bounds__(kSelectThreads, 1)
+calibrate_fused_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P, int64_t n,
+                       unsigned long long k0, const int32_t *__restrict__ pred, int64_t m,
+                       int32_t *__restrict__ out, SelectState *st, int32_t *q_dev_out,
+                       int32_t *status, int in_regs, int pred_in_regs) {
+  pdl_prologue();
+  __shared__ uint32_t sh[kBins];
+  __shared__ unsigned long long s_warp[kSelectThreads / 32];
+  __shared__ uint32_t s_lo;
+  __shared__ int s_w;
+  __shared__ unsigned long long s_k;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t T = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + tid;
+  const bool pvec = (reinterpret_cast<uintptr_t>(pred) % 16 == 0) &&
+                    (reinterpret_cast<uintptr_t>(out) % 16 == 0);
+  const bool svec = (reinterpret_cast<uintptr_t>(L) % 16 == 0) &&
+                    (reinterpret_cast<uintptr_t>(P) % 16 == 0);
+  // the predictions do not depend on q: their loads overlap the select
+  int32_t pv[kRegItems];
+  if (pred_in_regs) load_items(pred, m, t, T, pvec, pv);
+  uint32_t sv[kRegItems];
+  if (in_regs) {
+    int32_t a[kRegItems], b[kRegItems];
+    load_items(L, n, t, T, svec, a);
+    load_items(P, n, t, T, svec, b);
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {  // issue all loads first
-        const int64_t i = i0 + u * stride + threadIdx.x;
-        ok[u] = i < n4;
-        a[u] = ok[u] ? __ldg(L4 + i) : make_int4(0, 0, 0, 0);
-        b[u] = ok[u] ? __ldg(P4 + i) : make_int4(0, 0, 0, 0);
+    for (int i = 0; i < kRegItems; ++i) sv[i] = score(a[i], b[i]);
+  }
+
+  uint32_t lo = 0;
+  int wlog = 32;
+  unsigned long long k = k0;
+  for (int pass = 0; pass < kPasses && wlog > 0; ++pass) {
+    for (int b = tid; b < kBins; b += blockDim.x) sh[b] = 0;
+    __syncthreads();
+    const int shift = wlog > kStepBits ? wlog - kStepBits : 0;
+    // First pass: the zero scores (about half of a length residual's scores)
+    // are counted by one ballot per warp and every other lane adds alone,
+    // since its bin is a single value or a narrow range.  Later passes
+    // aggregate the lanes of each bin with a match, as no bin of a range is
+    // known to be hot.  Every lane of a warp calls this together.
+    auto visit = [&](uint32_t s, bool valid) {
+      if (pass == 0) {
+        const int d = first_bin(s);
+        const unsigned zeros = __ballot_sync(0xffffffffu, valid && d == 0);
+        if (zeros && lane == __ffs(zeros) - 1) atomicAdd(&sh[0], static_cast<uint32_t>(__popc(zeros)));
+        if (valid && d > 0) atomicAdd(&sh[d], 1u);
+      } else {
+        const uint32_t r = s - lo;  // wlog <= 24 here
+        if (s < lo || r >= (1u << wlog)) valid = false;
+        const int d = valid ? static_cast<int>(r >> shift) : -1;
+        const unsigned peers = __match_any_sync(0xffffffffu, d);
+        if (valid && lane == __ffs(peers) - 1)
+          atomicAdd(&sh[d], static_cast<uint32_t>(__popc(peers)));
       }
+    };
+    if (in_regs) {
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        visit(score(a[u].x, b[u].x), ok[u]);
-        visit(score(a[u].y, b[u].y), ok[u]);
-        visit(score(a[u].z, b[u].z), ok[u]);
-        visit(score(a[u].w, b[u].w), ok[u]);
+      for (int i = 0; i < kRegItems; ++i)
+        visit(sv[i], 4 * (t + (i / 4) * T) + (i % 4) < n);
+    } else {
+      // whole blocks step together, so every lane of a warp visits
+      for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x; 4 * base < n; base += T) {
+        const int64_t i4 = base + tid;
+        int32_t a[4], b[4];
+        if (svec && 4 * i4 + 4 <= n) {
+          const int4 x = __ldg(reinterpret_cast<const int4 *>(L) + i4);
+          const int4 y = __ldg(reinterpret_cast<const int4 *>(P) + i4);
+          a[0] = x.x, a[1] = x.y, a[2] = x.z, a[3] = x.w;
+          b[0] = y.x, b[1] = y.y, b[2] = y.z, b[3] = y.w;
+        } else {
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const bool ok = 4 * i4 + c < n;
+            a[c] = ok ? __ldg(L + 4 * i4 + c) : 0;
+            b[c] = ok ? __ldg(P + 4 * i4 + c) : 0;
+          }
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) visit(score(a[c], b[c]), 4 * i4 + c < n);
       }
     }
-    tail_start = n4 * 4;
-  }
-  for (int64_t i0 = tail_start + b0; i0 < n; i0 += stride) {
-    const int64_t i = i0 + threadIdx.x;
-    const bool ok = i < n;
-    visit(ok ? score(__ldg(L + i), __ldg(P + i)) : 0u, ok);
-  }
-  __syncthreads();
+    __syncthreads();
+    // start each block's flush at a different bin so blocks do not collide
+    const int rot = static_cast<int>((blockIdx.x * 97u) % kBins);
+    for (int i = tid; i < kBins; i += blockDim.x) {
+      const int b = (i + rot) & (kBins - 1);
+      if (sh[b]) atomicAdd(&st->hist[pass][b], static_cast<unsigned long long>(sh[b]));
+    }
+    if (!grid_barrier(&st->bar, status, kSpinLimit)) return;
 
-  // start each block's flush at a different bin so blocks do not collide
-  const int rot = static_cast<int>((blockIdx.x * 97u) % kBins);
-  for (int i = threadIdx.x; i < kBins; i += blockDim.x) {
-    const int b = (i + rot) & (kBins - 1);
-    if (sh[b]) atomicAdd(&st->hist[PASS][b], static_cast<unsigned long long>(sh[b]));
-  }
-  // one thread publishes the block's flush (the barrier orders every thread's
-  // atomics before its fence, as a grid barrier does)
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    s_last = (atomicAdd(&st->done[PASS], 1u) == gridDim.x - 1);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-
-  // The last block: find the bin holding rank k inside the range.
-  const unsigned long long k =
-      PASS == 0 ? k0 : *reinterpret_cast<volatile unsigned long long *>(&st->k_rem);
-  constexpr int kPer = kBins / kSelectThreads;  // 4 consecutive bins per thread
-  unsigned long long c[kPer], tot = 0;
-#pragma unroll
-  for (int j = 0; j < kPer; ++j) {
-    c[j] = __ldcg(&st->hist[PASS][threadIdx.x * kPer + j]);
-    tot += c[j];
-  }
-  // exclusive scan of the per-thread totals
-  const int warp = threadIdx.x >> 5;
-  unsigned long long incl = tot;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    unsigned long long y = __shfl_up_sync(0xffffffffu, incl, off);
-    if (lane >= off) incl += y;
-  }
-  if (lane == 31) s_warp[warp] = incl;
-  __syncthreads();
-  unsigned long long excl = incl - tot;
-  for (int w = 0; w < warp; ++w) excl += s_warp[w];
-  if (excl < k && k <= excl + tot) {
-    unsigned long long cum = excl;
-    int d = 0;
+    // every block: the bin holding rank k inside the range (the same counts,
+    // so the same bin in every block)
+    constexpr int kPer = kBins / kSelectThreads;  // 4 consecutive bins per thread
+    unsigned long long c[kPer], tot = 0;
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {
-      if (k <= cum + c[j]) {
-        d = threadIdx.x * kPer + j;
-        break;
-      }
-      cum += c[j];
+      c[j] = __ldcg(&st->hist[pass][tid * kPer + j]);
+      tot += c[j];
     }
-    // the new range: the bin's values
-    uint32_t nlo;
-    int nw;
-    if constexpr (PASS == 0) {
-      if (d < static_cast<int>(kExactBins)) {
-        nlo = static_cast<uint32_t>(d);
-        nw = 0;
-      } else {
-        const int e = 10 + ((d - static_cast<int>(kExactBins)) >> kMantBits);
-        const uint32_t top = (1u << kMantBits) |
-                             static_cast<uint32_t>((d - static_cast<int>(kExactBins)) &
-                                                   ((1 << kMantBits) - 1));
-        nlo = top << (e - kMantBits);
-        nw = e - kMantBits;
+    unsigned long long incl = tot;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const unsigned long long y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    unsigned long long excl = incl - tot;
+    for (int w = 0; w < warp; ++w) excl += s_warp[w];
+    if (excl < k && k <= excl + tot) {
+      unsigned long long cum = excl;
+      int d = 0;
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) {
+        if (k <= cum + c[j]) {
+          d = tid * kPer + j;
+          break;
+        }
+        cum += c[j];
       }
+      // the new range: the bin's values
+      uint32_t nlo;
+      int nw;
+      if (pass == 0) {
+        if (d < static_cast<int>(kExactBins)) {
+          nlo = static_cast<uint32_t>(d);
+          nw = 0;
+        } else {
+          const int e = 10 + ((d - static_cast<int>(kExactBins)) >> kMantBits);
+          const uint32_t top = (1u << kMantBits) |
+                               static_cast<uint32_t>((d - static_cast<int>(kExactBins)) &
+                                                     ((1 << kMantBits) - 1));
+          nlo = top << (e - kMantBits);
+          nw = e - kMantBits;
+        }
+      } else {
+        nlo = lo + (static_cast<uint32_t>(d) << shift);
+        nw = shift;
+      }
+      s_lo = nlo;
+      s_w = nw;
+      s_k = k - cum;
+    }
+    __syncthreads();
+    lo = s_lo;
+    wlog = s_w;
+    k = s_k;
+    __syncthreads();  // s_lo, s_w, s_k and s_warp are written again next pass
+  }
+  // three passes always close the range: q = lo
+  const bool q_ok = lo <= 0x7fffffffu;
+  const int32_t q = q_ok ? static_cast<int32_t>(lo) : 0;
+  if (blockIdx.x == 0 && tid == 0) {
+    if (q_ok) {
+      st->q = q;
+      if (q_dev_out) *q_dev_out = q;
     } else {
-      nlo = lo + (static_cast<uint32_t>(d) << shift);
-      nw = shift;
-    }
-    st->lo = nlo;
-    st->wlog = nw;
-    st->k_rem = k - cum;
-    if (nw == 0) {
-      st->resolved = 1u;
-      if (nlo > 0x7fffffffu) {
-        flag_error(status, MAPS_E_RANGE);
-      } else {
-        st->q = static_cast<int32_t>(nlo);
-        if (q_dev_out) *q_dev_out = static_cast<int32_t>(nlo);
-      }
+      flag_error(status, MAPS_E_RANGE);
     }
   }
+  // U = pred + q (Eq. conformal_upper), saturated and flagged above INT32_MAX
+  bool bad = false;
+  auto bound_of = [&](int32_t p) {
+    long long u = static_cast<long long>(p) + q;
+    if (u > 0x7fffffffLL) {
+      bad = true;
+      u = 0x7fffffffLL;
+    }
+    return static_cast<int32_t>(u);
+  };
+  if (pred_in_regs) {
+#pragma unroll
+    for (int u = 0; u < kRegItems / 4; ++u) {
+      const int64_t i4 = t + u * T, e0 = 4 * i4;
+      if (pvec && e0 + 4 <= m) {
+        reinterpret_cast<int4 *>(out)[i4] =
+            make_int4(bound_of(pv[4 * u]), bound_of(pv[4 * u + 1]), bound_of(pv[4 * u + 2]),
+                      bound_of(pv[4 * u + 3]));
+      } else {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          if (e0 + c < m) out[e0 + c] = bound_of(pv[4 * u + c]);
+      }
+    }
+  } else {
+    for (int64_t i = t; i < m; i += T) out[i] = bound_of(__ldg(pred + i));
+  }
+  if (bad) flag_error(status, MAPS_E_RANGE);
 }
 
 // U = pred + q.  Four bounds per thread (one 128-bit load and store when
@@ -360,6 +414,17 @@ select_small_kernel(const int32_t *__restrict__ L, const int32_t *__restrict__ P
   if (__syncthreads_or(bad) && tid == 0) flag_error(status, MAPS_E_RANGE);
 }
 
+// Blocks of the fused kernel that can be resident at once (its grid limit as
+// a cooperative launch).
+int64_t fused_grid() {
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, calibrate_fused_kernel, kSelectThreads,
+                                                    0) != cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  return static_cast<int64_t>(per_sm) * sm_count();
+}
+
 inline int64_t conformal_rank(int64_t n, uint32_t alpha_ppm) {
   const int64_t num = static_cast<int64_t>(1000000u - alpha_ppm) * (n + 1);
   return (num + 999999) / 1000000;
@@ -406,15 +471,18 @@ int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
     if (m <= kSmallM) m = 0;
   } else {
     MAPS_TRY(cuda_ok(cudaMemsetAsync(st, 0, sizeof(SelectState), s)));
-    // one block of 1,024 threads per multiprocessor (its registers allow one),
-    // each reading at least a 128-bit word of both arrays per thread
-    const int g = static_cast<int>(std::min<int64_t>(std::max<int64_t>(1, (n + 4 * kSelectThreads - 1) /
-                                                                          (4 * kSelectThreads)),
-                                                     sm_count()));
-    launch_pdl(select_pass_kernel<0>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
-    launch_pdl(select_pass_kernel<1>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
-    launch_pdl(select_pass_kernel<2>, g, kSelectThreads, 0, s, true_len, pred_len, n, kk, st, q_dev_out, status);
-    MAPS_TRY(launch_ok());
+    // one block of 1,024 threads per multiprocessor (its registers allow
+    // one), at least a 128-bit word of both arrays per thread, and enough
+    // threads to hold the predictions in registers
+    const int64_t per = static_cast<int64_t>(kRegItems) * kSelectThreads;
+    const int64_t want = std::max<int64_t>({int64_t(1), (n + 4 * kSelectThreads - 1) / (4 * kSelectThreads),
+                                            (m + per - 1) / per});
+    const int64_t g = std::min<int64_t>(want, fused_grid());
+    const int in_regs = n <= per * g ? 1 : 0;
+    const int pred_in_regs = m <= per * g ? 1 : 0;
+    MAPS_TRY(launch_coop(calibrate_fused_kernel, g, kSelectThreads, 0, s, true_len, pred_len, n, kk,
+                         query_pred, m, bound_out, st, q_dev_out, status, in_regs, pred_in_regs));
+    m = 0;  // the bounds are written by the same kernel
   }
   if (m > 0) {
     const int64_t gb = (m + 1023) / 1024;

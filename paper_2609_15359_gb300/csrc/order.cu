@@ -122,7 +122,12 @@ static_assert(kSegMax % kMergeTile == 0, "merge tiles align with runs");
 // pair_budget(N), and a queue past the cap or past kPairRuns is merged.
 constexpr int kPairRuns = 16;
 __host__ __device__ __forceinline__ int64_t pair_budget(int64_t N) {
-  const int64_t b = 4 * (N / kSegMax);
+  // room for one queue of every entry (up to kPairRuns runs), and at larger
+  // N four pairs per chunk
+  const int64_t runs = (N + kSegMax - 1) / kSegMax;
+  const int64_t r = runs < kPairRuns ? runs : kPairRuns;
+  const int64_t per = 4 * (N / kSegMax);
+  const int64_t b = per > r * (r - 1) ? per : r * (r - 1);
   return b < 1024 ? b : 1024;
 }
 struct PairQueues {
@@ -1849,8 +1854,10 @@ int maps_order_local(int64_t N, int32_t D, const int32_t *dec, const int32_t *bo
   MAPS_TRY(cuda_ok(cudaFuncSetAttribute(order_finish_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         static_cast<int>(smem))));
-  // the global passes take tiles by ticket, so any resident grid completes them
-  MAPS_TRY(launch_coop(order_finish_kernel, std::min<int64_t>(tiles, finish_grid(smem)),
+  // the global passes take tiles by ticket, so any resident grid completes
+  // them; the pairwise ranks take one block per pair
+  MAPS_TRY(launch_coop(order_finish_kernel,
+                       std::min<int64_t>(std::max<int64_t>(tiles, w.pq.budget), finish_grid(smem)),
                        kPassThreads, smem, s, n_hi, N, D, dbits, w.counts, w.plan, w.dec_count,
                        seg_off_out, w.mt_off, w.mt_n, w.mt_t, w.pq, w.keyA, w.keyB, w.valA, w.valB,
                        w.hi_orig, perm_out, w.state, tiles, w.tickets, w.bar, status));
@@ -1874,7 +1881,7 @@ namespace {
 
 constexpr int64_t kStaticMaxN = 65536;  // entries
 constexpr int32_t kStaticMaxD = 4096;   // decoders
-constexpr size_t kStaticBytes = size_t(3) << 20;
+constexpr size_t kStaticBytes = size_t(5) << 20;
 static __device__ __align__(256) unsigned char g_order_scratch[kStaticBytes];
 
 // Device address of the static scratch on the current device.  The host-side

@@ -47,3 +47,14 @@ def test_binding_loads_and_host_only_queries(libmaps):
     big = M.lib.maps_dispatch_workspace_size(M.MODE_SNAPSHOT, 256, 65536, 65536)
     assert big > 2 * 256 * 1024 * 4  # look-back state for every tile and decoder
     assert M.lib.maps_order_local_workspace_size(10**6, 256) > 10**6 * 24
+
+
+def test_static_order_array_holds_its_largest_calls(libmaps):
+    """maps_order_local_static takes up to 65,536 entries and 4,096 decoders in
+    a fixed 5 MiB array: the workspace those calls need fits it, and a queue of
+    all 65,536 entries has room for its sixteen runs' pairwise ranks."""
+    from paper_2609_15359_gb300 import maps as M
+    for D in (1, 7, 256, 1024, 1025, 4096):
+        assert M.lib.maps_order_local_workspace_size(65536, D) <= 5 << 20
+    small = M.lib.maps_order_local_workspace_size(65536, 1)
+    assert small > 15 * 14 * 4608 * 2  # 210 run pairs of 16-bit counts

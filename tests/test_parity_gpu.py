@@ -220,6 +220,44 @@ def test_calibrate_grid_bucket_edges(M, ws, oracle, seed):
     assert {0, M.MAPS_E_RANGE} <= seen
 
 
+@pytest.mark.parametrize("n,m,shift", [
+    # more scores than the grid keeps in registers: every pass reads them again
+    (1300007, 4099, 0),
+    # more predictions than the grid keeps in registers, at an unaligned address
+    (20011, 1300003, 1),
+    # just past the one-block limit, no queries; then a ragged, unaligned few
+    (8193, 0, 0), (10001, 777, 1)])
+def test_calibrate_fused_register_limits(M, ws, oracle, n, m, shift):
+    """Calibration sets above the one-block limit take one cooperative kernel;
+    its scores and predictions live in registers up to eight per thread, else
+    they are read from memory: q, the bounds and the status match the oracle
+    either way."""
+    rng = np.random.default_rng(n + m)
+    L = rng.integers(0, 40000, n).astype(np.int32)
+    P = rng.integers(0, 40000, n).astype(np.int32)
+    P[: n // 5] = L[: n // 5]
+    query = rng.integers(0, 70000, m + shift).astype(np.int32)
+    Ld, Pd, Qd = dev(L), dev(P), dev(query)
+    U = torch.full((m + shift + 1,), -9, dtype=torch.int32, device="cuda")
+    qd = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for a in (1000, 100000, 999999):  # ranks within n at every size here
+        sto, qo = oracle.calibrate(L, P, a)
+        st, q = M.maps_calibrate(Ld, Pd, a, Qd[shift:] if m else None, U[shift:shift + m] if m else None,
+                                 qd, q_host=True, ws=ws)
+        assert st == sto == 0 and q == qo == int(host(qd)[0]), (n, m, a)
+        if m:
+            Uh = host(U)
+            assert np.array_equal(Uh[shift:shift + m], oracle.bound(query[shift:], qo)[1])
+            assert Uh[:shift].tolist() == [-9] * shift and Uh[shift + m] == -9
+    # a bound above INT32_MAX: the range error, the others still bounded
+    big = query[shift:].copy() if m else np.zeros(1, np.int32)
+    big[-1] = I32_MAX - 3
+    Ub = torch.empty(len(big), dtype=torch.int32, device="cuda")
+    st, q = M.maps_calibrate(Ld, Pd, 100000, dev(big), Ub, q_host=True, ws=ws)
+    assert st == M.MAPS_E_RANGE
+    assert np.array_equal(host(Ub)[:-1], oracle.bound(big[:-1], oracle.calibrate(L, P, 100000)[1])[1])
+
+
 @pytest.mark.parametrize("name", ["tiny", "d16", "d64", "large"])
 def test_calibrate_workloads(M, ws, oracle, name):
     w = W.make(name)
@@ -543,7 +581,12 @@ def test_order_bucketing_rounds_range_error(M, ws, oracle):
     # bounds in [2^20, 2^20 + 200): keys share their high bits
     (30000, 3, 2**20, 2**20 + 200, 0.5),
     # more decoders than the stable scatter takes, one long queue
-    (40000, 1100, 0, 2**31 - 1, 0.9)])
+    (40000, 1100, 0, 2**31 - 1, 0.9),
+    # every entry in one queue of 15 runs (ranked pairwise: 210 pairs)
+    (65536, 256, 0, 70000, 1.0),
+    # sixteen queues of about 16 runs each: the first to reserve their pairs within
+    # the budget are ranked pairwise, the others merged level by level
+    (1120000, 16, 0, 2**31 - 1, 0.0)])
 def test_order_long_queues(M, ws, oracle, N, D, blo, bhi, skew):
     rng = np.random.default_rng(N + D)
     dec = rng.integers(0, D, N).astype(np.int32)
