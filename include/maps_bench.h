@@ -46,6 +46,16 @@ int maps_test_withhold_lookback(int32_t tile, uint32_t spin_limit);
  * changes.  Returns MAPS_OK or MAPS_E_CUDA. */
 int maps_test_absent_block(int32_t block);
 
+/* Exercises the bounded grid barrier of maps_calibrate's cooperative kernel
+ * (calibration sets above 8,192 residuals): on the current device, later
+ * calls make block `block` of that kernel return at once, so the other
+ * blocks' barrier gives up after `spin_limit` polls (0: the library default),
+ * records MAPS_E_TIMEOUT (read with maps_check) and ends each block without
+ * another write: q and the bounds of that call are not written.  block = -1,
+ * spin_limit = 0 restores the normal behaviour.  Calls in flight must have
+ * finished before the settings change.  Returns MAPS_OK or MAPS_E_CUDA. */
+int maps_test_calibrate_absent_block(int32_t block, uint32_t spin_limit);
+
 #ifdef __cplusplus
 }
 #endif

@@ -23,6 +23,7 @@
 #include <algorithm>
 
 #include "maps_internal.cuh"
+#include "maps_bench.h"
 
 namespace maps {
 namespace {
@@ -34,6 +35,12 @@ constexpr uint32_t kExactBins = 1024;  // scores below this have a bin each
 constexpr int kMantBits = 7;           // bits after the leading one, first pass
 constexpr int kStepBits = 12;          // bits per later pass
 constexpr int kRegItems = 8;           // scores, and predictions, a thread keeps in registers
+
+// Test aid (maps_test_calibrate_absent_block): a block of the fused kernel
+// that returns at once (-1: none), so that the others' grid barrier runs out,
+// and the polls a barrier wait makes before it gives up.
+__device__ int32_t g_cal_absent_block = -1;
+__device__ uint32_t g_cal_spins = kSpinLimit;
 
 struct SelectState {
   unsigned long long hist[kPasses][kBins];  // global bin counts per pass
@@ -81,6 +88,7 @@ calibrate_fused_kernel(const int32_t *__restrict__ L, const int32_t *__restrict_
                        int32_t *__restrict__ out, SelectState *st, int32_t *q_dev_out,
                        int32_t *status, int in_regs, int pred_in_regs) {
   pdl_prologue();
+  if (static_cast<int>(blockIdx.x) == g_cal_absent_block) return;  // test aid, normally -1
   __shared__ uint32_t sh[kBins];
   __shared__ unsigned long long s_warp[kSelectThreads / 32];
   __shared__ uint32_t s_lo;
@@ -165,7 +173,7 @@ calibrate_fused_kernel(const int32_t *__restrict__ L, const int32_t *__restrict_
       const int b = (i + rot) & (kBins - 1);
       if (sh[b]) atomicAdd(&st->hist[pass][b], static_cast<unsigned long long>(sh[b]));
     }
-    if (!grid_barrier(&st->bar, status, kSpinLimit)) return;
+    if (!grid_barrier(&st->bar, status, g_cal_spins)) return;
 
     // every block: the bin holding rank k inside the range (the same counts,
     // so the same bin in every block)
@@ -494,6 +502,14 @@ int maps_calibrate(const int32_t *true_len, const int32_t *pred_len, int64_t n,
     MAPS_TRY(cuda_ok(cudaMemcpyAsync(q_host_out, &st->q, sizeof(int32_t), cudaMemcpyDeviceToHost, s)));
     return maps_check(ws, stream);
   }
+  return MAPS_OK;
+}
+
+int maps_test_calibrate_absent_block(int32_t block, uint32_t spin_limit) {
+  using namespace maps;
+  const uint32_t spins = spin_limit == 0 ? kSpinLimit : spin_limit;
+  MAPS_TRY(cuda_ok(cudaMemcpyToSymbol(g_cal_absent_block, &block, sizeof(block))));
+  MAPS_TRY(cuda_ok(cudaMemcpyToSymbol(g_cal_spins, &spins, sizeof(spins))));
   return MAPS_OK;
 }
 

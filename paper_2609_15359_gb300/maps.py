@@ -76,6 +76,7 @@ def _load():
         "maps_set_dispatch_events": ([vp, vp], ctypes.c_int),
         "maps_test_withhold_lookback": ([i32, u32], ctypes.c_int),
         "maps_test_absent_block": ([i32], ctypes.c_int),
+        "maps_test_calibrate_absent_block": ([i32, u32], ctypes.c_int),
         "maps_calibrate_workspace_size": ([i64, i64], sz),
         "maps_calibrate": ([vp, vp, i64, u32, vp, i64, vp, vp, vp, vp, sz, vp], ctypes.c_int),
         "maps_project_occupancy_workspace_size": ([i32, i32, i64], sz),
@@ -104,7 +105,7 @@ def _load():
 lib = _load()
 EXPORTS = ("maps_version", "maps_last_cuda_error", "maps_check", "maps_set_dispatch_events",
            "maps_test_withhold_lookback", "maps_test_absent_block",
-           "maps_calibrate_workspace_size", "maps_calibrate",
+           "maps_test_calibrate_absent_block", "maps_calibrate_workspace_size", "maps_calibrate",
            "maps_project_occupancy_workspace_size", "maps_project_occupancy",
            "maps_dispatch_workspace_size", "maps_dispatch",
            "maps_order_local_workspace_size", "maps_order_local", "maps_order_local_static",

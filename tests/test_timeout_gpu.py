@@ -1,5 +1,10 @@
 """A bounded device wait that runs out is reported, and the device stays usable.
 
+The calibration's cooperative kernel (calibration sets above 8,192 residuals)
+waits at a bounded grid barrier after each select pass; the test aid
+maps_test_calibrate_absent_block makes one of its blocks return at once, so
+the others' wait runs out.
+
 The local order's global form (arrival not in index order) sorts with
 decoupled look-back between tiles: each tile waits, bounded, for its
 predecessors' published counts.  The test aid maps_test_withhold_lookback
@@ -90,3 +95,36 @@ def test_order_grid_barrier_timeout_is_reported_and_the_next_call_is_exact(oracl
     assert M.maps_check(ws2) == 0 and sto == 0
     assert np.array_equal(perm.cpu().numpy(), po)
     assert np.array_equal(seg.cpu().numpy(), so)
+
+
+def test_calibrate_grid_barrier_timeout_is_reported_and_the_next_call_is_exact(oracle):
+    """Block 0 of the calibration's cooperative kernel is made absent, so the
+    other blocks' barrier after the first select pass runs out after a short
+    limit: the call reports MAPS_E_TIMEOUT and writes no bound, and the next
+    call on a fresh workspace gives the oracle's q and bounds exactly."""
+    if not torch.cuda.is_available():
+        pytest.fail("CUDA device required")
+    from paper_2609_15359_gb300 import maps as M
+    rng = np.random.default_rng(17)
+    n, m, a = 200_000, 5_000, 100_000
+    L = rng.integers(0, 40000, n).astype(np.int32)
+    P = rng.integers(0, 40000, n).astype(np.int32)
+    pred = rng.integers(0, 5000, m).astype(np.int32)
+    Ld, Pd, pd = (torch.from_numpy(x).cuda() for x in (L, P, pred))
+    U = torch.full((m + 1,), -9, dtype=torch.int32, device="cuda")
+    qd = torch.full((1,), -9, dtype=torch.int32, device="cuda")
+    ws = M.Workspace()
+    try:
+        assert M.lib.maps_test_calibrate_absent_block(0, 2000) == 0
+        st, _ = M.maps_calibrate(Ld, Pd, a, pd, U[:m], qd, ws=ws)
+        assert st == 0
+        assert M.maps_check(ws) == M.MAPS_E_TIMEOUT
+    finally:
+        assert M.lib.maps_test_calibrate_absent_block(-1, 0) == 0
+    assert (U.cpu().numpy() == -9).all() and int(qd.item()) == -9  # nothing written
+    sto, qo = oracle.calibrate(L, P, a)
+    _, Uo = oracle.bound(pred, qo)
+    ws2 = M.Workspace()
+    st, q = M.maps_calibrate(Ld, Pd, a, pd, U[:m], qd, q_host=True, ws=ws2)
+    assert st == sto == 0 and q == qo == int(qd.item())
+    assert np.array_equal(U[:m].cpu().numpy(), Uo) and int(U[m].item()) == -9
