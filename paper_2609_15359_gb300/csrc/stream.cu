@@ -727,9 +727,9 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
   // Without a headroom output and with the Q-first rule, a decoder whose peak
   // is provably within its capacity is decided by (Q, index) alone.
   const bool quick = headroom == nullptr && mc == 0;
-  // Fast path (at most 32 decoders, no headroom output, Q-first rule): take
-  // each candidate's choice by (Q, index) alone while checking that every
-  // decoder is feasible at that step, before any list is sorted.  For t < u,
+  // Fast path (at most 32 decoders, no headroom output, Q-first rule): the
+  // choices by (Q, index) alone, taken when every decoder is shown feasible at
+  // every step, before any list is sorted.  For t < u,
   // K(t) + t = S(t) + t (C(t) + 1) with S <= the decoder's b-sum and C <= n
   // while t < e_max, and K(t) + t = t after e_max, so decoder k's peak for a
   // candidate of horizon u, after the batch's earlier reservations on k, is
@@ -739,54 +739,118 @@ stream_dispatch_kernel(int D, int H, int nb, int mc, const int64_t *res_off, con
   // (each adds p + t + 1 for t < u).  While p + 1 + that bound <= cap for
   // every decoder, every decoder is feasible, so the rule picks the smallest
   // (Q, index), which is the choice taken: the decisions are the walk's, and
-  // the lists need no sorting.  A step where some decoder might not fit sends
-  // the whole batch to the walk (Q is written only on success).
-  if (quick && D <= 32 && warp == 0) {
-    const int k = lane;
-    const bool has = k < D;
-    const int n = has ? s_n[k] : 0, lo = has ? s_base[k] - k * nb : 0;
-    long long sb = 0;  // this decoder's b-sum and largest end step
-    int em = 1;
-    for (int i = 0; i < n; ++i) {
-      sb += uB[lo + i];
-      em = max(em, uE[lo + i]);
+  // the lists need no sorting.  If some decoder might not fit at some step
+  // the walk decides the whole batch (Q is written only on success).
+  // The picks of the Q-first rule have a closed form: taking the smallest
+  // (Q, index) and raising that Q by one, level by level, at level L every
+  // decoder with Q <= L takes one candidate, in index order.  So candidate j
+  // goes to level L, the smallest with cum(L) > j where
+  // cum(L) = sum over k of max(0, L - Q_k + 1), and there to the
+  // (j - cum(L - 1))-th decoder with Q <= L.  Each candidate's pick is found
+  // on its own; then one warp per decoder sums the reservations before each
+  // candidate (a scan) and checks the bound.
+  if (quick && D <= 32) {
+    __shared__ long long f_sb[32];
+    __shared__ int f_em[32], f_cnt[32], f_inv, f_miss;
+    if (tid == 0) {
+      f_inv = 0;
+      f_miss = 0;
     }
-    const long long cap = has ? s_cap[k] : 0;
-    int q = has ? s_q[k] : 0;
-    // checked once: every candidate valid, every Q stays within 21 bits (a Q
-    // grows by at most nb), and no K of the residents reaches INT32_MAX (so
-    // the tables' range checks could not fire); otherwise the walk handles
-    // the batch
-    bool invalid = has && (static_cast<long long>(q) + nb >= (1 << 21) ||
-                           sb + static_cast<long long>(em - 1) * (n + 1) > 0x7fffffffLL);
-    for (int j = lane; j < nb; j += 32) invalid |= (s_cp[j] | s_cu[j]) < 0;
-    bool fits = !__any_sync(0xffffffffu, invalid);
-    long long add = 0;
-    bool miss = false;  // some step where this lane's decoder might not fit
-    for (int j0 = 0; j0 < nb && fits; j0 += 32) {
-      const int j1 = min(nb, j0 + 32);
-      for (int j = j0; j < j1; ++j) {
-        const int32_t p = s_cp[j], U = s_cu[j];
+    __syncthreads();
+    if (warp < D) {  // decoder `warp`: its residents' b-sum and largest end step
+      const int k = warp, n = s_n[k], lo = s_base[k] - k * nb;
+      long long sb = 0;
+      int em = 1;
+      for (int i = lane; i < n; i += 32) {
+        sb += uB[lo + i];
+        em = max(em, uE[lo + i]);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        sb += __shfl_xor_sync(0xffffffffu, sb, off);
+        em = max(em, __shfl_xor_sync(0xffffffffu, em, off));
+      }
+      if (lane == 0) {
+        f_sb[k] = sb;
+        f_em[k] = em;
+        f_cnt[k] = 0;
+        // checked once: every Q stays within 21 bits (a Q grows by at most
+        // nb), and no K of the residents reaches INT32_MAX (so the tables'
+        // range checks could not fire); otherwise the walk handles the batch
+        if (static_cast<long long>(s_q[k]) + nb >= (1 << 21) ||
+            sb + static_cast<long long>(em - 1) * (n + 1) > 0x7fffffffLL)
+          f_inv = 1;
+      }
+    }
+    for (int j = tid; j < nb; j += kSt)
+      if ((s_cp[j] | s_cu[j]) < 0) f_inv = 1;  // every candidate valid
+    __syncthreads();
+    if (!f_inv) {
+      int qmin = 0x7fffffff;
+      for (int k = 0; k < D; ++k) qmin = min(qmin, s_q[k]);
+      auto cum = [&](int L) {  // picks made by the end of level L
+        int c = 0;
+        for (int k = 0; k < D; ++k) c += max(0, L - s_q[k] + 1);
+        return c;
+      };
+      for (int j = tid; j < nb; j += kSt) {
+        // the decoder at qmin alone takes nb picks by level qmin + nb - 1
+        int lo = qmin, hi = qmin + nb - 1;
+        while (lo < hi) {
+          const int mid = lo + (hi - lo) / 2;
+          if (cum(mid) > j)
+            hi = mid;
+          else
+            lo = mid + 1;
+        }
+        int r = j - (lo > qmin ? cum(lo - 1) : 0);
+        int pick = -1;
+        for (int k = 0; k < D; ++k)
+          if (s_q[k] <= lo && r-- == 0) {
+            pick = k;
+            break;
+          }
+        s_ch[j] = pick < 0 ? 0 : pick;
+        if (pick < 0) f_miss = 1;  // cannot happen; the walk would decide the batch
+      }
+    }
+    __syncthreads();
+    if (!f_inv && warp < D) {
+      const int k = warp, n = s_n[k], em = f_em[k];
+      const long long sb = f_sb[k], cap = s_cap[k];
+      long long carry = 0;  // p + u of this decoder's reservations so far
+      int cnt = 0;
+      bool miss = false;
+      for (int j0 = 0; j0 < nb; j0 += 32) {
+        const int j = j0 + lane;
+        const bool ok = j < nb;
+        const int32_t p = ok ? s_cp[j] : 0, U = ok ? s_cu[j] : 1;
         const int u = U < 1 ? 1 : (U > H ? H : U);
+        const bool mine = ok && s_ch[j] == k;
+        const long long w = mine ? static_cast<long long>(p) + u : 0;
+        long long incl = w;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const long long y = __shfl_up_sync(0xffffffffu, incl, off);
+          if (lane >= off) incl += y;
+        }
+        const long long add = carry + incl - w;  // the reservations before candidate j
         const long long b0 = max(sb + static_cast<long long>(min(u, em) - 1) * (n + 1),
                                  static_cast<long long>(u - 1));
-        miss |= has && static_cast<long long>(p) + 1 + b0 + add > cap;
-        const uint32_t key = has ? (static_cast<uint32_t>(q) << 10) | static_cast<uint32_t>(k) : 0xffffffffu;
-        const int bk = static_cast<int>(__reduce_min_sync(0xffffffffu, key) & 1023u);
-        if (lane == 0) s_ch[j] = bk;
-        if (lane == bk) {
-          q += 1;
-          add += static_cast<long long>(p) + u;
-        }
+        miss |= ok && static_cast<long long>(p) + 1 + b0 + add > cap;
+        carry += __shfl_sync(0xffffffffu, incl, 31);
+        cnt += __popc(__ballot_sync(0xffffffffu, mine));
       }
-      fits = !__any_sync(0xffffffffu, miss);  // a miss anywhere: the walk decides the batch
+      if (__any_sync(0xffffffffu, miss) && lane == 0) f_miss = 1;
+      if (lane == 0) f_cnt[k] = cnt;
     }
+    __syncthreads();
+    const bool fits = !f_inv && !f_miss;
     if (fits) {
-      __syncwarp();
-      for (int j = lane; j < nb; j += 32) choice[j] = s_ch[j];
-      if (has) s_q[k] = q;
+      for (int j = tid; j < nb; j += kSt) choice[j] = s_ch[j];
+      for (int k = tid; k < D; k += kSt) s_q[k] += f_cnt[k];
     }
-    if (lane == 0) s_fast = fits ? 1 : 0;
+    if (tid == 0) s_fast = fits ? 1 : 0;
   }
   __syncthreads();
 
