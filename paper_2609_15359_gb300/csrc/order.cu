@@ -980,15 +980,18 @@ __device__ unsigned long long seg_diff(SegSmem &sm, int n, int cur) {
 }
 
 // Small calls (1 <= N <= kSegMax entries, D <= kSmallOrderD): the whole
-// order in one block.  The entries are put in arrival order first unless
-// arrival is already non-decreasing along the index (a sort of (arrival,
-// index)); then a sort of (decoder, not promoted, promoted ? 0 : bound,
-// arrival position) gives the queue order (promoted entries keep their
-// arrival order).  Up to kBitonicN entries both sorts are bitonic networks
-// over unique keys (a few dozen barrier-separated stages); larger calls take
-// stable 9-bit LSD passes with the index in the keys' low bits.  The segment
-// offsets come from binary searches over the sorted decoders.  One launch
-// instead of a memset and four.
+// order in one block.  When arrival is non-decreasing along the index, one
+// sort of (decoder, not promoted, promoted ? 0 : bound, index) gives the
+// queue order.  Otherwise, when (decoder, not promoted, promoted ? 0 : bound,
+// arrival, index) fits 64 bits (the bit widths taken from the largest
+// arrival and the largest non-promoted bound), one sort on that key does;
+// else the entries are put in arrival order first (a sort of (arrival,
+// index)) and the first key's index is replaced by the arrival position.  Up
+// to kBitonicN entries the sorts are bitonic networks over unique keys (a
+// few dozen barrier-separated stages); larger calls take stable 9-bit LSD
+// passes with the index in the keys' low bits.  The segment offsets come
+// from binary searches over the sorted decoders.  One launch instead of a
+// memset and four.
 constexpr int kSmallOrderD = 4096;
 constexpr int kBitonicN = 1024;
 
@@ -1020,73 +1023,136 @@ order_small_kernel(int N, int D, int dbits, const int32_t *__restrict__ dec,
   pdl_prologue();
   extern __shared__ __align__(16) unsigned char small_raw[];
   SegSmem &sm = *reinterpret_cast<SegSmem *>(small_raw);
+  __shared__ uint32_t s_amax, s_umax;
   const int tid = threadIdx.x;
   const int ib = index_bits(N);
   const unsigned long long imask = (1ull << ib) - 1;
   bool bad = false, unsorted = false;
   const bool bit = N <= kBitonicN;
-  unsigned long long *k0 = bit ? reinterpret_cast<unsigned long long *>(small_raw) : sm.key[0];
-  for (int x = tid; x < N; x += kSegThreads) {
-    const int32_t a = __ldg(arrival + x);
-    if (a < 0) bad = true;
-    if (x + 1 < N && __ldg(arrival + x + 1) < a) unsorted = true;
-    k0[x] = (static_cast<unsigned long long>(a < 0 ? 0 : a) << ib) | static_cast<unsigned>(x);
+  if (tid == 0) {
+    s_amax = 0;
+    s_umax = 0;
   }
-  int P = 1;
-  while (P < N) P <<= 1;
-  unsorted = __syncthreads_or(unsorted) != 0;
-  int cur = 0;
   // the bitonic path's two key arrays sit back to back (the launch asks for
   // only 2 kBitonicN keys of shared memory then)
   unsigned long long *kb[2] = {reinterpret_cast<unsigned long long *>(small_raw),
                                reinterpret_cast<unsigned long long *>(small_raw) + kBitonicN};
+  unsigned long long *k0 = bit ? kb[0] : sm.key[0];
+  __syncthreads();
+  uint32_t amax = 0;
+  for (int x = tid; x < N; x += kSegThreads) {
+    const int32_t a = __ldg(arrival + x);
+    if (a < 0) bad = true;
+    if (x + 1 < N && __ldg(arrival + x + 1) < a) unsorted = true;
+    amax = max(amax, static_cast<uint32_t>(a < 0 ? 0 : a));
+    k0[x] = (static_cast<unsigned long long>(a < 0 ? 0 : a) << ib) | static_cast<unsigned>(x);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) amax = max(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+  if ((tid & 31) == 0) atomicMax(&s_amax, amax);
+  unsorted = __syncthreads_or(unsorted) != 0;
+  // arrival out of index order: when (decoder, not promoted, primary,
+  // arrival, index) fits 64 bits, one sort on that key gives the order;
+  // otherwise the entries are put in arrival order first
+  int ab = 0, ub = 0;
+  bool one = false;
   if (unsorted) {
-    if (bit) {
-      for (int x = N + tid; x < P; x += kSegThreads) kb[0][x] = ~0ull;
-      __syncthreads();
-      block_bitonic(kb[0], P);
-    } else {
-      cur = seg_lsd(sm, N, seg_diff(sm, N, 0), ib, ib + 31, 0);
+    uint32_t umax = 0;  // the largest bound of a non-promoted entry
+    for (int x = tid; x < N; x += kSegThreads) {
+      const int32_t u = __ldg(bound + x), w = __ldg(wait + x);
+      if (w <= max_wait && u > 0) umax = max(umax, static_cast<uint32_t>(u));
     }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) umax = max(umax, __shfl_xor_sync(0xffffffffu, umax, off));
+    if ((tid & 31) == 0) atomicMax(&s_umax, umax);
+    __syncthreads();
+    ab = bit_width(s_amax);
+    ub = bit_width(s_umax);
+    one = dbits + 1 + ub + ab + ib <= 64;
   }
-  unsigned long long *kin = bit ? kb[0] : sm.key[cur];
-  unsigned long long *kout = bit ? kb[1] : sm.key[cur ^ 1];
-  for (int t = tid; t < N; t += kSegThreads) {  // the queue keys, in arrival order
-    const int x = static_cast<int>(kin[t] & imask);
-    int32_t d = __ldg(dec + x);
-    const int32_t u = __ldg(bound + x), w = __ldg(wait + x);
-    if (d < 0 || d >= D) {
-      bad = true;
-      d = 0;
-    }
-    if (u < 0) bad = true;
-    const unsigned long long np = w > max_wait ? 0ull : 1ull;
-    const unsigned long long prim = np ? static_cast<unsigned long long>(u < 0 ? 0 : u) : 0ull;
-    // low bits: the arrival position for the bitonic sort (unique keys), the
-    // index for the stable passes
-    kout[t] = (((static_cast<unsigned long long>(d) << 32) | (np << 31) | prim) << ib) |
-              static_cast<unsigned>(bit ? t : x);
-  }
+  int P = 1;
+  while (P < N) P <<= 1;
+  int cur = 0;
   const unsigned long long *ks;  // the sorted queue keys
-  if (bit) {
-    for (int t = N + tid; t < P; t += kSegThreads) kout[t] = ~0ull;
-    __syncthreads();
-    block_bitonic(kout, P);
-    for (int t = tid; t < N; t += kSegThreads)  // arrival position -> index
-      perm[t] = static_cast<int32_t>(kin[kout[t] & imask] & imask);
-    ks = kout;
+  int dshift;                    // where their decoder field starts
+  if (one) {
+    for (int x = tid; x < N; x += kSegThreads) {  // each thread rewrites its own keys
+      const int32_t a = __ldg(arrival + x), u = __ldg(bound + x), w = __ldg(wait + x);
+      int32_t d = __ldg(dec + x);
+      if (d < 0 || d >= D) {
+        bad = true;
+        d = 0;
+      }
+      if (u < 0) bad = true;
+      const unsigned long long np = w > max_wait ? 0ull : 1ull;
+      const unsigned long long prim = np ? static_cast<unsigned long long>(u < 0 ? 0 : u) : 0ull;
+      unsigned long long key = (static_cast<unsigned long long>(d) << 1) | np;
+      key = (key << ub) | prim;
+      key = (key << ab) | static_cast<unsigned long long>(a < 0 ? 0 : a);
+      k0[x] = (key << ib) | static_cast<unsigned>(x);
+    }
+    if (bit) {
+      for (int x = N + tid; x < P; x += kSegThreads) k0[x] = ~0ull;
+      __syncthreads();
+      block_bitonic(k0, P);
+      ks = k0;
+    } else {
+      __syncthreads();
+      cur = seg_lsd(sm, N, seg_diff(sm, N, 0), ib, ib + ab + ub + 1 + dbits, 0);
+      ks = sm.key[cur];
+    }
+    for (int t = tid; t < N; t += kSegThreads) perm[t] = static_cast<int32_t>(ks[t] & imask);
+    dshift = ib + ab + ub + 1;
   } else {
-    __syncthreads();
-    cur ^= 1;
-    cur = seg_lsd(sm, N, seg_diff(sm, N, cur), ib, ib + 32 + dbits, cur);
-    for (int t = tid; t < N; t += kSegThreads) perm[t] = static_cast<int32_t>(sm.key[cur][t] & imask);
-    ks = sm.key[cur];
+    // k0 holds (arrival, index) keys, written before the barrier above
+    if (unsorted) {
+      if (bit) {
+        for (int x = N + tid; x < P; x += kSegThreads) kb[0][x] = ~0ull;
+        __syncthreads();
+        block_bitonic(kb[0], P);
+      } else {
+        cur = seg_lsd(sm, N, seg_diff(sm, N, 0), ib, ib + 31, 0);
+      }
+    }
+    unsigned long long *kin = bit ? kb[0] : sm.key[cur];
+    unsigned long long *kout = bit ? kb[1] : sm.key[cur ^ 1];
+    for (int t = tid; t < N; t += kSegThreads) {  // the queue keys, in arrival order
+      const int x = static_cast<int>(kin[t] & imask);
+      int32_t d = __ldg(dec + x);
+      const int32_t u = __ldg(bound + x), w = __ldg(wait + x);
+      if (d < 0 || d >= D) {
+        bad = true;
+        d = 0;
+      }
+      if (u < 0) bad = true;
+      const unsigned long long np = w > max_wait ? 0ull : 1ull;
+      const unsigned long long prim = np ? static_cast<unsigned long long>(u < 0 ? 0 : u) : 0ull;
+      // low bits: the arrival position for the bitonic sort (unique keys), the
+      // index for the stable passes
+      kout[t] = (((static_cast<unsigned long long>(d) << 32) | (np << 31) | prim) << ib) |
+                static_cast<unsigned>(bit ? t : x);
+    }
+    if (bit) {
+      for (int t = N + tid; t < P; t += kSegThreads) kout[t] = ~0ull;
+      __syncthreads();
+      block_bitonic(kout, P);
+      for (int t = tid; t < N; t += kSegThreads)  // arrival position -> index
+        perm[t] = static_cast<int32_t>(kin[kout[t] & imask] & imask);
+      ks = kout;
+    } else {
+      __syncthreads();
+      cur ^= 1;
+      cur = seg_lsd(sm, N, seg_diff(sm, N, cur), ib, ib + 32 + dbits, cur);
+      for (int t = tid; t < N; t += kSegThreads) perm[t] = static_cast<int32_t>(sm.key[cur][t] & imask);
+      ks = sm.key[cur];
+    }
+    dshift = ib + 32;
   }
   for (int d = tid; d <= D; d += kSegThreads) {  // entries of decoders below d
     int lo = 0, hi = N;
     while (lo < hi) {
       const int mid = (lo + hi) >> 1;
-      if (static_cast<long long>(ks[mid] >> (ib + 32)) < d)
+      if (static_cast<long long>(ks[mid] >> dshift) < d)
         lo = mid + 1;
       else
         hi = mid;

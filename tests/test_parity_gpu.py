@@ -555,6 +555,30 @@ def test_order_random(M, ws, oracle, N, D, sorted_arrival):
     assert np.array_equal(seg, so)
 
 
+@pytest.mark.parametrize("N,D,ubits,abits", [
+    # one-block calls with arrival out of index order: when (decoder, not
+    # promoted, bound, arrival, index) fits 64 bits one sort on it gives the
+    # order (bitonic, then stable passes), otherwise two sorts do
+    (700, 5, 15, 20), (3000, 40, 15, 20), (1000, 1, 31, 31), (4000, 300, 31, 31),
+    # exactly 64 bits, and one bit more
+    (1024, 16, 18, 31), (1024, 16, 19, 31)])
+def test_order_small_unsorted_key_widths(M, ws, oracle, N, D, ubits, abits):
+    rng = np.random.default_rng(N + D + ubits)
+    dec = rng.integers(0, D, N).astype(np.int32)
+    U = rng.integers(0, 2**ubits, N, dtype=np.int64).astype(np.int32)
+    wait = rng.integers(-10, 3000, N).astype(np.int32)
+    i = rng.integers(0, N)
+    U[i], wait[i] = 2**ubits - 1, 0  # the full width, on an entry that is not promoted
+    arr = rng.integers(0, 2**abits, N, dtype=np.int64).astype(np.int32)
+    arr[rng.integers(0, N)] = 2**abits - 1
+    arr[: N // 4] = arr[N // 4]  # ties on arrival
+    sto, po, so = oracle.order_local(D, dec, U, wait, arr, 1000)
+    st, perm, seg = gpu_order(M, ws, D, dec, U, wait, arr, 1000)
+    assert st == sto == 0
+    assert np.array_equal(perm, po)
+    assert np.array_equal(seg, so)
+
+
 def test_order_bucketing_rounds_range_error(M, ws, oracle):
     """An entry outside the decoder domain in a call whose bucketing blocks
     take several rounds: counted and placed at decoder 0 in both of its
