@@ -145,7 +145,9 @@ def test_golden_worked_example(M, ws, golden):
 # calibration
 # ---------------------------------------------------------------------------
 
-@pytest.mark.parametrize("n", [1, 2, 3, 9, 10, 1000, 4097, 65537, 1000003])
+# one-block sizes: a bitonic sort up to 2,048 scores, a radix select up to
+# 8,192; then the cooperative kernel
+@pytest.mark.parametrize("n", [1, 2, 3, 9, 10, 1000, 1024, 1025, 2048, 2049, 4097, 65537, 1000003])
 def test_calibrate_random(M, ws, oracle, n):
     rng = np.random.default_rng(n)
     L = rng.integers(-(2**31), 2**31, n, dtype=np.int64).astype(np.int32) if n % 2 else \
