@@ -64,16 +64,16 @@ L2_FLUSH_BYTES = 256 << 20
 # valid only for the kernel source it was taken on.
 TRAFFIC = {
     "dispatch_feasible": {"bytes": 0, "source": "dispatch.cu", "source_sha256": ""},
-    "calibrate": {"bytes": 12528384, "source": "calibrate.cu", "source_sha256":
-        "f911677ebf18557a3fe29062328fd3091e4376a7303344c0642bc1748c1f7e87"},
+    "calibrate": {"bytes": 12529152, "source": "calibrate.cu", "source_sha256":
+        "276186c42f8478d5e6974baf53e2af9bb81b825d1d070bb4995dfe8d2de38920"},
     "occupancy": {"bytes": 31169536, "source": "occupancy.cu", "source_sha256":
         "fd537e3019c8991f53d529abba17e1a23b2664a7f4477b0936c6a78e22aa0746"},
     "dispatch": {"bytes": 26562560, "source": "dispatch.cu", "source_sha256":
         "bc228a45bdc7bb49327bd4b8871778b2d0a6aa7e4c877112d9afa425f6628241"},
     "dispatch_scoring": {"bytes": 21107968, "source": "dispatch.cu", "source_sha256":
         "bc228a45bdc7bb49327bd4b8871778b2d0a6aa7e4c877112d9afa425f6628241"},
-    "order": {"bytes": 28038912, "source": "order.cu", "source_sha256":
-        "096437fff8f81cae667e81cdcfbdb6320c336a9bb200371bf585b5e1a2eccb37"},
+    "order": {"bytes": 28039168, "source": "order.cu", "source_sha256":
+        "9f99bc2e2751e755a279d07397d1df4fce876f9be2cfdee980f5c3fa25798411"},
 }
 KERNELS = {
     "calibrate": "calibrate_fused_kernel (maps_calibrate: select passes and bounds in one "
