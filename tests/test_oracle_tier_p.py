@@ -74,7 +74,7 @@ def test_tier_p_equals_tier_b_on_workloads(oracle, name, feasible):
 
 def test_tier_p_equals_tier_b_on_random_tiny_instances(oracle):
     rng = np.random.default_rng(2024)
-    for it in range(300):
+    for it in range(10_000):
         n = int(rng.integers(0, 40))
         L = rng.integers(0, 60, n).astype(np.int32)
         P = rng.integers(0, 60, n).astype(np.int32)
