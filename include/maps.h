@@ -21,6 +21,12 @@
  *           on it and return without waiting, except where a `_host` output
  *           is non-NULL: then the call synchronises the stream and returns
  *           the full status, data-dependent errors included.
+ * Grids.    maps_calibrate with more than 8,192 residuals and
+ *           maps_order_local past one block each launch one cooperative
+ *           kernel (every block resident at once, with bounded grid
+ *           barriers): such a launch starts when the multiprocessors it
+ *           needs are free, so it waits for other streams' kernels that hold
+ *           them.
  * Layout.   Arrays are dense and row-major; int32 unless stated.  K is
  *           [D][H].  Residents of decoder k are the index range
  *           [res_off[k], res_off[k+1]) of the resident arrays (CSR).
