@@ -862,6 +862,11 @@ def test_stream_golden(M, ws, stream_golden):
     # 200 decoders x batches of 256: the end-step tables would need about 800 KB of
     # shared memory, so the loop dispatches through the dense projection instead
     (3000, 200, 2048, 60000, 256, 300, 100000, 1000),
+    # 48 decoders: the shared-memory walk past one warp's decoders, with queues
+    (4000, 48, 4096, 30000, 64, 200, 100000, 1000),
+    # a window of 10,000 completions: once it holds more than 8,192 the quantile is
+    # taken by the cooperative calibration kernel inside the loop
+    (30000, 8, 16384, 262144, 512, 10000, 100000, 1000),
 ])
 def test_stream_prefix(M, ws, oracle, N, D, H, cap, B, Wn, a, mw):
     w = W.make_stream(n_requests=N)
