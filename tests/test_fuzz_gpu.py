@@ -4,13 +4,16 @@ succeeds.  Sizes start at zero; lengths fall in and out of the domain;
 horizons go down to one step; decoders may have no residents; values are
 drawn from small ranges so that ties are everywhere.  Each draw is seeded,
 and a failure reports its iteration."""
+import os
+
 import numpy as np
 import pytest
 import torch
 
 pytestmark = pytest.mark.gpu
 
-ITERATIONS = 3000
+# draws per test; MAPS_FUZZ_ITERATIONS runs a longer sweep
+ITERATIONS = int(os.environ.get("MAPS_FUZZ_ITERATIONS", "3000"))
 
 
 @pytest.fixture(scope="module")

@@ -5,13 +5,16 @@ index order, bounds of a few bits to the full 31.  Each output is compared
 element by element with the plain oracle (tier P), which the CPU tests pin
 to the by-definition one; the statuses must agree.  Each draw is seeded, and
 a failure reports its iteration."""
+import os
+
 import numpy as np
 import pytest
 import torch
 
 pytestmark = pytest.mark.gpu
 
-ITERATIONS = 100
+# draws per test; MAPS_FUZZ_ITERATIONS runs a longer sweep
+ITERATIONS = int(os.environ.get("MAPS_FUZZ_ITERATIONS", "100"))
 
 
 @pytest.fixture(scope="module")
