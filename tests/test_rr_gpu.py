@@ -2,6 +2,8 @@
 (maps_rr_pressure) against the plain oracle: every admission and completion
 time, every decoder's high-pressure metrics and waiting statistics, and each
 realisation's span -- bit for bit."""
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -88,3 +90,33 @@ def test_rr_errors(M, oracle):
     cfg = M.RRCfg(0, 1, 1, 1, 1)
     assert M.lib.maps_rr_pressure(cfg, 1, None, None, None, None, None, None, None, None, 0,
                                   None) == M.MAPS_E_INVALID
+
+
+def test_rr_random_sweep(M, oracle):
+    """Random configurations: 1 to 16 decoders, capacities from barely above
+    the largest footprint to ample, 1 to 3,000 requests in 1 to 6
+    realisations per call, thresholds from 1 ppm to 1, token times of 1 us
+    to 2 ms, and arrivals from simultaneous to sparse.  MAPS_FUZZ_ITERATIONS
+    runs a longer sweep."""
+    rng = np.random.default_rng(59)
+    for it in range(int(os.environ.get("MAPS_FUZZ_ITERATIONS", "40"))):
+        N = int(rng.integers(1, 17))
+        n = int(rng.integers(1, 3000))
+        n_real = int(rng.integers(1, 7))
+        out = rng.integers(1, int(rng.choice([5, 300, 3000])), (n_real, n))
+        C = int(out.max()) + int(rng.choice([1, 500, 5000, 100_000]))
+        prompt = np.minimum(rng.integers(0, 4000, (n_real, n)), C - out)
+        gaps = rng.integers(0, int(rng.choice([1, 3, 50_000, 2_000_000])), (n_real, n))
+        arr = np.cumsum(gaps, axis=1) + rng.integers(0, 10**6, (n_real, 1))
+        theta = int(rng.choice([1, 300_000, 850_000, 1_000_000]))
+        tok = int(rng.choice([1, 1000, 2000]))
+        st, adm, done, stats, tsim = gpu_rr(M, N, C, tok, theta, arr, prompt, out)
+        ref = [oracle.rr_pressure(N, C, tok, theta, arr[r], prompt[r], out[r]) for r in range(n_real)]
+        # one call covers every realisation: it succeeds when each of them does
+        assert (st == 0) == all(x[0] == 0 for x in ref), (it, N, C, n, st)
+        if st == 0:
+            for r, (_, a, d, s_, ts) in enumerate(ref):
+                assert np.array_equal(adm[r], a), (it, r)
+                assert np.array_equal(done[r], d), (it, r)
+                assert np.array_equal(stats[r], s_), (it, r)
+                assert tsim[r] == ts, (it, r)
